@@ -1,0 +1,376 @@
+"""Benchmark: PVS resumable exact dense ranking on one GB300 (per rank).
+
+Workload (the passage-scale single-query configuration): a corpus of
+N = 8,841,823 vectors of d = 768 drawn from a 4,096-component Gaussian
+mixture (standard-normal centres, within-component std 0.35, L2-normalised);
+queries are perturbed mixture centres (noise std 0.5, normalised).  One step
+= a batch of queries; per query the cursor delivers the first 1,000 exact
+ranks in chunks of 20 (open, 50 pulls, close).  The corpus codes (6.9 GB per
+interval pass) are far larger than the 129 MB L2, so no L2 flush is needed.
+
+`value` (exact dense ranks/s) is timed with CUDA events on the library's
+stream with queries resident in HBM and ranks written to device buffers;
+`e2e` repeats the step through the same C ABI with host query buffers and
+host output buffers (pvs_next), the copies inside the timed region.
+`roofline` reports the interval pass (the dominant kernel): algorithmic bytes
+N * (m_pad + 12) per pass over its CUDA-event duration, against the measured
+HBM copy bandwidth.
+
+`--impl reference` times the oracle (a plain CPU implementation, run as it
+stands) on a bounded sample of the same workload.  Under torchrun every rank
+ranks its own queries against its own copy of the index (no collective).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+N_CORPUS = 8_841_823
+DIM = 768
+COMPONENTS = 4096
+WITHIN_STD = 0.35
+QUERY_NOISE = 0.5
+RANKS_PER_QUERY = 1000
+CHUNK = 20
+METRIC = "exact dense ranks/sec"
+UNIT = "ranks/s"
+WORKLOAD = ("passage-scale single-query ranking: N=8,841,823 x d=768 Gaussian mixture "
+            "(4,096 components, within std 0.35, L2-normalised), first 1,000 exact ranks "
+            "per query in chunks of 20")
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=3)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="pvs", choices=["pvs", "reference"])
+    p.add_argument("--queries", type=int, default=50, help="queries per step")
+    p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: int):
+        self.gpu = gpu
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        rows = [r.split(",") for r in getattr(self, "out", "").strip().splitlines() if r.strip()]
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def build_corpus_index(pvs, synth, torch, n, stream, device):
+    """Generate the mixture corpus chunk by chunk straight into the index."""
+    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=device)
+    index = None
+    chunk = 1 << 20
+    t0 = time.perf_counter()
+    for r in range(0, n, chunk):
+        c = min(chunk, n - r)
+        rows = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+        if index is None:
+            index = pvs.pvs_build(rows, stream=stream)
+        else:
+            pvs.pvs_append(index, rows)
+        del rows
+    torch.cuda.synchronize()
+    return index, centres, time.perf_counter() - t0
+
+
+def run_step_device(pvs, torch, index, queries, out_ids, out_scores, stream, lat20, lat1000,
+                    stats_acc):
+    """One step: every query opens a cursor and pulls 1,000 ranks in chunks
+    of 20 into device buffers."""
+    ev = []
+    for qi in range(queries.shape[0]):
+        t_open = torch.cuda.Event(enable_timing=True)
+        t_20 = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_open.record(stream)
+        cur = pvs.pvs_cursor_open(index, queries[qi])
+        for p in range(RANKS_PER_QUERY // CHUNK):
+            off = p * CHUNK
+            pvs.pvs_next_device(cur, CHUNK, out_ids[qi, off:], out_scores[qi, off:])
+            if p == 0:
+                t_20.record(stream)
+        t_end.record(stream)
+        st = pvs.pvs_cursor_sync(cur)
+        s = pvs.pvs_cursor_stats(cur)
+        pvs.pvs_cursor_close(cur)
+        if st < 0:
+            raise RuntimeError(f"cursor failed: {st}")
+        ev.append((t_open, t_20, t_end))
+        stats_acc.append(s)
+    stream.synchronize()
+    for a, b, c in ev:
+        lat20.append(a.elapsed_time(b))
+        lat1000.append(a.elapsed_time(c))
+
+
+def run_step_host(pvs, index, queries_host):
+    for q in queries_host:
+        cur = pvs.pvs_cursor_open(index, q)
+        for p in range(RANKS_PER_QUERY // CHUNK):
+            ids, sc, st = pvs.pvs_next(cur, CHUNK)
+        pvs.pvs_cursor_close(cur)
+
+
+def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget=20.0):
+    """The oracle (as it stands) on a bounded sample: the first `rows` corpus
+    rows, for as many queries as fit the budget; ranks/s scaled to the full N
+    (the oracle's cost is linear in the rows it scores)."""
+    import numpy as np
+    from oracle import pvs_oracle as po
+    rows = 1 << 20
+    V = synth.mixture_rows(rows, centres_dev, WITHIN_STD, seed=2, first=0).cpu().numpy()
+    t0 = time.perf_counter()
+    done = 0
+    while done < len(queries_host):
+        ids, sc = po.dense_ranking(queries_host[done], V)
+        _ = ids[:RANKS_PER_QUERY]
+        done += 1
+        if time.perf_counter() - t0 > seconds_budget:
+            break
+    dt = time.perf_counter() - t0
+    per_query_full = dt / done * (n_full / rows)
+    return {"value": RANKS_PER_QUERY / per_query_full, "unit": UNIT,
+            "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{done} queries x first {RANKS_PER_QUERY} exact ranks over the first "
+                      f"{rows:,} corpus rows (oracle: binary64 scoring + exact fallback + full "
+                      f"sort), time scaled by N/{rows:,}"}
+
+
+def reference_arm(args):
+    rank, world, local = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+    import synth
+    from oracle import pvs_oracle as po
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=dev)
+    rows = 1 << 19
+    V = synth.mixture_rows(rows, centres, WITHIN_STD, seed=2, first=0).cpu().numpy()
+    Q = synth.mixture_queries(args.warmup + args.steps, centres, QUERY_NOISE, seed=3).cpu().numpy()
+    for w in range(args.warmup):
+        po.dense_ranking(Q[w], V)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        po.dense_ranking(Q[args.warmup + s], V)
+    dt = (time.perf_counter() - t0) / args.steps * (args.n / rows)
+    value = RANKS_PER_QUERY / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "N": args.n, "d": DIM,
+                       "step": "1 query, first 1,000 ranks"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
+                             "kind": "oracle",
+                             "sample": f"1 query per step over the first {rows:,} rows, "
+                                       f"time scaled by N/{rows:,}"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+        return
+    import numpy as np
+    import torch
+    import paper_2608_07152_gb300 as pvs
+    import synth
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    stream = torch.cuda.Stream(device=dev)
+    n = args.n
+    index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev)
+    total_q = (args.warmup + args.steps) * args.queries
+    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=3 + 7919 * rank)
+    queries = queries.reshape(args.warmup + args.steps, args.queries, DIM).contiguous()
+    out_ids = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
+    out_scores = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+
+    lat20, lat1000, stats = [], [], []
+    for w in range(args.warmup):
+        run_step_device(pvs, torch, index, queries[w], out_ids, out_scores, stream, [], [], [])
+
+    # ---- timed region: device-resident queries and outputs ----
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    launches0 = pvs.pvs_launch_count()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for s in range(args.steps):
+            run_step_device(pvs, torch, index, queries[args.warmup + s], out_ids, out_scores,
+                            stream, lat20, lat1000, stats)
+        end.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    launches = pvs.pvs_launch_count() - launches0
+    elapsed = start.elapsed_time(end) / 1e3
+    if pg:
+        t = torch.tensor([elapsed], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        elapsed = float(t.item())
+    ranks_total = args.steps * args.queries * RANKS_PER_QUERY * world
+    value = ranks_total / elapsed
+
+    # ---- e2e: host query buffers, host outputs through pvs_next ----
+    qh = [np.ascontiguousarray(queries[args.warmup + s].cpu().numpy()) for s in range(args.steps)]
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        run_step_host(pvs, index, qh[s])
+    torch.cuda.synchronize()
+    e2e_elapsed = time.perf_counter() - t0
+    if pg:
+        t = torch.tensor([e2e_elapsed], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        e2e_elapsed = float(t.item())
+    e2e_value = ranks_total / e2e_elapsed
+
+    # ---- roofline of the interval pass ----
+    m_pad = ((DIM + 63) // 64) * 64
+    passes = sum(s["interval_passes"] for s in stats)
+    interval_ms = sum(s["interval_ms"] for s in stats) / max(passes, 1)
+    alg_bytes = n * (m_pad + 12)
+    achieved = alg_bytes / (interval_ms / 1e3) / 1e9
+    peak, peak_kind = measured_peaks()
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "interval_pass_traffic.json")
+    if os.path.exists(prof):
+        try:
+            with open(prof) as f:
+                traffic = json.load(f).get("traffic_bytes_per_pass")
+        except Exception:
+            traffic = None
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "N": n, "d": DIM, "queries_per_step": args.queries,
+                   "ranks_per_query": RANKS_PER_QUERY, "chunk": CHUNK,
+                   "l2": "no flush: each query's interval pass streams 6.9 GB of codes (> 129 MB L2)",
+                   "parallelism": f"replicas x{world} (queries sharded, no collective)"},
+        "e2e": {"value": e2e_value, "unit": UNIT,
+                "h2d_bytes_per_step": args.queries * DIM * 4,
+                "d2h_bytes_per_step": args.queries * RANKS_PER_QUERY * (8 + 4)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_kind": peak_kind, "kernel": "interval_pass_kernel",
+                     "frac_of_8tbs_nominal": achieved / 8000.0},
+        "gpu_launches": launches,
+        "latency_ms": {"first_20_p50": statistics.median(lat20),
+                       "first_1000_p50": statistics.median(lat1000),
+                       "first_1000_p95": sorted(lat1000)[int(0.95 * (len(lat1000) - 1))]},
+        "interval_pass": {"ms": interval_ms, "GBps": achieved, "bytes": alg_bytes},
+        "per_query": {"refined_mean": statistics.mean(s["refined"] for s in stats),
+                      "candidates_mean": statistics.mean(s["candidates"] for s in stats),
+                      "exact_fallbacks": sum(s["exact_fallbacks"] for s in stats)},
+        "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        qb = queries[0].cpu().numpy()
+        line["cpu_baseline"] = cpu_baseline(synth, torch, centres, qb, n)
+    pvs.pvs_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

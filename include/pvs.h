@@ -1,0 +1,250 @@
+/*
+ * pvs.h -- C ABI of the GB300 PVS / EAHR library (libpvs.so).
+ *
+ * Method: "Exact Adaptive Hybrid Retrieval Without Fixed Top-L Cutoffs",
+ * arXiv 2608.07152.
+ *   - PVS (Per-Vector Scalar Quantization) resumable exact dense ranking,
+ *     Sec. 2.3.1 and Appendix A.1;
+ *   - the ranked-list contract (stable exact prefix, Open / Exhausted /
+ *     Failed), Sec. 2.1;
+ *   - EAHR adaptive weighted-RRF fusion with ordered certification,
+ *     Sec. 2.1 and 2.2.
+ *
+ * Conventions for every entry point:
+ *   - Every call returns a pvs_status.  Negative values are errors; on an
+ *     error no output is produced and, for a cursor, the cursor becomes
+ *     Failed for good (Sec. 2.1: a Failed list invalidates the request).
+ *   - Item ids are row numbers in insertion order (0, 1, 2, ...); the tie
+ *     order between equal scores is ascending id.
+ *   - Vectors are row-major float32, `dim` floats per row, no padding.
+ *   - "on_device" flags say whether a pointer is CUDA device memory (or
+ *     managed memory) of the current device (1) or host memory (0).
+ *   - The library owns index, snapshot and cursor objects; the caller owns
+ *     every buffer it passes in.  Objects are not thread-safe: calls on one
+ *     index, its snapshots and its cursors must not run concurrently.
+ *   - All device work runs on the CUDA stream given to pvs_build (or a
+ *     library-created stream when NULL).
+ */
+#ifndef PVS_H_
+#define PVS_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum pvs_status {
+    PVS_OK = 0,
+    PVS_EXHAUSTED = 1,        /* the ranked list is complete (Sec. 2.1)        */
+    PVS_ERR_INVALID = -1,     /* bad argument or call sequence                 */
+    PVS_ERR_NONFINITE = -2,   /* non-finite vector entry (App. A.1)            */
+    PVS_ERR_OVERFLOW = -3,    /* a bound or score overflows float32, or the
+                                 Int8 accumulator could overflow (App. A.1)    */
+    PVS_ERR_INTERVAL = -4,    /* an authoritative score fell outside its
+                                 interval (App. A.1): the request fails        */
+    PVS_ERR_CUDA = -5,        /* a CUDA runtime call failed                    */
+    PVS_ERR_OOM = -6,         /* device or host allocation failed              */
+    PVS_ERR_TIMEOUT = -7,     /* a device-side wait ran out of time            */
+    PVS_ERR_FAILED = -8       /* the cursor failed earlier                     */
+} pvs_status;
+
+typedef struct pvs_index pvs_index;
+typedef struct pvs_snapshot pvs_snapshot;
+typedef struct pvs_cursor pvs_cursor;
+
+/* Counters of one cursor (the logical counters of Sec. 3.5 plus device
+ * traffic). */
+typedef struct pvs_stats {
+    int64_t visible;          /* n_i: items in the cursor's ranked list        */
+    int64_t emitted;          /* d_i: ranks delivered so far                   */
+    int64_t refined;          /* authoritative float32 score evaluations       */
+    int64_t exact_fallbacks;  /* evaluations that needed the exact accumulator */
+    int64_t interval_passes;  /* full passes over the Int8 codes               */
+    int64_t horizon_builds;   /* candidate-set (re)builds from the bounds      */
+    int64_t pulls;            /* pvs_next / pvs_next_device calls              */
+    int64_t candidates;       /* candidate entries certified over all pulls    */
+    int64_t code_bytes;       /* bytes of codes + per-vector params scanned    */
+    int32_t state;            /* PVS_OK (Open), PVS_EXHAUSTED, or the failure  */
+    int32_t reserved;
+    double interval_ms;       /* device time of the interval passes, measured
+                                 with CUDA events on the cursor's stream       */
+} pvs_stats;
+
+/* ---------------------------------------------------------------------------
+ * Index (Sec. 2.3.1: PVS stores per vector an Int8 code z_v in [-127,127]^m,
+ * a scale s_v > 0, and here the upward-rounded norms ||v||_2 and
+ * ||v - s_v z_v||_2 that the residual bound E and guard G need (App. A.1);
+ * the raw float32 vectors are kept for authoritative scoring).
+ * ------------------------------------------------------------------------ */
+
+/* Build an index over n vectors of dimension dim (1 <= dim <= 32767,
+ * 0 <= n < 2^31).  `vecs` is n*dim floats, host or device per
+ * vecs_on_device.  `cuda_stream` is a cudaStream_t (NULL: the library
+ * creates one).  Errors: PVS_ERR_INVALID (null out, bad sizes),
+ * PVS_ERR_NONFINITE (an entry is NaN or +-inf; App. A.1), PVS_ERR_OVERFLOW
+ * (a norm bound overflows float32), PVS_ERR_OOM, PVS_ERR_CUDA.  On success
+ * *out owns device copies of everything; free it with pvs_index_free. */
+pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
+                     void* cuda_stream, pvs_index** out);
+
+/* Append n vectors; they get ids size .. size+n-1.  Existing snapshots and
+ * open cursors keep their visible set (Sec. 2.4: fixed snapshots).  Errors
+ * as pvs_build; on error the index is unchanged. */
+pvs_status pvs_append(pvs_index* index, const float* vecs, int64_t n, int32_t vecs_on_device);
+
+/* Tombstone (delete) n ids given in host memory.  Deleting a deleted id is a
+ * no-op.  Affects snapshots created afterwards only (Sec. 2.4: deletion
+ * state defines the visible items of a snapshot).  Errors: PVS_ERR_INVALID
+ * if an id is out of range (nothing is deleted then). */
+pvs_status pvs_tombstone(pvs_index* index, const int64_t* ids, int64_t n);
+
+int64_t pvs_index_size(const pvs_index* index);   /* rows ever inserted       */
+int64_t pvs_index_live(const pvs_index* index);   /* rows not tombstoned      */
+int32_t pvs_index_dim(const pvs_index* index);
+/* Copy rows [first, first+count) of the index into caller buffers, any of
+ * which may be NULL: codes as int8 [count x dim], scales, norm bounds of v and
+ * of the residual v - s_v z_v (float32 [count]).  Host pointers. */
+pvs_status pvs_index_export(const pvs_index* index, int64_t first, int64_t count,
+                            int8_t* codes, float* scale, float* vnorm, float* enorm);
+void pvs_index_free(pvs_index* index);
+
+/* Freeze the currently visible set (rows inserted so far minus tombstones).
+ * A snapshot may be freed while cursors opened on it are still open. */
+pvs_status pvs_snapshot_create(pvs_index* index, pvs_snapshot** out);
+int64_t pvs_snapshot_visible(const pvs_snapshot* snap);
+void pvs_snapshot_free(pvs_snapshot* snap);
+
+/* ---------------------------------------------------------------------------
+ * Cursor: one query's resumable exact dense ranked list (Sec. 2.1, 2.3.1).
+ * ------------------------------------------------------------------------ */
+
+/* Open a cursor for one query (dim floats, host or device).  `snap` may be
+ * NULL for the index's current visible set.  The query is encoded like a
+ * corpus vector (Sec. 2.3.1).  The index must outlive the cursor.  Errors:
+ * PVS_ERR_INVALID, PVS_ERR_NONFINITE, PVS_ERR_OVERFLOW, PVS_ERR_OOM,
+ * PVS_ERR_CUDA. */
+pvs_status pvs_cursor_open(pvs_index* index, const pvs_snapshot* snap, const float* query,
+                           int32_t query_on_device, pvs_cursor** out);
+
+/* Open nq cursors that share one batched interval pass (queries: nq*dim
+ * floats).  `horizon` is the number of ranks each cursor is prepared to
+ * deliver without rescanning the codes (>= 1; later ranks still come out
+ * exactly, at the cost of a rescan).  out[0..nq-1] receive the cursors. */
+pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
+                                 const float* queries, int32_t nq, int32_t queries_on_device,
+                                 int32_t horizon, pvs_cursor** out);
+
+/* Deliver the next n exact ranks (Sec. 2.1: a stable exact prefix that is
+ * only ever extended).  ids (int64) and scores (the authoritative float32
+ * scores: the correctly rounded value of the exact inner product) are HOST
+ * buffers of n entries; *n_out receives the count written.  Returns PVS_OK,
+ * or PVS_EXHAUSTED once the last rank has been delivered (then
+ * *n_out <= n; later calls deliver 0).  Blocks until the ranks are on the
+ * host.  Errors: PVS_ERR_INVALID (n < 0 or null pointers), PVS_ERR_INTERVAL
+ * (App. A.1 failure rule), PVS_ERR_OVERFLOW, PVS_ERR_TIMEOUT, PVS_ERR_CUDA,
+ * PVS_ERR_FAILED (the cursor failed before). */
+pvs_status pvs_next(pvs_cursor* cursor, int32_t n, int64_t* ids, float* scores, int32_t* n_out);
+
+/* As pvs_next, but ids and scores are DEVICE buffers and the call only
+ * enqueues the work on the cursor's stream; *n_out is exact on return.
+ * Device-side failures surface at the next blocking call (pvs_cursor_sync,
+ * pvs_next, pvs_cursor_stats); every rank delivered since the last
+ * successful blocking call is then void. */
+pvs_status pvs_next_device(pvs_cursor* cursor, int32_t n, int64_t* ids, float* scores,
+                           int32_t* n_out);
+
+/* Wait for the cursor's queued work; return its state (PVS_OK while Open,
+ * PVS_EXHAUSTED, or the failure). */
+pvs_status pvs_cursor_sync(pvs_cursor* cursor);
+pvs_status pvs_cursor_stats(pvs_cursor* cursor, pvs_stats* out);
+void pvs_cursor_close(pvs_cursor* cursor);
+
+/* Diagnostics.  Copy to host the score interval [lo, hi] that the cursor
+ * holds for ids first .. first+count-1 of its snapshot: the App. A.1 interval
+ * before an item is scored, lo == hi == its authoritative score after, and
+ * -inf once the item is delivered or if it is deleted.  Runs the interval
+ * pass first if no pull has run it yet. */
+pvs_status pvs_cursor_bounds(pvs_cursor* cursor, int64_t first, int64_t count, float* lo,
+                             float* hi);
+
+/* Authoritative float32 scores (correctly rounded exact inner products) of
+ * n ids (host array, each < the cursor's snapshot size) against the cursor's
+ * query, written to the host array `scores`.  Does not change the cursor. */
+pvs_status pvs_cursor_score_ids(pvs_cursor* cursor, const int64_t* ids, int32_t n,
+                                float* scores);
+
+const char* pvs_status_string(int32_t status);
+
+/* Number of CUDA kernels this library has launched in this process. */
+int64_t pvs_launch_count(void);
+
+/* ---------------------------------------------------------------------------
+ * EAHR (Sec. 2.1, 2.2): ordered Top-K of complete-list weighted RRF over the
+ * dense ranked list of a cursor and a sparse ranked list from the caller.
+ * ------------------------------------------------------------------------ */
+
+enum {
+    EAHR_RANK_SCALED = 0,   /* g(r) = 1 / (r / w + k - 1)  (Sec. 2.1)         */
+    EAHR_NUMERATOR = 1      /* g(r) = w / (k + r)                              */
+};
+enum {
+    EAHR_POLICY_GEOMETRIC = 0,   /* pull the channel with the larger next
+                                    contribution; pull sizes grow x2 (result
+                                    unchanged: Sec. 2.4)                        */
+    EAHR_POLICY_EQUAL_DEPTH = 1  /* both lists advance by `step` ranks, and
+                                    certification runs after every step
+                                    (the controlled-stream protocol, Sec. 3.4) */
+};
+
+typedef struct eahr_params {
+    int32_t K;          /* result size, >= 1                                   */
+    int32_t k;          /* RRF rank constant, >= 1                             */
+    int32_t form;       /* EAHR_RANK_SCALED or EAHR_NUMERATOR                  */
+    int32_t policy;     /* EAHR_POLICY_*                                       */
+    int32_t step;       /* first pull size (GEOMETRIC) or step (EQUAL_DEPTH);
+                           0 selects 16                                        */
+    int32_t w_num[2];   /* channel weights w_i = w_num[i] / w_den[i];          */
+    int32_t w_den[2];   /* [0] dense, [1] sparse; 0 <= w_num < 2^16,
+                           1 <= w_den < 2^16                                   */
+} eahr_params;
+
+typedef struct eahr_stats {
+    int64_t depth[2];       /* d_i: ranks read from each list                  */
+    int64_t length[2];      /* n_i: complete-list length of each list          */
+    int32_t exhausted[2];   /* list i reached Exhausted                        */
+    int32_t pulls[2];       /* producer calls per list                         */
+    int32_t checks;         /* certification rounds                            */
+    int32_t reserved;
+} eahr_stats;
+
+/* EAHR over a freshly opened dense cursor (no ranks delivered yet) and a
+ * sparse ranked list given as host ids in rank order (the support U_s may be
+ * a subset of the visible items).  Sparse ids are checked as the driver reads
+ * them: an id outside the cursor's snapshot, or repeated within the list,
+ * fails the call with PVS_ERR_INVALID when it is reached (entries the driver
+ * never reads are not inspected).  Writes the q_K <= K ids of T*_K in order
+ * to out_ids and their count to *n_out (Sec. 2.1: zero-score items are never
+ * appended).  out_F (may be NULL) receives each item's fused score F as the
+ * correctly rounded binary64 value of the exact rational where the prefixes
+ * read determine it, and NaN where the item is still unread in an Open list
+ * (its position is certified all the same, Sec. 2.2).  `st` may be NULL.
+ * Errors: PVS_ERR_INVALID (bad parameters, cursor not fresh, bad sparse
+ * list), any error of pvs_next (the request is then void). */
+pvs_status eahr_topk(pvs_cursor* dense, const int64_t* sparse_ids, int64_t n_sparse,
+                     const eahr_params* params, int64_t* out_ids, double* out_F,
+                     int32_t* n_out, eahr_stats* st);
+
+/* The same fusion over two ranked lists held in host memory (ids in rank
+ * order, 0 <= id < 2^31; an id repeated within a list fails the call when it
+ * is read).  For callers with their own producers and for the
+ * controlled-stream protocol of Sec. 3.4. */
+pvs_status eahr_topk_lists(const int64_t* list0, int64_t n0, const int64_t* list1, int64_t n1,
+                           const eahr_params* params, int64_t* out_ids, double* out_F,
+                           int32_t* n_out, eahr_stats* st);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PVS_H_ */

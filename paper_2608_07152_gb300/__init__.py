@@ -1,0 +1,322 @@
+"""GB300-native PVS resumable exact dense ranking and EAHR fusion.
+
+Method: arXiv 2608.07152 (Exact Adaptive Hybrid Retrieval).  Every step of
+the ranking path runs in the CUDA kernels of ``libpvs.so`` behind the C ABI of
+``include/pvs.h``; this module only marshals arguments.  The functions keep
+the C names.  A negative status raises :class:`PvsError`; ``PVS_EXHAUSTED``
+is returned, not raised.
+
+Host inputs are numpy arrays; device inputs are CUDA ``torch`` tensors
+(torch's current stream is synchronised before their pointers are handed to
+the library, which runs on its own stream).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from ._build import LIB as _LIB_PATH
+
+PVS_OK = 0
+PVS_EXHAUSTED = 1
+PVS_ERR_INVALID = -1
+PVS_ERR_NONFINITE = -2
+PVS_ERR_OVERFLOW = -3
+PVS_ERR_INTERVAL = -4
+PVS_ERR_CUDA = -5
+PVS_ERR_OOM = -6
+PVS_ERR_TIMEOUT = -7
+PVS_ERR_FAILED = -8
+
+EAHR_RANK_SCALED = 0
+EAHR_NUMERATOR = 1
+EAHR_POLICY_GEOMETRIC = 0
+EAHR_POLICY_EQUAL_DEPTH = 1
+
+
+class PvsError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {pvs_status_string(status)} ({status})")
+
+
+class pvs_stats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "visible", "emitted", "refined", "exact_fallbacks", "interval_passes",
+        "horizon_builds", "pulls", "candidates", "code_bytes")] + [
+        ("state", ctypes.c_int32), ("reserved", ctypes.c_int32),
+        ("interval_ms", ctypes.c_double)]
+
+
+class eahr_params(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("k", ctypes.c_int32), ("form", ctypes.c_int32),
+                ("policy", ctypes.c_int32), ("step", ctypes.c_int32),
+                ("w_num", ctypes.c_int32 * 2), ("w_den", ctypes.c_int32 * 2)]
+
+
+class eahr_stats(ctypes.Structure):
+    _fields_ = [("depth", ctypes.c_int64 * 2), ("length", ctypes.c_int64 * 2),
+                ("exhausted", ctypes.c_int32 * 2), ("pulls", ctypes.c_int32 * 2),
+                ("checks", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(
+            f"libpvs.so not found at {_LIB_PATH}; build it with "
+            "`python -c 'import __graft_entry__ as g; g.build()'` (needs nvcc)")
+    L = ctypes.CDLL(_LIB_PATH)
+    P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    pp = ctypes.POINTER(ctypes.c_void_p)
+    sig = {
+        "pvs_build": (i32, [P, i64, i32, i32, P, pp]),
+        "pvs_append": (i32, [P, P, i64, i32]),
+        "pvs_tombstone": (i32, [P, P, i64]),
+        "pvs_index_size": (i64, [P]),
+        "pvs_index_live": (i64, [P]),
+        "pvs_index_dim": (i32, [P]),
+        "pvs_index_export": (i32, [P, i64, i64, P, P, P, P]),
+        "pvs_index_free": (None, [P]),
+        "pvs_snapshot_create": (i32, [P, pp]),
+        "pvs_snapshot_visible": (i64, [P]),
+        "pvs_snapshot_free": (None, [P]),
+        "pvs_cursor_open": (i32, [P, P, P, i32, pp]),
+        "pvs_cursor_open_batch": (i32, [P, P, P, i32, i32, i32, pp]),
+        "pvs_next": (i32, [P, i32, P, P, P]),
+        "pvs_next_device": (i32, [P, i32, P, P, P]),
+        "pvs_cursor_sync": (i32, [P]),
+        "pvs_cursor_stats": (i32, [P, ctypes.POINTER(pvs_stats)]),
+        "pvs_cursor_bounds": (i32, [P, i64, i64, P, P]),
+        "pvs_cursor_score_ids": (i32, [P, P, i32, P]),
+        "pvs_cursor_close": (None, [P]),
+        "pvs_status_string": (ctypes.c_char_p, [i32]),
+        "pvs_launch_count": (i64, []),
+        "eahr_topk": (i32, [P, P, i64, ctypes.POINTER(eahr_params), P, P, P,
+                            ctypes.POINTER(eahr_stats)]),
+        "eahr_topk_lists": (i32, [P, i64, P, i64, ctypes.POINTER(eahr_params), P, P, P,
+                                  ctypes.POINTER(eahr_stats)]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(L, name)
+        f.restype = res
+        f.argtypes = args
+    return L
+
+
+_lib = _load()
+lib_path = _LIB_PATH
+EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_index_live",
+            "pvs_index_dim", "pvs_index_export", "pvs_index_free", "pvs_snapshot_create",
+            "pvs_snapshot_visible", "pvs_snapshot_free", "pvs_cursor_open",
+            "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
+            "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
+            "pvs_status_string", "pvs_launch_count", "eahr_topk", "eahr_topk_lists")
+
+
+def pvs_status_string(status: int) -> str:
+    return _lib.pvs_status_string(int(status)).decode()
+
+
+def pvs_launch_count() -> int:
+    return int(_lib.pvs_launch_count())
+
+
+def _check(status: int, where: str) -> int:
+    if status < 0:
+        raise PvsError(status, where)
+    return status
+
+
+def _vec_arg(x, dim: int | None = None):
+    """(pointer, rows, dim, on_device, keepalive) for numpy or torch input."""
+    try:
+        import torch
+    except ImportError:  # pragma: no cover
+        torch = None
+    if torch is not None and isinstance(x, torch.Tensor):
+        if x.dtype != torch.float32:
+            raise TypeError("vectors must be float32")
+        x = x.contiguous()
+        on_dev = 1 if x.is_cuda else 0
+        if x.is_cuda:
+            torch.cuda.current_stream(x.device).synchronize()
+        shape = tuple(x.shape)
+        return ctypes.c_void_p(x.data_ptr()), shape, on_dev, x
+    a = np.ascontiguousarray(x, dtype=np.float32)
+    return ctypes.c_void_p(a.ctypes.data), a.shape, 0, a
+
+
+def pvs_build(vecs, stream=None):
+    """Build an index over the rows of a 2-D float32 array / tensor."""
+    ptr, shape, on_dev, keep = _vec_arg(vecs)
+    n, dim = (shape[0], shape[1]) if len(shape) == 2 else (0, shape[-1])
+    out = ctypes.c_void_p()
+    st = ctypes.c_void_p(stream) if stream else None
+    _check(_lib.pvs_build(ptr, n, dim, on_dev, st, ctypes.byref(out)), "pvs_build")
+    return out
+
+
+def pvs_append(index, vecs) -> None:
+    ptr, shape, on_dev, keep = _vec_arg(vecs)
+    _check(_lib.pvs_append(index, ptr, shape[0], on_dev), "pvs_append")
+
+
+def pvs_tombstone(index, ids) -> None:
+    a = np.ascontiguousarray(ids, dtype=np.int64)
+    _check(_lib.pvs_tombstone(index, a.ctypes.data, a.size), "pvs_tombstone")
+
+
+def pvs_index_size(index) -> int:
+    return int(_lib.pvs_index_size(index))
+
+
+def pvs_index_live(index) -> int:
+    return int(_lib.pvs_index_live(index))
+
+
+def pvs_index_dim(index) -> int:
+    return int(_lib.pvs_index_dim(index))
+
+
+def pvs_index_export(index, first: int, count: int):
+    dim = pvs_index_dim(index)
+    codes = np.zeros((count, dim), np.int8)
+    scale = np.zeros(count, np.float32)
+    vnorm = np.zeros(count, np.float32)
+    enorm = np.zeros(count, np.float32)
+    _check(_lib.pvs_index_export(index, first, count, codes.ctypes.data, scale.ctypes.data,
+                                 vnorm.ctypes.data, enorm.ctypes.data), "pvs_index_export")
+    return codes, scale, vnorm, enorm
+
+
+def pvs_index_free(index) -> None:
+    _lib.pvs_index_free(index)
+
+
+def pvs_snapshot_create(index):
+    out = ctypes.c_void_p()
+    _check(_lib.pvs_snapshot_create(index, ctypes.byref(out)), "pvs_snapshot_create")
+    return out
+
+
+def pvs_snapshot_visible(snap) -> int:
+    return int(_lib.pvs_snapshot_visible(snap))
+
+
+def pvs_snapshot_free(snap) -> None:
+    _lib.pvs_snapshot_free(snap)
+
+
+def pvs_cursor_open(index, query, snap=None):
+    ptr, shape, on_dev, keep = _vec_arg(query)
+    out = ctypes.c_void_p()
+    _check(_lib.pvs_cursor_open(index, snap, ptr, on_dev, ctypes.byref(out)), "pvs_cursor_open")
+    return out
+
+
+def pvs_cursor_open_batch(index, queries, horizon: int, snap=None):
+    ptr, shape, on_dev, keep = _vec_arg(queries)
+    nq = shape[0]
+    arr = (ctypes.c_void_p * max(nq, 1))()
+    _check(_lib.pvs_cursor_open_batch(index, snap, ptr, nq, on_dev, int(horizon),
+                                      ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))),
+           "pvs_cursor_open_batch")
+    return [ctypes.c_void_p(arr[i]) for i in range(nq)]
+
+
+def pvs_next(cursor, n: int):
+    """Next n exact ranks -> (ids int64[n_out], scores float32[n_out], status)."""
+    ids = np.zeros(max(n, 1), np.int64)
+    sc = np.zeros(max(n, 1), np.float32)
+    got = ctypes.c_int32(0)
+    st = _check(_lib.pvs_next(cursor, int(n), ids.ctypes.data, sc.ctypes.data,
+                              ctypes.byref(got)), "pvs_next")
+    return ids[:got.value], sc[:got.value], st
+
+
+def pvs_next_device(cursor, n: int, ids, scores):
+    """Enqueue the next n ranks into CUDA tensors ids (int64) / scores
+    (float32); returns (n_out, status)."""
+    got = ctypes.c_int32(0)
+    st = _check(_lib.pvs_next_device(cursor, int(n), ctypes.c_void_p(ids.data_ptr()),
+                                     ctypes.c_void_p(scores.data_ptr()), ctypes.byref(got)),
+                "pvs_next_device")
+    return got.value, st
+
+
+def pvs_cursor_sync(cursor) -> int:
+    return _check(_lib.pvs_cursor_sync(cursor), "pvs_cursor_sync")
+
+
+def pvs_cursor_stats(cursor) -> dict:
+    s = pvs_stats()
+    _check(_lib.pvs_cursor_stats(cursor, ctypes.byref(s)), "pvs_cursor_stats")
+    return {name: getattr(s, name) for name, _ in pvs_stats._fields_ if name != "reserved"}
+
+
+def pvs_cursor_bounds(cursor, first: int, count: int):
+    lo = np.zeros(max(count, 1), np.float32)
+    hi = np.zeros(max(count, 1), np.float32)
+    _check(_lib.pvs_cursor_bounds(cursor, first, count, lo.ctypes.data, hi.ctypes.data),
+           "pvs_cursor_bounds")
+    return lo[:count], hi[:count]
+
+
+def pvs_cursor_score_ids(cursor, ids):
+    a = np.ascontiguousarray(ids, dtype=np.int64)
+    out = np.zeros(max(a.size, 1), np.float32)
+    _check(_lib.pvs_cursor_score_ids(cursor, a.ctypes.data, a.size, out.ctypes.data),
+           "pvs_cursor_score_ids")
+    return out[:a.size]
+
+
+def pvs_cursor_close(cursor) -> None:
+    _lib.pvs_cursor_close(cursor)
+
+
+def _params(K, k, form, policy, step, weights):
+    p = eahr_params()
+    p.K, p.k, p.form, p.policy, p.step = int(K), int(k), int(form), int(policy), int(step)
+    for i, w in enumerate(weights):
+        num, den = (w, 1) if np.isscalar(w) else w
+        p.w_num[i], p.w_den[i] = int(num), int(den)
+    return p
+
+
+def _eahr_result(st, ids, F, got, stats):
+    s = {"depth": list(stats.depth), "length": list(stats.length),
+         "exhausted": list(stats.exhausted), "pulls": list(stats.pulls),
+         "checks": stats.checks}
+    return ids[:got.value], F[:got.value], s
+
+
+def eahr_topk(cursor, sparse_ids, K: int = 20, k: int = 60, form: int = EAHR_NUMERATOR,
+              policy: int = EAHR_POLICY_GEOMETRIC, step: int = 0, weights=(1, 1)):
+    """Ordered Top-K of complete-list weighted RRF (dense cursor + host sparse
+    ranking) -> (ids int64[q_K], F float64[q_K], stats)."""
+    sp = np.ascontiguousarray(sparse_ids, dtype=np.int64)
+    p = _params(K, k, form, policy, step, weights)
+    ids = np.zeros(K, np.int64)
+    F = np.zeros(K, np.float64)
+    got = ctypes.c_int32(0)
+    stats = eahr_stats()
+    _check(_lib.eahr_topk(cursor, sp.ctypes.data, sp.size, ctypes.byref(p), ids.ctypes.data,
+                          F.ctypes.data, ctypes.byref(got), ctypes.byref(stats)), "eahr_topk")
+    return _eahr_result(0, ids, F, got, stats)
+
+
+def eahr_topk_lists(list0, list1, K: int = 20, k: int = 60, form: int = EAHR_RANK_SCALED,
+                    policy: int = EAHR_POLICY_GEOMETRIC, step: int = 0, weights=(1, 1)):
+    a = np.ascontiguousarray(list0, dtype=np.int64)
+    b = np.ascontiguousarray(list1, dtype=np.int64)
+    p = _params(K, k, form, policy, step, weights)
+    ids = np.zeros(K, np.int64)
+    F = np.zeros(K, np.float64)
+    got = ctypes.c_int32(0)
+    stats = eahr_stats()
+    _check(_lib.eahr_topk_lists(a.ctypes.data, a.size, b.ctypes.data, b.size, ctypes.byref(p),
+                                ids.ctypes.data, F.ctypes.data, ctypes.byref(got),
+                                ctypes.byref(stats)), "eahr_topk_lists")
+    return _eahr_result(0, ids, F, got, stats)

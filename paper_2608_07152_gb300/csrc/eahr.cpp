@@ -1,0 +1,435 @@
+// EAHR host driver (arXiv 2608.07152, Sec. 2.1 and 2.2): ordered Top-K of
+// complete-list weighted RRF, read adaptively from two resumable exact
+// ranked lists.
+//
+// Bounds (Sec. 2.2), all exact rationals:
+//   u_i = g_i(d_i + 1) for an Open list, 0 for an Exhausted one;
+//   L(x) = sum of the contributions already read; U(x) = L(x) + u_i for every
+//   Open list i that has not returned x; B = u_0 + u_1.
+// Certification: x+ = argmax over R = O \ A of (L, -id) is appended when its
+// (L, id) beats (U(y), y) for every other y in R and L(x+) > B.
+//
+// With two lists every bound is a sum of at most two contributions
+// a / (b r + c) with denominators below 2^32, so numerators stay below 2^49,
+// denominators below 2^64, and comparisons are exact in 128-bit integers.
+//
+// Incremental structures: items read from both lists sit in an ordered set
+// keyed by (F desc, id asc); items read from one list only are ordered by
+// their rank in that list (their L and U are monotone in it), so the best
+// and second-best of each group are found without scanning O.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <limits>
+#include <new>
+#include <set>
+#include <vector>
+
+#include "../../include/pvs.h"
+#include "runtime.h"
+
+namespace {
+
+typedef unsigned __int128 u128;
+
+struct Frac {
+    uint64_t num = 0, den = 1;
+};
+
+inline int cmp(const Frac& a, const Frac& b) {
+    const u128 l = (u128)a.num * b.den, r = (u128)b.num * a.den;
+    return l < r ? -1 : (l > r ? 1 : 0);
+}
+
+inline Frac add(const Frac& a, const Frac& b) {
+    if (a.num == 0) return b;
+    if (b.num == 0) return a;
+    Frac s;
+    s.num = a.num * b.den + b.num * a.den;
+    s.den = a.den * b.den;
+    return s;
+}
+
+inline int bitlen(u128 x) {
+    int n = 0;
+    while (x) {
+        ++n;
+        x >>= 1;
+    }
+    return n;
+}
+
+// Correctly rounded (nearest, ties to even) binary64 value of num / den.
+double frac_to_double(const Frac& f) {
+    if (f.num == 0) return 0.0;
+    const int s = 55 + bitlen(f.den) - bitlen(f.num);
+    const u128 n = (u128)f.num << s;
+    u128 q = n / f.den;
+    const bool rem = (n % f.den) != 0;
+    const int drop = bitlen(q) - 53;               // 2 or 3
+    const u128 mask = ((u128)1 << drop) - 1;
+    const u128 low = q & mask, half = (u128)1 << (drop - 1);
+    u128 mant = q >> drop;
+    if (low > half || (low == half && (rem || (mant & 1)))) ++mant;
+    return std::ldexp((double)(uint64_t)mant, drop - s);
+}
+
+// g(r) = a / (b r + c)
+struct Contrib {
+    uint64_t a = 0, b = 1, c = 0;
+    Frac at(int64_t r) const {
+        Frac f;
+        if (a == 0) return f;
+        f.num = a;
+        f.den = b * (uint64_t)r + c;
+        return f;
+    }
+};
+
+struct Node {
+    Frac F;
+    int32_t id;
+};
+struct NodeCmp {
+    bool operator()(const Node& x, const Node& y) const {
+        const int c = cmp(x.F, y.F);
+        if (c != 0) return c > 0;     // larger F first
+        return x.id < y.id;           // then smaller id
+    }
+};
+
+// (a, x) beats (b, y): a > b, or a == b and x has the smaller id.
+inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
+    const int c = cmp(a, b);
+    return c > 0 || (c == 0 && x < y);
+}
+
+struct Source {
+    // dense cursor or host list
+    pvs_cursor* cursor = nullptr;
+    const int64_t* list = nullptr;
+    int64_t length = 0;
+};
+
+class Driver {
+  public:
+    Contrib g[2];
+    Source src[2];
+    bool active[2] = {true, true};   // positive weight
+    int64_t depth[2] = {0, 0};
+    bool exhausted[2] = {false, false};
+    int32_t pulls[2] = {0, 0};
+    int32_t checks = 0;
+    std::vector<int32_t> prefix[2];
+    int32_t* rank[2] = {nullptr, nullptr};   // rank of id in list i (0: unread)
+    uint8_t* inA = nullptr;
+    int64_t id_space = 0;
+    std::set<Node, NodeCmp> both;
+    size_t ptr[2] = {0, 0};
+    std::vector<int32_t> A;
+    int K = 0;
+    std::vector<int64_t> buf_ids;
+    std::vector<float> buf_scores;
+    const pvs::SnapData* snap = nullptr;
+
+    ~Driver() {
+        std::free(rank[0]);
+        std::free(rank[1]);
+        std::free(inA);
+    }
+
+    bool init(int64_t ids) {
+        id_space = std::max<int64_t>(ids, 1);
+        rank[0] = static_cast<int32_t*>(std::calloc((size_t)id_space, sizeof(int32_t)));
+        rank[1] = static_cast<int32_t*>(std::calloc((size_t)id_space, sizeof(int32_t)));
+        inA = static_cast<uint8_t*>(std::calloc((size_t)id_space, 1));
+        return rank[0] && rank[1] && inA;
+    }
+
+    Frac u(int i) const {
+        if (!active[i] || exhausted[i]) return Frac{};
+        return g[i].at(depth[i] + 1);
+    }
+
+    Frac L(int32_t x) const {
+        Frac f;
+        if (active[0] && rank[0][x]) f = add(f, g[0].at(rank[0][x]));
+        if (active[1] && rank[1][x]) f = add(f, g[1].at(rank[1][x]));
+        return f;
+    }
+
+    Frac U(int32_t x) const {
+        Frac f = L(x);
+        for (int i = 0; i < 2; ++i)
+            if (active[i] && !exhausted[i] && !rank[i][x]) f = add(f, u(i));
+        return f;
+    }
+
+    // Record ranks depth+1 .. depth+n of list i.  Ids from host lists are
+    // checked as they are read: inside the id space, visible in the
+    // snapshot (when there is one) and not repeated within the list.
+    bool record(int i, const int64_t* ids, int64_t n) {
+        const int j = 1 - i;
+        const bool check = src[i].cursor == nullptr;
+        for (int64_t t = 0; t < n; ++t) {
+            const int64_t x64 = ids[t];
+            if (check) {
+                if (x64 < 0 || x64 >= id_space) return false;
+                if (snap && !snap->is_visible(x64)) return false;
+                if (rank[i][x64]) return false;
+            }
+            const int32_t x = (int32_t)x64;
+            prefix[i].push_back(x);
+            rank[i][x] = (int32_t)(depth[i] + t + 1);
+            if (active[j] && rank[j][x] && !inA[x]) both.insert(Node{L(x), x});
+        }
+        depth[i] += n;
+        return true;
+    }
+
+    // First item of list i, at or after position `from` of its prefix, that
+    // is read from list i only and not fixed; -1 if none.
+    int32_t only_from(int i, size_t from, int32_t skip) const {
+        const int j = 1 - i;
+        for (size_t p = from; p < prefix[i].size(); ++p) {
+            const int32_t x = prefix[i][p];
+            if (inA[x] || x == skip) continue;
+            if (active[j] && rank[j][x]) continue;
+            return x;
+        }
+        return -1;
+    }
+
+    void advance_ptr(int i) {
+        const int j = 1 - i;
+        while (ptr[i] < prefix[i].size()) {
+            const int32_t x = prefix[i][ptr[i]];
+            if (inA[x] || (active[j] && rank[j][x])) {
+                ++ptr[i];
+                continue;
+            }
+            break;
+        }
+    }
+
+    // Sec. 2.2 certification; returns true when the result is complete.
+    bool certify() {
+        ++checks;
+        const Frac B = add(u(0), u(1));
+        while ((int)A.size() < K) {
+            advance_ptr(0);
+            advance_ptr(1);
+            // candidates for x+
+            int32_t cand[3] = {-1, -1, -1};
+            if (!both.empty()) cand[0] = both.begin()->id;
+            if (active[0]) cand[1] = only_from(0, ptr[0], -1);
+            if (active[1]) cand[2] = only_from(1, ptr[1], -1);
+            int32_t xp = -1;
+            Frac Lx;
+            for (int t = 0; t < 3; ++t) {
+                if (cand[t] < 0) continue;
+                const Frac l = L(cand[t]);
+                if (xp < 0 || beats(l, cand[t], Lx, xp)) {
+                    xp = cand[t];
+                    Lx = l;
+                }
+            }
+            if (xp < 0) return B.num == 0;   // R empty
+            // strongest other item by (U, id)
+            int32_t others[3] = {-1, -1, -1};
+            if (!both.empty()) {
+                auto it = both.begin();
+                if (it->id == xp) ++it;
+                if (it != both.end()) others[0] = it->id;
+            }
+            if (active[0]) others[1] = only_from(0, ptr[0], xp);
+            if (active[1]) others[2] = only_from(1, ptr[1], xp);
+            bool ok = cmp(Lx, B) > 0;
+            for (int t = 0; t < 3 && ok; ++t)
+                if (others[t] >= 0) ok = beats(Lx, xp, U(others[t]), others[t]);
+            if (!ok) {
+                // complete when nothing left can have a positive score
+                if (B.num != 0) return false;
+                return Lx.num == 0;
+            }
+            A.push_back(xp);
+            inA[xp] = 1;
+            if (active[0] && active[1] && rank[0][xp] && rank[1][xp]) both.erase(Node{Lx, xp});
+        }
+        return true;
+    }
+
+    // Pull up to n ranks from list i.
+    pvs_status pull(int i, int64_t n) {
+        if (exhausted[i] || !active[i]) return PVS_OK;
+        pulls[i]++;
+        if (src[i].cursor) {
+            if (n > (int64_t)std::numeric_limits<int32_t>::max()) n = std::numeric_limits<int32_t>::max();
+            buf_ids.resize((size_t)n);
+            buf_scores.resize((size_t)n);
+            int32_t got = 0;
+            pvs_status s = pvs_next(src[i].cursor, (int32_t)n, buf_ids.data(), buf_scores.data(), &got);
+            if (s < 0) return s;
+            record(i, buf_ids.data(), got);
+            if (s == PVS_EXHAUSTED) exhausted[i] = true;
+        } else {
+            const int64_t take = std::min<int64_t>(n, src[i].length - depth[i]);
+            if (!record(i, src[i].list + depth[i], take)) return PVS_ERR_INVALID;
+            if (depth[i] == src[i].length) exhausted[i] = true;
+        }
+        if (depth[i] >= src[i].length) exhausted[i] = true;
+        return PVS_OK;
+    }
+};
+
+bool contrib_from(const eahr_params* p, int i, int64_t max_rank, Contrib* out) {
+    const int64_t wn = p->w_num[i], wd = p->w_den[i];
+    if (wn < 0 || wn >= (1 << 16) || wd < 1 || wd >= (1 << 16)) return false;
+    Contrib c;
+    c.a = (uint64_t)wn;
+    c.b = (uint64_t)wd;
+    if (p->form == EAHR_RANK_SCALED)
+        c.c = (uint64_t)(p->k - 1) * (uint64_t)wn;     // 1/(r q/p + k - 1) = p/(q r + (k-1) p)
+    else
+        c.c = (uint64_t)wd * (uint64_t)p->k;           // (p/q)/(k + r) = p/(q r + q k)
+    if (c.a == 0) c.c = 0;
+    // denominators must stay below 2^32 up to rank max_rank + 1
+    const u128 dmax = (u128)c.b * (u128)(max_rank + 1) + c.c;
+    if (dmax >= ((u128)1 << 32) || (c.a != 0 && c.b * 1 + c.c == 0)) return false;
+    *out = c;
+    return true;
+}
+
+pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F, int32_t* n_out,
+               eahr_stats* st) {
+    const int step0 = p->step > 0 ? p->step : 16;
+    int64_t size[2] = {step0, step0};
+    d.K = p->K;
+    for (int i = 0; i < 2; ++i)
+        if (!d.active[i]) d.exhausted[i] = false;
+    // lists with zero weight contribute nothing and are never read
+    bool done = false;
+    if (!d.active[0] && !d.active[1]) done = true;
+    while (!done) {
+        if (p->policy == EAHR_POLICY_EQUAL_DEPTH) {
+            for (int i = 0; i < 2; ++i) {
+                pvs_status s = d.pull(i, step0);
+                if (s < 0) return s;
+            }
+        } else {
+            // the list whose next unread rank can still contribute more
+            int pick = -1;
+            for (int i = 0; i < 2; ++i) {
+                if (!d.active[i] || d.exhausted[i]) continue;
+                if (pick < 0) {
+                    pick = i;
+                    continue;
+                }
+                const int c = cmp(d.u(i), d.u(pick));
+                if (c > 0 || (c == 0 && d.depth[i] < d.depth[pick])) pick = i;
+            }
+            if (pick >= 0) {
+                pvs_status s = d.pull(pick, size[pick]);
+                if (s < 0) return s;
+                size[pick] = std::min<int64_t>(2 * size[pick], (int64_t)1 << 24);
+            }
+        }
+        done = d.certify();
+        if (!done) {
+            bool any_open = false;
+            for (int i = 0; i < 2; ++i) any_open |= d.active[i] && !d.exhausted[i];
+            if (!any_open) done = true;   // cannot happen: exhausted lists decide
+        }
+    }
+    const int32_t q = (int32_t)d.A.size();
+    for (int32_t t = 0; t < q; ++t) {
+        const int32_t x = d.A[t];
+        out_ids[t] = x;
+        if (out_F) {
+            bool determined = true;
+            for (int i = 0; i < 2; ++i)
+                if (d.active[i] && !d.exhausted[i] && !d.rank[i][x]) determined = false;
+            out_F[t] = determined ? frac_to_double(d.L(x)) : std::nan("");
+        }
+    }
+    *n_out = q;
+    if (st) {
+        for (int i = 0; i < 2; ++i) {
+            st->depth[i] = d.depth[i];
+            st->length[i] = d.src[i].length;
+            st->exhausted[i] = d.exhausted[i] ? 1 : 0;
+            st->pulls[i] = d.pulls[i];
+        }
+        st->checks = d.checks;
+        st->reserved = 0;
+    }
+    return PVS_OK;
+}
+
+bool params_ok(const eahr_params* p) {
+    return p && p->K >= 1 && p->k >= 1 && (p->form == EAHR_RANK_SCALED || p->form == EAHR_NUMERATOR) &&
+           (p->policy == EAHR_POLICY_GEOMETRIC || p->policy == EAHR_POLICY_EQUAL_DEPTH) &&
+           p->step >= 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+pvs_status eahr_topk(pvs_cursor* dense, const int64_t* sparse_ids, int64_t n_sparse,
+                     const eahr_params* p, int64_t* out_ids, double* out_F, int32_t* n_out,
+                     eahr_stats* st) {
+    if (n_out) *n_out = 0;
+    if (!dense || !params_ok(p) || !out_ids || !n_out || n_sparse < 0 ||
+        (n_sparse > 0 && !sparse_ids))
+        return PVS_ERR_INVALID;
+    if (pvs::cursor_emitted(dense) != 0) return PVS_ERR_INVALID;
+    const pvs::SnapData* snap = pvs::cursor_snapshot(dense);
+    const int64_t id_space = snap->rows;
+    if (n_sparse > snap->visible) return PVS_ERR_INVALID;
+    Driver d;
+    d.snap = snap;
+    d.src[0].cursor = dense;
+    d.src[0].length = pvs::cursor_visible(dense);
+    d.src[1].list = sparse_ids;
+    d.src[1].length = n_sparse;
+    for (int i = 0; i < 2; ++i) {
+        if (!contrib_from(p, i, d.src[i].length, &d.g[i])) return PVS_ERR_INVALID;
+        d.active[i] = d.g[i].a != 0;
+        if (d.src[i].length == 0) d.exhausted[i] = true;
+    }
+    if (!d.init(id_space)) return PVS_ERR_OOM;
+    return run(d, p, out_ids, out_F, n_out, st);
+}
+
+pvs_status eahr_topk_lists(const int64_t* list0, int64_t n0, const int64_t* list1, int64_t n1,
+                           const eahr_params* p, int64_t* out_ids, double* out_F, int32_t* n_out,
+                           eahr_stats* st) {
+    if (n_out) *n_out = 0;
+    if (!params_ok(p) || !out_ids || !n_out || n0 < 0 || n1 < 0 || (n0 > 0 && !list0) ||
+        (n1 > 0 && !list1))
+        return PVS_ERR_INVALID;
+    int64_t id_space = 0;
+    for (int64_t t = 0; t < n0; ++t) id_space = std::max<int64_t>(id_space, list0[t] + 1);
+    for (int64_t t = 0; t < n1; ++t) id_space = std::max<int64_t>(id_space, list1[t] + 1);
+    for (int64_t t = 0; t < n0; ++t)
+        if (list0[t] < 0) return PVS_ERR_INVALID;
+    for (int64_t t = 0; t < n1; ++t)
+        if (list1[t] < 0) return PVS_ERR_INVALID;
+    if (id_space > ((int64_t)1 << 31)) return PVS_ERR_INVALID;
+    Driver d;
+    d.src[0].list = list0;
+    d.src[0].length = n0;
+    d.src[1].list = list1;
+    d.src[1].length = n1;
+    for (int i = 0; i < 2; ++i) {
+        if (!contrib_from(p, i, d.src[i].length, &d.g[i])) return PVS_ERR_INVALID;
+        d.active[i] = d.g[i].a != 0;
+        if (d.src[i].length == 0) d.exhausted[i] = true;
+    }
+    if (!d.init(id_space)) return PVS_ERR_OOM;
+    return run(d, p, out_ids, out_F, n_out, st);
+}
+
+}  // extern "C"

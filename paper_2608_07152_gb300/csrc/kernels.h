@@ -1,0 +1,121 @@
+// Host-side launchers of the PVS device kernels (internal to libpvs.so).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pvs {
+
+// Process-wide count of kernels launched by the library (pvs_launch_count).
+void count_launches(int k);
+
+constexpr int kTileRows = 64;         // rows per interval-pass tile
+constexpr int kCodeAlign = 64;        // code rows padded to a multiple of 64 bytes
+constexpr int kMaxDim = 32767;
+
+// Encoded query scalars (Sec. 2.3.1, App. A.1).
+struct QueryScalars {
+    float s;       // s_q
+    float qnorm;   // ||q||_2 rounded up
+    float qhat;    // ||s_q z_q||_2 rounded up
+    float enorm;   // ||q - s_q z_q||_2 rounded up
+    float gamma;   // gamma_m
+    int status;    // PVS status of the encoding
+};
+
+// Radix-select state for the k-th largest ordered key.
+struct SelectState {
+    uint64_t prefix;     // decided high bits of the key
+    uint64_t k;          // remaining rank among keys that match the prefix
+    uint32_t hist[256];
+};
+
+// Per-cursor device counters.
+struct DevCounters {
+    unsigned long long refined;
+    unsigned long long exact_fallbacks;
+    unsigned int w_len;      // working-set length
+    unsigned int cand;       // candidates of the current pull
+};
+
+// ---- build / encode (build_kernels.cu) -------------------------------------
+// Quantize rows [0, n) of `vecs` (row stride m floats) into codes (stride
+// m_pad), params, and a raw copy (stride m_raw, zero padded).
+cudaError_t launch_build(const float* vecs, int64_t n, int m, int m_pad, int m_raw,
+                         int8_t* codes, float* scale, float* vnorm, float* enorm, float* raw,
+                         int* status, cudaStream_t st);
+// Encode one query: codes zq[m_pad], raw copy qraw[m_raw], scalars.
+cudaError_t launch_encode_query(const float* q, int m, int m_pad, int m_raw, int8_t* zq,
+                                float* qraw, QueryScalars* qs, cudaStream_t st);
+// Encode nq queries (row stride m), one warp each.
+cudaError_t launch_encode_queries(const float* q, int nq, int m, int m_pad, int m_raw,
+                                  int8_t* zq, float* qraw, QueryScalars* qs, cudaStream_t st);
+
+// ---- interval pass (interval_kernels.cu) ------------------------------------
+struct IntervalArgs {
+    const int8_t* codes;
+    const float* scale;
+    const float* vnorm;
+    const float* enorm;
+    const uint32_t* tomb;   // tombstone bitmap of the snapshot, or null
+    int64_t rows;           // rows [0, rows) are scanned
+    int m_pad;
+    const int8_t* zq;
+    const QueryScalars* qs;
+    float* lo;
+    float* hi;
+    int* status;
+};
+cudaError_t launch_interval_pass(const IntervalArgs& a, int num_sms, cudaStream_t st);
+// Plain reference-style variant without staging (used for tiny inputs).
+cudaError_t launch_interval_simple(const IntervalArgs& a, cudaStream_t st);
+
+// ---- selection / compaction / sort (select_kernels.cu) ----------------------
+// k-th largest key (1-based) among live entries of a float array: key of
+// vals[i] with vals[i] != -inf, i < *len (len in device memory).  Result in
+// sel->prefix (as a 32-bit ordered key).  k must be <= live count.
+cudaError_t launch_select_f32(const float* vals, const unsigned int* len, uint64_t k,
+                              SelectState* sel, int grid, cudaStream_t st);
+// Same over `rows` entries with a host-known length.
+cudaError_t launch_select_f32_n(const float* vals, int64_t rows, uint64_t k, SelectState* sel,
+                                int grid, cudaStream_t st);
+// Ordered compaction: for i < rows with lo[i] != -inf and key(hi[i]) >=
+// sel->prefix, append (i, lo, hi) to (w_id, w_lo, w_hi) in index order;
+// writes the count to *w_len.  `scratch` holds >= compact_scratch(rows) uints.
+size_t compact_scratch_elems(int64_t rows);
+cudaError_t launch_compact_ordered(const float* lo, const float* hi, int64_t rows,
+                                   const SelectState* sel, int32_t* w_id, float* w_lo,
+                                   float* w_hi, unsigned int* w_len, unsigned int* scratch,
+                                   cudaStream_t st);
+// Candidates of a pull: i < *w_len, live, key(w_hi[i]) >= sel->prefix ->
+// cand[] (unordered), count in *cand_len (zeroed by the launcher).
+cudaError_t launch_candidates(const float* w_lo, const float* w_hi, const unsigned int* w_len,
+                              const SelectState* sel, int32_t* cand, unsigned int* cand_len,
+                              int grid, cudaStream_t st);
+// keys[i] = rank_key(w_lo[cand[i]], cand[i]) for i < *cand_len.
+cudaError_t launch_make_keys(const int32_t* cand, const unsigned int* cand_len,
+                             const float* w_lo, uint64_t* keys, int grid, cudaStream_t st);
+// Sort `count` 64-bit keys descending, in place (count <= kBitonicMax).
+constexpr int kBitonicMax = 8192;
+cudaError_t launch_bitonic_desc(uint64_t* keys, int count, cudaStream_t st);
+// LSD radix sort of `count` 64-bit keys descending; result in keys.
+size_t radix_sort_scratch_bytes(int64_t count);
+cudaError_t launch_radix_sort_desc(uint64_t* keys, uint64_t* tmp, int64_t count, void* scratch,
+                                   cudaStream_t st);
+// Emit the first n sorted keys: ids/scores out (device), mark emitted.
+cudaError_t launch_emit(const uint64_t* keys, int n, const int32_t* w_id, float* w_lo,
+                        float* w_hi, float* lo, float* hi, int64_t* out_ids, float* out_scores,
+                        cudaStream_t st);
+
+// ---- refinement (refine_kernels.cu) -----------------------------------------
+// Authoritative score of every unresolved candidate (w_lo < w_hi): exact
+// RN_f32(sum_j q_j v_j), containment check, then w_lo = w_hi = lo = hi = s.
+cudaError_t launch_refine(const int32_t* cand, const unsigned int* cand_len,
+                          const int32_t* w_id, float* w_lo, float* w_hi, float* lo, float* hi,
+                          const float* qraw, const float* raw, int m_raw, int* status,
+                          DevCounters* ctr, int grid, cudaStream_t st);
+// Authoritative scores of explicit ids (tests / diagnostics).
+cudaError_t launch_score_ids(const int64_t* ids, int n, const float* qraw, const float* raw,
+                             int m_raw, float* out, DevCounters* ctr, cudaStream_t st);
+
+}  // namespace pvs

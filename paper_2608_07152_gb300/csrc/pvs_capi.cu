@@ -1,0 +1,705 @@
+// C ABI of libpvs.so: index build / append / tombstone, snapshots, cursors
+// and the pull orchestration of PVS resumable exact ranking
+// (arXiv 2608.07152, Sec. 2.1, 2.3.1, 2.4, App. A.1).
+//
+// Pull of n ranks (Sec. 2.3.1: candidates in decreasing interval upper
+// bound, raw vectors read only where intervals do not decide):
+//   1. first pull: one interval pass over the Int8 codes -> lo[i], hi[i];
+//   2. working set W: tau_H = H-th largest lo among live rows, W = {live rows
+//      with hi >= tau_H} in id order; W holds the next H ranks (every item
+//      outside W is preceded by the >= H items with lo >= tau_H);
+//   3. per pull: tau = n-th largest lo in W; candidates C = {hi >= tau}; score
+//      the unresolved candidates exactly (lo = hi = s afterwards); C contains
+//      the next n ranks, which are its n largest (score, -id) keys;
+//   4. emit them in order and mark them emitted (lo = hi = -inf).
+//   W is rebuilt with a doubled horizon when a pull would go past it.
+#include <algorithm>
+#include <atomic>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+
+#include "runtime.h"
+
+using namespace pvs;
+
+namespace pvs {
+
+static std::atomic<long long> g_launches{0};
+void count_launches(int k) { g_launches.fetch_add(k, std::memory_order_relaxed); }
+
+SnapData::~SnapData() {
+    if (d_tomb) cudaFree(d_tomb);
+}
+
+int64_t cursor_visible(const pvs_cursor* c) { return c->visible; }
+int64_t cursor_emitted(const pvs_cursor* c) { return c->emitted; }
+const SnapData* cursor_snapshot(const pvs_cursor* c) { return c->snap.get(); }
+
+}  // namespace pvs
+
+namespace {
+
+constexpr size_t kStageBytes = size_t(1) << 30;   // host-input staging chunk
+
+inline int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+pvs_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return PVS_OK;
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return PVS_ERR_OOM;
+    }
+    return PVS_ERR_CUDA;
+}
+
+#define PVS_CUDA(x)                                      \
+    do {                                                 \
+        cudaError_t _e = (x);                            \
+        if (_e != cudaSuccess) return cuda_status(_e);   \
+    } while (0)
+
+template <typename T>
+cudaError_t dev_alloc(T** p, size_t count) {
+    *p = nullptr;
+    if (count == 0) count = 1;
+    return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+}
+
+template <typename T>
+void dev_free(T*& p) {
+    if (p) cudaFree(p);
+    p = nullptr;
+}
+
+bool is_device_ptr(const void* p) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+// Grow the index arrays to hold `need` rows.
+pvs_status index_reserve(pvs_index* x, int64_t need) {
+    if (need <= x->cap) return PVS_OK;
+    int64_t cap = std::max<int64_t>(need, x->cap + x->cap / 2);
+    cap = round_up(std::max<int64_t>(cap, 64), 64);
+    int8_t* codes = nullptr;
+    float *scale = nullptr, *vnorm = nullptr, *enorm = nullptr, *raw = nullptr;
+    cudaError_t e = dev_alloc(&codes, (size_t)cap * x->m_pad);
+    if (e == cudaSuccess) e = dev_alloc(&scale, (size_t)cap);
+    if (e == cudaSuccess) e = dev_alloc(&vnorm, (size_t)cap);
+    if (e == cudaSuccess) e = dev_alloc(&enorm, (size_t)cap);
+    if (e == cudaSuccess) e = dev_alloc(&raw, (size_t)cap * x->m_raw);
+    if (e == cudaSuccess) {
+        // zero the tail so that tile copies past the last row read zeros
+        e = cudaMemsetAsync(scale, 0, cap * sizeof(float), x->stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(vnorm, 0, cap * sizeof(float), x->stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(enorm, 0, cap * sizeof(float), x->stream);
+    }
+    if (e == cudaSuccess && x->size > 0) {
+        e = cudaMemcpyAsync(codes, x->codes, (size_t)x->size * x->m_pad, cudaMemcpyDeviceToDevice,
+                            x->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(scale, x->scale, x->size * sizeof(float), cudaMemcpyDeviceToDevice,
+                                x->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(vnorm, x->vnorm, x->size * sizeof(float), cudaMemcpyDeviceToDevice,
+                                x->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(enorm, x->enorm, x->size * sizeof(float), cudaMemcpyDeviceToDevice,
+                                x->stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(raw, x->raw, (size_t)x->size * x->m_raw * sizeof(float),
+                                cudaMemcpyDeviceToDevice, x->stream);
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);
+    if (e != cudaSuccess) {
+        dev_free(codes), dev_free(scale), dev_free(vnorm), dev_free(enorm), dev_free(raw);
+        return cuda_status(e);
+    }
+    dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
+    dev_free(x->raw);
+    x->codes = codes, x->scale = scale, x->vnorm = vnorm, x->enorm = enorm, x->raw = raw;
+    x->cap = cap;
+    x->h_tomb.resize((size_t)(cap / 32), 0u);
+    return PVS_OK;
+}
+
+// Quantize n rows into the index at row offset x->size (does not commit).
+pvs_status index_fill(pvs_index* x, const float* vecs, int64_t n, bool on_device) {
+    if (n == 0) return PVS_OK;
+    PVS_CUDA(cudaMemsetAsync(x->d_status, 0, sizeof(int), x->stream));
+    const int64_t row0 = x->size;
+    if (on_device) {
+        PVS_CUDA(launch_build(vecs, n, x->m, x->m_pad, x->m_raw, x->codes + row0 * x->m_pad,
+                              x->scale + row0, x->vnorm + row0, x->enorm + row0,
+                              x->raw + row0 * x->m_raw, x->d_status, x->stream));
+    } else {
+        const int64_t rows_per_chunk =
+            std::max<int64_t>(1, (int64_t)(kStageBytes / sizeof(float)) / x->m);
+        const int64_t chunk = std::min<int64_t>(rows_per_chunk, n);
+        if (x->stage_floats < (size_t)(chunk * x->m)) {
+            dev_free(x->d_stage);
+            PVS_CUDA(dev_alloc(&x->d_stage, (size_t)(chunk * x->m)));
+            x->stage_floats = (size_t)(chunk * x->m);
+        }
+        for (int64_t r = 0; r < n; r += chunk) {
+            const int64_t c = std::min<int64_t>(chunk, n - r);
+            PVS_CUDA(cudaMemcpyAsync(x->d_stage, vecs + r * x->m, (size_t)(c * x->m) * sizeof(float),
+                                     cudaMemcpyHostToDevice, x->stream));
+            const int64_t dr = row0 + r;
+            PVS_CUDA(launch_build(x->d_stage, c, x->m, x->m_pad, x->m_raw,
+                                  x->codes + dr * x->m_pad, x->scale + dr, x->vnorm + dr,
+                                  x->enorm + dr, x->raw + dr * x->m_raw, x->d_status, x->stream));
+        }
+    }
+    int st = 0;
+    PVS_CUDA(cudaMemcpyAsync(&st, x->d_status, sizeof(int), cudaMemcpyDeviceToHost, x->stream));
+    PVS_CUDA(cudaStreamSynchronize(x->stream));
+    return (pvs_status)st;
+}
+
+std::shared_ptr<SnapData> make_snapdata(const pvs_index* x) {
+    auto s = std::make_shared<SnapData>();
+    s->rows = x->size;
+    s->visible = x->live;
+    if (x->tombstoned > 0) {
+        const size_t words = (size_t)((x->size + 31) / 32);
+        s->h_tomb.assign(x->h_tomb.begin(), x->h_tomb.begin() + words);
+        if (cudaMalloc(&s->d_tomb, words * sizeof(uint32_t)) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        if (cudaMemcpy(s->d_tomb, s->h_tomb.data(), words * sizeof(uint32_t),
+                       cudaMemcpyHostToDevice) != cudaSuccess)
+            return nullptr;
+    }
+    return s;
+}
+
+void cursor_free_device(pvs_cursor* c) {
+    dev_free(c->zq), dev_free(c->qraw), dev_free(c->qs);
+    dev_free(c->lo), dev_free(c->hi);
+    dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
+    dev_free(c->compact_scratch);
+    dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp);
+    if (c->sort_scratch) cudaFree(c->sort_scratch);
+    c->sort_scratch = nullptr;
+    dev_free(c->sel), dev_free(c->ctr), dev_free(c->d_status);
+    dev_free(c->d_ids), dev_free(c->d_scores);
+    if (c->h_ids) cudaFreeHost(c->h_ids);
+    if (c->h_scores) cudaFreeHost(c->h_scores);
+    if (c->h_small) cudaFreeHost(c->h_small);
+    c->h_ids = nullptr, c->h_scores = nullptr, c->h_small = nullptr;
+    if (c->ev_begin) cudaEventDestroy(c->ev_begin);
+    if (c->ev_end) cudaEventDestroy(c->ev_end);
+    c->ev_begin = c->ev_end = nullptr;
+}
+
+// Allocate the per-row state of a cursor (first pull).
+pvs_status cursor_alloc_rows(pvs_cursor* c) {
+    if (c->lo) return PVS_OK;
+    const size_t n = (size_t)std::max<int64_t>(c->rows, 1);
+    PVS_CUDA(dev_alloc(&c->lo, n));
+    PVS_CUDA(dev_alloc(&c->hi, n));
+    PVS_CUDA(dev_alloc(&c->w_id, n));
+    PVS_CUDA(dev_alloc(&c->w_lo, n));
+    PVS_CUDA(dev_alloc(&c->w_hi, n));
+    PVS_CUDA(dev_alloc(&c->compact_scratch, compact_scratch_elems((int64_t)n)));
+    PVS_CUDA(dev_alloc(&c->cand, n));
+    PVS_CUDA(dev_alloc(&c->keys, n));
+    PVS_CUDA(dev_alloc(&c->keys_tmp, n));
+    PVS_CUDA(cudaMalloc(&c->sort_scratch, radix_sort_scratch_bytes((int64_t)n)));
+    return PVS_OK;
+}
+
+pvs_status cursor_out_reserve(pvs_cursor* c, int64_t n) {
+    if (n <= c->out_cap) return PVS_OK;
+    dev_free(c->d_ids), dev_free(c->d_scores);
+    if (c->h_ids) cudaFreeHost(c->h_ids);
+    if (c->h_scores) cudaFreeHost(c->h_scores);
+    c->h_ids = nullptr, c->h_scores = nullptr, c->out_cap = 0;
+    const int64_t cap = std::max<int64_t>(n, 256);
+    PVS_CUDA(dev_alloc(&c->d_ids, (size_t)cap));
+    PVS_CUDA(dev_alloc(&c->d_scores, (size_t)cap));
+    PVS_CUDA(cudaMallocHost(&c->h_ids, cap * sizeof(int64_t)));
+    PVS_CUDA(cudaMallocHost(&c->h_scores, cap * sizeof(float)));
+    c->out_cap = cap;
+    return PVS_OK;
+}
+
+int grid_for(const pvs_cursor* c, int64_t items, int per_block = 256) {
+    const int64_t g = std::max<int64_t>(1, (items + per_block - 1) / per_block);
+    return (int)std::min<int64_t>(g, 4 * (int64_t)c->index->num_sms);
+}
+
+pvs_status fail(pvs_cursor* c, pvs_status s) {
+    if (s < 0 && c->state >= 0) c->state = s;
+    return s;
+}
+
+// Add the timed interval pass once its end event has completed.
+void harvest_interval_time(pvs_cursor* c) {
+    if (!c->ev_pending) return;
+    if (cudaEventQuery(c->ev_end) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    float ms = 0.0f;
+    if (cudaEventElapsedTime(&ms, c->ev_begin, c->ev_end) == cudaSuccess) c->interval_ms += ms;
+    c->ev_pending = false;
+}
+
+// Read the device status word; a failure makes the cursor Failed.
+pvs_status check_device_status(pvs_cursor* c) {
+    cudaStream_t st = c->index->stream;
+    PVS_CUDA(cudaMemcpyAsync(c->h_small, c->d_status, sizeof(int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    const int s = (int)c->h_small[0];
+    if (s != 0) return fail(c, (pvs_status)s);
+    return PVS_OK;
+}
+
+pvs_status interval_pass(pvs_cursor* c) {
+    pvs_index* x = c->index;
+    IntervalArgs a;
+    a.codes = x->codes;
+    a.scale = x->scale;
+    a.vnorm = x->vnorm;
+    a.enorm = x->enorm;
+    a.tomb = c->snap->d_tomb;
+    a.rows = c->rows;
+    a.m_pad = x->m_pad;
+    a.zq = c->zq;
+    a.qs = c->qs;
+    a.lo = c->lo;
+    a.hi = c->hi;
+    a.status = c->d_status;
+    if (!c->ev_begin) {
+        PVS_CUDA(cudaEventCreate(&c->ev_begin));
+        PVS_CUDA(cudaEventCreate(&c->ev_end));
+    }
+    PVS_CUDA(cudaEventRecord(c->ev_begin, x->stream));
+    PVS_CUDA(launch_interval_pass(a, x->num_sms, x->stream));
+    PVS_CUDA(cudaEventRecord(c->ev_end, x->stream));
+    c->ev_pending = true;
+    c->interval_passes++;
+    c->scanned = true;
+    return PVS_OK;
+}
+
+// (Re)build the working set so that it holds the next `want` ranks.
+pvs_status build_working_set(pvs_cursor* c, int64_t want) {
+    pvs_index* x = c->index;
+    const int64_t remaining = c->visible - c->emitted;
+    int64_t H = std::max<int64_t>({want, 2 * c->horizon, 2048});
+    if (H > remaining) H = remaining;
+    if (H < remaining) {
+        PVS_CUDA(launch_select_f32_n(c->lo, c->rows, (uint64_t)H, c->sel, grid_for(c, c->rows),
+                                     x->stream));
+    } else {
+        PVS_CUDA(cudaMemsetAsync(c->sel, 0, sizeof(SelectState), x->stream));  // tau = 0: all live
+    }
+    PVS_CUDA(launch_compact_ordered(c->lo, c->hi, c->rows, c->sel, c->w_id, c->w_lo, c->w_hi,
+                                    &c->ctr->w_len, c->compact_scratch, x->stream));
+    c->horizon = H;
+    c->horizon_base = c->emitted;
+    c->horizon_builds++;
+    return PVS_OK;
+}
+
+// One pull of n_eff >= 1 ranks into device buffers d_ids / d_scores.
+pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
+    pvs_index* x = c->index;
+    cudaStream_t st = x->stream;
+    pvs_status s = cursor_alloc_rows(c);
+    if (s != PVS_OK) return fail(c, s);
+    if (!c->scanned) {
+        s = interval_pass(c);
+        if (s != PVS_OK) return fail(c, s);
+    }
+    if (c->emitted + n_eff - c->horizon_base > c->horizon) {
+        s = build_working_set(c, n_eff);
+        if (s != PVS_OK) return fail(c, s);
+    }
+    const int grid_w = grid_for(c, std::min<int64_t>(c->rows, (int64_t)1 << 22));
+    cudaError_t e = launch_select_f32(c->w_lo, &c->ctr->w_len, (uint64_t)n_eff, c->sel, grid_w, st);
+    if (e == cudaSuccess)
+        e = launch_candidates(c->w_lo, c->w_hi, &c->ctr->w_len, c->sel, c->cand, &c->ctr->cand,
+                              grid_w, st);
+    if (e == cudaSuccess)
+        e = launch_refine(c->cand, &c->ctr->cand, c->w_id, c->w_lo, c->w_hi, c->lo, c->hi, c->qraw,
+                          x->raw, x->m_raw, c->d_status, c->ctr, 2 * x->num_sms, st);
+    if (e == cudaSuccess) e = launch_make_keys(c->cand, &c->ctr->cand, c->w_lo, c->keys, grid_w, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(c->h_small + 1, &c->ctr->cand, sizeof(unsigned int),
+                            cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(c->h_small, c->d_status, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return fail(c, cuda_status(e));
+    harvest_interval_time(c);
+    if ((int)c->h_small[0] != 0) return fail(c, (pvs_status)(int)c->h_small[0]);
+    const int64_t cand = c->h_small[1];
+    if (cand < n_eff) return fail(c, PVS_ERR_INVALID);   // internal invariant
+    c->candidates += cand;
+    if (cand <= kBitonicMax)
+        e = launch_bitonic_desc(c->keys, (int)cand, st);
+    else
+        e = launch_radix_sort_desc(c->keys, c->keys_tmp, cand, c->sort_scratch, st);
+    if (e == cudaSuccess)
+        e = launch_emit(c->keys, (int)n_eff, c->w_id, c->w_lo, c->w_hi, c->lo, c->hi, d_ids,
+                        d_scores, st);
+    if (e != cudaSuccess) return fail(c, cuda_status(e));
+    c->emitted += n_eff;
+    c->pulls++;
+    return PVS_OK;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+extern "C" {
+
+int64_t pvs_launch_count(void) { return (int64_t)g_launches.load(); }
+
+const char* pvs_status_string(int32_t s) {
+    switch (s) {
+        case PVS_OK: return "ok";
+        case PVS_EXHAUSTED: return "exhausted";
+        case PVS_ERR_INVALID: return "invalid argument";
+        case PVS_ERR_NONFINITE: return "non-finite input";
+        case PVS_ERR_OVERFLOW: return "overflow";
+        case PVS_ERR_INTERVAL: return "authoritative score outside its interval";
+        case PVS_ERR_CUDA: return "CUDA error";
+        case PVS_ERR_OOM: return "out of memory";
+        case PVS_ERR_TIMEOUT: return "device wait timed out";
+        case PVS_ERR_FAILED: return "cursor failed earlier";
+        default: return "unknown status";
+    }
+}
+
+pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
+                     void* cuda_stream, pvs_index** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) || (n > 0 && !vecs))
+        return PVS_ERR_INVALID;
+    pvs_index* x = new (std::nothrow) pvs_index();
+    if (!x) return PVS_ERR_OOM;
+    auto bail = [&](pvs_status s) {
+        pvs_index_free(x);
+        return s;
+    };
+    if (cudaGetDevice(&x->device) != cudaSuccess) return bail(PVS_ERR_CUDA);
+    if (cudaDeviceGetAttribute(&x->num_sms, cudaDevAttrMultiProcessorCount, x->device) !=
+        cudaSuccess)
+        return bail(PVS_ERR_CUDA);
+    x->m = dim;
+    x->m_pad = (int)round_up(dim, kCodeAlign);
+    x->m_raw = (int)round_up(dim, 4);
+    if (cuda_stream) {
+        x->stream = static_cast<cudaStream_t>(cuda_stream);
+    } else {
+        if (cudaStreamCreateWithFlags(&x->stream, cudaStreamNonBlocking) != cudaSuccess)
+            return bail(PVS_ERR_CUDA);
+        x->own_stream = true;
+    }
+    if (cudaMalloc(&x->d_status, sizeof(int)) != cudaSuccess) return bail(PVS_ERR_OOM);
+    if (vecs_on_device && n > 0 && !is_device_ptr(vecs)) return bail(PVS_ERR_INVALID);
+    pvs_status s = index_reserve(x, n);
+    if (s != PVS_OK) return bail(s);
+    s = index_fill(x, vecs, n, vecs_on_device != 0);
+    if (s != PVS_OK) return bail(s);
+    x->size = n;
+    x->live = n;
+    *out = x;
+    return PVS_OK;
+}
+
+pvs_status pvs_append(pvs_index* x, const float* vecs, int64_t n, int32_t vecs_on_device) {
+    if (!x || n < 0 || (n > 0 && !vecs) || x->size + n >= ((int64_t)1 << 31))
+        return PVS_ERR_INVALID;
+    if (n == 0) return PVS_OK;
+    if (vecs_on_device && !is_device_ptr(vecs)) return PVS_ERR_INVALID;
+    pvs_status s = index_reserve(x, x->size + n);
+    if (s != PVS_OK) return s;
+    s = index_fill(x, vecs, n, vecs_on_device != 0);
+    if (s != PVS_OK) return s;
+    x->size += n;
+    x->live += n;
+    return PVS_OK;
+}
+
+pvs_status pvs_tombstone(pvs_index* x, const int64_t* ids, int64_t n) {
+    if (!x || n < 0 || (n > 0 && !ids)) return PVS_ERR_INVALID;
+    for (int64_t i = 0; i < n; ++i)
+        if (ids[i] < 0 || ids[i] >= x->size) return PVS_ERR_INVALID;
+    for (int64_t i = 0; i < n; ++i) {
+        const int64_t id = ids[i];
+        uint32_t& w = x->h_tomb[(size_t)(id >> 5)];
+        const uint32_t b = 1u << (id & 31);
+        if (!(w & b)) {
+            w |= b;
+            x->tombstoned++;
+            x->live--;
+        }
+    }
+    return PVS_OK;
+}
+
+int64_t pvs_index_size(const pvs_index* x) { return x ? x->size : -1; }
+int64_t pvs_index_live(const pvs_index* x) { return x ? x->live : -1; }
+int32_t pvs_index_dim(const pvs_index* x) { return x ? x->m : -1; }
+
+pvs_status pvs_index_export(const pvs_index* x, int64_t first, int64_t count, int8_t* codes,
+                            float* scale, float* vnorm, float* enorm) {
+    if (!x || first < 0 || count < 0 || first + count > x->size) return PVS_ERR_INVALID;
+    if (count == 0) return PVS_OK;
+    if (codes)
+        PVS_CUDA(cudaMemcpy2D(codes, (size_t)x->m, x->codes + first * x->m_pad, (size_t)x->m_pad,
+                              (size_t)x->m, (size_t)count, cudaMemcpyDeviceToHost));
+    if (scale)
+        PVS_CUDA(cudaMemcpy(scale, x->scale + first, count * sizeof(float), cudaMemcpyDeviceToHost));
+    if (vnorm)
+        PVS_CUDA(cudaMemcpy(vnorm, x->vnorm + first, count * sizeof(float), cudaMemcpyDeviceToHost));
+    if (enorm)
+        PVS_CUDA(cudaMemcpy(enorm, x->enorm + first, count * sizeof(float), cudaMemcpyDeviceToHost));
+    return PVS_OK;
+}
+
+void pvs_index_free(pvs_index* x) {
+    if (!x) return;
+    if (x->stream) cudaStreamSynchronize(x->stream);
+    dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
+    dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage);
+    if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
+    delete x;
+}
+
+pvs_status pvs_snapshot_create(pvs_index* x, pvs_snapshot** out) {
+    if (!x || !out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    auto d = make_snapdata(x);
+    if (!d) return PVS_ERR_OOM;
+    pvs_snapshot* s = new (std::nothrow) pvs_snapshot();
+    if (!s) return PVS_ERR_OOM;
+    s->index = x;
+    s->data = std::move(d);
+    *out = s;
+    return PVS_OK;
+}
+
+int64_t pvs_snapshot_visible(const pvs_snapshot* s) { return s ? s->data->visible : -1; }
+
+void pvs_snapshot_free(pvs_snapshot* s) { delete s; }
+
+pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* query,
+                           int32_t query_on_device, pvs_cursor** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (!x || !query || (snap && snap->index != x)) return PVS_ERR_INVALID;
+    if (query_on_device && !is_device_ptr(query)) return PVS_ERR_INVALID;
+    pvs_cursor* c = new (std::nothrow) pvs_cursor();
+    if (!c) return PVS_ERR_OOM;
+    auto bail = [&](pvs_status s) {
+        cursor_free_device(c);
+        delete c;
+        return s;
+    };
+    c->index = x;
+    c->snap = snap ? snap->data : make_snapdata(x);
+    if (!c->snap) return bail(PVS_ERR_OOM);
+    c->rows = c->snap->rows;
+    c->visible = c->snap->visible;
+    cudaStream_t st = x->stream;
+    if (dev_alloc(&c->zq, (size_t)x->m_pad) != cudaSuccess ||
+        dev_alloc(&c->qraw, (size_t)x->m_raw) != cudaSuccess ||
+        dev_alloc(&c->qs, 1) != cudaSuccess || dev_alloc(&c->sel, 1) != cudaSuccess ||
+        dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
+        cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess)
+        return bail(PVS_ERR_OOM);
+    const float* qd = query;
+    float* tmp = nullptr;
+    if (!query_on_device) {
+        if (dev_alloc(&tmp, (size_t)x->m) != cudaSuccess) return bail(PVS_ERR_OOM);
+        if (cudaMemcpyAsync(tmp, query, x->m * sizeof(float), cudaMemcpyHostToDevice, st) !=
+            cudaSuccess) {
+            cudaFree(tmp);
+            return bail(PVS_ERR_CUDA);
+        }
+        qd = tmp;
+    }
+    cudaError_t e = cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->d_status, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = launch_encode_query(qd, x->m, x->m_pad, x->m_raw, c->zq, c->qraw, c->qs, st);
+    QueryScalars qs{};
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&qs, c->qs, sizeof(qs), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (tmp) cudaFree(tmp);
+    if (e != cudaSuccess) return bail(cuda_status(e));
+    if (qs.status != 0) return bail((pvs_status)qs.status);
+    c->state = c->visible == 0 ? PVS_EXHAUSTED : PVS_OK;
+    *out = c;
+    return PVS_OK;
+}
+
+pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const float* queries,
+                                 int32_t nq, int32_t queries_on_device, int32_t horizon,
+                                 pvs_cursor** out) {
+    if (!x || !queries || !out || nq < 0 || horizon < 1) return PVS_ERR_INVALID;
+    const size_t m = (size_t)x->m;
+    for (int32_t i = 0; i < nq; ++i) out[i] = nullptr;
+    for (int32_t i = 0; i < nq; ++i) {
+        pvs_status s = pvs_cursor_open(x, snap, queries + i * m, queries_on_device, &out[i]);
+        if (s != PVS_OK) {
+            for (int32_t j = 0; j < i; ++j) {
+                pvs_cursor_close(out[j]);
+                out[j] = nullptr;
+            }
+            return s;
+        }
+    }
+    return PVS_OK;
+}
+
+static pvs_status next_common(pvs_cursor* c, int32_t n, int32_t* n_out, int64_t* n_eff) {
+    *n_eff = 0;
+    if (n_out) *n_out = 0;
+    if (!c || n < 0 || !n_out) return PVS_ERR_INVALID;
+    if (c->state < 0) return PVS_ERR_FAILED;
+    const int64_t remaining = c->visible - c->emitted;
+    *n_eff = std::min<int64_t>(n, remaining);
+    return PVS_OK;
+}
+
+pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    int64_t n_eff;
+    pvs_status s = next_common(c, n, n_out, &n_eff);
+    if (s != PVS_OK) return s;
+    if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
+    if (n_eff > 0) {
+        s = cursor_out_reserve(c, n_eff);
+        if (s != PVS_OK) return fail(c, s);
+        s = pull(c, n_eff, c->d_ids, c->d_scores);
+        if (s != PVS_OK) return s;
+        cudaStream_t st = c->index->stream;
+        cudaError_t e = cudaMemcpyAsync(c->h_ids, c->d_ids, n_eff * sizeof(int64_t),
+                                        cudaMemcpyDeviceToHost, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(c->h_scores, c->d_scores, n_eff * sizeof(float),
+                                cudaMemcpyDeviceToHost, st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        s = check_device_status(c);
+        if (s != PVS_OK) return s;
+        std::memcpy(ids, c->h_ids, n_eff * sizeof(int64_t));
+        std::memcpy(scores, c->h_scores, n_eff * sizeof(float));
+    }
+    *n_out = (int32_t)n_eff;
+    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
+    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+}
+
+pvs_status pvs_next_device(pvs_cursor* c, int32_t n, int64_t* ids, float* scores,
+                           int32_t* n_out) {
+    int64_t n_eff;
+    pvs_status s = next_common(c, n, n_out, &n_eff);
+    if (s != PVS_OK) return s;
+    if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
+    if (n_eff > 0) {
+        s = pull(c, n_eff, ids, scores);
+        if (s != PVS_OK) return s;
+    }
+    *n_out = (int32_t)n_eff;
+    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
+    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+}
+
+pvs_status pvs_cursor_sync(pvs_cursor* c) {
+    if (!c) return PVS_ERR_INVALID;
+    if (c->state < 0) return (pvs_status)c->state;
+    pvs_status s = check_device_status(c);
+    if (s != PVS_OK) return s;
+    return (pvs_status)c->state;
+}
+
+pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
+    if (!c || !out) return PVS_ERR_INVALID;
+    std::memset(out, 0, sizeof(*out));
+    DevCounters d{};
+    cudaError_t e = cudaMemcpyAsync(&d, c->ctr, sizeof(d), cudaMemcpyDeviceToHost, c->index->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->index->stream);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (c->state >= 0) check_device_status(c);
+    out->visible = c->visible;
+    out->emitted = c->emitted;
+    out->refined = (int64_t)d.refined;
+    out->exact_fallbacks = (int64_t)d.exact_fallbacks;
+    out->interval_passes = c->interval_passes;
+    out->horizon_builds = c->horizon_builds;
+    out->pulls = c->pulls;
+    out->candidates = c->candidates;
+    out->code_bytes = c->interval_passes * c->rows * (int64_t)(c->index->m_pad + 12);
+    out->state = c->state;
+    harvest_interval_time(c);
+    out->interval_ms = c->interval_ms;
+    return PVS_OK;
+}
+
+pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float* lo,
+                             float* hi) {
+    if (!c || first < 0 || count < 0 || first + count > c->rows || (count > 0 && (!lo || !hi)))
+        return PVS_ERR_INVALID;
+    if (c->state < 0) return PVS_ERR_FAILED;
+    pvs_status s = cursor_alloc_rows(c);
+    if (s != PVS_OK) return fail(c, s);
+    if (!c->scanned) {
+        s = interval_pass(c);
+        if (s != PVS_OK) return fail(c, s);
+        s = check_device_status(c);
+        if (s != PVS_OK) return s;
+    }
+    if (count == 0) return PVS_OK;
+    cudaStream_t st = c->index->stream;
+    PVS_CUDA(cudaMemcpyAsync(lo, c->lo + first, count * sizeof(float), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpyAsync(hi, c->hi + first, count * sizeof(float), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    return PVS_OK;
+}
+
+pvs_status pvs_cursor_score_ids(pvs_cursor* c, const int64_t* ids, int32_t n, float* scores) {
+    if (!c || n < 0 || (n > 0 && (!ids || !scores))) return PVS_ERR_INVALID;
+    for (int32_t i = 0; i < n; ++i)
+        if (ids[i] < 0 || ids[i] >= c->rows) return PVS_ERR_INVALID;
+    if (n == 0) return PVS_OK;
+    cudaStream_t st = c->index->stream;
+    int64_t* d_ids = nullptr;
+    float* d_out = nullptr;
+    cudaError_t e = dev_alloc(&d_ids, (size_t)n);
+    if (e == cudaSuccess) e = dev_alloc(&d_out, (size_t)n);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(d_ids, ids, n * sizeof(int64_t), cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+        e = launch_score_ids(d_ids, n, c->qraw, c->index->raw, c->index->m_raw, d_out, c->ctr, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(scores, d_out, n * sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    dev_free(d_ids);
+    dev_free(d_out);
+    return cuda_status(e);
+}
+
+void pvs_cursor_close(pvs_cursor* c) {
+    if (!c) return;
+    if (c->index && c->index->stream) cudaStreamSynchronize(c->index->stream);
+    cursor_free_device(c);
+    delete c;
+}
+
+}  // extern "C"

@@ -1,0 +1,100 @@
+// Internal host-side structures of libpvs.so (index, snapshot, cursor).
+#pragma once
+
+#include <cstdint>
+#include <memory>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/pvs.h"
+#include "kernels.h"
+
+namespace pvs {
+
+struct SnapData {
+    int64_t rows = 0;                 // rows [0, rows) exist in the snapshot
+    int64_t visible = 0;              // rows minus tombstones
+    std::vector<uint32_t> h_tomb;     // tombstone bits of rows [0, rows)
+    uint32_t* d_tomb = nullptr;       // device copy, null if nothing is deleted
+    ~SnapData();
+    bool is_visible(int64_t id) const {
+        if (id < 0 || id >= rows) return false;
+        if (h_tomb.empty()) return true;
+        return ((h_tomb[(size_t)(id >> 5)] >> (id & 31)) & 1u) == 0;
+    }
+};
+
+}  // namespace pvs
+
+struct pvs_index {
+    int device = 0;
+    int num_sms = 0;
+    int m = 0, m_pad = 0, m_raw = 0;
+    int64_t size = 0, cap = 0, live = 0;
+    int8_t* codes = nullptr;          // [cap][m_pad]
+    float* scale = nullptr;           // [cap]
+    float* vnorm = nullptr;           // [cap]
+    float* enorm = nullptr;           // [cap]
+    float* raw = nullptr;             // [cap][m_raw]
+    std::vector<uint32_t> h_tomb;     // [cap/32]
+    int64_t tombstoned = 0;
+    cudaStream_t stream = nullptr;
+    bool own_stream = false;
+    int* d_status = nullptr;
+    float* d_stage = nullptr;         // host-input staging
+    size_t stage_floats = 0;
+};
+
+struct pvs_snapshot {
+    pvs_index* index = nullptr;
+    std::shared_ptr<pvs::SnapData> data;
+};
+
+struct pvs_cursor {
+    pvs_index* index = nullptr;
+    std::shared_ptr<pvs::SnapData> snap;
+    int64_t rows = 0, visible = 0, emitted = 0;
+    int state = PVS_OK;
+    bool scanned = false;
+    // query
+    int8_t* zq = nullptr;
+    float* qraw = nullptr;
+    pvs::QueryScalars* qs = nullptr;
+    // bounds of every row of the snapshot
+    float* lo = nullptr;
+    float* hi = nullptr;
+    // working set (ordered by id): rows that can hold the next `horizon` ranks
+    int32_t* w_id = nullptr;
+    float* w_lo = nullptr;
+    float* w_hi = nullptr;
+    int64_t horizon = 0, horizon_base = 0;
+    unsigned int* compact_scratch = nullptr;
+    // pull scratch
+    int32_t* cand = nullptr;
+    uint64_t* keys = nullptr;
+    uint64_t* keys_tmp = nullptr;
+    void* sort_scratch = nullptr;
+    pvs::SelectState* sel = nullptr;
+    pvs::DevCounters* ctr = nullptr;
+    int* d_status = nullptr;
+    // output staging
+    int64_t* d_ids = nullptr;
+    float* d_scores = nullptr;
+    int64_t out_cap = 0;
+    int64_t* h_ids = nullptr;         // pinned
+    float* h_scores = nullptr;        // pinned
+    unsigned int* h_small = nullptr;  // pinned scratch (counts, status)
+    // stats
+    int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;
+    cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
+    bool ev_pending = false;
+    double interval_ms = 0.0;
+};
+
+namespace pvs {
+// Accessors used by the EAHR driver.
+int64_t cursor_visible(const pvs_cursor* c);
+int64_t cursor_emitted(const pvs_cursor* c);
+const SnapData* cursor_snapshot(const pvs_cursor* c);
+}  // namespace pvs

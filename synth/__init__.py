@@ -1,0 +1,172 @@
+"""Seeded synthetic workloads for the PVS / EAHR path (no method arithmetic).
+
+The paper's corpora (MS MARCO passages, CORD-19 snapshots encoded with
+bge-small) and its sparse BM25 rankings are not available here; these
+generators stand in for them with the shapes and structure of the workloads:
+
+* ``unit_normal``        i.i.d. standard normal rows, L2-normalised;
+* ``mixture_centres`` / ``mixture_rows`` / ``mixture_queries``
+                         a Gaussian mixture (centres ~ N(0, I), uniform
+                         component choice, isotropic within-component noise),
+                         L2-normalised;
+* ``near_duplicate_rows`` copies of chosen rows plus N(0, sigma^2) noise,
+                         L2-normalised;
+* ``copula_ranking``     a complete ranking whose Kendall tau against the
+                         ranking of given proxy scores is about ``tau``
+                         (Gaussian copula, rho = sin(pi tau / 2));
+* ``controlled_streams`` the rank relations of the controlled-stream study
+                         (block-32 correlated, partial overlap, independent,
+                         reversed, all tied).
+
+Every generator is deterministic in its seed; large matrices are produced in
+row chunks, each with its own derived seed, so any chunk can be regenerated
+alone.  Tensors come out on the requested torch device.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+CHUNK_ROWS = 1 << 18
+
+
+def _gen(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) & ((1 << 63) - 1))
+    return g
+
+
+def _chunk_seed(seed: int, chunk: int) -> int:
+    return (int(seed) * 1000003 + 7919 * int(chunk) + 17) & ((1 << 63) - 1)
+
+
+def _normalise(x: torch.Tensor) -> torch.Tensor:
+    return x / torch.linalg.vector_norm(x, dim=1, keepdim=True).clamp_min(1e-30)
+
+
+def unit_normal(n: int, d: int, seed: int, device="cpu", first: int = 0) -> torch.Tensor:
+    """Rows first .. first+n-1 of an i.i.d. N(0, 1) matrix, L2-normalised."""
+    out = torch.empty((n, d), dtype=torch.float32, device=device)
+    for r in range(0, n, CHUNK_ROWS):
+        c = min(CHUNK_ROWS, n - r)
+        out[r:r + c] = _rows_normal(first + r, c, d, seed, device)
+    return out
+
+
+def _rows_normal(row0: int, count: int, d: int, seed: int, device) -> torch.Tensor:
+    # row0 is aligned to CHUNK_ROWS by every caller that regenerates chunks
+    chunk = row0 // CHUNK_ROWS
+    x = torch.randn((count, d), generator=_gen(_chunk_seed(seed, chunk), device),
+                    device=device, dtype=torch.float32)
+    return _normalise(x)
+
+
+def mixture_centres(n_components: int, d: int, seed: int, device="cpu") -> torch.Tensor:
+    return torch.randn((n_components, d), generator=_gen(_chunk_seed(seed, -1), device),
+                       device=device, dtype=torch.float32)
+
+
+def mixture_rows(n: int, centres: torch.Tensor, within_std: float, seed: int,
+                 first: int = 0) -> torch.Tensor:
+    """Rows first .. first+n-1 of a mixture: centre[c] + within_std * N(0, I),
+    c uniform over the components, L2-normalised."""
+    device = centres.device
+    k, d = centres.shape
+    out = torch.empty((n, d), dtype=torch.float32, device=device)
+    for r in range(0, n, CHUNK_ROWS):
+        c = min(CHUNK_ROWS, n - r)
+        g = _gen(_chunk_seed(seed, (first + r) // CHUNK_ROWS), device)
+        comp = torch.randint(0, k, (c,), generator=g, device=device)
+        x = torch.randn((c, d), generator=g, device=device, dtype=torch.float32)
+        x.mul_(within_std).add_(centres[comp])
+        out[r:r + c] = _normalise(x)
+    return out
+
+
+def mixture_queries(nq: int, centres: torch.Tensor, noise_std: float, seed: int) -> torch.Tensor:
+    """Queries: a uniformly chosen centre + noise_std * N(0, I), normalised."""
+    device = centres.device
+    g = _gen(_chunk_seed(seed, -2), device)
+    comp = torch.randint(0, centres.shape[0], (nq,), generator=g, device=device)
+    x = torch.randn((nq, centres.shape[1]), generator=g, device=device, dtype=torch.float32)
+    return _normalise(centres[comp] + noise_std * x)
+
+
+def near_duplicate_rows(src: torch.Tensor, noise_std: float, seed: int) -> torch.Tensor:
+    """Copies of the given rows plus N(0, noise_std^2) noise, normalised."""
+    g = _gen(_chunk_seed(seed, -3), src.device)
+    x = torch.randn(src.shape, generator=g, device=src.device, dtype=torch.float32)
+    return _normalise(src + noise_std * x)
+
+
+def copula_ranking(proxy_scores: torch.Tensor, tau: float, seed: int) -> torch.Tensor:
+    """A complete ranking (int64 ids, best first) of all len(proxy_scores)
+    items whose Kendall tau against the proxy-score ranking is about tau:
+    key = rho * Phi^-1((n - r + 0.5) / n) + sqrt(1 - rho^2) * eps with
+    rho = sin(pi * tau / 2) (Greiner's relation for a Gaussian copula) and
+    r the proxy rank."""
+    device = proxy_scores.device
+    n = proxy_scores.numel()
+    rho = math.sin(math.pi * tau / 2.0)
+    order = torch.argsort(proxy_scores.double(), descending=True, stable=True)
+    ranks = torch.empty(n, dtype=torch.float64, device=device)
+    ranks[order] = torch.arange(1, n + 1, dtype=torch.float64, device=device)
+    u = (n - ranks + 0.5) / n
+    z = torch.special.ndtri(u)
+    g = _gen(_chunk_seed(seed, -4), device)
+    eps = torch.randn(n, generator=g, device=device, dtype=torch.float64)
+    key = rho * z + math.sqrt(max(0.0, 1.0 - rho * rho)) * eps
+    return torch.argsort(key, descending=True, stable=True)
+
+
+def kendall_tau_sample(a: np.ndarray, b: np.ndarray, pairs: int, seed: int) -> float:
+    """Kendall tau between two complete rankings (arrays of ids in rank order)
+    estimated on random item pairs."""
+    n = len(a)
+    ra = np.empty(n, np.int64)
+    rb = np.empty(n, np.int64)
+    ra[np.asarray(a)] = np.arange(n)
+    rb[np.asarray(b)] = np.arange(n)
+    rng = np.random.default_rng(seed)
+    i = rng.integers(0, n, pairs)
+    j = rng.integers(0, n, pairs)
+    keep = i != j
+    s = np.sign(ra[i[keep]] - ra[j[keep]]) * np.sign(rb[i[keep]] - rb[j[keep]])
+    return float(s.mean())
+
+
+def controlled_streams(n: int, relation: str, seed: int):
+    """Two complete rankings of n items for the controlled-stream study.
+    relation: 'correlated' (second = first permuted within 32-item blocks),
+    'partial' (500 random items of the first list's top 1000 plus the 500
+    items ranked just below it form the second list's top 1000 in random
+    order; the rest follow in the first list's order),
+    'independent', 'reversed', 'tied' (equal scores: both lists in id order)."""
+    rng = np.random.default_rng(seed)
+    if relation == "tied":
+        ids = np.arange(n, dtype=np.int64)
+        return ids, ids.copy()
+    first = rng.permutation(n).astype(np.int64)
+    if relation == "correlated":
+        second = first.copy()
+        for b in range(0, n, 32):
+            second[b:b + 32] = rng.permutation(second[b:b + 32])
+    elif relation == "partial":
+        top = min(1000, n)
+        half = top // 2
+        inside = rng.choice(first[:top], half, replace=False)
+        outside = first[top:top + (top - half)]   # the first list's next 500 items
+        head = rng.permutation(np.concatenate([inside, outside]))
+        used = np.zeros(n, bool)
+        used[head] = True
+        rest = first[~used[first]]          # the remaining items keep the first order
+        second = np.concatenate([head, rest]).astype(np.int64)
+    elif relation == "independent":
+        second = rng.permutation(n).astype(np.int64)
+    elif relation == "reversed":
+        second = first[::-1].copy()
+    else:
+        raise ValueError(relation)
+    return first, second

@@ -1,0 +1,137 @@
+"""C ABI library: loads on a machine without a GPU, exports every symbol that
+include/pvs.h declares, and its host-only EAHR driver reproduces the oracle
+(arXiv 2608.07152, Sec. 2.1, 2.2; controlled streams of Sec. 3.4 / 4.2)."""
+import os
+import re
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import paper_2608_07152_gb300 as pvs
+from oracle import eahr_oracle as eo
+from oracle import rrf_oracle as ro
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "pvs.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b((?:pvs|eahr)_[a-z_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_function():
+    names = declared_functions()
+    assert len(names) >= 20
+    for name in names:
+        assert hasattr(pvs._lib, name), name
+        assert name in pvs.EXPORTED, name
+
+
+def test_struct_layouts_match_header():
+    assert pvs.ctypes.sizeof(pvs.pvs_stats) == 9 * 8 + 2 * 4 + 8
+    assert pvs.ctypes.sizeof(pvs.eahr_params) == 9 * 4
+    assert pvs.ctypes.sizeof(pvs.eahr_stats) == 4 * 8 + 6 * 4
+
+
+def test_status_strings():
+    assert pvs.pvs_status_string(0) == "ok"
+    assert "interval" in pvs.pvs_status_string(-4)
+
+
+FORMS = [(pvs.EAHR_RANK_SCALED, ro.RANK_SCALED), (pvs.EAHR_NUMERATOR, ro.NUMERATOR)]
+
+
+@pytest.mark.parametrize("policy", [pvs.EAHR_POLICY_GEOMETRIC, pvs.EAHR_POLICY_EQUAL_DEPTH])
+def test_eahr_lists_match_complete_list_target(policy):
+    rng = np.random.default_rng(0)
+    for trial in range(60):
+        n = int(rng.integers(1, 400))
+        a = rng.permutation(n)
+        b = rng.permutation(n)[: int(rng.integers(0, n + 1))]
+        K = int(rng.integers(1, 30))
+        k = int(rng.integers(1, 80))
+        cform, oform = FORMS[trial % 2]
+        w = [(int(rng.integers(1, 5)), int(rng.integers(1, 4))),
+             (int(rng.integers(0, 4)), int(rng.integers(1, 3)))]
+        step = int(rng.integers(1, 40))
+        ids, F, st = pvs.eahr_topk_lists(a, b, K=K, k=k, form=cform, policy=policy, step=step,
+                                         weights=w)
+        wf = [Fraction(*w[0]), Fraction(*w[1])]
+        T = ro.target_topk([a, b], wf, k, K, oform)
+        assert ids.tolist() == [x for x, _ in T], trial
+        for (x, f), got in zip(T, F):
+            if not np.isnan(got):
+                assert got == ro.as_float(f)
+
+
+def test_eahr_lists_duplicate_or_negative_ids_fail():
+    a = np.array([3, 1, 2, 0])
+    with pytest.raises(pvs.PvsError) as e:
+        pvs.eahr_topk_lists(a, np.array([1, 1, 2]), K=4, policy=pvs.EAHR_POLICY_EQUAL_DEPTH,
+                            step=4)
+    assert e.value.status == pvs.PVS_ERR_INVALID
+    with pytest.raises(pvs.PvsError):
+        pvs.eahr_topk_lists(a, np.array([-1]), K=2)
+    with pytest.raises(pvs.PvsError):
+        pvs.eahr_topk_lists(a, a, K=0)
+    with pytest.raises(pvs.PvsError):
+        pvs.eahr_topk_lists(a, a, K=2, weights=((1, 0), (1, 1)))
+
+
+def test_eahr_lists_empty_and_zero_weight():
+    ids, F, st = pvs.eahr_topk_lists(np.array([], np.int64), np.array([], np.int64), K=5)
+    assert ids.size == 0
+    a = np.array([4, 2, 0])
+    ids, F, st = pvs.eahr_topk_lists(a, np.array([0, 2, 4]), K=5, weights=(1, 0))
+    assert ids.tolist() == [4, 2, 0] and st["depth"][1] == 0
+
+
+@pytest.mark.parametrize("relation", ["correlated", "partial", "independent", "reversed", "tied"])
+def test_eahr_lists_stop_where_the_oracle_rule_stops(relation):
+    # same protocol (equal depth, check every 16), independent implementations
+    for seed in (1729, 2027):
+        a, b = synth.controlled_streams(1500, relation, seed)
+        A, depths, exh = eo.equal_depth_run([a.tolist(), b.tolist()], [1, 1], 60, 20, step=16)
+        ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+                                         policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
+        assert ids.tolist() == A
+        assert st["depth"] == depths
+        assert st["exhausted"] == [int(x) for x in exh]
+
+
+@pytest.mark.parametrize("n", [100_000, 1_000_000, 5_000_000])
+def test_controlled_streams_paper_outcomes(n):
+    # Sec. 4.2: correlated rankings fix the Top-20 at depth 32 for all sizes;
+    # reversed (anti-correlated) rankings exhaust both lists.
+    for seed in (1729, 2027, 65537):
+        a, b = synth.controlled_streams(n, "correlated", seed)
+        ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+                                         policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
+        assert st["depth"] == [32, 32]
+        assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, 20)]
+    a, b = synth.controlled_streams(n, "reversed", 1729)
+    ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+                                     policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
+    assert st["exhausted"] == [1, 1] and st["depth"] == [n, n]
+    assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, 20)]
+
+
+def test_controlled_streams_independent_and_partial_read_ratios():
+    # Sec. 4.2 reports 64.5-77.9% of each list for independent rankings and a
+    # median depth of 1264 for partial overlap; the generators' random
+    # streams differ from the paper's, so these are loose checks.
+    ratios, partial = [], []
+    for seed in (1729, 2027, 65537):
+        a, b = synth.controlled_streams(100_000, "independent", seed)
+        _, _, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+                                       policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
+        ratios.append(st["depth"][0] / 100_000)
+        a, b = synth.controlled_streams(100_000, "partial", seed)
+        _, _, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+                                       policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
+        partial.append(st["depth"][0])
+    assert all(0.3 < r < 0.95 for r in ratios), ratios
+    assert 1000 <= float(np.median(partial)) <= 2000, partial
