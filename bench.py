@@ -76,6 +76,23 @@ def measured_peaks():
         return 6800.0, "fallback"
 
 
+def interval_traffic(n_rows: int):
+    """DRAM bytes per interval pass from the committed ncu capture, scaled by
+    rows; None when the kernel source changed since the capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "interval_pass_kernel_passage_8.8Mx768_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        with open(os.path.join(ROOT, d["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != d["source_sha256"]:
+                return None
+        per_row = (d["captured_dram_bytes_read"] + d["captured_dram_bytes_write"]) / d["captured_rows"]
+        return per_row * n_rows
+    except Exception:
+        return None
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled during the timed region."""
 
@@ -325,14 +342,7 @@ def main():
     alg_bytes = n * (m_pad + 12)
     achieved = alg_bytes / (interval_ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
-    traffic = None
-    prof = os.path.join(ROOT, "profiles", "interval_pass_traffic.json")
-    if os.path.exists(prof):
-        try:
-            with open(prof) as f:
-                traffic = json.load(f).get("traffic_bytes_per_pass")
-        except Exception:
-            traffic = None
+    traffic = interval_traffic(n)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
