@@ -180,6 +180,43 @@ const char* pvs_status_string(int32_t status);
 int64_t pvs_launch_count(void);
 
 /* ---------------------------------------------------------------------------
+ * Allocation-free exact ranking.  The paper has no counterpart to this entry
+ * point; it exists for callers that cannot allocate device memory where they
+ * need a ranking: code running while a CUDA stream is being captured into a
+ * graph (cudaMalloc is not permitted during most capture modes), and
+ * services whose memory pool owns the device memory budget.
+ * ------------------------------------------------------------------------ */
+
+/* Largest vector count pvs_rank_exact_noalloc accepts. */
+#define PVS_NOALLOC_MAX_VECTORS 8192
+
+/* Rank n <= PVS_NOALLOC_MAX_VECTORS row-major float32 vectors `vecs`
+ * (n x dim, DEVICE memory) against one query (dim floats, DEVICE memory) by
+ * authoritative score -- the correctly rounded exact inner product, the same
+ * score and order (score descending, ties by ascending row number) as
+ * pvs_next -- and write the first `top` <= n row numbers and scores to the
+ * DEVICE buffers out_ids (int64) and out_scores (float32).  Work is queued
+ * on `cuda_stream` (a cudaStream_t; NULL for the legacy default stream) and
+ * the call returns after it has finished.
+ *
+ * Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ * Its scratch is one static device array of 8192 64-bit keys plus a status
+ * word (64 KiB + 256 B) that every GPU loading the library holds until the
+ * process exits.  All calls share that array; it keeps the last call's keys,
+ * the status word is cleared by every call, and calls whose device work
+ * overlaps (e.g. on two streams at once) race on it.  The first call on a
+ * device looks up the array's device address (cudaGetSymbolAddress) with that
+ * device current; make that first call before any stream capture begins.
+ *
+ * Errors: PVS_ERR_INVALID when n > PVS_NOALLOC_MAX_VECTORS, n < 0, top > n,
+ * dim outside [1, 32767], or a pointer is not device memory;
+ * PVS_ERR_NONFINITE for a NaN or infinite entry; PVS_ERR_OVERFLOW when a
+ * score overflows float32; PVS_ERR_CUDA when a CUDA call fails. */
+pvs_status pvs_rank_exact_noalloc(const float* query, const float* vecs, int32_t n, int32_t dim,
+                                  int32_t top, int64_t* out_ids, float* out_scores,
+                                  void* cuda_stream);
+
+/* ---------------------------------------------------------------------------
  * EAHR (Sec. 2.1, 2.2): ordered Top-K of complete-list weighted RRF over the
  * dense ranked list of a cursor and a sparse ranked list from the caller.
  * ------------------------------------------------------------------------ */

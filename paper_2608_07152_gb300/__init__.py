@@ -93,6 +93,7 @@ def _load() -> ctypes.CDLL:
         "pvs_cursor_close": (None, [P]),
         "pvs_status_string": (ctypes.c_char_p, [i32]),
         "pvs_launch_count": (i64, []),
+        "pvs_rank_exact_noalloc": (i32, [P, P, i32, i32, i32, P, P, P]),
         "eahr_topk": (i32, [P, P, i64, ctypes.POINTER(eahr_params), P, P, P,
                             ctypes.POINTER(eahr_stats)]),
         "eahr_topk_lists": (i32, [P, i64, P, i64, ctypes.POINTER(eahr_params), P, P, P,
@@ -112,7 +113,8 @@ EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_i
             "pvs_snapshot_visible", "pvs_snapshot_free", "pvs_cursor_open",
             "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
-            "pvs_status_string", "pvs_launch_count", "eahr_topk", "eahr_topk_lists")
+            "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
+            "eahr_topk_lists")
 
 
 def pvs_status_string(status: int) -> str:
@@ -274,6 +276,28 @@ def pvs_cursor_score_ids(cursor, ids):
 
 def pvs_cursor_close(cursor) -> None:
     _lib.pvs_cursor_close(cursor)
+
+
+PVS_NOALLOC_MAX_VECTORS = 8192
+
+
+def pvs_rank_exact_noalloc(query, vecs, top: int, out_ids, out_scores) -> int:
+    """Allocation-free exact ranking of the rows of `vecs` against `query`
+    (both contiguous float32 CUDA tensors) into the caller's CUDA tensors
+    out_ids (int64, >= top) and out_scores (float32, >= top).  Neither this
+    wrapper nor the library allocates device memory: callers that cannot
+    (code inside a stream capture, pool-managed services) pass tensors they
+    already own.  Runs on torch's current stream and returns after it."""
+    import torch
+    for t in (query, vecs, out_ids, out_scores):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()):
+            raise TypeError("pvs_rank_exact_noalloc takes contiguous CUDA tensors")
+    n, dim = (vecs.shape[0], vecs.shape[1]) if vecs.dim() == 2 else (0, query.shape[-1])
+    stream = torch.cuda.current_stream(vecs.device).cuda_stream
+    return _check(_lib.pvs_rank_exact_noalloc(
+        ctypes.c_void_p(query.data_ptr()), ctypes.c_void_p(vecs.data_ptr()), int(n), int(dim),
+        int(top), ctypes.c_void_p(out_ids.data_ptr()), ctypes.c_void_p(out_scores.data_ptr()),
+        ctypes.c_void_p(stream) if stream else None), "pvs_rank_exact_noalloc")
 
 
 def _params(K, k, form, policy, step, weights):

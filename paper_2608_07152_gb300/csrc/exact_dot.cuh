@@ -1,0 +1,170 @@
+// Exact authoritative float32 score of one vector, computed by one warp
+// (arXiv 2608.07152 Sec. 2.3.1 authoritative scores; App. A.1).
+//
+// The score is RN_f32 of the exact inner product sum_j q_j v_j:
+//   * every product of two float32 values is exact in binary64; lanes
+//     accumulate S = sum p_j and A = sum |p_j| in binary64 and reduce them;
+//   * |S - exact| <= (m - 1) u A / (1 - (m - 1) u) with u = 2^-53 for any
+//     summation order; with beta = 4 m u A the whole interval
+//     [RD(S - beta), RU(S + beta)] rounds to one float32 value in all but
+//     rare cases, and that value is the answer;
+//   * otherwise the warp sums the products exactly in a fixed-point
+//     accumulator (20 signed 32-bit digits in int64 slots, weight 2^-352 for
+//     the lowest bit) and rounds the exact sum to nearest-even.
+#pragma once
+
+#include "pvs_common.cuh"
+
+namespace pvs {
+
+constexpr int kAccDigits = 20;
+constexpr int kAccBase = 352;   // bit 0 of the accumulator has weight 2^-352
+
+// Add one exact binary64 product into the per-lane fixed-point accumulator.
+__device__ inline void acc_add(long long* acc, double p) {
+    if (p == 0.0) return;
+    const unsigned long long bits = (unsigned long long)__double_as_longlong(p);
+    const int bexp = (int)((bits >> 52) & 0x7ff);           // normal: |p| >= 2^-298
+    const unsigned long long mant = (bits & 0xfffffffffffffull) | (1ull << 52);
+    const int pos = bexp - 1075 + kAccBase;                 // weight of mant's bit 0
+    const int d = pos >> 5, o = pos & 31;
+    // products of finite float32 values always land in range; anything else
+    // (callers check finiteness first) is ignored rather than written out of bounds
+    if (bexp == 0 || bexp == 0x7ff || pos < 0 || d + 2 >= kAccDigits) return;
+    unsigned long long w0, rest;
+    if (o == 0) {
+        w0 = mant & 0xffffffffull;
+        rest = mant >> 32;
+    } else {
+        w0 = (mant & ((1ull << (32 - o)) - 1ull)) << o;
+        rest = mant >> (32 - o);
+    }
+    const unsigned long long w1 = rest & 0xffffffffull, w2 = rest >> 32;
+    if (bits >> 63) {
+        acc[d] -= (long long)w0;
+        acc[d + 1] -= (long long)w1;
+        acc[d + 2] -= (long long)w2;
+    } else {
+        acc[d] += (long long)w0;
+        acc[d + 1] += (long long)w1;
+        acc[d + 2] += (long long)w2;
+    }
+}
+
+// Round the exact value held in normalised digits (magnitude, sign) to the
+// nearest float32, ties to even.
+__device__ inline float acc_round(const unsigned int* mag, bool negative) {
+    int top = -1;
+    for (int k = kAccDigits - 1; k >= 0; --k)
+        if (mag[k]) {
+            top = 32 * k + 31 - __clz(mag[k]);
+            break;
+        }
+    if (top < 0) return 0.0f;
+    auto bit = [&](int i) -> unsigned int {
+        return i < 0 ? 0u : (mag[i >> 5] >> (i & 31)) & 1u;
+    };
+    const int sub_lsb = -149 + kAccBase;     // bit index of 2^-149
+    int lsb = top - 23;
+    if (lsb < sub_lsb) lsb = sub_lsb;
+    unsigned long long M = 0;
+    for (int i = top; i >= lsb; --i) M = (M << 1) | bit(i);
+    const unsigned int rbit = bit(lsb - 1);
+    bool sticky = false;
+    for (int i = lsb - 2; i >= 0 && !sticky; --i) sticky = bit(i) != 0;
+    if (rbit && (sticky || (M & 1ull))) ++M;
+    // M <= 2^24; value = M * 2^(lsb - kAccBase), exact in binary64
+    double v = (double)M * pow2d(lsb - kAccBase);
+    float f = __double2float_rn(v);   // exact when representable; inf on overflow
+    return negative ? -f : f;
+}
+
+// Products q_j * v_j of one lane, visited in a fixed order: float4 loads for
+// 16-byte aligned rows whose length is a multiple of 4 (the index layout),
+// scalar loads otherwise.
+template <bool kVec4, typename F>
+__device__ inline void for_lane_products(const float* __restrict__ q, const float* __restrict__ v,
+                                         int m, F&& f) {
+    const int lane = threadIdx.x & 31;
+    if constexpr (kVec4) {
+        const float4* q4 = reinterpret_cast<const float4*>(q);
+        const float4* v4 = reinterpret_cast<const float4*>(v);
+        for (int j = lane; j < (m >> 2); j += kWarp) {
+            const float4 a = __ldg(q4 + j), b = __ldg(v4 + j);
+            f(__dmul_rn((double)a.x, (double)b.x), __dmul_rn((double)a.y, (double)b.y),
+              __dmul_rn((double)a.z, (double)b.z), __dmul_rn((double)a.w, (double)b.w));
+        }
+    } else {
+        for (int j = lane; j < m; j += kWarp)
+            f(__dmul_rn((double)__ldg(q + j), (double)__ldg(v + j)), 0.0, 0.0, 0.0);
+    }
+}
+
+// One warp: exact RN_f32(sum q_j v_j) over m finite entries.
+template <bool kVec4>
+__device__ inline float exact_dot_warp_impl(const float* __restrict__ q,
+                                            const float* __restrict__ v, int m,
+                                            bool* used_fallback) {
+    double S = 0.0, A = 0.0;
+    for_lane_products<kVec4>(q, v, m, [&](double p0, double p1, double p2, double p3) {
+        S = __dadd_rn(S, __dadd_rn(__dadd_rn(p0, p1), __dadd_rn(p2, p3)));
+        A = __dadd_rn(A, __dadd_rn(__dadd_rn(fabs(p0), fabs(p1)), __dadd_rn(fabs(p2), fabs(p3))));
+    });
+    S = warp_sum(S);
+    A = warp_sum(A);
+    const double beta = __dmul_ru(A, 4.0 * (double)m * 0x1p-53);
+    const float flo = __double2float_rn(__dsub_rd(S, beta));
+    const float fhi = __double2float_rn(__dadd_ru(S, beta));
+    if (flo == fhi) {
+        *used_fallback = false;
+        return flo == 0.0f ? 0.0f : flo;
+    }
+    // exact fallback
+    *used_fallback = true;
+    long long acc[kAccDigits];
+#pragma unroll
+    for (int k = 0; k < kAccDigits; ++k) acc[k] = 0;
+    for_lane_products<kVec4>(q, v, m, [&](double p0, double p1, double p2, double p3) {
+        acc_add(acc, p0);
+        acc_add(acc, p1);
+        acc_add(acc, p2);
+        acc_add(acc, p3);
+    });
+#pragma unroll
+    for (int k = 0; k < kAccDigits; ++k) acc[k] = warp_sum(acc[k]);
+    // normalise: carry-propagate signed digits into 32-bit digits
+    unsigned int mag[kAccDigits];
+    long long carry = 0;
+#pragma unroll
+    for (int k = 0; k < kAccDigits; ++k) {
+        const long long x = acc[k] + carry;
+        mag[k] = (unsigned int)(x & 0xffffffffll);
+        carry = x >> 32;   // arithmetic shift: floor division
+    }
+    const bool negative = carry < 0;
+    if (negative) {  // two's complement negate over all digits
+        unsigned long long c = 1;
+#pragma unroll
+        for (int k = 0; k < kAccDigits; ++k) {
+            const unsigned long long x = (unsigned long long)(~mag[k]) + c;
+            mag[k] = (unsigned int)x;
+            c = x >> 32;
+        }
+    }
+    return acc_round(mag, negative);
+}
+
+// Index rows: 16-byte aligned, m_raw a multiple of 4 (zero padded).
+__device__ inline float exact_dot_warp(const float* __restrict__ q, const float* __restrict__ v,
+                                       int m_raw, bool* used_fallback) {
+    return exact_dot_warp_impl<true>(q, v, m_raw, used_fallback);
+}
+
+// Any row of m float32 values.
+__device__ inline float exact_dot_warp_any(const float* __restrict__ q,
+                                           const float* __restrict__ v, int m,
+                                           bool* used_fallback) {
+    return exact_dot_warp_impl<false>(q, v, m, used_fallback);
+}
+
+}  // namespace pvs
