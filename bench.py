@@ -164,12 +164,43 @@ def build_corpus_index(pvs, synth, torch, n, stream, device):
     return index, centres, time.perf_counter() - t0
 
 
-def run_step_device(pvs, torch, index, queries, out_ids, out_scores, stream, lat20, lat1000,
-                    stats_acc):
+PIPELINE = 2   # queries in flight, each on its own stream
+
+
+def _finish(pvs, cur, stats_acc):
+    st = pvs.pvs_cursor_sync(cur)
+    s = pvs.pvs_cursor_stats(cur)
+    pvs.pvs_cursor_close(cur)
+    if st < 0:
+        raise RuntimeError(f"cursor failed: {st}")
+    if stats_acc is not None:
+        stats_acc.append(s)
+
+
+def run_step_device(pvs, index, queries, out_ids, out_scores, streams, stats_acc):
     """One step: every query opens a cursor and pulls 1,000 ranks in chunks
-    of 20 into device buffers."""
-    ev = []
+    of 20 into device buffers.  Up to PIPELINE queries are in flight on their
+    own streams, so one query's pulls overlap the next query's interval pass;
+    every pull is still a separate pvs_next_device call."""
+    pending = []
     for qi in range(queries.shape[0]):
+        slot = qi % PIPELINE
+        cur = pvs.pvs_cursor_open(index, queries[qi])
+        pvs.pvs_cursor_set_stream(cur, streams[slot])
+        for p in range(RANKS_PER_QUERY // CHUNK):
+            off = p * CHUNK
+            pvs.pvs_next_device(cur, CHUNK, out_ids[slot, off:], out_scores[slot, off:])
+        pending.append(cur)
+        if len(pending) >= PIPELINE:
+            _finish(pvs, pending.pop(0), stats_acc)
+    while pending:
+        _finish(pvs, pending.pop(0), stats_acc)
+
+
+def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, count):
+    """Latency to the first 20 and first 1,000 ranks, one query at a time."""
+    lat20, lat1000 = [], []
+    for qi in range(count):
         t_open = torch.cuda.Event(enable_timing=True)
         t_20 = torch.cuda.Event(enable_timing=True)
         t_end = torch.cuda.Event(enable_timing=True)
@@ -177,29 +208,42 @@ def run_step_device(pvs, torch, index, queries, out_ids, out_scores, stream, lat
         cur = pvs.pvs_cursor_open(index, queries[qi])
         for p in range(RANKS_PER_QUERY // CHUNK):
             off = p * CHUNK
-            pvs.pvs_next_device(cur, CHUNK, out_ids[qi, off:], out_scores[qi, off:])
+            pvs.pvs_next_device(cur, CHUNK, out_ids[0, off:], out_scores[0, off:])
             if p == 0:
                 t_20.record(stream)
         t_end.record(stream)
-        st = pvs.pvs_cursor_sync(cur)
-        s = pvs.pvs_cursor_stats(cur)
-        pvs.pvs_cursor_close(cur)
-        if st < 0:
-            raise RuntimeError(f"cursor failed: {st}")
-        ev.append((t_open, t_20, t_end))
-        stats_acc.append(s)
-    stream.synchronize()
-    for a, b, c in ev:
-        lat20.append(a.elapsed_time(b))
-        lat1000.append(a.elapsed_time(c))
+        _finish(pvs, cur, None)
+        stream.synchronize()
+        lat20.append(t_open.elapsed_time(t_20))
+        lat1000.append(t_open.elapsed_time(t_end))
+    return lat20, lat1000
 
 
-def run_step_host(pvs, index, queries_host):
-    for q in queries_host:
-        cur = pvs.pvs_cursor_open(index, q)
-        for p in range(RANKS_PER_QUERY // CHUNK):
-            ids, sc, st = pvs.pvs_next(cur, CHUNK)
-        pvs.pvs_cursor_close(cur)
+def run_step_host(pvs, torch, index, queries_host, streams):
+    """The same step through host buffers (pvs_next); PIPELINE host threads
+    each drive their own cursors and stream."""
+    import threading
+
+    errors = []
+
+    def worker(k):
+        try:
+            for q in queries_host[k::PIPELINE]:
+                cur = pvs.pvs_cursor_open(index, q)
+                pvs.pvs_cursor_set_stream(cur, streams[k])
+                for p in range(RANKS_PER_QUERY // CHUNK):
+                    pvs.pvs_next(cur, CHUNK)
+                pvs.pvs_cursor_close(cur)
+        except Exception as e:  # surfaced below
+            errors.append(e)
+
+    threads = [threading.Thread(target=worker, args=(k,)) for k in range(PIPELINE)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    if errors:
+        raise errors[0]
 
 
 def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget=20.0):
@@ -287,13 +331,14 @@ def main():
     total_q = (args.warmup + args.steps) * args.queries
     queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=3 + 7919 * rank)
     queries = queries.reshape(args.warmup + args.steps, args.queries, DIM).contiguous()
-    out_ids = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
-    out_scores = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    out_ids = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
+    out_scores = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    streams = [torch.cuda.Stream(device=dev) for _ in range(PIPELINE)]
     torch.cuda.synchronize()
 
-    lat20, lat1000, stats = [], [], []
+    stats = []
     for w in range(args.warmup):
-        run_step_device(pvs, torch, index, queries[w], out_ids, out_scores, stream, [], [], [])
+        run_step_device(pvs, index, queries[w], out_ids, out_scores, streams, None)
 
     # ---- timed region: device-resident queries and outputs ----
     if pg:
@@ -304,9 +349,15 @@ def main():
     end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         start.record(stream)
+        for s_ in streams:
+            s_.wait_event(start)
         for s in range(args.steps):
-            run_step_device(pvs, torch, index, queries[args.warmup + s], out_ids, out_scores,
-                            stream, lat20, lat1000, stats)
+            run_step_device(pvs, index, queries[args.warmup + s], out_ids, out_scores, streams,
+                            stats)
+        for s_ in streams:                      # join every stream's work
+            done = torch.cuda.Event()
+            done.record(s_)
+            stream.wait_event(done)
         end.record(stream)
         stream.synchronize()
     torch.cuda.synchronize()
@@ -326,9 +377,13 @@ def main():
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for s in range(args.steps):
-        run_step_host(pvs, index, qh[s])
+        run_step_host(pvs, torch, index, qh[s], streams)
     torch.cuda.synchronize()
     e2e_elapsed = time.perf_counter() - t0
+
+    # ---- latency, one query at a time ----
+    lat20, lat1000 = measure_latency(pvs, torch, index, queries[args.warmup],
+                                     out_ids, out_scores, stream, min(args.queries, 20))
     if pg:
         t = torch.tensor([e2e_elapsed], device=dev)
         pg.all_reduce(t, op=pg.ReduceOp.MAX)

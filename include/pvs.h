@@ -20,10 +20,14 @@
  *   - "on_device" flags say whether a pointer is CUDA device memory (or
  *     managed memory) of the current device (1) or host memory (0).
  *   - The library owns index, snapshot and cursor objects; the caller owns
- *     every buffer it passes in.  Objects are not thread-safe: calls on one
- *     index, its snapshots and its cursors must not run concurrently.
- *   - All device work runs on the CUDA stream given to pvs_build (or a
- *     library-created stream when NULL).
+ *     every buffer it passes in.  Threads: distinct cursors of one index may
+ *     be opened, pulled and closed from different host threads at once; a
+ *     single cursor must not be used by two threads at once, and index
+ *     mutations (pvs_append, pvs_tombstone, pvs_index_free) must not overlap
+ *     any other call on that index.
+ *   - Index work runs on the CUDA stream given to pvs_build (or a
+ *     library-created stream when NULL); a cursor's work runs on that stream
+ *     too unless pvs_cursor_set_stream moves it.
  */
 #ifndef PVS_H_
 #define PVS_H_
@@ -153,6 +157,13 @@ pvs_status pvs_next(pvs_cursor* cursor, int32_t n, int64_t* ids, float* scores, 
  * successful blocking call is then void. */
 pvs_status pvs_next_device(pvs_cursor* cursor, int32_t n, int64_t* ids, float* scores,
                            int32_t* n_out);
+
+/* Run the cursor's later device work on `cuda_stream` (a cudaStream_t; NULL:
+ * back to the index's stream), after waiting for its queued work.  Cursors on
+ * different streams overlap on the device: one query's pulls can run while
+ * another query's interval pass streams the codes.  Ordering against work
+ * the caller queues elsewhere is the caller's. */
+pvs_status pvs_cursor_set_stream(pvs_cursor* cursor, void* cuda_stream);
 
 /* Wait for the cursor's queued work; return its state (PVS_OK while Open,
  * PVS_EXHAUSTED, or the failure). */

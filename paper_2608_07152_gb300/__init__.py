@@ -87,6 +87,7 @@ def _load() -> ctypes.CDLL:
         "pvs_next": (i32, [P, i32, P, P, P]),
         "pvs_next_device": (i32, [P, i32, P, P, P]),
         "pvs_cursor_sync": (i32, [P]),
+        "pvs_cursor_set_stream": (i32, [P, P]),
         "pvs_cursor_stats": (i32, [P, ctypes.POINTER(pvs_stats)]),
         "pvs_cursor_bounds": (i32, [P, i64, i64, P, P]),
         "pvs_cursor_score_ids": (i32, [P, P, i32, P]),
@@ -112,6 +113,7 @@ EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_i
             "pvs_index_dim", "pvs_index_export", "pvs_index_free", "pvs_snapshot_create",
             "pvs_snapshot_visible", "pvs_snapshot_free", "pvs_cursor_open",
             "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
+            "pvs_cursor_set_stream",
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
             "eahr_topk_lists")
@@ -250,6 +252,13 @@ def pvs_next_device(cursor, n: int, ids, scores):
 
 def pvs_cursor_sync(cursor) -> int:
     return _check(_lib.pvs_cursor_sync(cursor), "pvs_cursor_sync")
+
+
+def pvs_cursor_set_stream(cursor, stream) -> None:
+    """stream: a torch.cuda.Stream, a raw cudaStream_t handle, or None."""
+    handle = getattr(stream, "cuda_stream", stream)
+    _check(_lib.pvs_cursor_set_stream(cursor, ctypes.c_void_p(handle) if handle else None),
+           "pvs_cursor_set_stream")
 
 
 def pvs_cursor_stats(cursor) -> dict:

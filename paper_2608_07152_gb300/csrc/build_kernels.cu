@@ -47,8 +47,10 @@ cudaError_t launch_build(const float* vecs, int64_t n, int m, int m_pad, int m_r
 
 // Query encoding: the same quantizer, plus ||s_q z_q|| rounded up and
 // gamma_m = RU(a / RD(1 - a)), a = (8m + 64) 2^-23 (App. A.1).
-__global__ void encode_kernel(const float* __restrict__ q, int nq, int m, int m_pad, int m_raw,
-                              int8_t* __restrict__ zq, float* __restrict__ qraw,
+// q and qraw may be the same buffer (a host query staged in qraw): the raw
+// copy then rewrites the values it read.
+__global__ void encode_kernel(const float* q, int nq, int m, int m_pad, int m_raw,
+                              int8_t* __restrict__ zq, float* qraw,
                               QueryScalars* __restrict__ qs) {
     const int lane = threadIdx.x & 31;
     const int qi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);

@@ -36,7 +36,30 @@ struct DevCounters {
     unsigned long long exact_fallbacks;
     unsigned int w_len;      // working-set length
     unsigned int cand;       // candidates of the current pull
+    unsigned long long cand_total;   // candidates over fused pulls
 };
+
+// ---- fused single-CTA pull (pull_kernel.cu) ----------------------------------
+constexpr int kPullFusedMax = 256;   // largest pull served by one fused launch
+struct PullArgs {
+    int32_t* w_id;
+    float* w_lo;
+    float* w_hi;
+    const unsigned int* w_len;
+    float* lo;                // bounds of every row (kept in step with the working set)
+    float* hi;
+    const float* qraw;
+    const float* raw;
+    int m_raw;
+    int n;                    // ranks to emit, 1 .. kPullFusedMax
+    int32_t* cand;            // scratch, >= working-set capacity
+    unsigned long long* keys; // scratch, >= working-set capacity
+    int64_t* out_ids;         // device
+    float* out_scores;        // device
+    int* status;
+    DevCounters* ctr;
+};
+cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
 
 // ---- build / encode (build_kernels.cu) -------------------------------------
 // Quantize rows [0, n) of `vecs` (row stride m floats) into codes (stride

@@ -200,10 +200,34 @@ void cursor_free_device(pvs_cursor* c) {
     c->ev_begin = c->ev_end = nullptr;
 }
 
-// Allocate the per-row state of a cursor (first pull).
+// Host-side state of a fresh cursor; device buffers are kept for reuse.
+void cursor_reset(pvs_cursor* c) {
+    c->index = nullptr;
+    c->snap.reset();
+    c->rows = c->visible = c->emitted = 0;
+    c->state = PVS_OK;
+    c->scanned = false;
+    c->horizon = c->horizon_base = 0;
+    c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
+    c->ev_pending = false;
+    c->interval_ms = 0.0;
+}
+
+constexpr size_t kCursorPool = 4;   // closed cursors kept per index
+
+// Allocate the per-row state of a cursor (first pull); a pooled cursor keeps
+// buffers that are large enough.
 pvs_status cursor_alloc_rows(pvs_cursor* c) {
-    if (c->lo) return PVS_OK;
+    if (c->lo && c->cap_rows >= c->rows) return PVS_OK;
+    dev_free(c->lo), dev_free(c->hi);
+    dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
+    dev_free(c->compact_scratch);
+    dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp);
+    if (c->sort_scratch) cudaFree(c->sort_scratch);
+    c->sort_scratch = nullptr;
+    c->cap_rows = 0;
     const size_t n = (size_t)std::max<int64_t>(c->rows, 1);
+    c->cap_rows = (int64_t)n;
     PVS_CUDA(dev_alloc(&c->lo, n));
     PVS_CUDA(dev_alloc(&c->hi, n));
     PVS_CUDA(dev_alloc(&c->w_id, n));
@@ -256,7 +280,7 @@ void harvest_interval_time(pvs_cursor* c) {
 
 // Read the device status word; a failure makes the cursor Failed.
 pvs_status check_device_status(pvs_cursor* c) {
-    cudaStream_t st = c->index->stream;
+    cudaStream_t st = c->stream;
     PVS_CUDA(cudaMemcpyAsync(c->h_small, c->d_status, sizeof(int), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaStreamSynchronize(st));
     const int s = (int)c->h_small[0];
@@ -283,9 +307,16 @@ pvs_status interval_pass(pvs_cursor* c) {
         PVS_CUDA(cudaEventCreate(&c->ev_begin));
         PVS_CUDA(cudaEventCreate(&c->ev_end));
     }
-    PVS_CUDA(cudaEventRecord(c->ev_begin, x->stream));
-    PVS_CUDA(launch_interval_pass(a, x->num_sms, x->stream));
-    PVS_CUDA(cudaEventRecord(c->ev_end, x->stream));
+    // Interval passes of one index run one after another: each saturates
+    // HBM, so overlapping two gains nothing; pulls of other cursors still
+    // overlap the pass.  The pass waits for the previous pass's end event.
+    std::lock_guard<std::mutex> lock(x->pass_mutex);
+    if (!x->pass_done) PVS_CUDA(cudaEventCreateWithFlags(&x->pass_done, cudaEventDisableTiming));
+    else PVS_CUDA(cudaStreamWaitEvent(c->stream, x->pass_done, 0));
+    PVS_CUDA(cudaEventRecord(c->ev_begin, c->stream));
+    PVS_CUDA(launch_interval_pass(a, x->num_sms, c->stream));
+    PVS_CUDA(cudaEventRecord(c->ev_end, c->stream));
+    PVS_CUDA(cudaEventRecord(x->pass_done, c->stream));
     c->ev_pending = true;
     c->interval_passes++;
     c->scanned = true;
@@ -300,12 +331,12 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     if (H > remaining) H = remaining;
     if (H < remaining) {
         PVS_CUDA(launch_select_f32_n(c->lo, c->rows, (uint64_t)H, c->sel, grid_for(c, c->rows),
-                                     x->stream));
+                                     c->stream));
     } else {
-        PVS_CUDA(cudaMemsetAsync(c->sel, 0, sizeof(SelectState), x->stream));  // tau = 0: all live
+        PVS_CUDA(cudaMemsetAsync(c->sel, 0, sizeof(SelectState), c->stream));  // tau = 0: all live
     }
     PVS_CUDA(launch_compact_ordered(c->lo, c->hi, c->rows, c->sel, c->w_id, c->w_lo, c->w_hi,
-                                    &c->ctr->w_len, c->compact_scratch, x->stream));
+                                    &c->ctr->w_len, c->compact_scratch, c->stream));
     c->horizon = H;
     c->horizon_base = c->emitted;
     c->horizon_builds++;
@@ -315,7 +346,7 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
 // One pull of n_eff >= 1 ranks into device buffers d_ids / d_scores.
 pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
     pvs_index* x = c->index;
-    cudaStream_t st = x->stream;
+    cudaStream_t st = c->stream;
     pvs_status s = cursor_alloc_rows(c);
     if (s != PVS_OK) return fail(c, s);
     if (!c->scanned) {
@@ -325,6 +356,31 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
     if (c->emitted + n_eff - c->horizon_base > c->horizon) {
         s = build_working_set(c, n_eff);
         if (s != PVS_OK) return fail(c, s);
+    }
+    if (n_eff <= kPullFusedMax) {
+        // one launch, no host round trip; failures surface at the next sync
+        PullArgs a;
+        a.w_id = c->w_id;
+        a.w_lo = c->w_lo;
+        a.w_hi = c->w_hi;
+        a.w_len = &c->ctr->w_len;
+        a.lo = c->lo;
+        a.hi = c->hi;
+        a.qraw = c->qraw;
+        a.raw = x->raw;
+        a.m_raw = x->m_raw;
+        a.n = (int)n_eff;
+        a.cand = c->cand;
+        a.keys = reinterpret_cast<unsigned long long*>(c->keys);
+        a.out_ids = d_ids;
+        a.out_scores = d_scores;
+        a.status = c->d_status;
+        a.ctr = c->ctr;
+        cudaError_t e = launch_pull_fused(a, 2 * x->num_sms, st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        c->emitted += n_eff;
+        c->pulls++;
+        return PVS_OK;
     }
     const int grid_w = grid_for(c, std::min<int64_t>(c->rows, (int64_t)1 << 22));
     cudaError_t e = launch_select_f32(c->w_lo, &c->ctr->w_len, (uint64_t)n_eff, c->sel, grid_w, st);
@@ -368,6 +424,13 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
 extern "C" {
 
 int64_t pvs_launch_count(void) { return (int64_t)g_launches.load(); }
+
+pvs_status pvs_cursor_set_stream(pvs_cursor* c, void* cuda_stream) {
+    if (!c || !c->index) return PVS_ERR_INVALID;
+    PVS_CUDA(cudaStreamSynchronize(c->stream));
+    c->stream = cuda_stream ? static_cast<cudaStream_t>(cuda_stream) : c->index->stream;
+    return PVS_OK;
+}
 
 const char* pvs_status_string(int32_t s) {
     switch (s) {
@@ -477,8 +540,14 @@ pvs_status pvs_index_export(const pvs_index* x, int64_t first, int64_t count, in
 void pvs_index_free(pvs_index* x) {
     if (!x) return;
     if (x->stream) cudaStreamSynchronize(x->stream);
+    for (pvs_cursor* c : x->cursor_pool) {
+        cursor_free_device(c);
+        delete c;
+    }
+    x->cursor_pool.clear();
     dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
     dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage);
+    if (x->pass_done) cudaEventDestroy(x->pass_done);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
 }
@@ -506,43 +575,52 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
     *out = nullptr;
     if (!x || !query || (snap && snap->index != x)) return PVS_ERR_INVALID;
     if (query_on_device && !is_device_ptr(query)) return PVS_ERR_INVALID;
-    pvs_cursor* c = new (std::nothrow) pvs_cursor();
-    if (!c) return PVS_ERR_OOM;
+    pvs_cursor* c = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(x->pool_mutex);
+        if (!x->cursor_pool.empty()) {   // reuse a closed cursor's buffers
+            c = x->cursor_pool.back();
+            x->cursor_pool.pop_back();
+        }
+    }
+    if (!c) {
+        c = new (std::nothrow) pvs_cursor();
+        if (!c) return PVS_ERR_OOM;
+    }
     auto bail = [&](pvs_status s) {
         cursor_free_device(c);
         delete c;
         return s;
     };
+    cursor_reset(c);
     c->index = x;
+    c->stream = x->stream;
     c->snap = snap ? snap->data : make_snapdata(x);
     if (!c->snap) return bail(PVS_ERR_OOM);
     c->rows = c->snap->rows;
     c->visible = c->snap->visible;
-    cudaStream_t st = x->stream;
-    if (dev_alloc(&c->zq, (size_t)x->m_pad) != cudaSuccess ||
-        dev_alloc(&c->qraw, (size_t)x->m_raw) != cudaSuccess ||
-        dev_alloc(&c->qs, 1) != cudaSuccess || dev_alloc(&c->sel, 1) != cudaSuccess ||
-        dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
-        cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess)
+    cudaStream_t st = c->stream;
+    if (!c->zq &&
+        (dev_alloc(&c->zq, (size_t)x->m_pad) != cudaSuccess ||
+         dev_alloc(&c->qraw, (size_t)x->m_raw) != cudaSuccess ||
+         dev_alloc(&c->qs, 1) != cudaSuccess || dev_alloc(&c->sel, 1) != cudaSuccess ||
+         dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
+         cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess))
         return bail(PVS_ERR_OOM);
+    // a host query is staged in the cursor's raw query buffer, which the
+    // encoder then rewrites in place with the same values (plus zero padding)
     const float* qd = query;
-    float* tmp = nullptr;
+    cudaError_t e = cudaSuccess;
     if (!query_on_device) {
-        if (dev_alloc(&tmp, (size_t)x->m) != cudaSuccess) return bail(PVS_ERR_OOM);
-        if (cudaMemcpyAsync(tmp, query, x->m * sizeof(float), cudaMemcpyHostToDevice, st) !=
-            cudaSuccess) {
-            cudaFree(tmp);
-            return bail(PVS_ERR_CUDA);
-        }
-        qd = tmp;
+        e = cudaMemcpyAsync(c->qraw, query, x->m * sizeof(float), cudaMemcpyHostToDevice, st);
+        qd = c->qraw;
     }
-    cudaError_t e = cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), st);
     if (e == cudaSuccess) e = cudaMemsetAsync(c->d_status, 0, sizeof(int), st);
     if (e == cudaSuccess) e = launch_encode_query(qd, x->m, x->m_pad, x->m_raw, c->zq, c->qraw, c->qs, st);
     QueryScalars qs{};
     if (e == cudaSuccess) e = cudaMemcpyAsync(&qs, c->qs, sizeof(qs), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
-    if (tmp) cudaFree(tmp);
     if (e != cudaSuccess) return bail(cuda_status(e));
     if (qs.status != 0) return bail((pvs_status)qs.status);
     c->state = c->visible == 0 ? PVS_EXHAUSTED : PVS_OK;
@@ -589,7 +667,7 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         if (s != PVS_OK) return fail(c, s);
         s = pull(c, n_eff, c->d_ids, c->d_scores);
         if (s != PVS_OK) return s;
-        cudaStream_t st = c->index->stream;
+        cudaStream_t st = c->stream;
         cudaError_t e = cudaMemcpyAsync(c->h_ids, c->d_ids, n_eff * sizeof(int64_t),
                                         cudaMemcpyDeviceToHost, st);
         if (e == cudaSuccess)
@@ -633,8 +711,8 @@ pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
     if (!c || !out) return PVS_ERR_INVALID;
     std::memset(out, 0, sizeof(*out));
     DevCounters d{};
-    cudaError_t e = cudaMemcpyAsync(&d, c->ctr, sizeof(d), cudaMemcpyDeviceToHost, c->index->stream);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(c->index->stream);
+    cudaError_t e = cudaMemcpyAsync(&d, c->ctr, sizeof(d), cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) return cuda_status(e);
     if (c->state >= 0) check_device_status(c);
     out->visible = c->visible;
@@ -644,7 +722,7 @@ pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
     out->interval_passes = c->interval_passes;
     out->horizon_builds = c->horizon_builds;
     out->pulls = c->pulls;
-    out->candidates = c->candidates;
+    out->candidates = c->candidates + (int64_t)d.cand_total;
     out->code_bytes = c->interval_passes * c->rows * (int64_t)(c->index->m_pad + 12);
     out->state = c->state;
     harvest_interval_time(c);
@@ -666,7 +744,7 @@ pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float*
         if (s != PVS_OK) return s;
     }
     if (count == 0) return PVS_OK;
-    cudaStream_t st = c->index->stream;
+    cudaStream_t st = c->stream;
     PVS_CUDA(cudaMemcpyAsync(lo, c->lo + first, count * sizeof(float), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaMemcpyAsync(hi, c->hi + first, count * sizeof(float), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaStreamSynchronize(st));
@@ -678,7 +756,7 @@ pvs_status pvs_cursor_score_ids(pvs_cursor* c, const int64_t* ids, int32_t n, fl
     for (int32_t i = 0; i < n; ++i)
         if (ids[i] < 0 || ids[i] >= c->rows) return PVS_ERR_INVALID;
     if (n == 0) return PVS_OK;
-    cudaStream_t st = c->index->stream;
+    cudaStream_t st = c->stream;
     int64_t* d_ids = nullptr;
     float* d_out = nullptr;
     cudaError_t e = dev_alloc(&d_ids, (size_t)n);
@@ -697,7 +775,17 @@ pvs_status pvs_cursor_score_ids(pvs_cursor* c, const int64_t* ids, int32_t n, fl
 
 void pvs_cursor_close(pvs_cursor* c) {
     if (!c) return;
-    if (c->index && c->index->stream) cudaStreamSynchronize(c->index->stream);
+    pvs_index* x = c->index;
+    if (x) cudaStreamSynchronize(c->stream);
+    harvest_interval_time(c);
+    if (x) {
+        std::lock_guard<std::mutex> lock(x->pool_mutex);
+        if (x->cursor_pool.size() < kCursorPool) {   // keep the buffers for the next cursor
+            cursor_reset(c);
+            x->cursor_pool.push_back(c);
+            return;
+        }
+    }
     cursor_free_device(c);
     delete c;
 }

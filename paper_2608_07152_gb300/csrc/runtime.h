@@ -3,6 +3,7 @@
 
 #include <cstdint>
 #include <memory>
+#include <mutex>
 #include <vector>
 
 #include <cuda_runtime.h>
@@ -44,6 +45,10 @@ struct pvs_index {
     int* d_status = nullptr;
     float* d_stage = nullptr;         // host-input staging
     size_t stage_floats = 0;
+    std::vector<pvs_cursor*> cursor_pool;   // closed cursors whose buffers are reused
+    std::mutex pool_mutex;                  // cursors may open / close on several threads
+    std::mutex pass_mutex;                  // orders interval passes of this index
+    cudaEvent_t pass_done = nullptr;        // end of the last interval pass queued
 };
 
 struct pvs_snapshot {
@@ -53,6 +58,7 @@ struct pvs_snapshot {
 
 struct pvs_cursor {
     pvs_index* index = nullptr;
+    cudaStream_t stream = nullptr;    // where this cursor's device work runs
     std::shared_ptr<pvs::SnapData> snap;
     int64_t rows = 0, visible = 0, emitted = 0;
     int state = PVS_OK;
@@ -61,7 +67,8 @@ struct pvs_cursor {
     int8_t* zq = nullptr;
     float* qraw = nullptr;
     pvs::QueryScalars* qs = nullptr;
-    // bounds of every row of the snapshot
+    // bounds of every row of the snapshot (buffers hold cap_rows rows)
+    int64_t cap_rows = 0;
     float* lo = nullptr;
     float* hi = nullptr;
     // working set (ordered by id): rows that can hold the next `horizon` ranks

@@ -355,6 +355,60 @@ def test_eahr_topk_matches_complete_list_fusion(tau):
         pvs.pvs_index_free(index)
 
 
+def test_cursors_on_separate_streams_and_threads_match_oracle():
+    """Interleaved pulls of cursors on their own streams (their interval
+    passes serialised per index, pulls overlapping) and cursors driven from
+    two host threads both give the oracle's rankings."""
+    import threading
+    centres = synth.mixture_centres(32, 128, seed=50, device="cpu")
+    V = synth.mixture_rows(20_000, centres, 0.35, seed=51).numpy()
+    qs = synth.mixture_queries(6, centres, 0.5, seed=52).numpy()
+    refs = [po.dense_ranking(q, V) for q in qs]
+    index = pvs.pvs_build(V)
+    try:
+        streams = [torch.cuda.Stream() for _ in range(4)]
+        ids_t = torch.zeros((4, 250), dtype=torch.int64, device="cuda")
+        sc_t = torch.zeros((4, 250), dtype=torch.float32, device="cuda")
+        curs = []
+        for k in range(4):
+            c = pvs.pvs_cursor_open(index, qs[k])
+            pvs.pvs_cursor_set_stream(c, streams[k])
+            curs.append(c)
+        for p in range(10):
+            for k, c in enumerate(curs):
+                pvs.pvs_next_device(c, 25, ids_t[k, 25 * p:], sc_t[k, 25 * p:])
+        for c in curs:
+            assert pvs.pvs_cursor_sync(c) == pvs.PVS_OK
+            pvs.pvs_cursor_close(c)
+        torch.cuda.synchronize()
+        for k in range(4):
+            assert np.array_equal(ids_t[k].cpu().numpy(), refs[k][0][:250])
+            assert np.array_equal(sc_t[k].cpu().numpy(), refs[k][1][:250])
+
+        results, errors = {}, []
+
+        def worker(k):
+            try:
+                c = pvs.pvs_cursor_open(index, qs[k])
+                pvs.pvs_cursor_set_stream(c, streams[k % 2])
+                got = [pvs.pvs_next(c, 40)[0] for _ in range(5)]
+                pvs.pvs_cursor_close(c)
+                results[k] = np.concatenate(got)
+            except Exception as e:
+                errors.append(e)
+
+        threads = [threading.Thread(target=worker, args=(k,)) for k in (4, 5)]
+        for t in threads:
+            t.start()
+        for t in threads:
+            t.join()
+        assert not errors
+        for k in (4, 5):
+            assert np.array_equal(results[k], refs[k][0][:200])
+    finally:
+        pvs.pvs_index_free(index)
+
+
 def test_eahr_rejects_bad_sparse_lists_and_used_cursors():
     V = np.random.default_rng(0).standard_normal((200, 32)).astype(np.float32)
     index = pvs.pvs_build(V)
