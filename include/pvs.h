@@ -73,6 +73,7 @@ typedef struct pvs_stats {
     int32_t reserved;
     double interval_ms;       /* device time of the interval passes, measured
                                  with CUDA events on the cursor's stream       */
+    int64_t batch_passes;     /* batched tensor-core passes that served it     */
 } pvs_stats;
 
 /* ---------------------------------------------------------------------------
@@ -131,13 +132,28 @@ void pvs_snapshot_free(pvs_snapshot* snap);
 pvs_status pvs_cursor_open(pvs_index* index, const pvs_snapshot* snap, const float* query,
                            int32_t query_on_device, pvs_cursor** out);
 
-/* Open nq cursors that share one batched interval pass (queries: nq*dim
- * floats).  `horizon` is the number of ranks each cursor is prepared to
- * deliver without rescanning the codes (>= 1; later ranks still come out
- * exactly, at the cost of a rescan).  out[0..nq-1] receive the cursors. */
+/* Open nq cursors (queries: nq*dim floats) whose intervals come from one
+ * tensor-core pass per group of up to 256 queries (the Int8 dot products of
+ * all queries as one exact bf16 GEMM, Sec. 2.3.1 intervals in its
+ * epilogue).  Each cursor keeps only the rows that can hold its first
+ * ranks: `horizon` (>= 1) is the number of ranks it is prepared for; it can
+ * usually deliver about three times that many before it needs a
+ * single-query interval pass, and later ranks still come out exactly, at the
+ * cost of that pass.  out[0..nq-1] receive the cursors; they run on the
+ * index's stream.  Errors as pvs_cursor_open; on error no cursor is
+ * returned. */
 pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
                                  const float* queries, int32_t nq, int32_t queries_on_device,
                                  int32_t horizon, pvs_cursor** out);
+
+/* The next n ranks of each of nc cursors in one set of launches (all
+ * cursors of one index and one stream).  Row i of ids / scores (nc x n,
+ * int64 / float32, device or host per outputs_on_device) receives cursor i's
+ * ranks and n_out[i] (host) their count.  Semantics per cursor as pvs_next
+ * (host outputs: blocking, statuses checked) or pvs_next_device (device
+ * outputs: queued).  Returns PVS_OK or the first error. */
+pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
+                          int64_t* ids, float* scores, int32_t* n_out);
 
 /* Deliver the next n exact ranks (Sec. 2.1: a stable exact prefix that is
  * only ever extended).  ids (int64) and scores (the authoritative float32
@@ -186,6 +202,13 @@ pvs_status pvs_cursor_score_ids(pvs_cursor* cursor, const int64_t* ids, int32_t 
                                 float* scores);
 
 const char* pvs_status_string(int32_t status);
+
+/* Diagnostics.  Score intervals of every row of `snap` (NULL: the current
+ * visible set) for 1 <= nq <= 256 queries, computed by the tensor-core
+ * batched pass; host outputs lo / hi of nq x rows floats (row-major by
+ * query; -inf for deleted rows). */
+pvs_status pvs_batch_bounds(pvs_index* index, const pvs_snapshot* snap, const float* queries,
+                            int32_t nq, int32_t queries_on_device, float* lo, float* hi);
 
 /* Number of CUDA kernels this library has launched in this process. */
 int64_t pvs_launch_count(void);

@@ -47,7 +47,7 @@ class pvs_stats(ctypes.Structure):
         "visible", "emitted", "refined", "exact_fallbacks", "interval_passes",
         "horizon_builds", "pulls", "candidates", "code_bytes")] + [
         ("state", ctypes.c_int32), ("reserved", ctypes.c_int32),
-        ("interval_ms", ctypes.c_double)]
+        ("interval_ms", ctypes.c_double), ("batch_passes", ctypes.c_int64)]
 
 
 class eahr_params(ctypes.Structure):
@@ -88,6 +88,8 @@ def _load() -> ctypes.CDLL:
         "pvs_next_device": (i32, [P, i32, P, P, P]),
         "pvs_cursor_sync": (i32, [P]),
         "pvs_cursor_set_stream": (i32, [P, P]),
+        "pvs_next_batch": (i32, [P, i32, i32, i32, P, P, P]),
+        "pvs_batch_bounds": (i32, [P, P, P, i32, i32, P, P]),
         "pvs_cursor_stats": (i32, [P, ctypes.POINTER(pvs_stats)]),
         "pvs_cursor_bounds": (i32, [P, i64, i64, P, P]),
         "pvs_cursor_score_ids": (i32, [P, P, i32, P]),
@@ -113,7 +115,7 @@ EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_i
             "pvs_index_dim", "pvs_index_export", "pvs_index_free", "pvs_snapshot_create",
             "pvs_snapshot_visible", "pvs_snapshot_free", "pvs_cursor_open",
             "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
-            "pvs_cursor_set_stream",
+            "pvs_cursor_set_stream", "pvs_next_batch", "pvs_batch_bounds",
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
             "eahr_topk_lists")
@@ -248,6 +250,41 @@ def pvs_next_device(cursor, n: int, ids, scores):
                                      ctypes.c_void_p(scores.data_ptr()), ctypes.byref(got)),
                 "pvs_next_device")
     return got.value, st
+
+
+def pvs_next_batch(cursors, n: int, ids=None, scores=None):
+    """Next n ranks of every cursor.  Without ids/scores: host outputs, returns
+    (ids int64[nc, n], scores float32[nc, n], n_out int32[nc]); with CUDA
+    tensors ids / scores of shape [nc, >= n] (row stride n): queued, returns
+    n_out."""
+    nc = len(cursors)
+    arr = (ctypes.c_void_p * max(nc, 1))(*[c.value if isinstance(c, ctypes.c_void_p) else c
+                                            for c in cursors])
+    n_out = np.zeros(max(nc, 1), np.int32)
+    if ids is None:
+        h_ids = np.zeros((max(nc, 1), max(n, 1)), np.int64)
+        h_sc = np.zeros((max(nc, 1), max(n, 1)), np.float32)
+        _check(_lib.pvs_next_batch(arr, nc, int(n), 0, h_ids.ctypes.data, h_sc.ctypes.data,
+                                   n_out.ctypes.data), "pvs_next_batch")
+        return h_ids[:nc, :n], h_sc[:nc, :n], n_out[:nc]
+    _check(_lib.pvs_next_batch(arr, nc, int(n), 1, ctypes.c_void_p(ids.data_ptr()),
+                               ctypes.c_void_p(scores.data_ptr()), n_out.ctypes.data),
+           "pvs_next_batch")
+    return n_out[:nc]
+
+
+def pvs_batch_bounds(index, queries, snap=None, rows=None):
+    """Tensor-core intervals of every row for nq <= 256 queries ->
+    (lo, hi) float32[nq, rows]; `rows` is the snapshot's row count (default:
+    the index's current size, right for snap=None)."""
+    ptr, shape, on_dev, keep = _vec_arg(queries)
+    nq = shape[0]
+    rows = int(_lib.pvs_index_size(index)) if rows is None else int(rows)
+    lo = np.zeros((nq, max(rows, 1)), np.float32)
+    hi = np.zeros((nq, max(rows, 1)), np.float32)
+    _check(_lib.pvs_batch_bounds(index, snap, ptr, nq, on_dev, lo.ctypes.data, hi.ctypes.data),
+           "pvs_batch_bounds")
+    return lo[:, :rows], hi[:, :rows]
 
 
 def pvs_cursor_sync(cursor) -> int:

@@ -60,6 +60,40 @@ struct PullArgs {
     DevCounters* ctr;
 };
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
+// Many cursors at once (args_dev: device array of ncursors PullArgs).
+cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
+                              cudaStream_t st);
+cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
+                                cudaStream_t st);
+
+// ---- batched open support (pull_kernel.cu, batch_support.cu) ----------------
+constexpr int kWsSortMax = 8192;     // largest per-query working set of a batched open
+struct WsDst {                       // a cursor's working-set arrays
+    int32_t* w_id;
+    float* w_lo;
+    float* w_hi;
+    unsigned int* w_len;
+};
+struct QueryDst {                    // a cursor's query buffers
+    int8_t* zq;
+    float* qraw;
+    QueryScalars* qs;
+};
+cudaError_t launch_batch_tau(const float* dump_lo, int64_t ld, unsigned int nsample, int nq,
+                             unsigned int k, float* tau, cudaStream_t st);
+cudaError_t launch_ws_sort(const int32_t* w_id_b, const float* w_lo_b, const float* w_hi_b,
+                           int cap, const unsigned int* w_len_b, const WsDst* dst, int nq,
+                           cudaStream_t st);
+cudaError_t launch_norm_max(const float* vnorm, const float* enorm, int64_t rows,
+                            unsigned int* out, cudaStream_t st);
+cudaError_t launch_rmax(const QueryScalars* qs, int nq, const unsigned int* maxes, float* rmax,
+                        cudaStream_t st);
+cudaError_t launch_copy_queries(const int8_t* zq_b, const float* qraw_b, const QueryScalars* qs_b,
+                                const QueryDst* dst, int nq, int m_pad, int m_raw,
+                                cudaStream_t st);
+cudaError_t launch_scatter_ws(const int32_t* w_id, const float* w_lo, const float* w_hi,
+                              const unsigned int* w_len, float* lo, float* hi, int grid,
+                              cudaStream_t st);
 
 // ---- build / encode (build_kernels.cu) -------------------------------------
 // Quantize rows [0, n) of `vecs` (row stride m floats) into codes (stride
@@ -129,6 +163,36 @@ cudaError_t launch_radix_sort_desc(uint64_t* keys, uint64_t* tmp, int64_t count,
 cudaError_t launch_emit(const uint64_t* keys, int n, const int32_t* w_id, float* w_lo,
                         float* w_hi, float* lo, float* hi, int64_t* out_ids, float* out_scores,
                         cudaStream_t st);
+
+// ---- batched interval pass on the tensor cores (batch_gemm.cu) --------------
+struct BatchArgs {
+    int64_t rows;                 // corpus rows [0, rows) are scanned
+    int m_pad;                    // K (multiple of 64)
+    int nq, nq_pad;               // queries; nq_pad multiple of 32, <= 256
+    const float* scale;
+    const float* vnorm;
+    const float* enorm;
+    const uint32_t* tomb;         // tombstones of the snapshot, or null
+    const QueryScalars* qs;       // [nq]
+    int mode;                     // 0: dump, 1: filter
+    int tile_stride;              // process 128-row tiles 0, s, 2s, ...
+    float* dump_lo;               // dump: [nq][dump_ld], row (i*128 + r) of tile i*s
+    float* dump_hi;
+    int64_t dump_ld;
+    const float* tau;             // filter: [nq] thresholds
+    const float* rmax;            // filter: [nq] upper bound of the interval half-width
+    int32_t* w_id;                // filter: [nq][w_cap] working sets (unordered)
+    float* w_lo;
+    float* w_hi;
+    int w_cap;
+    unsigned int* w_len;          // [nq] (may exceed w_cap: overflow)
+    unsigned int* h_eff;          // [nq] rows with lo >= tau
+    int* status;
+};
+cudaError_t launch_batch_intervals(const BatchArgs& a, const uint16_t* codes_bf16,
+                                   const uint16_t* qcodes_bf16, int num_sms, cudaStream_t st);
+cudaError_t launch_codes_to_bf16(const int8_t* src, uint16_t* dst, int64_t count,
+                                 cudaStream_t st);
 
 // ---- refinement (refine_kernels.cu) -----------------------------------------
 // Authoritative score of every unresolved candidate (w_lo < w_hi): exact

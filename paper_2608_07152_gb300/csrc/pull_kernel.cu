@@ -137,8 +137,7 @@ __device__ inline void bitonic_desc_smem(unsigned long long* sk, int pow2) {
 
 // Steps 1-2 (one CTA): tau and the candidate list; the count goes to
 // ctr->cand for the refinement and emission launches.
-__global__ void __launch_bounds__(kPullThreads, 2) pull_select_kernel(PullArgs a) {
-    __shared__ PullShared sh;
+__device__ inline void pull_select_body(const PullArgs& a, PullShared& sh) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const unsigned int len = *a.w_len;
     const int n = a.n;
@@ -180,10 +179,20 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_select_kernel(PullArgs a
     }
 }
 
+__global__ void __launch_bounds__(kPullThreads, 2) pull_select_kernel(PullArgs a) {
+    __shared__ PullShared sh;
+    pull_select_body(a, sh);
+}
+
+// One CTA per cursor.
+__global__ void __launch_bounds__(kPullThreads, 2) pull_select_batch_kernel(const PullArgs* args) {
+    __shared__ PullShared sh;
+    pull_select_body(args[blockIdx.x], sh);
+}
+
 // Steps 4-5 (one CTA): order the candidates (all scored by now) and emit the
 // first n.
-__global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) {
-    __shared__ PullShared sh;
+__device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const unsigned int c = a.ctr->cand;
     const int n = a.n;
@@ -244,9 +253,21 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) 
         a.out_scores[r] = rank_key_score(k);
         a.w_lo[w] = -INFINITY;
         a.w_hi[w] = -INFINITY;
-        a.lo[id] = -INFINITY;
-        a.hi[id] = -INFINITY;
+        if (a.lo) {
+            a.lo[id] = -INFINITY;
+            a.hi[id] = -INFINITY;
+        }
     }
+}
+
+__global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) {
+    __shared__ PullShared sh;
+    pull_emit_body(a, sh);
+}
+
+__global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const PullArgs* args) {
+    __shared__ PullShared sh;
+    pull_emit_body(args[blockIdx.x], sh);
 }
 
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st) {
@@ -262,6 +283,114 @@ cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t s
     if (e != cudaSuccess) return e;
     count_launches(1);
     pull_emit_kernel<<<1, kPullThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+// ---- batched open: per-query thresholds and ordered working sets --------------
+
+struct RowKeys {   // live lower bounds of one query's dump row
+    const float* lo;
+    __device__ bool valid(unsigned int i) const { return lo[i] != -INFINITY; }
+    __device__ uint32_t key(unsigned int i) const { return fkey(lo[i]); }
+};
+
+// One CTA per query: tau[q] = k-th largest live lower bound among the sampled
+// rows (dump row q), or -inf if fewer than k are live.
+__global__ void __launch_bounds__(kPullThreads, 2) batch_tau_kernel(const float* dump_lo,
+                                                                    int64_t ld,
+                                                                    unsigned int nsample,
+                                                                    unsigned int k, float* tau) {
+    __shared__ PullShared sh;
+    const int q = blockIdx.x, t = threadIdx.x;
+    const RowKeys src{dump_lo + (int64_t)q * ld};
+    if (t == 0) {
+        sh.prefix = 0;
+        sh.k = k;
+    }
+    __syncthreads();
+    const int shifts32[3] = {21, 10, 0}, bits32[3] = {11, 11, 10};
+    for (int p = 0; p < 3; ++p) {
+        block_histogram<uint32_t>(sh, nsample, shifts32[p], bits32[p], (uint32_t)sh.prefix, src);
+        if (t == 0) sh.ok = 0;
+        __syncthreads();
+        block_pick_digit(sh, shifts32[p]);
+        if (!sh.ok) {
+            if (t == 0) tau[q] = -INFINITY;
+            return;
+        }
+    }
+    if (t == 0) tau[q] = fkey_inv((uint32_t)sh.prefix);
+}
+
+cudaError_t launch_batch_tau(const float* dump_lo, int64_t ld, unsigned int nsample, int nq,
+                             unsigned int k, float* tau, cudaStream_t st) {
+    if (nq <= 0) return cudaSuccess;
+    count_launches(1);
+    batch_tau_kernel<<<nq, kPullThreads, 0, st>>>(dump_lo, ld, nsample, k, tau);
+    return cudaGetLastError();
+}
+
+// One CTA per query: the unordered working set written by the filter pass
+// (ids, bounds at [q * cap, ...)) is sorted by id into the cursor's own
+// arrays, so that working-set index order is id order.
+__global__ void __launch_bounds__(kPullThreads) ws_sort_kernel(const int32_t* w_id_b,
+                                                               const float* w_lo_b,
+                                                               const float* w_hi_b, int cap,
+                                                               const unsigned int* w_len_b,
+                                                               const WsDst* dst) {
+    extern __shared__ unsigned long long keys[];
+    const int q = blockIdx.x, t = threadIdx.x;
+    const unsigned int len = w_len_b[q];
+    const WsDst d = dst[q];
+    if (len > (unsigned int)cap) {          // overflow: the cursor rescans instead
+        if (t == 0) *d.w_len = 0;
+        return;
+    }
+    int pow2 = 1;
+    while (pow2 < (int)len) pow2 <<= 1;
+    const int64_t base = (int64_t)q * cap;
+    for (int i = t; i < pow2; i += kPullThreads)
+        keys[i] = i < (int)len ? ((unsigned long long)(0xffffffffu - (uint32_t)w_id_b[base + i]) << 32) |
+                                     (unsigned int)i
+                               : 0ull;
+    __syncthreads();
+    bitonic_desc_smem(keys, pow2);
+    for (int r = t; r < (int)len; r += kPullThreads) {
+        const unsigned int pos = (unsigned int)(keys[r] & 0xffffffffull);
+        d.w_id[r] = w_id_b[base + pos];
+        d.w_lo[r] = w_lo_b[base + pos];
+        d.w_hi[r] = w_hi_b[base + pos];
+    }
+    if (t == 0) *d.w_len = len;
+}
+
+cudaError_t launch_ws_sort(const int32_t* w_id_b, const float* w_lo_b, const float* w_hi_b,
+                           int cap, const unsigned int* w_len_b, const WsDst* dst, int nq,
+                           cudaStream_t st) {
+    if (nq <= 0) return cudaSuccess;
+    if (cap > kWsSortMax) return cudaErrorInvalidValue;
+    int pow2 = 1;
+    while (pow2 < cap) pow2 <<= 1;
+    const size_t smem = (size_t)pow2 * sizeof(unsigned long long);
+    cudaError_t e = cudaFuncSetAttribute(ws_sort_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    count_launches(1);
+    ws_sort_kernel<<<nq, kPullThreads, smem, st>>>(w_id_b, w_lo_b, w_hi_b, cap, w_len_b, dst);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
+                              cudaStream_t st) {
+    if (ncursors <= 0) return cudaSuccess;
+    count_launches(1);
+    pull_select_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    e = launch_refine_batch(args_dev, ncursors, refine_blocks_per_cursor, st);
+    if (e != cudaSuccess) return e;
+    count_launches(1);
+    pull_emit_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);
     return cudaGetLastError();
 }
 

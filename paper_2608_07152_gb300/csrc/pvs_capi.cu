@@ -123,6 +123,8 @@ pvs_status index_reserve(pvs_index* x, int64_t need) {
     }
     dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
     dev_free(x->raw);
+    dev_free(x->codes_bf16);   // rebuilt on demand at the new capacity
+    x->bf16_rows = 0;
     x->codes = codes, x->scale = scale, x->vnorm = vnorm, x->enorm = enorm, x->raw = raw;
     x->cap = cap;
     x->h_tomb.resize((size_t)(cap / 32), 0u);
@@ -207,8 +209,10 @@ void cursor_reset(pvs_cursor* c) {
     c->rows = c->visible = c->emitted = 0;
     c->state = PVS_OK;
     c->scanned = false;
+    c->batch_ws = false;
     c->horizon = c->horizon_base = 0;
     c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
+    c->batch_passes = 0;
     c->ev_pending = false;
     c->interval_ms = 0.0;
 }
@@ -217,28 +221,45 @@ constexpr size_t kCursorPool = 4;   // closed cursors kept per index
 
 // Allocate the per-row state of a cursor (first pull); a pooled cursor keeps
 // buffers that are large enough.
-pvs_status cursor_alloc_rows(pvs_cursor* c) {
+// Bounds of every row of the snapshot (single-query interval pass).
+pvs_status cursor_alloc_full(pvs_cursor* c) {
     if (c->lo && c->cap_rows >= c->rows) return PVS_OK;
-    dev_free(c->lo), dev_free(c->hi);
+    dev_free(c->lo), dev_free(c->hi), dev_free(c->compact_scratch);
+    c->cap_rows = 0;
+    const size_t n = (size_t)std::max<int64_t>(c->rows, 1);
+    PVS_CUDA(dev_alloc(&c->lo, n));
+    PVS_CUDA(dev_alloc(&c->hi, n));
+    PVS_CUDA(dev_alloc(&c->compact_scratch, compact_scratch_elems((int64_t)n)));
+    c->cap_rows = (int64_t)n;
+    return PVS_OK;
+}
+
+// Working-set arrays and pull scratch for up to `cap` entries (contents are
+// not preserved when they grow).
+pvs_status cursor_alloc_ws(pvs_cursor* c, int64_t cap) {
+    cap = std::max<int64_t>(cap, 1);
+    if (c->w_id && c->cap_w >= cap) return PVS_OK;
     dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
-    dev_free(c->compact_scratch);
     dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp);
     if (c->sort_scratch) cudaFree(c->sort_scratch);
     c->sort_scratch = nullptr;
-    c->cap_rows = 0;
-    const size_t n = (size_t)std::max<int64_t>(c->rows, 1);
-    c->cap_rows = (int64_t)n;
-    PVS_CUDA(dev_alloc(&c->lo, n));
-    PVS_CUDA(dev_alloc(&c->hi, n));
+    c->cap_w = 0;
+    const size_t n = (size_t)cap;
     PVS_CUDA(dev_alloc(&c->w_id, n));
     PVS_CUDA(dev_alloc(&c->w_lo, n));
     PVS_CUDA(dev_alloc(&c->w_hi, n));
-    PVS_CUDA(dev_alloc(&c->compact_scratch, compact_scratch_elems((int64_t)n)));
     PVS_CUDA(dev_alloc(&c->cand, n));
     PVS_CUDA(dev_alloc(&c->keys, n));
     PVS_CUDA(dev_alloc(&c->keys_tmp, n));
     PVS_CUDA(cudaMalloc(&c->sort_scratch, radix_sort_scratch_bytes((int64_t)n)));
+    c->cap_w = cap;
     return PVS_OK;
+}
+
+pvs_status cursor_alloc_rows(pvs_cursor* c) {
+    pvs_status s = cursor_alloc_full(c);
+    if (s != PVS_OK) return s;
+    return cursor_alloc_ws(c, c->rows);
 }
 
 pvs_status cursor_out_reserve(pvs_cursor* c, int64_t n) {
@@ -344,19 +365,50 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
 }
 
 // One pull of n_eff >= 1 ranks into device buffers d_ids / d_scores.
+// Full bounds for a cursor whose working set came from a batched pass: a
+// single-query interval pass, then the working set's resolved scores and
+// delivered items are carried over before the working set is rebuilt.
+pvs_status rescan_from_batch(pvs_cursor* c) {
+    pvs_status s = cursor_alloc_full(c);
+    if (s != PVS_OK) return s;
+    s = interval_pass(c);
+    if (s != PVS_OK) return s;
+    PVS_CUDA(launch_scatter_ws(c->w_id, c->w_lo, c->w_hi, &c->ctr->w_len, c->lo, c->hi,
+                               grid_for(c, c->cap_w), c->stream));
+    // the working set is rebuilt from the full bounds; its arrays may grow
+    PVS_CUDA(cudaStreamSynchronize(c->stream));
+    s = cursor_alloc_ws(c, c->rows);
+    if (s != PVS_OK) return s;
+    c->batch_ws = false;
+    c->horizon = 0;   // the next pull rebuilds the working set from the full bounds
+    return PVS_OK;
+}
+
+// Make the cursor's working set hold the next n_eff ranks.
+pvs_status prepare_pull(pvs_cursor* c, int64_t n_eff) {
+    pvs_status s;
+    if (!c->scanned && !c->batch_ws) {
+        s = cursor_alloc_rows(c);
+        if (s != PVS_OK) return s;
+        s = interval_pass(c);
+        if (s != PVS_OK) return s;
+    }
+    if (c->emitted + n_eff - c->horizon_base > c->horizon) {
+        if (c->batch_ws) {
+            s = rescan_from_batch(c);
+            if (s != PVS_OK) return s;
+        }
+        s = build_working_set(c, n_eff);
+        if (s != PVS_OK) return s;
+    }
+    return PVS_OK;
+}
+
 pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
     pvs_index* x = c->index;
     cudaStream_t st = c->stream;
-    pvs_status s = cursor_alloc_rows(c);
+    pvs_status s = prepare_pull(c, n_eff);
     if (s != PVS_OK) return fail(c, s);
-    if (!c->scanned) {
-        s = interval_pass(c);
-        if (s != PVS_OK) return fail(c, s);
-    }
-    if (c->emitted + n_eff - c->horizon_base > c->horizon) {
-        s = build_working_set(c, n_eff);
-        if (s != PVS_OK) return fail(c, s);
-    }
     if (n_eff <= kPullFusedMax) {
         // one launch, no host round trip; failures surface at the next sync
         PullArgs a;
@@ -413,6 +465,257 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
     if (e != cudaSuccess) return fail(c, cuda_status(e));
     c->emitted += n_eff;
     c->pulls++;
+    return PVS_OK;
+}
+
+// ---------------------------------------------------------------------------
+// batched open: one tensor-core interval pass for up to kBatchMax queries
+// ---------------------------------------------------------------------------
+constexpr int kBatchMax = 256;
+
+// Stream-ordered scratch that is released (stream-ordered) at scope exit.
+struct DevBuf {
+    cudaStream_t st = nullptr;
+    std::vector<void*> ptrs;
+    explicit DevBuf(cudaStream_t s = nullptr) : st(s) {}
+    template <typename T>
+    T* get(size_t count) {
+        void* p = nullptr;
+        if (cudaMallocAsync(&p, std::max<size_t>(count, 1) * sizeof(T), st) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        ptrs.push_back(p);
+        return static_cast<T*>(p);
+    }
+    ~DevBuf() {
+        for (void* p : ptrs) cudaFreeAsync(p, st);
+    }
+};
+
+struct BatchQueries {
+    int nq = 0, nq_pad = 0;
+    int8_t* zq = nullptr;          // [nq][m_pad]
+    float* qraw = nullptr;         // [nq][m_raw]
+    QueryScalars* qs = nullptr;    // [nq]
+    uint16_t* qcodes = nullptr;    // [nq_pad][m_pad] bf16, zero rows past nq
+};
+
+// bf16 copy of every code row (the tensor-core pass reads it).
+pvs_status ensure_bf16(pvs_index* x) {
+    if (!x->codes_bf16) {
+        PVS_CUDA(dev_alloc(&x->codes_bf16, (size_t)std::max<int64_t>(x->cap, 1) * x->m_pad));
+        x->bf16_rows = 0;
+    }
+    if (x->bf16_rows < x->size) {
+        const int64_t r0 = x->bf16_rows;
+        PVS_CUDA(launch_codes_to_bf16(x->codes + r0 * x->m_pad, x->codes_bf16 + r0 * x->m_pad,
+                                      (x->size - r0) * x->m_pad, x->stream));
+        x->bf16_rows = x->size;
+    }
+    return PVS_OK;
+}
+
+// Encode nq queries on the index stream; checks their status (waits).
+pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_device, DevBuf& buf,
+                        BatchQueries* bq) {
+    cudaStream_t st = x->stream;
+    bq->nq = nq;
+    bq->nq_pad = (int)round_up(nq, 32);
+    bq->zq = buf.get<int8_t>((size_t)nq * x->m_pad);
+    bq->qraw = buf.get<float>((size_t)nq * x->m_raw);
+    bq->qs = buf.get<QueryScalars>((size_t)nq);
+    bq->qcodes = buf.get<uint16_t>((size_t)bq->nq_pad * x->m_pad);
+    const float* qd = queries;
+    if (!on_device) {
+        float* tmp = buf.get<float>((size_t)nq * x->m);
+        if (!tmp) return PVS_ERR_OOM;
+        PVS_CUDA(cudaMemcpyAsync(tmp, queries, (size_t)nq * x->m * sizeof(float),
+                                 cudaMemcpyHostToDevice, st));
+        qd = tmp;
+    }
+    if (!bq->zq || !bq->qraw || !bq->qs || !bq->qcodes) return PVS_ERR_OOM;
+    PVS_CUDA(launch_encode_queries(qd, nq, x->m, x->m_pad, x->m_raw, bq->zq, bq->qraw, bq->qs, st));
+    PVS_CUDA(cudaMemsetAsync(bq->qcodes, 0, (size_t)bq->nq_pad * x->m_pad * sizeof(uint16_t), st));
+    PVS_CUDA(launch_codes_to_bf16(bq->zq, bq->qcodes, (int64_t)nq * x->m_pad, st));
+    {
+        std::lock_guard<std::mutex> lock(x->pass_mutex);
+        pvs_status s = ensure_bf16(x);
+        if (s != PVS_OK) return s;
+    }
+    std::vector<QueryScalars> h(nq);
+    PVS_CUDA(cudaMemcpyAsync(h.data(), bq->qs, nq * sizeof(QueryScalars), cudaMemcpyDeviceToHost,
+                             st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    for (int i = 0; i < nq; ++i)
+        if (h[i].status != 0) return (pvs_status)h[i].status;
+    return PVS_OK;
+}
+
+// A cursor with its small buffers, fresh counters and the given snapshot.
+pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs_cursor** out) {
+    pvs_cursor* c = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(x->pool_mutex);
+        if (!x->cursor_pool.empty()) {
+            c = x->cursor_pool.back();
+            x->cursor_pool.pop_back();
+        }
+    }
+    if (!c) {
+        c = new (std::nothrow) pvs_cursor();
+        if (!c) return PVS_ERR_OOM;
+    }
+    cursor_reset(c);
+    c->index = x;
+    c->stream = x->stream;
+    c->snap = sd;
+    c->rows = sd->rows;
+    c->visible = sd->visible;
+    *out = c;
+    if (!c->zq &&
+        (dev_alloc(&c->zq, (size_t)x->m_pad) != cudaSuccess ||
+         dev_alloc(&c->qraw, (size_t)x->m_raw) != cudaSuccess ||
+         dev_alloc(&c->qs, 1) != cudaSuccess || dev_alloc(&c->sel, 1) != cudaSuccess ||
+         dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
+         cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess))
+        return PVS_ERR_OOM;
+    PVS_CUDA(cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), c->stream));
+    PVS_CUDA(cudaMemsetAsync(c->d_status, 0, sizeof(int), c->stream));
+    c->state = c->visible == 0 ? PVS_EXHAUSTED : PVS_OK;
+    return PVS_OK;
+}
+
+// Up to kBatchMax cursors from one batched pass:
+//   1. encode the queries; bf16 query codes for the MMA;
+//   2. thresholds: on every 16th 128-row tile (every tile for small corpora)
+//      the pass dumps all intervals; tau_q = the k-th largest lower bound of
+//      query q there, k sized so that about 3x the horizon rows of the whole
+//      corpus reach it;
+//   3. the filter pass appends every row with hi >= tau_q to query q's
+//      working set and counts the rows with lo >= tau_q: those rows precede
+//      every row outside the working set, so the cursor can deliver that many
+//      ranks before it needs a single-query pass;
+//   4. each working set is sorted by id into its cursor.
+// A query whose working set overflows, or whose count is 0, falls back to a
+// single-query interval pass at its first pull.
+pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
+                            const float* queries, int nq, bool on_device, int horizon,
+                            pvs_cursor** out) {
+    cudaStream_t st = x->stream;
+    DevBuf buf(st);
+    BatchQueries bq;
+    pvs_status s = encode_batch(x, queries, nq, on_device, buf, &bq);
+    if (s != PVS_OK) return s;
+    for (int i = 0; i < nq; ++i) {
+        s = acquire_cursor(x, sd, &out[i]);
+        if (s != PVS_OK) return s;
+    }
+    QueryDst* d_qd = buf.get<QueryDst>((size_t)nq);
+    if (!d_qd) return PVS_ERR_OOM;
+    {
+        std::vector<QueryDst> qd(nq);
+        for (int i = 0; i < nq; ++i) qd[i] = QueryDst{out[i]->zq, out[i]->qraw, out[i]->qs};
+        PVS_CUDA(cudaMemcpyAsync(d_qd, qd.data(), nq * sizeof(QueryDst), cudaMemcpyHostToDevice, st));
+        PVS_CUDA(launch_copy_queries(bq.zq, bq.qraw, bq.qs, d_qd, nq, x->m_pad, x->m_raw, st));
+        PVS_CUDA(cudaStreamSynchronize(st));   // qd (host) is read by the copy above
+    }
+    const int64_t rows = sd->rows;
+    if (rows == 0) return PVS_OK;
+
+    const int64_t ntiles = (rows + 127) / 128;
+    const int stride = ntiles >= 64 ? 16 : 1;
+    const int64_t ld = ((ntiles + stride - 1) / stride) * 128;
+    const unsigned int k_s =
+        stride == 1 ? (unsigned int)horizon : (unsigned int)((3 * (int64_t)horizon + 15) / 16 + 8);
+    const int w_cap = (int)std::min<int64_t>({(int64_t)kWsSortMax, 16 * (int64_t)horizon + 1024,
+                                              std::max<int64_t>(rows, 1)});
+    float* dlo = buf.get<float>((size_t)nq * ld);
+    float* dhi = buf.get<float>((size_t)nq * ld);
+    float* tau = buf.get<float>((size_t)nq);
+    float* rmax = buf.get<float>((size_t)nq);
+    unsigned int* maxes = buf.get<unsigned int>(2);
+    int* status = buf.get<int>(1);
+    int32_t* wid = buf.get<int32_t>((size_t)nq * w_cap);
+    float* wlo = buf.get<float>((size_t)nq * w_cap);
+    float* whi = buf.get<float>((size_t)nq * w_cap);
+    unsigned int* wlen = buf.get<unsigned int>((size_t)nq);
+    unsigned int* heff = buf.get<unsigned int>((size_t)nq);
+    WsDst* d_ws = buf.get<WsDst>((size_t)nq);
+    if (!dlo || !dhi || !tau || !rmax || !maxes || !status || !wid || !wlo || !whi || !wlen ||
+        !heff || !d_ws)
+        return PVS_ERR_OOM;
+    PVS_CUDA(cudaMemsetAsync(status, 0, sizeof(int), st));
+    PVS_CUDA(cudaMemsetAsync(wlen, 0, nq * sizeof(unsigned int), st));
+    PVS_CUDA(cudaMemsetAsync(heff, 0, nq * sizeof(unsigned int), st));
+
+    BatchArgs a{};
+    a.rows = rows;
+    a.m_pad = x->m_pad;
+    a.nq = nq;
+    a.nq_pad = bq.nq_pad;
+    a.scale = x->scale;
+    a.vnorm = x->vnorm;
+    a.enorm = x->enorm;
+    a.tomb = sd->d_tomb;
+    a.qs = bq.qs;
+    a.status = status;
+    // 2. thresholds from the sampled tiles
+    a.mode = 0;
+    a.tile_stride = stride;
+    a.dump_lo = dlo;
+    a.dump_hi = dhi;
+    a.dump_ld = ld;
+    PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
+    PVS_CUDA(launch_batch_tau(dlo, ld, (unsigned int)ld, nq, k_s, tau, st));
+    PVS_CUDA(launch_norm_max(x->vnorm, x->enorm, rows, maxes, st));
+    PVS_CUDA(launch_rmax(bq.qs, nq, maxes, rmax, st));
+    // 3. the filter pass over every row
+    a.mode = 1;
+    a.tile_stride = 1;
+    a.dump_lo = a.dump_hi = nullptr;
+    a.dump_ld = 0;
+    a.tau = tau;
+    a.rmax = rmax;
+    a.w_id = wid;
+    a.w_lo = wlo;
+    a.w_hi = whi;
+    a.w_cap = w_cap;
+    a.w_len = wlen;
+    a.h_eff = heff;
+    {
+        std::lock_guard<std::mutex> lock(x->pass_mutex);   // one HBM pass at a time
+        if (x->pass_done) PVS_CUDA(cudaStreamWaitEvent(st, x->pass_done, 0));
+        PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
+        if (!x->pass_done)
+            PVS_CUDA(cudaEventCreateWithFlags(&x->pass_done, cudaEventDisableTiming));
+        PVS_CUDA(cudaEventRecord(x->pass_done, st));
+    }
+    // 4. ordered working sets into the cursors
+    std::vector<WsDst> ws(nq);
+    for (int i = 0; i < nq; ++i) {
+        s = cursor_alloc_ws(out[i], w_cap);
+        if (s != PVS_OK) return s;
+        ws[i] = WsDst{out[i]->w_id, out[i]->w_lo, out[i]->w_hi, &out[i]->ctr->w_len};
+    }
+    PVS_CUDA(cudaMemcpyAsync(d_ws, ws.data(), nq * sizeof(WsDst), cudaMemcpyHostToDevice, st));
+    PVS_CUDA(launch_ws_sort(wid, wlo, whi, w_cap, wlen, d_ws, nq, st));
+    std::vector<unsigned int> h_wlen(nq), h_heff(nq);
+    int h_status = 0;
+    PVS_CUDA(cudaMemcpyAsync(h_wlen.data(), wlen, nq * sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpyAsync(h_heff.data(), heff, nq * sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpyAsync(&h_status, status, sizeof(int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    if (h_status != 0) return (pvs_status)h_status;
+    for (int i = 0; i < nq; ++i) {
+        pvs_cursor* c = out[i];
+        if (h_wlen[i] <= (unsigned int)w_cap && h_heff[i] > 0) {
+            c->batch_ws = true;
+            c->horizon = h_heff[i];
+            c->horizon_base = 0;
+        }
+        c->batch_passes = 1;
+    }
     return PVS_OK;
 }
 
@@ -546,7 +849,7 @@ void pvs_index_free(pvs_index* x) {
     }
     x->cursor_pool.clear();
     dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
-    dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage);
+    dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage), dev_free(x->codes_bf16);
     if (x->pass_done) cudaEventDestroy(x->pass_done);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
@@ -632,17 +935,159 @@ pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const f
                                  int32_t nq, int32_t queries_on_device, int32_t horizon,
                                  pvs_cursor** out) {
     if (!x || !queries || !out || nq < 0 || horizon < 1) return PVS_ERR_INVALID;
-    const size_t m = (size_t)x->m;
+    if (queries_on_device && !is_device_ptr(queries)) return PVS_ERR_INVALID;
     for (int32_t i = 0; i < nq; ++i) out[i] = nullptr;
-    for (int32_t i = 0; i < nq; ++i) {
-        pvs_status s = pvs_cursor_open(x, snap, queries + i * m, queries_on_device, &out[i]);
+    std::shared_ptr<SnapData> sd = snap ? snap->data : make_snapdata(x);
+    if (!sd) return PVS_ERR_OOM;
+    for (int32_t g0 = 0; g0 < nq; g0 += kBatchMax) {
+        const int32_t g = std::min<int32_t>(kBatchMax, nq - g0);
+        pvs_status s = open_batch_group(x, sd, queries + (size_t)g0 * x->m, g,
+                                        queries_on_device != 0, horizon, out + g0);
         if (s != PVS_OK) {
-            for (int32_t j = 0; j < i; ++j) {
-                pvs_cursor_close(out[j]);
+            for (int32_t j = 0; j < nq; ++j) {
+                if (out[j]) pvs_cursor_close(out[j]);
                 out[j] = nullptr;
             }
             return s;
         }
+    }
+    return PVS_OK;
+}
+
+pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float* queries,
+                            int32_t nq, int32_t queries_on_device, float* lo, float* hi) {
+    if (!x || !queries || !lo || !hi || nq < 1 || nq > kBatchMax) return PVS_ERR_INVALID;
+    if (queries_on_device && !is_device_ptr(queries)) return PVS_ERR_INVALID;
+    std::shared_ptr<SnapData> sd = snap ? snap->data : make_snapdata(x);
+    if (!sd) return PVS_ERR_OOM;
+    const int64_t rows = sd->rows;
+    if (rows == 0) return PVS_OK;
+    cudaStream_t st = x->stream;
+    DevBuf buf(st);
+    BatchQueries bq;
+    pvs_status s = encode_batch(x, queries, nq, queries_on_device, buf, &bq);
+    if (s != PVS_OK) return s;
+    const int64_t ntiles = (rows + 127) / 128;
+    const int64_t ld = ntiles * 128;
+    float* dlo = buf.get<float>((size_t)nq * ld);
+    float* dhi = buf.get<float>((size_t)nq * ld);
+    int* status = buf.get<int>(1);
+    if (!dlo || !dhi || !status) return PVS_ERR_OOM;
+    PVS_CUDA(cudaMemsetAsync(status, 0, sizeof(int), st));
+    BatchArgs a{};
+    a.rows = rows;
+    a.m_pad = x->m_pad;
+    a.nq = nq;
+    a.nq_pad = bq.nq_pad;
+    a.scale = x->scale;
+    a.vnorm = x->vnorm;
+    a.enorm = x->enorm;
+    a.tomb = sd->d_tomb;
+    a.qs = bq.qs;
+    a.mode = 0;
+    a.tile_stride = 1;
+    a.dump_lo = dlo;
+    a.dump_hi = dhi;
+    a.dump_ld = ld;
+    a.status = status;
+    PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
+    int h_status = 0;
+    PVS_CUDA(cudaMemcpyAsync(&h_status, status, sizeof(int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpy2DAsync(lo, rows * sizeof(float), dlo, ld * sizeof(float),
+                               rows * sizeof(float), nq, cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpy2DAsync(hi, rows * sizeof(float), dhi, ld * sizeof(float),
+                               rows * sizeof(float), nq, cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    return (pvs_status)h_status;
+}
+
+pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
+                          int64_t* ids, float* scores, int32_t* n_out) {
+    if (!cursors || nc < 0 || n < 0 || !n_out || (nc > 0 && n > 0 && (!ids || !scores)))
+        return PVS_ERR_INVALID;
+    if (nc == 0) return PVS_OK;
+    pvs_index* x = cursors[0] ? cursors[0]->index : nullptr;
+    if (!x) return PVS_ERR_INVALID;
+    cudaStream_t st = cursors[0]->stream;
+    for (int32_t i = 0; i < nc; ++i) {
+        n_out[i] = 0;
+        if (!cursors[i] || cursors[i]->index != x || cursors[i]->stream != st)
+            return PVS_ERR_INVALID;
+    }
+    for (int32_t i = 0; i < nc; ++i)
+        if (cursors[i]->state < 0) return PVS_ERR_FAILED;
+    const bool fused = n <= kPullFusedMax;
+    if (!fused) {   // large pulls: one cursor at a time
+        pvs_status worst = PVS_OK;
+        for (int32_t i = 0; i < nc; ++i) {
+            pvs_status s = outputs_on_device
+                               ? pvs_next_device(cursors[i], n, ids + (int64_t)i * n,
+                                                 scores + (int64_t)i * n, &n_out[i])
+                               : pvs_next(cursors[i], n, ids + (int64_t)i * n,
+                                          scores + (int64_t)i * n, &n_out[i]);
+            if (s < 0) return s;
+        }
+        return worst;
+    }
+    DevBuf buf(st);   // released in stream order after the launches that read it
+    int64_t* d_ids = outputs_on_device ? ids : buf.get<int64_t>((size_t)nc * n);
+    float* d_scores = outputs_on_device ? scores : buf.get<float>((size_t)nc * n);
+    PullArgs* d_args = buf.get<PullArgs>((size_t)nc);
+    if (!d_ids || !d_scores || !d_args) return PVS_ERR_OOM;
+    std::vector<PullArgs> args;
+    std::vector<int32_t> who;
+    args.reserve(nc);
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        const int64_t n_eff = std::min<int64_t>(n, c->visible - c->emitted);
+        n_out[i] = (int32_t)n_eff;
+        if (n_eff <= 0) continue;
+        pvs_status s = prepare_pull(c, n_eff);
+        if (s != PVS_OK) return fail(c, s);
+        PullArgs a;
+        a.w_id = c->w_id;
+        a.w_lo = c->w_lo;
+        a.w_hi = c->w_hi;
+        a.w_len = &c->ctr->w_len;
+        a.lo = c->scanned ? c->lo : nullptr;
+        a.hi = c->scanned ? c->hi : nullptr;
+        a.qraw = c->qraw;
+        a.raw = x->raw;
+        a.m_raw = x->m_raw;
+        a.n = (int)n_eff;
+        a.cand = c->cand;
+        a.keys = reinterpret_cast<unsigned long long*>(c->keys);
+        a.out_ids = d_ids + (int64_t)i * n;
+        a.out_scores = d_scores + (int64_t)i * n;
+        a.status = c->d_status;
+        a.ctr = c->ctr;
+        args.push_back(a);
+        who.push_back(i);
+    }
+    if (!args.empty()) {
+        PVS_CUDA(cudaMemcpyAsync(d_args, args.data(), args.size() * sizeof(PullArgs),
+                                 cudaMemcpyHostToDevice, st));
+        PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, st));
+    }
+    for (int32_t i : who) {
+        cursors[i]->emitted += n_out[i];
+        cursors[i]->pulls++;
+    }
+    pvs_status result = PVS_OK;
+    if (!outputs_on_device) {
+        PVS_CUDA(cudaMemcpyAsync(ids, d_ids, (size_t)nc * n * sizeof(int64_t),
+                                 cudaMemcpyDeviceToHost, st));
+        PVS_CUDA(cudaMemcpyAsync(scores, d_scores, (size_t)nc * n * sizeof(float),
+                                 cudaMemcpyDeviceToHost, st));
+        for (int32_t i : who) {
+            pvs_status s = check_device_status(cursors[i]);
+            if (s != PVS_OK) result = s;
+        }
+        if (result != PVS_OK) return result;
+    }
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
     }
     return PVS_OK;
 }
@@ -727,6 +1172,7 @@ pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
     out->state = c->state;
     harvest_interval_time(c);
     out->interval_ms = c->interval_ms;
+    out->batch_passes = c->batch_passes;
     return PVS_OK;
 }
 
@@ -735,14 +1181,18 @@ pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float*
     if (!c || first < 0 || count < 0 || first + count > c->rows || (count > 0 && (!lo || !hi)))
         return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
-    pvs_status s = cursor_alloc_rows(c);
-    if (s != PVS_OK) return fail(c, s);
-    if (!c->scanned) {
+    pvs_status s = PVS_OK;
+    if (c->batch_ws) {
+        s = rescan_from_batch(c);
+        if (s != PVS_OK) return fail(c, s);
+    } else if (!c->scanned) {
+        s = cursor_alloc_rows(c);
+        if (s != PVS_OK) return fail(c, s);
         s = interval_pass(c);
         if (s != PVS_OK) return fail(c, s);
-        s = check_device_status(c);
-        if (s != PVS_OK) return s;
     }
+    s = check_device_status(c);
+    if (s != PVS_OK) return s;
     if (count == 0) return PVS_OK;
     cudaStream_t st = c->stream;
     PVS_CUDA(cudaMemcpyAsync(lo, c->lo + first, count * sizeof(float), cudaMemcpyDeviceToHost, st));

@@ -8,16 +8,18 @@
 
 namespace pvs {
 
-__global__ void __launch_bounds__(256) refine_kernel(
-    const int32_t* __restrict__ cand, const unsigned int* cand_len, const int32_t* __restrict__ w_id,
-    float* w_lo, float* w_hi, float* lo, float* hi, const float* __restrict__ qraw,
-    const float* __restrict__ raw, int m_raw, int* status, DevCounters* ctr) {
+// Warps warp0, warp0 + nwarps, ... of the launch score candidates of one
+// cursor.  lo / hi (bounds of every row) may be null for a cursor that only
+// holds a working set.
+__device__ inline void refine_warps(const int32_t* __restrict__ cand, const unsigned int* cand_len,
+                                    const int32_t* __restrict__ w_id, float* w_lo, float* w_hi,
+                                    float* lo, float* hi, const float* __restrict__ qraw,
+                                    const float* __restrict__ raw, int m_raw, int* status,
+                                    DevCounters* ctr, int64_t warp0, int64_t nwarps) {
     const int lane = threadIdx.x & 31;
     const int64_t n = *cand_len;
-    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
     unsigned long long refined = 0, fallbacks = 0;
-    for (int64_t i = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n;
-         i += warps) {
+    for (int64_t i = warp0; i < n; i += nwarps) {
         const int32_t w = cand[i];
         const float l = w_lo[w], h = w_hi[w];
         if (!(l < h)) continue;    // resolved: lo == hi is the exact score
@@ -31,14 +33,46 @@ __global__ void __launch_bounds__(256) refine_kernel(
             else if (s < l || s > h) set_status(status, PVS_ERR_INTERVAL);
             w_lo[w] = s;
             w_hi[w] = s;
-            lo[id] = s;
-            hi[id] = s;
+            if (lo) {
+                lo[id] = s;
+                hi[id] = s;
+            }
         }
     }
     if (lane == 0 && refined) {
         atomicAdd(&ctr->refined, refined);
         if (fallbacks) atomicAdd(&ctr->exact_fallbacks, fallbacks);
     }
+}
+
+__global__ void __launch_bounds__(256) refine_kernel(
+    const int32_t* __restrict__ cand, const unsigned int* cand_len, const int32_t* __restrict__ w_id,
+    float* w_lo, float* w_hi, float* lo, float* hi, const float* __restrict__ qraw,
+    const float* __restrict__ raw, int m_raw, int* status, DevCounters* ctr) {
+    refine_warps(cand, cand_len, w_id, w_lo, w_hi, lo, hi, qraw, raw, m_raw, status, ctr,
+                 (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5),
+                 (int64_t)gridDim.x * (blockDim.x >> 5));
+}
+
+// Many cursors at once: blocks_per_cursor consecutive blocks serve cursor
+// blockIdx.x / blocks_per_cursor.
+__global__ void __launch_bounds__(256) refine_batch_kernel(const PullArgs* args,
+                                                           int blocks_per_cursor) {
+    const PullArgs& a = args[blockIdx.x / blocks_per_cursor];
+    const int64_t warps_per_block = blockDim.x >> 5;
+    refine_warps(a.cand, &a.ctr->cand, a.w_id, a.w_lo, a.w_hi, a.lo, a.hi, a.qraw, a.raw,
+                 a.m_raw, a.status, a.ctr,
+                 (int64_t)(blockIdx.x % blocks_per_cursor) * warps_per_block + (threadIdx.x >> 5),
+                 (int64_t)blocks_per_cursor * warps_per_block);
+}
+
+cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
+                                cudaStream_t st) {
+    if (ncursors <= 0) return cudaSuccess;
+    count_launches(1);
+    refine_batch_kernel<<<ncursors * blocks_per_cursor, 256, 0, st>>>(args_dev,
+                                                                       blocks_per_cursor);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_refine(const int32_t* cand, const unsigned int* cand_len,

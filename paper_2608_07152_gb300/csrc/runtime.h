@@ -49,6 +49,9 @@ struct pvs_index {
     std::mutex pool_mutex;                  // cursors may open / close on several threads
     std::mutex pass_mutex;                  // orders interval passes of this index
     cudaEvent_t pass_done = nullptr;        // end of the last interval pass queued
+    // bf16 copy of the codes for the tensor-core batched pass (built on demand)
+    uint16_t* codes_bf16 = nullptr;         // [cap][m_pad]
+    int64_t bf16_rows = 0;                  // rows converted so far
 };
 
 struct pvs_snapshot {
@@ -72,6 +75,8 @@ struct pvs_cursor {
     float* lo = nullptr;
     float* hi = nullptr;
     // working set (ordered by id): rows that can hold the next `horizon` ranks
+    int64_t cap_w = 0;                // capacity of the working-set arrays
+    bool batch_ws = false;            // working set came from a batched pass (no full bounds)
     int32_t* w_id = nullptr;
     float* w_lo = nullptr;
     float* w_hi = nullptr;
@@ -94,6 +99,7 @@ struct pvs_cursor {
     unsigned int* h_small = nullptr;  // pinned scratch (counts, status)
     // stats
     int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;
+    int64_t batch_passes = 0;         // batched (tensor-core) passes this cursor took part in
     cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
     bool ev_pending = false;
     double interval_ms = 0.0;

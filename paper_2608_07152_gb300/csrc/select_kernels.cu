@@ -405,8 +405,10 @@ __global__ void emit_kernel(const uint64_t* __restrict__ keys, int n, const int3
     out_scores[i] = rank_key_score(k);
     w_lo[w] = -INFINITY;
     w_hi[w] = -INFINITY;
-    lo[id] = -INFINITY;
-    hi[id] = -INFINITY;
+    if (lo) {
+        lo[id] = -INFINITY;
+        hi[id] = -INFINITY;
+    }
 }
 
 cudaError_t launch_emit(const uint64_t* keys, int n, const int32_t* w_id, float* w_lo,

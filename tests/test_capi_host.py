@@ -30,10 +30,29 @@ def test_library_exports_every_declared_function():
         assert name in pvs.EXPORTED, name
 
 
-def test_struct_layouts_match_header():
-    assert pvs.ctypes.sizeof(pvs.pvs_stats) == 9 * 8 + 2 * 4 + 8
-    assert pvs.ctypes.sizeof(pvs.eahr_params) == 9 * 4
-    assert pvs.ctypes.sizeof(pvs.eahr_stats) == 4 * 8 + 6 * 4
+def test_struct_layouts_match_header(tmp_path):
+    """The binding's ctypes structures match the C compiler's layout of the
+    structures in include/pvs.h (size and every field offset)."""
+    import subprocess
+    structs = {"pvs_stats": pvs.pvs_stats, "eahr_params": pvs.eahr_params,
+               "eahr_stats": pvs.eahr_stats}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "pvs.h"', "int main(void) {"]
+    for name, cls in structs.items():
+        lines.append(f'printf("{name} size %zu\\n", sizeof({name}));')
+        for field, _ in cls._fields_:
+            lines.append(f'printf("{name} {field} %zu\\n", offsetof({name}, {field}));')
+    lines.append("return 0; }")
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                   check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout
+    c_layout = {tuple(l.split()[:2]): int(l.split()[2]) for l in out.splitlines()}
+    for name, cls in structs.items():
+        assert pvs.ctypes.sizeof(cls) == c_layout[(name, "size")], name
+        for field, _ in cls._fields_:
+            assert getattr(cls, field).offset == c_layout[(name, field)], (name, field)
 
 
 def test_status_strings():
