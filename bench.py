@@ -56,6 +56,9 @@ def parse():
     p.add_argument("--queries", type=int, default=50, help="queries per step")
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--workload", default="passage", choices=["passage", "batched"],
+                   help="passage: single-query ranking (default); batched: 256-query "
+                        "tensor-core batches")
     return p.parse_args()
 
 
@@ -146,15 +149,15 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def build_corpus_index(pvs, synth, torch, n, stream, device):
+def build_corpus_index(pvs, synth, torch, n, stream, device, components=COMPONENTS, seed=2):
     """Generate the mixture corpus chunk by chunk straight into the index."""
-    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=device)
+    centres = synth.mixture_centres(components, DIM, seed=seed, device=device)
     index = None
     chunk = 1 << 20
     t0 = time.perf_counter()
     for r in range(0, n, chunk):
         c = min(chunk, n - r)
-        rows = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+        rows = synth.mixture_rows(c, centres, WITHIN_STD, seed=seed, first=r)
         if index is None:
             index = pvs.pvs_build(rows, stream=stream)
         else:
@@ -306,6 +309,122 @@ def reference_arm(args):
     print(json.dumps(line), flush=True)
 
 
+BATCH_N = 1_000_000
+BATCH_COMPONENTS = 1024
+BATCH_Q = 256
+BATCH_RANKS = 200
+BATCH_CHUNK = 50
+BATCH_WORKLOAD = ("batched queries: N=1,000,000 x d=768 Gaussian mixture (1,024 components, "
+                  "within std 0.35), 256 concurrent queries per batch, first 200 exact ranks "
+                  "per query in chunks of 50")
+
+
+def bf16_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """Batched workload: one step = one batch of 256 queries opened together
+    (one tensor-core interval pass), then 4 batched pulls of 50 ranks."""
+    stream = torch.cuda.Stream(device=dev)
+    n = BATCH_N if args.n == N_CORPUS else args.n
+    index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev,
+                                                 components=BATCH_COMPONENTS, seed=4)
+    nb = args.warmup + args.steps
+    queries = synth.mixture_queries(nb * BATCH_Q, centres, QUERY_NOISE, seed=5 + 7919 * rank)
+    queries = queries.reshape(nb, BATCH_Q, DIM).contiguous()
+    ids_t = torch.empty((BATCH_Q, BATCH_CHUNK), dtype=torch.int64, device=dev)
+    sc_t = torch.empty((BATCH_Q, BATCH_CHUNK), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+
+    def step(qb, stats):
+        curs = pvs.pvs_cursor_open_batch(index, qb, horizon=BATCH_RANKS)
+        for _ in range(BATCH_RANKS // BATCH_CHUNK):
+            pvs.pvs_next_batch(curs, BATCH_CHUNK, ids_t, sc_t)
+        for c in curs:
+            if pvs.pvs_cursor_sync(c) < 0:
+                raise RuntimeError("cursor failed")
+        if stats is not None:
+            stats.extend(pvs.pvs_cursor_stats(c) for c in curs)
+        for c in curs:
+            pvs.pvs_cursor_close(c)
+
+    for w in range(args.warmup):
+        step(queries[w], None)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    stats = []
+    launches0 = pvs.pvs_launch_count()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for s in range(args.steps):
+            step(queries[args.warmup + s], stats)
+        end.record(stream)
+        stream.synchronize()
+    launches = pvs.pvs_launch_count() - launches0
+    elapsed = start.elapsed_time(end) / 1e3
+    if pg:
+        t = torch.tensor([elapsed], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        elapsed = float(t.item())
+    ranks_total = args.steps * BATCH_Q * BATCH_RANKS * world
+    value = ranks_total / elapsed
+
+    # e2e: host queries, host outputs
+    qh = [np.ascontiguousarray(queries[args.warmup + s].cpu().numpy()) for s in range(args.steps)]
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        curs = pvs.pvs_cursor_open_batch(index, qh[s], horizon=BATCH_RANKS)
+        for _ in range(BATCH_RANKS // BATCH_CHUNK):
+            pvs.pvs_next_batch(curs, BATCH_CHUNK)
+        for c in curs:
+            pvs.pvs_cursor_close(c)
+    e2e_elapsed = time.perf_counter() - t0
+    e2e_value = ranks_total / e2e_elapsed
+
+    batch_ms = statistics.mean(s["batch_ms"] for s in stats)   # one filter pass per batch
+    flops = 2.0 * BATCH_Q * n * DIM
+    achieved = flops / (batch_ms / 1e3) / 1e12
+    peak, peak_kind = bf16_peak()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": BATCH_WORKLOAD, "N": n, "d": DIM, "queries_per_batch": BATCH_Q,
+                   "ranks_per_query": BATCH_RANKS, "chunk": BATCH_CHUNK,
+                   "l2": "no flush: each batch pass streams 1.5 GB of bf16 codes (> 129 MB L2)",
+                   "parallelism": f"replicas x{world}"},
+        "e2e": {"value": e2e_value, "unit": UNIT,
+                "h2d_bytes_per_step": BATCH_Q * DIM * 4,
+                "d2h_bytes_per_step": BATCH_Q * BATCH_RANKS * (8 + 4)},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "kernel": "batch_interval_kernel (filter pass)"},
+        "gpu_launches": launches,
+        "batch_pass_ms": batch_ms,
+        "per_query": {"refined_mean": statistics.mean(s["refined"] for s in stats),
+                      "single_query_passes": sum(s["interval_passes"] for s in stats)},
+        "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    pvs.pvs_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -324,6 +443,9 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
+    if args.workload == "batched":
+        main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
 
     stream = torch.cuda.Stream(device=dev)
     n = args.n

@@ -74,6 +74,8 @@ typedef struct pvs_stats {
     double interval_ms;       /* device time of the interval passes, measured
                                  with CUDA events on the cursor's stream       */
     int64_t batch_passes;     /* batched tensor-core passes that served it     */
+    double batch_ms;          /* device time of that batched pass (shared by
+                                 the cursors of its group), CUDA events       */
 } pvs_stats;
 
 /* ---------------------------------------------------------------------------

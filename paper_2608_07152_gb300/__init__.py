@@ -47,7 +47,8 @@ class pvs_stats(ctypes.Structure):
         "visible", "emitted", "refined", "exact_fallbacks", "interval_passes",
         "horizon_builds", "pulls", "candidates", "code_bytes")] + [
         ("state", ctypes.c_int32), ("reserved", ctypes.c_int32),
-        ("interval_ms", ctypes.c_double), ("batch_passes", ctypes.c_int64)]
+        ("interval_ms", ctypes.c_double), ("batch_passes", ctypes.c_int64),
+        ("batch_ms", ctypes.c_double)]
 
 
 class eahr_params(ctypes.Structure):

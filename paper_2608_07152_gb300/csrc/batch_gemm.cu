@@ -7,16 +7,18 @@
 // and every partial sum stays below 2^24, so fp32 accumulation is exact and
 // D holds the exact integers.
 //
-// Persistent kernel, one CTA per SM, 6 warps:
+// Persistent kernel, one CTA per SM, 18 warps:
 //   warp 0     TMA producer: A tile (128 rows x 64 bf16) and B tile (Qp x 64)
 //              per K chunk into a 4-stage ring, 128-byte swizzle;
 //   warp 1     allocates 512 TMEM columns, issues tcgen05.mma (M=128, N=Qp,
 //              K=16) x 4 per chunk, commits each stage back to the producer
 //              and each finished tile to the epilogue;
-//   warps 2-5  epilogue: one TMEM lane (= one corpus row) per thread,
-//              tcgen05.ld of 32 query columns at a time, then the interval
-//              arithmetic of App. A.1 in the same operation order as the
-//              single-query pass.
+//   warps 2-17 epilogue: one TMEM lane (= one corpus row) per thread; the
+//              four warps that share a TMEM lane quarter split the query
+//              columns (32 at a time, tcgen05.ld), so every scheduler has
+//              four epilogue warps to hide load and arithmetic latency; then
+//              the interval arithmetic of App. A.1 in the same operation
+//              order as the single-query pass.
 // Two TMEM accumulators (2 x 256 columns) let the epilogue of tile i run
 // under the MMAs of tile i+1.
 //
@@ -44,7 +46,8 @@ constexpr int kStages = 4;
 constexpr int kStageA = kBM * kBK * 2;        // 16 KB
 constexpr int kStageB = kMaxBN * kBK * 2;     // 32 KB
 constexpr int kStageBytes = kStageA + kStageB;
-constexpr int kBatchThreads = 192;
+constexpr int kEpiWarps = 16;   // 4 per TMEM lane quarter: latency hiding for the epilogue
+constexpr int kBatchThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
 
 struct BatchShared {
@@ -55,8 +58,7 @@ struct BatchShared {
     uint32_t tmem_base;
     int abort;
     QueryScalars qs[kMaxBN];
-    float tau[kMaxBN];
-    float rmax[kMaxBN];
+    float4 flt[kMaxBN];   // filter: (s_q, rmax_q, tau_q, 0)
 };
 
 // The abort flag is written and polled by different warps.
@@ -67,9 +69,10 @@ __device__ __forceinline__ void raise_abort(BatchShared& sh) {
     *reinterpret_cast<volatile int*>(&sh.abort) = 1;
 }
 
-__device__ __forceinline__ void interval_of(int dot, const QueryScalars& q, float sv, float vn,
+// fdot: the exact dot product as the fp32 accumulator holds it (an integer
+// below 2^24, so it equals the float conversion of the int32 dot product).
+__device__ __forceinline__ void interval_of(float fdot, const QueryScalars& q, float sv, float vn,
                                             float en, float& lo, float& hi) {
-    const float fdot = __int2float_rn(dot);
     const float c = __fmul_rn(__fmul_rn(q.s, sv), fdot);
     const float E = __fadd_ru(__fmul_ru(q.enorm, vn), __fmul_ru(q.qhat, en));
     const float G = __fmul_ru(__fadd_ru(__fadd_ru(fabsf(c), E), __fmul_ru(q.qnorm, vn)), q.gamma);
@@ -97,8 +100,8 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
     for (int i = threadIdx.x; i < kMaxBN; i += blockDim.x) {
         if (i < nq) {
             sh.qs[i] = a.qs[i];
-            sh.tau[i] = a.tau ? a.tau[i] : -INFINITY;
-            sh.rmax[i] = a.rmax ? a.rmax[i] : INFINITY;
+            sh.flt[i] = make_float4(a.qs[i].s, a.rmax ? a.rmax[i] : INFINITY,
+                                    a.tau ? a.tau[i] : -INFINITY, 0.0f);
         }
     }
     if (threadIdx.x == 0) {
@@ -108,7 +111,7 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&sh.tfull[b], 1);
-            mbar_init(&sh.tempty[b], 4);
+            mbar_init(&sh.tempty[b], kEpiWarps);
         }
         sh.abort = 0;
         mbar_fence_init();
@@ -198,6 +201,7 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
     } else {
         // ---------------- epilogue ----------------
         const int quarter = warp & 3;               // TMEM lanes 32*quarter ..
+        const int cgroup = (warp - 2) >> 2;         // this warp's share of the 32-column chunks
         const int r_in_tile = quarter * 32 + lane;
         int it = 0;
         for (int64_t i = blockIdx.x; i < niter; i += gridDim.x, ++it) {
@@ -220,7 +224,7 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
                 en = __ldg(a.enorm + row);
             }
             const int64_t srow = i * kBM + r_in_tile;   // row of the dump arrays
-            for (int cc = 0; cc < nqp / 32; ++cc) {
+            for (int cc = cgroup; cc < nqp / 32; cc += kEpiWarps / 4) {
                 uint32_t r[32];
                 tc::ld_32x32b_x32(tmem + ((uint32_t)(quarter * 32) << 16) +
                                       (uint32_t)(b * kMaxBN + cc * 32),
@@ -230,21 +234,22 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
                 for (int j = 0; j < 32; ++j) {
                     const int q = cc * 32 + j;
                     if (q >= nq) break;
-                    const int dot = __float2int_rn(__uint_as_float(r[j]));
+                    const float fdot = __uint_as_float(r[j]);
                     const QueryScalars& qs = sh.qs[q];
                     if (a.mode == 0) {
                         float lo = -INFINITY, hi = -INFINITY;
-                        if (live) interval_of(dot, qs, sv, vn, en, lo, hi);
+                        if (live) interval_of(fdot, qs, sv, vn, en, lo, hi);
                         if (live && (!isfinite(lo) || !isfinite(hi)))
                             set_status(a.status, PVS_ERR_OVERFLOW);
                         a.dump_lo[(int64_t)q * a.dump_ld + srow] = lo;
-                        a.dump_hi[(int64_t)q * a.dump_ld + srow] = hi;
+                        if (a.dump_hi) a.dump_hi[(int64_t)q * a.dump_ld + srow] = hi;
                     } else if (live) {
-                        const float c = __fmul_rn(__fmul_rn(qs.s, sv), __int2float_rn(dot));
-                        const float tau = sh.tau[q];
-                        if (__fadd_ru(c, sh.rmax[q]) < tau) continue;   // hi < tau for sure
+                        const float4 f = sh.flt[q];
+                        const float c = __fmul_rn(__fmul_rn(f.x, sv), fdot);
+                        const float tau = f.z;
+                        if (__fadd_ru(c, f.y) < tau) continue;   // hi < tau for sure
                         float lo, hi;
-                        interval_of(dot, qs, sv, vn, en, lo, hi);
+                        interval_of(fdot, qs, sv, vn, en, lo, hi);
                         if (!isfinite(lo) || !isfinite(hi)) set_status(a.status, PVS_ERR_OVERFLOW);
                         if (hi < tau) continue;
                         const unsigned int pos = atomicAdd(&a.w_len[q], 1u);

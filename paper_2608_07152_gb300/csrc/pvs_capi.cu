@@ -213,11 +213,20 @@ void cursor_reset(pvs_cursor* c) {
     c->horizon = c->horizon_base = 0;
     c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
     c->batch_passes = 0;
+    c->batch_ms = 0.0;
     c->ev_pending = false;
     c->interval_ms = 0.0;
 }
 
-constexpr size_t kCursorPool = 4;   // closed cursors kept per index
+// Closed cursors kept per index for reuse: at most kCursorPool of them and
+// kCursorPoolBytes of device buffers (batched opens reuse hundreds of small
+// cursors; single-query cursors hold buffers for every row).
+constexpr size_t kCursorPool = 1024;
+constexpr size_t kCursorPoolBytes = size_t(4) << 30;
+
+size_t cursor_device_bytes(const pvs_cursor* c) {
+    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096;
+}
 
 // Allocate the per-row state of a cursor (first pull); a pooled cursor keeps
 // buffers that are large enough.
@@ -560,6 +569,7 @@ pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs
         if (!x->cursor_pool.empty()) {
             c = x->cursor_pool.back();
             x->cursor_pool.pop_back();
+            x->pool_bytes -= cursor_device_bytes(c);
         }
     }
     if (!c) {
@@ -623,15 +633,22 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     const int64_t rows = sd->rows;
     if (rows == 0) return PVS_OK;
 
+    // Sample every stride-th tile and take tau_q = the k_s-th largest sampled
+    // lower bound, k_s = 1.5 H / stride + 4: about 1.5 H rows of the corpus
+    // reach it.  It misses the horizon (fewer than H rows reach it) only when
+    // at least k_s of the top-H rows were sampled; that count is about
+    // Poisson(H / stride), so this happens for well under 1 % of the queries
+    // (H = 200: stride 12, k_s = 29, mean 16.7), which then rescan.
     const int64_t ntiles = (rows + 127) / 128;
-    const int stride = ntiles >= 64 ? 16 : 1;
+    int stride = (int)std::min<int64_t>(16, std::max<int64_t>(1, (3 * (int64_t)horizon) / 48));
+    if (ntiles < 8 * (int64_t)stride) stride = 1;
     const int64_t ld = ((ntiles + stride - 1) / stride) * 128;
     const unsigned int k_s =
-        stride == 1 ? (unsigned int)horizon : (unsigned int)((3 * (int64_t)horizon + 15) / 16 + 8);
-    const int w_cap = (int)std::min<int64_t>({(int64_t)kWsSortMax, 16 * (int64_t)horizon + 1024,
-                                              std::max<int64_t>(rows, 1)});
+        stride == 1 ? (unsigned int)horizon
+                    : (unsigned int)((3 * (int64_t)horizon + 2 * stride - 1) / (2 * stride) + 4);
+    const int w_cap = (int)std::min<int64_t>((int64_t)kWsSortMax, std::max<int64_t>(rows, 1));
     float* dlo = buf.get<float>((size_t)nq * ld);
-    float* dhi = buf.get<float>((size_t)nq * ld);
+    float* dhi = dlo;   // the sampling pass needs the lower bounds only
     float* tau = buf.get<float>((size_t)nq);
     float* rmax = buf.get<float>((size_t)nq);
     unsigned int* maxes = buf.get<unsigned int>(2);
@@ -664,7 +681,7 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     a.mode = 0;
     a.tile_stride = stride;
     a.dump_lo = dlo;
-    a.dump_hi = dhi;
+    a.dump_hi = nullptr;
     a.dump_ld = ld;
     PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
     PVS_CUDA(launch_batch_tau(dlo, ld, (unsigned int)ld, nq, k_s, tau, st));
@@ -683,10 +700,15 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     a.w_cap = w_cap;
     a.w_len = wlen;
     a.h_eff = heff;
+    cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+    PVS_CUDA(cudaEventCreate(&ev0));
+    PVS_CUDA(cudaEventCreate(&ev1));
     {
         std::lock_guard<std::mutex> lock(x->pass_mutex);   // one HBM pass at a time
         if (x->pass_done) PVS_CUDA(cudaStreamWaitEvent(st, x->pass_done, 0));
+        PVS_CUDA(cudaEventRecord(ev0, st));
         PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
+        PVS_CUDA(cudaEventRecord(ev1, st));
         if (!x->pass_done)
             PVS_CUDA(cudaEventCreateWithFlags(&x->pass_done, cudaEventDisableTiming));
         PVS_CUDA(cudaEventRecord(x->pass_done, st));
@@ -706,6 +728,10 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     PVS_CUDA(cudaMemcpyAsync(h_heff.data(), heff, nq * sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaMemcpyAsync(&h_status, status, sizeof(int), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaStreamSynchronize(st));
+    float pass_ms = 0.0f;
+    cudaEventElapsedTime(&pass_ms, ev0, ev1);
+    cudaEventDestroy(ev0);
+    cudaEventDestroy(ev1);
     if (h_status != 0) return (pvs_status)h_status;
     for (int i = 0; i < nq; ++i) {
         pvs_cursor* c = out[i];
@@ -715,6 +741,7 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
             c->horizon_base = 0;
         }
         c->batch_passes = 1;
+        c->batch_ms = pass_ms;   // the filter pass, shared by the group's cursors
     }
     return PVS_OK;
 }
@@ -848,6 +875,7 @@ void pvs_index_free(pvs_index* x) {
         delete c;
     }
     x->cursor_pool.clear();
+    x->pool_bytes = 0;
     dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
     dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage), dev_free(x->codes_bf16);
     if (x->pass_done) cudaEventDestroy(x->pass_done);
@@ -884,6 +912,7 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
         if (!x->cursor_pool.empty()) {   // reuse a closed cursor's buffers
             c = x->cursor_pool.back();
             x->cursor_pool.pop_back();
+            x->pool_bytes -= cursor_device_bytes(c);
         }
     }
     if (!c) {
@@ -1173,6 +1202,7 @@ pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
     harvest_interval_time(c);
     out->interval_ms = c->interval_ms;
     out->batch_passes = c->batch_passes;
+    out->batch_ms = c->batch_ms;
     return PVS_OK;
 }
 
@@ -1230,7 +1260,10 @@ void pvs_cursor_close(pvs_cursor* c) {
     harvest_interval_time(c);
     if (x) {
         std::lock_guard<std::mutex> lock(x->pool_mutex);
-        if (x->cursor_pool.size() < kCursorPool) {   // keep the buffers for the next cursor
+        const size_t bytes = cursor_device_bytes(c);
+        if (x->cursor_pool.size() < kCursorPool &&
+            x->pool_bytes + bytes <= kCursorPoolBytes) {   // keep the buffers for the next cursor
+            x->pool_bytes += bytes;
             cursor_reset(c);
             x->cursor_pool.push_back(c);
             return;

@@ -46,6 +46,7 @@ struct pvs_index {
     float* d_stage = nullptr;         // host-input staging
     size_t stage_floats = 0;
     std::vector<pvs_cursor*> cursor_pool;   // closed cursors whose buffers are reused
+    size_t pool_bytes = 0;                  // device bytes held by pooled cursors
     std::mutex pool_mutex;                  // cursors may open / close on several threads
     std::mutex pass_mutex;                  // orders interval passes of this index
     cudaEvent_t pass_done = nullptr;        // end of the last interval pass queued
@@ -100,6 +101,7 @@ struct pvs_cursor {
     // stats
     int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;
     int64_t batch_passes = 0;         // batched (tensor-core) passes this cursor took part in
+    double batch_ms = 0.0;            // device time of that pass (shared by its cursors)
     cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
     bool ev_pending = false;
     double interval_ms = 0.0;
