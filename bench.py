@@ -342,34 +342,40 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     sc_t = torch.empty((BATCH_Q, BATCH_CHUNK), dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
 
-    def step(qb, stats):
+    def step(qb, pass_ms, stats=None):
         curs = pvs.pvs_cursor_open_batch(index, qb, horizon=BATCH_RANKS)
         for _ in range(BATCH_RANKS // BATCH_CHUNK):
             pvs.pvs_next_batch(curs, BATCH_CHUNK, ids_t, sc_t)
-        for c in curs:
-            if pvs.pvs_cursor_sync(c) < 0:
-                raise RuntimeError("cursor failed")
-        if stats is not None:
-            stats.extend(pvs.pvs_cursor_stats(c) for c in curs)
-        for c in curs:
-            pvs.pvs_cursor_close(c)
+        if stats is None:
+            states = pvs.pvs_cursor_sync_batch(curs)   # one wait for every cursor's status
+        else:
+            st = pvs.pvs_cursor_stats_batch(curs)
+            stats.extend(st)
+            states = [x["state"] for x in st]
+        if any(x < 0 for x in states):
+            raise RuntimeError("cursor failed")
+        if pass_ms is not None:   # device time of this batch's filter pass (CUDA events)
+            pass_ms.append(pvs.pvs_cursor_stats(curs[0])["batch_ms"])
+        pvs.pvs_cursor_close_batch(curs)
 
     for w in range(args.warmup):
         step(queries[w], None)
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
-    stats = []
+    pass_ms = []
     launches0 = pvs.pvs_launch_count()
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         start.record(stream)
         for s in range(args.steps):
-            step(queries[args.warmup + s], stats)
+            step(queries[args.warmup + s], pass_ms)
         end.record(stream)
         stream.synchronize()
     launches = pvs.pvs_launch_count() - launches0
+    stats = []   # per-query counters from one more (untimed) batch of the same queries
+    step(queries[args.warmup], None, stats)
     elapsed = start.elapsed_time(end) / 1e3
     if pg:
         t = torch.tensor([elapsed], device=dev)
@@ -386,12 +392,11 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         curs = pvs.pvs_cursor_open_batch(index, qh[s], horizon=BATCH_RANKS)
         for _ in range(BATCH_RANKS // BATCH_CHUNK):
             pvs.pvs_next_batch(curs, BATCH_CHUNK)
-        for c in curs:
-            pvs.pvs_cursor_close(c)
+        pvs.pvs_cursor_close_batch(curs)
     e2e_elapsed = time.perf_counter() - t0
     e2e_value = ranks_total / e2e_elapsed
 
-    batch_ms = statistics.mean(s["batch_ms"] for s in stats)   # one filter pass per batch
+    batch_ms = statistics.mean(pass_ms)   # one filter pass per batch
     flops = 2.0 * BATCH_Q * n * DIM
     achieved = flops / (batch_ms / 1e3) / 1e12
     peak, peak_kind = bf16_peak()

@@ -189,6 +189,22 @@ pvs_status pvs_cursor_sync(pvs_cursor* cursor);
 pvs_status pvs_cursor_stats(pvs_cursor* cursor, pvs_stats* out);
 void pvs_cursor_close(pvs_cursor* cursor);
 
+/* Batch forms of pvs_cursor_sync, pvs_cursor_stats and pvs_cursor_close for
+ * the nc cursors of a batched open (a host array of nc non-null cursors; no
+ * cursor twice).  They gather the device status words (and counters) of all
+ * cursors that share a stream with one launch, one copy and one wait, instead
+ * of one round trip per cursor.  pvs_cursor_sync_batch writes each cursor's
+ * state to states[i] (host, nc entries: PVS_OK, PVS_EXHAUSTED or the
+ * failure; a device failure makes that cursor Failed as pvs_cursor_sync
+ * does) and returns PVS_OK unless the call itself failed (PVS_ERR_INVALID
+ * for a null array or cursor, PVS_ERR_CUDA, PVS_ERR_OOM).
+ * pvs_cursor_stats_batch writes out[i] (host, nc entries) as
+ * pvs_cursor_stats would.  pvs_cursor_close_batch waits for each distinct
+ * stream once, then closes every cursor; null entries are skipped. */
+pvs_status pvs_cursor_sync_batch(pvs_cursor** cursors, int32_t nc, int32_t* states);
+pvs_status pvs_cursor_stats_batch(pvs_cursor** cursors, int32_t nc, pvs_stats* out);
+void pvs_cursor_close_batch(pvs_cursor** cursors, int32_t nc);
+
 /* Diagnostics.  Copy to host the score interval [lo, hi] that the cursor
  * holds for ids first .. first+count-1 of its snapshot: the App. A.1 interval
  * before an item is scored, lo == hi == its authoritative score after, and

@@ -125,9 +125,14 @@ def round_real_to_f32(s64: float, residual_sign: int) -> np.float32:
 
     RN_f32(x) == RN_f32(s64) unless s64 is exactly halfway between two
     adjacent float32 values (then x's side of s64 decides), because every
-    such halfway point is itself a binary64 number.
+    such halfway point is itself a binary64 number.  A result that rounds to
+    zero is returned as +0: the score orders by value and -0 == +0, so the
+    sign of a zero carries nothing, and one canonical zero makes scores
+    comparable bit for bit.
     """
     f = np.float32(s64)
+    if f == 0:
+        return np.float32(0.0)                  # a score that rounds to zero is +0
     if not np.isfinite(f) or float(f) == s64:
         return f
     g = np.nextafter(f, np.float32(math.inf) if s64 > float(f) else np.float32(-math.inf))
@@ -176,6 +181,7 @@ def exact_scores(q: np.ndarray, V: np.ndarray, block: int = 1 << 16) -> np.ndarr
         out[b0:b0 + block][ok] = lo[ok]
         for i in np.nonzero(~ok)[0]:
             out[b0 + i] = exact_score_one(q, V[b0 + i])
+    out[out == 0] = np.float32(0.0)             # canonical +0, as round_real_to_f32
     return out
 
 

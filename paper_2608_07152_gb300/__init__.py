@@ -95,6 +95,9 @@ def _load() -> ctypes.CDLL:
         "pvs_cursor_bounds": (i32, [P, i64, i64, P, P]),
         "pvs_cursor_score_ids": (i32, [P, P, i32, P]),
         "pvs_cursor_close": (None, [P]),
+        "pvs_cursor_sync_batch": (i32, [P, i32, P]),
+        "pvs_cursor_stats_batch": (i32, [P, i32, P]),
+        "pvs_cursor_close_batch": (None, [P, i32]),
         "pvs_status_string": (ctypes.c_char_p, [i32]),
         "pvs_launch_count": (i64, []),
         "pvs_rank_exact_noalloc": (i32, [P, P, i32, i32, i32, P, P, P]),
@@ -118,6 +121,7 @@ EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_i
             "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
             "pvs_cursor_set_stream", "pvs_next_batch", "pvs_batch_bounds",
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
+            "pvs_cursor_sync_batch", "pvs_cursor_stats_batch", "pvs_cursor_close_batch",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
             "eahr_topk_lists")
 
@@ -253,14 +257,18 @@ def pvs_next_device(cursor, n: int, ids, scores):
     return got.value, st
 
 
+def _cursor_array(cursors):
+    return (ctypes.c_void_p * max(len(cursors), 1))(
+        *[c.value if isinstance(c, ctypes.c_void_p) else c for c in cursors])
+
+
 def pvs_next_batch(cursors, n: int, ids=None, scores=None):
     """Next n ranks of every cursor.  Without ids/scores: host outputs, returns
     (ids int64[nc, n], scores float32[nc, n], n_out int32[nc]); with CUDA
     tensors ids / scores of shape [nc, >= n] (row stride n): queued, returns
     n_out."""
     nc = len(cursors)
-    arr = (ctypes.c_void_p * max(nc, 1))(*[c.value if isinstance(c, ctypes.c_void_p) else c
-                                            for c in cursors])
+    arr = _cursor_array(cursors)
     n_out = np.zeros(max(nc, 1), np.int32)
     if ids is None:
         h_ids = np.zeros((max(nc, 1), max(n, 1)), np.int64)
@@ -323,6 +331,27 @@ def pvs_cursor_score_ids(cursor, ids):
 
 def pvs_cursor_close(cursor) -> None:
     _lib.pvs_cursor_close(cursor)
+
+
+def pvs_cursor_sync_batch(cursors):
+    """States (int32[nc]) of many cursors after one wait per stream."""
+    states = np.zeros(max(len(cursors), 1), np.int32)
+    _check(_lib.pvs_cursor_sync_batch(_cursor_array(cursors), len(cursors),
+                                      states.ctypes.data), "pvs_cursor_sync_batch")
+    return states[:len(cursors)]
+
+
+def pvs_cursor_stats_batch(cursors) -> list:
+    out = (pvs_stats * max(len(cursors), 1))()
+    _check(_lib.pvs_cursor_stats_batch(_cursor_array(cursors), len(cursors),
+                                       ctypes.cast(out, ctypes.c_void_p)),
+           "pvs_cursor_stats_batch")
+    return [{name: getattr(out[i], name) for name, _ in pvs_stats._fields_ if name != "reserved"}
+            for i in range(len(cursors))]
+
+
+def pvs_cursor_close_batch(cursors) -> None:
+    _lib.pvs_cursor_close_batch(_cursor_array(cursors), len(cursors))
 
 
 PVS_NOALLOC_MAX_VECTORS = 8192

@@ -1,8 +1,10 @@
 // Small kernels around the batched interval pass: corpus maxima of the norm
 // bounds, the per-query upper bound rmax_q of the interval half-width (the
 // cheap pre-filter of the filter pass), copying batch-encoded queries into the
-// cursors' own buffers, and carrying a working set's state (resolved scores,
-// delivered items) into freshly computed full bounds when a cursor rescans.
+// cursors' own buffers, carrying a working set's state (resolved scores,
+// delivered items) into freshly computed full bounds when a cursor rescans,
+// and gathering the status words and counters of many cursors so that a
+// batch is checked with one copy and one synchronisation.
 #include "kernels.h"
 #include "pvs_common.cuh"
 
@@ -69,7 +71,11 @@ __global__ void copy_query_kernel(const int8_t* __restrict__ zq_b, const float* 
     const QueryDst d = dst[q];
     for (int j = threadIdx.x; j < m_pad; j += blockDim.x) d.zq[j] = zq_b[(int64_t)q * m_pad + j];
     for (int j = threadIdx.x; j < m_raw; j += blockDim.x) d.qraw[j] = qraw_b[(int64_t)q * m_raw + j];
-    if (threadIdx.x == 0) *d.qs = qs_b[q];
+    if (threadIdx.x == 0) {
+        *d.qs = qs_b[q];
+        *d.ctr = DevCounters{};
+        *d.status = 0;
+    }
 }
 
 cudaError_t launch_copy_queries(const int8_t* zq_b, const float* qraw_b, const QueryScalars* qs_b,
@@ -106,6 +112,22 @@ cudaError_t launch_scatter_ws(const int32_t* w_id, const float* w_lo, const floa
                               cudaStream_t st) {
     count_launches(1);
     scatter_ws_kernel<<<grid, 256, 0, st>>>(w_id, w_lo, w_hi, w_len, lo, hi);
+    return cudaGetLastError();
+}
+
+__global__ void gather_state_kernel(const CursorRef* __restrict__ refs, int n, int* status_out,
+                                    DevCounters* ctr_out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    status_out[i] = *refs[i].status;
+    if (ctr_out) ctr_out[i] = *refs[i].ctr;
+}
+
+cudaError_t launch_gather_state(const CursorRef* refs, int n, int* status_out,
+                                DevCounters* ctr_out, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    count_launches(1);
+    gather_state_kernel<<<(n + 255) / 256, 256, 0, st>>>(refs, n, status_out, ctr_out);
     return cudaGetLastError();
 }
 

@@ -76,7 +76,7 @@ __device__ inline float acc_round(const unsigned int* mag, bool negative) {
     // M <= 2^24; value = M * 2^(lsb - kAccBase), exact in binary64
     double v = (double)M * pow2d(lsb - kAccBase);
     float f = __double2float_rn(v);   // exact when representable; inf on overflow
-    return negative ? -f : f;
+    return (negative && f != 0.0f) ? -f : f;   // a result that rounds to zero is +0
 }
 
 // Products q_j * v_j of one lane, visited in a fixed order: float4 loads for
@@ -158,6 +158,114 @@ __device__ inline float exact_dot_warp_impl(const float* __restrict__ q,
 __device__ inline float exact_dot_warp(const float* __restrict__ q, const float* __restrict__ v,
                                        int m_raw, bool* used_fallback) {
     return exact_dot_warp_impl<true>(q, v, m_raw, used_fallback);
+}
+
+// Fast form on the float32 pipe (binary64 throughput is a small fraction of
+// float32 throughput on this part).  Error-free transformations (Knuth's
+// TwoSum; TwoProduct with one fused multiply-add, as in Ogita, Rump and Oishi,
+// "Accurate sum and dot product", 2005) split every product and every partial
+// sum of the main accumulator s into its rounded value and exact error; the
+// errors are summed in float32 into c.  Bookkeeping that makes the result
+// rigorous for any summation order:
+//   * exact = s + (sum of all error terms) + d, where |d| <= m 2^-150 covers
+//     the only inexact step, a TwoProduct error term that underflows;
+//   * every float32 addition of the error sum satisfies x + y = fl(x + y)(1 + e)
+//     with |e| <= 2^-24, so |c - sum of error terms| <= 2^-24 sum |fl(node)|
+//     over the additions that built c; a holds that sum rounded upward.
+// The enclosure [RD(s + c - beta), RU(s + c + beta)] with beta = 2^-24 a +
+// m 2^-150 is formed in binary64 once per row; when it rounds to one float32
+// value that value is the answer, otherwise exact_dot_warp decides.
+// Out of line so that the rare ambiguous case does not cost the fast loop
+// registers.
+static __device__ __noinline__ float exact_dot_warp_slow(const float* __restrict__ q,
+                                                  const float* __restrict__ v, int m_raw,
+                                                  bool* used_fallback) {
+    return exact_dot_warp_impl<true>(q, v, m_raw, used_fallback);
+}
+
+__device__ inline void two_sum_f(float a, float b, float& s, float& e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+struct EftAcc {
+    float s = 0.0f, c = 0.0f, a1 = 0.0f, a2 = 0.0f;
+    __device__ inline void add_product(float x, float y) {
+        const float p = __fmul_rn(x, y);
+        const float ep = __fmaf_rn(x, y, -p);
+        float es;
+        two_sum_f(s, p, s, es);
+        const float t = __fadd_rn(ep, es);
+        c = __fadd_rn(c, t);
+        a1 = __fadd_ru(a1, fabsf(t));
+        a2 = __fadd_ru(a2, fabsf(c));
+    }
+    // Merge another lane's accumulator (commutative: every lane of a butterfly
+    // ends with the same bits).
+    __device__ inline void merge(float s2, float c2, float a12, float a22) {
+        float es;
+        two_sum_f(s, s2, s, es);
+        const float cc = __fadd_rn(c, c2);
+        const float c3 = __fadd_rn(cc, es);
+        a1 = __fadd_ru(__fadd_ru(a1, a12), fabsf(cc));
+        a2 = __fadd_ru(__fadd_ru(a2, a22), fabsf(c3));
+        c = c3;
+    }
+};
+
+// Index rows: 16-byte aligned, m_raw a multiple of 4 (zero padded).
+__device__ inline float exact_dot_warp_eft(const float* __restrict__ q,
+                                           const float* __restrict__ v, int m_raw,
+                                           bool* used_fallback) {
+    const int lane = threadIdx.x & 31;
+    const float4* q4 = reinterpret_cast<const float4*>(q);
+    const float4* v4 = reinterpret_cast<const float4*>(v);
+    EftAcc acc;
+    constexpr int kBatch = 4;   // float4 pairs a lane has in flight
+    const int n4 = m_raw >> 2;
+#pragma unroll 1
+    for (int j0 = lane; j0 < n4; j0 += kWarp * kBatch) {
+        float4 x[kBatch], y[kBatch];
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int j = j0 + kWarp * b;
+            if (j < n4) {
+                x[b] = __ldg(q4 + j);
+                y[b] = __ldg(v4 + j);
+            } else {
+                x[b] = y[b] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            acc.add_product(x[b].x, y[b].x);
+            acc.add_product(x[b].y, y[b].y);
+            acc.add_product(x[b].z, y[b].z);
+            acc.add_product(x[b].w, y[b].w);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float s2 = __shfl_xor_sync(0xffffffffu, acc.s, off);
+        const float c2 = __shfl_xor_sync(0xffffffffu, acc.c, off);
+        const float a12 = __shfl_xor_sync(0xffffffffu, acc.a1, off);
+        const float a22 = __shfl_xor_sync(0xffffffffu, acc.a2, off);
+        acc.merge(s2, c2, a12, a22);
+    }
+    if (isfinite(acc.s) && isfinite(acc.c)) {
+        const double a = __dadd_ru((double)acc.a1, (double)acc.a2);
+        const double beta = __dadd_ru(a * 0x1p-24, (double)m_raw * 0x1p-150);
+        const double sc_lo = __dadd_rd((double)acc.s, (double)acc.c);
+        const double sc_hi = __dadd_ru((double)acc.s, (double)acc.c);
+        const float flo = __double2float_rn(__dsub_rd(sc_lo, beta));
+        const float fhi = __double2float_rn(__dadd_ru(sc_hi, beta));
+        if (flo == fhi) {
+            *used_fallback = false;
+            return flo == 0.0f ? 0.0f : flo;
+        }
+    }
+    return exact_dot_warp_slow(q, v, m_raw, used_fallback);
 }
 
 // Any row of m float32 values.

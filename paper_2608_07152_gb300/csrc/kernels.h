@@ -39,6 +39,12 @@ struct DevCounters {
     unsigned long long cand_total;   // candidates over fused pulls
 };
 
+// Where one cursor keeps its device status word and counters.
+struct CursorRef {
+    const int* status;
+    const DevCounters* ctr;
+};
+
 // ---- fused single-CTA pull (pull_kernel.cu) ----------------------------------
 constexpr int kPullFusedMax = 256;   // largest pull served by one fused launch
 struct PullArgs {
@@ -74,10 +80,12 @@ struct WsDst {                       // a cursor's working-set arrays
     float* w_hi;
     unsigned int* w_len;
 };
-struct QueryDst {                    // a cursor's query buffers
+struct QueryDst {                    // a cursor's query buffers and fresh device state
     int8_t* zq;
     float* qraw;
     QueryScalars* qs;
+    DevCounters* ctr;                // zeroed by the copy
+    int* status;                     // zeroed by the copy
 };
 cudaError_t launch_batch_tau(const float* dump_lo, int64_t ld, unsigned int nsample, int nq,
                              unsigned int k, float* tau, cudaStream_t st);
@@ -191,6 +199,9 @@ struct BatchArgs {
 };
 cudaError_t launch_batch_intervals(const BatchArgs& a, const uint16_t* codes_bf16,
                                    const uint16_t* qcodes_bf16, int num_sms, cudaStream_t st);
+// status_out[i] = *refs[i].status; ctr_out[i] = *refs[i].ctr (ctr_out may be null).
+cudaError_t launch_gather_state(const CursorRef* refs, int n, int* status_out,
+                                DevCounters* ctr_out, cudaStream_t st);
 cudaError_t launch_codes_to_bf16(const int8_t* src, uint16_t* dst, int64_t count,
                                  cudaStream_t st);
 

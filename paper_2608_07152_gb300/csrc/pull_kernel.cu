@@ -296,13 +296,16 @@ struct RowKeys {   // live lower bounds of one query's dump row
 
 // One CTA per query: tau[q] = k-th largest live lower bound among the sampled
 // rows (dump row q), or -inf if fewer than k are live.
-__global__ void __launch_bounds__(kPullThreads, 2) batch_tau_kernel(const float* dump_lo,
-                                                                    int64_t ld,
-                                                                    unsigned int nsample,
-                                                                    unsigned int k, float* tau) {
-    __shared__ PullShared sh;
-    const int q = blockIdx.x, t = threadIdx.x;
-    const RowKeys src{dump_lo + (int64_t)q * ld};
+//   1. every thread takes the maximum key of its share of the row (float4
+//      loads, several in flight); the k-th largest of these maxima, t0, is a
+//      lower bound of the answer: k threads each hold a value >= t0;
+//   2. the values >= t0 (usually a few times k) are gathered into shared
+//      memory and sorted; the k-th of them is the answer.
+// When k exceeds the thread count, fewer than k threads saw a live value, or
+// more than kPullSortCap values reach t0, a three-pass radix select decides.
+__device__ inline void tau_radix(PullShared& sh, const RowKeys& src, unsigned int nsample,
+                                 unsigned int k, float* out) {
+    const int t = threadIdx.x;
     if (t == 0) {
         sh.prefix = 0;
         sh.k = k;
@@ -315,11 +318,74 @@ __global__ void __launch_bounds__(kPullThreads, 2) batch_tau_kernel(const float*
         __syncthreads();
         block_pick_digit(sh, shifts32[p]);
         if (!sh.ok) {
-            if (t == 0) tau[q] = -INFINITY;
+            if (t == 0) *out = -INFINITY;
             return;
         }
     }
-    if (t == 0) tau[q] = fkey_inv((uint32_t)sh.prefix);
+    if (t == 0) *out = fkey_inv((uint32_t)sh.prefix);
+}
+
+__global__ void __launch_bounds__(kPullThreads, 2) batch_tau_kernel(const float* dump_lo,
+                                                                    int64_t ld,
+                                                                    unsigned int nsample,
+                                                                    unsigned int k, float* tau) {
+    __shared__ PullShared sh;
+    const int q = blockIdx.x, t = threadIdx.x;
+    const float* row = dump_lo + (int64_t)q * ld;
+    const RowKeys src{row};
+    if (k == 0 || k > (unsigned int)kPullThreads) {
+        tau_radix(sh, src, nsample, k, &tau[q]);
+        return;
+    }
+    // 1. per-thread maxima (key 0: no live value; every live key is larger)
+    const unsigned int n4 = nsample >> 2;
+    const float4* row4 = reinterpret_cast<const float4*>(row);
+    auto live_key = [](float v) -> uint32_t { return v == -INFINITY ? 0u : fkey(v); };
+    uint32_t mx = 0;
+#pragma unroll 4
+    for (unsigned int i = t; i < n4; i += kPullThreads) {
+        const float4 v = __ldg(row4 + i);
+        mx = max(mx, max(max(live_key(v.x), live_key(v.y)), max(live_key(v.z), live_key(v.w))));
+    }
+    for (unsigned int i = 4 * n4 + t; i < nsample; i += kPullThreads) mx = max(mx, live_key(row[i]));
+    sh.sk[t] = ((unsigned long long)mx << 32) | (unsigned int)t;
+    __syncthreads();
+    bitonic_desc_smem(sh.sk, kPullThreads);
+    const uint32_t t0 = (uint32_t)(sh.sk[k - 1] >> 32);
+    __syncthreads();
+    if (t0 == 0) {   // fewer than k threads saw a live value
+        tau_radix(sh, src, nsample, k, &tau[q]);
+        return;
+    }
+    // 2. gather the values >= t0
+    if (t == 0) sh.count = 0;
+    __syncthreads();
+    auto take = [&](float v) {
+        const uint32_t key = live_key(v);
+        if (key >= t0) {
+            const unsigned int pos = atomicAdd(&sh.count, 1u);
+            if (pos < (unsigned int)kPullSortCap) sh.sk[pos] = (unsigned long long)key << 32;
+        }
+    };
+#pragma unroll 4
+    for (unsigned int i = t; i < n4; i += kPullThreads) {
+        const float4 v = __ldg(row4 + i);
+        take(v.x), take(v.y), take(v.z), take(v.w);
+    }
+    for (unsigned int i = 4 * n4 + t; i < nsample; i += kPullThreads) take(row[i]);
+    __syncthreads();
+    const unsigned int cnt = sh.count;
+    if (cnt > (unsigned int)kPullSortCap) {
+        __syncthreads();
+        tau_radix(sh, src, nsample, k, &tau[q]);
+        return;
+    }
+    int pow2 = 1;
+    while (pow2 < (int)cnt) pow2 <<= 1;
+    for (int i = (int)cnt + t; i < pow2; i += kPullThreads) sh.sk[i] = 0ull;
+    __syncthreads();
+    bitonic_desc_smem(sh.sk, pow2);
+    if (t == 0) tau[q] = fkey_inv((uint32_t)(sh.sk[k - 1] >> 32));
 }
 
 cudaError_t launch_batch_tau(const float* dump_lo, int64_t ld, unsigned int nsample, int nq,

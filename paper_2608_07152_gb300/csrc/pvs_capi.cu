@@ -485,12 +485,16 @@ constexpr int kBatchMax = 256;
 // Stream-ordered scratch that is released (stream-ordered) at scope exit.
 struct DevBuf {
     cudaStream_t st = nullptr;
+    cudaMemPool_t pool = nullptr;
     std::vector<void*> ptrs;
-    explicit DevBuf(cudaStream_t s = nullptr) : st(s) {}
+    DevBuf(cudaStream_t s, cudaMemPool_t p) : st(s), pool(p) {}
     template <typename T>
     T* get(size_t count) {
         void* p = nullptr;
-        if (cudaMallocAsync(&p, std::max<size_t>(count, 1) * sizeof(T), st) != cudaSuccess) {
+        const size_t bytes = std::max<size_t>(count, 1) * sizeof(T);
+        const cudaError_t e = pool ? cudaMallocFromPoolAsync(&p, bytes, pool, st)
+                                   : cudaMallocAsync(&p, bytes, st);
+        if (e != cudaSuccess) {
             cudaGetLastError();
             return nullptr;
         }
@@ -501,6 +505,60 @@ struct DevBuf {
         for (void* p : ptrs) cudaFreeAsync(p, st);
     }
 };
+
+// Status words (and, if ctr is given, counters) of n cursors that share
+// stream st: one gather launch, one copy back, one synchronisation.
+pvs_status gather_state(pvs_cursor* const* cs, int n, cudaStream_t st, int* status,
+                        DevCounters* ctr) {
+    if (n <= 0) return PVS_OK;
+    DevBuf buf(st, cs[0]->index->scratch_pool);
+    CursorRef* d_refs = buf.get<CursorRef>((size_t)n);
+    int* d_status = buf.get<int>((size_t)n);
+    DevCounters* d_ctr = ctr ? buf.get<DevCounters>((size_t)n) : nullptr;
+    if (!d_refs || !d_status || (ctr && !d_ctr)) return PVS_ERR_OOM;
+    std::vector<CursorRef> refs((size_t)n);
+    for (int i = 0; i < n; ++i) refs[(size_t)i] = CursorRef{cs[i]->d_status, cs[i]->ctr};
+    PVS_CUDA(cudaMemcpyAsync(d_refs, refs.data(), (size_t)n * sizeof(CursorRef),
+                             cudaMemcpyHostToDevice, st));
+    PVS_CUDA(launch_gather_state(d_refs, n, d_status, d_ctr, st));
+    PVS_CUDA(cudaMemcpyAsync(status, d_status, (size_t)n * sizeof(int), cudaMemcpyDeviceToHost,
+                             st));
+    if (ctr)
+        PVS_CUDA(cudaMemcpyAsync(ctr, d_ctr, (size_t)n * sizeof(DevCounters),
+                                 cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaStreamSynchronize(st));
+    return PVS_OK;
+}
+
+// gather_state over cursors on any mix of streams: one round per stream.
+pvs_status gather_state_any(pvs_cursor* const* cs, int n, int* status, DevCounters* ctr) {
+    std::vector<cudaStream_t> streams;
+    for (int i = 0; i < n; ++i)
+        if (std::find(streams.begin(), streams.end(), cs[i]->stream) == streams.end())
+            streams.push_back(cs[i]->stream);
+    std::vector<pvs_cursor*> group;
+    std::vector<int> where, g_status;
+    std::vector<DevCounters> g_ctr;
+    for (cudaStream_t st : streams) {
+        group.clear();
+        where.clear();
+        for (int i = 0; i < n; ++i)
+            if (cs[i]->stream == st) {
+                group.push_back(cs[i]);
+                where.push_back(i);
+            }
+        g_status.assign(group.size(), 0);
+        g_ctr.assign(ctr ? group.size() : 0, DevCounters{});
+        pvs_status s = gather_state(group.data(), (int)group.size(), st, g_status.data(),
+                                    ctr ? g_ctr.data() : nullptr);
+        if (s != PVS_OK) return s;
+        for (size_t j = 0; j < group.size(); ++j) {
+            status[where[j]] = g_status[j];
+            if (ctr) ctr[where[j]] = g_ctr[j];
+        }
+    }
+    return PVS_OK;
+}
 
 struct BatchQueries {
     int nq = 0, nq_pad = 0;
@@ -526,8 +584,11 @@ pvs_status ensure_bf16(pvs_index* x) {
 }
 
 // Encode nq queries on the index stream; checks their status (waits).
+// Encode nq queries for the batched pass.  With check_now the call waits and
+// reports a non-finite query; otherwise the caller reads bq->qs[i].status
+// later, at its own synchronisation point.
 pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_device, DevBuf& buf,
-                        BatchQueries* bq) {
+                        BatchQueries* bq, bool check_now = true) {
     cudaStream_t st = x->stream;
     bq->nq = nq;
     bq->nq_pad = (int)round_up(nq, 32);
@@ -552,6 +613,7 @@ pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_devi
         pvs_status s = ensure_bf16(x);
         if (s != PVS_OK) return s;
     }
+    if (!check_now) return PVS_OK;
     std::vector<QueryScalars> h(nq);
     PVS_CUDA(cudaMemcpyAsync(h.data(), bq->qs, nq * sizeof(QueryScalars), cudaMemcpyDeviceToHost,
                              st));
@@ -562,7 +624,10 @@ pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_devi
 }
 
 // A cursor with its small buffers, fresh counters and the given snapshot.
-pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs_cursor** out) {
+// With zero_state false the caller zeroes the counters and status word on the
+// device itself (the batched open does it in its query copy).
+pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs_cursor** out,
+                          bool zero_state = true) {
     pvs_cursor* c = nullptr;
     {
         std::lock_guard<std::mutex> lock(x->pool_mutex);
@@ -590,8 +655,10 @@ pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs
          dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
          cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess))
         return PVS_ERR_OOM;
-    PVS_CUDA(cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), c->stream));
-    PVS_CUDA(cudaMemsetAsync(c->d_status, 0, sizeof(int), c->stream));
+    if (zero_state) {
+        PVS_CUDA(cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), c->stream));
+        PVS_CUDA(cudaMemsetAsync(c->d_status, 0, sizeof(int), c->stream));
+    }
     c->state = c->visible == 0 ? PVS_EXHAUSTED : PVS_OK;
     return PVS_OK;
 }
@@ -613,25 +680,35 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
                             const float* queries, int nq, bool on_device, int horizon,
                             pvs_cursor** out) {
     cudaStream_t st = x->stream;
-    DevBuf buf(st);
+    DevBuf buf(st, x->scratch_pool);
     BatchQueries bq;
-    pvs_status s = encode_batch(x, queries, nq, on_device, buf, &bq);
+    // one synchronisation at the end: query statuses are read with the pass's
+    pvs_status s = encode_batch(x, queries, nq, on_device, buf, &bq, /*check_now=*/false);
     if (s != PVS_OK) return s;
     for (int i = 0; i < nq; ++i) {
-        s = acquire_cursor(x, sd, &out[i]);
+        s = acquire_cursor(x, sd, &out[i], /*zero_state=*/false);
         if (s != PVS_OK) return s;
     }
     QueryDst* d_qd = buf.get<QueryDst>((size_t)nq);
     if (!d_qd) return PVS_ERR_OOM;
     {
+        // a pageable source is staged before cudaMemcpyAsync returns
         std::vector<QueryDst> qd(nq);
-        for (int i = 0; i < nq; ++i) qd[i] = QueryDst{out[i]->zq, out[i]->qraw, out[i]->qs};
+        for (int i = 0; i < nq; ++i)
+            qd[i] = QueryDst{out[i]->zq, out[i]->qraw, out[i]->qs, out[i]->ctr, out[i]->d_status};
         PVS_CUDA(cudaMemcpyAsync(d_qd, qd.data(), nq * sizeof(QueryDst), cudaMemcpyHostToDevice, st));
         PVS_CUDA(launch_copy_queries(bq.zq, bq.qraw, bq.qs, d_qd, nq, x->m_pad, x->m_raw, st));
-        PVS_CUDA(cudaStreamSynchronize(st));   // qd (host) is read by the copy above
     }
+    std::vector<QueryScalars> h_qs(nq);
     const int64_t rows = sd->rows;
-    if (rows == 0) return PVS_OK;
+    if (rows == 0) {
+        PVS_CUDA(cudaMemcpyAsync(h_qs.data(), bq.qs, nq * sizeof(QueryScalars),
+                                 cudaMemcpyDeviceToHost, st));
+        PVS_CUDA(cudaStreamSynchronize(st));
+        for (int i = 0; i < nq; ++i)
+            if (h_qs[i].status != 0) return (pvs_status)h_qs[i].status;
+        return PVS_OK;
+    }
 
     // Sample every stride-th tile and take tau_q = the k_s-th largest sampled
     // lower bound, k_s = 1.5 H / stride + 4: about 1.5 H rows of the corpus
@@ -727,11 +804,15 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     PVS_CUDA(cudaMemcpyAsync(h_wlen.data(), wlen, nq * sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaMemcpyAsync(h_heff.data(), heff, nq * sizeof(unsigned int), cudaMemcpyDeviceToHost, st));
     PVS_CUDA(cudaMemcpyAsync(&h_status, status, sizeof(int), cudaMemcpyDeviceToHost, st));
+    PVS_CUDA(cudaMemcpyAsync(h_qs.data(), bq.qs, nq * sizeof(QueryScalars), cudaMemcpyDeviceToHost,
+                             st));
     PVS_CUDA(cudaStreamSynchronize(st));
     float pass_ms = 0.0f;
     cudaEventElapsedTime(&pass_ms, ev0, ev1);
     cudaEventDestroy(ev0);
     cudaEventDestroy(ev1);
+    for (int i = 0; i < nq; ++i)   // a non-finite query fails the batch
+        if (h_qs[i].status != 0) return (pvs_status)h_qs[i].status;
     if (h_status != 0) return (pvs_status)h_status;
     for (int i = 0; i < nq; ++i) {
         pvs_cursor* c = out[i];
@@ -805,6 +886,18 @@ pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_
         x->own_stream = true;
     }
     if (cudaMalloc(&x->d_status, sizeof(int)) != cudaSuccess) return bail(PVS_ERR_OOM);
+    {
+        cudaMemPoolProps props{};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = x->device;
+        if (cudaMemPoolCreate(&x->scratch_pool, &props) != cudaSuccess) {
+            x->scratch_pool = nullptr;
+            return bail(PVS_ERR_CUDA);
+        }
+        uint64_t keep = UINT64_MAX;
+        cudaMemPoolSetAttribute(x->scratch_pool, cudaMemPoolAttrReleaseThreshold, &keep);
+    }
     if (vecs_on_device && n > 0 && !is_device_ptr(vecs)) return bail(PVS_ERR_INVALID);
     pvs_status s = index_reserve(x, n);
     if (s != PVS_OK) return bail(s);
@@ -879,6 +972,7 @@ void pvs_index_free(pvs_index* x) {
     dev_free(x->codes), dev_free(x->scale), dev_free(x->vnorm), dev_free(x->enorm);
     dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage), dev_free(x->codes_bf16);
     if (x->pass_done) cudaEventDestroy(x->pass_done);
+    if (x->scratch_pool) cudaMemPoolDestroy(x->scratch_pool);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
 }
@@ -992,7 +1086,7 @@ pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float*
     const int64_t rows = sd->rows;
     if (rows == 0) return PVS_OK;
     cudaStream_t st = x->stream;
-    DevBuf buf(st);
+    DevBuf buf(st, x->scratch_pool);
     BatchQueries bq;
     pvs_status s = encode_batch(x, queries, nq, queries_on_device, buf, &bq);
     if (s != PVS_OK) return s;
@@ -1058,7 +1152,7 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         }
         return worst;
     }
-    DevBuf buf(st);   // released in stream order after the launches that read it
+    DevBuf buf(st, x->scratch_pool);   // released in stream order after the launches that read it
     int64_t* d_ids = outputs_on_device ? ids : buf.get<int64_t>((size_t)nc * n);
     float* d_scores = outputs_on_device ? scores : buf.get<float>((size_t)nc * n);
     PullArgs* d_args = buf.get<PullArgs>((size_t)nc);
@@ -1108,10 +1202,14 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
                                  cudaMemcpyDeviceToHost, st));
         PVS_CUDA(cudaMemcpyAsync(scores, d_scores, (size_t)nc * n * sizeof(float),
                                  cudaMemcpyDeviceToHost, st));
-        for (int32_t i : who) {
-            pvs_status s = check_device_status(cursors[i]);
-            if (s != PVS_OK) result = s;
-        }
+        std::vector<pvs_cursor*> pulled;
+        for (int32_t i : who) pulled.push_back(cursors[i]);
+        std::vector<int> dev_status(pulled.size(), 0);
+        pvs_status s = gather_state(pulled.data(), (int)pulled.size(), st, dev_status.data(),
+                                    nullptr);
+        if (s != PVS_OK) return s;
+        for (size_t j = 0; j < pulled.size(); ++j)
+            if (dev_status[j] != 0) result = fail(pulled[j], (pvs_status)dev_status[j]);
         if (result != PVS_OK) return result;
     }
     for (int32_t i = 0; i < nc; ++i) {
@@ -1181,14 +1279,8 @@ pvs_status pvs_cursor_sync(pvs_cursor* c) {
     return (pvs_status)c->state;
 }
 
-pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
-    if (!c || !out) return PVS_ERR_INVALID;
+static void fill_stats(pvs_cursor* c, const DevCounters& d, pvs_stats* out) {
     std::memset(out, 0, sizeof(*out));
-    DevCounters d{};
-    cudaError_t e = cudaMemcpyAsync(&d, c->ctr, sizeof(d), cudaMemcpyDeviceToHost, c->stream);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
-    if (e != cudaSuccess) return cuda_status(e);
-    if (c->state >= 0) check_device_status(c);
     out->visible = c->visible;
     out->emitted = c->emitted;
     out->refined = (int64_t)d.refined;
@@ -1203,6 +1295,51 @@ pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
     out->interval_ms = c->interval_ms;
     out->batch_passes = c->batch_passes;
     out->batch_ms = c->batch_ms;
+}
+
+pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
+    if (!c || !out) return PVS_ERR_INVALID;
+    std::memset(out, 0, sizeof(*out));
+    DevCounters d{};
+    cudaError_t e = cudaMemcpyAsync(&d, c->ctr, sizeof(d), cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (c->state >= 0) check_device_status(c);
+    fill_stats(c, d, out);
+    return PVS_OK;
+}
+
+static bool valid_cursor_list(pvs_cursor* const* cs, int32_t nc) {
+    if (!cs || nc < 0) return false;
+    for (int32_t i = 0; i < nc; ++i)
+        if (!cs[i] || !cs[i]->index) return false;
+    return true;
+}
+
+pvs_status pvs_cursor_sync_batch(pvs_cursor** cursors, int32_t nc, int32_t* states) {
+    if (!valid_cursor_list(cursors, nc) || (nc > 0 && !states)) return PVS_ERR_INVALID;
+    std::vector<int> dev_status((size_t)nc, 0);
+    pvs_status s = gather_state_any(cursors, nc, dev_status.data(), nullptr);
+    if (s != PVS_OK) return s;
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        if (c->state >= 0 && dev_status[(size_t)i] != 0) fail(c, (pvs_status)dev_status[(size_t)i]);
+        states[i] = c->state;
+    }
+    return PVS_OK;
+}
+
+pvs_status pvs_cursor_stats_batch(pvs_cursor** cursors, int32_t nc, pvs_stats* out) {
+    if (!valid_cursor_list(cursors, nc) || (nc > 0 && !out)) return PVS_ERR_INVALID;
+    std::vector<int> dev_status((size_t)nc, 0);
+    std::vector<DevCounters> d((size_t)nc, DevCounters{});
+    pvs_status s = gather_state_any(cursors, nc, dev_status.data(), d.data());
+    if (s != PVS_OK) return s;
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        if (c->state >= 0 && dev_status[(size_t)i] != 0) fail(c, (pvs_status)dev_status[(size_t)i]);
+        fill_stats(c, d[(size_t)i], &out[i]);
+    }
     return PVS_OK;
 }
 
@@ -1253,10 +1390,10 @@ pvs_status pvs_cursor_score_ids(pvs_cursor* c, const int64_t* ids, int32_t n, fl
     return cuda_status(e);
 }
 
-void pvs_cursor_close(pvs_cursor* c) {
-    if (!c) return;
+// Return a cursor's buffers to its index's pool (or free them); the caller
+// has waited for the cursor's stream.
+static void release_cursor(pvs_cursor* c) {
     pvs_index* x = c->index;
-    if (x) cudaStreamSynchronize(c->stream);
     harvest_interval_time(c);
     if (x) {
         std::lock_guard<std::mutex> lock(x->pool_mutex);
@@ -1271,6 +1408,27 @@ void pvs_cursor_close(pvs_cursor* c) {
     }
     cursor_free_device(c);
     delete c;
+}
+
+void pvs_cursor_close(pvs_cursor* c) {
+    if (!c) return;
+    if (c->index) cudaStreamSynchronize(c->stream);
+    release_cursor(c);
+}
+
+void pvs_cursor_close_batch(pvs_cursor** cursors, int32_t nc) {
+    if (!cursors || nc <= 0) return;
+    std::vector<cudaStream_t> synced;
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        if (!c || !c->index) continue;
+        if (std::find(synced.begin(), synced.end(), c->stream) == synced.end()) {
+            cudaStreamSynchronize(c->stream);
+            synced.push_back(c->stream);
+        }
+    }
+    for (int32_t i = 0; i < nc; ++i)
+        if (cursors[i]) release_cursor(cursors[i]);
 }
 
 }  // extern "C"

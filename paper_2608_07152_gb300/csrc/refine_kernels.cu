@@ -1,7 +1,7 @@
 // Authoritative float32 scores of PVS candidates (Sec. 2.3.1: raw vectors are
 // read only for candidates the intervals do not order; App. A.1: a score
 // outside its interval fails the request).  The score itself is computed by
-// exact_dot_warp (exact_dot.cuh): RN_f32 of the exact inner product.
+// exact_dot_warp_eft (exact_dot.cuh): RN_f32 of the exact inner product.
 #include "exact_dot.cuh"
 #include "kernels.h"
 #include "pvs_common.cuh"
@@ -10,7 +10,9 @@ namespace pvs {
 
 // Warps warp0, warp0 + nwarps, ... of the launch score candidates of one
 // cursor.  lo / hi (bounds of every row) may be null for a cursor that only
-// holds a working set.
+// holds a working set.  A warp fetches the metadata of its next 32
+// candidates at once (lane j holds candidate j) and broadcasts it with
+// shuffles, so each candidate waits on its row alone.
 __device__ inline void refine_warps(const int32_t* __restrict__ cand, const unsigned int* cand_len,
                                     const int32_t* __restrict__ w_id, float* w_lo, float* w_hi,
                                     float* lo, float* hi, const float* __restrict__ qraw,
@@ -19,23 +21,39 @@ __device__ inline void refine_warps(const int32_t* __restrict__ cand, const unsi
     const int lane = threadIdx.x & 31;
     const int64_t n = *cand_len;
     unsigned long long refined = 0, fallbacks = 0;
-    for (int64_t i = warp0; i < n; i += nwarps) {
-        const int32_t w = cand[i];
-        const float l = w_lo[w], h = w_hi[w];
-        if (!(l < h)) continue;    // resolved: lo == hi is the exact score
-        const int32_t id = w_id[w];
-        bool fb;
-        const float s = exact_dot_warp(qraw, raw + (int64_t)id * m_raw, m_raw, &fb);
-        if (lane == 0) {
-            ++refined;
-            fallbacks += fb;
-            if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
-            else if (s < l || s > h) set_status(status, PVS_ERR_INTERVAL);
-            w_lo[w] = s;
-            w_hi[w] = s;
-            if (lo) {
-                lo[id] = s;
-                hi[id] = s;
+#pragma unroll 1
+    for (int64_t base = warp0; base < n; base += 32 * nwarps) {
+        const int64_t mine = base + lane * nwarps;
+        int32_t w = 0, id = 0;
+        float l = 0.0f, h = 0.0f;   // l == h: nothing to do
+        if (mine < n) {
+            w = cand[mine];
+            l = w_lo[w];
+            h = w_hi[w];
+            id = w_id[w];
+        }
+        const int64_t left = (n - base + nwarps - 1) / nwarps;   // candidates of this warp left
+        const int cnt = left < 32 ? (int)left : 32;
+#pragma unroll 1
+        for (int j = 0; j < cnt; ++j) {
+            const float lj = __shfl_sync(0xffffffffu, l, j);
+            const float hj = __shfl_sync(0xffffffffu, h, j);
+            const int32_t wj = __shfl_sync(0xffffffffu, w, j);
+            const int32_t idj = __shfl_sync(0xffffffffu, id, j);
+            if (!(lj < hj)) continue;    // resolved: lo == hi is the exact score
+            bool fb;
+            const float s = exact_dot_warp_eft(qraw, raw + (int64_t)idj * m_raw, m_raw, &fb);
+            if (lane == 0) {
+                ++refined;
+                fallbacks += fb;
+                if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
+                else if (s < lj || s > hj) set_status(status, PVS_ERR_INTERVAL);
+                w_lo[wj] = s;
+                w_hi[wj] = s;
+                if (lo) {
+                    lo[idj] = s;
+                    hi[idj] = s;
+                }
             }
         }
     }
@@ -91,7 +109,7 @@ __global__ void score_ids_kernel(const int64_t* ids, int n, const float* qraw, c
     const int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (i >= n) return;
     bool fb;
-    const float s = exact_dot_warp(qraw, raw + ids[i] * m_raw, m_raw, &fb);
+    const float s = exact_dot_warp_eft(qraw, raw + ids[i] * m_raw, m_raw, &fb);
     if (lane == 0) {
         out[i] = s;
         if (fb) atomicAdd(&ctr->exact_fallbacks, 1ull);

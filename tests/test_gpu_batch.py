@@ -101,3 +101,57 @@ def test_open_batch_groups_snapshots_and_device_outputs():
     finally:
         pvs.pvs_snapshot_free(snap)
         pvs.pvs_index_free(index)
+
+
+def test_batch_sync_stats_and_close_agree_with_per_cursor_calls():
+    V, Q = _mixture(4_000, 96, 40, seed=21, comps=16)
+    index = pvs.pvs_build(V)
+    side = torch.cuda.Stream()
+    try:
+        curs = pvs.pvs_cursor_open_batch(index, Q, horizon=30)
+        ids, sc, n_out = pvs.pvs_next_batch(curs, 25)
+        assert all(n_out == 25)
+        # two cursors move to another stream: the batch helpers group by stream
+        for c in curs[:2]:
+            pvs.pvs_cursor_set_stream(c, side)
+        for c in curs[:2]:
+            i2, s2, n2 = pvs.pvs_next(c, 10)
+        states = pvs.pvs_cursor_sync_batch(curs)
+        assert list(states) == [pvs.pvs_cursor_sync(c) for c in curs]
+        assert all(s == pvs.PVS_OK for s in states)
+        many = pvs.pvs_cursor_stats_batch(curs)
+        one = [pvs.pvs_cursor_stats(c) for c in curs]
+        for a, b in zip(many, one):
+            for key in ("visible", "emitted", "refined", "exact_fallbacks", "pulls",
+                        "candidates", "state", "batch_passes"):
+                assert a[key] == b[key], key
+        assert [s["emitted"] for s in many[:3]] == [35, 35, 25]
+        for i in (0, 5, 39):
+            ref_ids, ref_sc = po.dense_ranking(Q[i], V, np.ones(len(V), bool))
+            assert np.array_equal(ids[i], ref_ids[:25])
+            assert np.array_equal(sc[i], ref_sc[:25])
+        pvs.pvs_cursor_close_batch(curs)
+        assert len(pvs.pvs_cursor_sync_batch([])) == 0
+        pvs.pvs_cursor_close_batch([])
+    finally:
+        pvs.pvs_index_free(index)
+
+
+def test_open_batch_rejects_a_non_finite_query_and_stays_usable():
+    V, Q = _mixture(2_000, 64, 8, seed=31, comps=8)
+    index = pvs.pvs_build(V)
+    try:
+        bad = Q.copy()
+        bad[5, 3] = np.nan
+        with pytest.raises(pvs.PvsError) as err:
+            pvs.pvs_cursor_open_batch(index, bad, horizon=20)
+        assert err.value.status == pvs.PVS_ERR_NONFINITE
+        curs = pvs.pvs_cursor_open_batch(index, Q, horizon=20)
+        ids, sc, n_out = pvs.pvs_next_batch(curs, 20)
+        for i in range(len(Q)):
+            ref_ids, ref_sc = po.dense_ranking(Q[i], V, np.ones(len(V), bool))
+            assert np.array_equal(ids[i], ref_ids[:20])
+            assert np.array_equal(sc[i], ref_sc[:20])
+        pvs.pvs_cursor_close_batch(curs)
+    finally:
+        pvs.pvs_index_free(index)

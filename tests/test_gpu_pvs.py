@@ -154,6 +154,39 @@ def test_exact_scores_match_oracle_including_halfway_cases():
         pvs.pvs_index_free(index)
 
 
+def test_exact_scores_at_extreme_magnitudes():
+    """Rows whose float32 products overflow (but cancel) or underflow: the
+    float32 error-free path must hand these to the binary64 / exact paths."""
+    m = 64
+    rng = np.random.default_rng(17)
+    big = (rng.standard_normal((60, m)) * 1e10).astype(np.float32)
+    big[:, 0], big[:, 1] = 3e19, -3e19          # products beyond float32 range cancel
+    big[1, 1] = 3e19                            # exact score beyond float32 range: inf
+    big[2, 0] = np.nextafter(np.float32(3e19), np.float32(np.inf))
+    tiny = (rng.standard_normal((60, m)) * 2.0 ** -75).astype(np.float32)
+    tiny[0] = 0.0
+    tiny[0, :3] = 2.0 ** -75
+    V = np.concatenate([big, tiny])
+    qb = (rng.standard_normal(m) * 1e10).astype(np.float32)
+    qb[0] = qb[1] = 3e19
+    qb_c = (rng.standard_normal(m) * 1e19).astype(np.float32)
+    qt = np.zeros(m, np.float32)
+    qt[:3] = 2.0 ** -75
+    qt[3:] = (rng.standard_normal(m - 3) * 2.0 ** -75).astype(np.float32)
+    index = pvs.pvs_build(V)
+    try:
+        for query in (qb, qb_c, qt):
+            cur = pvs.pvs_cursor_open(index, query)
+            try:
+                got = pvs.pvs_cursor_score_ids(cur, np.arange(V.shape[0]))
+            finally:
+                pvs.pvs_cursor_close(cur)
+            ref = po.exact_scores(query, V)
+            assert np.array_equal(got.view(np.uint32), ref.view(np.uint32))
+    finally:
+        pvs.pvs_index_free(index)
+
+
 def test_exact_fallback_path_is_taken_and_exact():
     m = 64
     q = np.zeros(m, np.float32)

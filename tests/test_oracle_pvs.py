@@ -285,6 +285,32 @@ def test_exact_scores_cancellation_is_exactly_zero():
     assert po.exact_scores(q, v[None])[0] == np.float32(1.0)
 
 
+def test_exact_scores_in_the_subnormal_range_and_canonical_zero():
+    """Products below the float32 range: scores are the rational rounding
+    (including subnormal results), and any score that rounds to zero is +0."""
+    rng = np.random.default_rng(11)
+    m = 64
+    V = (rng.standard_normal((80, m)) * 2.0 ** -75).astype(np.float32)
+    q = (rng.standard_normal(m) * 2.0 ** -75).astype(np.float32)
+    s = po.exact_scores(q, V)
+    zeros = 0
+    for i in range(V.shape[0]):
+        want = f32_round_exact(exact_dot(q, V[i]))
+        assert s[i] == want, i
+        assert po.exact_score_one(q, V[i]).view(np.uint32) == s[i].view(np.uint32)
+        if want == 0:
+            zeros += 1
+            assert s[i].view(np.uint32) == 0, i          # +0, never -0
+    assert zeros > 0
+    # exact value -2^-151: rounds to zero from below
+    tiny = np.float32(2.0 ** -75)
+    z = po.exact_scores(np.array([tiny], np.float32), np.array([[-tiny / 2]], np.float32))
+    assert z.view(np.uint32)[0] == 0
+    # 3 * 2^-150 lies between 2^-149 and 2^-148, nearer the latter
+    three = po.exact_score_one(np.full(3, tiny, np.float32), np.full(3, tiny, np.float32))
+    assert three == np.float32(2.0 ** -148)
+
+
 def test_dense_ranking_brute_force_with_ties():
     rng = np.random.default_rng(4)
     base = rng.integers(-2, 3, (6, 5)).astype(np.float32)
