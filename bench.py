@@ -314,6 +314,7 @@ BATCH_COMPONENTS = 1024
 BATCH_Q = 256
 BATCH_RANKS = 200
 BATCH_CHUNK = 50
+BATCH_PIPELINE = 2   # batches in flight, each driven by its own host thread and stream
 BATCH_WORKLOAD = ("batched queries: N=1,000,000 x d=768 Gaussian mixture (1,024 components, "
                   "within std 0.35), 256 concurrent queries per batch, first 200 exact ranks "
                   "per query in chunks of 50")
@@ -328,9 +329,30 @@ def bf16_peak():
         return 1900.0, "fallback"
 
 
+def _run_threads(worker, nthreads):
+    import threading
+    errors = []
+
+    def guarded(k):
+        try:
+            worker(k)
+        except Exception as e:  # surfaced below
+            errors.append(e)
+
+    threads = [threading.Thread(target=guarded, args=(k,)) for k in range(nthreads)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    if errors:
+        raise errors[0]
+
+
 def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     """Batched workload: one step = one batch of 256 queries opened together
-    (one tensor-core interval pass), then 4 batched pulls of 50 ranks."""
+    (one tensor-core interval pass), then 4 batched pulls of 50 ranks.
+    BATCH_PIPELINE host threads drive alternate batches on their own streams,
+    so one batch's pulls overlap the next batch's open."""
     stream = torch.cuda.Stream(device=dev)
     n = BATCH_N if args.n == N_CORPUS else args.n
     index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev,
@@ -338,14 +360,15 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     nb = args.warmup + args.steps
     queries = synth.mixture_queries(nb * BATCH_Q, centres, QUERY_NOISE, seed=5 + 7919 * rank)
     queries = queries.reshape(nb, BATCH_Q, DIM).contiguous()
-    ids_t = torch.empty((BATCH_Q, BATCH_CHUNK), dtype=torch.int64, device=dev)
-    sc_t = torch.empty((BATCH_Q, BATCH_CHUNK), dtype=torch.float32, device=dev)
+    streams = [torch.cuda.Stream(device=dev) for _ in range(BATCH_PIPELINE)]
+    ids_t = torch.empty((BATCH_PIPELINE, BATCH_Q, BATCH_CHUNK), dtype=torch.int64, device=dev)
+    sc_t = torch.empty((BATCH_PIPELINE, BATCH_Q, BATCH_CHUNK), dtype=torch.float32, device=dev)
     torch.cuda.synchronize()
 
-    def step(qb, pass_ms, stats=None):
-        curs = pvs.pvs_cursor_open_batch(index, qb, horizon=BATCH_RANKS)
+    def step(qb, slot, pass_ms, stats=None):
+        curs = pvs.pvs_cursor_open_batch(index, qb, horizon=BATCH_RANKS, stream=streams[slot])
         for _ in range(BATCH_RANKS // BATCH_CHUNK):
-            pvs.pvs_next_batch(curs, BATCH_CHUNK, ids_t, sc_t)
+            pvs.pvs_next_batch(curs, BATCH_CHUNK, ids_t[slot], sc_t[slot])
         if stats is None:
             states = pvs.pvs_cursor_sync_batch(curs)   # one wait for every cursor's status
         else:
@@ -358,8 +381,14 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
             pass_ms.append(pvs.pvs_cursor_stats(curs[0])["batch_ms"])
         pvs.pvs_cursor_close_batch(curs)
 
-    for w in range(args.warmup):
-        step(queries[w], None)
+    def run(batches, pass_ms):
+        def worker(k):
+            torch.cuda.set_device(dev)
+            for b in batches[k::BATCH_PIPELINE]:
+                step(queries[b], k, pass_ms)
+        _run_threads(worker, BATCH_PIPELINE)
+
+    run(list(range(args.warmup)), None)
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
@@ -369,13 +398,18 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     end = torch.cuda.Event(enable_timing=True)
     with ClockSampler(local) as clk:
         start.record(stream)
-        for s in range(args.steps):
-            step(queries[args.warmup + s], pass_ms)
+        for s_ in streams:
+            s_.wait_event(start)
+        run(list(range(args.warmup, nb)), pass_ms)
+        for s_ in streams:                      # join every stream's work
+            done = torch.cuda.Event()
+            done.record(s_)
+            stream.wait_event(done)
         end.record(stream)
         stream.synchronize()
     launches = pvs.pvs_launch_count() - launches0
     stats = []   # per-query counters from one more (untimed) batch of the same queries
-    step(queries[args.warmup], None, stats)
+    step(queries[args.warmup], 0, None, stats)
     elapsed = start.elapsed_time(end) / 1e3
     if pg:
         t = torch.tensor([elapsed], device=dev)
@@ -384,15 +418,21 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     ranks_total = args.steps * BATCH_Q * BATCH_RANKS * world
     value = ranks_total / elapsed
 
-    # e2e: host queries, host outputs
-    qh = [np.ascontiguousarray(queries[args.warmup + s].cpu().numpy()) for s in range(args.steps)]
+    # e2e: host queries, host outputs, the same threads and streams
+    qh = [np.ascontiguousarray(queries[b].cpu().numpy()) for b in range(nb)]
     torch.cuda.synchronize()
+
+    def e2e_worker(k):
+        torch.cuda.set_device(dev)
+        for b in range(args.warmup + k, nb, BATCH_PIPELINE):
+            curs = pvs.pvs_cursor_open_batch(index, qh[b], horizon=BATCH_RANKS,
+                                             stream=streams[k])
+            for _ in range(BATCH_RANKS // BATCH_CHUNK):
+                pvs.pvs_next_batch(curs, BATCH_CHUNK)
+            pvs.pvs_cursor_close_batch(curs)
+
     t0 = time.perf_counter()
-    for s in range(args.steps):
-        curs = pvs.pvs_cursor_open_batch(index, qh[s], horizon=BATCH_RANKS)
-        for _ in range(BATCH_RANKS // BATCH_CHUNK):
-            pvs.pvs_next_batch(curs, BATCH_CHUNK)
-        pvs.pvs_cursor_close_batch(curs)
+    _run_threads(e2e_worker, BATCH_PIPELINE)
     e2e_elapsed = time.perf_counter() - t0
     e2e_value = ranks_total / e2e_elapsed
 
@@ -407,6 +447,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         "data": "synthetic",
         "config": {"workload": BATCH_WORKLOAD, "N": n, "d": DIM, "queries_per_batch": BATCH_Q,
                    "ranks_per_query": BATCH_RANKS, "chunk": BATCH_CHUNK,
+                   "batches_in_flight": BATCH_PIPELINE,
                    "l2": "no flush: each batch pass streams 1.5 GB of bf16 codes (> 129 MB L2)",
                    "parallelism": f"replicas x{world}"},
         "e2e": {"value": e2e_value, "unit": UNIT,

@@ -141,12 +141,15 @@ pvs_status pvs_cursor_open(pvs_index* index, const pvs_snapshot* snap, const flo
  * ranks: `horizon` (>= 1) is the number of ranks it is prepared for; it can
  * usually deliver about three times that many before it needs a
  * single-query interval pass, and later ranks still come out exactly, at the
- * cost of that pass.  out[0..nq-1] receive the cursors; they run on the
- * index's stream.  Errors as pvs_cursor_open; on error no cursor is
- * returned. */
+ * cost of that pass.  The work runs on `cuda_stream` (a cudaStream_t; NULL:
+ * the index's stream), and so do the cursors afterwards: batched opens on
+ * different streams from different threads overlap on the device (their
+ * full passes over the codes still run one at a time).  The call returns
+ * once the cursors are ready.  out[0..nq-1] receive the cursors.  Errors as
+ * pvs_cursor_open; on error no cursor is returned. */
 pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
                                  const float* queries, int32_t nq, int32_t queries_on_device,
-                                 int32_t horizon, pvs_cursor** out);
+                                 int32_t horizon, void* cuda_stream, pvs_cursor** out);
 
 /* The next n ranks of each of nc cursors in one set of launches (all
  * cursors of one index and one stream).  Row i of ids / scores (nc x n,

@@ -84,7 +84,7 @@ def _load() -> ctypes.CDLL:
         "pvs_snapshot_visible": (i64, [P]),
         "pvs_snapshot_free": (None, [P]),
         "pvs_cursor_open": (i32, [P, P, P, i32, pp]),
-        "pvs_cursor_open_batch": (i32, [P, P, P, i32, i32, i32, pp]),
+        "pvs_cursor_open_batch": (i32, [P, P, P, i32, i32, i32, P, pp]),
         "pvs_next": (i32, [P, i32, P, P, P]),
         "pvs_next_device": (i32, [P, i32, P, P, P]),
         "pvs_cursor_sync": (i32, [P]),
@@ -227,14 +227,29 @@ def pvs_cursor_open(index, query, snap=None):
     return out
 
 
-def pvs_cursor_open_batch(index, queries, horizon: int, snap=None):
+class CursorBatch(tuple):
+    """The cursors of a batched open (immutable), with the C array of their
+    handles built once for the batch calls."""
+
+    def __new__(cls, handles):
+        self = super().__new__(cls, [ctypes.c_void_p(h) for h in handles])
+        self._arr = (ctypes.c_void_p * max(len(handles), 1))(*handles)
+        return self
+
+
+def pvs_cursor_open_batch(index, queries, horizon: int, snap=None, stream=None):
+    """Open one cursor per query row -> CursorBatch.  stream: a
+    torch.cuda.Stream or raw cudaStream_t for the open and the cursors (None:
+    the index's stream)."""
     ptr, shape, on_dev, keep = _vec_arg(queries)
     nq = shape[0]
     arr = (ctypes.c_void_p * max(nq, 1))()
+    handle = getattr(stream, "cuda_stream", stream)
     _check(_lib.pvs_cursor_open_batch(index, snap, ptr, nq, on_dev, int(horizon),
+                                      ctypes.c_void_p(handle) if handle else None,
                                       ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))),
            "pvs_cursor_open_batch")
-    return [ctypes.c_void_p(arr[i]) for i in range(nq)]
+    return CursorBatch([arr[i] for i in range(nq)])
 
 
 def pvs_next(cursor, n: int):
@@ -258,6 +273,8 @@ def pvs_next_device(cursor, n: int, ids, scores):
 
 
 def _cursor_array(cursors):
+    if isinstance(cursors, CursorBatch):
+        return cursors._arr
     return (ctypes.c_void_p * max(len(cursors), 1))(
         *[c.value if isinstance(c, ctypes.c_void_p) else c for c in cursors])
 

@@ -172,9 +172,8 @@ __device__ inline float exact_dot_warp(const float* __restrict__ q, const float*
 //   * every float32 addition of the error sum satisfies x + y = fl(x + y)(1 + e)
 //     with |e| <= 2^-24, so |c - sum of error terms| <= 2^-24 sum |fl(node)|
 //     over the additions that built c; a holds that sum rounded upward.
-// The enclosure [RD(s + c - beta), RU(s + c + beta)] with beta = 2^-24 a +
-// m 2^-150 is formed in binary64 once per row; when it rounds to one float32
-// value that value is the answer, otherwise exact_dot_warp decides.
+// The decision is taken in float32 too (below); rows it cannot settle go to
+// the binary64 / exact path.
 // Out of line so that the rare ambiguous case does not cost the fast loop
 // registers.
 static __device__ __noinline__ float exact_dot_warp_slow(const float* __restrict__ q,
@@ -214,37 +213,13 @@ struct EftAcc {
     }
 };
 
-// Index rows: 16-byte aligned, m_raw a multiple of 4 (zero padded).
-__device__ inline float exact_dot_warp_eft(const float* __restrict__ q,
-                                           const float* __restrict__ v, int m_raw,
-                                           bool* used_fallback) {
-    const int lane = threadIdx.x & 31;
-    const float4* q4 = reinterpret_cast<const float4*>(q);
-    const float4* v4 = reinterpret_cast<const float4*>(v);
-    EftAcc acc;
-    constexpr int kBatch = 4;   // float4 pairs a lane has in flight
-    const int n4 = m_raw >> 2;
-#pragma unroll 1
-    for (int j0 = lane; j0 < n4; j0 += kWarp * kBatch) {
-        float4 x[kBatch], y[kBatch];
-#pragma unroll
-        for (int b = 0; b < kBatch; ++b) {
-            const int j = j0 + kWarp * b;
-            if (j < n4) {
-                x[b] = __ldg(q4 + j);
-                y[b] = __ldg(v4 + j);
-            } else {
-                x[b] = y[b] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-            }
-        }
-#pragma unroll
-        for (int b = 0; b < kBatch; ++b) {
-            acc.add_product(x[b].x, y[b].x);
-            acc.add_product(x[b].y, y[b].y);
-            acc.add_product(x[b].z, y[b].z);
-            acc.add_product(x[b].w, y[b].w);
-        }
-    }
+// Butterfly merge of the lanes' accumulators, then the float32 decision:
+// r = RN(s + c) with its exact error e2 (TwoSum), so exact = r + e2 + d with
+// |d| <= 2^-24 a + m 2^-149 (the error-sum and underflow bounds, rounded up).
+// Within half the gap around r on either side (a quarter of an ulp below a
+// power of two) the nearest float32 is r.  Returns false when that does not
+// settle the row (then the binary64 / exact path must).
+__device__ inline bool eft_finish(EftAcc acc, int m_raw, float* out) {
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
         const float s2 = __shfl_xor_sync(0xffffffffu, acc.s, off);
@@ -253,17 +228,84 @@ __device__ inline float exact_dot_warp_eft(const float* __restrict__ q,
         const float a22 = __shfl_xor_sync(0xffffffffu, acc.a2, off);
         acc.merge(s2, c2, a12, a22);
     }
-    if (isfinite(acc.s) && isfinite(acc.c)) {
-        const double a = __dadd_ru((double)acc.a1, (double)acc.a2);
-        const double beta = __dadd_ru(a * 0x1p-24, (double)m_raw * 0x1p-150);
-        const double sc_lo = __dadd_rd((double)acc.s, (double)acc.c);
-        const double sc_hi = __dadd_ru((double)acc.s, (double)acc.c);
-        const float flo = __double2float_rn(__dsub_rd(sc_lo, beta));
-        const float fhi = __double2float_rn(__dadd_ru(sc_hi, beta));
-        if (flo == fhi) {
-            *used_fallback = false;
-            return flo == 0.0f ? 0.0f : flo;
+    float r, e2;
+    two_sum_f(acc.s, acc.c, r, e2);
+    const float ar = fabsf(r);
+    if (!(ar >= 0x1p-100f && ar <= 0x1p+126f && isfinite(acc.c))) return false;
+    const float a = __fadd_ru(acc.a1, acc.a2);
+    const float bound = __fadd_ru(fabsf(e2), __fadd_ru(__fmul_ru(a, 0x1p-24f),
+                                                       __fmul_ru((float)m_raw, 0x1p-149f)));
+    const unsigned int bits = __float_as_uint(ar);
+    const float ulp = __uint_as_float(bits & 0x7f800000u) * 0x1p-23f;
+    const float half_gap = (bits & 0x007fffffu) ? ulp * 0.5f : ulp * 0.25f;
+    if (!(bound < half_gap)) return false;
+    *out = r;
+    return true;
+}
+
+// Index rows: 16-byte aligned, m_raw a multiple of 4 (zero padded).  q_fast
+// holds the same values as q and may point to shared memory (it is read with
+// generic loads); q (global) serves the out-of-line exact path.  Up to
+// kBatch float4 of the row are in flight per lane: a row of up to
+// 4 * 32 * kBatch values costs one round trip to memory.
+__device__ inline float exact_dot_warp_eft(const float* q_fast, const float* __restrict__ q,
+                                           const float* __restrict__ v, int m_raw,
+                                           bool* used_fallback) {
+    const int lane = threadIdx.x & 31;
+    const float4* q4 = reinterpret_cast<const float4*>(q_fast);
+    const float4* v4 = reinterpret_cast<const float4*>(v);
+    EftAcc acc;
+    constexpr int kBatch = 8;
+    const int n4 = m_raw >> 2;
+#pragma unroll 1
+    for (int j0 = lane; j0 < n4; j0 += kWarp * kBatch) {
+        float4 y[kBatch];
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int j = j0 + kWarp * b;
+            y[b] = j < n4 ? __ldg(v4 + j) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         }
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int j = j0 + kWarp * b;
+            if (j < n4) {
+                const float4 x = q4[j];
+                acc.add_product(x.x, y[b].x);
+                acc.add_product(x.y, y[b].y);
+                acc.add_product(x.z, y[b].z);
+                acc.add_product(x.w, y[b].w);
+            }
+        }
+    }
+    float r;
+    if (eft_finish(acc, m_raw, &r)) {
+        *used_fallback = false;
+        return r;
+    }
+    return exact_dot_warp_slow(q, v, m_raw, used_fallback);
+}
+
+// The same score with the row already in shared memory (v_sh, generic loads);
+// v (global) is the same row for the exact path.
+__device__ inline float exact_dot_warp_eft_smem(const float* q_fast, const float* __restrict__ q,
+                                                const float* v_sh, const float* __restrict__ v,
+                                                int m_raw, bool* used_fallback) {
+    const int lane = threadIdx.x & 31;
+    const float4* q4 = reinterpret_cast<const float4*>(q_fast);
+    const float4* v4 = reinterpret_cast<const float4*>(v_sh);
+    EftAcc acc;
+    const int n4 = m_raw >> 2;
+    for (int j = lane; j < n4; j += kWarp) {
+        const float4 x = q4[j], y = v4[j];
+        acc.add_product(x.x, y.x);
+        acc.add_product(x.y, y.y);
+        acc.add_product(x.z, y.z);
+        acc.add_product(x.w, y.w);
+    }
+    float r;
+    if (eft_finish(acc, m_raw, &r)) {
+        *used_fallback = false;
+        return r;
     }
     return exact_dot_warp_slow(q, v, m_raw, used_fallback);
 }

@@ -68,9 +68,9 @@ struct PullArgs {
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
 // Many cursors at once (args_dev: device array of ncursors PullArgs).
 cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
-                              cudaStream_t st);
+                              int m_raw, cudaStream_t st);
 cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
-                                cudaStream_t st);
+                                int m_raw, cudaStream_t st);
 
 // ---- batched open support (pull_kernel.cu, batch_support.cu) ----------------
 constexpr int kWsSortMax = 8192;     // largest per-query working set of a batched open

@@ -55,6 +55,12 @@ __device__ inline bool mbar_wait(uint64_t* bar, uint32_t parity) {
     }
 }
 
+// Order this thread's earlier generic-proxy accesses of shared memory (and
+// those of the threads it synchronised with) before its later bulk copies.
+__device__ inline void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ inline uint64_t l2_evict_first_policy() {
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));

@@ -447,13 +447,13 @@ cudaError_t launch_ws_sort(const int32_t* w_id_b, const float* w_lo_b, const flo
 }
 
 cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
-                              cudaStream_t st) {
+                              int m_raw, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
     count_launches(1);
     pull_select_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    e = launch_refine_batch(args_dev, ncursors, refine_blocks_per_cursor, st);
+    e = launch_refine_batch(args_dev, ncursors, refine_blocks_per_cursor, m_raw, st);
     if (e != cudaSuccess) return e;
     count_launches(1);
     pull_emit_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);

@@ -568,17 +568,23 @@ struct BatchQueries {
     uint16_t* qcodes = nullptr;    // [nq_pad][m_pad] bf16, zero rows past nq
 };
 
-// bf16 copy of every code row (the tensor-core pass reads it).
-pvs_status ensure_bf16(pvs_index* x) {
+// bf16 copy of every code row (the tensor-core pass reads it), extended on
+// stream st; st then waits for the last conversion, whichever stream ran it.
+// Caller holds x->pass_mutex.
+pvs_status ensure_bf16(pvs_index* x, cudaStream_t st) {
     if (!x->codes_bf16) {
         PVS_CUDA(dev_alloc(&x->codes_bf16, (size_t)std::max<int64_t>(x->cap, 1) * x->m_pad));
         x->bf16_rows = 0;
     }
+    if (!x->bf16_ready) PVS_CUDA(cudaEventCreateWithFlags(&x->bf16_ready, cudaEventDisableTiming));
     if (x->bf16_rows < x->size) {
         const int64_t r0 = x->bf16_rows;
         PVS_CUDA(launch_codes_to_bf16(x->codes + r0 * x->m_pad, x->codes_bf16 + r0 * x->m_pad,
-                                      (x->size - r0) * x->m_pad, x->stream));
+                                      (x->size - r0) * x->m_pad, st));
         x->bf16_rows = x->size;
+        PVS_CUDA(cudaEventRecord(x->bf16_ready, st));
+    } else {
+        PVS_CUDA(cudaStreamWaitEvent(st, x->bf16_ready, 0));
     }
     return PVS_OK;
 }
@@ -588,8 +594,7 @@ pvs_status ensure_bf16(pvs_index* x) {
 // reports a non-finite query; otherwise the caller reads bq->qs[i].status
 // later, at its own synchronisation point.
 pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_device, DevBuf& buf,
-                        BatchQueries* bq, bool check_now = true) {
-    cudaStream_t st = x->stream;
+                        BatchQueries* bq, cudaStream_t st, bool check_now = true) {
     bq->nq = nq;
     bq->nq_pad = (int)round_up(nq, 32);
     bq->zq = buf.get<int8_t>((size_t)nq * x->m_pad);
@@ -610,7 +615,7 @@ pvs_status encode_batch(pvs_index* x, const float* queries, int nq, bool on_devi
     PVS_CUDA(launch_codes_to_bf16(bq->zq, bq->qcodes, (int64_t)nq * x->m_pad, st));
     {
         std::lock_guard<std::mutex> lock(x->pass_mutex);
-        pvs_status s = ensure_bf16(x);
+        pvs_status s = ensure_bf16(x, st);
         if (s != PVS_OK) return s;
     }
     if (!check_now) return PVS_OK;
@@ -678,16 +683,16 @@ pvs_status acquire_cursor(pvs_index* x, const std::shared_ptr<SnapData>& sd, pvs
 // single-query interval pass at its first pull.
 pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
                             const float* queries, int nq, bool on_device, int horizon,
-                            pvs_cursor** out) {
-    cudaStream_t st = x->stream;
+                            cudaStream_t st, pvs_cursor** out) {
     DevBuf buf(st, x->scratch_pool);
     BatchQueries bq;
     // one synchronisation at the end: query statuses are read with the pass's
-    pvs_status s = encode_batch(x, queries, nq, on_device, buf, &bq, /*check_now=*/false);
+    pvs_status s = encode_batch(x, queries, nq, on_device, buf, &bq, st, /*check_now=*/false);
     if (s != PVS_OK) return s;
     for (int i = 0; i < nq; ++i) {
         s = acquire_cursor(x, sd, &out[i], /*zero_state=*/false);
         if (s != PVS_OK) return s;
+        out[i]->stream = st;
     }
     QueryDst* d_qd = buf.get<QueryDst>((size_t)nq);
     if (!d_qd) return PVS_ERR_OOM;
@@ -832,11 +837,33 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
 // ===========================================================================
 // C ABI
 // ===========================================================================
+// The index's device is current for the duration of a call (the CUDA
+// runtime's current device belongs to the calling host thread).
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        int cur = -1;
+        if (dev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != dev &&
+            cudaSetDevice(dev) == cudaSuccess)
+            prev = cur;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+static int index_device(const pvs_index* x) { return x ? x->device : -1; }
+static int cursor_device(const pvs_cursor* c) { return c && c->index ? c->index->device : -1; }
+static int first_cursor_device(pvs_cursor* const* cs, int32_t nc) {
+    return cs && nc > 0 ? cursor_device(cs[0]) : -1;
+}
+
 extern "C" {
 
 int64_t pvs_launch_count(void) { return (int64_t)g_launches.load(); }
 
 pvs_status pvs_cursor_set_stream(pvs_cursor* c, void* cuda_stream) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c || !c->index) return PVS_ERR_INVALID;
     PVS_CUDA(cudaStreamSynchronize(c->stream));
     c->stream = cuda_stream ? static_cast<cudaStream_t>(cuda_stream) : c->index->stream;
@@ -910,6 +937,7 @@ pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_
 }
 
 pvs_status pvs_append(pvs_index* x, const float* vecs, int64_t n, int32_t vecs_on_device) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || n < 0 || (n > 0 && !vecs) || x->size + n >= ((int64_t)1 << 31))
         return PVS_ERR_INVALID;
     if (n == 0) return PVS_OK;
@@ -924,6 +952,7 @@ pvs_status pvs_append(pvs_index* x, const float* vecs, int64_t n, int32_t vecs_o
 }
 
 pvs_status pvs_tombstone(pvs_index* x, const int64_t* ids, int64_t n) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || n < 0 || (n > 0 && !ids)) return PVS_ERR_INVALID;
     for (int64_t i = 0; i < n; ++i)
         if (ids[i] < 0 || ids[i] >= x->size) return PVS_ERR_INVALID;
@@ -946,6 +975,7 @@ int32_t pvs_index_dim(const pvs_index* x) { return x ? x->m : -1; }
 
 pvs_status pvs_index_export(const pvs_index* x, int64_t first, int64_t count, int8_t* codes,
                             float* scale, float* vnorm, float* enorm) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || first < 0 || count < 0 || first + count > x->size) return PVS_ERR_INVALID;
     if (count == 0) return PVS_OK;
     if (codes)
@@ -961,6 +991,7 @@ pvs_status pvs_index_export(const pvs_index* x, int64_t first, int64_t count, in
 }
 
 void pvs_index_free(pvs_index* x) {
+    DeviceGuard device_guard(index_device(x));
     if (!x) return;
     if (x->stream) cudaStreamSynchronize(x->stream);
     for (pvs_cursor* c : x->cursor_pool) {
@@ -973,11 +1004,13 @@ void pvs_index_free(pvs_index* x) {
     dev_free(x->raw), dev_free(x->d_status), dev_free(x->d_stage), dev_free(x->codes_bf16);
     if (x->pass_done) cudaEventDestroy(x->pass_done);
     if (x->scratch_pool) cudaMemPoolDestroy(x->scratch_pool);
+    if (x->bf16_ready) cudaEventDestroy(x->bf16_ready);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
 }
 
 pvs_status pvs_snapshot_create(pvs_index* x, pvs_snapshot** out) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || !out) return PVS_ERR_INVALID;
     *out = nullptr;
     auto d = make_snapdata(x);
@@ -992,10 +1025,14 @@ pvs_status pvs_snapshot_create(pvs_index* x, pvs_snapshot** out) {
 
 int64_t pvs_snapshot_visible(const pvs_snapshot* s) { return s ? s->data->visible : -1; }
 
-void pvs_snapshot_free(pvs_snapshot* s) { delete s; }
+void pvs_snapshot_free(pvs_snapshot* s) {
+    DeviceGuard device_guard(s ? index_device(s->index) : -1);
+    delete s;
+}
 
 pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* query,
                            int32_t query_on_device, pvs_cursor** out) {
+    DeviceGuard device_guard(index_device(x));
     if (!out) return PVS_ERR_INVALID;
     *out = nullptr;
     if (!x || !query || (snap && snap->index != x)) return PVS_ERR_INVALID;
@@ -1056,7 +1093,8 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
 
 pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const float* queries,
                                  int32_t nq, int32_t queries_on_device, int32_t horizon,
-                                 pvs_cursor** out) {
+                                 void* cuda_stream, pvs_cursor** out) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || !queries || !out || nq < 0 || horizon < 1) return PVS_ERR_INVALID;
     if (queries_on_device && !is_device_ptr(queries)) return PVS_ERR_INVALID;
     for (int32_t i = 0; i < nq; ++i) out[i] = nullptr;
@@ -1065,7 +1103,10 @@ pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const f
     for (int32_t g0 = 0; g0 < nq; g0 += kBatchMax) {
         const int32_t g = std::min<int32_t>(kBatchMax, nq - g0);
         pvs_status s = open_batch_group(x, sd, queries + (size_t)g0 * x->m, g,
-                                        queries_on_device != 0, horizon, out + g0);
+                                        queries_on_device != 0, horizon,
+                                        cuda_stream ? static_cast<cudaStream_t>(cuda_stream)
+                                                    : x->stream,
+                                        out + g0);
         if (s != PVS_OK) {
             for (int32_t j = 0; j < nq; ++j) {
                 if (out[j]) pvs_cursor_close(out[j]);
@@ -1079,6 +1120,7 @@ pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const f
 
 pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float* queries,
                             int32_t nq, int32_t queries_on_device, float* lo, float* hi) {
+    DeviceGuard device_guard(index_device(x));
     if (!x || !queries || !lo || !hi || nq < 1 || nq > kBatchMax) return PVS_ERR_INVALID;
     if (queries_on_device && !is_device_ptr(queries)) return PVS_ERR_INVALID;
     std::shared_ptr<SnapData> sd = snap ? snap->data : make_snapdata(x);
@@ -1088,7 +1130,7 @@ pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float*
     cudaStream_t st = x->stream;
     DevBuf buf(st, x->scratch_pool);
     BatchQueries bq;
-    pvs_status s = encode_batch(x, queries, nq, queries_on_device, buf, &bq);
+    pvs_status s = encode_batch(x, queries, nq, queries_on_device, buf, &bq, st);
     if (s != PVS_OK) return s;
     const int64_t ntiles = (rows + 127) / 128;
     const int64_t ld = ntiles * 128;
@@ -1126,6 +1168,7 @@ pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float*
 
 pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
                           int64_t* ids, float* scores, int32_t* n_out) {
+    DeviceGuard device_guard(first_cursor_device(cursors, nc));
     if (!cursors || nc < 0 || n < 0 || !n_out || (nc > 0 && n > 0 && (!ids || !scores)))
         return PVS_ERR_INVALID;
     if (nc == 0) return PVS_OK;
@@ -1190,7 +1233,7 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
     if (!args.empty()) {
         PVS_CUDA(cudaMemcpyAsync(d_args, args.data(), args.size() * sizeof(PullArgs),
                                  cudaMemcpyHostToDevice, st));
-        PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, st));
+        PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, x->m_raw, st));
     }
     for (int32_t i : who) {
         cursors[i]->emitted += n_out[i];
@@ -1230,6 +1273,7 @@ static pvs_status next_common(pvs_cursor* c, int32_t n, int32_t* n_out, int64_t*
 }
 
 pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    DeviceGuard device_guard(cursor_device(c));
     int64_t n_eff;
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
@@ -1258,6 +1302,7 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
 
 pvs_status pvs_next_device(pvs_cursor* c, int32_t n, int64_t* ids, float* scores,
                            int32_t* n_out) {
+    DeviceGuard device_guard(cursor_device(c));
     int64_t n_eff;
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
@@ -1272,6 +1317,7 @@ pvs_status pvs_next_device(pvs_cursor* c, int32_t n, int64_t* ids, float* scores
 }
 
 pvs_status pvs_cursor_sync(pvs_cursor* c) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c) return PVS_ERR_INVALID;
     if (c->state < 0) return (pvs_status)c->state;
     pvs_status s = check_device_status(c);
@@ -1298,6 +1344,7 @@ static void fill_stats(pvs_cursor* c, const DevCounters& d, pvs_stats* out) {
 }
 
 pvs_status pvs_cursor_stats(pvs_cursor* c, pvs_stats* out) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c || !out) return PVS_ERR_INVALID;
     std::memset(out, 0, sizeof(*out));
     DevCounters d{};
@@ -1317,6 +1364,7 @@ static bool valid_cursor_list(pvs_cursor* const* cs, int32_t nc) {
 }
 
 pvs_status pvs_cursor_sync_batch(pvs_cursor** cursors, int32_t nc, int32_t* states) {
+    DeviceGuard device_guard(first_cursor_device(cursors, nc));
     if (!valid_cursor_list(cursors, nc) || (nc > 0 && !states)) return PVS_ERR_INVALID;
     std::vector<int> dev_status((size_t)nc, 0);
     pvs_status s = gather_state_any(cursors, nc, dev_status.data(), nullptr);
@@ -1330,6 +1378,7 @@ pvs_status pvs_cursor_sync_batch(pvs_cursor** cursors, int32_t nc, int32_t* stat
 }
 
 pvs_status pvs_cursor_stats_batch(pvs_cursor** cursors, int32_t nc, pvs_stats* out) {
+    DeviceGuard device_guard(first_cursor_device(cursors, nc));
     if (!valid_cursor_list(cursors, nc) || (nc > 0 && !out)) return PVS_ERR_INVALID;
     std::vector<int> dev_status((size_t)nc, 0);
     std::vector<DevCounters> d((size_t)nc, DevCounters{});
@@ -1345,6 +1394,7 @@ pvs_status pvs_cursor_stats_batch(pvs_cursor** cursors, int32_t nc, pvs_stats* o
 
 pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float* lo,
                              float* hi) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c || first < 0 || count < 0 || first + count > c->rows || (count > 0 && (!lo || !hi)))
         return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
@@ -1369,6 +1419,7 @@ pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float*
 }
 
 pvs_status pvs_cursor_score_ids(pvs_cursor* c, const int64_t* ids, int32_t n, float* scores) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c || n < 0 || (n > 0 && (!ids || !scores))) return PVS_ERR_INVALID;
     for (int32_t i = 0; i < n; ++i)
         if (ids[i] < 0 || ids[i] >= c->rows) return PVS_ERR_INVALID;
@@ -1411,12 +1462,14 @@ static void release_cursor(pvs_cursor* c) {
 }
 
 void pvs_cursor_close(pvs_cursor* c) {
+    DeviceGuard device_guard(cursor_device(c));
     if (!c) return;
     if (c->index) cudaStreamSynchronize(c->stream);
     release_cursor(c);
 }
 
 void pvs_cursor_close_batch(pvs_cursor** cursors, int32_t nc) {
+    DeviceGuard device_guard(first_cursor_device(cursors, nc));
     if (!cursors || nc <= 0) return;
     std::vector<cudaStream_t> synced;
     for (int32_t i = 0; i < nc; ++i) {

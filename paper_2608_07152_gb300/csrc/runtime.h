@@ -53,6 +53,7 @@ struct pvs_index {
     // bf16 copy of the codes for the tensor-core batched pass (built on demand)
     uint16_t* codes_bf16 = nullptr;         // [cap][m_pad]
     int64_t bf16_rows = 0;                  // rows converted so far
+    cudaEvent_t bf16_ready = nullptr;       // end of the last conversion (any stream)
     // stream-ordered scratch of batched calls; keeps its memory between calls
     // (the device's default pool hands memory back at every synchronisation)
     cudaMemPool_t scratch_pool = nullptr;

@@ -155,3 +155,41 @@ def test_open_batch_rejects_a_non_finite_query_and_stays_usable():
         pvs.pvs_cursor_close_batch(curs)
     finally:
         pvs.pvs_index_free(index)
+
+
+def test_batched_opens_on_two_threads_and_streams():
+    import threading
+    V, Q = _mixture(6_000, 128, 64, seed=41, comps=16)
+    index = pvs.pvs_build(V)
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    results, errors = {}, []
+
+    def worker(k):
+        try:
+            for rep in range(3):
+                part = Q[k * 32:(k + 1) * 32]
+                curs = pvs.pvs_cursor_open_batch(index, part, horizon=40, stream=streams[k])
+                ids, sc, n_out = pvs.pvs_next_batch(curs, 40)
+                assert all(pvs.pvs_cursor_sync_batch(curs) >= 0)
+                pvs.pvs_cursor_close_batch(curs)
+                results[(k, rep)] = (ids.copy(), sc.copy())
+        except Exception as e:
+            errors.append(e)
+
+    try:
+        threads = [threading.Thread(target=worker, args=(k,)) for k in range(2)]
+        for t in threads:
+            t.start()
+        for t in threads:
+            t.join()
+        assert not errors, errors
+        vis = np.ones(len(V), bool)
+        for k in range(2):
+            for i in (0, 13, 31):
+                ref_ids, ref_sc = po.dense_ranking(Q[k * 32 + i], V, vis)
+                for rep in range(3):
+                    ids, sc = results[(k, rep)]
+                    assert np.array_equal(ids[i], ref_ids[:40])
+                    assert np.array_equal(sc[i], ref_sc[:40])
+    finally:
+        pvs.pvs_index_free(index)
