@@ -248,6 +248,7 @@ __device__ inline bool eft_finish(EftAcc acc, int m_raw, float* out) {
 // generic loads); q (global) serves the out-of-line exact path.  Up to
 // kBatch float4 of the row are in flight per lane: a row of up to
 // 4 * 32 * kBatch values costs one round trip to memory.
+template <int kBatch = 8>
 __device__ inline float exact_dot_warp_eft(const float* q_fast, const float* __restrict__ q,
                                            const float* __restrict__ v, int m_raw,
                                            bool* used_fallback) {
@@ -255,7 +256,6 @@ __device__ inline float exact_dot_warp_eft(const float* q_fast, const float* __r
     const float4* q4 = reinterpret_cast<const float4*>(q_fast);
     const float4* v4 = reinterpret_cast<const float4*>(v);
     EftAcc acc;
-    constexpr int kBatch = 8;
     const int n4 = m_raw >> 2;
 #pragma unroll 1
     for (int j0 = lane; j0 < n4; j0 += kWarp * kBatch) {

@@ -67,6 +67,10 @@ struct PullArgs {
 };
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
 // Many cursors at once (args_dev: device array of ncursors PullArgs).
+// One launch per pull (n <= kPullFusedMax): a cluster of CTAs selects,
+// refines and emits (one cluster per cursor in the batch form).
+cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st);
+cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st);
 cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
                               int m_raw, cudaStream_t st);
 cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,

@@ -36,6 +36,7 @@ struct PullShared {
     unsigned long long prefix;
     unsigned long long k;
     unsigned int count;
+    unsigned int cand_n;
     int ok;
 };
 
@@ -190,56 +191,11 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_select_batch_kernel(cons
     pull_select_body(args[blockIdx.x], sh);
 }
 
-// Steps 4-5 (one CTA): order the candidates (all scored by now) and emit the
-// first n.
-__device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const unsigned int c = a.ctr->cand;
+// Sort the m keys in sh.sk (descending) and emit the first n: ids, scores,
+// and -inf bounds for the delivered rows.
+__device__ inline void emit_sorted(const PullArgs& a, PullShared& sh, int m) {
+    const int t = threadIdx.x;
     const int n = a.n;
-    if (c < (unsigned int)n) {      // only after a failure recorded by the select step
-        if (t == 0) set_status(a.status, PVS_ERR_INVALID);
-        return;
-    }
-    int m;   // keys in sh.sk to sort
-    if (c <= (unsigned int)kPullSortCap) {
-        for (unsigned int j = t; j < c; j += kPullThreads) {
-            const int32_t w = a.cand[j];
-            sh.sk[j] = rank_key(a.w_lo[w], (uint32_t)w);
-        }
-        m = (int)c;
-    } else {
-        for (unsigned int j = t; j < c; j += kPullThreads) {
-            const int32_t w = a.cand[j];
-            a.keys[j] = rank_key(a.w_lo[w], (uint32_t)w);
-        }
-        if (t == 0) {
-            sh.prefix = 0;
-            sh.k = (unsigned long long)n;
-        }
-        __syncthreads();
-        const CandKeys ck{a.keys};
-        const int shifts64[6] = {53, 42, 31, 20, 9, 0}, bits64[6] = {11, 11, 11, 11, 11, 9};
-        for (int p = 0; p < 6; ++p) {
-            block_histogram<unsigned long long>(sh, c, shifts64[p], bits64[p], sh.prefix, ck);
-            block_pick_digit(sh, shifts64[p]);
-        }
-        const unsigned long long kth = sh.prefix;   // keys are unique: exactly n keys >= kth
-        if (t == 0) sh.count = 0;
-        __syncthreads();
-        for (unsigned int i0 = warp * 32; i0 < c; i0 += kPullThreads) {
-            const unsigned int i = i0 + lane;
-            const unsigned long long kv = i < c ? a.keys[i] : 0ull;
-            const bool f = i < c && kv >= kth;
-            const unsigned int bal = __ballot_sync(0xffffffffu, f);
-            unsigned int base = 0;
-            if (lane == 0 && bal) base = atomicAdd(&sh.count, (unsigned int)__popc(bal));
-            base = __shfl_sync(0xffffffffu, base, 0);
-            const unsigned int pos = base + __popc(bal & ((1u << lane) - 1u));
-            if (f && pos < (unsigned int)kPullSortCap) sh.sk[pos] = kv;
-        }
-        __syncthreads();
-        m = n;
-    }
     int pow2 = 1;
     while (pow2 < m) pow2 <<= 1;
     for (int j = m + t; j < pow2; j += kPullThreads) sh.sk[j] = 0ull;
@@ -260,6 +216,70 @@ __device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
     }
 }
 
+// More than kPullSortCap candidates (a list in global memory; the selection
+// uses sh.hist): keys to a.keys, radix selection of the n-th largest key,
+// the n largest into sh.sk.  Out of line: rare, and register-hungry.
+static __device__ __noinline__ void emit_many(const PullArgs& a, PullShared& sh,
+                                              const int32_t* cand, unsigned int c) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int n = a.n;
+    for (unsigned int j = t; j < c; j += kPullThreads) {
+        const int32_t w = cand[j];
+        a.keys[j] = rank_key(a.w_lo[w], (uint32_t)w);
+    }
+    if (t == 0) {
+        sh.prefix = 0;
+        sh.k = (unsigned long long)n;
+    }
+    __syncthreads();
+    const CandKeys ck{a.keys};
+    const int shifts64[6] = {53, 42, 31, 20, 9, 0}, bits64[6] = {11, 11, 11, 11, 11, 9};
+    for (int p = 0; p < 6; ++p) {
+        block_histogram<unsigned long long>(sh, c, shifts64[p], bits64[p], sh.prefix, ck);
+        block_pick_digit(sh, shifts64[p]);
+    }
+    const unsigned long long kth = sh.prefix;   // keys are unique: exactly n keys >= kth
+    if (t == 0) sh.count = 0;
+    __syncthreads();
+    for (unsigned int i0 = warp * 32; i0 < c; i0 += kPullThreads) {
+        const unsigned int i = i0 + lane;
+        const unsigned long long kv = i < c ? a.keys[i] : 0ull;
+        const bool f = i < c && kv >= kth;
+        const unsigned int bal = __ballot_sync(0xffffffffu, f);
+        unsigned int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(&sh.count, (unsigned int)__popc(bal));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        const unsigned int pos = base + __popc(bal & ((1u << lane) - 1u));
+        if (f && pos < (unsigned int)kPullSortCap) sh.sk[pos] = kv;
+    }
+    __syncthreads();
+    emit_sorted(a, sh, n);
+}
+
+// Steps 4-5 (one CTA): order the candidates (all scored by now) and emit the
+// first n.
+__device__ inline void pull_emit_list(const PullArgs& a, PullShared& sh, const int32_t* cand,
+                                      unsigned int c) {
+    const int t = threadIdx.x;
+    if (c < (unsigned int)a.n) {      // only after a failure recorded by the select step
+        if (t == 0) set_status(a.status, PVS_ERR_INVALID);
+        return;
+    }
+    if (c > (unsigned int)kPullSortCap) {
+        emit_many(a, sh, cand, c);
+        return;
+    }
+    for (unsigned int j = t; j < c; j += kPullThreads) {
+        const int32_t w = cand[j];
+        sh.sk[j] = rank_key(a.w_lo[w], (uint32_t)w);
+    }
+    emit_sorted(a, sh, (int)c);
+}
+
+__device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
+    pull_emit_list(a, sh, a.cand, a.ctr->cand);
+}
+
 __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) {
     __shared__ PullShared sh;
     pull_emit_body(a, sh);
@@ -268,6 +288,223 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) 
 __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const PullArgs* args) {
     __shared__ PullShared sh;
     pull_emit_body(args[blockIdx.x], sh);
+}
+
+// ---- one launch per pull: a cluster of kPullCluster CTAs ----------------------
+// Every CTA of the cluster derives tau and the candidate list itself (the same
+// set; its order may differ), refines the candidates it owns (working-set
+// index modulo the cluster's warps), and after a cluster barrier with
+// release / acquire semantics CTA 0 orders the candidates and emits.
+//   tau: every thread takes the largest live lower bound of its share; in
+//   every warp the j-th largest of these, j = ceil(n / warps), bounds the
+//   answer from below, and so does t0, their minimum (each warp holds j values
+//   >= t0).  One more pass gathers the live rows with hi >= t0 (every row with
+//   lo >= t0 among them); tau is the n-th largest lower bound of the gathered
+//   rows and the candidates are those with hi >= tau.  If more rows than
+//   kPullSortCap reach t0, CTA 0 runs the radix selection instead.
+constexpr int kPullCluster = 8;
+constexpr int kPullClusterWarps = kPullCluster * kPullWarps;
+
+__device__ inline uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ inline void cluster_barrier() {
+    asm volatile(
+        "barrier.cluster.arrive.release.aligned;\n\t"
+        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// The j-th largest of the warp's 32 values (each lane one value).
+__device__ inline uint32_t warp_jth_largest(uint32_t v, int j) {
+    uint32_t out = 0;
+    for (int it = 0; it < j; ++it) {
+        out = __reduce_max_sync(0xffffffffu, v);
+        const unsigned int holders = __ballot_sync(0xffffffffu, v == out);
+        if ((int)(threadIdx.x & 31) == __ffs(holders) - 1) v = 0;
+    }
+    return out;
+}
+
+// 1: the candidate list is in sh.hist (int32) with sh.cand_n entries;
+// 0: more than kPullSortCap rows reach t0 (the radix path must select);
+// -1: fewer than n live rows.  Every CTA reaches the same outcome.
+__device__ inline int pull_select_fast(const PullArgs& a, PullShared& sh) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const unsigned int len = *a.w_len;
+    const int n = a.n;
+    uint32_t mx = 0;   // 0: no live row (every live key is larger)
+    for (unsigned int i = t; i < len; i += kPullThreads) {
+        const float l = a.w_lo[i];
+        if (l != -INFINITY) mx = max(mx, fkey(l));
+    }
+    const uint32_t wj = warp_jth_largest(mx, (n + kPullWarps - 1) / kPullWarps);
+    if (lane == 0) sh.warp_tot[warp] = wj;
+    if (t == 0) {
+        sh.count = 0;
+        sh.cand_n = 0;
+        sh.ok = 0;
+    }
+    __syncthreads();
+    uint32_t t0 = 0xffffffffu;
+    for (int w = 0; w < kPullWarps; ++w) t0 = min(t0, sh.warp_tot[w]);
+    for (unsigned int i0 = warp * 32; i0 < len; i0 += kPullThreads) {
+        const unsigned int i = i0 + lane;
+        bool f = false;
+        uint32_t lk = 0, hk = 0;
+        if (i < len) {
+            const float l = a.w_lo[i];
+            if (l != -INFINITY) {
+                hk = fkey(a.w_hi[i]);
+                lk = fkey(l);
+                f = hk >= t0;
+            }
+        }
+        const unsigned int bal = __ballot_sync(0xffffffffu, f);
+        unsigned int base = 0;
+        if (lane == 0 && bal) base = atomicAdd(&sh.count, (unsigned int)__popc(bal));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        const unsigned int pos = base + __popc(bal & ((1u << lane) - 1u));
+        if (f && pos < (unsigned int)kPullSortCap) {
+            sh.hist[pos] = lk;
+            sh.sk[pos] = ((unsigned long long)hk << 32) | i;
+        }
+    }
+    __syncthreads();
+    const unsigned int g = sh.count;
+    if (g > (unsigned int)kPullSortCap) return 0;
+    // tau: the lower-bound key v with #{> v} < n <= #{>= v}
+    for (unsigned int e = t; e < g; e += kPullThreads) {
+        const uint32_t le = sh.hist[e];
+        unsigned int gt = 0, ge = 0;
+        for (unsigned int f = 0; f < g; ++f) {
+            const uint32_t lf = sh.hist[f];
+            gt += lf > le;
+            ge += lf >= le;
+        }
+        if (gt < (unsigned int)n && (unsigned int)n <= ge) {
+            sh.prefix = le;   // every writer writes the same value
+            sh.ok = 1;
+        }
+    }
+    __syncthreads();
+    if (!sh.ok) return -1;
+    const uint32_t tau = (uint32_t)sh.prefix;
+    int32_t* list = reinterpret_cast<int32_t*>(sh.hist);   // the lower bounds are done with
+    for (unsigned int e = t; e < g; e += kPullThreads) {
+        const unsigned long long v = sh.sk[e];
+        if ((uint32_t)(v >> 32) >= tau) list[atomicAdd(&sh.cand_n, 1u)] = (int32_t)(uint32_t)v;
+    }
+    __syncthreads();
+    return 1;
+}
+
+// Exact scores of the candidates this warp owns (index modulo the cluster's warps).
+__device__ inline void cluster_refine(const PullArgs& a, const int32_t* cand, unsigned int c,
+                                      unsigned int gwarp) {
+    const int lane = threadIdx.x & 31;
+    unsigned long long refined = 0, fallbacks = 0;
+    for (unsigned int j0 = 0; j0 < c; j0 += 32) {
+        const unsigned int j = j0 + lane;
+        int32_t w = 0, id = 0;
+        float l = 0.0f, h = 0.0f;
+        bool own = false;
+        if (j < c) {
+            w = cand[j];
+            if ((unsigned int)w % kPullClusterWarps == gwarp) {
+                l = a.w_lo[w];
+                h = a.w_hi[w];
+                own = l < h;   // lo == hi: already the exact score
+                if (own) id = a.w_id[w];
+            }
+        }
+        unsigned int mine = __ballot_sync(0xffffffffu, own);
+        while (mine) {
+            const int b = __ffs(mine) - 1;
+            mine &= mine - 1;
+            const int32_t wb = __shfl_sync(0xffffffffu, w, b);
+            const int32_t idb = __shfl_sync(0xffffffffu, id, b);
+            const float lb = __shfl_sync(0xffffffffu, l, b);
+            const float hb = __shfl_sync(0xffffffffu, h, b);
+            bool fb;
+            const float s = exact_dot_warp_eft<2>(a.qraw, a.qraw, a.raw + (int64_t)idb * a.m_raw,
+                                                  a.m_raw, &fb);
+            if (lane == 0) {
+                ++refined;
+                fallbacks += fb;
+                if (!isfinite(s)) set_status(a.status, PVS_ERR_OVERFLOW);
+                else if (s < lb || s > hb) set_status(a.status, PVS_ERR_INTERVAL);
+                a.w_lo[wb] = s;
+                a.w_hi[wb] = s;
+                if (a.lo) {
+                    a.lo[idb] = s;
+                    a.hi[idb] = s;
+                }
+            }
+        }
+    }
+    if (lane == 0 && refined) {
+        atomicAdd(&a.ctr->refined, refined);
+        if (fallbacks) atomicAdd(&a.ctr->exact_fallbacks, fallbacks);
+    }
+}
+
+static __device__ __noinline__ void pull_select_radix(const PullArgs& a, PullShared& sh) {
+    pull_select_body(a, sh);
+}
+
+__device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
+    const uint32_t rank = cluster_ctarank();
+    const int mode = pull_select_fast(a, sh);
+    if (mode == 0 && rank == 0) pull_select_radix(a, sh);   // list and count in global memory
+    cluster_barrier();   // the fallback list is visible to every CTA
+    const int32_t* cand = mode == 1 ? reinterpret_cast<const int32_t*>(sh.hist) : a.cand;
+    const unsigned int c = mode == 1 ? sh.cand_n : (mode == 0 ? a.ctr->cand : 0u);
+    cluster_refine(a, cand, c, rank * kPullWarps + (threadIdx.x >> 5));
+    cluster_barrier();   // every exact score is visible to CTA 0
+    if (rank != 0) return;
+    if (mode == -1) {    // fewer than n live rows: the working set was too small
+        if (threadIdx.x == 0) {
+            set_status(a.status, PVS_ERR_INVALID);
+            a.ctr->cand = 0;
+        }
+        return;
+    }
+    if (mode == 1 && threadIdx.x == 0) {
+        a.ctr->cand = c;
+        a.ctr->cand_total += c;
+    }
+    pull_emit_list(a, sh, cand, c);
+}
+
+__global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThreads, 2)
+    pull_cluster_kernel(PullArgs a) {
+    __shared__ PullShared sh;
+    pull_cluster_body(a, sh);
+}
+
+// One cluster per cursor.
+__global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThreads, 2)
+    pull_cluster_batch_kernel(const PullArgs* args) {
+    __shared__ PullShared sh;
+    pull_cluster_body(args[blockIdx.x / kPullCluster], sh);
+}
+
+cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
+    if (a.n <= 0) return cudaSuccess;
+    if (a.n > kPullFusedMax) return cudaErrorInvalidValue;
+    count_launches(1);
+    pull_cluster_kernel<<<kPullCluster, kPullThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st) {
+    if (ncursors <= 0) return cudaSuccess;
+    count_launches(1);
+    pull_cluster_batch_kernel<<<ncursors * kPullCluster, kPullThreads, 0, st>>>(args_dev);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st) {

@@ -210,6 +210,7 @@ void cursor_reset(pvs_cursor* c) {
     c->state = PVS_OK;
     c->scanned = false;
     c->batch_ws = false;
+    c->fresh_ws = false;
     c->horizon = c->horizon_base = 0;
     c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
     c->batch_passes = 0;
@@ -370,6 +371,7 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     c->horizon = H;
     c->horizon_base = c->emitted;
     c->horizon_builds++;
+    c->fresh_ws = true;
     return PVS_OK;
 }
 
@@ -437,8 +439,12 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
         a.out_scores = d_scores;
         a.status = c->d_status;
         a.ctr = c->ctr;
-        cudaError_t e = launch_pull_fused(a, 2 * x->num_sms, st);
+        // the first pull of a working set refines most of it: spread that
+        // over every SM; later pulls take one cluster launch
+        cudaError_t e = c->fresh_ws ? launch_pull_fused(a, 2 * x->num_sms, st)
+                                    : launch_pull_cluster(a, st);
         if (e != cudaSuccess) return fail(c, cuda_status(e));
+        c->fresh_ws = false;
         c->emitted += n_eff;
         c->pulls++;
         return PVS_OK;
@@ -823,6 +829,7 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
         pvs_cursor* c = out[i];
         if (h_wlen[i] <= (unsigned int)w_cap && h_heff[i] > 0) {
             c->batch_ws = true;
+            c->fresh_ws = true;
             c->horizon = h_heff[i];
             c->horizon_base = 0;
         }
@@ -1233,11 +1240,17 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
     if (!args.empty()) {
         PVS_CUDA(cudaMemcpyAsync(d_args, args.data(), args.size() * sizeof(PullArgs),
                                  cudaMemcpyHostToDevice, st));
-        PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, x->m_raw, st));
+        bool fresh = false;
+        for (int32_t i : who) fresh = fresh || cursors[i]->fresh_ws;
+        if (fresh)   // first pull of new working sets: refinement on every SM
+            PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, x->m_raw, st));
+        else
+            PVS_CUDA(launch_pull_cluster_batch(d_args, (int)args.size(), st));
     }
     for (int32_t i : who) {
         cursors[i]->emitted += n_out[i];
         cursors[i]->pulls++;
+        cursors[i]->fresh_ws = false;
     }
     pvs_status result = PVS_OK;
     if (!outputs_on_device) {

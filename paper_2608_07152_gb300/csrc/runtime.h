@@ -82,6 +82,7 @@ struct pvs_cursor {
     // working set (ordered by id): rows that can hold the next `horizon` ranks
     int64_t cap_w = 0;                // capacity of the working-set arrays
     bool batch_ws = false;            // working set came from a batched pass (no full bounds)
+    bool fresh_ws = false;            // no pull since the working set was built (many candidates)
     int32_t* w_id = nullptr;
     float* w_lo = nullptr;
     float* w_hi = nullptr;

@@ -282,6 +282,38 @@ def test_ties_and_degenerate_queries():
         pvs.pvs_index_free(index)
 
 
+def test_many_tied_rows_take_the_radix_selection_paths():
+    """6,000 identical rows above 1,500 others: after the first pull more than
+    2,048 working-set rows reach the selection's lower bound, so the one-launch
+    pull falls back to the radix selection, and the emission orders more than
+    2,048 candidates."""
+    rng = np.random.default_rng(23)
+    m = 64
+    q = rng.standard_normal(m).astype(np.float32)
+    top = (q / np.linalg.norm(q)).astype(np.float32)
+    V = np.concatenate([np.tile(top, (6_000, 1)),
+                        (rng.standard_normal((1_500, m)) * 0.05).astype(np.float32)])
+    V = V[rng.permutation(len(V))]
+    index = pvs.pvs_build(V)
+    try:
+        ref_ids, ref_sc = po.dense_ranking(q, V, np.ones(len(V), bool))
+        cur = pvs.pvs_cursor_open(index, q)
+        try:
+            got_i, got_s = [], []
+            for _ in range(8):
+                i, sc, _ = pvs.pvs_next(cur, 100)
+                got_i.append(i)
+                got_s.append(sc)
+            st = pvs.pvs_cursor_stats(cur)
+        finally:
+            pvs.pvs_cursor_close(cur)
+        assert np.array_equal(np.concatenate(got_i), ref_ids[:800])
+        assert np.array_equal(np.concatenate(got_s), ref_sc[:800])
+        assert st["state"] >= 0
+    finally:
+        pvs.pvs_index_free(index)
+
+
 def test_empty_index_and_zero_pulls():
     index = pvs.pvs_build(np.zeros((0, 64), np.float32))
     try:
