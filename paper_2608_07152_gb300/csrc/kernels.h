@@ -37,6 +37,14 @@ struct DevCounters {
     unsigned int w_len;      // working-set length
     unsigned int cand;       // candidates of the current pull
     unsigned long long cand_total;   // candidates over fused pulls
+    // frontier carried between one-launch pulls: every live working-set row
+    // with hi >= front_bound (a float key) is among the front_n entries of
+    // PullArgs::front, and at least front_k live rows have lo >= front_bound;
+    // front_k == 0: no frontier
+    unsigned int front_n;
+    unsigned int front_bound;
+    unsigned int front_k;
+    unsigned int front_pad;
 };
 
 // Where one cursor keeps its device status word and counters.
@@ -64,6 +72,7 @@ struct PullArgs {
     float* out_scores;        // device
     int* status;
     DevCounters* ctr;
+    int32_t* front;           // frontier of working-set indices, kFrontCap entries
 };
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
 // Many cursors at once (args_dev: device array of ncursors PullArgs).
@@ -78,6 +87,7 @@ cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int bloc
 
 // ---- batched open support (pull_kernel.cu, batch_support.cu) ----------------
 constexpr int kWsSortMax = 8192;     // largest per-query working set of a batched open
+constexpr int kFrontCap = 2048;      // frontier entries (the one-launch pull's gather capacity)
 struct WsDst {                       // a cursor's working-set arrays
     int32_t* w_id;
     float* w_lo;

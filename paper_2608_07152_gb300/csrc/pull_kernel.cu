@@ -91,17 +91,23 @@ __device__ inline void block_histogram(PullShared& sh, unsigned int len, int shi
     const int top = shift + bits;
     const KeyT hmask = top >= (int)(8 * sizeof(KeyT)) ? (KeyT)0 : ~(KeyT)0 << top;
     const unsigned int dmask = (1u << bits) - 1u;
-    for (unsigned int i0 = warp * 32; i0 < len; i0 += kPullThreads) {
-        const unsigned int i = i0 + lane;
-        KeyT key = 0;
-        bool valid = i < len && src.valid(i);
-        if (valid) {
-            key = src.key(i);
-            valid = (key & hmask) == (prefix & hmask);
+    constexpr int kUnroll = 4;   // loads in flight per thread before the histogram updates
+    for (unsigned int i0 = warp * 32; i0 < len; i0 += kPullThreads * kUnroll) {
+        KeyT key[kUnroll];
+        bool valid[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const unsigned int i = i0 + u * kPullThreads + lane;
+            valid[u] = i < len && src.valid(i);
+            key[u] = valid[u] ? src.key(i) : (KeyT)0;
         }
-        const unsigned int d = valid ? (unsigned int)((key >> shift) & dmask) : (0x10000u + lane);
-        const unsigned int peers = __match_any_sync(0xffffffffu, d);
-        if (valid && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[d], (unsigned int)__popc(peers));
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const bool v = valid[u] && (key[u] & hmask) == (prefix & hmask);
+            const unsigned int d = v ? (unsigned int)((key[u] >> shift) & dmask) : (0x10000u + lane);
+            const unsigned int peers = __match_any_sync(0xffffffffu, d);
+            if (v && lane == __ffs(peers) - 1) atomicAdd(&sh.hist[d], (unsigned int)__popc(peers));
+        }
     }
     __syncthreads();
 }
@@ -164,6 +170,7 @@ __device__ inline void pull_select_body(const PullArgs& a, PullShared& sh) {
         }
     }
     const uint32_t tau = (uint32_t)sh.prefix;
+#pragma unroll 4
     for (unsigned int i0 = warp * 32; i0 < len; i0 += kPullThreads) {
         const unsigned int i = i0 + lane;
         const bool f = i < len && a.w_lo[i] != -INFINITY && fkey(a.w_hi[i]) >= tau;
@@ -277,6 +284,7 @@ __device__ inline void pull_emit_list(const PullArgs& a, PullShared& sh, const i
 }
 
 __device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
+    if (threadIdx.x == 0) a.ctr->front_k = 0;   // rows leave without the frontier's count
     pull_emit_list(a, sh, a.cand, a.ctr->cand);
 }
 
@@ -317,69 +325,184 @@ __device__ inline void cluster_barrier() {
         "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-// The j-th largest of the warp's 32 values (each lane one value).
-__device__ inline uint32_t warp_jth_largest(uint32_t v, int j) {
-    uint32_t out = 0;
-    for (int it = 0; it < j; ++it) {
-        out = __reduce_max_sync(0xffffffffu, v);
-        const unsigned int holders = __ballot_sync(0xffffffffu, v == out);
-        if ((int)(threadIdx.x & 31) == __ffs(holders) - 1) v = 0;
-    }
-    return out;
+// Execution barrier of the cluster without memory ordering.
+__device__ inline void cluster_barrier_relaxed() {
+    asm volatile(
+        "barrier.cluster.arrive.relaxed.aligned;\n\t"
+        "barrier.cluster.wait.aligned;" ::: "memory");
 }
 
-// 1: the candidate list is in sh.hist (int32) with sh.cand_n entries;
-// 0: more than kPullSortCap rows reach t0 (the radix path must select);
-// -1: fewer than n live rows.  Every CTA reaches the same outcome.
-__device__ inline int pull_select_fast(const PullArgs& a, PullShared& sh) {
+
+// Rows whose lower bound may reach the frontier bound: kFrontMult times the
+// ranks of the pull that builds it (the frontier then serves later pulls).
+constexpr int kFrontMult = 6;
+static_assert(kFrontCap == kPullSortCap, "the frontier is the gathered set");
+
+struct FastSelect {
+    int mode;            // 1: list in sh.hist (sh.cand_n entries); 0: radix fallback; -1: < n live
+    bool from_front;     // the rows came from the carried frontier
+    bool new_front;      // a whole-set gather at the wide bound: it can become the frontier
+    uint32_t t0;         // the bound of the gather
+    unsigned int g;      // rows gathered (hi >= t0)
+    unsigned int l;      // of them with lo >= t0
+};
+
+// Gather, with one shared-memory atomic per row that reaches t0 (few do),
+// (hi key, index) of the live rows with hi >= t0 into sh.sk (count sh.count)
+// and the lo keys of those with lo >= t0 into sh.hist (count sh.cand_n).
+// Rows: the frontier's len entries, or working-set indices 0 .. len-1.
+__device__ inline void gather_rows(const PullArgs& a, PullShared& sh, bool from_front,
+                                   unsigned int len, uint32_t t0) {
+    const int t = threadIdx.x;
+    auto take = [&](float l, float h, unsigned int i) {
+        if (l == -INFINITY) return;
+        const uint32_t hk = fkey(h);
+        if (hk < t0) return;
+        const unsigned int pos = atomicAdd(&sh.count, 1u);
+        if (pos < (unsigned int)kPullSortCap) sh.sk[pos] = ((unsigned long long)hk << 32) | i;
+        const uint32_t lk = fkey(l);
+        if (lk >= t0) {
+            const unsigned int q = atomicAdd(&sh.cand_n, 1u);
+            if (q < (unsigned int)kPullSortCap) sh.hist[q] = lk;
+        }
+    };
+    if (from_front) {
+        for (unsigned int e = t; e < len; e += kPullThreads) {
+            const int32_t w = a.front[e];
+            take(a.w_lo[w], a.w_hi[w], (unsigned int)w);
+        }
+    } else {
+        const unsigned int len4 = len >> 2;   // working-set arrays are 16-byte aligned
+        const float4* lo4 = reinterpret_cast<const float4*>(a.w_lo);
+        const float4* hi4 = reinterpret_cast<const float4*>(a.w_hi);
+#pragma unroll 4
+        for (unsigned int i = t; i < len4; i += kPullThreads) {
+            const float4 l = lo4[i], h = hi4[i];
+            take(l.x, h.x, 4 * i);
+            take(l.y, h.y, 4 * i + 1);
+            take(l.z, h.z, 4 * i + 2);
+            take(l.w, h.w, 4 * i + 3);
+        }
+        for (unsigned int i = 4 * len4 + t; i < len; i += kPullThreads) take(a.w_lo[i], a.w_hi[i], i);
+    }
+    __syncthreads();
+}
+
+// Selection for the one-launch pull; every CTA of the cluster reaches the
+// same outcome.  Rows come from the frontier when it still holds at least n
+// rows with lo >= its bound, else from the whole working set (then t0 comes
+// from the per-thread maxima, for kFrontMult * n ranks).  Gathered: (hi key,
+// index) of the rows with hi >= t0 in sh.sk; lo keys of those with lo >= t0
+// in sh.hist, among which tau is the n-th largest.
+__device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const unsigned int len = *a.w_len;
     const int n = a.n;
-    uint32_t mx = 0;   // 0: no live row (every live key is larger)
-    for (unsigned int i = t; i < len; i += kPullThreads) {
-        const float l = a.w_lo[i];
-        if (l != -INFINITY) mx = max(mx, fkey(l));
-    }
-    const uint32_t wj = warp_jth_largest(mx, (n + kPullWarps - 1) / kPullWarps);
-    if (lane == 0) sh.warp_tot[warp] = wj;
-    if (t == 0) {
-        sh.count = 0;
-        sh.cand_n = 0;
-        sh.ok = 0;
-    }
-    __syncthreads();
-    uint32_t t0 = 0xffffffffu;
-    for (int w = 0; w < kPullWarps; ++w) t0 = min(t0, sh.warp_tot[w]);
-    for (unsigned int i0 = warp * 32; i0 < len; i0 += kPullThreads) {
-        const unsigned int i = i0 + lane;
-        bool f = false;
-        uint32_t lk = 0, hk = 0;
-        if (i < len) {
-            const float l = a.w_lo[i];
-            if (l != -INFINITY) {
-                hk = fkey(a.w_hi[i]);
-                lk = fkey(l);
-                f = hk >= t0;
+    FastSelect r{1, false, false, 0u, 0u, 0u};
+    const unsigned int fk = a.ctr->front_k;
+    r.from_front = a.front != nullptr && fk >= (unsigned int)n;
+    r.new_front = !r.from_front && a.front != nullptr;
+    unsigned int len;
+    uint32_t t0_tight = 0;   // whole-set pass: the bound for n rows (t0 is for kFrontMult n)
+    if (r.from_front) {
+        len = a.ctr->front_n;
+        r.t0 = a.ctr->front_bound;
+        if (t == 0) {
+            sh.count = 0;
+            sh.cand_n = 0;
+            sh.ok = 0;
+        }
+        __syncthreads();
+    } else {
+        len = *a.w_len;
+        uint32_t mx = 0;   // 0: no live row (every live key is larger)
+        auto live_key = [](float l) -> uint32_t { return l == -INFINITY ? 0u : fkey(l); };
+        const unsigned int len4 = len >> 2;   // working-set arrays are 16-byte aligned
+        // a small set goes one row per thread so that every warp holds rows
+        const bool vec = len4 >= (unsigned int)kPullThreads;
+        if (vec) {
+            const float4* lo4 = reinterpret_cast<const float4*>(a.w_lo);
+#pragma unroll 4
+            for (unsigned int i = t; i < len4; i += kPullThreads) {
+                const float4 l = lo4[i];
+                mx = max(mx, max(max(live_key(l.x), live_key(l.y)), max(live_key(l.z), live_key(l.w))));
             }
+            for (unsigned int i = 4 * len4 + t; i < len; i += kPullThreads)
+                mx = max(mx, live_key(a.w_lo[i]));
+        } else {
+            for (unsigned int i = t; i < len; i += kPullThreads) mx = max(mx, live_key(a.w_lo[i]));
         }
-        const unsigned int bal = __ballot_sync(0xffffffffu, f);
-        unsigned int base = 0;
-        if (lane == 0 && bal) base = atomicAdd(&sh.count, (unsigned int)__popc(bal));
-        base = __shfl_sync(0xffffffffu, base, 0);
-        const unsigned int pos = base + __popc(bal & ((1u << lane) - 1u));
-        if (f && pos < (unsigned int)kPullSortCap) {
-            sh.hist[pos] = lk;
-            sh.sk[pos] = ((unsigned long long)hk << 32) | i;
+        const int busy_warps =
+            max(1, min(kPullWarps, (int)((min(len, (unsigned int)kPullThreads) + 31) / 32)));
+        // Every warp lists its j2 largest thread maxima (values of distinct
+        // rows); the R-th largest of the listed values bounds the R-th largest
+        // live lower bound from below.  R = n (over each warp's first j1
+        // values; the warps that hold rows list at least n) gives the tight
+        // bound; R = kFrontMult n, at most their j2 values each, the wide one.
+        // Threads without live rows list zeros (a bound of 0 gathers every row).
+        const int j1 = min(32, (n + busy_warps - 1) / busy_warps);
+        const int j2 = r.new_front ? max(j1, min(32, (kFrontMult * n + busy_warps - 1) / busy_warps))
+                                   : j1;
+        const unsigned int r2 = min((unsigned int)(kFrontMult * n), (unsigned int)(busy_warps * j2));
+        for (int it = 0; it < j2; ++it) {
+            const uint32_t top = __reduce_max_sync(0xffffffffu, mx);
+            const unsigned int holders = __ballot_sync(0xffffffffu, mx == top);
+            if (lane == __ffs(holders) - 1) mx = 0;
+            if (lane == 0) sh.hist[warp * j2 + it] = top;
         }
+        if (t == 0) {
+            sh.count = 0;
+            sh.cand_n = 0;
+            sh.ok = 0;
+            sh.warp_tot[0] = 0;   // wide bound
+            sh.warp_tot[1] = 0;   // tight bound
+        }
+        __syncthreads();
+        const int nv = kPullWarps * j2;
+        for (int e = t; e < nv; e += kPullThreads) {
+            const uint32_t v = sh.hist[e];
+            unsigned int gt = 0, ge = 0, gt1 = 0, ge1 = 0;
+            for (int f = 0; f < nv; ++f) {
+                const uint32_t u = sh.hist[f];
+                const bool first = (f % j2) < j1;
+                gt += u > v;
+                ge += u >= v;
+                gt1 += first && u > v;
+                ge1 += first && u >= v;
+            }
+            if (gt < r2 && r2 <= ge) sh.warp_tot[0] = v;                       // same value from every writer
+            if ((e % j2) < j1 && gt1 < (unsigned int)n && (unsigned int)n <= ge1) sh.warp_tot[1] = v;
+        }
+        __syncthreads();
+        r.t0 = sh.warp_tot[0];
+        t0_tight = sh.warp_tot[1];
+        __syncthreads();   // sh.hist is the gather's buffer
     }
-    __syncthreads();
-    const unsigned int g = sh.count;
-    if (g > (unsigned int)kPullSortCap) return 0;
-    // tau: the lower-bound key v with #{> v} < n <= #{>= v}
-    for (unsigned int e = t; e < g; e += kPullThreads) {
+    for (int attempt = 0;; ++attempt) {
+        gather_rows(a, sh, r.from_front, len, r.t0);
+        r.g = sh.count;
+        r.l = sh.cand_n;
+        if (r.g <= (unsigned int)kPullSortCap) break;
+        if (r.from_front || attempt > 0 || t0_tight <= r.t0) {
+            r.mode = 0;
+            return r;
+        }
+        // too many rows reach the wide bound: gather again at the bound for
+        // n rows (no frontier from this pull)
+        r.t0 = t0_tight;
+        r.new_front = false;
+        __syncthreads();
+        if (t == 0) {
+            sh.count = 0;
+            sh.cand_n = 0;
+        }
+        __syncthreads();
+    }
+    // tau: the lower-bound key v with #{> v} < n <= #{>= v} among the l rows
+    // with lo >= t0 (the n-th largest is one of them when l >= n)
+    for (unsigned int e = t; e < r.l; e += kPullThreads) {
         const uint32_t le = sh.hist[e];
         unsigned int gt = 0, ge = 0;
-        for (unsigned int f = 0; f < g; ++f) {
+        for (unsigned int f = 0; f < r.l; ++f) {
             const uint32_t lf = sh.hist[f];
             gt += lf > le;
             ge += lf >= le;
@@ -390,15 +513,20 @@ __device__ inline int pull_select_fast(const PullArgs& a, PullShared& sh) {
         }
     }
     __syncthreads();
-    if (!sh.ok) return -1;
+    if (!sh.ok) {
+        r.mode = -1;
+        return r;
+    }
     const uint32_t tau = (uint32_t)sh.prefix;
+    if (t == 0) sh.cand_n = 0;
+    __syncthreads();
     int32_t* list = reinterpret_cast<int32_t*>(sh.hist);   // the lower bounds are done with
-    for (unsigned int e = t; e < g; e += kPullThreads) {
+    for (unsigned int e = t; e < r.g; e += kPullThreads) {
         const unsigned long long v = sh.sk[e];
         if ((uint32_t)(v >> 32) >= tau) list[atomicAdd(&sh.cand_n, 1u)] = (int32_t)(uint32_t)v;
     }
     __syncthreads();
-    return 1;
+    return r;
 }
 
 // Exact scores of the candidates this warp owns (index modulo the cluster's warps).
@@ -416,11 +544,20 @@ __device__ inline void cluster_refine(const PullArgs& a, const int32_t* cand, un
             if ((unsigned int)w % kPullClusterWarps == gwarp) {
                 l = a.w_lo[w];
                 h = a.w_hi[w];
+                id = a.w_id[w];
                 own = l < h;   // lo == hi: already the exact score
-                if (own) id = a.w_id[w];
             }
         }
         unsigned int mine = __ballot_sync(0xffffffffu, own);
+        // start every owned row on its way into L1 (one 128-byte line per lane
+        // per step) before scoring the first
+        const int lines = (a.m_raw * (int)sizeof(float) + 127) >> 7;
+        for (unsigned int pm = mine; pm; pm &= pm - 1) {
+            const int32_t idp = __shfl_sync(0xffffffffu, id, __ffs(pm) - 1);
+            const char* row = reinterpret_cast<const char*>(a.raw + (int64_t)idp * a.m_raw);
+            for (int ln = lane; ln < lines; ln += 32)
+                asm volatile("prefetch.global.L1 [%0];" ::"l"(row + (ln << 7)));
+        }
         while (mine) {
             const int b = __ffs(mine) - 1;
             mine &= mine - 1;
@@ -457,9 +594,18 @@ static __device__ __noinline__ void pull_select_radix(const PullArgs& a, PullSha
 
 __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
     const uint32_t rank = cluster_ctarank();
-    const int mode = pull_select_fast(a, sh);
-    if (mode == 0 && rank == 0) pull_select_radix(a, sh);   // list and count in global memory
-    cluster_barrier();   // the fallback list is visible to every CTA
+    const FastSelect fs = pull_select_fast(a, sh);
+    const int mode = fs.mode;
+    // Every CTA has read the working set before any CTA writes a score into
+    // it.  In the fast path that ordering is all this barrier carries; after
+    // the radix fallback it also publishes CTA 0's list (the outcome is the
+    // same in every CTA).
+    if (mode == 0) {
+        if (rank == 0) pull_select_radix(a, sh);   // list and count in global memory
+        cluster_barrier();
+    } else {
+        cluster_barrier_relaxed();
+    }
     const int32_t* cand = mode == 1 ? reinterpret_cast<const int32_t*>(sh.hist) : a.cand;
     const unsigned int c = mode == 1 ? sh.cand_n : (mode == 0 ? a.ctr->cand : 0u);
     cluster_refine(a, cand, c, rank * kPullWarps + (threadIdx.x >> 5));
@@ -476,6 +622,24 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
         a.ctr->cand = c;
         a.ctr->cand_total += c;
     }
+    // the frontier for the next pulls (every CTA has read the old one by now):
+    // a whole-set gather becomes the frontier; a frontier pull uses up n of
+    // its rows with lo >= bound (rows only leave that set by being emitted)
+    if (threadIdx.x == 0) {   // (without a frontier buffer: any old frontier is void)
+        if (mode == 1 && fs.from_front) {
+            a.ctr->front_k -= (unsigned int)a.n;
+        } else if (mode == 1 && fs.new_front) {
+            a.ctr->front_n = fs.g;
+            a.ctr->front_bound = fs.t0;
+            a.ctr->front_k = fs.l >= (unsigned int)a.n ? fs.l - (unsigned int)a.n : 0u;
+        } else {
+            a.ctr->front_k = 0;
+        }
+    }
+    if (mode == 1 && fs.new_front)
+        for (unsigned int e = threadIdx.x; e < fs.g; e += kPullThreads)
+            a.front[e] = (int32_t)(uint32_t)sh.sk[e];
+    __syncthreads();   // sh.sk is the emission's sort buffer
     pull_emit_list(a, sh, cand, c);
 }
 

@@ -188,7 +188,7 @@ void cursor_free_device(pvs_cursor* c) {
     dev_free(c->lo), dev_free(c->hi);
     dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
     dev_free(c->compact_scratch);
-    dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp);
+    dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp), dev_free(c->front);
     if (c->sort_scratch) cudaFree(c->sort_scratch);
     c->sort_scratch = nullptr;
     dev_free(c->sel), dev_free(c->ctr), dev_free(c->d_status);
@@ -226,7 +226,7 @@ constexpr size_t kCursorPool = 1024;
 constexpr size_t kCursorPoolBytes = size_t(4) << 30;
 
 size_t cursor_device_bytes(const pvs_cursor* c) {
-    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096;
+    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096 + kFrontCap * 4;
 }
 
 // Allocate the per-row state of a cursor (first pull); a pooled cursor keeps
@@ -248,6 +248,7 @@ pvs_status cursor_alloc_full(pvs_cursor* c) {
 // not preserved when they grow).
 pvs_status cursor_alloc_ws(pvs_cursor* c, int64_t cap) {
     cap = std::max<int64_t>(cap, 1);
+    if (!c->front) PVS_CUDA(dev_alloc(&c->front, (size_t)kFrontCap));
     if (c->w_id && c->cap_w >= cap) return PVS_OK;
     dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
     dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp);
@@ -372,6 +373,7 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     c->horizon_base = c->emitted;
     c->horizon_builds++;
     c->fresh_ws = true;
+    PVS_CUDA(cudaMemsetAsync(&c->ctr->front_k, 0, sizeof(unsigned int), c->stream));   // new indices
     return PVS_OK;
 }
 
@@ -439,6 +441,7 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
         a.out_scores = d_scores;
         a.status = c->d_status;
         a.ctr = c->ctr;
+        a.front = c->front;
         // the first pull of a working set refines most of it: spread that
         // over every SM; later pulls take one cluster launch
         cudaError_t e = c->fresh_ws ? launch_pull_fused(a, 2 * x->num_sms, st)
@@ -450,7 +453,10 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
         return PVS_OK;
     }
     const int grid_w = grid_for(c, std::min<int64_t>(c->rows, (int64_t)1 << 22));
-    cudaError_t e = launch_select_f32(c->w_lo, &c->ctr->w_len, (uint64_t)n_eff, c->sel, grid_w, st);
+    // rows leave without the one-launch pull's frontier count: drop the frontier
+    cudaError_t e = cudaMemsetAsync(&c->ctr->front_k, 0, sizeof(unsigned int), st);
+    if (e == cudaSuccess)
+        e = launch_select_f32(c->w_lo, &c->ctr->w_len, (uint64_t)n_eff, c->sel, grid_w, st);
     if (e == cudaSuccess)
         e = launch_candidates(c->w_lo, c->w_hi, &c->ctr->w_len, c->sel, c->cand, &c->ctr->cand,
                               grid_w, st);
@@ -1234,6 +1240,7 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         a.out_scores = d_scores + (int64_t)i * n;
         a.status = c->d_status;
         a.ctr = c->ctr;
+        a.front = nullptr;   // a few pulls per batch: a frontier would not pay for itself
         args.push_back(a);
         who.push_back(i);
     }

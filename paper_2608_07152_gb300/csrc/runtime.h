@@ -90,6 +90,7 @@ struct pvs_cursor {
     unsigned int* compact_scratch = nullptr;
     // pull scratch
     int32_t* cand = nullptr;
+    int32_t* front = nullptr;         // frontier of the one-launch pull (kFrontCap entries)
     uint64_t* keys = nullptr;
     uint64_t* keys_tmp = nullptr;
     void* sort_scratch = nullptr;
