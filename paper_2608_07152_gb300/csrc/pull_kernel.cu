@@ -276,6 +276,35 @@ __device__ inline void pull_emit_list(const PullArgs& a, PullShared& sh, const i
         emit_many(a, sh, cand, c);
         return;
     }
+    if (c <= (unsigned int)kPullThreads) {
+        // one candidate per thread: its rank is the number of larger keys (keys
+        // are unique), and its id is loaded with its score
+        unsigned long long key = 0;
+        int32_t w = 0, id = 0;
+        if (t < (int)c) {
+            w = cand[t];
+            const float sc = a.w_lo[w];
+            id = a.w_id[w];
+            key = rank_key(sc, (uint32_t)w);
+            sh.sk[t] = key;
+        }
+        __syncthreads();
+        if (t < (int)c) {
+            unsigned int r = 0;
+            for (unsigned int f = 0; f < c; ++f) r += sh.sk[f] > key;
+            if (r < (unsigned int)a.n) {
+                a.out_ids[r] = id;
+                a.out_scores[r] = rank_key_score(key);
+                a.w_lo[w] = -INFINITY;
+                a.w_hi[w] = -INFINITY;
+                if (a.lo) {
+                    a.lo[id] = -INFINITY;
+                    a.hi[id] = -INFINITY;
+                }
+            }
+        }
+        return;
+    }
     for (unsigned int j = t; j < c; j += kPullThreads) {
         const int32_t w = cand[j];
         sh.sk[j] = rank_key(a.w_lo[w], (uint32_t)w);
