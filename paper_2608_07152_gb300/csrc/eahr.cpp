@@ -13,17 +13,19 @@
 // a / (b r + c) with denominators below 2^32, so numerators stay below 2^49,
 // denominators below 2^64, and comparisons are exact in 128-bit integers.
 //
-// Incremental structures: items read from both lists sit in an ordered set
-// keyed by (F desc, id asc); items read from one list only are ordered by
-// their rank in that list (their L and U are monotone in it), so the best
-// and second-best of each group are found without scanning O.
+// Incremental structures: items read from both lists (their F is final)
+// are kept best-first by (F desc, id asc), but only the K + 2 best of them:
+// certification looks at the best two, and items leave this group only from
+// the top, at most K times, so nothing further down can ever be looked at.
+// Items read from one list only are ordered by their rank in that list
+// (their L and U are monotone in it), so the best and second-best of each
+// group are found without scanning O.
 #include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
 #include <limits>
 #include <new>
-#include <set>
 #include <vector>
 
 #include "../../include/pvs.h"
@@ -99,6 +101,19 @@ struct NodeCmp {
     }
 };
 
+// The best `cap` items read from both lists, best first.
+struct TopBoth {
+    std::vector<Node> v;
+    size_t cap = 2;
+    bool empty() const { return v.empty(); }
+    void insert(const Node& n) {
+        if (v.size() == cap && !NodeCmp()(n, v.back())) return;   // not above the worst kept
+        v.insert(std::upper_bound(v.begin(), v.end(), n, NodeCmp()), n);
+        if (v.size() > cap) v.pop_back();
+    }
+    void pop_front() { v.erase(v.begin()); }
+};
+
 // (a, x) beats (b, y): a > b, or a == b and x has the smaller id.
 inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
     const int c = cmp(a, b);
@@ -125,7 +140,7 @@ class Driver {
     int32_t* rank[2] = {nullptr, nullptr};   // rank of id in list i (0: unread)
     uint8_t* inA = nullptr;
     int64_t id_space = 0;
-    std::set<Node, NodeCmp> both;
+    TopBoth both;
     size_t ptr[2] = {0, 0};
     std::vector<int32_t> A;
     int K = 0;
@@ -222,7 +237,7 @@ class Driver {
             advance_ptr(1);
             // candidates for x+
             int32_t cand[3] = {-1, -1, -1};
-            if (!both.empty()) cand[0] = both.begin()->id;
+            if (!both.empty()) cand[0] = both.v[0].id;
             if (active[0]) cand[1] = only_from(0, ptr[0], -1);
             if (active[1]) cand[2] = only_from(1, ptr[1], -1);
             int32_t xp = -1;
@@ -239,9 +254,8 @@ class Driver {
             // strongest other item by (U, id)
             int32_t others[3] = {-1, -1, -1};
             if (!both.empty()) {
-                auto it = both.begin();
-                if (it->id == xp) ++it;
-                if (it != both.end()) others[0] = it->id;
+                size_t k = both.v[0].id == xp ? 1 : 0;
+                if (k < both.v.size()) others[0] = both.v[k].id;
             }
             if (active[0]) others[1] = only_from(0, ptr[0], xp);
             if (active[1]) others[2] = only_from(1, ptr[1], xp);
@@ -255,7 +269,8 @@ class Driver {
             }
             A.push_back(xp);
             inA[xp] = 1;
-            if (active[0] && active[1] && rank[0][xp] && rank[1][xp]) both.erase(Node{Lx, xp});
+            // read from both lists: then it was the best of that group
+            if (active[0] && active[1] && rank[0][xp] && rank[1][xp]) both.pop_front();
         }
         return true;
     }
@@ -306,6 +321,7 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
     const int step0 = p->step > 0 ? p->step : 16;
     int64_t size[2] = {step0, step0};
     d.K = p->K;
+    d.both.cap = (size_t)p->K + 2;
     for (int i = 0; i < 2; ++i)
         if (!d.active[i]) d.exhausted[i] = false;
     // lists with zero weight contribute nothing and are never read
