@@ -56,14 +56,20 @@ def parse():
     p.add_argument("--queries", type=int, default=50, help="queries per step")
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--workload", default="passage", choices=["passage", "batched", "eahr"],
+    p.add_argument("--workload", default="passage",
+                   choices=["passage", "batched", "eahr", "snapshots"],
                    help="passage: single-query ranking (default); batched: 256-query "
                         "tensor-core batches; eahr: EAHR Top-20 fusion over the passage "
-                        "corpus and copula sparse rankings")
+                        "corpus and copula sparse rankings; snapshots: near-duplicate "
+                        "corpus, five snapshots, EAHR Top-20")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
                    help="queries at tau = -0.5 (both lists are read to the end)")
+    p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
+    p.add_argument("--oracle-check", action="store_true",
+                   help="snapshots: compare the first query's first 1,000 dense ranks of every "
+                        "snapshot with the oracle and count near-tie swaps")
     return p.parse_args()
 
 
@@ -602,6 +608,133 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+SNAP_N = 2_000_000
+SNAP_DIM = 1024
+SNAP_DUP = 0.2          # near-duplicate share of the base corpus
+SNAP_DUP_STD = 1e-4     # their noise (standard deviation)
+SNAP_STEPS = 5
+SNAP_APPEND = 0.1       # of the base size, per snapshot
+SNAP_TOMB = 0.02        # of the live rows, per snapshot
+SNAP_TAU = 0.2
+
+
+def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """Adversarial ties and snapshots: a 2,000,000 x 1,024 mixture corpus whose
+    last 20 % are near-duplicates of earlier rows (copies + N(0, 1e-4^2),
+    normalised); snapshot 1 is that corpus, every later snapshot appends 10 %
+    new mixture rows and tombstones 2 % of the live rows.  Per snapshot, 100
+    queries run EAHR Top-20 with a sparse channel that is a Gaussian-copula
+    ranking (Kendall tau 0.2) of the snapshot's visible ids."""
+    n0 = SNAP_N if args.n == N_CORPUS else args.n
+    d = SNAP_DIM
+    stream = torch.cuda.Stream(device=dev)
+    centres = synth.mixture_centres(COMPONENTS, d, seed=5, device=dev)
+    total = n0 + (SNAP_STEPS - 1) * int(SNAP_APPEND * n0)
+    rows = torch.empty((total, d), dtype=torch.float32, device=dev)
+    n_mix = n0 - int(SNAP_DUP * n0)
+    t0 = time.perf_counter()
+    rows[:n_mix] = synth.mixture_rows(n_mix, centres, WITHIN_STD, seed=5)
+    g = torch.Generator(device=dev)
+    g.manual_seed(55)
+    src = torch.randint(0, n_mix, (n0 - n_mix,), generator=g, device=dev)
+    rows[n_mix:n0] = synth.near_duplicate_rows(rows[src], SNAP_DUP_STD, seed=56)
+    index = pvs.pvs_build(rows[:n0], stream=stream.cuda_stream)
+    torch.cuda.synchronize()
+    build_s = time.perf_counter() - t0
+    visible = torch.ones(total, dtype=torch.bool, device=dev)
+    visible[n0:] = False
+    rng = np.random.default_rng(57 + rank)
+    queries = synth.mixture_queries(SNAP_STEPS * args.snap_queries + 2, centres, QUERY_NOISE,
+                                    seed=58 + 7919 * rank)
+    launches0 = pvs.pvs_launch_count()
+    per_snap = []
+    size = n0
+    qi = 0
+    lat_all = []
+    with ClockSampler(local) as clk:
+        for step in range(SNAP_STEPS):
+            if step > 0:   # grow and delete, then freeze
+                add = int(SNAP_APPEND * n0)
+                rows[size:size + add] = synth.mixture_rows(add, centres, WITHIN_STD,
+                                                           seed=60 + step)
+                pvs.pvs_append(index, rows[size:size + add])
+                visible[size:size + add] = True
+                size += add
+                live = torch.nonzero(visible[:size]).squeeze(1).cpu().numpy()
+                dead = rng.choice(live, int(SNAP_TOMB * live.size), replace=False)
+                pvs.pvs_tombstone(index, dead)
+                visible[torch.from_numpy(dead).to(dev)] = False
+            snap = pvs.pvs_snapshot_create(index)
+            vis_ids = torch.nonzero(visible[:size]).squeeze(1)
+            lat, depth, ex_any, ex_both, near_ties, swaps = [], [], 0, 0, None, None
+            for j in range(args.snap_queries):
+                q = queries[qi]
+                qi += 1
+                proxy = rows[vis_ids] @ q
+                sparse = vis_ids[synth.copula_ranking(proxy, SNAP_TAU, 900 + qi)].cpu().numpy()
+                torch.cuda.synchronize()
+                t = time.perf_counter()
+                cur = pvs.pvs_cursor_open(index, q, snap)
+                ids, F, st = pvs.eahr_topk(cur, sparse, K=EAHR_K, k=EAHR_RRF_K,
+                                           form=pvs.EAHR_NUMERATOR)
+                pvs.pvs_cursor_close(cur)
+                lat.append((time.perf_counter() - t) * 1e3)
+                depth.append(st["depth"][0])
+                ex_any += int(st["exhausted"][0] or st["exhausted"][1])
+                ex_both += int(st["exhausted"][0] and st["exhausted"][1])
+                if j == 0:   # near ties among the first 1,000 dense ranks of this snapshot
+                    cur = pvs.pvs_cursor_open(index, q, snap)
+                    d_ids, d_sc, _ = pvs.pvs_next(cur, 1000)
+                    pvs.pvs_cursor_close(cur)
+                    a = d_sc[:-1].astype(np.float64)
+                    b = d_sc[1:].astype(np.float64)
+                    near_ties = int(np.sum(np.abs(a - b) < 2.0 ** -20 *
+                                           np.maximum(np.abs(a), np.abs(b))))
+                    if args.oracle_check:
+                        from oracle import pvs_oracle as po
+                        vis_host = visible[:size].cpu().numpy()
+                        ref_ids, _ = po.dense_ranking(q.cpu().numpy(),
+                                                      rows[:size].cpu().numpy(), vis_host)
+                        swaps = int(np.sum(ref_ids[:len(d_ids)] != d_ids))
+            pvs.pvs_snapshot_free(snap)
+            lat_all.extend(lat)
+            per_snap.append({
+                "snapshot": step + 1, "rows": size, "visible": int(vis_ids.numel()),
+                "queries": args.snap_queries,
+                "latency_ms_p50": float(np.median(lat)), "latency_ms_p95": float(np.percentile(lat, 95)),
+                "dense_depth_p50": float(np.median(depth)),
+                "exhaustion_rate_any": ex_any / args.snap_queries,
+                "exhaustion_rate_both": ex_both / args.snap_queries,
+                "near_tie_pairs_first_1000": near_ties,
+                "oracle_mismatches_first_1000": swaps})
+    launches = pvs.pvs_launch_count() - launches0
+    p50 = float(np.median(lat_all))
+    line = {
+        "metric": "EAHR Top-20 latency (p50 over five snapshots)", "value": p50, "unit": "ms",
+        "n_gpus": world, "steps": len(lat_all), "warmup": 0, "ms_per_step": float(np.mean(lat_all)),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "int8",
+        "data": "synthetic",
+        "config": {"workload": "adversarial ties + snapshots: N=2,000,000 x d=1,024 mixture with "
+                               "20% near-duplicates (std 1e-4), +10% appended and 2% tombstoned "
+                               "per snapshot, 5 snapshots, EAHR Top-20, sparse Kendall tau 0.2",
+                   "N": n0, "d": d, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
+                   "l2": "no flush: every query's interval pass streams >= 2 GB of codes",
+                   "parallelism": f"replicas x{world}"},
+        "e2e": {"value": p50, "unit": "ms", "h2d_bytes_per_step": d * 4,
+                "d2h_bytes_per_step": EAHR_K * (8 + 8)},
+        "snapshots": per_snap,
+        "gpu_launches": launches,
+        "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    pvs.pvs_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -625,6 +758,9 @@ def main():
         return
     if args.workload == "eahr":
         main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
+    if args.workload == "snapshots":
+        main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
     stream = torch.cuda.Stream(device=dev)
