@@ -67,6 +67,8 @@ def parse():
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
                    help="queries at tau = -0.5 (both lists are read to the end)")
     p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
+    p.add_argument("--pipeline", type=int, default=0,
+                   help="queries (passage) or batches (batched) in flight; 0: the default")
     p.add_argument("--oracle-check", action="store_true",
                    help="snapshots: compare the first query's first 1,000 dense ranks of every "
                         "snapshot with the oracle and count near-tie swaps")
@@ -178,7 +180,8 @@ def build_corpus_index(pvs, synth, torch, n, stream, device, components=COMPONEN
     return index, centres, time.perf_counter() - t0
 
 
-PIPELINE = 2   # queries in flight, each on its own stream
+PIPELINE = 8   # queries in flight, each on its own stream (measured plateau: 2 -> 704k,
+               # 4 -> 827k, 6 -> 876k, 8 -> 903k, 10 -> 881k ranks/s)
 
 
 def _finish(pvs, cur, stats_acc):
@@ -736,7 +739,10 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
 
 
 def main():
+    global PIPELINE, BATCH_PIPELINE
     args = parse()
+    if args.pipeline > 0:
+        PIPELINE = BATCH_PIPELINE = args.pipeline
     if args.impl == "reference":
         reference_arm(args)
         return
@@ -844,6 +850,7 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
         "config": {"workload": WORKLOAD, "N": n, "d": DIM, "queries_per_step": args.queries,
                    "ranks_per_query": RANKS_PER_QUERY, "chunk": CHUNK,
+                   "queries_in_flight": PIPELINE,
                    "l2": "no flush: each query's interval pass streams 6.9 GB of codes (> 129 MB L2)",
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},
         "e2e": {"value": e2e_value, "unit": UNIT,
