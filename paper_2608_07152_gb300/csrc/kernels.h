@@ -73,6 +73,7 @@ struct PullArgs {
     int* status;
     DevCounters* ctr;
     int32_t* front;           // frontier of working-set indices, kFrontCap entries
+    int* status_mirror;       // pinned host word: the status after the pull (null: none)
 };
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
 // Many cursors at once (args_dev: device array of ncursors PullArgs).

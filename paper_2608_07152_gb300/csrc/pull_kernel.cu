@@ -312,9 +312,18 @@ __device__ inline void pull_emit_list(const PullArgs& a, PullShared& sh, const i
     emit_sorted(a, sh, (int)c);
 }
 
+// The status word as it stands after a pull, into the caller's pinned host
+// word (host-buffer pulls then need no separate copy).
+__device__ inline void mirror_status(const PullArgs& a) {
+    __syncthreads();
+    if (threadIdx.x == 0 && a.status_mirror)
+        *reinterpret_cast<volatile int*>(a.status_mirror) = *reinterpret_cast<volatile int*>(a.status);
+}
+
 __device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {
     if (threadIdx.x == 0) a.ctr->front_k = 0;   // rows leave without the frontier's count
     pull_emit_list(a, sh, a.cand, a.ctr->cand);
+    mirror_status(a);
 }
 
 __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) {
@@ -645,6 +654,7 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
             set_status(a.status, PVS_ERR_INVALID);
             a.ctr->cand = 0;
         }
+        mirror_status(a);
         return;
     }
     if (mode == 1 && threadIdx.x == 0) {
@@ -670,6 +680,7 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
             a.front[e] = (int32_t)(uint32_t)sh.sk[e];
     __syncthreads();   // sh.sk is the emission's sort buffer
     pull_emit_list(a, sh, cand, c);
+    mirror_status(a);
 }
 
 __global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThreads, 2)

@@ -417,7 +417,10 @@ pvs_status prepare_pull(pvs_cursor* c, int64_t n_eff) {
     return PVS_OK;
 }
 
-pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
+// status_mirror: a pinned host word the one-launch path sets to the status
+// after the pull (host-buffer pulls); null for device-buffer pulls.
+pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores,
+                int* status_mirror = nullptr) {
     pvs_index* x = c->index;
     cudaStream_t st = c->stream;
     pvs_status s = prepare_pull(c, n_eff);
@@ -442,6 +445,7 @@ pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores) {
         a.status = c->d_status;
         a.ctr = c->ctr;
         a.front = c->front;
+        a.status_mirror = status_mirror;
         // the first pull of a working set refines most of it: spread that
         // over every SM; later pulls take one cluster launch
         cudaError_t e = c->fresh_ws ? launch_pull_fused(a, 2 * x->num_sms, st)
@@ -1241,6 +1245,7 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         a.status = c->d_status;
         a.ctr = c->ctr;
         a.front = nullptr;   // a few pulls per batch: a frontier would not pay for itself
+        a.status_mirror = nullptr;
         args.push_back(a);
         who.push_back(i);
     }
@@ -1298,7 +1303,23 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
     if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
-    if (n_eff > 0) {
+    if (n_eff > 0 && n_eff <= kPullFusedMax) {
+        // the kernels write ids, scores and the status word straight into the
+        // cursor's pinned host buffers: one launch, one wait
+        s = cursor_out_reserve(c, n_eff);
+        if (s != PVS_OK) return fail(c, s);
+        int* mirror = reinterpret_cast<int*>(c->h_small) + 2;
+        *mirror = 0;
+        s = pull(c, n_eff, c->h_ids, c->h_scores, mirror);
+        if (s != PVS_OK) return s;
+        cudaError_t e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        harvest_interval_time(c);
+        const int dev_status = *reinterpret_cast<volatile int*>(mirror);
+        if (dev_status != 0) return fail(c, (pvs_status)dev_status);
+        std::memcpy(ids, c->h_ids, n_eff * sizeof(int64_t));
+        std::memcpy(scores, c->h_scores, n_eff * sizeof(float));
+    } else if (n_eff > 0) {
         s = cursor_out_reserve(c, n_eff);
         if (s != PVS_OK) return fail(c, s);
         s = pull(c, n_eff, c->d_ids, c->d_scores);
