@@ -82,6 +82,27 @@ def dist_env():
     return rank, world, local
 
 
+def query_seed(base: int, rank: int) -> int:
+    """Every rank draws its own queries (weak scaling: the work is sharded by
+    query, each rank against its own replica of the index)."""
+    return base + 7919 * rank
+
+
+def slowest(pg, seconds: float, device) -> float:
+    """The job's time: the maximum over ranks (no-op without a process group)."""
+    if pg is None:
+        return seconds
+    import torch
+    t = torch.tensor([seconds], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput: every rank's units over the slowest rank's time."""
+    return units_per_rank * world / seconds
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -374,7 +395,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev,
                                                  components=BATCH_COMPONENTS, seed=4)
     nb = args.warmup + args.steps
-    queries = synth.mixture_queries(nb * BATCH_Q, centres, QUERY_NOISE, seed=5 + 7919 * rank)
+    queries = synth.mixture_queries(nb * BATCH_Q, centres, QUERY_NOISE, seed=query_seed(5, rank))
     queries = queries.reshape(nb, BATCH_Q, DIM).contiguous()
     streams = [torch.cuda.Stream(device=dev) for _ in range(BATCH_PIPELINE)]
     ids_t = torch.empty((BATCH_PIPELINE, BATCH_Q, BATCH_CHUNK), dtype=torch.int64, device=dev)
@@ -427,12 +448,9 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     stats = []   # per-query counters from one more (untimed) batch of the same queries
     step(queries[args.warmup], 0, None, stats)
     elapsed = start.elapsed_time(end) / 1e3
-    if pg:
-        t = torch.tensor([elapsed], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = slowest(pg, elapsed, dev)
     ranks_total = args.steps * BATCH_Q * BATCH_RANKS * world
-    value = ranks_total / elapsed
+    value = job_rate(args.steps * BATCH_Q * BATCH_RANKS, world, elapsed)
 
     # e2e: host queries, host outputs, the same threads and streams
     qh = [np.ascontiguousarray(queries[b].cpu().numpy()) for b in range(nb)]
@@ -515,7 +533,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     torch.cuda.synchronize()
     build_s = time.perf_counter() - t0
     total_q = 2 * args.eahr_queries + args.eahr_exhaust_queries + 2
-    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=3 + 7919 * rank)
+    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
 
     def sparse_for(q, tau, seed):
         proxy = rows @ q
@@ -557,7 +575,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
             for j in range(count):
                 q = queries[qi]
                 qi += 1
-                sp, proxy = sparse_for(q, tau, 1000 + 7919 * rank + qi)
+                sp, proxy = sparse_for(q, tau, query_seed(1000, rank) + qi)
                 if j == 0:   # realised Kendall tau of the generated channel
                     dense_order = torch.argsort(proxy, descending=True, stable=True).cpu().numpy()
                     ktau = synth.kendall_tau_sample(dense_order, sp, 200_000, seed=qi)
@@ -648,7 +666,7 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     visible[n0:] = False
     rng = np.random.default_rng(57 + rank)
     queries = synth.mixture_queries(SNAP_STEPS * args.snap_queries + 2, centres, QUERY_NOISE,
-                                    seed=58 + 7919 * rank)
+                                    seed=query_seed(58, rank))
     launches0 = pvs.pvs_launch_count()
     per_snap = []
     size = n0
@@ -773,7 +791,7 @@ def main():
     n = args.n
     index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev)
     total_q = (args.warmup + args.steps) * args.queries
-    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=3 + 7919 * rank)
+    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
     queries = queries.reshape(args.warmup + args.steps, args.queries, DIM).contiguous()
     out_ids = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
     out_scores = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
@@ -807,12 +825,9 @@ def main():
     torch.cuda.synchronize()
     launches = pvs.pvs_launch_count() - launches0
     elapsed = start.elapsed_time(end) / 1e3
-    if pg:
-        t = torch.tensor([elapsed], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = slowest(pg, elapsed, dev)
     ranks_total = args.steps * args.queries * RANKS_PER_QUERY * world
-    value = ranks_total / elapsed
+    value = job_rate(args.steps * args.queries * RANKS_PER_QUERY, world, elapsed)
 
     # ---- e2e: host query buffers, host outputs through pvs_next ----
     qh = [np.ascontiguousarray(queries[args.warmup + s].cpu().numpy()) for s in range(args.steps)]
@@ -828,10 +843,7 @@ def main():
     # ---- latency, one query at a time ----
     lat20, lat1000 = measure_latency(pvs, torch, index, queries[args.warmup],
                                      out_ids, out_scores, stream, min(args.queries, 20))
-    if pg:
-        t = torch.tensor([e2e_elapsed], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_elapsed = float(t.item())
+    e2e_elapsed = slowest(pg, e2e_elapsed, dev)
     e2e_value = ranks_total / e2e_elapsed
 
     # ---- roofline of the interval pass ----
