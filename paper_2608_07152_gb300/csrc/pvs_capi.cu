@@ -165,6 +165,14 @@ pvs_status index_fill(pvs_index* x, const float* vecs, int64_t n, bool on_device
     return (pvs_status)st;
 }
 
+// Corpus maxima of the norm bounds over rows [0, size); waits for them.
+pvs_status refresh_norm_maxes(pvs_index* x) {
+    if (!x->norm_maxes) PVS_CUDA(dev_alloc(&x->norm_maxes, 2));
+    PVS_CUDA(launch_norm_max(x->vnorm, x->enorm, x->size, x->norm_maxes, x->stream));
+    PVS_CUDA(cudaStreamSynchronize(x->stream));
+    return PVS_OK;
+}
+
 std::shared_ptr<SnapData> make_snapdata(const pvs_index* x) {
     auto s = std::make_shared<SnapData>();
     s->rows = x->size;
@@ -732,24 +740,23 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     }
 
     // Sample every stride-th tile and take tau_q = the k_s-th largest sampled
-    // lower bound, k_s = 1.5 H / stride + 4: about 1.5 H rows of the corpus
-    // reach it.  It misses the horizon (fewer than H rows reach it) only when
-    // at least k_s of the top-H rows were sampled; that count is about
-    // Poisson(H / stride), so this happens for well under 1 % of the queries
-    // (H = 200: stride 12, k_s = 29, mean 16.7), which then rescan.
+    // lower bound, k_s = 2 H / stride + 4: about 2 H rows of the corpus reach
+    // it.  It misses the horizon (fewer than H rows reach it) only when at
+    // least k_s of the top-H rows were sampled; that count is about
+    // Poisson(H / stride), so this happens for about 1e-5 of the queries
+    // (H = 200: stride 12, k_s = 38, mean 16.7), which then rescan.
     const int64_t ntiles = (rows + 127) / 128;
     int stride = (int)std::min<int64_t>(16, std::max<int64_t>(1, (3 * (int64_t)horizon) / 48));
     if (ntiles < 8 * (int64_t)stride) stride = 1;
     const int64_t ld = ((ntiles + stride - 1) / stride) * 128;
     const unsigned int k_s =
         stride == 1 ? (unsigned int)horizon
-                    : (unsigned int)((3 * (int64_t)horizon + 2 * stride - 1) / (2 * stride) + 4);
+                    : (unsigned int)((2 * (int64_t)horizon + stride - 1) / stride + 4);
     const int w_cap = (int)std::min<int64_t>((int64_t)kWsSortMax, std::max<int64_t>(rows, 1));
     float* dlo = buf.get<float>((size_t)nq * ld);
     float* dhi = dlo;   // the sampling pass needs the lower bounds only
     float* tau = buf.get<float>((size_t)nq);
     float* rmax = buf.get<float>((size_t)nq);
-    unsigned int* maxes = buf.get<unsigned int>(2);
     int* status = buf.get<int>(1);
     int32_t* wid = buf.get<int32_t>((size_t)nq * w_cap);
     float* wlo = buf.get<float>((size_t)nq * w_cap);
@@ -757,7 +764,7 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     unsigned int* wlen = buf.get<unsigned int>((size_t)nq);
     unsigned int* heff = buf.get<unsigned int>((size_t)nq);
     WsDst* d_ws = buf.get<WsDst>((size_t)nq);
-    if (!dlo || !dhi || !tau || !rmax || !maxes || !status || !wid || !wlo || !whi || !wlen ||
+    if (!dlo || !dhi || !tau || !rmax || !status || !wid || !wlo || !whi || !wlen ||
         !heff || !d_ws)
         return PVS_ERR_OOM;
     PVS_CUDA(cudaMemsetAsync(status, 0, sizeof(int), st));
@@ -783,8 +790,7 @@ pvs_status open_batch_group(pvs_index* x, const std::shared_ptr<SnapData>& sd,
     a.dump_ld = ld;
     PVS_CUDA(launch_batch_intervals(a, x->codes_bf16, bq.qcodes, x->num_sms, st));
     PVS_CUDA(launch_batch_tau(dlo, ld, (unsigned int)ld, nq, k_s, tau, st));
-    PVS_CUDA(launch_norm_max(x->vnorm, x->enorm, rows, maxes, st));
-    PVS_CUDA(launch_rmax(bq.qs, nq, maxes, rmax, st));
+    PVS_CUDA(launch_rmax(bq.qs, nq, x->norm_maxes, rmax, st));   // maxima over all rows: a valid bound
     // 3. the filter pass over every row
     a.mode = 1;
     a.tile_stride = 1;
@@ -949,6 +955,8 @@ pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_
     if (s != PVS_OK) return bail(s);
     x->size = n;
     x->live = n;
+    s = refresh_norm_maxes(x);
+    if (s != PVS_OK) return bail(s);
     *out = x;
     return PVS_OK;
 }
@@ -965,7 +973,7 @@ pvs_status pvs_append(pvs_index* x, const float* vecs, int64_t n, int32_t vecs_o
     if (s != PVS_OK) return s;
     x->size += n;
     x->live += n;
-    return PVS_OK;
+    return refresh_norm_maxes(x);
 }
 
 pvs_status pvs_tombstone(pvs_index* x, const int64_t* ids, int64_t n) {
@@ -1022,6 +1030,7 @@ void pvs_index_free(pvs_index* x) {
     if (x->pass_done) cudaEventDestroy(x->pass_done);
     if (x->scratch_pool) cudaMemPoolDestroy(x->scratch_pool);
     if (x->bf16_ready) cudaEventDestroy(x->bf16_ready);
+    dev_free(x->norm_maxes);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
 }

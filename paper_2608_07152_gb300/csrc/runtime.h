@@ -54,6 +54,9 @@ struct pvs_index {
     uint16_t* codes_bf16 = nullptr;         // [cap][m_pad]
     int64_t bf16_rows = 0;                  // rows converted so far
     cudaEvent_t bf16_ready = nullptr;       // end of the last conversion (any stream)
+    // max vnorm and max enorm (float bits) over every row; refreshed by build and
+    // append (upper bounds for any snapshot), read by the batched pass
+    unsigned int* norm_maxes = nullptr;
     // stream-ordered scratch of batched calls; keeps its memory between calls
     // (the device's default pool hands memory back at every synchronisation)
     cudaMemPool_t scratch_pool = nullptr;
