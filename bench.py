@@ -349,7 +349,7 @@ BATCH_COMPONENTS = 1024
 BATCH_Q = 256
 BATCH_RANKS = 200
 BATCH_CHUNK = 50
-BATCH_PIPELINE = 2   # batches in flight, each driven by its own host thread and stream
+BATCH_PIPELINE = 4   # batches in flight, each driven by its own host thread and stream
 BATCH_WORKLOAD = ("batched queries: N=1,000,000 x d=768 Gaussian mixture (1,024 components, "
                   "within std 0.35), 256 concurrent queries per batch, first 200 exact ranks "
                   "per query in chunks of 50")

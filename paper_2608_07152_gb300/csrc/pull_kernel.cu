@@ -336,7 +336,7 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const 
     pull_emit_body(args[blockIdx.x], sh);
 }
 
-// ---- one launch per pull: a cluster of kPullCluster CTAs ----------------------
+// ---- one launch per pull: a cluster of CTAs per cursor -------------------------
 // Every CTA of the cluster derives tau and the candidate list itself (the same
 // set; its order may differ), refines the candidates it owns (working-set
 // index modulo the cluster's warps), and after a cluster barrier with
@@ -348,8 +348,8 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const 
 //   lo >= t0 among them); tau is the n-th largest lower bound of the gathered
 //   rows and the candidates are those with hi >= tau.  If more rows than
 //   kPullSortCap reach t0, CTA 0 runs the radix selection instead.
-constexpr int kPullCluster = 8;
-constexpr int kPullClusterWarps = kPullCluster * kPullWarps;
+constexpr int kPullCluster = 8;        // single cursor: the whole pull in one cluster of 8
+constexpr int kPullClusterBatch = 2;   // batched pulls: many cursors at once, 2 CTAs each
 
 __device__ inline uint32_t cluster_ctarank() {
     uint32_t r;
@@ -569,7 +569,7 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
 
 // Exact scores of the candidates this warp owns (index modulo the cluster's warps).
 __device__ inline void cluster_refine(const PullArgs& a, const int32_t* cand, unsigned int c,
-                                      unsigned int gwarp) {
+                                      unsigned int gwarp, unsigned int cluster_warps) {
     const int lane = threadIdx.x & 31;
     unsigned long long refined = 0, fallbacks = 0;
     for (unsigned int j0 = 0; j0 < c; j0 += 32) {
@@ -579,7 +579,7 @@ __device__ inline void cluster_refine(const PullArgs& a, const int32_t* cand, un
         bool own = false;
         if (j < c) {
             w = cand[j];
-            if ((unsigned int)w % kPullClusterWarps == gwarp) {
+            if ((unsigned int)w % cluster_warps == gwarp) {
                 l = a.w_lo[w];
                 h = a.w_hi[w];
                 id = a.w_id[w];
@@ -630,6 +630,7 @@ static __device__ __noinline__ void pull_select_radix(const PullArgs& a, PullSha
     pull_select_body(a, sh);
 }
 
+template <int kCtas>
 __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
     const uint32_t rank = cluster_ctarank();
     const FastSelect fs = pull_select_fast(a, sh);
@@ -646,7 +647,7 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
     }
     const int32_t* cand = mode == 1 ? reinterpret_cast<const int32_t*>(sh.hist) : a.cand;
     const unsigned int c = mode == 1 ? sh.cand_n : (mode == 0 ? a.ctr->cand : 0u);
-    cluster_refine(a, cand, c, rank * kPullWarps + (threadIdx.x >> 5));
+    cluster_refine(a, cand, c, rank * kPullWarps + (threadIdx.x >> 5), kCtas * kPullWarps);
     cluster_barrier();   // every exact score is visible to CTA 0
     if (rank != 0) return;
     if (mode == -1) {    // fewer than n live rows: the working set was too small
@@ -686,14 +687,14 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
 __global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThreads, 2)
     pull_cluster_kernel(PullArgs a) {
     __shared__ PullShared sh;
-    pull_cluster_body(a, sh);
+    pull_cluster_body<kPullCluster>(a, sh);
 }
 
 // One cluster per cursor.
-__global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThreads, 2)
+__global__ void __cluster_dims__(kPullClusterBatch, 1, 1) __launch_bounds__(kPullThreads, 2)
     pull_cluster_batch_kernel(const PullArgs* args) {
     __shared__ PullShared sh;
-    pull_cluster_body(args[blockIdx.x / kPullCluster], sh);
+    pull_cluster_body<kPullClusterBatch>(args[blockIdx.x / kPullClusterBatch], sh);
 }
 
 cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
@@ -707,7 +708,7 @@ cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
 cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
     count_launches(1);
-    pull_cluster_batch_kernel<<<ncursors * kPullCluster, kPullThreads, 0, st>>>(args_dev);
+    pull_cluster_batch_kernel<<<ncursors * kPullClusterBatch, kPullThreads, 0, st>>>(args_dev);
     return cudaGetLastError();
 }
 
