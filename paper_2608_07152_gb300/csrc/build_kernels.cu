@@ -102,7 +102,9 @@ cudaError_t launch_encode_queries(const float* q, int nq, int m, int m_pad, int 
                                   int8_t* zq, float* qraw, QueryScalars* qs, cudaStream_t st) {
     if (nq <= 0) return cudaSuccess;
     count_launches(1);
-    encode_kernel<<<(nq + 7) / 8, 256, 0, st>>>(q, nq, m, m_pad, m_raw, zq, qraw, qs);
+    // one warp per block: the queries spread over every SM (their norm bounds
+    // use binary64, whose per-SM rate is low on this part)
+    encode_kernel<<<nq, 32, 0, st>>>(q, nq, m, m_pad, m_raw, zq, qraw, qs);
     return cudaGetLastError();
 }
 
