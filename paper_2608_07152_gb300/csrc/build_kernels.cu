@@ -45,48 +45,135 @@ cudaError_t launch_build(const float* vecs, int64_t n, int m, int m_pad, int m_r
     return cudaGetLastError();
 }
 
-// Query encoding: the same quantizer, plus ||s_q z_q|| rounded up and
-// gamma_m = RU(a / RD(1 - a)), a = (8m + 64) 2^-23 (App. A.1).
+// Queries: one block of kEncThreads per query, the quantizer of
+// quantize_row_warp spread over its warps (maxima and exact integer sums do
+// not depend on the order, so the results are bit-identical), plus the
+// query-side scalars of App. A.1: ||s_q z_q|| rounded up and
+// gamma_m = RU(a / RD(1 - a)), a = (8m + 64) 2^-23.
 // q and qraw may be the same buffer (a host query staged in qraw): the raw
-// copy then rewrites the values it read.
-__global__ void encode_kernel(const float* q, int nq, int m, int m_pad, int m_raw,
-                              int8_t* __restrict__ zq, float* qraw,
-                              QueryScalars* __restrict__ qs) {
-    const int lane = threadIdx.x & 31;
-    const int qi = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+// copy, after every read of the first pass, rewrites the values it read.
+constexpr int kEncThreads = 256;
+constexpr int kEncWarps = kEncThreads / kWarp;
+
+__global__ void __launch_bounds__(kEncThreads) encode_kernel(const float* q, int nq, int m,
+                                                            int m_pad, int m_raw,
+                                                            int8_t* __restrict__ zq, float* qraw,
+                                                            QueryScalars* __restrict__ qs) {
+    __shared__ float s_f[kEncWarps];
+    __shared__ double s_d[kEncWarps];
+    __shared__ long long s_a[kEncWarps], s_b[kEncWarps];
+    __shared__ int s_i[kEncWarps];
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int qi = blockIdx.x;
     if (qi >= nq) return;
     const float* v = q + (int64_t)qi * m;
     int8_t* z = zq + (int64_t)qi * m_pad;
-    RowQuant r = quantize_row_warp(v, m, m_pad, z);
-    float* dst = qraw + (int64_t)qi * m_raw;
-    for (int j = lane; j < m_raw; j += kWarp) dst[j] = j < m ? v[j] : 0.0f;
-    __syncwarp();
-    // ||q_hat||: values s_q z_j are exact in binary64
-    float qhat = 0.0f;
-    if (r.status == 0) {
-        double M = 0.0;
-        for (int j = lane; j < m; j += kWarp)
-            M = fmax(M, fabs(__dmul_rn((double)r.s, (double)z[j])));
-        M = warp_max(M);
-        long long T = 0;
-        int e = M > 0.0 ? norm_exponent(M) : 0;
-        if (M > 0.0)
-            for (int j = lane; j < m; j += kWarp)
-                T += norm_term(__dmul_rn((double)r.s, (double)z[j]), e);
-        T = warp_sum(T);
-        qhat = norm_finish(T, e);
-        if (isinf(qhat)) r.status = PVS_ERR_OVERFLOW;
+    auto block_max_f = [&](float x) {
+        x = warp_max(x);
+        if (lane == 0) s_f[warp] = x;
+        __syncthreads();
+        float r = s_f[0];
+        for (int w = 1; w < kEncWarps; ++w) r = fmaxf(r, s_f[w]);
+        __syncthreads();
+        return r;
+    };
+    auto block_max_d = [&](double x) {
+        x = warp_max(x);
+        if (lane == 0) s_d[warp] = x;
+        __syncthreads();
+        double r = s_d[0];
+        for (int w = 1; w < kEncWarps; ++w) r = fmax(r, s_d[w]);
+        __syncthreads();
+        return r;
+    };
+    auto block_sum2 = [&](long long& x, long long& y) {
+        x = warp_sum(x);
+        y = warp_sum(y);
+        if (lane == 0) {
+            s_a[warp] = x;
+            s_b[warp] = y;
+        }
+        __syncthreads();
+        x = 0;
+        y = 0;
+        for (int w = 0; w < kEncWarps; ++w) {
+            x += s_a[w];
+            y += s_b[w];
+        }
+        __syncthreads();
+    };
+    // finiteness and max |q_j|
+    float maxabs = 0.0f;
+    bool finite = true;
+    for (int j = t; j < m; j += kEncThreads) {
+        const float x = v[j];
+        finite &= isfinite(x);
+        maxabs = fmaxf(maxabs, fabsf(x));
     }
-    if (lane == 0) {
-        float a = (float)((8.0 * (double)m + 64.0) * 0x1p-23);   // exact
-        float den = __fsub_rd(1.0f, a);
-        QueryScalars out;
-        out.s = r.s;
-        out.qnorm = r.vnorm;
-        out.qhat = qhat;
-        out.enorm = r.enorm;
-        out.gamma = __fdiv_ru(a, den);
-        out.status = r.status;
+    finite = __all_sync(0xffffffffu, finite);
+    if (lane == 0) s_i[warp] = finite;
+    maxabs = block_max_f(maxabs);   // (its barrier publishes s_i)
+    for (int w = 0; w < kEncWarps; ++w) finite &= s_i[w] != 0;
+    for (int j = t; j < m_raw; j += kEncThreads) qraw[(int64_t)qi * m_raw + j] = j < m ? v[j] : 0.0f;
+    QueryScalars out{};
+    out.status = 0;
+    if (finite) {
+        float s;
+        if (maxabs == 0.0f) {
+            s = 1.0f;
+        } else {
+            s = __fdiv_rn(maxabs, 127.0f);
+            if (s == 0.0f) s = __uint_as_float(1u);  // 2^-149
+        }
+        // codes and residual maximum (each thread later reads only its own codes)
+        double emax = 0.0;
+        for (int j = t; j < m_pad; j += kEncThreads) {
+            int c = 0;
+            if (j < m && maxabs != 0.0f) {
+                const float tq = __fdiv_rn(v[j], s);
+                float rt = roundf(tq);                     // half away from zero
+                rt = fminf(fmaxf(rt, -127.0f), 127.0f);
+                c = (int)rt;
+                const double e = __dsub_rn((double)v[j], __dmul_rn((double)s, (double)c));  // exact
+                emax = fmax(emax, fabs(e));
+            }
+            z[j] = (int8_t)c;
+        }
+        emax = block_max_d(emax);
+        // norm bounds of q and of its residual
+        long long Tv = 0, Te = 0;
+        const int ev = maxabs > 0.0f ? norm_exponent((double)maxabs) : 0;
+        const int ee = emax > 0.0 ? norm_exponent(emax) : 0;
+        for (int j = t; j < m; j += kEncThreads) {
+            const double x = (double)v[j];
+            if (maxabs > 0.0f) Tv += norm_term(x, ev);
+            if (emax > 0.0) {
+                const int c = z[j];
+                Te += norm_term(__dsub_rn(x, __dmul_rn((double)s, (double)c)), ee);
+            }
+        }
+        block_sum2(Tv, Te);
+        out.s = s;
+        out.qnorm = norm_finish(Tv, ev);
+        out.enorm = norm_finish(Te, ee);
+        if (isinf(out.qnorm) || isinf(out.enorm)) out.status = PVS_ERR_OVERFLOW;
+        // ||q_hat||: the values s z_j are exact in binary64
+        double M = 0.0;
+        for (int j = t; j < m; j += kEncThreads) M = fmax(M, fabs(__dmul_rn((double)s, (double)z[j])));
+        M = block_max_d(M);
+        long long T = 0, unused = 0;
+        const int e = M > 0.0 ? norm_exponent(M) : 0;
+        if (M > 0.0)
+            for (int j = t; j < m; j += kEncThreads) T += norm_term(__dmul_rn((double)s, (double)z[j]), e);
+        block_sum2(T, unused);
+        out.qhat = norm_finish(T, e);
+        if (out.status == 0 && isinf(out.qhat)) out.status = PVS_ERR_OVERFLOW;
+    } else {
+        out.status = PVS_ERR_NONFINITE;
+    }
+    if (t == 0) {
+        const float a = (float)((8.0 * (double)m + 64.0) * 0x1p-23);   // exact
+        out.gamma = __fdiv_ru(a, __fsub_rd(1.0f, a));
         qs[qi] = out;
     }
 }
@@ -94,7 +181,7 @@ __global__ void encode_kernel(const float* q, int nq, int m, int m_pad, int m_ra
 cudaError_t launch_encode_query(const float* q, int m, int m_pad, int m_raw, int8_t* zq,
                                 float* qraw, QueryScalars* qs, cudaStream_t st) {
     count_launches(1);
-    encode_kernel<<<1, 32, 0, st>>>(q, 1, m, m_pad, m_raw, zq, qraw, qs);
+    encode_kernel<<<1, kEncThreads, 0, st>>>(q, 1, m, m_pad, m_raw, zq, qraw, qs);
     return cudaGetLastError();
 }
 
@@ -102,9 +189,7 @@ cudaError_t launch_encode_queries(const float* q, int nq, int m, int m_pad, int 
                                   int8_t* zq, float* qraw, QueryScalars* qs, cudaStream_t st) {
     if (nq <= 0) return cudaSuccess;
     count_launches(1);
-    // one warp per block: the queries spread over every SM (their norm bounds
-    // use binary64, whose per-SM rate is low on this part)
-    encode_kernel<<<nq, 32, 0, st>>>(q, nq, m, m_pad, m_raw, zq, qraw, qs);
+    encode_kernel<<<nq, kEncThreads, 0, st>>>(q, nq, m, m_pad, m_raw, zq, qraw, qs);
     return cudaGetLastError();
 }
 
