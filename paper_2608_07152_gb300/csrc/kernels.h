@@ -40,11 +40,12 @@ struct DevCounters {
     // frontier carried between one-launch pulls: every live working-set row
     // with hi >= front_bound (a float key) is among the front_n entries of
     // PullArgs::front, and at least front_k live rows have lo >= front_bound;
-    // front_k == 0: no frontier
+    // front_k == 0: no frontier.  front_hint: the multiple of n the next
+    // whole-set gather starts with (0: the widest).
     unsigned int front_n;
     unsigned int front_bound;
     unsigned int front_k;
-    unsigned int front_pad;
+    unsigned int front_hint;
 };
 
 // Where one cursor keeps its device status word and counters.
@@ -88,7 +89,7 @@ cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int bloc
 
 // ---- batched open support (pull_kernel.cu, batch_support.cu) ----------------
 constexpr int kWsSortMax = 8192;     // largest per-query working set of a batched open
-constexpr int kFrontCap = 2048;      // frontier entries (the one-launch pull's gather capacity)
+constexpr int kFrontCap = 4096;      // frontier entries (the one-launch pull's gather capacity)
 struct WsDst {                       // a cursor's working-set arrays
     int32_t* w_id;
     float* w_lo;

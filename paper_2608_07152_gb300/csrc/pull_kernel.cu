@@ -374,20 +374,25 @@ __device__ inline void cluster_barrier_relaxed() {
 // Rows whose lower bound may reach the frontier bound: kFrontMult times the
 // ranks of the pull that builds it (the frontier then serves later pulls).
 constexpr int kFrontMult = 6;
-static_assert(kFrontCap == kPullSortCap, "the frontier is the gathered set");
+// The gather keeps working-set indices only (in the bytes of sh.sk): twice the
+// rows of (key, index) pairs in the same shared memory.
+constexpr int kGatherCap = kPullSortCap * 2;
+static_assert(kFrontCap == kGatherCap, "the frontier is the gathered set");
 
 struct FastSelect {
     int mode;            // 1: list in sh.hist (sh.cand_n entries); 0: radix fallback; -1: < n live
     bool from_front;     // the rows came from the carried frontier
-    bool new_front;      // a whole-set gather at the wide bound: it can become the frontier
+    bool new_front;      // a whole-set gather at a wide bound: it can become the frontier
     uint32_t t0;         // the bound of the gather
     unsigned int g;      // rows gathered (hi >= t0)
     unsigned int l;      // of them with lo >= t0
+    unsigned int mult;   // the gather's bound was for mult * n rows (1: the tight bound)
 };
 
 // Gather, with one shared-memory atomic per row that reaches t0 (few do),
-// (hi key, index) of the live rows with hi >= t0 into sh.sk (count sh.count)
-// and the lo keys of those with lo >= t0 into sh.hist (count sh.cand_n).
+// the working-set indices of the live rows with hi >= t0 into the bytes of
+// sh.sk (count sh.count, capacity kGatherCap) and the lo keys of those with
+// lo >= t0 into sh.hist (count sh.cand_n, capacity kPullSortCap).
 // Rows: the frontier's len entries, or working-set indices 0 .. len-1.
 __device__ inline void gather_rows(const PullArgs& a, PullShared& sh, bool from_front,
                                    unsigned int len, uint32_t t0) {
@@ -397,7 +402,7 @@ __device__ inline void gather_rows(const PullArgs& a, PullShared& sh, bool from_
         const uint32_t hk = fkey(h);
         if (hk < t0) return;
         const unsigned int pos = atomicAdd(&sh.count, 1u);
-        if (pos < (unsigned int)kPullSortCap) sh.sk[pos] = ((unsigned long long)hk << 32) | i;
+        if (pos < (unsigned int)kGatherCap) reinterpret_cast<uint32_t*>(sh.sk)[pos] = i;
         const uint32_t lk = fkey(l);
         if (lk >= t0) {
             const unsigned int q = atomicAdd(&sh.cand_n, 1u);
@@ -435,12 +440,15 @@ __device__ inline void gather_rows(const PullArgs& a, PullShared& sh, bool from_
 __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int n = a.n;
-    FastSelect r{1, false, false, 0u, 0u, 0u};
+    FastSelect r{1, false, false, 0u, 0u, 0u, 1u};
     const unsigned int fk = a.ctr->front_k;
     r.from_front = a.front != nullptr && fk >= (unsigned int)n;
     r.new_front = !r.from_front && a.front != nullptr;
     unsigned int len;
-    uint32_t t0_tight = 0;   // whole-set pass: the bound for n rows (t0 is for kFrontMult n)
+    // whole-set pass: bounds for mult * n rows, widest first; the cursor's hint
+    // (front_hint) starts deep cursors, whose wide gathers overflow, lower
+    const unsigned int hint = a.ctr->front_hint == 3u ? 3u : (unsigned int)kFrontMult;
+    uint32_t t0_mid = 0, t0_tight = 0;
     if (r.from_front) {
         len = a.ctr->front_n;
         r.t0 = a.ctr->front_bound;
@@ -478,9 +486,11 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
         // bound; R = kFrontMult n, at most their j2 values each, the wide one.
         // Threads without live rows list zeros (a bound of 0 gathers every row).
         const int j1 = min(32, (n + busy_warps - 1) / busy_warps);
-        const int j2 = r.new_front ? max(j1, min(32, (kFrontMult * n + busy_warps - 1) / busy_warps))
-                                   : j1;
-        const unsigned int r2 = min((unsigned int)(kFrontMult * n), (unsigned int)(busy_warps * j2));
+        const int j2 = r.new_front
+                           ? max(j1, min(32, ((int)hint * n + busy_warps - 1) / busy_warps))
+                           : j1;
+        const unsigned int r2 = min(hint * (unsigned int)n, (unsigned int)(busy_warps * j2));
+        const unsigned int rm = min(3u * (unsigned int)n, r2);
         for (int it = 0; it < j2; ++it) {
             const uint32_t top = __reduce_max_sync(0xffffffffu, mx);
             const unsigned int holders = __ballot_sync(0xffffffffu, mx == top);
@@ -493,6 +503,7 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
             sh.ok = 0;
             sh.warp_tot[0] = 0;   // wide bound
             sh.warp_tot[1] = 0;   // tight bound
+            sh.warp_tot[2] = 0;   // middle bound (3 n rows)
         }
         __syncthreads();
         const int nv = kPullWarps * j2;
@@ -508,26 +519,36 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
                 ge1 += first && u >= v;
             }
             if (gt < r2 && r2 <= ge) sh.warp_tot[0] = v;                       // same value from every writer
+            if (gt < rm && rm <= ge) sh.warp_tot[2] = v;
             if ((e % j2) < j1 && gt1 < (unsigned int)n && (unsigned int)n <= ge1) sh.warp_tot[1] = v;
         }
         __syncthreads();
         r.t0 = sh.warp_tot[0];
+        r.mult = r.new_front ? hint : 1u;
+        t0_mid = sh.warp_tot[2];
         t0_tight = sh.warp_tot[1];
         __syncthreads();   // sh.hist is the gather's buffer
     }
-    for (int attempt = 0;; ++attempt) {
+    for (;;) {
         gather_rows(a, sh, r.from_front, len, r.t0);
         r.g = sh.count;
         r.l = sh.cand_n;
-        if (r.g <= (unsigned int)kPullSortCap) break;
-        if (r.from_front || attempt > 0 || t0_tight <= r.t0) {
+        if (r.g <= (unsigned int)kGatherCap && r.l <= (unsigned int)kPullSortCap) break;
+        // too many rows reach this bound: gather again at the next tighter one
+        // (3 n rows, still a frontier; then n rows, none)
+        uint32_t next = 0;
+        if (!r.from_front && r.mult > 3u && t0_mid > r.t0) {
+            next = t0_mid;
+            r.mult = 3u;
+        } else if (!r.from_front && r.mult > 1u && t0_tight > r.t0) {
+            next = t0_tight;
+            r.mult = 1u;
+            r.new_front = false;
+        } else {
             r.mode = 0;
             return r;
         }
-        // too many rows reach the wide bound: gather again at the bound for
-        // n rows (no frontier from this pull)
-        r.t0 = t0_tight;
-        r.new_front = false;
+        r.t0 = next;
         __syncthreads();
         if (t == 0) {
             sh.count = 0;
@@ -536,9 +557,40 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
         __syncthreads();
     }
     // tau: the lower-bound key v with #{> v} < n <= #{>= v} among the l rows
-    // with lo >= t0 (the n-th largest is one of them when l >= n)
+    // with lo >= t0 (the n-th largest is one of them when l >= n).  Counting
+    // is quadratic in l; for a long list a bound t_sub <= the n-th largest
+    // (the n-th largest of the warps' listed top thread maxima, listed past
+    // the keys) leaves only the entries >= t_sub to count.
+    uint32_t t_sub = 0;
+    const int jn = (n + kPullWarps - 1) / kPullWarps;
+    if (r.l > 256 && r.l + (unsigned int)(kPullWarps * jn) <= (unsigned int)kPullSortCap) {
+        uint32_t mx = 0;
+        for (unsigned int e = t; e < r.l; e += kPullThreads) mx = max(mx, sh.hist[e]);
+        uint32_t* listed = sh.hist + r.l;
+        for (int it = 0; it < jn; ++it) {
+            const uint32_t top = __reduce_max_sync(0xffffffffu, mx);
+            const unsigned int holders = __ballot_sync(0xffffffffu, mx == top);
+            if (lane == __ffs(holders) - 1) mx = 0;
+            if (lane == 0) listed[warp * jn + it] = top;
+        }
+        if (t == 0) sh.warp_tot[2] = 0;
+        __syncthreads();
+        const int nv = kPullWarps * jn;
+        for (int e = t; e < nv; e += kPullThreads) {
+            const uint32_t v = listed[e];
+            unsigned int gt = 0, ge = 0;
+            for (int f = 0; f < nv; ++f) {
+                gt += listed[f] > v;
+                ge += listed[f] >= v;
+            }
+            if (gt < (unsigned int)n && (unsigned int)n <= ge) sh.warp_tot[2] = v;
+        }
+        __syncthreads();
+        t_sub = sh.warp_tot[2];
+    }
     for (unsigned int e = t; e < r.l; e += kPullThreads) {
         const uint32_t le = sh.hist[e];
+        if (le < t_sub) continue;   // below the n-th largest
         unsigned int gt = 0, ge = 0;
         for (unsigned int f = 0; f < r.l; ++f) {
             const uint32_t lf = sh.hist[f];
@@ -558,12 +610,19 @@ __device__ inline FastSelect pull_select_fast(const PullArgs& a, PullShared& sh)
     const uint32_t tau = (uint32_t)sh.prefix;
     if (t == 0) sh.cand_n = 0;
     __syncthreads();
+    // candidates: gathered rows with hi >= tau (no score has been written yet:
+    // the cluster's first barrier comes after the selection)
     int32_t* list = reinterpret_cast<int32_t*>(sh.hist);   // the lower bounds are done with
+    const uint32_t* gidx = reinterpret_cast<const uint32_t*>(sh.sk);
     for (unsigned int e = t; e < r.g; e += kPullThreads) {
-        const unsigned long long v = sh.sk[e];
-        if ((uint32_t)(v >> 32) >= tau) list[atomicAdd(&sh.cand_n, 1u)] = (int32_t)(uint32_t)v;
+        const uint32_t w = gidx[e];
+        if (fkey(a.w_hi[w]) >= tau) {
+            const unsigned int pos = atomicAdd(&sh.cand_n, 1u);
+            if (pos < (unsigned int)kPullSortCap) list[pos] = (int32_t)w;
+        }
     }
     __syncthreads();
+    if (sh.cand_n > (unsigned int)kPullSortCap) r.mode = 0;   // (the same in every CTA)
     return r;
 }
 
@@ -675,10 +734,16 @@ __device__ inline void pull_cluster_body(const PullArgs& a, PullShared& sh) {
         } else {
             a.ctr->front_k = 0;
         }
+        // where to start the next whole-set gather: the wide bound again while
+        // its gathers fit with room to spare, else the middle one
+        if (mode == 1 && !fs.from_front)
+            a.ctr->front_hint = (fs.mult == (unsigned int)kFrontMult ||
+                                 (fs.mult == 3u && fs.g < (unsigned int)kGatherCap / 4))
+                                    ? (unsigned int)kFrontMult : 3u;
     }
     if (mode == 1 && fs.new_front)
         for (unsigned int e = threadIdx.x; e < fs.g; e += kPullThreads)
-            a.front[e] = (int32_t)(uint32_t)sh.sk[e];
+            a.front[e] = (int32_t)reinterpret_cast<const uint32_t*>(sh.sk)[e];
     __syncthreads();   // sh.sk is the emission's sort buffer
     pull_emit_list(a, sh, cand, c);
     mirror_status(a);

@@ -381,7 +381,8 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     c->horizon_base = c->emitted;
     c->horizon_builds++;
     c->fresh_ws = true;
-    PVS_CUDA(cudaMemsetAsync(&c->ctr->front_k, 0, sizeof(unsigned int), c->stream));   // new indices
+    // new indices: no frontier, default hint (front_k and front_hint are adjacent)
+    PVS_CUDA(cudaMemsetAsync(&c->ctr->front_k, 0, 2 * sizeof(unsigned int), c->stream));
     return PVS_OK;
 }
 
