@@ -1,16 +1,20 @@
 // Exact authoritative float32 score of one vector, computed by one warp
 // (arXiv 2608.07152 Sec. 2.3.1 authoritative scores; App. A.1).
 //
-// The score is RN_f32 of the exact inner product sum_j q_j v_j:
-//   * every product of two float32 values is exact in binary64; lanes
-//     accumulate S = sum p_j and A = sum |p_j| in binary64 and reduce them;
-//   * |S - exact| <= (m - 1) u A / (1 - (m - 1) u) with u = 2^-53 for any
-//     summation order; with beta = 4 m u A the whole interval
-//     [RD(S - beta), RU(S + beta)] rounds to one float32 value in all but
-//     rare cases, and that value is the answer;
-//   * otherwise the warp sums the products exactly in a fixed-point
-//     accumulator (20 signed 32-bit digits in int64 slots, weight 2^-352 for
-//     the lowest bit) and rounds the exact sum to nearest-even.
+// The score is RN_f32 of the exact inner product sum_j q_j v_j.  Three
+// layers, each deciding only when its error bound proves the rounding:
+//   1. exact_dot_warp_eft (the common path, float32 pipe): error-free
+//      transformations of every product and partial sum with a bounded
+//      error sum, decided in float32 (see below);
+//   2. exact_dot_warp_impl, binary64: every product of two float32 values is
+//      exact in binary64; lanes accumulate S = sum p_j and A = sum |p_j|;
+//      |S - exact| <= (m - 1) u A / (1 - (m - 1) u) with u = 2^-53 for any
+//      summation order, and with beta = 4 m u A the interval
+//      [RD(S - beta), RU(S + beta)] rounding to one float32 value decides;
+//   3. otherwise the warp sums the products exactly in a fixed-point
+//      accumulator (20 signed 32-bit digits in int64 slots, weight 2^-352 for
+//      the lowest bit) and rounds the exact sum to nearest-even.
+// A result that rounds to zero is +0.
 #pragma once
 
 #include "pvs_common.cuh"

@@ -1,23 +1,25 @@
-// PVS pull without a host round trip (Sec. 2.3.1 incremental ranking,
-// Sec. 2.1 exact prefix): three launches turn the cursor's working set into
-// the next n exact ranks.
-//   1. tau = n-th largest lower bound among live working-set entries: radix
-//      select over ordered float keys, 11/11/10-bit digits, shared-memory
-//      histograms updated once per distinct digit per warp (match.any);
+// PVS pulls without a host round trip (Sec. 2.3.1 incremental ranking,
+// Sec. 2.1 exact prefix): the cursor's working set becomes the next n exact
+// ranks in these steps:
+//   1. tau = n-th largest lower bound among live working-set entries;
 //   2. candidates = live entries with hi >= tau (a superset of every item that
-//      can hold one of the next n ranks), compacted with warp ballots;
-//   3. every unresolved candidate (lo < hi) is scored exactly, one warp each
-//      on every SM (refine_kernel: the binary64 arithmetic is slow per SM on
-//      this part, so it is spread over the whole GPU), checked against its
-//      interval (App. A.1) and marked resolved (lo = hi = score) in the
-//      working set and the full bounds;
-//   4. the candidates' rank keys (score desc, id asc) are sorted in shared
-//      memory (bitonic, up to kPullSortCap); a larger candidate set first
-//      selects its n largest keys with a 64-bit radix select;
-//   5. the first n keys are written out and marked emitted (-inf).
-// Steps 1-2 and 4-5 each run in one CTA of 512 threads (<= 64 registers each)
-// with ~25 KB of shared memory, so they fit on an SM beside another cursor's
-// interval-pass CTA.
+//      can hold one of the next n ranks);
+//   3. every unresolved candidate (lo < hi) is scored exactly
+//      (exact_dot.cuh), checked against its interval (App. A.1) and marked
+//      resolved (lo = hi = score) in the working set and the full bounds;
+//   4. the candidates are ordered by rank key (score desc, id asc);
+//   5. the first n are written out and marked emitted (-inf).
+// Two forms:
+//   * three launches (the first pull of a fresh working set, which refines
+//     most of it, and every batched first pull): one CTA selects by radix
+//     select over ordered float keys (11/11/10-bit digits, shared-memory
+//     histograms, match.any aggregation), refinement runs on every SM
+//     (refine_kernels.cu), one CTA orders and emits;
+//   * one cluster launch (every later pull): each CTA of the cluster selects
+//     from the cursor's frontier or the whole working set, the CTAs split the
+//     refinement, and CTA 0 emits after a cluster barrier.
+// Every CTA has 512 threads (<= 64 registers) and ~25 KB of shared memory, so
+// it fits on an SM beside another cursor's interval-pass CTA.
 #include "exact_dot.cuh"
 #include "kernels.h"
 #include "pvs_common.cuh"
