@@ -55,6 +55,42 @@ __device__ inline bool mbar_wait(uint64_t* bar, uint32_t parity) {
     }
 }
 
+// ---- thread-block clusters ----------------------------------------------------
+__device__ inline uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Every thread of every CTA of the cluster; release/acquire ordering.
+__device__ inline void cluster_barrier() {
+    asm volatile(
+        "barrier.cluster.arrive.release.aligned;\n\t"
+        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Execution barrier of the cluster without memory ordering.
+__device__ inline void cluster_barrier_relaxed() {
+    asm volatile(
+        "barrier.cluster.arrive.relaxed.aligned;\n\t"
+        "barrier.cluster.wait.aligned;" ::: "memory");
+}
+
+// shared::cluster address of the variable at `p` in the CTA of cluster rank `rank`.
+__device__ inline uint32_t cluster_map(const void* p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+    return r;
+}
+
+// One arrival on an mbarrier of any CTA of the cluster, with the default
+// (CTA-scope) ordering: enough where the arrival only hands back a resource
+// whose last use has completed (a TMEM buffer after tcgen05.wait::ld), not
+// data written to memory.
+__device__ inline void mbar_arrive_remote(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
 // Order this thread's earlier generic-proxy accesses of shared memory (and
 // those of the threads it synchronised with) before its later bulk copies.
 __device__ inline void fence_proxy_async_smem() {

@@ -22,6 +22,7 @@
 // it fits on an SM beside another cursor's interval-pass CTA.
 #include "exact_dot.cuh"
 #include "kernels.h"
+#include "pipeline.cuh"
 #include "pvs_common.cuh"
 
 namespace pvs {
@@ -352,25 +353,6 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const 
 //   kPullSortCap reach t0, CTA 0 runs the radix selection instead.
 constexpr int kPullCluster = 8;        // single cursor: the whole pull in one cluster of 8
 constexpr int kPullClusterBatch = 2;   // batched pulls: many cursors at once, 2 CTAs each
-
-__device__ inline uint32_t cluster_ctarank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
-__device__ inline void cluster_barrier() {
-    asm volatile(
-        "barrier.cluster.arrive.release.aligned;\n\t"
-        "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// Execution barrier of the cluster without memory ordering.
-__device__ inline void cluster_barrier_relaxed() {
-    asm volatile(
-        "barrier.cluster.arrive.relaxed.aligned;\n\t"
-        "barrier.cluster.wait.aligned;" ::: "memory");
-}
 
 
 // Rows whose lower bound may reach the frontier bound: kFrontMult times the
