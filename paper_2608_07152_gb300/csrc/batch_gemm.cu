@@ -73,7 +73,10 @@ struct BatchShared {
     uint32_t tmem_base;
     int abort;
     QueryScalars qs[kMaxBN];
-    float4 flt[kMaxBN];   // filter: (s_q, rmax_q, tau_q, 0)
+    // filter: s_q, rmax_q (upper bound of the half-width), tau_q per query
+    alignas(16) float fs[kMaxBN];
+    alignas(16) float frm[kMaxBN];
+    alignas(16) float ftau[kMaxBN];
 };
 
 template <int kCta>
@@ -100,6 +103,27 @@ __device__ __forceinline__ void interval_of(float fdot, const QueryScalars& q, f
     const float r = __fadd_ru(E, G);
     lo = __fsub_rd(c, r);
     hi = __fadd_ru(c, r);
+}
+
+// Two fp32 lanes per instruction (f32x2), each lane rounded as its scalar
+// counterpart.
+__device__ __forceinline__ uint64_t pack2(float x, float y) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+    return r;
+}
+__device__ __forceinline__ void unpack2(uint64_t v, float& x, float& y) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
+}
+__device__ __forceinline__ uint64_t mul2_rn(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t add2_ru(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rp.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
 }
 
 // kCta = 2: the two CTAs of each cluster form a pair (cluster rank 0 is the
@@ -132,10 +156,13 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
     for (int i = threadIdx.x; i < kMaxBN; i += blockDim.x) {
         if (i < nq) {
             sh.qs[i] = a.qs[i];
-            sh.flt[i] = make_float4(a.qs[i].s, a.rmax ? a.rmax[i] : INFINITY,
-                                    a.tau ? a.tau[i] : -INFINITY, 0.0f);
-        } else {
-            sh.flt[i] = make_float4(0.0f, 0.0f, INFINITY, 0.0f);   // padding: never kept
+            sh.fs[i] = a.qs[i].s;
+            sh.frm[i] = a.rmax ? a.rmax[i] : INFINITY;
+            sh.ftau[i] = a.tau ? a.tau[i] : -INFINITY;
+        } else {   // padding columns: never candidates
+            sh.fs[i] = 0.0f;
+            sh.frm[i] = 0.0f;
+            sh.ftau[i] = INFINITY;
         }
     }
     if (threadIdx.x == 0) {
@@ -310,9 +337,8 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
             const int64_t srow = i * kBM + r_in_tile;   // row of the dump arrays
             const uint32_t tcol = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(b * kMaxBN);
             for (int cc = cgroup; real && cc < nqp / 32; cc += kEpiWarps / 4) {
-                // 32 query columns, read from TMEM 8 at a time (registers
-                // indexed by constants only)
                 if (a.mode == 0) {
+                    // 32 query columns, read from TMEM 8 at a time
                     for (int g = 0; g < 4; ++g) {
                         uint32_t r[8];
                         tc::ld_32x32b_x8(tcol + (uint32_t)(cc * 32 + g * 8), r);
@@ -332,37 +358,55 @@ __global__ void __launch_bounds__(kBatchThreads, 1)
                     continue;
                 }
                 // filter, step 1: which of the 32 queries keep this row (bit
-                // j of pmask); rows whose lower bound reaches tau are counted
-                // at once (no result is waited for).  Per group of 8 queries a
-                // branch-free test c + rmax_q >= tau_q marks the candidates
-                // (every other pair has hi < tau for sure); only those get
-                // the full interval.
-                uint32_t pmask = 0;
-                for (int g = 0; g < 4; ++g) {
-                    uint32_t r[8];
-                    tc::ld_32x32b_x8(tcol + (uint32_t)(cc * 32 + g * 8), r);
+                // k of pmask); rows whose lower bound reaches tau are counted
+                // at once (no result is waited for).  A branch-free test
+                // RU(c + rmax_q) >= tau_q marks the candidates (every other
+                // pair has hi < tau for sure), two queries per f32x2
+                // instruction with the roundings of c in the interval; only
+                // the candidates get the full interval.
+                uint32_t cand = 0;
+                {
+                    uint32_t r[32];
+                    tc::ld_32x32b_x32(tcol + (uint32_t)(cc * 32), r);
                     tc::wait_ld();
-                    uint32_t cand = 0;
+                    const uint64_t sv2 = pack2(sv, sv);
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const float4 f = sh.flt[cc * 32 + g * 8 + k];
-                        const float c = __fmul_rn(__fmul_rn(f.x, sv), __uint_as_float(r[k]));
-                        cand |= (uint32_t)(!(__fadd_ru(c, f.y) < f.z)) << k;
+                    for (int k = 0; k < 32; k += 4) {
+                        const int q = cc * 32 + k;
+                        const float4 s4 = *reinterpret_cast<const float4*>(&sh.fs[q]);
+                        const float4 m4 = *reinterpret_cast<const float4*>(&sh.frm[q]);
+                        const float4 t4 = *reinterpret_cast<const float4*>(&sh.ftau[q]);
+                        const uint64_t c01 = mul2_rn(mul2_rn(pack2(s4.x, s4.y), sv2),
+                                                     pack2(__uint_as_float(r[k]),
+                                                           __uint_as_float(r[k + 1])));
+                        const uint64_t c23 = mul2_rn(mul2_rn(pack2(s4.z, s4.w), sv2),
+                                                     pack2(__uint_as_float(r[k + 2]),
+                                                           __uint_as_float(r[k + 3])));
+                        float u0, u1, u2, u3;
+                        unpack2(add2_ru(c01, pack2(m4.x, m4.y)), u0, u1);
+                        unpack2(add2_ru(c23, pack2(m4.z, m4.w)), u2, u3);
+                        cand |= ((uint32_t)!(u0 < t4.x) << k) | ((uint32_t)!(u1 < t4.y) << (k + 1)) |
+                                ((uint32_t)!(u2 < t4.z) << (k + 2)) |
+                                ((uint32_t)!(u3 < t4.w) << (k + 3));
                     }
-                    if (!live) cand = 0;
-                    if (cand == 0) continue;
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const int q = cc * 32 + g * 8 + k;
-                        if (!((cand >> k) & 1u) || q >= nq) continue;
-                        const float tau = sh.flt[q].z;
-                        float lo, hi;
-                        interval_of(__uint_as_float(r[k]), sh.qs[q], sv, vn, en, lo, hi);
-                        if (!isfinite(lo) || !isfinite(hi)) set_status(a.status, PVS_ERR_OVERFLOW);
-                        if (hi < tau) continue;
-                        pmask |= 1u << (g * 8 + k);
-                        if (lo >= tau) atomicAdd(&a.h_eff[q], 1u);
-                    }
+                }
+                if (!live) cand = 0;
+                uint32_t pmask = 0;
+                uint32_t rest = __reduce_or_sync(0xffffffffu, cand);
+                while (rest != 0) {   // the same for the whole warp; rare
+                    const int k = __ffs(rest) - 1;
+                    rest &= rest - 1u;
+                    const uint32_t v = tc::ld_32x32b_x1(tcol + (uint32_t)(cc * 32 + k));
+                    tc::wait_ld();
+                    const int q = cc * 32 + k;
+                    if (!((cand >> k) & 1u) || q >= nq) continue;
+                    const float tau = sh.ftau[q];
+                    float lo, hi;
+                    interval_of(__uint_as_float(v), sh.qs[q], sv, vn, en, lo, hi);
+                    if (!isfinite(lo) || !isfinite(hi)) set_status(a.status, PVS_ERR_OVERFLOW);
+                    if (hi < tau) continue;
+                    pmask |= 1u << k;
+                    if (lo >= tau) atomicAdd(&a.h_eff[q], 1u);
                 }
                 // step 2: lane j reserves room for every row of the warp that
                 // query cc*32+j keeps (one atomic round trip for the chunk)
