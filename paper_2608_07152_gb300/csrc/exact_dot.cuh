@@ -259,7 +259,9 @@ __device__ inline float exact_dot_warp_eft(const float* q_fast, const float* __r
     const int lane = threadIdx.x & 31;
     const float4* q4 = reinterpret_cast<const float4*>(q_fast);
     const float4* v4 = reinterpret_cast<const float4*>(v);
-    EftAcc acc;
+    // two independent accumulators (components x, z and y, w) halve the
+    // dependency chains; they merge like two lanes of the butterfly
+    EftAcc acc, acc2;
     const int n4 = m_raw >> 2;
 #pragma unroll 1
     for (int j0 = lane; j0 < n4; j0 += kWarp * kBatch) {
@@ -275,12 +277,13 @@ __device__ inline float exact_dot_warp_eft(const float* q_fast, const float* __r
             if (j < n4) {
                 const float4 x = q4[j];
                 acc.add_product(x.x, y[b].x);
-                acc.add_product(x.y, y[b].y);
+                acc2.add_product(x.y, y[b].y);
                 acc.add_product(x.z, y[b].z);
-                acc.add_product(x.w, y[b].w);
+                acc2.add_product(x.w, y[b].w);
             }
         }
     }
+    acc.merge(acc2.s, acc2.c, acc2.a1, acc2.a2);
     float r;
     if (eft_finish(acc, m_raw, &r)) {
         *used_fallback = false;
@@ -297,15 +300,16 @@ __device__ inline float exact_dot_warp_eft_smem(const float* q_fast, const float
     const int lane = threadIdx.x & 31;
     const float4* q4 = reinterpret_cast<const float4*>(q_fast);
     const float4* v4 = reinterpret_cast<const float4*>(v_sh);
-    EftAcc acc;
+    EftAcc acc, acc2;   // two dependency chains, merged as in the butterfly
     const int n4 = m_raw >> 2;
     for (int j = lane; j < n4; j += kWarp) {
         const float4 x = q4[j], y = v4[j];
         acc.add_product(x.x, y.x);
-        acc.add_product(x.y, y.y);
+        acc2.add_product(x.y, y.y);
         acc.add_product(x.z, y.z);
-        acc.add_product(x.w, y.w);
+        acc2.add_product(x.w, y.w);
     }
+    acc.merge(acc2.s, acc2.c, acc2.a1, acc2.a2);
     float r;
     if (eft_finish(acc, m_raw, &r)) {
         *used_fallback = false;
