@@ -12,6 +12,9 @@ Modules
                  (Sec. 2.3.1, Appendix A.1; the bound arithmetic is in
                  ``pvs_ref.c``), the authoritative float32 score and the
                  complete dense ranking (Sec. 2.1).
+``pbm_oracle``   PBM sparse scores S(x) and range bounds H(R) in the fixed
+                 float32 term order (Sec. 2.3.2, Appendix A.2), block
+                 maxima, and the complete sparse ranking (Sec. 2.1).
 ``rrf_oracle``   complete-list weighted RRF and the target T*_K (Sec. 2.1),
                  in exact rational arithmetic.
 ``eahr_oracle``  the ordered certification rule of Sec. 2.2 applied to given
