@@ -63,6 +63,12 @@ class eahr_stats(ctypes.Structure):
                 ("checks", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class pbm_stats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "items", "emitted", "ranges", "ranges_expanded", "postings_visited", "items_scored",
+        "pulls", "rounds")] + [("state", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 def _load() -> ctypes.CDLL:
     if not os.path.exists(_LIB_PATH):
         raise ImportError(
@@ -105,6 +111,17 @@ def _load() -> ctypes.CDLL:
                             ctypes.POINTER(eahr_stats)]),
         "eahr_topk_lists": (i32, [P, i64, P, i64, ctypes.POINTER(eahr_params), P, P, P,
                                   ctypes.POINTER(eahr_stats)]),
+        "pbm_build": (i32, [P, i32, P, P, i64, i64, i32, i32, P, pp]),
+        "pbm_index_items": (i64, [P]),
+        "pbm_index_ranges": (i64, [P]),
+        "pbm_index_free": (None, [P]),
+        "pbm_cursor_open": (i32, [P, P, P, i32, pp]),
+        "pbm_next": (i32, [P, i32, P, P, P]),
+        "pbm_cursor_range_bounds": (i32, [P, i64, i64, P]),
+        "pbm_cursor_stats": (i32, [P, ctypes.POINTER(pbm_stats)]),
+        "pbm_cursor_close": (None, [P]),
+        "eahr_topk_pbm": (i32, [P, P, ctypes.POINTER(eahr_params), P, P, P,
+                                ctypes.POINTER(eahr_stats)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -123,7 +140,9 @@ EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_i
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_cursor_sync_batch", "pvs_cursor_stats_batch", "pvs_cursor_close_batch",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
-            "eahr_topk_lists")
+            "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
+            "pbm_index_free", "pbm_cursor_open", "pbm_next", "pbm_cursor_range_bounds",
+            "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm")
 
 
 def pvs_status_string(status: int) -> str:
@@ -436,4 +455,109 @@ def eahr_topk_lists(list0, list1, K: int = 20, k: int = 60, form: int = EAHR_RAN
     _check(_lib.eahr_topk_lists(a.ctypes.data, a.size, b.ctypes.data, b.size, ctypes.byref(p),
                                 ids.ctypes.data, F.ctypes.data, ctypes.byref(got),
                                 ctypes.byref(stats)), "eahr_topk_lists")
+    return _eahr_result(0, ids, F, got, stats)
+
+
+# --------------------------------------------------------------------------
+# PBM sparse rank generator (Sec. 2.3.2, App. A.2; include/pbm.h)
+# --------------------------------------------------------------------------
+
+def _array_arg(x, dtype):
+    """(pointer, size, on_device, keepalive) of a 1-D numpy or torch array."""
+    try:
+        import torch
+    except ImportError:  # pragma: no cover
+        torch = None
+    if torch is not None and isinstance(x, torch.Tensor):
+        tdt = {np.int64: torch.int64, np.int32: torch.int32, np.float32: torch.float32}[dtype]
+        if x.dtype != tdt:
+            raise TypeError(f"expected {tdt}")
+        x = x.contiguous()
+        if x.is_cuda:
+            torch.cuda.current_stream(x.device).synchronize()
+        return ctypes.c_void_p(x.data_ptr()), x.numel(), 1 if x.is_cuda else 0, x
+    a = np.ascontiguousarray(x, dtype=dtype)
+    return ctypes.c_void_p(a.ctypes.data), a.size, 0, a
+
+
+def pbm_build(term_off, docs, imps, n_items: int, block: int = 0, stream=None):
+    """PBM index from term-major postings (numpy or torch; all three on the
+    same side): term_off int64 [n_terms + 1], docs int32, imps float32."""
+    o, n_off, dev_o, ko = _array_arg(term_off, np.int64)
+    d, n_d, dev_d, kd = _array_arg(docs, np.int32)
+    p, n_p, dev_p, kp = _array_arg(imps, np.float32)
+    if not (dev_o == dev_d == dev_p):
+        raise ValueError("postings arrays must all be on the host or all on the device")
+    if n_d != n_p:
+        raise ValueError("one impact per posting")
+    out = ctypes.c_void_p()
+    st = ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else stream)
+    _check(_lib.pbm_build(o, n_off - 1, d, p, n_d, int(n_items), int(block), dev_o, st,
+                          ctypes.byref(out)), "pbm_build")
+    return out
+
+
+def pbm_index_items(index) -> int:
+    return int(_lib.pbm_index_items(index))
+
+
+def pbm_index_ranges(index) -> int:
+    return int(_lib.pbm_index_ranges(index))
+
+
+def pbm_index_free(index) -> None:
+    _lib.pbm_index_free(index)
+
+
+def pbm_cursor_open(index, terms, weights):
+    t = np.ascontiguousarray(terms, dtype=np.int32)
+    w = np.ascontiguousarray(weights, dtype=np.float32)
+    if t.shape != w.shape:
+        raise ValueError("one weight per query term")
+    out = ctypes.c_void_p()
+    _check(_lib.pbm_cursor_open(index, t.ctypes.data, w.ctypes.data, t.size, ctypes.byref(out)),
+           "pbm_cursor_open")
+    return out
+
+
+def pbm_next(cursor, n: int):
+    """Next up to n sparse ranks -> (ids int64, scores float32, status)."""
+    ids = np.empty(max(int(n), 1), np.int64)
+    sc = np.empty(max(int(n), 1), np.float32)
+    got = ctypes.c_int32(0)
+    s = _check(_lib.pbm_next(cursor, int(n), ids.ctypes.data, sc.ctypes.data,
+                             ctypes.byref(got)), "pbm_next")
+    return ids[:got.value], sc[:got.value], s
+
+
+def pbm_cursor_range_bounds(cursor, first: int, count: int):
+    """H_hat(R) of ranges first .. first+count-1 as computed at open."""
+    H = np.empty(max(int(count), 1), np.float32)
+    _check(_lib.pbm_cursor_range_bounds(cursor, int(first), int(count), H.ctypes.data),
+           "pbm_cursor_range_bounds")
+    return H[:int(count)]
+
+
+def pbm_cursor_stats(cursor) -> dict:
+    st = pbm_stats()
+    _check(_lib.pbm_cursor_stats(cursor, ctypes.byref(st)), "pbm_cursor_stats")
+    return {n: getattr(st, n) for n, _ in pbm_stats._fields_ if n != "reserved"}
+
+
+def pbm_cursor_close(cursor) -> None:
+    _lib.pbm_cursor_close(cursor)
+
+
+def eahr_topk_pbm(cursor, sparse_cursor, K: int = 20, k: int = 60, form: int = EAHR_NUMERATOR,
+                  policy: int = EAHR_POLICY_GEOMETRIC, step: int = 0, weights=(1, 1)):
+    """Ordered Top-K of complete-list weighted RRF with the sparse ranks pulled
+    from a PBM cursor -> (ids int64[q_K], F float64[q_K], stats)."""
+    p = _params(K, k, form, policy, step, weights)
+    ids = np.zeros(K, np.int64)
+    F = np.zeros(K, np.float64)
+    got = ctypes.c_int32(0)
+    stats = eahr_stats()
+    _check(_lib.eahr_topk_pbm(cursor, sparse_cursor, ctypes.byref(p), ids.ctypes.data,
+                              F.ctypes.data, ctypes.byref(got), ctypes.byref(stats)),
+           "eahr_topk_pbm")
     return _eahr_result(0, ids, F, got, stats)

@@ -28,6 +28,7 @@
 #include <new>
 #include <vector>
 
+#include "../../include/pbm.h"
 #include "../../include/pvs.h"
 #include "runtime.h"
 
@@ -121,8 +122,9 @@ inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
 }
 
 struct Source {
-    // dense cursor or host list
+    // dense cursor, sparse PBM cursor or host list
     pvs_cursor* cursor = nullptr;
+    pbm_cursor* sparse = nullptr;
     const int64_t* list = nullptr;
     int64_t length = 0;
 };
@@ -186,7 +188,7 @@ class Driver {
     // snapshot (when there is one) and not repeated within the list.
     bool record(int i, const int64_t* ids, int64_t n) {
         const int j = 1 - i;
-        const bool check = src[i].cursor == nullptr;
+        const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr;
         for (int64_t t = 0; t < n; ++t) {
             const int64_t x64 = ids[t];
             if (check) {
@@ -279,12 +281,15 @@ class Driver {
     pvs_status pull(int i, int64_t n) {
         if (exhausted[i] || !active[i]) return PVS_OK;
         pulls[i]++;
-        if (src[i].cursor) {
+        if (src[i].cursor || src[i].sparse) {
             if (n > (int64_t)std::numeric_limits<int32_t>::max()) n = std::numeric_limits<int32_t>::max();
             buf_ids.resize((size_t)n);
             buf_scores.resize((size_t)n);
             int32_t got = 0;
-            pvs_status s = pvs_next(src[i].cursor, (int32_t)n, buf_ids.data(), buf_scores.data(), &got);
+            pvs_status s =
+                src[i].cursor
+                    ? pvs_next(src[i].cursor, (int32_t)n, buf_ids.data(), buf_scores.data(), &got)
+                    : pbm_next(src[i].sparse, (int32_t)n, buf_ids.data(), buf_scores.data(), &got);
             if (s < 0) return s;
             record(i, buf_ids.data(), got);
             if (s == PVS_EXHAUSTED) exhausted[i] = true;
@@ -445,6 +450,32 @@ pvs_status eahr_topk_lists(const int64_t* list0, int64_t n0, const int64_t* list
         if (d.src[i].length == 0) d.exhausted[i] = true;
     }
     if (!d.init(id_space)) return PVS_ERR_OOM;
+    return run(d, p, out_ids, out_F, n_out, st);
+}
+
+pvs_status eahr_topk_pbm(pvs_cursor* dense, pbm_cursor* sparse, const eahr_params* p,
+                         int64_t* out_ids, double* out_F, int32_t* n_out, eahr_stats* st) {
+    if (n_out) *n_out = 0;
+    if (!dense || !sparse || !params_ok(p) || !out_ids || !n_out) return PVS_ERR_INVALID;
+    if (pvs::cursor_emitted(dense) != 0) return PVS_ERR_INVALID;
+    pbm_stats ps;
+    if (pbm_cursor_stats(sparse, &ps) != PVS_OK || ps.emitted != 0 || ps.state < 0)
+        return PVS_ERR_INVALID;
+    const pvs::SnapData* snap = pvs::cursor_snapshot(dense);
+    // both channels rank the same items: every row of the snapshot, no deletions
+    if (ps.items != snap->rows || snap->visible != snap->rows) return PVS_ERR_INVALID;
+    Driver d;
+    d.snap = snap;
+    d.src[0].cursor = dense;
+    d.src[0].length = pvs::cursor_visible(dense);
+    d.src[1].sparse = sparse;
+    d.src[1].length = ps.items;
+    for (int i = 0; i < 2; ++i) {
+        if (!contrib_from(p, i, d.src[i].length, &d.g[i])) return PVS_ERR_INVALID;
+        d.active[i] = d.g[i].a != 0;
+        if (d.src[i].length == 0) d.exhausted[i] = true;
+    }
+    if (!d.init(snap->rows)) return PVS_ERR_OOM;
     return run(d, p, out_ids, out_F, n_out, st);
 }
 

@@ -1,0 +1,498 @@
+// C ABI of the PBM sparse rank generator (include/pbm.h): arXiv 2608.07152
+// Sec. 2.3.2 and App. A.2; ranked-list contract of Sec. 2.1.
+//
+// A pull repeats two device steps until the next ranks are certified:
+//   1. K = max over unexpanded ranges R of key(H(R), first id of R), and the
+//      number of scored items in the pool with K < key < (last key emitted):
+//      those items precede every unexpanded item, so they are the next ranks;
+//   2. if fewer than asked are certified and ranges remain, expand the E
+//      unexpanded ranges of largest H (E doubles every round of a pull).
+// The certified items are then emitted in key order.  The pool is
+// append-only: emission runs in strictly decreasing key order, so the items
+// not yet emitted are exactly the pool keys below the last emitted key.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/pbm.h"
+#include "kernels.h"
+#include "pbm_kernels.h"
+#include "pvs_common.cuh"
+
+namespace {
+
+constexpr int kDefaultBlock = 128;
+constexpr uint64_t kCollectCap = 65536;   // windows up to this size are sorted whole
+
+pvs_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return PVS_OK;
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return PVS_ERR_OOM;
+    }
+    return PVS_ERR_CUDA;
+}
+
+#define PBM_CUDA(x)                                      \
+    do {                                                 \
+        cudaError_t _e = (x);                            \
+        if (_e != cudaSuccess) return cuda_status(_e);   \
+    } while (0)
+
+template <typename T>
+cudaError_t dalloc(T** p, size_t count) {
+    *p = nullptr;
+    return cudaMalloc(reinterpret_cast<void**>(p), (count ? count : 1) * sizeof(T));
+}
+
+template <typename T>
+void dfree(T*& p) {
+    if (p) cudaFree(p);
+    p = nullptr;
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        int cur = -1;
+        if (dev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != dev &&
+            cudaSetDevice(dev) == cudaSuccess)
+            prev = cur;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct pbm_index {
+    int device = 0;
+    int num_sms = 0;
+    cudaStream_t stream = nullptr;
+    bool own_stream = false;
+    int64_t n_items = 0, n_postings = 0, nb = 0, n_ranges = 0, nchunk = 0;
+    int32_t n_terms = 0;
+    int block = kDefaultBlock;
+    int64_t* term_off = nullptr;    // [n_terms + 1]
+    int32_t* docs = nullptr;        // [n_postings]
+    float* imps = nullptr;          // [n_postings]
+    int32_t* blk_range = nullptr;   // [nb]
+    int64_t* blk_pbeg = nullptr;    // [nb + 1]
+    float* blk_max = nullptr;       // [nb]
+    int64_t* blk_off = nullptr;     // [n_terms + 1]
+};
+
+struct pbm_cursor {
+    pbm_index* index = nullptr;
+    cudaStream_t stream = nullptr;
+    int nq = 0;
+    int32_t* terms = nullptr;
+    float* weights = nullptr;
+    int64_t* starts = nullptr;        // [nq][nchunk + 1]
+    float* H = nullptr;               // [n_ranges], as computed at open
+    float* Hlive = nullptr;           // [n_ranges], -inf once expanded
+    uint64_t* pool = nullptr;         // [n_items] rank keys of scored items
+    int32_t* list = nullptr;          // [n_ranges] ranges picked in a round
+    pvs::PbmCounters* ctr = nullptr;  // device
+    pvs::PbmCounters* h_ctr = nullptr;   // pinned mirror
+    unsigned long long* sel64 = nullptr;   // [258]
+    uint64_t* buf = nullptr;          // gathered keys
+    uint64_t* tmp = nullptr;
+    size_t buf_cap = 0;
+    void* sort_scratch = nullptr;
+    int64_t* out_ids = nullptr;
+    float* out_scores = nullptr;
+    uint64_t last_key = ~0ull;
+    int64_t emitted = 0, pulls = 0, rounds = 0;
+    int state = PVS_OK;
+};
+
+namespace {
+
+pvs_status fail(pbm_cursor* c, pvs_status s) {
+    if (s < 0 && c->state >= 0) c->state = s;
+    return s;
+}
+
+void free_cursor(pbm_cursor* c) {
+    if (!c) return;
+    dfree(c->terms);
+    dfree(c->weights);
+    dfree(c->starts);
+    dfree(c->H);
+    dfree(c->Hlive);
+    dfree(c->pool);
+    dfree(c->list);
+    dfree(c->ctr);
+    if (c->h_ctr) cudaFreeHost(c->h_ctr);
+    dfree(c->sel64);
+    dfree(c->buf);
+    dfree(c->tmp);
+    if (c->sort_scratch) cudaFree(c->sort_scratch);
+    dfree(c->out_ids);
+    dfree(c->out_scores);
+    delete c;
+}
+
+// Gather / sort buffers for at least `count` keys.
+pvs_status ensure_buffers(pbm_cursor* c, uint64_t count) {
+    const uint64_t need = std::max<uint64_t>(count, kCollectCap);
+    if (c->buf_cap >= need) return PVS_OK;
+    dfree(c->buf);
+    dfree(c->tmp);
+    if (c->sort_scratch) cudaFree(c->sort_scratch);
+    c->sort_scratch = nullptr;
+    dfree(c->out_ids);
+    dfree(c->out_scores);
+    c->buf_cap = 0;
+    PBM_CUDA(dalloc(&c->buf, need));
+    PBM_CUDA(dalloc(&c->tmp, need));
+    PBM_CUDA(cudaMalloc(&c->sort_scratch, pvs::radix_sort_scratch_bytes((int64_t)need)));
+    PBM_CUDA(dalloc(&c->out_ids, need));
+    PBM_CUDA(dalloc(&c->out_scores, need));
+    c->buf_cap = need;
+    return PVS_OK;
+}
+
+pvs_status sort_desc(pbm_cursor* c, uint64_t count) {
+    if (count <= 1) return PVS_OK;
+    if (count <= (uint64_t)pvs::kBitonicMax)
+        PBM_CUDA(pvs::launch_bitonic_desc(c->buf, (int)count, c->stream));
+    else
+        PBM_CUDA(pvs::launch_radix_sort_desc(c->buf, c->tmp, (int64_t)count, c->sort_scratch,
+                                             c->stream));
+    return PVS_OK;
+}
+
+pvs_status read_counters(pbm_cursor* c) {
+    PBM_CUDA(cudaMemcpyAsync(c->h_ctr, c->ctr, sizeof(pvs::PbmCounters), cudaMemcpyDeviceToHost,
+                             c->stream));
+    PBM_CUDA(cudaStreamSynchronize(c->stream));
+    if (c->h_ctr->status != 0) return (pvs_status)c->h_ctr->status;
+    return PVS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+pvs_status pbm_build(const int64_t* term_off, int32_t n_terms, const int32_t* docs,
+                     const float* imps, int64_t n_postings, int64_t n_items, int32_t block,
+                     int32_t on_device, void* cuda_stream, pbm_index** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (block == 0) block = kDefaultBlock;
+    if (n_terms < 0 || n_items < 1 || n_items >= ((int64_t)1 << 31) || n_postings < 0 ||
+        n_postings >= ((int64_t)1 << 32) - 1 || block < 1 || block > pvs::kPbmMaxBlock ||
+        !term_off || (n_postings > 0 && (!docs || !imps)))
+        return PVS_ERR_INVALID;
+    // the offsets are small: check them on the host
+    std::vector<int64_t> off((size_t)n_terms + 1);
+    if (on_device) {
+        if (cudaMemcpy(off.data(), term_off, off.size() * sizeof(int64_t),
+                       cudaMemcpyDeviceToHost) != cudaSuccess)
+            return PVS_ERR_CUDA;
+    } else {
+        std::memcpy(off.data(), term_off, off.size() * sizeof(int64_t));
+    }
+    if (off[0] != 0 || off[(size_t)n_terms] != n_postings) return PVS_ERR_INVALID;
+    for (int32_t t = 0; t < n_terms; ++t)
+        if (off[(size_t)t + 1] < off[(size_t)t]) return PVS_ERR_INVALID;
+
+    pbm_index* x = new (std::nothrow) pbm_index();
+    if (!x) return PVS_ERR_OOM;
+    auto bail = [&](pvs_status s) {
+        pbm_index_free(x);
+        return s;
+    };
+    if (cudaGetDevice(&x->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&x->num_sms, cudaDevAttrMultiProcessorCount, x->device) !=
+            cudaSuccess)
+        return bail(PVS_ERR_CUDA);
+    if (cuda_stream) {
+        x->stream = static_cast<cudaStream_t>(cuda_stream);
+    } else {
+        if (cudaStreamCreateWithFlags(&x->stream, cudaStreamNonBlocking) != cudaSuccess)
+            return bail(PVS_ERR_CUDA);
+        x->own_stream = true;
+    }
+    x->n_items = n_items;
+    x->n_terms = n_terms;
+    x->n_postings = n_postings;
+    x->block = block;
+    x->n_ranges = (n_items + block - 1) / block;
+    x->nchunk = (x->n_ranges + pvs::kPbmChunk - 1) / pvs::kPbmChunk;
+    cudaStream_t st = x->stream;
+    const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    if (dalloc(&x->term_off, off.size()) != cudaSuccess ||
+        dalloc(&x->docs, (size_t)n_postings) != cudaSuccess ||
+        dalloc(&x->imps, (size_t)n_postings) != cudaSuccess ||
+        dalloc(&x->blk_off, (size_t)n_terms + 1) != cudaSuccess)
+        return bail(PVS_ERR_OOM);
+    if (cudaMemcpyAsync(x->term_off, off.data(), off.size() * sizeof(int64_t),
+                        cudaMemcpyHostToDevice, st) != cudaSuccess ||
+        (n_postings > 0 &&
+         (cudaMemcpyAsync(x->docs, docs, (size_t)n_postings * sizeof(int32_t), kind, st) !=
+              cudaSuccess ||
+          cudaMemcpyAsync(x->imps, imps, (size_t)n_postings * sizeof(float), kind, st) !=
+              cudaSuccess)))
+        return bail(PVS_ERR_CUDA);
+
+    // blocks: starts marked and counted, then written once their number is known
+    uint8_t* flags = nullptr;
+    unsigned int* scratch = nullptr;
+    int* status = nullptr;
+    unsigned long long* nb_dev = nullptr;
+    auto free_tmp = [&]() {
+        dfree(flags);
+        dfree(scratch);
+        dfree(status);
+        dfree(nb_dev);
+    };
+    auto bail2 = [&](pvs_status s) {
+        free_tmp();
+        return bail(s);
+    };
+    if (dalloc(&flags, (size_t)n_postings) != cudaSuccess ||
+        dalloc(&scratch, pvs::pbm_scan_scratch_elems(n_postings)) != cudaSuccess ||
+        dalloc(&status, 1) != cudaSuccess || dalloc(&nb_dev, 1) != cudaSuccess)
+        return bail2(PVS_ERR_OOM);
+    if (cudaMemsetAsync(status, 0, sizeof(int), st) != cudaSuccess ||
+        pvs::launch_pbm_mark(x->term_off, n_terms, x->docs, x->imps, n_postings, n_items, block,
+                             flags, status, st) != cudaSuccess ||
+        pvs::launch_pbm_count_blocks(flags, n_postings, scratch, nb_dev, st) != cudaSuccess)
+        return bail2(PVS_ERR_CUDA);
+    int h_status = 0;
+    unsigned long long h_nb = 0;
+    if (cudaMemcpyAsync(&h_status, status, sizeof(int), cudaMemcpyDeviceToHost, st) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(&h_nb, nb_dev, sizeof(h_nb), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return bail2(PVS_ERR_CUDA);
+    if (h_status != 0) return bail2((pvs_status)h_status);
+    x->nb = (int64_t)h_nb;
+    if (dalloc(&x->blk_range, (size_t)x->nb) != cudaSuccess ||
+        dalloc(&x->blk_pbeg, (size_t)x->nb + 1) != cudaSuccess ||
+        dalloc(&x->blk_max, (size_t)x->nb) != cudaSuccess)
+        return bail2(PVS_ERR_OOM);
+    const int64_t p_end = n_postings;
+    if (pvs::launch_pbm_write_blocks(flags, x->docs, n_postings, block, scratch, x->blk_range,
+                                     x->blk_pbeg, st) != cudaSuccess ||
+        cudaMemcpyAsync(x->blk_pbeg + x->nb, &p_end, sizeof(int64_t), cudaMemcpyHostToDevice,
+                        st) != cudaSuccess ||
+        pvs::launch_pbm_block_max(x->blk_pbeg, x->imps, x->nb, x->blk_max, st) != cudaSuccess ||
+        pvs::launch_pbm_term_blocks(x->term_off, n_terms, x->blk_pbeg, x->nb, x->blk_off, st) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+        return bail2(PVS_ERR_CUDA);
+    free_tmp();
+    *out = x;
+    return PVS_OK;
+}
+
+int64_t pbm_index_items(const pbm_index* x) { return x ? x->n_items : 0; }
+int64_t pbm_index_ranges(const pbm_index* x) { return x ? x->n_ranges : 0; }
+
+void pbm_index_free(pbm_index* x) {
+    if (!x) return;
+    DeviceGuard device_guard(x->device);
+    if (x->stream) cudaStreamSynchronize(x->stream);
+    dfree(x->term_off);
+    dfree(x->docs);
+    dfree(x->imps);
+    dfree(x->blk_range);
+    dfree(x->blk_pbeg);
+    dfree(x->blk_max);
+    dfree(x->blk_off);
+    if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
+    delete x;
+}
+
+pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weights, int32_t nq,
+                           pbm_cursor** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (!x || nq < 0 || nq > pvs::kPbmMaxTerms || (nq > 0 && (!terms || !weights)))
+        return PVS_ERR_INVALID;
+    DeviceGuard device_guard(x->device);
+    std::vector<int32_t> sorted(terms, terms + nq);
+    std::sort(sorted.begin(), sorted.end());
+    for (int i = 0; i < nq; ++i) {
+        if (sorted[i] < 0 || sorted[i] >= x->n_terms) return PVS_ERR_INVALID;
+        if (i > 0 && sorted[i] == sorted[i - 1]) return PVS_ERR_INVALID;   // Q is a set
+    }
+    for (int i = 0; i < nq; ++i) {
+        if (!std::isfinite(weights[i])) return PVS_ERR_NONFINITE;
+        if (weights[i] < 0.0f) return PVS_ERR_INVALID;
+    }
+    pbm_cursor* c = new (std::nothrow) pbm_cursor();
+    if (!c) return PVS_ERR_OOM;
+    c->index = x;
+    c->stream = x->stream;
+    c->nq = nq;
+    auto bail = [&](pvs_status s) {
+        free_cursor(c);
+        return s;
+    };
+    if (dalloc(&c->terms, (size_t)nq) != cudaSuccess ||
+        dalloc(&c->weights, (size_t)nq) != cudaSuccess ||
+        dalloc(&c->starts, (size_t)nq * (size_t)(x->nchunk + 1)) != cudaSuccess ||
+        dalloc(&c->H, (size_t)x->n_ranges) != cudaSuccess ||
+        dalloc(&c->Hlive, (size_t)x->n_ranges) != cudaSuccess ||
+        dalloc(&c->pool, (size_t)x->n_items) != cudaSuccess ||
+        dalloc(&c->list, (size_t)x->n_ranges) != cudaSuccess ||
+        dalloc(&c->ctr, 1) != cudaSuccess ||
+        dalloc(&c->sel64, 258) != cudaSuccess ||
+        cudaMallocHost(reinterpret_cast<void**>(&c->h_ctr), sizeof(pvs::PbmCounters)) !=
+            cudaSuccess)
+        return bail(PVS_ERR_OOM);
+    std::memset(c->h_ctr, 0, sizeof(pvs::PbmCounters));
+    cudaStream_t st = c->stream;
+    const pvs::PbmQuery q{c->terms, c->weights, nq};
+    if ((nq > 0 &&
+         (cudaMemcpyAsync(c->terms, terms, (size_t)nq * sizeof(int32_t), cudaMemcpyHostToDevice,
+                          st) != cudaSuccess ||
+          cudaMemcpyAsync(c->weights, weights, (size_t)nq * sizeof(float),
+                          cudaMemcpyHostToDevice, st) != cudaSuccess)) ||
+        cudaMemsetAsync(c->ctr, 0, sizeof(pvs::PbmCounters), st) != cudaSuccess ||
+        pvs::launch_pbm_starts(q, x->blk_off, x->blk_range, x->nchunk, c->starts, st) !=
+            cudaSuccess ||
+        pvs::launch_pbm_bounds(q, c->starts, x->blk_range, x->blk_max, x->n_ranges, x->nchunk,
+                               c->H, c->Hlive, &c->ctr->status, st) != cudaSuccess)
+        return bail(PVS_ERR_CUDA);
+    if (cudaStreamSynchronize(st) != cudaSuccess) return bail(PVS_ERR_CUDA);   // query copies
+    *out = c;
+    return PVS_OK;
+}
+
+pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    if (n_out) *n_out = 0;
+    if (!c) return PVS_ERR_INVALID;
+    if (c->state < 0) return PVS_ERR_FAILED;
+    if (n < 1 || !ids || !scores || !n_out) return PVS_ERR_INVALID;
+    pbm_index* x = c->index;
+    DeviceGuard device_guard(x->device);
+    if (c->emitted == x->n_items) {
+        c->state = PVS_EXHAUSTED;
+        return PVS_EXHAUSTED;
+    }
+    cudaStream_t st = c->stream;
+    ++c->pulls;
+    const uint64_t need = (uint64_t)std::min<int64_t>(n, x->n_items - c->emitted);
+    uint64_t E = std::max<uint64_t>(8, 2 * ((need + x->block - 1) / x->block));
+    uint64_t window = 0;
+    for (;;) {
+        cudaError_t e = pvs::launch_pbm_kmax(c->Hlive, x->n_ranges, x->block, c->ctr, st);
+        if (e == cudaSuccess) e = pvs::launch_pbm_window(c->pool, c->last_key, c->ctr, st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        pvs_status s = read_counters(c);
+        if (s != PVS_OK) return fail(c, s);
+        window = c->h_ctr->window;
+        const uint64_t unexpanded = (uint64_t)x->n_ranges - c->h_ctr->ranges_expanded;
+        if (window >= need || unexpanded == 0) break;
+        // expand the E unexpanded ranges of largest bound (ties may add more)
+        ++c->rounds;
+        const uint64_t k = std::min(E, unexpanded);
+        const int grid = x->num_sms * 4;
+        pvs::PbmExpandArgs a{};
+        a.list = c->list;
+        a.q = pvs::PbmQuery{c->terms, c->weights, c->nq};
+        a.starts = c->starts;
+        a.nchunk = x->nchunk;
+        a.blk_range = x->blk_range;
+        a.blk_pbeg = x->blk_pbeg;
+        a.docs = x->docs;
+        a.imps = x->imps;
+        a.n_items = x->n_items;
+        a.block = x->block;
+        a.Hlive = c->Hlive;
+        a.pool = c->pool;
+        a.ctr = c->ctr;
+        e = pvs::launch_pbm_pick(c->Hlive, x->n_ranges, x->block, k, c->sel64, c->list, c->ctr,
+                                 st);
+        if (e == cudaSuccess) e = pvs::launch_pbm_expand(a, (int)std::min<uint64_t>(k, grid), st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        E *= 2;
+    }
+    const uint64_t m = std::min<uint64_t>(need, window);
+    if (m > 0) {
+        pvs_status s = ensure_buffers(c, std::min<uint64_t>(window, kCollectCap) + m);
+        if (s != PVS_OK) return fail(c, s);
+        uint64_t count = window;
+        cudaError_t e = cudaSuccess;
+        if (window <= kCollectCap) {
+            e = pvs::launch_pbm_collect(c->pool, nullptr, c->last_key, c->buf, c->buf_cap, c->ctr,
+                                        st);
+        } else {
+            // the m-th largest key of the window first, then the m keys from it on
+            e = pvs::launch_pbm_select64(c->pool, c->ctr, c->last_key, m, c->sel64, st);
+            if (e == cudaSuccess)
+                e = pvs::launch_pbm_collect(c->pool, c->sel64, c->last_key, c->buf, c->buf_cap,
+                                            c->ctr, st);
+            count = m;
+        }
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        s = sort_desc(c, count);
+        if (s != PVS_OK) return fail(c, s);
+        if (pvs::launch_pbm_emit(c->buf, (int)m, c->out_ids, c->out_scores, st) != cudaSuccess ||
+            cudaMemcpyAsync(ids, c->out_ids, m * sizeof(int64_t), cudaMemcpyDeviceToHost, st) !=
+                cudaSuccess ||
+            cudaMemcpyAsync(scores, c->out_scores, m * sizeof(float), cudaMemcpyDeviceToHost,
+                            st) != cudaSuccess)
+            return fail(c, PVS_ERR_CUDA);
+        s = read_counters(c);   // also waits for the outputs
+        if (s != PVS_OK) return fail(c, s);
+        if (c->h_ctr->collected != count) return fail(c, PVS_ERR_INVALID);   // internal invariant
+        c->last_key = pvs::rank_key(scores[m - 1], (uint32_t)ids[m - 1]);
+        c->emitted += (int64_t)m;
+    }
+    *n_out = (int32_t)m;
+    if (c->emitted == x->n_items) {
+        c->state = PVS_EXHAUSTED;
+        return PVS_EXHAUSTED;
+    }
+    return PVS_OK;
+}
+
+pvs_status pbm_cursor_range_bounds(pbm_cursor* c, int64_t first, int64_t count, float* H) {
+    if (!c || !H || first < 0 || count < 0 || first + count > c->index->n_ranges)
+        return PVS_ERR_INVALID;
+    DeviceGuard device_guard(c->index->device);
+    if (count == 0) return PVS_OK;
+    PBM_CUDA(cudaMemcpyAsync(H, c->H + first, (size_t)count * sizeof(float),
+                             cudaMemcpyDeviceToHost, c->stream));
+    PBM_CUDA(cudaStreamSynchronize(c->stream));
+    return c->state < 0 ? (pvs_status)c->state : PVS_OK;
+}
+
+pvs_status pbm_cursor_stats(pbm_cursor* c, pbm_stats* out) {
+    if (!c || !out) return PVS_ERR_INVALID;
+    DeviceGuard device_guard(c->index->device);
+    pvs_status s = read_counters(c);
+    if (s != PVS_OK && c->state >= 0) c->state = s;
+    out->items = c->index->n_items;
+    out->emitted = c->emitted;
+    out->ranges = c->index->n_ranges;
+    out->ranges_expanded = (int64_t)c->h_ctr->ranges_expanded;
+    out->postings_visited = (int64_t)c->h_ctr->postings;
+    out->items_scored = (int64_t)c->h_ctr->items;
+    out->pulls = c->pulls;
+    out->rounds = c->rounds;
+    out->state = c->state;
+    out->reserved = 0;
+    return PVS_OK;
+}
+
+void pbm_cursor_close(pbm_cursor* c) {
+    if (!c) return;
+    DeviceGuard device_guard(c->index ? c->index->device : -1);
+    if (c->stream) cudaStreamSynchronize(c->stream);
+    free_cursor(c);
+}
+
+}  // extern "C"

@@ -1,0 +1,108 @@
+// Host-side launchers of the PBM device kernels (internal to libpvs.so).
+// Method: arXiv 2608.07152 Sec. 2.3.2 (Posting Block-Max), App. A.2.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "kernels.h"
+
+namespace pvs {
+
+constexpr int kPbmMaxTerms = 1024;     // query terms
+constexpr int kPbmChunk = 1024;        // ranges per chunk of the bound pass
+constexpr int kPbmMaxBlock = 4096;     // ids per range
+
+// Device counters of a PBM cursor (one struct, mirrored to pinned memory).
+struct PbmCounters {
+    unsigned long long pool_len;         // scored items appended to the pool
+    unsigned long long kmax;             // max rank key over unexpanded ranges (0: none)
+    unsigned long long window;           // pool keys in (kmax, last)
+    unsigned long long ranges_expanded;
+    unsigned long long postings;
+    unsigned long long items;
+    unsigned long long picked;           // ranges picked in the current round
+    unsigned long long collected;        // pool keys gathered for an emission
+    int status;
+    int pad;
+};
+
+// ---- index build -------------------------------------------------------------
+// Marks posting i as the first of its block (new term or new range of
+// `block` ids), checks ids and impacts; flags[i] = 1 for a block start.
+cudaError_t launch_pbm_mark(const int64_t* term_off, int n_terms, const int32_t* docs,
+                            const float* imps, int64_t n_postings, int64_t n_items, int block,
+                            uint8_t* flags, int* status, cudaStream_t st);
+// Blocks from the start flags, in two steps: count (tile counts scanned in
+// `scratch`, the block total in *nb_out) and, once the block arrays are
+// allocated, write blk_range[b] and blk_pbeg[b] for every block start.
+size_t pbm_scan_scratch_elems(int64_t n_postings);
+cudaError_t launch_pbm_count_blocks(const uint8_t* flags, int64_t n_postings,
+                                    unsigned int* scratch, unsigned long long* nb_out,
+                                    cudaStream_t st);
+cudaError_t launch_pbm_write_blocks(const uint8_t* flags, const int32_t* docs, int64_t n_postings,
+                                    int block, const unsigned int* scratch, int32_t* blk_range,
+                                    int64_t* blk_pbeg, cudaStream_t st);
+// blk_max from blk_pbeg (run after the block count is known).
+cudaError_t launch_pbm_block_max(const int64_t* blk_pbeg, const float* imps, int64_t nb,
+                                 float* blk_max, cudaStream_t st);
+// blk_off[t] = first block whose postings start at or after term_off[t].
+cudaError_t launch_pbm_term_blocks(const int64_t* term_off, int n_terms, const int64_t* blk_pbeg,
+                                   int64_t nb, int64_t* blk_off, cudaStream_t st);
+
+// ---- query open ----------------------------------------------------------------
+struct PbmQuery {
+    const int32_t* terms;     // [nq]
+    const float* weights;     // [nq]
+    int nq;
+};
+// starts[i * (nchunk + 1) + k] = first block of query term i with range >= k * kPbmChunk.
+cudaError_t launch_pbm_starts(const PbmQuery& q, const int64_t* blk_off, const int32_t* blk_range,
+                              int64_t nchunk, int64_t* starts, cudaStream_t st);
+// H[r] (and Hlive[r] = H[r]) for every range, term by term in query order.
+cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const int32_t* blk_range,
+                              const float* blk_max, int64_t n_ranges, int64_t nchunk, float* H,
+                              float* Hlive, int* status, cudaStream_t st);
+
+// ---- pulls ---------------------------------------------------------------------
+// ctr->kmax = max over ranges with Hlive != -inf of rank_key(Hlive[r], r * block).
+cudaError_t launch_pbm_kmax(const float* Hlive, int64_t n_ranges, int block, PbmCounters* ctr,
+                            cudaStream_t st);
+// ctr->window = #{pool keys k: ctr->kmax < k < hi} over ctr->pool_len keys.
+cudaError_t launch_pbm_window(const uint64_t* pool, uint64_t hi, PbmCounters* ctr,
+                              cudaStream_t st);
+// The k unexpanded ranges with the largest keys key(Hlive[r], r * block)
+// (k <= unexpanded ranges) go to list, ctr->picked = k; sel64 holds 2 + 256
+// words of selection state.
+cudaError_t launch_pbm_pick(const float* Hlive, int64_t n_ranges, int block, uint64_t k,
+                            unsigned long long* sel64, int32_t* list, PbmCounters* ctr,
+                            cudaStream_t st);
+struct PbmExpandArgs {
+    const int32_t* list;          // picked ranges; count in ctr->picked
+    PbmQuery q;
+    const int64_t* starts;
+    int64_t nchunk;
+    const int32_t* blk_range;
+    const int64_t* blk_pbeg;
+    const int32_t* docs;
+    const float* imps;
+    int64_t n_items;
+    int block;
+    float* Hlive;
+    uint64_t* pool;
+    PbmCounters* ctr;
+};
+cudaError_t launch_pbm_expand(const PbmExpandArgs& a, int grid, cudaStream_t st);
+// Pool keys k with ctr->kmax < k < hi and k >= *from (from may be null)
+// appended to out in any order (ctr->collected counts them; at most cap written).
+cudaError_t launch_pbm_collect(const uint64_t* pool, const unsigned long long* from, uint64_t hi,
+                               uint64_t* out, uint64_t cap, PbmCounters* ctr, cudaStream_t st);
+// 64-bit radix selection: sel64[0] = the k-th largest (1-based) pool key k'
+// with ctr->kmax < k' < hi; sel64 holds 2 + 256 words of state.
+cudaError_t launch_pbm_select64(const uint64_t* pool, const PbmCounters* ctr, uint64_t hi,
+                                uint64_t k, unsigned long long* sel64, cudaStream_t st);
+// ids[i], scores[i] of the first m keys of a descending key array.
+cudaError_t launch_pbm_emit(const uint64_t* keys, int m, int64_t* ids, float* scores,
+                            cudaStream_t st);
+
+}  // namespace pvs

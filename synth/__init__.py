@@ -16,7 +16,14 @@ generators stand in for them with the shapes and structure of the workloads:
                          (Gaussian copula, rho = sin(pi tau / 2));
 * ``controlled_streams`` the rank relations of the controlled-stream study
                          (block-32 correlated, partial overlap, independent,
-                         reversed, all tied).
+                         reversed, all tied);
+* ``bm25_postings`` / ``sparse_queries``
+                         a stand-in for BM25 impact postings: term draws from
+                         a Zipf law (the most frequent ranks removed like
+                         stopwords), term frequencies from repeated draws,
+                         BM25 weights (k1 = 0.9, b = 0.4) from the corpus's own
+                         document frequencies and lengths, as term-major CSR;
+                         queries of a few distinct terms of weight 1.
 
 Every generator is deterministic in its seed; large matrices are produced in
 row chunks, each with its own derived seed, so any chunk can be regenerated
@@ -170,3 +177,85 @@ def controlled_streams(n: int, relation: str, seed: int):
     else:
         raise ValueError(relation)
     return first, second
+
+
+# --------------------------------------------------------------------------
+# sparse (BM25 impact) postings
+# --------------------------------------------------------------------------
+
+def _zipf_cdf(n_terms: int, exponent: float, skip: int, device) -> torch.Tensor:
+    r = torch.arange(1, n_terms + 1, dtype=torch.float64, device=device) + skip
+    w = r.pow(-exponent)
+    c = torch.cumsum(w, 0)
+    return c / c[-1]
+
+
+def bm25_postings(n_items: int, n_terms: int, mean_tokens: float, seed: int, device="cpu",
+                  exponent: float = 1.0, skip: int = 100, k1: float = 0.9, b: float = 0.4):
+    """Term-major postings (term_off int64 [n_terms + 1], docs int32, imps
+    float32) of a synthetic corpus with BM25 impacts.
+
+    Each item draws Poisson(mean_tokens) tokens; each token is a term drawn
+    from a Zipf law over ranks skip+1 .. skip+n_terms (the first `skip`
+    ranks play the removed stopwords).  Repeated draws of a term give its
+    term frequency tf.  The impact of term t on item x is the BM25 weight
+    idf_t * tf (k1 + 1) / (tf + k1 (1 - b + b dl_x / avgdl)) with
+    idf_t = ln(1 + (N - df_t + 0.5) / (df_t + 0.5)), computed in float64 and
+    stored as float32.  Postings of a term are in ascending item id."""
+    cdf = _zipf_cdf(n_terms, exponent, skip, device)
+    g = _gen(_chunk_seed(seed, -11), device)
+    dl = torch.poisson(torch.full((n_items,), float(mean_tokens), dtype=torch.float64,
+                                  device=device), generator=g).to(torch.int64)
+    keys = []
+    step = 1 << 16
+    for c0 in range(0, n_items, step):
+        c1 = min(n_items, c0 + step)
+        lens = dl[c0:c1]
+        total = int(lens.sum().item())
+        if total == 0:
+            continue
+        gc = _gen(_chunk_seed(seed, c0 // step), device)
+        u = torch.rand(total, generator=gc, dtype=torch.float64, device=device)
+        terms = torch.searchsorted(cdf, u).clamp_max(n_terms - 1)
+        docs = torch.repeat_interleave(torch.arange(c0, c1, device=device), lens)
+        keys.append(terms * n_items + docs)
+    if keys:
+        key = torch.sort(torch.cat(keys)).values
+        uniq, tf = torch.unique_consecutive(key, return_counts=True)
+    else:
+        uniq = torch.empty(0, dtype=torch.int64, device=device)
+        tf = torch.empty(0, dtype=torch.int64, device=device)
+    term = uniq // n_items
+    docs = (uniq % n_items).to(torch.int32)
+    df = torch.bincount(term, minlength=n_terms)
+    term_off = torch.zeros(n_terms + 1, dtype=torch.int64, device=device)
+    term_off[1:] = torch.cumsum(df, 0)
+    dlf = dl.to(torch.float64)
+    avgdl = float(dlf.mean().item()) if n_items else 1.0
+    avgdl = max(avgdl, 1e-9)
+    idf = torch.log1p((n_items - df.to(torch.float64) + 0.5) / (df.to(torch.float64) + 0.5))
+    tff = tf.to(torch.float64)
+    norm = k1 * (1.0 - b + b * dlf[docs.to(torch.int64)] / avgdl)
+    imps = (idf[term] * tff * (k1 + 1.0) / (tff + norm)).to(torch.float32)
+    return term_off, docs, imps
+
+
+def sparse_queries(nq: int, term_off: torch.Tensor, seed: int, mean_terms: float = 5.0,
+                   min_df: int = 1):
+    """nq queries of 1 + Poisson(mean_terms - 1) distinct terms (capped by
+    the vocabulary), drawn with probability proportional to the document
+    frequency among terms with at least min_df postings, each of weight 1
+    (a query term counted once).  Returns a list of (terms int32, weights
+    float32) numpy pairs; terms keep the order they were drawn in."""
+    off = term_off.detach().cpu().numpy().astype(np.int64)
+    df = np.diff(off)
+    ok = np.flatnonzero(df >= min_df)
+    rng = np.random.default_rng(int(seed) & ((1 << 63) - 1))
+    p = df[ok].astype(np.float64)
+    p /= p.sum()
+    out = []
+    for _ in range(nq):
+        k = min(ok.size, 1 + int(rng.poisson(max(mean_terms - 1.0, 0.0))))
+        t = rng.choice(ok, size=k, replace=False, p=p).astype(np.int32)
+        out.append((t, np.ones(k, np.float32)))
+    return out

@@ -1,5 +1,5 @@
 """C ABI library: loads on a machine without a GPU, exports every symbol that
-include/pvs.h declares, and its host-only EAHR driver reproduces the oracle
+include/*.h declares (pvs.h and pbm.h), and its host-only EAHR driver reproduces the oracle
 (arXiv 2608.07152, Sec. 2.1, 2.2; controlled streams of Sec. 3.4 / 4.2)."""
 import os
 import re
@@ -17,14 +17,21 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 def declared_functions():
-    text = open(os.path.join(ROOT, "include", "pvs.h")).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b((?:pvs|eahr)_[a-z_]+)\s*\(", text)))
+    names = set()
+    inc = os.path.join(ROOT, "include")
+    for h in sorted(os.listdir(inc)):
+        if not h.endswith(".h"):
+            continue
+        text = open(os.path.join(inc, h)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        names |= set(re.findall(r"\b((?:pvs|eahr|pbm)_[a-z_]+)\s*\(", text))
+    return sorted(names)
 
 
 def test_library_exports_every_declared_function():
     names = declared_functions()
-    assert len(names) >= 20
+    assert len(names) >= 30
+    assert "pbm_next" in names and "eahr_topk_pbm" in names
     for name in names:
         assert hasattr(pvs._lib, name), name
         assert name in pvs.EXPORTED, name
@@ -32,11 +39,12 @@ def test_library_exports_every_declared_function():
 
 def test_struct_layouts_match_header(tmp_path):
     """The binding's ctypes structures match the C compiler's layout of the
-    structures in include/pvs.h (size and every field offset)."""
+    structures in include/pvs.h and include/pbm.h (size and every field offset)."""
     import subprocess
     structs = {"pvs_stats": pvs.pvs_stats, "eahr_params": pvs.eahr_params,
-               "eahr_stats": pvs.eahr_stats}
-    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "pvs.h"', "int main(void) {"]
+               "eahr_stats": pvs.eahr_stats, "pbm_stats": pvs.pbm_stats}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "pvs.h"', '#include "pbm.h"',
+             "int main(void) {"]
     for name, cls in structs.items():
         lines.append(f'printf("{name} size %zu\\n", sizeof({name}));')
         for field, _ in cls._fields_:

@@ -1,0 +1,225 @@
+"""PBM sparse rank generator through the C ABI against the oracle
+(arXiv 2608.07152 Sec. 2.1, Sec. 2.3.2, App. A.2).
+
+Every emitted rank and score is compared bit for bit with the oracle's
+complete sparse ranking; the range bounds with the oracle's H_hat(R).
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2608_07152_gb300 as pvs
+import synth
+from oracle import pbm_oracle as po
+from oracle import pvs_oracle as pvo
+from oracle import rrf_oracle as ro
+
+pytestmark = pytest.mark.gpu
+
+
+def csr(n_terms, postings):
+    off, docs, imps = [0], [], []
+    for t in range(n_terms):
+        for d, p in postings.get(t, []):
+            docs.append(d)
+            imps.append(p)
+        off.append(len(docs))
+    return np.array(off, np.int64), np.array(docs, np.int32), np.array(imps, np.float32)
+
+
+def random_postings(rng, n_items, n_terms, max_df, integer=False):
+    postings = {}
+    for t in range(n_terms):
+        k = int(rng.integers(0, max_df + 1))
+        if k == 0:
+            continue
+        d = np.sort(rng.choice(n_items, size=min(k, n_items), replace=False))
+        p = (rng.integers(1, 4, size=d.size).astype(np.float32) if integer
+             else rng.gamma(2.0, 1.1, size=d.size).astype(np.float32))
+        postings[t] = list(zip(d.tolist(), p.tolist()))
+    return csr(n_terms, postings)
+
+
+def pull_all(cur, chunks, n_items):
+    ids, sc = [], []
+    k = 0
+    while True:
+        n = chunks[k % len(chunks)]
+        k += 1
+        i, s, st = pvs.pbm_next(cur, n)
+        ids.append(i)
+        sc.append(s)
+        if st == pvs.PVS_EXHAUSTED:
+            assert sum(len(x) for x in ids) == n_items
+            break
+        assert len(i) == n
+    return np.concatenate(ids), np.concatenate(sc)
+
+
+def check_against_oracle(off, docs, imps, n_items, terms, weights, block, chunks):
+    index = pvs.pbm_build(off, docs, imps, n_items, block=block)
+    try:
+        cur = pvs.pbm_cursor_open(index, terms, weights)
+        try:
+            nr = pvs.pbm_index_ranges(index)
+            H = pvs.pbm_cursor_range_bounds(cur, 0, nr)
+            ref_H = po.range_bounds(terms, weights, off, docs, imps, n_items, block)
+            assert np.array_equal(H.view(np.uint32), ref_H.view(np.uint32))
+            ids, sc = pull_all(cur, chunks, n_items)
+            stats = pvs.pbm_cursor_stats(cur)
+        finally:
+            pvs.pbm_cursor_close(cur)
+    finally:
+        pvs.pbm_index_free(index)
+    ref_ids, ref_sc = po.sparse_ranking(terms, weights, off, docs, imps, n_items)
+    assert np.array_equal(ids, ref_ids)
+    assert np.array_equal(sc.view(np.uint32), ref_sc.view(np.uint32))
+    assert stats["emitted"] == n_items and stats["state"] == pvs.PVS_EXHAUSTED
+    return stats
+
+
+def test_hand_worked_case():
+    off, docs, imps = csr(3, {0: [(0, 1.5), (2, 0.5), (4, 3.0)], 1: [(3, 7.0)],
+                              2: [(0, 4.0), (1, 2.0)]})
+    check_against_oracle(off, docs, imps, 6, [0, 2], [2.0, 0.5], 2, [1])
+    check_against_oracle(off, docs, imps, 6, [2, 0], [0.5, 2.0], 4, [4])
+
+
+@pytest.mark.parametrize("block", [1, 2, 7, 16, 128, 4096])
+def test_random_instances_every_block_size(block):
+    rng = np.random.default_rng(100 + block)
+    for trial in range(3):
+        n_items = int(rng.integers(50, 3000))
+        n_terms = 40
+        off, docs, imps = random_postings(rng, n_items, n_terms, max_df=n_items // 3)
+        nq = int(rng.integers(1, 9))
+        terms = rng.choice(n_terms, size=nq, replace=False).astype(np.int32)
+        weights = rng.gamma(1.5, 0.8, size=nq).astype(np.float32)
+        chunks = [int(x) for x in rng.integers(1, 300, size=5)]
+        check_against_oracle(off, docs, imps, n_items, terms, weights, block, chunks)
+
+
+def test_ties_zero_weights_and_empty_terms():
+    rng = np.random.default_rng(7)
+    n_items, n_terms = 1500, 30
+    off, docs, imps = random_postings(rng, n_items, n_terms, max_df=400, integer=True)
+    # integer impacts and weights: many exactly tied scores, ordered by id
+    terms = np.array([3, 11, 0, 25], np.int32)
+    check_against_oracle(off, docs, imps, n_items, terms, np.ones(4, np.float32), 16, [37, 5])
+    # a zero weight contributes nothing; a term without postings neither
+    empty = [t for t in range(n_terms) if off[t] == off[t + 1]]
+    terms2 = np.array([3, 11] + empty[:1], np.int32)
+    w2 = np.array([0.0, 2.0] + [1.0] * len(empty[:1]), np.float32)
+    check_against_oracle(off, docs, imps, n_items, terms2, w2, 64, [100])
+    # no query terms: every score is 0 and the ranking is id order
+    check_against_oracle(off, docs, imps, n_items, np.zeros(0, np.int32),
+                         np.zeros(0, np.float32), 16, [999])
+
+
+def test_bm25_corpus_deep_pulls_and_large_windows():
+    n_items, n_terms = 150_000, 20_000
+    off, docs, imps = synth.bm25_postings(n_items, n_terms, 30.0, seed=21)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    queries = synth.sparse_queries(3, torch.from_numpy(off), seed=22, mean_terms=5.0)
+    for qi, (terms, weights) in enumerate(queries):
+        # chunks of 20, then large pulls (windows above the sort-everything
+        # size go through the 64-bit selection)
+        stats = check_against_oracle(off, docs, imps, n_items, terms, weights, 128,
+                                     [20] * 50 + [70_000, 100_000])
+        q_postings = sum(int(off[t + 1] - off[t]) for t in terms)
+        assert stats["postings_visited"] == q_postings      # every posting once, at the end
+        assert stats["items_scored"] == n_items
+
+
+def test_first_ranks_touch_few_ranges():
+    n_items, n_terms = 400_000, 30_000
+    off, docs, imps = synth.bm25_postings(n_items, n_terms, 30.0, seed=31)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    terms, weights = synth.sparse_queries(1, torch.from_numpy(off), seed=32, mean_terms=4.0)[0]
+    ref_ids, ref_sc = po.sparse_ranking(terms, weights, off, docs, imps, n_items)
+    index = pvs.pbm_build(torch.from_numpy(off).cuda(), torch.from_numpy(docs).cuda(),
+                          torch.from_numpy(imps).cuda(), n_items)
+    try:
+        cur = pvs.pbm_cursor_open(index, terms, weights)
+        try:
+            got_i, got_s = [], []
+            for _ in range(10):
+                i, s, st = pvs.pbm_next(cur, 20)
+                assert st == pvs.PVS_OK and len(i) == 20
+                got_i.append(i)
+                got_s.append(s)
+            stats = pvs.pbm_cursor_stats(cur)
+        finally:
+            pvs.pbm_cursor_close(cur)
+    finally:
+        pvs.pbm_index_free(index)
+    assert np.array_equal(np.concatenate(got_i), ref_ids[:200])
+    assert np.array_equal(np.concatenate(got_s).view(np.uint32), ref_sc[:200].view(np.uint32))
+    # the bounds let PBM leave most ranges unexpanded for a short prefix
+    assert stats["ranges_expanded"] < stats["ranges"]
+
+
+def test_invalid_inputs_fail_loudly():
+    off, docs, imps = csr(2, {0: [(1, 1.0), (3, 2.0)], 1: [(0, 0.5)]})
+    def build_err(o, d, p, n=4, block=0):
+        with pytest.raises(pvs.PvsError) as e:
+            pvs.pbm_build(o, d, p, n, block=block)
+        return e.value.status
+    assert build_err(off, docs, np.array([1.0, -1.0, 0.5], np.float32)) == pvs.PVS_ERR_INVALID
+    assert build_err(off, docs, np.array([1.0, np.nan, 0.5], np.float32)) == pvs.PVS_ERR_NONFINITE
+    assert build_err(off, np.array([3, 1, 0], np.int32), imps) == pvs.PVS_ERR_INVALID
+    assert build_err(off, docs, imps, n=3) == pvs.PVS_ERR_INVALID           # id 3 out of range
+    assert build_err(np.array([0, 3, 2], np.int64), docs, imps) == pvs.PVS_ERR_INVALID
+    assert build_err(off, docs, imps, block=5000) == pvs.PVS_ERR_INVALID
+    index = pvs.pbm_build(off, docs, imps, 4)
+    try:
+        for terms, w, code in (([0, 0], [1.0, 1.0], pvs.PVS_ERR_INVALID),
+                               ([0, 2], [1.0, 1.0], pvs.PVS_ERR_INVALID),
+                               ([0], [-1.0], pvs.PVS_ERR_INVALID),
+                               ([1], [float("inf")], pvs.PVS_ERR_NONFINITE)):
+            with pytest.raises(pvs.PvsError) as e:
+                pvs.pbm_cursor_open(index, terms, w)
+            assert e.value.status == code
+        cur = pvs.pbm_cursor_open(index, [0, 1], [1.0, 1.0])
+        try:
+            with pytest.raises(pvs.PvsError):
+                pvs.pbm_next(cur, 0)
+            i, s, st = pvs.pbm_next(cur, 10)
+            assert st == pvs.PVS_EXHAUSTED and i.tolist() == [3, 1, 0, 2]
+            i, s, st = pvs.pbm_next(cur, 10)
+            assert st == pvs.PVS_EXHAUSTED and len(i) == 0
+        finally:
+            pvs.pbm_cursor_close(cur)
+    finally:
+        pvs.pbm_index_free(index)
+
+
+@pytest.mark.parametrize("tau_terms", [3, 6])
+def test_eahr_with_pbm_matches_complete_list_fusion(tau_terms):
+    n, m = 30_000, 64
+    V = synth.unit_normal(n, m, seed=41).numpy()
+    q = synth.unit_normal(1, m, seed=42).numpy()[0]
+    off, docs, imps = synth.bm25_postings(n, 5_000, 25.0, seed=43)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    terms, weights = synth.sparse_queries(1, torch.from_numpy(off), seed=44,
+                                          mean_terms=float(tau_terms))[0]
+    dense_ids, _ = pvo.dense_ranking(q, V)
+    sparse_ids, _ = po.sparse_ranking(terms, weights, off, docs, imps, n)
+    T = ro.target_topk_large([dense_ids, sparse_ids], [1, 1], 60, 20, ro.NUMERATOR)
+    dindex = pvs.pvs_build(V)
+    sindex = pvs.pbm_build(off, docs, imps, n)
+    try:
+        dcur = pvs.pvs_cursor_open(dindex, q)
+        scur = pvs.pbm_cursor_open(sindex, terms, weights)
+        try:
+            ids, F, st = pvs.eahr_topk_pbm(dcur, scur, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+        finally:
+            pvs.pbm_cursor_close(scur)
+            pvs.pvs_cursor_close(dcur)
+    finally:
+        pvs.pbm_index_free(sindex)
+        pvs.pvs_index_free(dindex)
+    assert ids.tolist() == [x for x, _ in T]
+    for (x, f), got in zip(T, F):
+        if not np.isnan(got):
+            assert got == ro.as_float(f)
