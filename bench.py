@@ -57,11 +57,12 @@ def parse():
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="passage",
-                   choices=["passage", "batched", "eahr", "snapshots"],
+                   choices=["passage", "batched", "eahr", "snapshots", "sparse"],
                    help="passage: single-query ranking (default); batched: 256-query "
                         "tensor-core batches; eahr: EAHR Top-20 fusion over the passage "
                         "corpus and copula sparse rankings; snapshots: near-duplicate "
-                        "corpus, five snapshots, EAHR Top-20")
+                        "corpus, five snapshots, EAHR Top-20; sparse: PBM sparse ranks "
+                        "over a synthetic BM25 corpus")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
@@ -629,6 +630,138 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+SPARSE_TERMS = 500_000      # vocabulary of the synthetic BM25 corpus
+SPARSE_TOKENS = 40.0        # mean tokens per item (Poisson)
+SPARSE_QUERY_TERMS = 5.0    # mean distinct terms per query
+SPARSE_RANKS = 1000
+SPARSE_CHUNK = 20
+
+
+def build_sparse_index(pvs, synth, torch, n, dev, seed):
+    """Synthetic BM25 postings generated on the device and the PBM index."""
+    t0 = time.perf_counter()
+    off, docs, imps = synth.bm25_postings(n, SPARSE_TERMS, SPARSE_TOKENS, seed=seed, device=dev)
+    torch.cuda.synchronize()
+    t1 = time.perf_counter()
+    index = pvs.pbm_build(off, docs, imps, n)
+    torch.cuda.synchronize()
+    return index, (off, docs, imps), t1 - t0, time.perf_counter() - t1
+
+
+def sparse_complete(torch, n, post, terms, weights, dev):
+    """The complete sparse ranking in plain torch (the comparator): every
+    query term's postings scattered into a score per item, then a full stable
+    sort; returns the first SPARSE_RANKS ids (host) and the time in ms."""
+    off, docs, imps = post
+    torch.cuda.synchronize()
+    t = time.perf_counter()
+    sc = torch.zeros(n, dtype=torch.float32, device=dev)
+    for term, w in zip(terms.tolist(), weights.tolist()):
+        a, b = int(off[term]), int(off[term + 1])
+        sc.index_put_((docs[a:b].long(),), imps[a:b] * w, accumulate=True)
+    order = torch.argsort(sc, descending=True, stable=True)
+    head = order[:SPARSE_RANKS].cpu()
+    return head, (time.perf_counter() - t) * 1e3
+
+
+def main_sparse(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """PBM sparse ranking over a passage-scale synthetic BM25 corpus: per
+    query, open a cursor and pull the first 1,000 exact sparse ranks in
+    chunks of 20 (host outputs).  Queries run one after another; each rank
+    drives its own index replica.  Beside it, the complete sparse ranking in
+    plain torch (score every posting of the query terms, sort all N)."""
+    n = args.n
+    index, post, gen_s, build_s = build_sparse_index(pvs, synth, torch, n, dev, seed=8)
+    off_h = post[0].cpu()
+    nqs = args.warmup + args.steps
+    queries = synth.sparse_queries(nqs, off_h, seed=query_seed(9, rank),
+                                   mean_terms=SPARSE_QUERY_TERMS, min_df=2)
+
+    def one(terms, weights):
+        t0 = time.perf_counter()
+        cur = pvs.pbm_cursor_open(index, terms, weights)
+        first = None
+        got = []
+        for c in range(SPARSE_RANKS // SPARSE_CHUNK):
+            ids, _, st = pvs.pbm_next(cur, SPARSE_CHUNK)
+            got.append(ids)
+            if c == 0:
+                first = time.perf_counter() - t0
+        total = time.perf_counter() - t0
+        stats = pvs.pbm_cursor_stats(cur)
+        pvs.pbm_cursor_close(cur)
+        return total, first, stats, np.concatenate(got)
+
+    for w in range(args.warmup):
+        one(*queries[w])
+        sparse_complete(torch, n, post, queries[w][0], queries[w][1], dev)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    launches0 = pvs.pvs_launch_count()
+    lat, first, st_all = [], [], []
+    t0 = time.perf_counter()
+    with ClockSampler(local) as clk:
+        for j in range(args.warmup, nqs):
+            total, f, stats, _ = one(*queries[j])
+            lat.append(total)
+            first.append(f)
+            st_all.append(stats)
+    elapsed = slowest(pg, time.perf_counter() - t0, dev)
+    launches = pvs.pvs_launch_count() - launches0
+    cmp_ms, mismatches = [], 0
+    for j in range(args.warmup, min(nqs, args.warmup + 20)):
+        head, ms = sparse_complete(torch, n, post, queries[j][0], queries[j][1], dev)
+        cmp_ms.append(ms)
+    check = None
+    if args.oracle_check:
+        from oracle import pbm_oracle as po
+        o, d, i = (x.cpu().numpy() for x in post)
+        check = {"queries": 0, "mismatches": 0}
+        for j in range(args.warmup, min(nqs, args.warmup + 3)):
+            _, _, _, ids = one(*queries[j])
+            ref, _ = po.sparse_ranking(queries[j][0], queries[j][1], o, d, i, n)
+            check["queries"] += 1
+            check["mismatches"] += int(not np.array_equal(ids, ref[:SPARSE_RANKS]))
+    value = job_rate(args.steps * SPARSE_RANKS, world, elapsed)
+    med = lambda k: float(np.median([s[k] for s in st_all]))
+    line = {
+        "metric": "exact sparse ranks/sec (PBM)", "value": value, "unit": "ranks/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": elapsed * 1e3 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "PBM sparse ranking: synthetic BM25 impact postings over "
+                               f"N={n:,} items (vocabulary {SPARSE_TERMS:,}, Zipf terms, "
+                               f"Poisson({SPARSE_TOKENS:g}) tokens per item, k1=0.9 b=0.4), "
+                               f"queries of 1+Poisson({SPARSE_QUERY_TERMS - 1:g}) terms, "
+                               f"first {SPARSE_RANKS} ranks in chunks of {SPARSE_CHUNK}",
+                   "N": n, "ranks_per_query": SPARSE_RANKS, "chunk": SPARSE_CHUNK,
+                   "postings": int(post[1].numel()), "block": 128,
+                   "l2": "no flush: queries run back to back on one index",
+                   "parallelism": f"replicas x{world}"},
+        "e2e": {"value": value, "unit": "ranks/s",
+                "h2d_bytes_per_step": int(np.mean([8 * len(q[0]) for q in queries])),
+                "d2h_bytes_per_step": SPARSE_RANKS * 12},
+        "latency_ms": {"first_20_p50": float(np.median(first)) * 1e3,
+                       "first_1000_p50": float(np.median(lat)) * 1e3,
+                       "first_1000_p95": float(np.percentile(lat, 95)) * 1e3},
+        "per_query": {"ranges_expanded_p50": med("ranges_expanded"), "ranges": st_all[0]["ranges"],
+                      "postings_visited_p50": med("postings_visited"),
+                      "rounds_p50": med("rounds")},
+        "complete_sparse_ranking_ms_p50": float(np.median(cmp_ms)) if cmp_ms else None,
+        "oracle_check": check,
+        "gpu_launches": launches,
+        "generate_s": gen_s, "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    pvs.pbm_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 SNAP_N = 2_000_000
 SNAP_DIM = 1024
 SNAP_DUP = 0.2          # near-duplicate share of the base corpus
@@ -785,6 +918,9 @@ def main():
         return
     if args.workload == "snapshots":
         main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
+    if args.workload == "sparse":
+        main_sparse(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
     stream = torch.cuda.Stream(device=dev)

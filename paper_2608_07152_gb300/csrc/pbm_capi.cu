@@ -1,12 +1,15 @@
 // C ABI of the PBM sparse rank generator (include/pbm.h): arXiv 2608.07152
 // Sec. 2.3.2 and App. A.2; ranked-list contract of Sec. 2.1.
 //
-// A pull repeats two device steps until the next ranks are certified:
-//   1. K = max over unexpanded ranges R of key(H(R), first id of R), and the
-//      number of scored items in the pool with K < key < (last key emitted):
-//      those items precede every unexpanded item, so they are the next ranks;
-//   2. if fewer than asked are certified and ranges remain, expand the E
-//      unexpanded ranges of largest H (E doubles every round of a pull).
+// The ranges' keys key(H(R), first id of R) are sorted once, descending, at
+// open, and ranges are expanded in that order.  A pull repeats two device
+// steps until the next ranks are certified:
+//   1. K = the key of the first unexpanded range in that order (the largest
+//      unexpanded key), and the number of scored items in the pool with
+//      K < key < (last key emitted): those items precede every unexpanded
+//      item, so they are the next ranks;
+//   2. if fewer than asked are certified and ranges remain, expand the next E
+//      ranges (E doubles every round and carries over between pulls).
 // The certified items are then emitted in key order.  The pool is
 // append-only: emission runs in strictly decreasing key order, so the items
 // not yet emitted are exactly the pool keys below the last emitted key.
@@ -26,7 +29,7 @@
 namespace {
 
 constexpr int kDefaultBlock = 128;
-constexpr uint64_t kCollectCap = 65536;   // windows up to this size are sorted whole
+constexpr uint64_t kCollectCap = 65536;   // smallest gather buffer (keys)
 
 pvs_status cuda_status(cudaError_t e) {
     if (e == cudaSuccess) return PVS_OK;
@@ -95,9 +98,8 @@ struct pbm_cursor {
     float* weights = nullptr;
     int64_t* starts = nullptr;        // [nq][nchunk + 1]
     float* H = nullptr;               // [n_ranges], as computed at open
-    float* Hlive = nullptr;           // [n_ranges], -inf once expanded
+    uint64_t* rkeys = nullptr;        // [n_ranges] range keys, sorted descending at open
     uint64_t* pool = nullptr;         // [n_items] rank keys of scored items
-    int32_t* list = nullptr;          // [n_ranges] ranges picked in a round
     pvs::PbmCounters* ctr = nullptr;  // device
     pvs::PbmCounters* h_ctr = nullptr;   // pinned mirror
     unsigned long long* sel64 = nullptr;   // [258]
@@ -107,7 +109,11 @@ struct pbm_cursor {
     void* sort_scratch = nullptr;
     int64_t* out_ids = nullptr;
     float* out_scores = nullptr;
+    int64_t* h_ids = nullptr;         // pinned: ranks of a pull served by the finish kernel
+    float* h_scores = nullptr;
     uint64_t last_key = ~0ull;
+    int64_t next = 0;                 // ranges expanded (a prefix of the sorted order)
+    uint64_t E = 64;                  // ranges to expand in the next round
     int64_t emitted = 0, pulls = 0, rounds = 0;
     int state = PVS_OK;
 };
@@ -125,9 +131,8 @@ void free_cursor(pbm_cursor* c) {
     dfree(c->weights);
     dfree(c->starts);
     dfree(c->H);
-    dfree(c->Hlive);
+    dfree(c->rkeys);
     dfree(c->pool);
-    dfree(c->list);
     dfree(c->ctr);
     if (c->h_ctr) cudaFreeHost(c->h_ctr);
     dfree(c->sel64);
@@ -136,6 +141,8 @@ void free_cursor(pbm_cursor* c) {
     if (c->sort_scratch) cudaFree(c->sort_scratch);
     dfree(c->out_ids);
     dfree(c->out_scores);
+    if (c->h_ids) cudaFreeHost(c->h_ids);
+    if (c->h_scores) cudaFreeHost(c->h_scores);
     delete c;
 }
 
@@ -343,13 +350,16 @@ pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weig
         dalloc(&c->weights, (size_t)nq) != cudaSuccess ||
         dalloc(&c->starts, (size_t)nq * (size_t)(x->nchunk + 1)) != cudaSuccess ||
         dalloc(&c->H, (size_t)x->n_ranges) != cudaSuccess ||
-        dalloc(&c->Hlive, (size_t)x->n_ranges) != cudaSuccess ||
+        dalloc(&c->rkeys, (size_t)x->n_ranges) != cudaSuccess ||
         dalloc(&c->pool, (size_t)x->n_items) != cudaSuccess ||
-        dalloc(&c->list, (size_t)x->n_ranges) != cudaSuccess ||
         dalloc(&c->ctr, 1) != cudaSuccess ||
         dalloc(&c->sel64, 258) != cudaSuccess ||
         cudaMallocHost(reinterpret_cast<void**>(&c->h_ctr), sizeof(pvs::PbmCounters)) !=
-            cudaSuccess)
+            cudaSuccess ||
+        cudaMallocHost(reinterpret_cast<void**>(&c->h_ids),
+                       pvs::kPbmFastWindow * sizeof(int64_t)) != cudaSuccess ||
+        cudaMallocHost(reinterpret_cast<void**>(&c->h_scores),
+                       pvs::kPbmFastWindow * sizeof(float)) != cudaSuccess)
         return bail(PVS_ERR_OOM);
     std::memset(c->h_ctr, 0, sizeof(pvs::PbmCounters));
     cudaStream_t st = c->stream;
@@ -363,7 +373,17 @@ pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weig
         pvs::launch_pbm_starts(q, x->blk_off, x->blk_range, x->nchunk, c->starts, st) !=
             cudaSuccess ||
         pvs::launch_pbm_bounds(q, c->starts, x->blk_range, x->blk_max, x->n_ranges, x->nchunk,
-                               c->H, c->Hlive, &c->ctr->status, st) != cudaSuccess)
+                               c->H, &c->ctr->status, st) != cudaSuccess ||
+        pvs::launch_pbm_range_keys(c->H, x->n_ranges, x->block, c->rkeys, st) != cudaSuccess)
+        return bail(PVS_ERR_CUDA);
+    // the expansion order: range keys sorted descending (the sort's scratch is
+    // the gather buffers, sized for at least n_ranges keys)
+    if (ensure_buffers(c, (uint64_t)x->n_ranges) != PVS_OK) return bail(PVS_ERR_OOM);
+    if (x->n_ranges > 1 &&
+        ((uint64_t)x->n_ranges <= (uint64_t)pvs::kBitonicMax
+             ? pvs::launch_bitonic_desc(c->rkeys, (int)x->n_ranges, st)
+             : pvs::launch_radix_sort_desc(c->rkeys, c->tmp, x->n_ranges, c->sort_scratch, st)) !=
+            cudaSuccess)
         return bail(PVS_ERR_CUDA);
     if (cudaStreamSynchronize(st) != cudaSuccess) return bail(PVS_ERR_CUDA);   // query copies
     *out = c;
@@ -384,23 +404,35 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     cudaStream_t st = c->stream;
     ++c->pulls;
     const uint64_t need = (uint64_t)std::min<int64_t>(n, x->n_items - c->emitted);
-    uint64_t E = std::max<uint64_t>(8, 2 * ((need + x->block - 1) / x->block));
+    uint64_t E = std::max<uint64_t>(c->E, 2 * ((need + x->block - 1) / x->block));
     uint64_t window = 0;
+    uint64_t last = 0;   // size of the last expansion of this pull
+    bool served = false;
     for (;;) {
-        cudaError_t e = pvs::launch_pbm_kmax(c->Hlive, x->n_ranges, x->block, c->ctr, st);
-        if (e == cudaSuccess) e = pvs::launch_pbm_window(c->pool, c->last_key, c->ctr, st);
+        // the certified window, gathered; a window of at most kPbmFastWindow
+        // keys that covers the pull is sorted and written to pinned memory in
+        // the same step (one synchronisation)
+        cudaError_t e = pvs::launch_pbm_window(c->rkeys, c->next, x->n_ranges, c->pool,
+                                               c->last_key, c->buf, c->buf_cap, c->ctr, st);
+        if (e == cudaSuccess)
+            e = pvs::launch_pbm_finish(c->buf, c->ctr, need, c->h_ids, c->h_scores, c->h_ctr,
+                                       st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
         if (e != cudaSuccess) return fail(c, cuda_status(e));
-        pvs_status s = read_counters(c);
-        if (s != PVS_OK) return fail(c, s);
-        window = c->h_ctr->window;
-        const uint64_t unexpanded = (uint64_t)x->n_ranges - c->h_ctr->ranges_expanded;
+        if (c->h_ctr->status != 0) return fail(c, (pvs_status)c->h_ctr->status);
+        window = c->h_ctr->collected;
+        if (window >= need && window <= (uint64_t)pvs::kPbmFastWindow) {
+            served = true;
+            break;
+        }
+        const uint64_t unexpanded = (uint64_t)(x->n_ranges - c->next);
         if (window >= need || unexpanded == 0) break;
-        // expand the E unexpanded ranges of largest bound (ties may add more)
+        // expand the next E ranges of the sorted order
         ++c->rounds;
         const uint64_t k = std::min(E, unexpanded);
-        const int grid = x->num_sms * 4;
         pvs::PbmExpandArgs a{};
-        a.list = c->list;
+        a.ranges = c->rkeys + c->next;
+        a.count = (int64_t)k;
         a.q = pvs::PbmQuery{c->terms, c->weights, c->nq};
         a.starts = c->starts;
         a.nchunk = x->nchunk;
@@ -410,34 +442,31 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         a.imps = x->imps;
         a.n_items = x->n_items;
         a.block = x->block;
-        a.Hlive = c->Hlive;
         a.pool = c->pool;
         a.ctr = c->ctr;
-        e = pvs::launch_pbm_pick(c->Hlive, x->n_ranges, x->block, k, c->sel64, c->list, c->ctr,
-                                 st);
-        if (e == cudaSuccess) e = pvs::launch_pbm_expand(a, (int)std::min<uint64_t>(k, grid), st);
+        e = pvs::launch_pbm_expand(a, (int)std::min<uint64_t>(k, (uint64_t)x->num_sms * 4), st);
         if (e != cudaSuccess) return fail(c, cuda_status(e));
+        c->next += (int64_t)k;
+        last = k;
         E *= 2;
     }
+    // the next pull starts from the size of the expansion that last sufficed
+    if (last) c->E = std::max<uint64_t>(16, last);
     const uint64_t m = std::min<uint64_t>(need, window);
-    if (m > 0) {
-        pvs_status s = ensure_buffers(c, std::min<uint64_t>(window, kCollectCap) + m);
+    if (served) {
+        std::memcpy(ids, c->h_ids, m * sizeof(int64_t));
+        std::memcpy(scores, c->h_scores, m * sizeof(float));
+    } else if (m > 0) {
+        // large window: the m-th largest key first (or the whole window when
+        // it fits the gather buffer), then a device sort of the m keys
+        pvs_status s = ensure_buffers(c, m);
         if (s != PVS_OK) return fail(c, s);
-        uint64_t count = window;
-        cudaError_t e = cudaSuccess;
-        if (window <= kCollectCap) {
-            e = pvs::launch_pbm_collect(c->pool, nullptr, c->last_key, c->buf, c->buf_cap, c->ctr,
+        cudaError_t e = pvs::launch_pbm_select64(c->pool, c->ctr, c->last_key, m, c->sel64, st);
+        if (e == cudaSuccess)
+            e = pvs::launch_pbm_collect(c->pool, c->sel64, c->last_key, c->buf, c->buf_cap, c->ctr,
                                         st);
-        } else {
-            // the m-th largest key of the window first, then the m keys from it on
-            e = pvs::launch_pbm_select64(c->pool, c->ctr, c->last_key, m, c->sel64, st);
-            if (e == cudaSuccess)
-                e = pvs::launch_pbm_collect(c->pool, c->sel64, c->last_key, c->buf, c->buf_cap,
-                                            c->ctr, st);
-            count = m;
-        }
         if (e != cudaSuccess) return fail(c, cuda_status(e));
-        s = sort_desc(c, count);
+        s = sort_desc(c, m);
         if (s != PVS_OK) return fail(c, s);
         if (pvs::launch_pbm_emit(c->buf, (int)m, c->out_ids, c->out_scores, st) != cudaSuccess ||
             cudaMemcpyAsync(ids, c->out_ids, m * sizeof(int64_t), cudaMemcpyDeviceToHost, st) !=
@@ -447,7 +476,9 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
             return fail(c, PVS_ERR_CUDA);
         s = read_counters(c);   // also waits for the outputs
         if (s != PVS_OK) return fail(c, s);
-        if (c->h_ctr->collected != count) return fail(c, PVS_ERR_INVALID);   // internal invariant
+        if (c->h_ctr->collected != m) return fail(c, PVS_ERR_INVALID);   // internal invariant
+    }
+    if (m > 0) {
         c->last_key = pvs::rank_key(scores[m - 1], (uint32_t)ids[m - 1]);
         c->emitted += (int64_t)m;
     }

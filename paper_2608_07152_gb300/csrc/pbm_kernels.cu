@@ -284,7 +284,7 @@ __global__ void __launch_bounds__(256) pbm_bounds_kernel(PbmQuery q,
                                                          const int32_t* __restrict__ blk_range,
                                                          const float* __restrict__ blk_max,
                                                          int64_t n_ranges, int64_t nchunk,
-                                                         float* H, float* Hlive, int* status) {
+                                                         float* H, int* status) {
     __shared__ float h[kPbmChunk];
     const int64_t k = blockIdx.x;
     const int64_t r0 = k * kPbmChunk;
@@ -307,17 +307,16 @@ __global__ void __launch_bounds__(256) pbm_bounds_kernel(PbmQuery q,
         const float v = h[x];
         if (!isfinite(v)) set_status(status, PVS_ERR_OVERFLOW);
         H[r0 + x] = v;
-        Hlive[r0 + x] = v;
     }
 }
 
 cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const int32_t* blk_range,
                               const float* blk_max, int64_t n_ranges, int64_t nchunk, float* H,
-                              float* Hlive, int* status, cudaStream_t st) {
+                              int* status, cudaStream_t st) {
     if (nchunk <= 0) return cudaSuccess;
     count_launches(1);
     pbm_bounds_kernel<<<(unsigned)nchunk, 256, 0, st>>>(q, starts, blk_range, blk_max, n_ranges,
-                                                        nchunk, H, Hlive, status);
+                                                        nchunk, H, status);
     return cudaGetLastError();
 }
 
@@ -325,122 +324,117 @@ cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const in
 // pulls
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ unsigned long long warp_max_u64(unsigned long long v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long y = __shfl_xor_sync(0xffffffffu, v, o);
-        v = y > v ? y : v;
-    }
-    return v;
-}
-
-__global__ void pbm_kmax_kernel(const float* __restrict__ Hlive, int64_t n, int block,
-                                PbmCounters* ctr) {
-    unsigned long long m = 0;
+__global__ void pbm_range_keys_kernel(const float* __restrict__ H, int64_t n, int block,
+                                      uint64_t* rkeys) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n; r += stride) {
-        const float h = Hlive[r];
-        if (h != -INFINITY) {
-            const unsigned long long key = rank_key(h, (uint32_t)(r * block));
-            m = key > m ? key : m;
-        }
-    }
-    m = warp_max_u64(m);
-    if ((threadIdx.x & 31) == 0 && m != 0) atomicMax(&ctr->kmax, m);
+    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n; r += stride)
+        rkeys[r] = rank_key(H[r], (uint32_t)(r * block));
 }
 
-cudaError_t launch_pbm_kmax(const float* Hlive, int64_t n_ranges, int block, PbmCounters* ctr,
-                            cudaStream_t st) {
-    cudaError_t e = cudaMemsetAsync(&ctr->kmax, 0, sizeof(unsigned long long), st);
-    if (e != cudaSuccess) return e;
+cudaError_t launch_pbm_range_keys(const float* H, int64_t n_ranges, int block, uint64_t* rkeys,
+                                  cudaStream_t st) {
+    if (n_ranges <= 0) return cudaSuccess;
     count_launches(1);
-    pbm_kmax_kernel<<<grid_for(n_ranges, 256, 152 * 4), 256, 0, st>>>(Hlive, n_ranges, block, ctr);
+    pbm_range_keys_kernel<<<grid_for(n_ranges, 256, 152 * 4), 256, 0, st>>>(H, n_ranges, block,
+                                                                            rkeys);
     return cudaGetLastError();
 }
 
-__global__ void pbm_window_kernel(const uint64_t* __restrict__ pool, uint64_t hi,
-                                  PbmCounters* ctr) {
-    const unsigned long long lo = ctr->kmax;
+__global__ void pbm_window_kernel(const uint64_t* __restrict__ sorted, int64_t next,
+                                  int64_t n_ranges, const uint64_t* __restrict__ pool,
+                                  uint64_t hi, uint64_t* out, uint64_t cap, PbmCounters* ctr) {
+    const unsigned long long lo = next < n_ranges ? sorted[next] : 0ull;
+    if (blockIdx.x == 0 && threadIdx.x == 0) ctr->kmax = lo;
     const int64_t n = (int64_t)ctr->pool_len;
-    unsigned int c = 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const uint64_t k = pool[i];
-        c += (k > lo && k < hi) ? 1u : 0u;
-    }
-    c = warp_sum(c);
-    if ((threadIdx.x & 31) == 0 && c) atomicAdd(&ctr->window, (unsigned long long)c);
-}
-
-cudaError_t launch_pbm_window(const uint64_t* pool, uint64_t hi, PbmCounters* ctr,
-                              cudaStream_t st) {
-    cudaError_t e = cudaMemsetAsync(&ctr->window, 0, sizeof(unsigned long long), st);
-    if (e != cudaSuccess) return e;
-    count_launches(1);
-    pbm_window_kernel<<<152 * 4, 256, 0, st>>>(pool, hi, ctr);
-    return cudaGetLastError();
-}
-
-// Range keys: key(H, first id) of unexpanded ranges, 0 for expanded ones.
-__device__ __forceinline__ unsigned long long range_key(const float* Hlive, int64_t r, int block) {
-    const float h = Hlive[r];
-    return h == -INFINITY ? 0ull : rank_key(h, (uint32_t)(r * block));
-}
-
-__global__ void pbm_rsel_hist_kernel(const float* __restrict__ Hlive, int64_t n, int block,
-                                     int shift, unsigned long long* sel) {
-    __shared__ unsigned int h[256];
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) h[i] = 0;
-    __syncthreads();
-    const unsigned long long prefix = sel[0];
-    const int up = shift + 8;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n; r += stride) {
-        const unsigned long long k = range_key(Hlive, r, block);
-        if (k == 0) continue;
-        if (up < 64 && (k >> up) != (prefix >> up)) continue;
-        atomicAdd(&h[(k >> shift) & 0xffu], 1u);
-    }
-    __syncthreads();
-    for (int i = threadIdx.x; i < 256; i += blockDim.x)
-        if (h[i]) atomicAdd(&sel[2 + i], (unsigned long long)h[i]);
-}
-
-__global__ void pbm_sel_init_kernel(unsigned long long* sel, unsigned long long k);
-__global__ void pbm_sel_pick_kernel(int shift, unsigned long long* sel);
-
-__global__ void pbm_pick_kernel(const float* __restrict__ Hlive, int64_t n, int block,
-                                const unsigned long long* sel, int32_t* list, PbmCounters* ctr) {
-    const unsigned long long t = sel[0];
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < n; r += stride) {
-        const unsigned long long k = range_key(Hlive, r, block);
-        if (k != 0 && k >= t) {
-            const unsigned long long pos = atomicAdd(&ctr->picked, 1ull);
-            list[pos] = (int32_t)r;
+    const int lane = threadIdx.x & 31;
+    // whole warps iterate together so that the appends can be aggregated
+    for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < n;
+         i0 += stride) {
+        const int64_t i = i0 + lane;
+        uint64_t k = 0;
+        bool take = false;
+        if (i < n) {
+            k = pool[i];
+            take = k > lo && k < hi;
+        }
+        const unsigned int m = __ballot_sync(0xffffffffu, take);
+        if (m == 0) continue;
+        unsigned long long base = 0;
+        if (lane == 0) base = atomicAdd(&ctr->collected, (unsigned long long)__popc(m));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (take) {
+            const unsigned long long pos = base + __popc(m & ((1u << lane) - 1u));
+            if (pos < cap) out[pos] = k;
         }
     }
 }
 
-cudaError_t launch_pbm_pick(const float* Hlive, int64_t n_ranges, int block, uint64_t k,
-                            unsigned long long* sel64, int32_t* list, PbmCounters* ctr,
-                            cudaStream_t st) {
-    cudaError_t e = cudaMemsetAsync(&ctr->picked, 0, sizeof(unsigned long long), st);
+cudaError_t launch_pbm_window(const uint64_t* sorted, int64_t next, int64_t n_ranges,
+                              const uint64_t* pool, uint64_t hi, uint64_t* out, uint64_t cap,
+                              PbmCounters* ctr, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(&ctr->collected, 0, sizeof(unsigned long long), st);
     if (e != cudaSuccess) return e;
-    const int grid = grid_for(n_ranges, 256, 152 * 4);
     count_launches(1);
-    pbm_sel_init_kernel<<<1, 256, 0, st>>>(sel64, (unsigned long long)k);
-    for (int shift = 56; shift >= 0; shift -= 8) {
-        count_launches(2);
-        pbm_rsel_hist_kernel<<<grid, 256, 0, st>>>(Hlive, n_ranges, block, shift, sel64);
-        pbm_sel_pick_kernel<<<1, 32, 0, st>>>(shift, sel64);
-    }
-    count_launches(1);
-    pbm_pick_kernel<<<grid, 256, 0, st>>>(Hlive, n_ranges, block, sel64, list, ctr);
+    pbm_window_kernel<<<152 * 4, 256, 0, st>>>(sorted, next, n_ranges, pool, hi, out, cap, ctr);
     return cudaGetLastError();
 }
 
-// One CTA per picked range at a time: the range's block of every query term
+constexpr int kFinishThreads = 1024;
+
+__global__ void __launch_bounds__(kFinishThreads) pbm_finish_kernel(const uint64_t* keys_in,
+                                                                    const PbmCounters* ctr,
+                                                                    uint64_t need, int64_t* h_ids,
+                                                                    float* h_scores,
+                                                                    PbmCounters* h_mirror) {
+    extern __shared__ uint64_t keys[];
+    const unsigned long long count = ctr->collected;
+    if (need > 0 && count >= need && count <= (unsigned long long)kPbmFastWindow) {
+        int pow2 = 1;
+        while ((unsigned long long)pow2 < count) pow2 <<= 1;
+        for (int i = threadIdx.x; i < pow2; i += blockDim.x)
+            keys[i] = (unsigned long long)i < count ? keys_in[i] : 0ull;   // 0 sorts last
+        __syncthreads();
+        // bitonic sort, descending
+        for (int k = 2; k <= pow2; k <<= 1) {
+            for (int j = k >> 1; j > 0; j >>= 1) {
+                for (int i = threadIdx.x; i < pow2; i += blockDim.x) {
+                    const int ixj = i ^ j;
+                    if (ixj > i) {
+                        const uint64_t a = keys[i], b = keys[ixj];
+                        const bool swap = (i & k) == 0 ? a < b : a > b;
+                        if (swap) {
+                            keys[i] = b;
+                            keys[ixj] = a;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        for (int i = threadIdx.x; (unsigned long long)i < need; i += blockDim.x) {
+            h_ids[i] = (int64_t)rank_key_id(keys[i]);
+            h_scores[i] = rank_key_score(keys[i]);
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) *h_mirror = *ctr;
+}
+
+cudaError_t launch_pbm_finish(const uint64_t* keys, const PbmCounters* ctr, uint64_t need,
+                              int64_t* h_ids, float* h_scores, PbmCounters* h_mirror,
+                              cudaStream_t st) {
+    cudaError_t e = cudaFuncSetAttribute(pbm_finish_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kPbmFastWindow * (int)sizeof(uint64_t));
+    if (e != cudaSuccess) return e;
+    count_launches(1);
+    pbm_finish_kernel<<<1, kFinishThreads, kPbmFastWindow * sizeof(uint64_t), st>>>(
+        keys, ctr, need, h_ids, h_scores, h_mirror);
+    return cudaGetLastError();
+}
+
+// One CTA per range at a time: the range's block of every query term
 // (binary search within the term's blocks of the range's chunk), then the
 // postings term by term in query order into the items' float32 scores,
 // then every item of the range goes to the pool with its rank key.
@@ -454,10 +448,9 @@ __global__ void __launch_bounds__(kExpandThreads) pbm_expand_kernel(PbmExpandArg
     __shared__ unsigned long long base_sh;
     const int nq = a.q.nq;
     for (int i = threadIdx.x; i < nq; i += blockDim.x) w[i] = a.q.weights[i];
-    const unsigned long long picked = a.ctr->picked;
     const int64_t per = a.nchunk + 1;
-    for (unsigned long long e = blockIdx.x; e < picked; e += gridDim.x) {
-        const int64_t r = a.list[e];
+    for (int64_t e = blockIdx.x; e < a.count; e += gridDim.x) {
+        const int64_t r = (int64_t)rank_key_id(a.ranges[e]) / a.block;
         const int64_t k = r / kPbmChunk;
         const int64_t first = r * a.block;
         const int64_t rest = a.n_items - first;
@@ -494,7 +487,6 @@ __global__ void __launch_bounds__(kExpandThreads) pbm_expand_kernel(PbmExpandArg
             atomicAdd(&a.ctr->ranges_expanded, 1ull);
             atomicAdd(&a.ctr->postings, visited);
             atomicAdd(&a.ctr->items, (unsigned long long)cnt);
-            a.Hlive[r] = -INFINITY;
         }
         __syncthreads();
         const unsigned long long base = base_sh;

@@ -21,7 +21,6 @@ struct PbmCounters {
     unsigned long long ranges_expanded;
     unsigned long long postings;
     unsigned long long items;
-    unsigned long long picked;           // ranges picked in the current round
     unsigned long long collected;        // pool keys gathered for an emission
     int status;
     int pad;
@@ -59,26 +58,32 @@ struct PbmQuery {
 // starts[i * (nchunk + 1) + k] = first block of query term i with range >= k * kPbmChunk.
 cudaError_t launch_pbm_starts(const PbmQuery& q, const int64_t* blk_off, const int32_t* blk_range,
                               int64_t nchunk, int64_t* starts, cudaStream_t st);
-// H[r] (and Hlive[r] = H[r]) for every range, term by term in query order.
+// H[r] for every range, term by term in query order.
 cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const int32_t* blk_range,
                               const float* blk_max, int64_t n_ranges, int64_t nchunk, float* H,
-                              float* Hlive, int* status, cudaStream_t st);
+                              int* status, cudaStream_t st);
 
 // ---- pulls ---------------------------------------------------------------------
-// ctr->kmax = max over ranges with Hlive != -inf of rank_key(Hlive[r], r * block).
-cudaError_t launch_pbm_kmax(const float* Hlive, int64_t n_ranges, int block, PbmCounters* ctr,
-                            cudaStream_t st);
-// ctr->window = #{pool keys k: ctr->kmax < k < hi} over ctr->pool_len keys.
-cudaError_t launch_pbm_window(const uint64_t* pool, uint64_t hi, PbmCounters* ctr,
+// rkeys[r] = key(H[r], r * block): the ranges' competition keys (sorted once,
+// descending, at open; the ranges are then expanded in that order).
+cudaError_t launch_pbm_range_keys(const float* H, int64_t n_ranges, int block, uint64_t* rkeys,
+                                  cudaStream_t st);
+// ctr->kmax = sorted[next] (0 once every range is expanded) and the pool
+// keys k with ctr->kmax < k < hi (the certified window): counted in
+// ctr->collected, the first `cap` of them (any order) written to out.
+cudaError_t launch_pbm_window(const uint64_t* sorted, int64_t next, int64_t n_ranges,
+                              const uint64_t* pool, uint64_t hi, uint64_t* out, uint64_t cap,
+                              PbmCounters* ctr, cudaStream_t st);
+// One CTA: when need <= ctr->collected <= kPbmFastWindow, sorts the collected
+// keys and writes the first `need` ids / scores to h_ids / h_scores; always
+// copies *ctr to *h_mirror last.  h_* may be pinned host memory.
+constexpr int kPbmFastWindow = 8192;
+cudaError_t launch_pbm_finish(const uint64_t* keys, const PbmCounters* ctr, uint64_t need,
+                              int64_t* h_ids, float* h_scores, PbmCounters* h_mirror,
                               cudaStream_t st);
-// The k unexpanded ranges with the largest keys key(Hlive[r], r * block)
-// (k <= unexpanded ranges) go to list, ctr->picked = k; sel64 holds 2 + 256
-// words of selection state.
-cudaError_t launch_pbm_pick(const float* Hlive, int64_t n_ranges, int block, uint64_t k,
-                            unsigned long long* sel64, int32_t* list, PbmCounters* ctr,
-                            cudaStream_t st);
 struct PbmExpandArgs {
-    const int32_t* list;          // picked ranges; count in ctr->picked
+    const uint64_t* ranges;       // sorted range keys of the ranges to expand
+    int64_t count;                // how many
     PbmQuery q;
     const int64_t* starts;
     int64_t nchunk;
@@ -88,7 +93,6 @@ struct PbmExpandArgs {
     const float* imps;
     int64_t n_items;
     int block;
-    float* Hlive;
     uint64_t* pool;
     PbmCounters* ctr;
 };
