@@ -57,12 +57,13 @@ def parse():
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="passage",
-                   choices=["passage", "batched", "eahr", "snapshots", "sparse"],
+                   choices=["passage", "batched", "eahr", "snapshots", "sparse", "hybrid"],
                    help="passage: single-query ranking (default); batched: 256-query "
                         "tensor-core batches; eahr: EAHR Top-20 fusion over the passage "
                         "corpus and copula sparse rankings; snapshots: near-duplicate "
                         "corpus, five snapshots, EAHR Top-20; sparse: PBM sparse ranks "
-                        "over a synthetic BM25 corpus")
+                        "over a synthetic BM25 corpus; hybrid: EAHR Top-20 over PVS and PBM "
+                        "on the same items")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
@@ -762,6 +763,141 @@ def main_sparse(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+HYBRID_TOPIC_TERMS = 64     # topic block per mixture component
+HYBRID_TOPIC_SHARE = 0.3    # share of an item's tokens drawn from its topic block
+
+
+def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """EAHR end to end with both generators on the GPU: PVS over the passage
+    mixture corpus (dense) and PBM over a topical synthetic BM25 corpus of
+    the same items (sparse: a share of every item's tokens comes from its
+    mixture component's term block, and each query draws terms from its own
+    component's block, so the two rankings agree in part).  Timed per query:
+    both cursors opened, eahr_topk_pbm, both closed.  Beside it, the
+    exhaustive comparator in plain torch: fp32 dense scores of every row and a
+    full sort, the complete sparse ranking, and complete-list fusion."""
+    n = args.n
+    stream = torch.cuda.Stream(device=dev)
+    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=dev)
+    t0 = time.perf_counter()
+    rows = torch.empty((n, DIM), dtype=torch.float32, device=dev)
+    chunk = 1 << 20
+    for r in range(0, n, chunk):
+        c = min(chunk, n - r)
+        rows[r:r + c] = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+    index = pvs.pvs_build(rows, stream=stream.cuda_stream)
+    torch.cuda.synchronize()
+    dense_build_s = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    comps = synth.mixture_components(n, COMPONENTS, seed=2, device=dev)
+    off, docs, imps = synth.bm25_postings(n, SPARSE_TERMS, SPARSE_TOKENS, seed=10, device=dev,
+                                          topic_of=comps, topic_terms=HYBRID_TOPIC_TERMS,
+                                          topic_share=HYBRID_TOPIC_SHARE)
+    del comps
+    sindex = pvs.pbm_build(off, docs, imps, n)
+    torch.cuda.synchronize()
+    sparse_build_s = time.perf_counter() - t0
+    nq = 2 + args.eahr_queries
+    dq = synth.mixture_queries(nq, centres, QUERY_NOISE, seed=query_seed(12, rank))
+    qc = synth.mixture_query_components(nq, COMPONENTS, seed=query_seed(12, rank), device=dev)
+    sq = synth.topical_queries(qc, off, SPARSE_TERMS, HYBRID_TOPIC_TERMS,
+                               seed=query_seed(13, rank))
+
+    def one(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        dcur = pvs.pvs_cursor_open(index, dq[i])
+        scur = pvs.pbm_cursor_open(sindex, *sq[i])
+        ids, F, st = pvs.eahr_topk_pbm(dcur, scur, K=EAHR_K, k=EAHR_RRF_K,
+                                       form=pvs.EAHR_NUMERATOR)
+        ps = pvs.pbm_cursor_stats(scur)
+        pvs.pbm_cursor_close(scur)
+        pvs.pvs_cursor_close(dcur)
+        ms = (time.perf_counter() - t) * 1e3
+        if len(ids) != EAHR_K:
+            raise RuntimeError("EAHR returned a short list")
+        return ms, st, ps
+
+    def full_orders(i):
+        sc = rows @ dq[i]
+        dorder = torch.argsort(sc, descending=True, stable=True)
+        ss = torch.zeros(n, dtype=torch.float32, device=dev)
+        for term, w in zip(sq[i][0].tolist(), sq[i][1].tolist()):
+            a, b = int(off[term]), int(off[term + 1])
+            ss.index_put_((docs[a:b].long(),), imps[a:b] * w, accumulate=True)
+        sorder = torch.argsort(ss, descending=True, stable=True)
+        return dorder, sorder
+
+    def comparator(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        dorder, sorder = full_orders(i)
+        ar = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
+        rd = torch.empty(n, dtype=torch.float64, device=dev)
+        rd[dorder] = ar
+        rs = torch.empty(n, dtype=torch.float64, device=dev)
+        rs[sorder] = ar
+        fused = 1.0 / (EAHR_RRF_K + rd) + 1.0 / (EAHR_RRF_K + rs)
+        torch.topk(fused, EAHR_K).indices.cpu()
+        return (time.perf_counter() - t) * 1e3
+
+    for w in range(2):
+        one(w)
+        comparator(w)
+    dorder, sorder = full_orders(2)
+    ktau = synth.kendall_tau_sample(dorder.cpu().numpy(), sorder.cpu().numpy(), 200_000, seed=5)
+    del dorder, sorder
+    if pg:
+        pg.barrier()
+    launches0 = pvs.pvs_launch_count()
+    lat, dd, ds, ex, rexp = [], [], [], 0, []
+    with ClockSampler(local) as clk:
+        for i in range(2, nq):
+            ms, st, ps = one(i)
+            lat.append(ms)
+            dd.append(st["depth"][0])
+            ds.append(st["depth"][1])
+            ex += int(st["exhausted"][0] and st["exhausted"][1])
+            rexp.append(ps["ranges_expanded"])
+    launches = pvs.pvs_launch_count() - launches0
+    cmp_ms = [comparator(i) for i in range(2, min(nq, 22))]
+    line = {
+        "metric": "EAHR Top-20 latency, PVS dense + PBM sparse (p50)",
+        "value": float(np.median(lat)), "unit": "ms", "n_gpus": world, "steps": len(lat),
+        "warmup": 2, "ms_per_step": float(np.mean(lat)), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": f"EAHR over PVS (passage mixture N={n:,} x d={DIM}) and PBM "
+                               f"(topical synthetic BM25 over the same items: vocabulary "
+                               f"{SPARSE_TERMS:,} + {COMPONENTS} x {HYBRID_TOPIC_TERMS} topic "
+                               f"terms, topic share {HYBRID_TOPIC_SHARE}), weighted RRF "
+                               f"1/(60+rank), K={EAHR_K}",
+                   "N": n, "d": DIM, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
+                   "postings": int(docs.numel()),
+                   "l2": "no flush: every query's interval pass streams 6.9 GB of codes",
+                   "parallelism": f"replicas x{world}"},
+        "e2e": {"value": float(np.median(lat)), "unit": "ms",
+                "h2d_bytes_per_step": DIM * 4 + int(np.mean([8 * len(q[0]) for q in sq])),
+                "d2h_bytes_per_step": EAHR_K * 16},
+        "latency_ms": {"p50": float(np.median(lat)), "p95": float(np.percentile(lat, 95)),
+                       "p99": float(np.percentile(lat, 99))},
+        "kendall_tau_dense_sparse": ktau,
+        "dense_depth_p50": float(np.median(dd)), "sparse_depth_p50": float(np.median(ds)),
+        "both_exhausted": ex, "pbm_ranges_expanded_p50": float(np.median(rexp)),
+        "pbm_ranges": pvs.pbm_index_ranges(sindex),
+        "exhaustive_torch_ms_p50": float(np.median(cmp_ms)),
+        "gpu_launches": launches,
+        "dense_build_s": dense_build_s, "sparse_build_s": sparse_build_s,
+        "clocks": clk.summary(),
+    }
+    pvs.pbm_index_free(sindex)
+    pvs.pvs_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 SNAP_N = 2_000_000
 SNAP_DIM = 1024
 SNAP_DUP = 0.2          # near-duplicate share of the base corpus
@@ -921,6 +1057,9 @@ def main():
         return
     if args.workload == "sparse":
         main_sparse(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
+    if args.workload == "hybrid":
+        main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
     stream = torch.cuda.Stream(device=dev)

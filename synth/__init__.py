@@ -17,13 +17,17 @@ generators stand in for them with the shapes and structure of the workloads:
 * ``controlled_streams`` the rank relations of the controlled-stream study
                          (block-32 correlated, partial overlap, independent,
                          reversed, all tied);
-* ``bm25_postings`` / ``sparse_queries``
+* ``bm25_postings`` / ``sparse_queries`` / ``topical_queries``
                          a stand-in for BM25 impact postings: term draws from
                          a Zipf law (the most frequent ranks removed like
                          stopwords), term frequencies from repeated draws,
                          BM25 weights (k1 = 0.9, b = 0.4) from the corpus's own
                          document frequencies and lengths, as term-major CSR;
-                         queries of a few distinct terms of weight 1.
+                         optionally a share of each item's tokens from a
+                         block of terms of its topic (its mixture component,
+                         see ``mixture_components``), so that sparse and
+                         dense rankings agree in part; queries of a few
+                         distinct terms of weight 1.
 
 Every generator is deterministic in its seed; large matrices are produced in
 row chunks, each with its own derived seed, so any chunk can be regenerated
@@ -90,6 +94,23 @@ def mixture_rows(n: int, centres: torch.Tensor, within_std: float, seed: int,
         x.mul_(within_std).add_(centres[comp])
         out[r:r + c] = _normalise(x)
     return out
+
+
+def mixture_components(n: int, n_components: int, seed: int, device="cpu") -> torch.Tensor:
+    """The mixture component of rows 0 .. n-1 of mixture_rows(seed=seed) on
+    the same device type: the same generator draws, replayed."""
+    out = torch.empty(n, dtype=torch.int64, device=device)
+    for r in range(0, n, CHUNK_ROWS):
+        c = min(CHUNK_ROWS, n - r)
+        g = _gen(_chunk_seed(seed, r // CHUNK_ROWS), device)
+        out[r:r + c] = torch.randint(0, n_components, (c,), generator=g, device=device)
+    return out
+
+
+def mixture_query_components(nq: int, n_components: int, seed: int, device="cpu") -> torch.Tensor:
+    """The component of each query of mixture_queries(seed=seed), replayed."""
+    g = _gen(_chunk_seed(seed, -2), device)
+    return torch.randint(0, n_components, (nq,), generator=g, device=device)
 
 
 def mixture_queries(nq: int, centres: torch.Tensor, noise_std: float, seed: int) -> torch.Tensor:
@@ -191,7 +212,8 @@ def _zipf_cdf(n_terms: int, exponent: float, skip: int, device) -> torch.Tensor:
 
 
 def bm25_postings(n_items: int, n_terms: int, mean_tokens: float, seed: int, device="cpu",
-                  exponent: float = 1.0, skip: int = 100, k1: float = 0.9, b: float = 0.4):
+                  exponent: float = 1.0, skip: int = 100, k1: float = 0.9, b: float = 0.4,
+                  topic_of=None, topic_terms: int = 0, topic_share: float = 0.0):
     """Term-major postings (term_off int64 [n_terms + 1], docs int32, imps
     float32) of a synthetic corpus with BM25 impacts.
 
@@ -201,8 +223,19 @@ def bm25_postings(n_items: int, n_terms: int, mean_tokens: float, seed: int, dev
     term frequency tf.  The impact of term t on item x is the BM25 weight
     idf_t * tf (k1 + 1) / (tf + k1 (1 - b + b dl_x / avgdl)) with
     idf_t = ln(1 + (N - df_t + 0.5) / (df_t + 0.5)), computed in float64 and
-    stored as float32.  Postings of a term are in ascending item id."""
+    stored as float32.  Postings of a term are in ascending item id.
+
+    Topics (optional): with topic_of[x] the topic of item x (e.g. its mixture
+    component), each token is, with probability topic_share, a uniform draw
+    from the item's own block of topic_terms terms, numbered after the
+    n_terms background terms (the vocabulary then has n_terms +
+    n_topics * topic_terms terms, n_topics = max(topic_of) + 1)."""
     cdf = _zipf_cdf(n_terms, exponent, skip, device)
+    n_topics = 0
+    if topic_of is not None and topic_terms > 0:
+        topic_of = topic_of.to(device=device, dtype=torch.int64)
+        n_topics = int(topic_of.max().item()) + 1
+    vocab = n_terms + n_topics * topic_terms
     g = _gen(_chunk_seed(seed, -11), device)
     dl = torch.poisson(torch.full((n_items,), float(mean_tokens), dtype=torch.float64,
                                   device=device), generator=g).to(torch.int64)
@@ -218,6 +251,11 @@ def bm25_postings(n_items: int, n_terms: int, mean_tokens: float, seed: int, dev
         u = torch.rand(total, generator=gc, dtype=torch.float64, device=device)
         terms = torch.searchsorted(cdf, u).clamp_max(n_terms - 1)
         docs = torch.repeat_interleave(torch.arange(c0, c1, device=device), lens)
+        if n_topics:
+            pick = torch.rand(total, generator=gc, device=device) < topic_share
+            j = torch.randint(0, topic_terms, (total,), generator=gc, device=device)
+            topical = n_terms + topic_of[docs] * topic_terms + j
+            terms = torch.where(pick, topical, terms)
         keys.append(terms * n_items + docs)
     if keys:
         key = torch.sort(torch.cat(keys)).values
@@ -227,8 +265,8 @@ def bm25_postings(n_items: int, n_terms: int, mean_tokens: float, seed: int, dev
         tf = torch.empty(0, dtype=torch.int64, device=device)
     term = uniq // n_items
     docs = (uniq % n_items).to(torch.int32)
-    df = torch.bincount(term, minlength=n_terms)
-    term_off = torch.zeros(n_terms + 1, dtype=torch.int64, device=device)
+    df = torch.bincount(term, minlength=vocab)
+    term_off = torch.zeros(vocab + 1, dtype=torch.int64, device=device)
     term_off[1:] = torch.cumsum(df, 0)
     dlf = dl.to(torch.float64)
     avgdl = float(dlf.mean().item()) if n_items else 1.0
@@ -258,4 +296,31 @@ def sparse_queries(nq: int, term_off: torch.Tensor, seed: int, mean_terms: float
         k = min(ok.size, 1 + int(rng.poisson(max(mean_terms - 1.0, 0.0))))
         t = rng.choice(ok, size=k, replace=False, p=p).astype(np.int32)
         out.append((t, np.ones(k, np.float32)))
+    return out
+
+
+def topical_queries(query_topics, term_off: torch.Tensor, n_terms: int, topic_terms: int,
+                    seed: int, mean_topic: float = 2.0, mean_background: float = 2.0,
+                    min_df: int = 2):
+    """Sparse queries that match the topical corpus of bm25_postings: query i
+    takes 1 + Poisson(mean_topic - 1) distinct terms of its topic's block
+    (those with postings) and Poisson(mean_background) distinct background
+    terms drawn in proportion to their document frequency, all of weight 1,
+    topic terms first.  Returns a list of (terms int32, weights float32)."""
+    off = term_off.detach().cpu().numpy().astype(np.int64)
+    df = np.diff(off)
+    bg = np.flatnonzero(df[:n_terms] >= min_df)
+    p = df[bg].astype(np.float64)
+    p /= p.sum()
+    rng = np.random.default_rng(int(seed) & ((1 << 63) - 1))
+    out = []
+    for c in np.asarray(query_topics.detach().cpu() if hasattr(query_topics, "detach")
+                        else query_topics).tolist():
+        block = n_terms + int(c) * topic_terms + np.arange(topic_terms)
+        block = block[df[block] > 0]
+        kt = min(block.size, 1 + int(rng.poisson(max(mean_topic - 1.0, 0.0))))
+        kb = min(bg.size, int(rng.poisson(mean_background)))
+        t = np.concatenate([rng.choice(block, size=kt, replace=False),
+                            rng.choice(bg, size=kb, replace=False, p=p)]).astype(np.int32)
+        out.append((t, np.ones(t.size, np.float32)))
     return out
