@@ -10,8 +10,10 @@ Modules
 -------
 ``pvs_oracle``   PVS quantization, norm bounds, gamma_m, score intervals
                  (Sec. 2.3.1, Appendix A.1; the bound arithmetic is in
-                 ``pvs_ref.c``), the authoritative float32 score and the
-                 complete dense ranking (Sec. 2.1).
+                 ``pvs_ref.c``), the one-scale quantization of the
+                 scalar-quantization ablation (Sec. 3.5, 4.4), the
+                 authoritative float32 score and the complete dense ranking
+                 (Sec. 2.1).
 ``pbm_oracle``   PBM sparse scores S(x) and range bounds H(R) in the fixed
                  float32 term order (Sec. 2.3.2, Appendix A.2), block
                  maxima, and the complete sparse ranking (Sec. 2.1).

@@ -47,6 +47,10 @@ def lib() -> ctypes.CDLL:
             L.orc_gamma.argtypes = [i32]
             L.orc_quantize.restype = i32
             L.orc_quantize.argtypes = [P, i64, i32, P, i32, P, P, P, P]
+            L.orc_global_scale.restype = ctypes.c_float
+            L.orc_global_scale.argtypes = [P, i64, i32]
+            L.orc_quantize_fixed.restype = i32
+            L.orc_quantize_fixed.argtypes = [P, i64, i32, P, i32, ctypes.c_float, P, P, P, P]
             L.orc_qhat_norm.restype = f32
             L.orc_qhat_norm.argtypes = [P, f32, i32, P]
             L.orc_interval_one.restype = None

@@ -12,6 +12,11 @@ Paper: arXiv 2608.07152.
                gamma_m >= a_m / (1 - a_m), a_m = (8m + 64) eps_f32, outward
                rounded endpoints, failure on non-finite input.
 
+Scalar-quantization intervals (the rank-generator ablation of Sec. 3.5 and
+4.4; the paper gives no construction; reading): one scale s = RN(max |v_j| /
+127) over the whole corpus in place of every s_v, with the same codes,
+residual bounds and intervals (``global_scale``, ``quantize_global``).
+
 Authoritative float32 score (the paper fixes no summation order; reading):
 the correctly rounded (to nearest, ties to even) float32 value of the exact
 real inner product sum_j q_j v_j.  It lies within every interval the guard
@@ -59,6 +64,32 @@ def quantize(V: np.ndarray, ldz: int | None = None) -> Quantized:
     st = _clib.lib().orc_quantize(_ptr(V), n, m, _ptr(Z), ldz, _ptr(s), _ptr(vn),
                                   _ptr(en), _ptr(scratch))
     return Quantized(Z, s, vn, en, int(st))
+
+
+def global_scale(V: np.ndarray) -> np.float32:
+    """Scalar-quantization intervals (the ablation of Sec. 3.5 / 4.4): one
+    scale RN(max |v_j| / 127) for the whole corpus (NaN for non-finite input)."""
+    V = np.ascontiguousarray(V, dtype=np.float32)
+    n, m = V.shape
+    return np.float32(_clib.lib().orc_global_scale(_ptr(V), n, m))
+
+
+def quantize_global(V: np.ndarray, s=None, ldz: int | None = None) -> Quantized:
+    """Quantize every row with one scale s (default: global_scale(V)); codes,
+    residuals and norm bounds as Sec. 2.3.1 with s in place of s_v.  Status 3
+    marks a row whose codes would leave [-127, 127]."""
+    V = np.ascontiguousarray(V, dtype=np.float32)
+    n, m = V.shape
+    ldz = m if ldz is None else ldz
+    s = global_scale(V) if s is None else np.float32(s)
+    Z = np.zeros((n, ldz), dtype=np.int8)
+    sv = np.zeros(n, np.float32)
+    vn = np.zeros(n, np.float32)
+    en = np.zeros(n, np.float32)
+    scratch = np.zeros(max(m, 1), np.float64)
+    st = _clib.lib().orc_quantize_fixed(_ptr(V), n, m, _ptr(Z), ldz, float(s), _ptr(sv),
+                                        _ptr(vn), _ptr(en), _ptr(scratch))
+    return Quantized(Z, sv, vn, en, int(st))
 
 
 def norm_bound(x) -> np.float32:

@@ -191,6 +191,60 @@ int32_t orc_quantize(const float* V, int64_t n, int32_t m, int8_t* Z, int32_t ld
     return status;
 }
 
+/* Scalar-quantization intervals (the ablation of Sec. 3.5 / 4.4; reading of
+ * this library): one scale for the whole corpus, s = RN(max_{v,j} |v_j| /
+ * 127) (1 for an all-zero corpus, the smallest subnormal if the quotient
+ * underflows), the same codes, residuals and norm bounds as Sec. 2.3.1 per
+ * vector with s in place of s_v.  Returns the scale, or NaN if an entry is
+ * not finite. */
+float orc_global_scale(const float* V, int64_t n, int32_t m) {
+    float maxabs = 0.0f;
+    for (int64_t i = 0; i < n * (int64_t)m; ++i) {
+        if (!isfinite(V[i])) return NAN;
+        float a = fabsf(V[i]);
+        if (a > maxabs) maxabs = a;
+    }
+    if (maxabs == 0.0f) return 1.0f;
+    float s = f32_op(FE_TONEAREST, '/', maxabs, 127.0f);
+    if (s == 0.0f) s = ldexpf(1.0f, -149);
+    return s;
+}
+
+/* Quantize n vectors with the given scale s: z_j = round_half_away(RN(v_j /
+ * s)); returns 0, 1 for a non-finite entry, 2 for a norm bound that
+ * overflows, 3 when a code would leave [-127, 127] (the vector is outside the
+ * scale's range: the index rejects it rather than clip). */
+int32_t orc_quantize_fixed(const float* V, int64_t n, int32_t m, int8_t* Z, int32_t ldz,
+                           float s, float* s_out, float* vnorm, float* enorm, double* scratch) {
+    int32_t status = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        const float* v = V + i * (int64_t)m;
+        int8_t* z = Z + i * (int64_t)ldz;
+        for (int32_t j = m; j < ldz; ++j) z[j] = 0;
+        int32_t st = 0;
+        for (int32_t j = 0; j < m; ++j) {
+            if (!isfinite(v[j])) st = 1;
+        }
+        if (!st) {
+            for (int32_t j = 0; j < m; ++j) {
+                float t = f32_op(FE_TONEAREST, '/', v[j], s);
+                double r = round_half_away((double)t);
+                if (r > 127.0 || r < -127.0) st = 3;
+                z[j] = (int8_t)(r > 127.0 ? 127 : (r < -127.0 ? -127 : r));
+            }
+            for (int32_t j = 0; j < m; ++j) scratch[j] = (double)v[j];
+            vnorm[i] = orc_norm_bound(scratch, m);
+            for (int32_t j = 0; j < m; ++j)
+                scratch[j] = (double)v[j] - (double)s * (double)z[j];
+            enorm[i] = orc_norm_bound(scratch, m);
+            if (!st && (isinf(vnorm[i]) || isinf(enorm[i]))) st = 2;
+        }
+        s_out[i] = s;
+        if (st && !status) status = st;
+    }
+    return status;
+}
+
 /* qhat_up = norm_bound(s_q * z_q). */
 float orc_qhat_norm(const int8_t* zq, float sq, int32_t m, double* scratch) {
     for (int32_t j = 0; j < m; ++j) scratch[j] = (double)sq * (double)zq[j];

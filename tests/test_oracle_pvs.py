@@ -325,3 +325,72 @@ def test_dense_ranking_brute_force_with_ties():
     vis[::3] = False
     ids2, _ = po.dense_ranking(q, V, vis)
     assert ids2.tolist() == [i for i in expected if vis[i]]
+
+
+# ---------------------------------------------------------------------------
+# scalar-quantization intervals (one scale for the corpus; ablation of
+# Sec. 3.5 / 4.4, reading of this library)
+# ---------------------------------------------------------------------------
+
+def test_global_scale_is_f32_of_corpus_maxabs_over_127():
+    rng = np.random.default_rng(61)
+    V = (rng.standard_normal((40, 24)) * rng.gamma(1.0, 2.0, size=(40, 1))).astype(np.float32)
+    s = po.global_scale(V)
+    mx = Fraction(float(np.abs(V).max()))
+    # s = RN_f32(mx / 127): the float32 nearest to the exact quotient
+    cands = sorted({np.float32(float(mx / 127)), np.nextafter(np.float32(float(mx / 127)), 0),
+                    np.nextafter(np.float32(float(mx / 127)), np.inf)},
+                   key=lambda c: (abs(Fraction(float(c)) - mx / 127), int(np.float32(c).view(np.uint32)) & 1))
+    assert s == cands[0]
+    assert po.global_scale(np.zeros((3, 5), np.float32)) == np.float32(1.0)
+    bad = V.copy()
+    bad[3, 4] = np.inf
+    assert np.isnan(po.global_scale(bad))
+
+
+def test_global_quantization_reduces_to_per_vector_when_every_row_has_the_corpus_max():
+    # rows with one common infinity norm: the global scale is every row's own
+    # scale, so codes, residual bounds and intervals coincide with Sec. 2.3.1
+    rng = np.random.default_rng(62)
+    V = rng.standard_normal((64, 32)).astype(np.float32)
+    V /= np.abs(V).max(axis=1, keepdims=True)
+    V[np.arange(64), rng.integers(0, 32, 64)] = np.where(rng.random(64) < 0.5, 1.0, -1.0)
+    Qp = po.quantize(V)
+    Qg = po.quantize_global(V)
+    assert Qg.status == 0
+    assert np.array_equal(Qp.s, Qg.s)
+    assert np.array_equal(Qp.z, Qg.z)
+    assert np.array_equal(Qp.vnorm.view(np.uint32), Qg.vnorm.view(np.uint32))
+    assert np.array_equal(Qp.enorm.view(np.uint32), Qg.enorm.view(np.uint32))
+
+
+@pytest.mark.parametrize("seed", [63, 64])
+def test_global_quantization_intervals_contain_the_exact_scores(seed):
+    rng = np.random.default_rng(seed)
+    m = 48
+    # rows of very different norms: the global scale is coarse for the small ones
+    V = (rng.standard_normal((300, m)) * rng.gamma(0.7, 1.0, size=(300, 1))).astype(np.float32)
+    q = rng.standard_normal(m).astype(np.float32)
+    Qg = po.quantize_global(V)
+    assert Qg.status == 0
+    qe = po.encode_query(q)
+    lo, hi = po.intervals(qe, Qg, m)
+    s = po.exact_scores(q, V)
+    assert np.all(lo <= s) and np.all(s <= hi)
+    # coarser codes, wider intervals than per-vector quantization on average
+    lo_p, hi_p = po.intervals(qe, po.quantize(V), m)
+    assert np.mean(hi - lo) > np.mean(hi_p - lo_p)
+    # a row of all-small entries has all-zero codes and its residual is itself
+    tiny = np.full((1, m), 1e-3 * float(po.global_scale(V)), np.float32)
+    Qt = po.quantize_global(tiny, s=po.global_scale(V))
+    assert Qt.status == 0 and not Qt.z.any()
+    assert Qt.enorm[0] == Qt.vnorm[0]
+
+
+def test_global_quantization_rejects_rows_outside_the_range():
+    V = np.array([[1.0, -0.5, 0.25]], np.float32)
+    s = po.global_scale(V)
+    ok = po.quantize_global(np.array([[1.0, 0.0, 0.0]], np.float32), s=s)
+    assert ok.status == 0 and ok.z[0, 0] == 127
+    out = po.quantize_global(np.array([[1.5, 0.0, 0.0]], np.float32), s=s)
+    assert out.status == 3
