@@ -53,6 +53,20 @@ typedef enum pvs_status {
     PVS_ERR_FAILED = -8       /* the cursor failed earlier                     */
 } pvs_status;
 
+/* Corpus quantization of an index (pvs_build_ex). */
+typedef enum pvs_quantization {
+    PVS_QUANT_PER_VECTOR = 0,   /* PVS: each vector its own scale (Sec. 2.3.1)             */
+    PVS_QUANT_GLOBAL = 1        /* scalar-quantization intervals: one scale for the corpus,
+                                   the rank-generator ablation of Sec. 3.5 / 4.4           */
+} pvs_quantization;
+
+/* Rank generator of a cursor (pvs_cursor_set_generator). */
+typedef enum pvs_generator {
+    PVS_GEN_INTERVALS = 0,      /* score intervals, selective exact evaluation (default)   */
+    PVS_GEN_FULL_SCAN = 1       /* exhaustive float32 scanning: every visible row scored
+                                   exactly, one full sort (ablation, Sec. 3.5 / 4.4)       */
+} pvs_generator;
+
 typedef struct pvs_index pvs_index;
 typedef struct pvs_snapshot pvs_snapshot;
 typedef struct pvs_cursor pvs_cursor;
@@ -94,6 +108,18 @@ typedef struct pvs_stats {
  * *out owns device copies of everything; free it with pvs_index_free. */
 pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
                      void* cuda_stream, pvs_index** out);
+
+/* pvs_build with a choice of corpus quantization.  PVS_QUANT_GLOBAL gives
+ * the scalar-quantization-interval index of the rank-generator ablation
+ * (Sec. 3.5, 4.4; the paper gives no construction, reading of this
+ * library): one scale s = RN(max_{v,j} |v_j| / 127) over the n vectors, the
+ * codes, norm bounds and intervals of Sec. 2.3.1 / App. A.1 with s in place
+ * of every s_v; queries keep their own scale.  pvs_append on such an index
+ * uses the same s and fails with PVS_ERR_INVALID for a vector whose codes
+ * would leave [-127, 127].  Errors as pvs_build, and PVS_ERR_INVALID for an
+ * unknown quantization. */
+pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
+                        void* cuda_stream, int32_t quantization, pvs_index** out);
 
 /* Append n vectors; they get ids size .. size+n-1.  Existing snapshots and
  * open cursors keep their visible set (Sec. 2.4: fixed snapshots).  Errors
@@ -185,6 +211,14 @@ pvs_status pvs_next_device(pvs_cursor* cursor, int32_t n, int64_t* ids, float* s
  * another query's interval pass streams the codes.  Ordering against work
  * the caller queues elsewhere is the caller's. */
 pvs_status pvs_cursor_set_stream(pvs_cursor* cursor, void* cuda_stream);
+
+/* Choose the cursor's rank generator (pvs_generator) before its first pull:
+ * PVS_GEN_INTERVALS (default) or PVS_GEN_FULL_SCAN (every visible row scored
+ * exactly at the first pull, then one full sort; pulls read it in order).
+ * Both produce the same ranking.  Cursors of pvs_cursor_open_batch keep
+ * PVS_GEN_INTERVALS.  Errors: PVS_ERR_INVALID (unknown generator, a cursor
+ * already pulled, a batched cursor). */
+pvs_status pvs_cursor_set_generator(pvs_cursor* cursor, int32_t generator);
 
 /* Wait for the cursor's queued work; return its state (PVS_OK while Open,
  * PVS_EXHAUSTED, or the failure). */

@@ -30,6 +30,11 @@ PVS_ERR_OOM = -6
 PVS_ERR_TIMEOUT = -7
 PVS_ERR_FAILED = -8
 
+PVS_QUANT_PER_VECTOR = 0
+PVS_QUANT_GLOBAL = 1
+PVS_GEN_INTERVALS = 0
+PVS_GEN_FULL_SCAN = 1
+
 EAHR_RANK_SCALED = 0
 EAHR_NUMERATOR = 1
 EAHR_POLICY_GEOMETRIC = 0
@@ -79,6 +84,8 @@ def _load() -> ctypes.CDLL:
     pp = ctypes.POINTER(ctypes.c_void_p)
     sig = {
         "pvs_build": (i32, [P, i64, i32, i32, P, pp]),
+        "pvs_build_ex": (i32, [P, i64, i32, i32, P, i32, pp]),
+        "pvs_cursor_set_generator": (i32, [P, i32]),
         "pvs_append": (i32, [P, P, i64, i32]),
         "pvs_tombstone": (i32, [P, P, i64]),
         "pvs_index_size": (i64, [P]),
@@ -132,7 +139,7 @@ def _load() -> ctypes.CDLL:
 
 _lib = _load()
 lib_path = _LIB_PATH
-EXPORTED = ("pvs_build", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_index_live",
+EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append", "pvs_tombstone", "pvs_index_size", "pvs_index_live",
             "pvs_index_dim", "pvs_index_export", "pvs_index_free", "pvs_snapshot_create",
             "pvs_snapshot_visible", "pvs_snapshot_free", "pvs_cursor_open",
             "pvs_cursor_open_batch", "pvs_next", "pvs_next_device", "pvs_cursor_sync",
@@ -178,14 +185,24 @@ def _vec_arg(x, dim: int | None = None):
     return ctypes.c_void_p(a.ctypes.data), a.shape, 0, a
 
 
-def pvs_build(vecs, stream=None):
-    """Build an index over the rows of a 2-D float32 array / tensor."""
+def pvs_build(vecs, stream=None, quantization: int = PVS_QUANT_PER_VECTOR):
+    """Build an index over the rows of a 2-D float32 array / tensor
+    (quantization: PVS_QUANT_PER_VECTOR, or PVS_QUANT_GLOBAL for the
+    scalar-quantization-interval index of the ablation, via pvs_build_ex)."""
     ptr, shape, on_dev, keep = _vec_arg(vecs)
     n, dim = (shape[0], shape[1]) if len(shape) == 2 else (0, shape[-1])
     out = ctypes.c_void_p()
     st = ctypes.c_void_p(stream) if stream else None
-    _check(_lib.pvs_build(ptr, n, dim, on_dev, st, ctypes.byref(out)), "pvs_build")
+    if quantization == PVS_QUANT_PER_VECTOR:
+        _check(_lib.pvs_build(ptr, n, dim, on_dev, st, ctypes.byref(out)), "pvs_build")
+    else:
+        _check(_lib.pvs_build_ex(ptr, n, dim, on_dev, st, int(quantization), ctypes.byref(out)),
+               "pvs_build_ex")
     return out
+
+
+def pvs_build_ex(vecs, quantization: int, stream=None):
+    return pvs_build(vecs, stream=stream, quantization=quantization)
 
 
 def pvs_append(index, vecs) -> None:
@@ -334,6 +351,11 @@ def pvs_batch_bounds(index, queries, snap=None, rows=None):
 
 def pvs_cursor_sync(cursor) -> int:
     return _check(_lib.pvs_cursor_sync(cursor), "pvs_cursor_sync")
+
+
+def pvs_cursor_set_generator(cursor, generator: int) -> None:
+    """PVS_GEN_INTERVALS (default) or PVS_GEN_FULL_SCAN, before the first pull."""
+    _check(_lib.pvs_cursor_set_generator(cursor, int(generator)), "pvs_cursor_set_generator")
 
 
 def pvs_cursor_set_stream(cursor, stream) -> None:

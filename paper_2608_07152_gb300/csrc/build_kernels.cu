@@ -15,13 +15,15 @@ __global__ void __launch_bounds__(256) build_kernel(const float* __restrict__ ve
                                                     float* __restrict__ scale,
                                                     float* __restrict__ vnorm,
                                                     float* __restrict__ enorm,
-                                                    float* __restrict__ raw, int* status) {
+                                                    float* __restrict__ raw, int* status,
+                                                    const float* fixed_scale) {
     const int lane = threadIdx.x & 31;
     const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    const float fs = fixed_scale ? *fixed_scale : 0.0f;
     for (int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < n;
          row += warps) {
         const float* v = vecs + row * (int64_t)m;
-        RowQuant r = quantize_row_warp(v, m, m_pad, codes + row * (int64_t)m_pad);
+        RowQuant r = quantize_row_warp(v, m, m_pad, codes + row * (int64_t)m_pad, fs);
         float* dst = raw + row * (int64_t)m_raw;
         for (int j = lane; j < m_raw; j += kWarp) dst[j] = j < m ? v[j] : 0.0f;
         if (lane == 0) {
@@ -35,13 +37,52 @@ __global__ void __launch_bounds__(256) build_kernel(const float* __restrict__ ve
 
 cudaError_t launch_build(const float* vecs, int64_t n, int m, int m_pad, int m_raw,
                          int8_t* codes, float* scale, float* vnorm, float* enorm, float* raw,
-                         int* status, cudaStream_t st) {
+                         int* status, cudaStream_t st, const float* fixed_scale) {
     if (n <= 0) return cudaSuccess;
     int64_t blocks = (n + 7) / 8;
     if (blocks > 152 * 64) blocks = 152 * 64;
     count_launches(1);
     build_kernel<<<(unsigned)blocks, 256, 0, st>>>(vecs, n, m, m_pad, m_raw, codes, scale, vnorm,
-                                                   enorm, raw, status);
+                                                   enorm, raw, status, fixed_scale);
+    return cudaGetLastError();
+}
+
+// Largest |v_j| over count floats, as float bits (nonnegative floats order
+// like their bits; a NaN entry wins and makes the scale NaN, and the build
+// then reports the non-finite row).
+__global__ void maxabs_kernel(const float* __restrict__ v, int64_t count, unsigned int* out) {
+    unsigned int m = 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += stride)
+        m = max(m, __float_as_uint(fabsf(v[i])));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((threadIdx.x & 31) == 0 && m) atomicMax(out, m);
+}
+
+// s = RN(maxabs / 127), 1 for an all-zero corpus, 2^-149 if the quotient underflows.
+__global__ void scale_from_maxabs_kernel(const unsigned int* maxabs_bits, float* s) {
+    const float mx = __uint_as_float(*maxabs_bits);
+    float v = 1.0f;
+    if (mx != 0.0f) {
+        v = __fdiv_rn(mx, 127.0f);
+        if (v == 0.0f) v = __uint_as_float(1u);
+    }
+    *s = v;
+}
+
+cudaError_t launch_maxabs(const float* v, int64_t count, unsigned int* out, cudaStream_t st) {
+    if (count <= 0) return cudaSuccess;
+    int64_t blocks = (count + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    count_launches(1);
+    maxabs_kernel<<<(unsigned)blocks, 256, 0, st>>>(v, count, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scale_from_maxabs(const unsigned int* maxabs_bits, float* s, cudaStream_t st) {
+    count_launches(1);
+    scale_from_maxabs_kernel<<<1, 1, 0, st>>>(maxabs_bits, s);
     return cudaGetLastError();
 }
 

@@ -122,9 +122,25 @@ cudaError_t launch_scatter_ws(const int32_t* w_id, const float* w_lo, const floa
 // ---- build / encode (build_kernels.cu) -------------------------------------
 // Quantize rows [0, n) of `vecs` (row stride m floats) into codes (stride
 // m_pad), params, and a raw copy (stride m_raw, zero padded).
+// fixed_scale (device, may be null): one scale for every row (scalar-
+// quantization intervals) instead of each row's own.
 cudaError_t launch_build(const float* vecs, int64_t n, int m, int m_pad, int m_raw,
                          int8_t* codes, float* scale, float* vnorm, float* enorm, float* raw,
-                         int* status, cudaStream_t st);
+                         int* status, cudaStream_t st, const float* fixed_scale = nullptr);
+// *out = max(*out, bits of max |v_i|) over count floats (*out zeroed by the caller).
+cudaError_t launch_maxabs(const float* v, int64_t count, unsigned int* out, cudaStream_t st);
+// *s = RN(maxabs / 127) (1 for 0; 2^-149 if the quotient underflows).
+cudaError_t launch_scale_from_maxabs(const unsigned int* maxabs_bits, float* s, cudaStream_t st);
+
+// ---- exhaustive float32 scanning (scan_kernels.cu) ---------------------------
+// keys[row] = rank_key(authoritative score, row) for every visible row < rows
+// (0 for a deleted row); ctr->refined counts the scored rows.
+cudaError_t launch_scan_scores(const float* qraw, const float* raw, int m_raw, int64_t rows,
+                               const uint32_t* tomb, uint64_t* keys, int* status,
+                               DevCounters* ctr, cudaStream_t st);
+// ids / scores of keys[0 .. n); *mirror = *status afterwards when mirror is set.
+cudaError_t launch_scan_emit(const uint64_t* keys, int64_t n, int64_t* ids, float* scores,
+                             const int* status, int* mirror, cudaStream_t st);
 // Encode one query: codes zq[m_pad], raw copy qraw[m_raw], scalars.
 cudaError_t launch_encode_query(const float* q, int m, int m_pad, int m_raw, int8_t* zq,
                                 float* qraw, QueryScalars* qs, cudaStream_t st);

@@ -14,6 +14,7 @@
 //   4. emit them in order and mark them emitted (lo = hi = -inf).
 //   W is rebuilt with a doubled horizon when a pull would go past it.
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <cstdio>
 #include <cstring>
@@ -139,7 +140,7 @@ pvs_status index_fill(pvs_index* x, const float* vecs, int64_t n, bool on_device
     if (on_device) {
         PVS_CUDA(launch_build(vecs, n, x->m, x->m_pad, x->m_raw, x->codes + row0 * x->m_pad,
                               x->scale + row0, x->vnorm + row0, x->enorm + row0,
-                              x->raw + row0 * x->m_raw, x->d_status, x->stream));
+                              x->raw + row0 * x->m_raw, x->d_status, x->stream, x->gscale));
     } else {
         const int64_t rows_per_chunk =
             std::max<int64_t>(1, (int64_t)(kStageBytes / sizeof(float)) / x->m);
@@ -156,7 +157,8 @@ pvs_status index_fill(pvs_index* x, const float* vecs, int64_t n, bool on_device
             const int64_t dr = row0 + r;
             PVS_CUDA(launch_build(x->d_stage, c, x->m, x->m_pad, x->m_raw,
                                   x->codes + dr * x->m_pad, x->scale + dr, x->vnorm + dr,
-                                  x->enorm + dr, x->raw + dr * x->m_raw, x->d_status, x->stream));
+                                  x->enorm + dr, x->raw + dr * x->m_raw, x->d_status, x->stream,
+                                  x->gscale));
         }
     }
     int st = 0;
@@ -208,6 +210,10 @@ void cursor_free_device(pvs_cursor* c) {
     if (c->ev_begin) cudaEventDestroy(c->ev_begin);
     if (c->ev_end) cudaEventDestroy(c->ev_end);
     c->ev_begin = c->ev_end = nullptr;
+    dev_free(c->scan_keys), dev_free(c->scan_tmp);
+    if (c->scan_scratch) cudaFree(c->scan_scratch);
+    c->scan_scratch = nullptr;
+    c->scan_cap = 0;
 }
 
 // Host-side state of a fresh cursor; device buffers are kept for reuse.
@@ -225,6 +231,8 @@ void cursor_reset(pvs_cursor* c) {
     c->batch_ms = 0.0;
     c->ev_pending = false;
     c->interval_ms = 0.0;
+    c->generator = PVS_GEN_INTERVALS;
+    c->scan_ready = false;
 }
 
 // Closed cursors kept per index for reuse: at most kCursorPool of them and
@@ -234,7 +242,8 @@ constexpr size_t kCursorPool = 1024;
 constexpr size_t kCursorPoolBytes = size_t(4) << 30;
 
 size_t cursor_device_bytes(const pvs_cursor* c) {
-    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096 + kFrontCap * 4;
+    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096 + kFrontCap * 4 +
+           (size_t)c->scan_cap * 20;
 }
 
 // Allocate the per-row state of a cursor (first pull); a pooled cursor keeps
@@ -428,8 +437,44 @@ pvs_status prepare_pull(pvs_cursor* c, int64_t n_eff) {
 
 // status_mirror: a pinned host word the one-launch path sets to the status
 // after the pull (host-buffer pulls); null for device-buffer pulls.
+// Exhaustive float32 scanning (PVS_GEN_FULL_SCAN): the first pull scores
+// every visible row exactly and sorts all keys once; every pull emits the
+// next keys of that order.
+pvs_status scan_pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores,
+                     int* status_mirror) {
+    pvs_index* x = c->index;
+    cudaStream_t st = c->stream;
+    if (!c->scan_ready) {
+        const int64_t rows = std::max<int64_t>(c->rows, 1);
+        if (c->scan_cap < rows) {
+            dev_free(c->scan_keys), dev_free(c->scan_tmp);
+            if (c->scan_scratch) cudaFree(c->scan_scratch);
+            c->scan_scratch = nullptr;
+            c->scan_cap = 0;
+            if (dev_alloc(&c->scan_keys, (size_t)rows) != cudaSuccess ||
+                dev_alloc(&c->scan_tmp, (size_t)rows) != cudaSuccess ||
+                cudaMalloc(&c->scan_scratch, radix_sort_scratch_bytes(rows)) != cudaSuccess)
+                return fail(c, PVS_ERR_OOM);
+            c->scan_cap = rows;
+        }
+        cudaError_t e = launch_scan_scores(c->qraw, x->raw, x->m_raw, c->rows, c->snap->d_tomb,
+                                           c->scan_keys, c->d_status, c->ctr, st);
+        if (e == cudaSuccess && c->rows > 1)
+            e = launch_radix_sort_desc(c->scan_keys, c->scan_tmp, c->rows, c->scan_scratch, st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        c->scan_ready = true;
+    }
+    cudaError_t e = launch_scan_emit(c->scan_keys + c->emitted, n_eff, d_ids, d_scores,
+                                     c->d_status, status_mirror, st);
+    if (e != cudaSuccess) return fail(c, cuda_status(e));
+    c->emitted += n_eff;
+    c->pulls++;
+    return PVS_OK;
+}
+
 pvs_status pull(pvs_cursor* c, int64_t n_eff, int64_t* d_ids, float* d_scores,
                 int* status_mirror = nullptr) {
+    if (c->generator == PVS_GEN_FULL_SCAN) return scan_pull(c, n_eff, d_ids, d_scores, status_mirror);
     pvs_index* x = c->index;
     cudaStream_t st = c->stream;
     pvs_status s = prepare_pull(c, n_eff);
@@ -886,6 +931,14 @@ extern "C" {
 
 int64_t pvs_launch_count(void) { return (int64_t)g_launches.load(); }
 
+pvs_status pvs_cursor_set_generator(pvs_cursor* c, int32_t generator) {
+    if (!c || !c->index) return PVS_ERR_INVALID;
+    if (generator != PVS_GEN_INTERVALS && generator != PVS_GEN_FULL_SCAN) return PVS_ERR_INVALID;
+    if (c->pulls != 0 || c->emitted != 0 || c->batch_ws) return PVS_ERR_INVALID;
+    c->generator = generator;
+    return PVS_OK;
+}
+
 pvs_status pvs_cursor_set_stream(pvs_cursor* c, void* cuda_stream) {
     DeviceGuard device_guard(cursor_device(c));
     if (!c || !c->index) return PVS_ERR_INVALID;
@@ -912,9 +965,15 @@ const char* pvs_status_string(int32_t s) {
 
 pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
                      void* cuda_stream, pvs_index** out) {
+    return pvs_build_ex(vecs, n, dim, vecs_on_device, cuda_stream, PVS_QUANT_PER_VECTOR, out);
+}
+
+pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
+                        void* cuda_stream, int32_t quantization, pvs_index** out) {
     if (!out) return PVS_ERR_INVALID;
     *out = nullptr;
-    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) || (n > 0 && !vecs))
+    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) || (n > 0 && !vecs) ||
+        (quantization != PVS_QUANT_PER_VECTOR && quantization != PVS_QUANT_GLOBAL))
         return PVS_ERR_INVALID;
     pvs_index* x = new (std::nothrow) pvs_index();
     if (!x) return PVS_ERR_OOM;
@@ -950,6 +1009,29 @@ pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_
         cudaMemPoolSetAttribute(x->scratch_pool, cudaMemPoolAttrReleaseThreshold, &keep);
     }
     if (vecs_on_device && n > 0 && !is_device_ptr(vecs)) return bail(PVS_ERR_INVALID);
+    if (quantization == PVS_QUANT_GLOBAL) {
+        // one scale for the corpus: RN(max |v_j| / 127), from the largest entry
+        x->quant = PVS_QUANT_GLOBAL;
+        unsigned int* mx = nullptr;
+        if (dev_alloc(&x->gscale, 1) != cudaSuccess || dev_alloc(&mx, 1) != cudaSuccess) {
+            dev_free(mx);
+            return bail(PVS_ERR_OOM);
+        }
+        cudaError_t e = cudaMemsetAsync(mx, 0, sizeof(unsigned int), x->stream);
+        if (e == cudaSuccess && vecs_on_device) {
+            e = launch_maxabs(vecs, n * (int64_t)dim, mx, x->stream);
+        } else if (e == cudaSuccess) {
+            float m = 0.0f;
+            for (int64_t i = 0; i < n * (int64_t)dim; ++i) m = std::max(m, std::fabs(vecs[i]));
+            unsigned int bits;
+            std::memcpy(&bits, &m, sizeof bits);
+            e = cudaMemcpyAsync(mx, &bits, sizeof bits, cudaMemcpyHostToDevice, x->stream);
+        }
+        if (e == cudaSuccess) e = launch_scale_from_maxabs(mx, x->gscale, x->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(x->stream);
+        dev_free(mx);
+        if (e != cudaSuccess) return bail(cuda_status(e));
+    }
     pvs_status s = index_reserve(x, n);
     if (s != PVS_OK) return bail(s);
     s = index_fill(x, vecs, n, vecs_on_device != 0);
@@ -1032,6 +1114,7 @@ void pvs_index_free(pvs_index* x) {
     if (x->scratch_pool) cudaMemPoolDestroy(x->scratch_pool);
     if (x->bf16_ready) cudaEventDestroy(x->bf16_ready);
     dev_free(x->norm_maxes);
+    dev_free(x->gscale);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);
     delete x;
 }
@@ -1204,7 +1287,8 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
     cudaStream_t st = cursors[0]->stream;
     for (int32_t i = 0; i < nc; ++i) {
         n_out[i] = 0;
-        if (!cursors[i] || cursors[i]->index != x || cursors[i]->stream != st)
+        if (!cursors[i] || cursors[i]->index != x || cursors[i]->stream != st ||
+            cursors[i]->generator != PVS_GEN_INTERVALS)
             return PVS_ERR_INVALID;
     }
     for (int32_t i = 0; i < nc; ++i)
@@ -1446,7 +1530,8 @@ pvs_status pvs_cursor_stats_batch(pvs_cursor** cursors, int32_t nc, pvs_stats* o
 pvs_status pvs_cursor_bounds(pvs_cursor* c, int64_t first, int64_t count, float* lo,
                              float* hi) {
     DeviceGuard device_guard(cursor_device(c));
-    if (!c || first < 0 || count < 0 || first + count > c->rows || (count > 0 && (!lo || !hi)))
+    if (!c || first < 0 || count < 0 || first + count > c->rows || (count > 0 && (!lo || !hi)) ||
+        c->generator != PVS_GEN_INTERVALS)
         return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
     pvs_status s = PVS_OK;

@@ -126,8 +126,11 @@ struct RowQuant {
     int status;
 };
 
+// fixed_s > 0: one scale for the whole corpus (scalar-quantization
+// intervals) in place of the row's own; a code that would leave [-127, 127]
+// sets PVS_ERR_INVALID (the row is outside the scale's range).
 __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m, int m_pad,
-                                             int8_t* __restrict__ z) {
+                                             int8_t* __restrict__ z, float fixed_s = 0.0f) {
     const int lane = threadIdx.x & 31;
     float maxabs = 0.0f;
     bool finite = true;
@@ -146,7 +149,9 @@ __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m,
         return r;
     }
     float s;
-    if (maxabs == 0.0f) {
+    if (fixed_s > 0.0f) {
+        s = fixed_s;
+    } else if (maxabs == 0.0f) {
         s = 1.0f;
     } else {
         s = __fdiv_rn(maxabs, 127.0f);
@@ -154,11 +159,13 @@ __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m,
     }
     // codes and residual maximum
     double emax = 0.0;
+    bool out_of_range = false;
     for (int j = lane; j < m_pad; j += kWarp) {
         int c = 0;
         if (j < m && maxabs != 0.0f) {
             float t = __fdiv_rn(v[j], s);
             float rt = roundf(t);                      // half away from zero
+            out_of_range |= fabsf(rt) > 127.0f;
             rt = fminf(fmaxf(rt, -127.0f), 127.0f);
             c = (int)rt;
             double e = __dsub_rn((double)v[j], __dmul_rn((double)s, (double)c));  // exact
@@ -168,6 +175,7 @@ __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m,
     }
     __syncwarp();
     emax = warp_max(emax);
+    out_of_range = __any_sync(0xffffffffu, out_of_range) && fixed_s > 0.0f;
     // norm of v
     long long Tv = 0, Te = 0;
     int ev = maxabs > 0.0f ? norm_exponent((double)maxabs) : 0;
@@ -187,6 +195,7 @@ __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m,
     r.vnorm = norm_finish(Tv, ev);
     r.enorm = norm_finish(Te, ee);
     if (isinf(r.vnorm) || isinf(r.enorm)) r.status = PVS_ERR_OVERFLOW;
+    if (out_of_range) r.status = PVS_ERR_INVALID;
     return r;
 }
 

@@ -60,6 +60,9 @@ struct pvs_index {
     // stream-ordered scratch of batched calls; keeps its memory between calls
     // (the device's default pool hands memory back at every synchronisation)
     cudaMemPool_t scratch_pool = nullptr;
+    // scalar-quantization intervals: one scale for every row (else null)
+    int quant = PVS_QUANT_PER_VECTOR;
+    float* gscale = nullptr;                // device, one float
 };
 
 struct pvs_snapshot {
@@ -114,6 +117,13 @@ struct pvs_cursor {
     cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
     bool ev_pending = false;
     double interval_ms = 0.0;
+    // rank generator (PVS_GEN_*); exhaustive scanning keeps every row's key, sorted
+    int generator = PVS_GEN_INTERVALS;
+    bool scan_ready = false;
+    uint64_t* scan_keys = nullptr;
+    uint64_t* scan_tmp = nullptr;
+    void* scan_scratch = nullptr;
+    int64_t scan_cap = 0;
 };
 
 namespace pvs {
