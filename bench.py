@@ -57,18 +57,22 @@ def parse():
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="passage",
-                   choices=["passage", "batched", "eahr", "snapshots", "sparse", "hybrid"],
+                   choices=["passage", "batched", "eahr", "snapshots", "sparse", "hybrid",
+                            "ablation"],
                    help="passage: single-query ranking (default); batched: 256-query "
                         "tensor-core batches; eahr: EAHR Top-20 fusion over the passage "
                         "corpus and copula sparse rankings; snapshots: near-duplicate "
                         "corpus, five snapshots, EAHR Top-20; sparse: PBM sparse ranks "
                         "over a synthetic BM25 corpus; hybrid: EAHR Top-20 over PVS and PBM "
-                        "on the same items")
+                        "on the same items; ablation: PVS vs scalar-quantization intervals "
+                        "vs full scan")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
                    help="queries at tau = -0.5 (both lists are read to the end)")
     p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
+    p.add_argument("--ablation-queries", type=int, default=30,
+                   help="queries per generator in --workload ablation")
     p.add_argument("--pipeline", type=int, default=0,
                    help="queries (passage) or batches (batched) in flight; 0: the default")
     p.add_argument("--oracle-check", action="store_true",
@@ -763,6 +767,129 @@ def main_sparse(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+def main_ablation(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """Rank-generator ablation (the analogue of the paper's Table 1, dense
+    side) over the passage corpus: the same queries through PVS, scalar-
+    quantization intervals (an index with one scale for the corpus) and
+    exhaustive float32 scanning.  Per generator and query: (1) the first
+    1,000 ranks in chunks of 20 into host buffers; (2) EAHR Top-20 against a
+    tau = +0.5 copula sparse ranking (as --workload eahr).  Reported: paired
+    geometric-mean latency ratios to PVS and float32 evaluations per query."""
+    n = args.n
+    stream = torch.cuda.Stream(device=dev)
+    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=dev)
+    rows = torch.empty((n, DIM), dtype=torch.float32, device=dev)
+    chunk = 1 << 20
+    for r in range(0, n, chunk):
+        c = min(chunk, n - r)
+        rows[r:r + c] = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+    t0 = time.perf_counter()
+    idx_pvs = pvs.pvs_build(rows, stream=stream.cuda_stream)
+    torch.cuda.synchronize()
+    t1 = time.perf_counter()
+    idx_sq = pvs.pvs_build(rows, stream=stream.cuda_stream, quantization=pvs.PVS_QUANT_GLOBAL)
+    torch.cuda.synchronize()
+    t2 = time.perf_counter()
+    nq = 2 + args.ablation_queries
+    queries = synth.mixture_queries(nq, centres, QUERY_NOISE, seed=query_seed(14, rank))
+    gens = {"pvs": (idx_pvs, pvs.PVS_GEN_INTERVALS),
+            "scalar": (idx_sq, pvs.PVS_GEN_INTERVALS),
+            "scan": (idx_pvs, pvs.PVS_GEN_FULL_SCAN)}
+
+    def ranks(name, q):
+        index, gen = gens[name]
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        cur = pvs.pvs_cursor_open(index, q)
+        pvs.pvs_cursor_set_generator(cur, gen)
+        for _ in range(RANKS_PER_QUERY // CHUNK):
+            pvs.pvs_next(cur, CHUNK)
+        ev = pvs.pvs_cursor_stats(cur)["refined"]
+        pvs.pvs_cursor_close(cur)
+        return (time.perf_counter() - t) * 1e3, ev
+
+    def fused(name, q, sp):
+        index, gen = gens[name]
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        cur = pvs.pvs_cursor_open(index, q)
+        pvs.pvs_cursor_set_generator(cur, gen)
+        ids, F, st = pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR)
+        ev = pvs.pvs_cursor_stats(cur)["refined"]
+        pvs.pvs_cursor_close(cur)
+        return (time.perf_counter() - t) * 1e3, ev, ids
+
+    def sparse_for(q, seed):
+        return synth.copula_ranking(rows @ q, 0.5, seed).cpu().numpy()
+
+    for w in range(2):   # warm-up
+        sp = sparse_for(queries[w], 900 + w)
+        for name in gens:
+            ranks(name, queries[w])
+            fused(name, queries[w], sp)
+    launches0 = pvs.pvs_launch_count()
+    res = {name: {"ranks_ms": [], "ranks_evals": [], "eahr_ms": [], "eahr_evals": []}
+           for name in gens}
+    mismatch = 0
+    with ClockSampler(local) as clk:
+        for i in range(2, nq):
+            q = queries[i]
+            sp = sparse_for(q, 900 + i)
+            top = None
+            for name in gens:   # the same query through every generator
+                ms, ev = ranks(name, q)
+                res[name]["ranks_ms"].append(ms)
+                res[name]["ranks_evals"].append(ev)
+                ms, ev, ids = fused(name, q, sp)
+                res[name]["eahr_ms"].append(ms)
+                res[name]["eahr_evals"].append(ev)
+                if top is None:
+                    top = ids.tolist()
+                mismatch += int(ids.tolist() != top)
+    launches = pvs.pvs_launch_count() - launches0
+
+    def gmean_ratio(a, b):
+        return float(np.exp(np.mean(np.log(np.asarray(a) / np.asarray(b)))))
+
+    table = {}
+    for name, r in res.items():
+        table[name] = {
+            "first_1000_ms_p50": float(np.median(r["ranks_ms"])),
+            "first_1000_f32_evals_p50": float(np.median(r["ranks_evals"])),
+            "eahr_top20_ms_p50": float(np.median(r["eahr_ms"])),
+            "eahr_f32_evals_p50": float(np.median(r["eahr_evals"])),
+            "first_1000_ratio_to_pvs": gmean_ratio(r["ranks_ms"], res["pvs"]["ranks_ms"]),
+            "eahr_ratio_to_pvs": gmean_ratio(r["eahr_ms"], res["pvs"]["eahr_ms"]),
+        }
+    line = {
+        "metric": "rank-generator ablation: EAHR Top-20 latency ratio scalar/PVS, scan/PVS",
+        "value": table["scan"]["eahr_ratio_to_pvs"], "unit": "x (paired geometric mean)",
+        "n_gpus": world, "steps": nq - 2, "warmup": 2,
+        "ms_per_step": float(np.mean(res["pvs"]["eahr_ms"])), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": f"passage mixture N={n:,} x d={DIM}; generators: PVS (per-vector "
+                               "scales), scalar-quantization intervals (one scale for the "
+                               "corpus), exhaustive float32 scan; first 1,000 ranks in chunks "
+                               f"of {CHUNK}, and EAHR Top-{EAHR_K} against a tau=+0.5 copula "
+                               "sparse ranking",
+                   "N": n, "d": DIM, "parallelism": f"replicas x{world}"},
+        "e2e": {"value": table["scan"]["eahr_ratio_to_pvs"], "unit": "x",
+                "h2d_bytes_per_step": DIM * 4, "d2h_bytes_per_step": EAHR_K * 16},
+        "generators": table,
+        "eahr_results_differ": mismatch,
+        "gpu_launches": launches,
+        "build_s": {"pvs": t1 - t0, "scalar": t2 - t1},
+        "clocks": clk.summary(),
+    }
+    pvs.pvs_index_free(idx_sq)
+    pvs.pvs_index_free(idx_pvs)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 HYBRID_TOPIC_TERMS = 64     # topic block per mixture component
 HYBRID_TOPIC_SHARE = 0.3    # share of an item's tokens drawn from its topic block
 
@@ -1060,6 +1187,9 @@ def main():
         return
     if args.workload == "hybrid":
         main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
+    if args.workload == "ablation":
+        main_ablation(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
     stream = torch.cuda.Stream(device=dev)
