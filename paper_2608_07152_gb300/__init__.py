@@ -35,6 +35,10 @@ PVS_QUANT_GLOBAL = 1
 PVS_GEN_INTERVALS = 0
 PVS_GEN_FULL_SCAN = 1
 
+PVS_CHILD_DENSE = 0
+PVS_CHILD_SPARSE = 1
+PVS_CHILD_MERGE = 2
+
 EAHR_RANK_SCALED = 0
 EAHR_NUMERATOR = 1
 EAHR_POLICY_GEOMETRIC = 0
@@ -72,6 +76,17 @@ class pbm_stats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
         "items", "emitted", "ranges", "ranges_expanded", "postings_visited", "items_scored",
         "pulls", "rounds")] + [("state", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class pvs_merge_child(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("cursor", ctypes.c_void_p), ("id_offset", ctypes.c_int64)]
+
+
+class pvs_merge_stats_t(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "emitted", "read", "duplicates", "child_pulls", "id_space", "length")] + [
+        ("state", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 def _load() -> ctypes.CDLL:
@@ -129,6 +144,12 @@ def _load() -> ctypes.CDLL:
         "pbm_cursor_close": (None, [P]),
         "eahr_topk_pbm": (i32, [P, P, ctypes.POINTER(eahr_params), P, P, P,
                                 ctypes.POINTER(eahr_stats)]),
+        "pvs_merge_open": (i32, [P, i32, pp]),
+        "pvs_merge_next": (i32, [P, i32, P, P, P]),
+        "pvs_merge_stats_get": (i32, [P, ctypes.POINTER(pvs_merge_stats_t)]),
+        "pvs_merge_close": (None, [P]),
+        "eahr_topk_merge": (i32, [P, P, ctypes.POINTER(eahr_params), P, P, P,
+                                  ctypes.POINTER(eahr_stats)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -149,7 +170,8 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
             "pbm_index_free", "pbm_cursor_open", "pbm_next", "pbm_cursor_range_bounds",
-            "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm")
+            "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
+            "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge")
 
 
 def pvs_status_string(status: int) -> str:
@@ -582,4 +604,54 @@ def eahr_topk_pbm(cursor, sparse_cursor, K: int = 20, k: int = 60, form: int = E
     _check(_lib.eahr_topk_pbm(cursor, sparse_cursor, ctypes.byref(p), ids.ctypes.data,
                               F.ctypes.data, ctypes.byref(got), ctypes.byref(stats)),
            "eahr_topk_pbm")
+    return _eahr_result(0, ids, F, got, stats)
+
+
+# --------------------------------------------------------------------------
+# hierarchical Segment / Shard merging (Sec. 2.4; include/merge.h)
+# --------------------------------------------------------------------------
+
+def pvs_merge_open(children):
+    """children: a list of (kind, cursor, id_offset) with kind PVS_CHILD_DENSE
+    (pvs cursor), PVS_CHILD_SPARSE (pbm cursor) or PVS_CHILD_MERGE."""
+    arr = (pvs_merge_child * len(children))()
+    for i, (kind, cur, off) in enumerate(children):
+        arr[i].kind = int(kind)
+        arr[i].cursor = cur.value if isinstance(cur, ctypes.c_void_p) else cur
+        arr[i].id_offset = int(off)
+    out = ctypes.c_void_p()
+    _check(_lib.pvs_merge_open(arr, len(children), ctypes.byref(out)), "pvs_merge_open")
+    return out
+
+
+def pvs_merge_next(merge, n: int):
+    ids = np.empty(max(int(n), 1), np.int64)
+    sc = np.empty(max(int(n), 1), np.float32)
+    got = ctypes.c_int32(0)
+    s = _check(_lib.pvs_merge_next(merge, int(n), ids.ctypes.data, sc.ctypes.data,
+                                   ctypes.byref(got)), "pvs_merge_next")
+    return ids[:got.value], sc[:got.value], s
+
+
+def pvs_merge_stats(merge) -> dict:
+    st = pvs_merge_stats_t()
+    _check(_lib.pvs_merge_stats_get(merge, ctypes.byref(st)), "pvs_merge_stats_get")
+    return {n: getattr(st, n) for n, _ in pvs_merge_stats_t._fields_ if n != "reserved"}
+
+
+def pvs_merge_close(merge) -> None:
+    _lib.pvs_merge_close(merge)
+
+
+def eahr_topk_merge(dense_merge, sparse_merge, K: int = 20, k: int = 60,
+                    form: int = EAHR_NUMERATOR, policy: int = EAHR_POLICY_GEOMETRIC, step: int = 0,
+                    weights=(1, 1)):
+    p = _params(K, k, form, policy, step, weights)
+    ids = np.zeros(K, np.int64)
+    F = np.zeros(K, np.float64)
+    got = ctypes.c_int32(0)
+    stats = eahr_stats()
+    _check(_lib.eahr_topk_merge(dense_merge, sparse_merge, ctypes.byref(p), ids.ctypes.data,
+                                F.ctypes.data, ctypes.byref(got), ctypes.byref(stats)),
+           "eahr_topk_merge")
     return _eahr_result(0, ids, F, got, stats)

@@ -28,9 +28,17 @@
 #include <new>
 #include <vector>
 
+#include "../../include/merge.h"
 #include "../../include/pbm.h"
 #include "../../include/pvs.h"
 #include "runtime.h"
+
+// facts about merge cursors (merge.cu)
+namespace pvs {
+int64_t merge_id_space(const pvs_merge* m);
+int64_t merge_length(const pvs_merge* m);
+bool merge_fresh(const pvs_merge* m);
+}  // namespace pvs
 
 namespace {
 
@@ -122,9 +130,10 @@ inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
 }
 
 struct Source {
-    // dense cursor, sparse PBM cursor or host list
+    // dense cursor, sparse PBM cursor, merge cursor or host list
     pvs_cursor* cursor = nullptr;
     pbm_cursor* sparse = nullptr;
+    pvs_merge* merge = nullptr;
     const int64_t* list = nullptr;
     int64_t length = 0;
 };
@@ -188,7 +197,8 @@ class Driver {
     // snapshot (when there is one) and not repeated within the list.
     bool record(int i, const int64_t* ids, int64_t n) {
         const int j = 1 - i;
-        const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr;
+        const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
+                           src[i].merge == nullptr;
         for (int64_t t = 0; t < n; ++t) {
             const int64_t x64 = ids[t];
             if (check) {
@@ -281,7 +291,7 @@ class Driver {
     pvs_status pull(int i, int64_t n) {
         if (exhausted[i] || !active[i]) return PVS_OK;
         pulls[i]++;
-        if (src[i].cursor || src[i].sparse) {
+        if (src[i].cursor || src[i].sparse || src[i].merge) {
             if (n > (int64_t)std::numeric_limits<int32_t>::max()) n = std::numeric_limits<int32_t>::max();
             buf_ids.resize((size_t)n);
             buf_scores.resize((size_t)n);
@@ -289,7 +299,10 @@ class Driver {
             pvs_status s =
                 src[i].cursor
                     ? pvs_next(src[i].cursor, (int32_t)n, buf_ids.data(), buf_scores.data(), &got)
-                    : pbm_next(src[i].sparse, (int32_t)n, buf_ids.data(), buf_scores.data(), &got);
+                : src[i].sparse
+                    ? pbm_next(src[i].sparse, (int32_t)n, buf_ids.data(), buf_scores.data(), &got)
+                    : pvs_merge_next(src[i].merge, (int32_t)n, buf_ids.data(), buf_scores.data(),
+                                     &got);
             if (s < 0) return s;
             record(i, buf_ids.data(), got);
             if (s == PVS_EXHAUSTED) exhausted[i] = true;
@@ -476,6 +489,27 @@ pvs_status eahr_topk_pbm(pvs_cursor* dense, pbm_cursor* sparse, const eahr_param
         if (d.src[i].length == 0) d.exhausted[i] = true;
     }
     if (!d.init(snap->rows)) return PVS_ERR_OOM;
+    return run(d, p, out_ids, out_F, n_out, st);
+}
+
+pvs_status eahr_topk_merge(pvs_merge* dense, pvs_merge* sparse, const eahr_params* p,
+                           int64_t* out_ids, double* out_F, int32_t* n_out, eahr_stats* st) {
+    if (n_out) *n_out = 0;
+    if (!dense || !sparse || dense == sparse || !params_ok(p) || !out_ids || !n_out)
+        return PVS_ERR_INVALID;
+    if (!pvs::merge_fresh(dense) || !pvs::merge_fresh(sparse)) return PVS_ERR_INVALID;
+    const int64_t id_space = std::max(pvs::merge_id_space(dense), pvs::merge_id_space(sparse));
+    Driver d;
+    d.src[0].merge = dense;
+    d.src[0].length = pvs::merge_length(dense);
+    d.src[1].merge = sparse;
+    d.src[1].length = pvs::merge_length(sparse);
+    for (int i = 0; i < 2; ++i) {
+        if (!contrib_from(p, i, d.src[i].length, &d.g[i])) return PVS_ERR_INVALID;
+        d.active[i] = d.g[i].a != 0;
+        if (d.src[i].length == 0) d.exhausted[i] = true;
+    }
+    if (!d.init(id_space)) return PVS_ERR_OOM;
     return run(d, p, out_ids, out_F, n_out, st);
 }
 

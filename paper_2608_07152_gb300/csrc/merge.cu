@@ -1,0 +1,248 @@
+// Hierarchical Segment / Shard merging (include/merge.h): arXiv 2608.07152
+// Sec. 2.4, ranked-list contract of Sec. 2.1.
+//
+// Host code over device-backed children: a k-way merge of the children's
+// exact rankings under the rank key (score descending, id ascending).  Each
+// child keeps a buffer of ranks read but not yet delivered; before an item
+// is delivered, every child that is not exhausted has a non-empty buffer, so
+// the item precedes everything any child can still produce (each child's
+// later ranks have smaller keys than its buffered ones).  Refill sizes start
+// from the request size spread over the children and double per refill.
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <unordered_set>
+#include <vector>
+
+#include "../../include/merge.h"
+#include "pvs_common.cuh"
+#include "runtime.h"
+
+namespace {
+
+constexpr int32_t kMaxChildren = 1024;
+constexpr int64_t kMaxChunk = int64_t(1) << 20;
+
+struct Child {
+    int32_t kind = PVS_CHILD_DENSE;
+    void* cur = nullptr;
+    int64_t off = 0;
+    int64_t length = 0;      // list length (upper bound for merges)
+    int64_t id_space = 0;    // request ids of this child lie below this
+    std::vector<int64_t> ids;
+    std::vector<float> scores;
+    size_t head = 0;
+    bool exhausted = false;
+    int64_t chunk = 0;       // next refill size
+};
+
+}  // namespace
+
+struct pvs_merge {
+    std::vector<Child> ch;
+    int64_t id_space = 0, length = 0;
+    std::vector<uint64_t> seen;   // delivered request ids (bitmap)
+    uint64_t last_key = 0;
+    bool any = false;
+    int64_t emitted = 0, read = 0, dups = 0, child_pulls = 0;
+    int state = PVS_OK;
+};
+
+namespace {
+
+pvs_status fail(pvs_merge* m, pvs_status s) {
+    if (s < 0 && m->state >= 0) m->state = s;
+    return s;
+}
+
+// Facts about a fresh child: list length and id space (in its own ids).
+pvs_status describe(const pvs_merge_child& c, int64_t* length, int64_t* id_space) {
+    switch (c.kind) {
+        case PVS_CHILD_DENSE: {
+            pvs_cursor* p = static_cast<pvs_cursor*>(c.cursor);
+            pvs_stats st;
+            if (pvs_cursor_stats(p, &st) != PVS_OK || st.state < 0 || st.emitted != 0)
+                return PVS_ERR_INVALID;
+            *length = st.visible;
+            *id_space = pvs::cursor_snapshot(p)->rows;
+            return PVS_OK;
+        }
+        case PVS_CHILD_SPARSE: {
+            pbm_stats st;
+            if (pbm_cursor_stats(static_cast<pbm_cursor*>(c.cursor), &st) != PVS_OK ||
+                st.state < 0 || st.emitted != 0)
+                return PVS_ERR_INVALID;
+            *length = st.items;
+            *id_space = st.items;
+            return PVS_OK;
+        }
+        case PVS_CHILD_MERGE: {
+            pvs_merge* g = static_cast<pvs_merge*>(c.cursor);
+            if (g->state < 0 || g->emitted != 0 || g->read != 0) return PVS_ERR_INVALID;
+            *length = g->length;
+            *id_space = g->id_space;
+            return PVS_OK;
+        }
+        default:
+            return PVS_ERR_INVALID;
+    }
+}
+
+// Read up to n ranks of a child into its (empty) buffer.
+pvs_status refill(pvs_merge* m, Child& c, int64_t n) {
+    c.ids.resize((size_t)n);
+    c.scores.resize((size_t)n);
+    c.head = 0;
+    int32_t got = 0;
+    pvs_status s;
+    switch (c.kind) {
+        case PVS_CHILD_DENSE:
+            s = pvs_next(static_cast<pvs_cursor*>(c.cur), (int32_t)n, c.ids.data(), c.scores.data(),
+                         &got);
+            break;
+        case PVS_CHILD_SPARSE:
+            s = pbm_next(static_cast<pbm_cursor*>(c.cur), (int32_t)n, c.ids.data(), c.scores.data(),
+                         &got);
+            break;
+        default:
+            s = pvs_merge_next(static_cast<pvs_merge*>(c.cur), (int32_t)n, c.ids.data(),
+                               c.scores.data(), &got);
+            break;
+    }
+    ++m->child_pulls;
+    if (s < 0) {
+        c.ids.clear();
+        c.scores.clear();
+        return s;
+    }
+    c.ids.resize((size_t)got);
+    c.scores.resize((size_t)got);
+    for (auto& x : c.ids) x += c.off;
+    m->read += got;
+    if (s == PVS_EXHAUSTED) c.exhausted = true;
+    return PVS_OK;
+}
+
+bool seen(const pvs_merge* m, int64_t id) {
+    return (m->seen[(size_t)(id >> 6)] >> (id & 63)) & 1u;
+}
+
+}  // namespace
+
+extern "C" {
+
+pvs_status pvs_merge_open(const pvs_merge_child* children, int32_t count, pvs_merge** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (!children || count < 1 || count > kMaxChildren) return PVS_ERR_INVALID;
+    std::unordered_set<void*> distinct;
+    pvs_merge* m = new (std::nothrow) pvs_merge();
+    if (!m) return PVS_ERR_OOM;
+    m->ch.resize((size_t)count);
+    for (int32_t i = 0; i < count; ++i) {
+        const pvs_merge_child& c = children[i];
+        if (!c.cursor || c.id_offset < 0 || !distinct.insert(c.cursor).second) {
+            delete m;
+            return PVS_ERR_INVALID;
+        }
+        int64_t length = 0, space = 0;
+        if (describe(c, &length, &space) != PVS_OK) {
+            delete m;
+            return PVS_ERR_INVALID;
+        }
+        Child& d = m->ch[(size_t)i];
+        d.kind = c.kind;
+        d.cur = c.cursor;
+        d.off = c.id_offset;
+        d.length = length;
+        d.id_space = c.id_offset + space;
+        d.exhausted = length == 0;
+        m->id_space = std::max(m->id_space, d.id_space);
+        m->length += length;
+    }
+    if (m->id_space > ((int64_t)1 << 31)) {
+        delete m;
+        return PVS_ERR_INVALID;
+    }
+    m->seen.assign((size_t)((m->id_space + 63) / 64), 0ull);
+    *out = m;
+    return PVS_OK;
+}
+
+pvs_status pvs_merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    if (n_out) *n_out = 0;
+    if (!m) return PVS_ERR_INVALID;
+    if (m->state < 0) return PVS_ERR_FAILED;
+    if (n < 1 || !ids || !scores || !n_out) return PVS_ERR_INVALID;
+    const int64_t k = (int64_t)m->ch.size();
+    int32_t count = 0;
+    while (count < n) {
+        // every child that can still produce has a buffered head
+        for (Child& c : m->ch) {
+            if (c.head < c.ids.size() || c.exhausted) continue;
+            if (c.chunk == 0) c.chunk = std::max<int64_t>(16, 2 * ((n + k - 1) / k));
+            pvs_status s = refill(m, c, c.chunk);
+            if (s != PVS_OK) return fail(m, s);
+            c.chunk = std::min<int64_t>(c.chunk * 2, kMaxChunk);
+        }
+        Child* best = nullptr;
+        uint64_t best_key = 0;
+        for (Child& c : m->ch) {
+            if (c.head >= c.ids.size()) continue;
+            const uint64_t key = pvs::rank_key(c.scores[c.head], (uint32_t)c.ids[c.head]);
+            if (!best || key > best_key) {
+                best = &c;
+                best_key = key;
+            }
+        }
+        if (!best) break;   // every child exhausted and delivered
+        const int64_t id = best->ids[best->head];
+        const float sc = best->scores[best->head];
+        ++best->head;
+        if (m->any && best_key == m->last_key) {   // another copy with the same score
+            ++m->dups;
+            continue;
+        }
+        if (id < 0 || id >= m->id_space || seen(m, id))
+            return fail(m, PVS_ERR_INVALID);   // a copy with another score: conflict
+        m->seen[(size_t)(id >> 6)] |= 1ull << (id & 63);
+        ids[count] = id;
+        scores[count] = sc;
+        ++count;
+        m->last_key = best_key;
+        m->any = true;
+    }
+    m->emitted += count;
+    *n_out = count;
+    bool done = true;
+    for (const Child& c : m->ch) done = done && c.exhausted && c.head >= c.ids.size();
+    if (done) {
+        m->state = PVS_EXHAUSTED;
+        return PVS_EXHAUSTED;
+    }
+    return PVS_OK;
+}
+
+pvs_status pvs_merge_stats_get(pvs_merge* m, pvs_merge_stats* out) {
+    if (!m || !out) return PVS_ERR_INVALID;
+    out->emitted = m->emitted;
+    out->read = m->read;
+    out->duplicates = m->dups;
+    out->child_pulls = m->child_pulls;
+    out->id_space = m->id_space;
+    out->length = m->length;
+    out->state = m->state;
+    out->reserved = 0;
+    return PVS_OK;
+}
+
+void pvs_merge_close(pvs_merge* m) { delete m; }
+
+}  // extern "C"
+
+// Facts the EAHR driver needs about a merge cursor.
+namespace pvs {
+int64_t merge_id_space(const pvs_merge* m) { return m->id_space; }
+int64_t merge_length(const pvs_merge* m) { return m->length; }
+bool merge_fresh(const pvs_merge* m) { return m->state >= 0 && m->emitted == 0 && m->read == 0; }
+}  // namespace pvs

@@ -1,5 +1,5 @@
 """C ABI library: loads on a machine without a GPU, exports every symbol that
-include/*.h declares (pvs.h and pbm.h), and its host-only EAHR driver reproduces the oracle
+include/*.h declares (pvs.h, pbm.h and merge.h), and its host-only EAHR driver reproduces the oracle
 (arXiv 2608.07152, Sec. 2.1, 2.2; controlled streams of Sec. 3.4 / 4.2)."""
 import os
 import re
@@ -42,9 +42,10 @@ def test_struct_layouts_match_header(tmp_path):
     structures in include/pvs.h and include/pbm.h (size and every field offset)."""
     import subprocess
     structs = {"pvs_stats": pvs.pvs_stats, "eahr_params": pvs.eahr_params,
-               "eahr_stats": pvs.eahr_stats, "pbm_stats": pvs.pbm_stats}
+               "eahr_stats": pvs.eahr_stats, "pbm_stats": pvs.pbm_stats,
+               "pvs_merge_child": pvs.pvs_merge_child, "pvs_merge_stats": pvs.pvs_merge_stats_t}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "pvs.h"', '#include "pbm.h"',
-             "int main(void) {"]
+             '#include "merge.h"', "int main(void) {"]
     for name, cls in structs.items():
         lines.append(f'printf("{name} size %zu\\n", sizeof({name}));')
         for field, _ in cls._fields_:
