@@ -58,14 +58,14 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="passage",
                    choices=["passage", "batched", "eahr", "snapshots", "sparse", "hybrid",
-                            "ablation"],
+                            "ablation", "segments"],
                    help="passage: single-query ranking (default); batched: 256-query "
                         "tensor-core batches; eahr: EAHR Top-20 fusion over the passage "
                         "corpus and copula sparse rankings; snapshots: near-duplicate "
                         "corpus, five snapshots, EAHR Top-20; sparse: PBM sparse ranks "
                         "over a synthetic BM25 corpus; hybrid: EAHR Top-20 over PVS and PBM "
                         "on the same items; ablation: PVS vs scalar-quantization intervals "
-                        "vs full scan")
+                        "vs full scan; segments: EAHR over 8 merged Segments")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
@@ -890,6 +890,156 @@ def main_ablation(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+SEGMENTS = 8   # one Shard of eight immutable Segments, as the paper's TREC-DL setup
+
+
+def main_segments(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """Hierarchical merging at passage scale: the C2 corpus and the topical
+    BM25 corpus of --workload hybrid, each cut into 8 Segments of
+    consecutive ids (one Shard).  Per query, the same request twice:
+    unsegmented (one PVS index, one PBM index, eahr_topk_pbm) and segmented
+    (8 PVS and 8 PBM segment cursors under two merge cursors,
+    eahr_topk_merge); plus the first 1,000 dense ranks through one index and
+    through the merge.  The two Top-20 results must agree."""
+    n = args.n
+    stream = torch.cuda.Stream(device=dev)
+    centres = synth.mixture_centres(COMPONENTS, DIM, seed=2, device=dev)
+    rows = torch.empty((n, DIM), dtype=torch.float32, device=dev)
+    chunk = 1 << 20
+    for r in range(0, n, chunk):
+        c = min(chunk, n - r)
+        rows[r:r + c] = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+    bounds = [(n * i // SEGMENTS, n * (i + 1) // SEGMENTS) for i in range(SEGMENTS)]
+    t0 = time.perf_counter()
+    d_full = pvs.pvs_build(rows, stream=stream.cuda_stream)
+    d_seg = [pvs.pvs_build(rows[a:b], stream=stream.cuda_stream) for a, b in bounds]
+    del rows
+    torch.cuda.synchronize()
+    comps = synth.mixture_components(n, COMPONENTS, seed=2, device=dev)
+    off, docs, imps = synth.bm25_postings(n, SPARSE_TERMS, SPARSE_TOKENS, seed=10, device=dev,
+                                          topic_of=comps, topic_terms=HYBRID_TOPIC_TERMS,
+                                          topic_share=HYBRID_TOPIC_SHARE)
+    del comps
+    s_full = pvs.pbm_build(off, docs, imps, n)
+    term_of = torch.repeat_interleave(torch.arange(off.numel() - 1, device=dev),
+                                      off[1:] - off[:-1])
+    s_seg = []
+    for a, b in bounds:   # the postings of items a .. b-1, renumbered from 0
+        sel = torch.nonzero((docs >= a) & (docs < b)).squeeze(1)
+        cnt = torch.bincount(term_of[sel], minlength=off.numel() - 1)
+        o = torch.zeros(off.numel(), dtype=torch.int64, device=dev)
+        o[1:] = torch.cumsum(cnt, 0)
+        s_seg.append(pvs.pbm_build(o, (docs[sel] - a).to(torch.int32), imps[sel], b - a))
+    del term_of
+    torch.cuda.synchronize()
+    build_s = time.perf_counter() - t0
+    nq = 2 + args.eahr_queries
+    dq = synth.mixture_queries(nq, centres, QUERY_NOISE, seed=query_seed(15, rank))
+    qc = synth.mixture_query_components(nq, COMPONENTS, seed=query_seed(15, rank), device=dev)
+    sq = synth.topical_queries(qc, off, SPARSE_TERMS, HYBRID_TOPIC_TERMS,
+                               seed=query_seed(16, rank))
+
+    def unsegmented(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        dc = pvs.pvs_cursor_open(d_full, dq[i])
+        sc = pvs.pbm_cursor_open(s_full, *sq[i])
+        ids, _, _ = pvs.eahr_topk_pbm(dc, sc, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR)
+        pvs.pbm_cursor_close(sc)
+        pvs.pvs_cursor_close(dc)
+        return (time.perf_counter() - t) * 1e3, ids
+
+    def segmented(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        dcs = [pvs.pvs_cursor_open(x, dq[i]) for x in d_seg]
+        scs = [pvs.pbm_cursor_open(x, *sq[i]) for x in s_seg]
+        dm = pvs.pvs_merge_open([(pvs.PVS_CHILD_DENSE, c, a) for c, (a, _) in zip(dcs, bounds)])
+        sm = pvs.pvs_merge_open([(pvs.PVS_CHILD_SPARSE, c, a) for c, (a, _) in zip(scs, bounds)])
+        ids, _, _ = pvs.eahr_topk_merge(dm, sm, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR)
+        st = pvs.pvs_merge_stats(dm)
+        pvs.pvs_merge_close(dm)
+        pvs.pvs_merge_close(sm)
+        for c in dcs:
+            pvs.pvs_cursor_close(c)
+        for c in scs:
+            pvs.pbm_cursor_close(c)
+        return (time.perf_counter() - t) * 1e3, ids, st
+
+    def ranks_single(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        c = pvs.pvs_cursor_open(d_full, dq[i])
+        out = [pvs.pvs_next(c, CHUNK)[0] for _ in range(RANKS_PER_QUERY // CHUNK)]
+        pvs.pvs_cursor_close(c)
+        return (time.perf_counter() - t) * 1e3, np.concatenate(out)
+
+    def ranks_merged(i):
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        dcs = [pvs.pvs_cursor_open(x, dq[i]) for x in d_seg]
+        dm = pvs.pvs_merge_open([(pvs.PVS_CHILD_DENSE, c, a) for c, (a, _) in zip(dcs, bounds)])
+        out = [pvs.pvs_merge_next(dm, CHUNK)[0] for _ in range(RANKS_PER_QUERY // CHUNK)]
+        pvs.pvs_merge_close(dm)
+        for c in dcs:
+            pvs.pvs_cursor_close(c)
+        return (time.perf_counter() - t) * 1e3, np.concatenate(out)
+
+    for w in range(2):
+        unsegmented(w)
+        segmented(w)
+        ranks_single(w)
+        ranks_merged(w)
+    launches0 = pvs.pvs_launch_count()
+    lat_u, lat_s, lat_r1, lat_rm, differ, depth = [], [], [], [], 0, []
+    with ClockSampler(local) as clk:
+        for i in range(2, nq):
+            ms_u, ids_u = unsegmented(i)
+            ms_s, ids_s, st = segmented(i)
+            ms_1, r1 = ranks_single(i)
+            ms_m, rm = ranks_merged(i)
+            lat_u.append(ms_u)
+            lat_s.append(ms_s)
+            lat_r1.append(ms_1)
+            lat_rm.append(ms_m)
+            depth.append(st["emitted"])
+            differ += int(ids_u.tolist() != ids_s.tolist()) + int(not np.array_equal(r1, rm))
+    launches = pvs.pvs_launch_count() - launches0
+    line = {
+        "metric": "EAHR Top-20 latency over 8 Segments, PVS + PBM (p50)",
+        "value": float(np.median(lat_s)), "unit": "ms", "n_gpus": world, "steps": len(lat_s),
+        "warmup": 2, "ms_per_step": float(np.mean(lat_s)), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": f"one Shard of {SEGMENTS} Segments of consecutive ids over the "
+                               f"passage mixture (N={n:,} x d={DIM}) and the topical BM25 "
+                               "corpus of --workload hybrid; EAHR Top-20 over two merge "
+                               "cursors vs one index per channel",
+                   "N": n, "segments": SEGMENTS, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
+                   "parallelism": f"replicas x{world}"},
+        "e2e": {"value": float(np.median(lat_s)), "unit": "ms",
+                "h2d_bytes_per_step": SEGMENTS * DIM * 4, "d2h_bytes_per_step": EAHR_K * 16},
+        "eahr_ms": {"segmented_p50": float(np.median(lat_s)),
+                    "segmented_p95": float(np.percentile(lat_s, 95)),
+                    "unsegmented_p50": float(np.median(lat_u)),
+                    "unsegmented_p95": float(np.percentile(lat_u, 95))},
+        "first_1000_dense_ms": {"merged_8_p50": float(np.median(lat_rm)),
+                                "single_index_p50": float(np.median(lat_r1))},
+        "dense_merge_depth_p50": float(np.median(depth)),
+        "results_differ": differ,
+        "gpu_launches": launches, "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    for x in d_seg + [d_full]:
+        pvs.pvs_index_free(x)
+    for x in s_seg + [s_full]:
+        pvs.pbm_index_free(x)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 HYBRID_TOPIC_TERMS = 64     # topic block per mixture component
 HYBRID_TOPIC_SHARE = 0.3    # share of an item's tokens drawn from its topic block
 
@@ -1190,6 +1340,9 @@ def main():
         return
     if args.workload == "ablation":
         main_ablation(args, pvs, synth, torch, np, rank, world, local, dev, pg)
+        return
+    if args.workload == "segments":
+        main_segments(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
     stream = torch.cuda.Stream(device=dev)
