@@ -71,6 +71,8 @@ def parse():
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
                    help="queries at tau = -0.5 (both lists are read to the end)")
     p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
+    p.add_argument("--eahr-policy", default="geometric", choices=["geometric", "frozen", "equal"],
+                   help="EAHR scheduling policy of --workload eahr")
     p.add_argument("--ablation-queries", type=int, default=30,
                    help="queries per generator in --workload ablation")
     p.add_argument("--pipeline", type=int, default=0,
@@ -540,6 +542,8 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     build_s = time.perf_counter() - t0
     total_q = 2 * args.eahr_queries + args.eahr_exhaust_queries + 2
     queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
+    policy = {"geometric": pvs.EAHR_POLICY_GEOMETRIC, "frozen": pvs.EAHR_POLICY_FROZEN,
+              "equal": pvs.EAHR_POLICY_EQUAL_DEPTH}[args.eahr_policy]
 
     def sparse_for(q, tau, seed):
         proxy = rows @ q
@@ -564,7 +568,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     for w in range(2):
         sp, _ = sparse_for(queries[w], 0.5, 7 + w)
         cur = pvs.pvs_cursor_open(index, queries[w])
-        pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR)
+        pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR, policy=policy)
         pvs.pvs_cursor_close(cur)
         comparator(queries[w], torch.from_numpy(sp).to(dev))
     if pg:
@@ -589,7 +593,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                 t = time.perf_counter()
                 cur = pvs.pvs_cursor_open(index, q)
                 ids, F, st = pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K,
-                                           form=pvs.EAHR_NUMERATOR)
+                                           form=pvs.EAHR_NUMERATOR, policy=policy)
                 pvs.pvs_cursor_close(cur)
                 lat.append((time.perf_counter() - t) * 1e3)
                 if len(ids) != EAHR_K:
@@ -618,6 +622,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                                "(or --n), sparse channel a complete copula ranking of all N ids "
                                "(Kendall tau +0.5 / 0 / -0.5), weighted RRF 1/(60+rank), K=20",
                    "N": n, "d": DIM, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
+                   "policy": args.eahr_policy,
                    "l2": "no flush: every query's interval pass streams 6.9 GB of codes",
                    "parallelism": f"replicas x{world}"},
         "e2e": {"value": head["latency_ms_p50"], "unit": "ms",

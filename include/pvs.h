@@ -318,9 +318,18 @@ enum {
     EAHR_POLICY_GEOMETRIC = 0,   /* pull the channel with the larger next
                                     contribution; pull sizes grow x2 (result
                                     unchanged: Sec. 2.4)                        */
-    EAHR_POLICY_EQUAL_DEPTH = 1  /* both lists advance by `step` ranks, and
+    EAHR_POLICY_EQUAL_DEPTH = 1, /* both lists advance by `step` ranks, and
                                     certification runs after every step
                                     (the controlled-stream protocol, Sec. 3.4) */
+    EAHR_POLICY_FROZEN = 2       /* the paper's frozen scheduler (Sec. 3.5):
+                                    each step reads `step` ranks from the list
+                                    whose next unread rank contributes more; a
+                                    list skipped 16 steps in a row is advanced;
+                                    certification after every step through the
+                                    first 4K ranks read, then whenever access
+                                    has grown by clamp(access / 8, 64, 1024)
+                                    since the last check, and at once when a
+                                    list is exhausted                          */
 };
 
 typedef struct eahr_params {
@@ -328,8 +337,8 @@ typedef struct eahr_params {
     int32_t k;          /* RRF rank constant, >= 1                             */
     int32_t form;       /* EAHR_RANK_SCALED or EAHR_NUMERATOR                  */
     int32_t policy;     /* EAHR_POLICY_*                                       */
-    int32_t step;       /* first pull size (GEOMETRIC) or step (EQUAL_DEPTH);
-                           0 selects 16                                        */
+    int32_t step;       /* first pull size (GEOMETRIC) or step (EQUAL_DEPTH,
+                           FROZEN); 0 selects 16                               */
     int32_t w_num[2];   /* channel weights w_i = w_num[i] / w_den[i];          */
     int32_t w_den[2];   /* [0] dense, [1] sparse; 0 <= w_num < 2^16,
                            1 <= w_den < 2^16                                   */

@@ -43,6 +43,7 @@ EAHR_RANK_SCALED = 0
 EAHR_NUMERATOR = 1
 EAHR_POLICY_GEOMETRIC = 0
 EAHR_POLICY_EQUAL_DEPTH = 1
+EAHR_POLICY_FROZEN = 2
 
 
 class PvsError(RuntimeError):

@@ -345,8 +345,38 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
     // lists with zero weight contribute nothing and are never read
     bool done = false;
     if (!d.active[0] && !d.active[1]) done = true;
+    // frozen scheduler state (Sec. 3.5)
+    int skipped[2] = {0, 0};
+    int64_t next_check = 0;   // access at which the next sparse-cadence check falls due
+    const int64_t dense_checks = 4 * (int64_t)p->K;   // every step checked until 4K ranks are read
     while (!done) {
-        if (p->policy == EAHR_POLICY_EQUAL_DEPTH) {
+        if (p->policy == EAHR_POLICY_FROZEN) {
+            int pick = -1;
+            for (int i = 0; i < 2; ++i) {
+                if (!d.active[i] || d.exhausted[i]) continue;
+                if (pick < 0) {
+                    pick = i;
+                    continue;
+                }
+                const int c = cmp(d.u(i), d.u(pick));
+                if (c > 0 || (c == 0 && d.depth[i] < d.depth[pick])) pick = i;
+            }
+            if (pick >= 0) {
+                const int other = 1 - pick;
+                const bool other_open = d.active[other] && !d.exhausted[other];
+                if (other_open && skipped[other] >= 16) pick = other;   // fairness
+                const bool was[2] = {d.exhausted[0], d.exhausted[1]};
+                pvs_status s = d.pull(pick, step0);
+                if (s < 0) return s;
+                skipped[pick] = 0;
+                const int o = 1 - pick;
+                if (d.active[o] && !d.exhausted[o]) ++skipped[o];
+                const int64_t access = d.depth[0] + d.depth[1];
+                const bool newly = (d.exhausted[0] && !was[0]) || (d.exhausted[1] && !was[1]);
+                if (!(access <= dense_checks || newly || access >= next_check)) continue;
+                next_check = access + std::min<int64_t>(1024, std::max<int64_t>(64, access / 8));
+            }
+        } else if (p->policy == EAHR_POLICY_EQUAL_DEPTH) {
             for (int i = 0; i < 2; ++i) {
                 pvs_status s = d.pull(i, step0);
                 if (s < 0) return s;
@@ -403,7 +433,8 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
 
 bool params_ok(const eahr_params* p) {
     return p && p->K >= 1 && p->k >= 1 && (p->form == EAHR_RANK_SCALED || p->form == EAHR_NUMERATOR) &&
-           (p->policy == EAHR_POLICY_GEOMETRIC || p->policy == EAHR_POLICY_EQUAL_DEPTH) &&
+           (p->policy == EAHR_POLICY_GEOMETRIC || p->policy == EAHR_POLICY_EQUAL_DEPTH ||
+            p->policy == EAHR_POLICY_FROZEN) &&
            p->step >= 0;
 }
 

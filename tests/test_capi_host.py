@@ -72,7 +72,8 @@ def test_status_strings():
 FORMS = [(pvs.EAHR_RANK_SCALED, ro.RANK_SCALED), (pvs.EAHR_NUMERATOR, ro.NUMERATOR)]
 
 
-@pytest.mark.parametrize("policy", [pvs.EAHR_POLICY_GEOMETRIC, pvs.EAHR_POLICY_EQUAL_DEPTH])
+@pytest.mark.parametrize("policy", [pvs.EAHR_POLICY_GEOMETRIC, pvs.EAHR_POLICY_EQUAL_DEPTH,
+                                    pvs.EAHR_POLICY_FROZEN])
 def test_eahr_lists_match_complete_list_target(policy):
     rng = np.random.default_rng(0)
     for trial in range(60):
@@ -163,3 +164,73 @@ def test_controlled_streams_independent_and_partial_read_ratios():
         partial.append(st["depth"][0])
     assert all(0.3 < r < 0.95 for r in ratios), ratios
     assert 1000 <= float(np.median(partial)) <= 2000, partial
+
+
+def _frozen_schedule(a, b, K, step=16):
+    """The frozen scheduler's pull and check sequence (Sec. 3.5), replayed in
+    plain Python from the same rules on two complete lists of equal weight,
+    numerator RRF with k = 60, until the given number of checks is reached:
+    each step reads `step` ranks of the list whose next unread rank
+    contributes more (ties to the shallower list, then the dense one), a list
+    skipped 16 steps is read instead, and a check falls due after every step
+    until 4K ranks are read, when access reaches the last check's access plus
+    clamp(access / 8, 64, 1024), and when a list runs out."""
+    n = [len(a), len(b)]
+    depth = [0, 0]
+    skipped = [0, 0]
+    next_check = 0
+    checks = []
+    while depth[0] < n[0] or depth[1] < n[1]:
+        open_ = [depth[i] < n[i] for i in range(2)]
+        u = [Fraction(1, 60 + depth[i] + 1) if open_[i] else None for i in range(2)]
+        cand = [i for i in range(2) if open_[i]]
+        pick = cand[0]
+        for i in cand[1:]:
+            if u[i] > u[pick] or (u[i] == u[pick] and depth[i] < depth[pick]):
+                pick = i
+        other = 1 - pick
+        if open_[other] and skipped[other] >= 16:
+            pick = other
+        was = [not o for o in open_]
+        depth[pick] = min(n[pick], depth[pick] + step)
+        skipped[pick] = 0
+        if depth[1 - pick] < n[1 - pick]:
+            skipped[1 - pick] += 1
+        access = depth[0] + depth[1]
+        newly = any(depth[i] >= n[i] and not was[i] for i in range(2))
+        if access <= 4 * K or newly or access >= next_check:
+            next_check = access + min(1024, max(64, access // 8))
+            checks.append((depth[0], depth[1]))
+    return checks
+
+
+@pytest.mark.parametrize("relation", ["correlated", "independent", "reversed"])
+def test_frozen_scheduler_reads_and_checks_on_the_paper_cadence(relation):
+    a, b = synth.controlled_streams(3000, relation, 77)
+    ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                     policy=pvs.EAHR_POLICY_FROZEN)
+    # the result is the complete-list target (Sec. 2.4: the policy does not change it)
+    T = ro.target_topk([a, b], [1, 1], 60, 20, ro.NUMERATOR)
+    assert ids.tolist() == [x for x, _ in T]
+    # the driver stopped at one of the scheduled checks, after exactly as many
+    # checks as the replayed schedule has up to that depth
+    sched = _frozen_schedule(a, b, 20)
+    stop = (st["depth"][0], st["depth"][1])
+    assert stop in sched
+    assert st["checks"] == sched.index(stop) + 1
+    # every read was one step of at most 16 ranks
+    assert st["pulls"][0] * 16 >= st["depth"][0] and st["pulls"][1] * 16 >= st["depth"][1]
+
+
+def test_frozen_scheduler_fairness_advances_a_starved_list():
+    # dense weight 50: its next contribution stays larger for thousands of
+    # ranks, so only the fairness rule reads the sparse list
+    rng = np.random.default_rng(5)
+    a = rng.permutation(20_000)
+    b = rng.permutation(20_000)
+    ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                     policy=pvs.EAHR_POLICY_FROZEN, weights=(50, 1))
+    T = ro.target_topk([a, b], [50, 1], 60, 20, ro.NUMERATOR)
+    assert ids.tolist() == [x for x, _ in T]
+    steps = st["pulls"][0] + st["pulls"][1]
+    assert st["pulls"][1] >= steps // 17      # at least one sparse step in every 17
