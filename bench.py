@@ -71,6 +71,8 @@ def parse():
     p.add_argument("--eahr-exhaust-queries", type=int, default=10,
                    help="queries at tau = -0.5 (both lists are read to the end)")
     p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
+    p.add_argument("--eahr-levels", default="0.5,0,-0.5",
+                   help="Kendall tau levels of --workload eahr (comma-separated)")
     p.add_argument("--eahr-policy", default="geometric", choices=["geometric", "frozen", "equal"],
                    help="EAHR scheduling policy of --workload eahr")
     p.add_argument("--ablation-queries", type=int, default=30,
@@ -578,7 +580,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     qi = 2
     lat_all = []
     with ClockSampler(local) as clk:
-        for tau in EAHR_LEVELS:
+        for tau in [float(x) for x in args.eahr_levels.split(",")]:
             count = args.eahr_exhaust_queries if tau < 0 else args.eahr_queries
             lat, cmp_ms, dd, ds, ex, pulls = [], [], [], [], 0, []
             ktau = None
@@ -612,7 +614,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                 "sparse_depth_p50": float(np.median(ds)), "both_exhausted": ex,
                 "dense_pulls_p50": float(np.median(pulls))}
     launches = pvs.pvs_launch_count() - launches0
-    head = levels["+0.5"]
+    head = levels.get("+0.5", next(iter(levels.values())))
     line = {
         "metric": "EAHR Top-20 latency (p50, tau=+0.5)", "value": head["latency_ms_p50"],
         "unit": "ms", "n_gpus": world, "steps": sum(v["queries"] for v in levels.values()),
