@@ -317,10 +317,15 @@ __device__ inline void pull_emit_list(const PullArgs& a, PullShared& sh, const i
 
 // The status word as it stands after a pull, into the caller's pinned host
 // word (host-buffer pulls then need no separate copy).
+// Publishes the status word to pinned host memory last: the host may poll it
+// instead of synchronising, so the block's output writes are made visible to
+// the host first.
 __device__ inline void mirror_status(const PullArgs& a) {
     __syncthreads();
-    if (threadIdx.x == 0 && a.status_mirror)
+    if (threadIdx.x == 0 && a.status_mirror) {
+        __threadfence_system();
         *reinterpret_cast<volatile int*>(a.status_mirror) = *reinterpret_cast<volatile int*>(a.status);
+    }
 }
 
 __device__ inline void pull_emit_body(const PullArgs& a, PullShared& sh) {

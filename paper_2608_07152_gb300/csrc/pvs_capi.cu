@@ -16,10 +16,12 @@
 #include <algorithm>
 #include <cmath>
 #include <atomic>
+#include <chrono>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
 #include <new>
+#include <thread>
 
 #include "runtime.h"
 
@@ -325,6 +327,27 @@ void harvest_interval_time(pvs_cursor* c) {
     float ms = 0.0f;
     if (cudaEventElapsedTime(&ms, c->ev_begin, c->ev_end) == cudaSuccess) c->interval_ms += ms;
     c->ev_pending = false;
+}
+
+// A pinned status word that the last kernel of a pull writes after its
+// outputs (never a status value while pending).
+constexpr int kStatusPending = 0x7fffffff;
+
+// Wait for the status word to be published: spin, yielding every 256 reads,
+// for at most 2 s; false when it was not published in that time.
+bool wait_published(const int* word) {
+    const volatile int* w = word;
+    const auto t0 = std::chrono::steady_clock::now();
+    for (uint32_t i = 1;; ++i) {
+        if (*w != kStatusPending) {
+            std::atomic_thread_fence(std::memory_order_acquire);
+            return true;
+        }
+        if ((i & 255u) == 0) {
+            if (std::chrono::steady_clock::now() - t0 > std::chrono::seconds(2)) return false;
+            std::this_thread::yield();
+        }
+    }
 }
 
 // Read the device status word; a failure makes the cursor Failed.
@@ -1403,11 +1426,15 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         s = cursor_out_reserve(c, n_eff);
         if (s != PVS_OK) return fail(c, s);
         int* mirror = reinterpret_cast<int*>(c->h_small) + 2;
-        *mirror = 0;
+        *reinterpret_cast<volatile int*>(mirror) = kStatusPending;
         s = pull(c, n_eff, c->h_ids, c->h_scores, mirror);
         if (s != PVS_OK) return s;
-        cudaError_t e = cudaStreamSynchronize(c->stream);
-        if (e != cudaSuccess) return fail(c, cuda_status(e));
+        if (!wait_published(mirror)) {
+            // nothing published within the limit: an asynchronous error, or a
+            // very slow pull; the stream decides
+            cudaError_t e = cudaStreamSynchronize(c->stream);
+            if (e != cudaSuccess) return fail(c, cuda_status(e));
+        }
         harvest_interval_time(c);
         const int dev_status = *reinterpret_cast<volatile int*>(mirror);
         if (dev_status != 0) return fail(c, (pvs_status)dev_status);

@@ -58,7 +58,15 @@ __global__ void scan_emit_kernel(const uint64_t* __restrict__ keys, int64_t n, i
         ids[i] = (int64_t)rank_key_id(keys[i]);
         scores[i] = rank_key_score(keys[i]);
     }
-    if (mirror && blockIdx.x == 0 && threadIdx.x == 0) *mirror = *status;
+    // the status word is published last (the host may poll it): a launch that
+    // publishes is one block, and its writes are made visible to the host first
+    if (mirror) {
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            __threadfence_system();
+            *reinterpret_cast<volatile int*>(mirror) = *reinterpret_cast<const volatile int*>(status);
+        }
+    }
 }
 
 cudaError_t launch_scan_emit(const uint64_t* keys, int64_t n, int64_t* ids, float* scores,
@@ -66,6 +74,7 @@ cudaError_t launch_scan_emit(const uint64_t* keys, int64_t n, int64_t* ids, floa
     int64_t blocks = (n + 255) / 256;
     if (blocks < 1) blocks = 1;
     if (blocks > 152 * 4) blocks = 152 * 4;
+    if (mirror) blocks = 1;   // one block publishes after all of its writes
     count_launches(1);
     scan_emit_kernel<<<(unsigned)blocks, 256, 0, st>>>(keys, n, ids, scores, status, mirror);
     return cudaGetLastError();
