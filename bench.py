@@ -10,8 +10,11 @@ interval pass) are far larger than the 129 MB L2, so no L2 flush is needed.
 
 `value` (exact dense ranks/s) is timed with CUDA events on the library's
 stream with queries resident in HBM and ranks written to device buffers;
-`e2e` repeats the step through the same C ABI with host query buffers and
-host output buffers (pvs_next), the copies inside the timed region.
+`e2e` repeats the step through the library's native request executor
+(pvs_executor_run: host query buffers in pinned memory, host output buffers,
+every 20-rank page read through pvs_next onto the host before the next is
+requested, PIPELINE native worker threads), the copies inside the timed
+region.
 `roofline` reports the interval pass (the dominant kernel): algorithmic bytes
 N * (m_pad + 12) per pass over its CUDA-event duration, against the measured
 HBM copy bandwidth.
@@ -265,33 +268,6 @@ def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, cou
         lat20.append(t_open.elapsed_time(t_20))
         lat1000.append(t_open.elapsed_time(t_end))
     return lat20, lat1000
-
-
-def run_step_host(pvs, torch, index, queries_host, streams):
-    """The same step through host buffers (pvs_next); PIPELINE host threads
-    each drive their own cursors and stream."""
-    import threading
-
-    errors = []
-
-    def worker(k):
-        try:
-            for q in queries_host[k::PIPELINE]:
-                cur = pvs.pvs_cursor_open(index, q)
-                pvs.pvs_cursor_set_stream(cur, streams[k])
-                for p in range(RANKS_PER_QUERY // CHUNK):
-                    pvs.pvs_next(cur, CHUNK)
-                pvs.pvs_cursor_close(cur)
-        except Exception as e:  # surfaced below
-            errors.append(e)
-
-    threads = [threading.Thread(target=worker, args=(k,)) for k in range(PIPELINE)]
-    for t in threads:
-        t.start()
-    for t in threads:
-        t.join()
-    if errors:
-        raise errors[0]
 
 
 def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget=20.0):
@@ -1394,16 +1370,25 @@ def main():
     ranks_total = args.steps * args.queries * RANKS_PER_QUERY * world
     value = job_rate(args.steps * args.queries * RANKS_PER_QUERY, world, elapsed)
 
-    # ---- e2e: host query buffers, host outputs through pvs_next ----
-    qh = [np.ascontiguousarray(queries[args.warmup + s].cpu().numpy()) for s in range(args.steps)]
-    if pg:
-        pg.barrier()
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for s in range(args.steps):
-        run_step_host(pvs, torch, index, qh[s], streams)
-    torch.cuda.synchronize()
-    e2e_elapsed = time.perf_counter() - t0
+    # ---- e2e: pinned host queries, host outputs, through the native executor ----
+    qh = [queries[args.warmup + s].cpu().pin_memory() for s in range(args.steps)]
+    h_ids = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.int64).pin_memory()
+    h_sc = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.float32).pin_memory()
+    executor = pvs.pvs_executor_create(index, PIPELINE)
+    try:
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for s in range(args.steps):
+            _, _, n_got, _, rc = pvs.pvs_executor_run(executor, qh[s], RANKS_PER_QUERY, CHUNK,
+                                                      ids=h_ids, scores=h_sc)
+            if rc != pvs.PVS_OK or int(n_got.min()) != RANKS_PER_QUERY:
+                raise RuntimeError(f"executor run failed: {rc}")
+        torch.cuda.synchronize()
+        e2e_elapsed = time.perf_counter() - t0
+    finally:
+        pvs.pvs_executor_destroy(executor)
 
     # ---- latency, one query at a time ----
     lat20, lat1000 = measure_latency(pvs, torch, index, queries[args.warmup],
@@ -1432,7 +1417,9 @@ def main():
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},
         "e2e": {"value": e2e_value, "unit": UNIT,
                 "h2d_bytes_per_step": args.queries * DIM * 4,
-                "d2h_bytes_per_step": args.queries * RANKS_PER_QUERY * (8 + 4)},
+                "d2h_bytes_per_step": args.queries * RANKS_PER_QUERY * (8 + 4),
+                "path": f"pvs_executor_run: {PIPELINE} native workers, pages of {CHUNK} "
+                        "through pvs_next, pinned host queries and outputs"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_kind": peak_kind, "kernel": "interval_pass_kernel",

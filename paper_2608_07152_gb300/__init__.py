@@ -90,6 +90,11 @@ class pvs_merge_stats_t(ctypes.Structure):
         ("state", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class pvs_executor_stats_t(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in ("requests", "failed", "pages", "ranks")] + [
+        ("workers", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
 def _load() -> ctypes.CDLL:
     if not os.path.exists(_LIB_PATH):
         raise ImportError(
@@ -151,6 +156,10 @@ def _load() -> ctypes.CDLL:
         "pvs_merge_close": (None, [P]),
         "eahr_topk_merge": (i32, [P, P, ctypes.POINTER(eahr_params), P, P, P,
                                   ctypes.POINTER(eahr_stats)]),
+        "pvs_executor_create": (i32, [P, i32, pp]),
+        "pvs_executor_run": (i32, [P, P, P, i32, i32, i32, P, P, P, P]),
+        "pvs_executor_stats_get": (i32, [P, ctypes.POINTER(pvs_executor_stats_t)]),
+        "pvs_executor_destroy": (None, [P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -172,7 +181,9 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
             "pbm_index_free", "pbm_cursor_open", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
-            "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge")
+            "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge",
+            "pvs_executor_create", "pvs_executor_run", "pvs_executor_stats_get",
+            "pvs_executor_destroy")
 
 
 def pvs_status_string(status: int) -> str:
@@ -656,3 +667,70 @@ def eahr_topk_merge(dense_merge, sparse_merge, K: int = 20, k: int = 60,
                                 F.ctypes.data, ctypes.byref(got), ctypes.byref(stats)),
            "eahr_topk_merge")
     return _eahr_result(0, ids, F, got, stats)
+
+
+# --------------------------------------------------------------------------
+# native request executor (Sec. 2.1 paging over PVS cursors; include/executor.h)
+# --------------------------------------------------------------------------
+
+def pvs_executor_create(index, workers: int = 8):
+    """Start `workers` native worker threads (one CUDA stream each) for index."""
+    out = ctypes.c_void_p()
+    _check(_lib.pvs_executor_create(index, int(workers), ctypes.byref(out)), "pvs_executor_create")
+    return out
+
+
+def _host_buffer(x, dtype, shape, what):
+    """A host numpy array or CPU torch tensor of dtype and shape -> (pointer, array)."""
+    if x is None:
+        a = np.empty(shape, dtype)
+        return a.ctypes.data, a
+    if hasattr(x, "data_ptr"):
+        import torch
+        want = {np.int64: torch.int64, np.float32: torch.float32, np.int32: torch.int32}[dtype]
+        if x.is_cuda or x.dtype != want or tuple(x.shape) != tuple(shape) or not x.is_contiguous():
+            raise ValueError(f"{what}: want a contiguous CPU {want} tensor of shape {shape}")
+        return x.data_ptr(), x
+    if (not isinstance(x, np.ndarray) or x.dtype != dtype or x.shape != tuple(shape)
+            or not x.flags.c_contiguous):
+        raise ValueError(f"{what}: want a C-contiguous {np.dtype(dtype)} array of shape {shape}")
+    return x.ctypes.data, x
+
+
+def pvs_executor_run(ex, queries, ranks: int, page: int, snap=None, ids=None, scores=None,
+                     n_out=None, status=None):
+    """Serve one request per row of `queries` (host: numpy float32 or a CPU,
+    preferably pinned, torch float32 tensor): `ranks` ranks each, read in
+    pages of `page` through the host path.  Outputs may be given as host
+    buffers (numpy / CPU torch) to be filled in place.  Returns (ids [nq,
+    ranks], scores [nq, ranks], n_out [nq], status [nq], rc); raises
+    PvsError when the arguments are rejected (then nothing ran)."""
+    if hasattr(queries, "data_ptr"):
+        if queries.is_cuda or queries.dtype.itemsize != 4 or queries.dim() != 2:
+            raise ValueError("queries: want a 2-D CPU float32 tensor")
+        q = queries.contiguous()
+        qptr, nq = q.data_ptr(), q.shape[0]
+    else:
+        q = np.ascontiguousarray(queries, dtype=np.float32)
+        if q.ndim != 2:
+            raise ValueError("queries: want a 2-D array")
+        qptr, nq = q.ctypes.data, q.shape[0]
+    pi, ids = _host_buffer(ids, np.int64, (nq, ranks), "ids")
+    ps, scores = _host_buffer(scores, np.float32, (nq, ranks), "scores")
+    pn, n_out = _host_buffer(n_out, np.int32, (nq,), "n_out")
+    pst, status = _host_buffer(status, np.int32, (nq,), "status")
+    status[:] = 0
+    rc = _lib.pvs_executor_run(ex, snap, qptr, int(nq), int(ranks), int(page), pi, ps, pn, pst)
+    if rc < 0 and not any(int(v) == rc for v in status):
+        raise PvsError(rc, "pvs_executor_run")
+    return ids, scores, n_out, status, rc
+
+
+def pvs_executor_stats(ex) -> dict:
+    st = pvs_executor_stats_t()
+    _check(_lib.pvs_executor_stats_get(ex, ctypes.byref(st)), "pvs_executor_stats_get")
+    return {n: getattr(st, n) for n, _ in pvs_executor_stats_t._fields_ if n != "reserved"}
+
+
+def pvs_executor_destroy(ex) -> None:
+    _lib.pvs_executor_destroy(ex)

@@ -211,7 +211,8 @@ void cursor_free_device(pvs_cursor* c) {
     c->h_ids = nullptr, c->h_scores = nullptr, c->h_small = nullptr;
     if (c->ev_begin) cudaEventDestroy(c->ev_begin);
     if (c->ev_end) cudaEventDestroy(c->ev_end);
-    c->ev_begin = c->ev_end = nullptr;
+    if (c->ev_order) cudaEventDestroy(c->ev_order);
+    c->ev_begin = c->ev_end = c->ev_order = nullptr;
     dev_free(c->scan_keys), dev_free(c->scan_tmp);
     if (c->scan_scratch) cudaFree(c->scan_scratch);
     c->scan_scratch = nullptr;
@@ -1163,8 +1164,12 @@ void pvs_snapshot_free(pvs_snapshot* s) {
     delete s;
 }
 
-pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* query,
-                           int32_t query_on_device, pvs_cursor** out) {
+}  // extern "C"
+
+// Open a cursor whose device work runs on `stream` from the start (null: the
+// index's stream), ordered after the work queued so far on the index's stream.
+pvs_status pvs::cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const float* query,
+                               int32_t query_on_device, cudaStream_t stream, pvs_cursor** out) {
     DeviceGuard device_guard(index_device(x));
     if (!out) return PVS_ERR_INVALID;
     *out = nullptr;
@@ -1190,7 +1195,7 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
     };
     cursor_reset(c);
     c->index = x;
-    c->stream = x->stream;
+    c->stream = stream ? stream : x->stream;
     c->snap = snap ? snap->data : make_snapdata(x);
     if (!c->snap) return bail(PVS_ERR_OOM);
     c->rows = c->snap->rows;
@@ -1203,10 +1208,16 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
          dev_alloc(&c->ctr, 1) != cudaSuccess || dev_alloc(&c->d_status, 1) != cudaSuccess ||
          cudaMallocHost(&c->h_small, 16 * sizeof(unsigned int)) != cudaSuccess))
         return bail(PVS_ERR_OOM);
+    cudaError_t e = cudaSuccess;
+    if (st != x->stream) {   // after the index's queued builds and appends
+        if (!c->ev_order) e = cudaEventCreateWithFlags(&c->ev_order, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventRecord(c->ev_order, x->stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(st, c->ev_order, 0);
+        if (e != cudaSuccess) return bail(cuda_status(e));
+    }
     // a host query is staged in the cursor's raw query buffer, which the
     // encoder then rewrites in place with the same values (plus zero padding)
     const float* qd = query;
-    cudaError_t e = cudaSuccess;
     if (!query_on_device) {
         e = cudaMemcpyAsync(c->qraw, query, x->m * sizeof(float), cudaMemcpyHostToDevice, st);
         qd = c->qraw;
@@ -1214,14 +1225,22 @@ pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* 
     if (e == cudaSuccess) e = cudaMemsetAsync(c->ctr, 0, sizeof(DevCounters), st);
     if (e == cudaSuccess) e = cudaMemsetAsync(c->d_status, 0, sizeof(int), st);
     if (e == cudaSuccess) e = launch_encode_query(qd, x->m, x->m_pad, x->m_raw, c->zq, c->qraw, c->qs, st);
-    QueryScalars qs{};
-    if (e == cudaSuccess) e = cudaMemcpyAsync(&qs, c->qs, sizeof(qs), cudaMemcpyDeviceToHost, st);
+    int* enc_status = reinterpret_cast<int*>(c->h_small) + 3;   // pinned
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(enc_status, &c->qs->status, sizeof(int), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return bail(cuda_status(e));
-    if (qs.status != 0) return bail((pvs_status)qs.status);
+    if (*enc_status != 0) return bail((pvs_status)*enc_status);
     c->state = c->visible == 0 ? PVS_EXHAUSTED : PVS_OK;
     *out = c;
     return PVS_OK;
+}
+
+extern "C" {
+
+pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* query,
+                           int32_t query_on_device, pvs_cursor** out) {
+    return pvs::cursor_open_on(x, snap, query, query_on_device, nullptr, out);
 }
 
 pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const float* queries,

@@ -115,6 +115,7 @@ struct pvs_cursor {
     int64_t batch_passes = 0;         // batched (tensor-core) passes this cursor took part in
     double batch_ms = 0.0;            // device time of that pass (shared by its cursors)
     cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
+    cudaEvent_t ev_order = nullptr;   // orders a cursor's own stream after the index's
     bool ev_pending = false;
     double interval_ms = 0.0;
     // rank generator (PVS_GEN_*); exhaustive scanning keeps every row's key, sorted
@@ -131,4 +132,7 @@ namespace pvs {
 int64_t cursor_visible(const pvs_cursor* c);
 int64_t cursor_emitted(const pvs_cursor* c);
 const SnapData* cursor_snapshot(const pvs_cursor* c);
+// Open a cursor whose device work runs on `stream` (null: the index's stream).
+pvs_status cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const float* query,
+                          int32_t query_on_device, cudaStream_t stream, pvs_cursor** out);
 }  // namespace pvs

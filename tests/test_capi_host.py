@@ -1,5 +1,5 @@
 """C ABI library: loads on a machine without a GPU, exports every symbol that
-include/*.h declares (pvs.h, pbm.h and merge.h), and its host-only EAHR driver reproduces the oracle
+include/*.h declares (pvs.h, pbm.h, merge.h and executor.h), and its host-only EAHR driver reproduces the oracle
 (arXiv 2608.07152, Sec. 2.1, 2.2; controlled streams of Sec. 3.4 / 4.2)."""
 import os
 import re
@@ -32,6 +32,7 @@ def test_library_exports_every_declared_function():
     names = declared_functions()
     assert len(names) >= 30
     assert "pbm_next" in names and "eahr_topk_pbm" in names
+    assert "pvs_executor_run" in names
     for name in names:
         assert hasattr(pvs._lib, name), name
         assert name in pvs.EXPORTED, name
@@ -39,13 +40,14 @@ def test_library_exports_every_declared_function():
 
 def test_struct_layouts_match_header(tmp_path):
     """The binding's ctypes structures match the C compiler's layout of the
-    structures in include/pvs.h and include/pbm.h (size and every field offset)."""
+    structures in include/*.h (size and every field offset)."""
     import subprocess
     structs = {"pvs_stats": pvs.pvs_stats, "eahr_params": pvs.eahr_params,
                "eahr_stats": pvs.eahr_stats, "pbm_stats": pvs.pbm_stats,
-               "pvs_merge_child": pvs.pvs_merge_child, "pvs_merge_stats": pvs.pvs_merge_stats_t}
+               "pvs_merge_child": pvs.pvs_merge_child, "pvs_merge_stats": pvs.pvs_merge_stats_t,
+               "pvs_executor_stats": pvs.pvs_executor_stats_t}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "pvs.h"', '#include "pbm.h"',
-             '#include "merge.h"', "int main(void) {"]
+             '#include "merge.h"', '#include "executor.h"', "int main(void) {"]
     for name, cls in structs.items():
         lines.append(f'printf("{name} size %zu\\n", sizeof({name}));')
         for field, _ in cls._fields_:
@@ -234,3 +236,14 @@ def test_frozen_scheduler_fairness_advances_a_starved_list():
     assert ids.tolist() == [x for x, _ in T]
     steps = st["pulls"][0] + st["pulls"][1]
     assert st["pulls"][1] >= steps // 17      # at least one sparse step in every 17
+
+
+def test_executor_rejects_null_handles_without_a_gpu():
+    """Argument checks of include/executor.h that run before any device call."""
+    out = pvs.ctypes.c_void_p(123)
+    assert pvs._lib.pvs_executor_create(None, 4, pvs.ctypes.byref(out)) == pvs.PVS_ERR_INVALID
+    assert out.value is None
+    assert pvs._lib.pvs_executor_run(None, None, None, 1, 10, 5, None, None, None, None) == \
+        pvs.PVS_ERR_INVALID
+    assert pvs._lib.pvs_executor_stats_get(None, None) == pvs.PVS_ERR_INVALID
+    pvs._lib.pvs_executor_destroy(None)
