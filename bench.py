@@ -53,7 +53,7 @@ WORKLOAD = ("passage-scale single-query ranking: N=8,841,823 x d=768 Gaussian mi
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=3)
+    p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="pvs", choices=["pvs", "reference"])
     p.add_argument("--queries", type=int, default=50, help="queries per step")
@@ -144,38 +144,60 @@ def interval_traffic(n_rows: int, record="interval_pass_kernel_passage_8.8Mx768_
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    """nvidia-smi clocks and throttle reasons sampled during the timed region.
+
+    The sampler is started, and its first sample awaited, before the region
+    begins; a reader thread stamps every sample on arrival, and the summary
+    keeps the samples that arrived between the region's start and one
+    sampling period after its end."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    PERIOD_MS = 100
 
     def __init__(self, gpu: int):
         self.gpu = gpu
         self.proc = None
+        self.rows = []
+        self.t0 = self.t1 = 0.0
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.monotonic(), line))
 
     def __enter__(self):
+        import threading
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.PERIOD_MS)],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.reader = threading.Thread(target=self._read, daemon=True)
+            self.reader.start()
+            deadline = time.monotonic() + 5.0
+            while not self.rows and time.monotonic() < deadline and self.proc.poll() is None:
+                time.sleep(0.01)
         except Exception:
             self.proc = None
+        self.t0 = time.monotonic()
         return self
 
     def __exit__(self, *exc):
-        self.out = ""
+        self.t1 = time.monotonic()
         if self.proc is not None:
+            time.sleep(self.PERIOD_MS / 1e3)   # the sample taken at the end
             self.proc.terminate()
             try:
-                self.out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except Exception:
                 self.proc.kill()
+            self.reader.join(timeout=5)
         return False
 
     def summary(self):
-        rows = [r.split(",") for r in getattr(self, "out", "").strip().splitlines() if r.strip()]
+        late = self.t1 + self.PERIOD_MS / 1e3
+        rows = [r.split(",") for t, r in self.rows if self.t0 <= t <= late and r.strip()]
         sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for r in rows:
