@@ -1,6 +1,7 @@
 """C ABI library: loads on a machine without a GPU, exports every symbol that
 include/*.h declares (pvs.h, pbm.h, merge.h and executor.h), and its host-only EAHR driver reproduces the oracle
 (arXiv 2608.07152, Sec. 2.1, 2.2; controlled streams of Sec. 3.4 / 4.2)."""
+import json
 import os
 import re
 from fractions import Fraction
@@ -133,39 +134,48 @@ def test_eahr_lists_stop_where_the_oracle_rule_stops(relation):
         assert st["exhausted"] == [int(x) for x in exh]
 
 
-@pytest.mark.parametrize("n", [100_000, 1_000_000, 5_000_000])
+GOLDEN = json.load(open(os.path.join(ROOT, "tests", "golden", "controlled_streams.json")))
+PROTOCOL, OUTCOMES = GOLDEN["protocol"], GOLDEN["outcomes"]
+
+
+@pytest.mark.parametrize("n", PROTOCOL["collection_sizes"])
 def test_controlled_streams_paper_outcomes(n):
-    # Sec. 4.2: correlated rankings fix the Top-20 at depth 32 for all sizes;
-    # reversed (anti-correlated) rankings exhaust both lists.
-    for seed in (1729, 2027, 65537):
+    # the paper's printed outcomes (tests/golden/controlled_streams.json):
+    # correlated rankings fix the Top-20 at depth 32 for every size; reversed
+    # (anti-correlated) rankings exhaust both lists
+    K = PROTOCOL["K"]
+    for seed in PROTOCOL["seeds"]:
         a, b = synth.controlled_streams(n, "correlated", seed)
-        ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+        ids, F, st = pvs.eahr_topk_lists(a, b, K=K, k=60, form=pvs.EAHR_RANK_SCALED,
                                          policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
-        assert st["depth"] == [32, 32]
-        assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, 20)]
-    a, b = synth.controlled_streams(n, "reversed", 1729)
-    ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
+        assert st["depth"] == [OUTCOMES["correlated_depth"]] * 2
+        assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, K)]
+    a, b = synth.controlled_streams(n, "reversed", PROTOCOL["seeds"][0])
+    ids, F, st = pvs.eahr_topk_lists(a, b, K=K, k=60, form=pvs.EAHR_RANK_SCALED,
                                      policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
     assert st["exhausted"] == [1, 1] and st["depth"] == [n, n]
-    assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, 20)]
+    assert ids.tolist() == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, K)]
 
 
 def test_controlled_streams_independent_and_partial_read_ratios():
-    # Sec. 4.2 reports 64.5-77.9% of each list for independent rankings and a
-    # median depth of 1264 for partial overlap; the generators' random
-    # streams differ from the paper's, so these are loose checks.
+    # the paper prints 64.5-77.9% of each list for independent rankings and a
+    # median depth of 1264 for partial overlap; the generators' random streams
+    # differ from the paper's, so these are loose checks around those values
+    n = PROTOCOL["collection_sizes"][0]
+    lo, hi = OUTCOMES["independent_fraction_of_each_list"]
     ratios, partial = [], []
-    for seed in (1729, 2027, 65537):
-        a, b = synth.controlled_streams(100_000, "independent", seed)
+    for seed in PROTOCOL["seeds"]:
+        a, b = synth.controlled_streams(n, "independent", seed)
         _, _, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
                                        policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
-        ratios.append(st["depth"][0] / 100_000)
-        a, b = synth.controlled_streams(100_000, "partial", seed)
+        ratios.append(st["depth"][0] / n)
+        a, b = synth.controlled_streams(n, "partial", seed)
         _, _, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=pvs.EAHR_RANK_SCALED,
                                        policy=pvs.EAHR_POLICY_EQUAL_DEPTH, step=16)
         partial.append(st["depth"][0])
-    assert all(0.3 < r < 0.95 for r in ratios), ratios
-    assert 1000 <= float(np.median(partial)) <= 2000, partial
+    assert all(lo - 0.35 < r < hi + 0.17 for r in ratios), ratios
+    med = OUTCOMES["partial_overlap_median_depth"]
+    assert 0.8 * med <= float(np.median(partial)) <= 1.6 * med, partial
 
 
 def _frozen_schedule(a, b, K, step=16):

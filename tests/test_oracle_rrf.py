@@ -1,5 +1,7 @@
 """Pins of the RRF / EAHR oracle (arXiv 2608.07152, Sec. 2.1, 2.2, 3.4, 4.2)."""
 import itertools
+import json
+import os
 from fractions import Fraction
 
 import numpy as np
@@ -7,6 +9,7 @@ import pytest
 
 from oracle import eahr_oracle as eo
 from oracle import rrf_oracle as ro
+import synth
 
 F = Fraction
 
@@ -110,6 +113,39 @@ def test_correlated_block32_streams_fix_top20_at_depth_32(seed, n):
                                               [1, 1], 60, 20, step=16)
     assert depths == [32, 32] and not any(exhausted)
     assert A == [x for x, _ in ro.target_topk([first, second], [1, 1], 60, 20)]
+
+
+GOLDEN = json.load(open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden",
+                                   "controlled_streams.json")))
+
+
+@pytest.mark.parametrize("n", GOLDEN["protocol"]["collection_sizes"])
+def test_oracle_correlated_streams_at_the_printed_sizes(n):
+    """The paper's printed outcome (tests/golden/controlled_streams.json):
+    at every collection size and seed, correlated rankings fix the ordered
+    Top-20 at depth 32."""
+    K = GOLDEN["protocol"]["K"]
+    for seed in GOLDEN["protocol"]["seeds"]:
+        a, b = synth.controlled_streams(n, "correlated", seed)
+        A, depths, exhausted = eo.equal_depth_run([a.tolist(), b.tolist()], [1, 1], 60, K,
+                                                  step=16)
+        assert depths == [GOLDEN["outcomes"]["correlated_depth"]] * 2 and not any(exhausted)
+        assert A == [x for x, _ in ro.target_topk_large([a, b], [1, 1], 60, K)]
+
+
+def test_oracle_partial_overlap_depth_near_the_printed_median():
+    """The paper prints a median depth of 1264 for partial overlap (500 of
+    the first list's Top-1000 plus 500 outside items in the second list's
+    Top-1000); the random streams differ, so the check is loose."""
+    n = GOLDEN["protocol"]["collection_sizes"][0]
+    depths = []
+    for seed in GOLDEN["protocol"]["seeds"]:
+        a, b = synth.controlled_streams(n, "partial", seed)
+        _, d, exhausted = eo.equal_depth_run([a.tolist(), b.tolist()], [1, 1], 60, 20, step=16)
+        assert not any(exhausted)
+        depths.append(d[0])
+    med = GOLDEN["outcomes"]["partial_overlap_median_depth"]
+    assert 0.8 * med <= float(np.median(depths)) <= 1.6 * med, depths
 
 
 @pytest.mark.parametrize("seed", [1729, 2027, 65537])
