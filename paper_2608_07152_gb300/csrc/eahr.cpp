@@ -20,11 +20,17 @@
 // Items read from one list only are ordered by their rank in that list
 // (their L and U are monotone in it), so the best and second-best of each
 // group are found without scanning O.
+//
+// Per-request state indexed by id (two rank arrays and a flag array over the
+// id space: 80 MB at 8.8M ids) comes from a pool and goes back cleared: a
+// request clears only the entries it wrote, so its cost follows its depth,
+// not the id space (fresh zero pages cost a page fault per touched page).
 #include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
 #include <limits>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -129,6 +135,70 @@ inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
     return c > 0 || (c == 0 && x < y);
 }
 
+// Zeroed id-indexed arrays, kept for reuse (at most kPoolMax of them and
+// kPoolBytes in all; larger or surplus ones are freed).
+struct Workspace {
+    int32_t* rank[2] = {nullptr, nullptr};
+    uint8_t* flag = nullptr;
+    int64_t cap = 0;
+    size_t bytes() const { return (size_t)cap * (2 * sizeof(int32_t) + 1); }
+    void release() {
+        std::free(rank[0]);
+        std::free(rank[1]);
+        std::free(flag);
+        rank[0] = rank[1] = nullptr;
+        flag = nullptr;
+        cap = 0;
+    }
+};
+
+constexpr size_t kPoolMax = 16;
+constexpr size_t kPoolBytes = size_t(1) << 30;
+
+std::mutex g_pool_mutex;
+std::vector<Workspace> g_pool;
+size_t g_pool_bytes = 0;
+
+// A zeroed workspace of at least `ids` entries: the smallest pooled one that
+// fits, else a new one.
+bool acquire(int64_t ids, Workspace* out) {
+    {
+        std::lock_guard<std::mutex> lock(g_pool_mutex);
+        size_t best = g_pool.size();
+        for (size_t k = 0; k < g_pool.size(); ++k)
+            if (g_pool[k].cap >= ids && (best == g_pool.size() || g_pool[k].cap < g_pool[best].cap))
+                best = k;
+        if (best < g_pool.size()) {
+            *out = g_pool[best];
+            g_pool_bytes -= out->bytes();
+            g_pool.erase(g_pool.begin() + (std::ptrdiff_t)best);
+            return true;
+        }
+    }
+    Workspace w;
+    w.cap = ids;
+    w.rank[0] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
+    w.rank[1] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
+    w.flag = static_cast<uint8_t*>(std::calloc((size_t)ids, 1));
+    if (!w.rank[0] || !w.rank[1] || !w.flag) {
+        w.release();
+        return false;
+    }
+    *out = w;
+    return true;
+}
+
+// Return a workspace whose arrays are all zero again.
+void give_back(Workspace w) {
+    std::lock_guard<std::mutex> lock(g_pool_mutex);
+    if (g_pool.size() < kPoolMax && g_pool_bytes + w.bytes() <= kPoolBytes) {
+        g_pool_bytes += w.bytes();
+        g_pool.push_back(w);
+        return;
+    }
+    w.release();
+}
+
 struct Source {
     // dense cursor, sparse PBM cursor, merge cursor or host list
     pvs_cursor* cursor = nullptr;
@@ -159,18 +229,29 @@ class Driver {
     std::vector<float> buf_scores;
     const pvs::SnapData* snap = nullptr;
 
+    Workspace ws;
+
+    // Every entry written is an id of prefix[i] (rank[i]) or of A (inA):
+    // clear those, or whole arrays when that is cheaper, and pool them.
     ~Driver() {
-        std::free(rank[0]);
-        std::free(rank[1]);
-        std::free(inA);
+        if (!ws.flag) return;
+        for (int i = 0; i < 2; ++i) {
+            if ((int64_t)prefix[i].size() > ws.cap / 16)
+                std::memset(rank[i], 0, (size_t)ws.cap * sizeof(int32_t));
+            else
+                for (int32_t x : prefix[i]) rank[i][x] = 0;
+        }
+        for (int32_t x : A) inA[x] = 0;
+        give_back(ws);
     }
 
     bool init(int64_t ids) {
         id_space = std::max<int64_t>(ids, 1);
-        rank[0] = static_cast<int32_t*>(std::calloc((size_t)id_space, sizeof(int32_t)));
-        rank[1] = static_cast<int32_t*>(std::calloc((size_t)id_space, sizeof(int32_t)));
-        inA = static_cast<uint8_t*>(std::calloc((size_t)id_space, 1));
-        return rank[0] && rank[1] && inA;
+        if (!acquire(id_space, &ws)) return false;
+        rank[0] = ws.rank[0];
+        rank[1] = ws.rank[1];
+        inA = ws.flag;
+        return true;
     }
 
     Frac u(int i) const {
