@@ -136,18 +136,19 @@ inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
 }
 
 // Zeroed id-indexed arrays, kept for reuse (at most kPoolMax of them and
-// kPoolBytes in all; larger or surplus ones are freed).
+// kPoolBytes in all; larger or surplus ones are freed).  The two lists'
+// ranks of one id sit side by side (one cache line serves both lookups), and
+// the certified-set flags are a bitset (1.1 MB at 8.8M ids, cache-resident).
 struct Workspace {
-    int32_t* rank[2] = {nullptr, nullptr};
-    uint8_t* flag = nullptr;
+    int32_t* ranks = nullptr;    // [cap][2]
+    uint64_t* bits = nullptr;    // [(cap + 63) / 64]
     int64_t cap = 0;
-    size_t bytes() const { return (size_t)cap * (2 * sizeof(int32_t) + 1); }
+    size_t bytes() const { return (size_t)cap * 2 * sizeof(int32_t) + (size_t)(cap + 63) / 8; }
     void release() {
-        std::free(rank[0]);
-        std::free(rank[1]);
-        std::free(flag);
-        rank[0] = rank[1] = nullptr;
-        flag = nullptr;
+        std::free(ranks);
+        std::free(bits);
+        ranks = nullptr;
+        bits = nullptr;
         cap = 0;
     }
 };
@@ -177,10 +178,9 @@ bool acquire(int64_t ids, Workspace* out) {
     }
     Workspace w;
     w.cap = ids;
-    w.rank[0] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
-    w.rank[1] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
-    w.flag = static_cast<uint8_t*>(std::calloc((size_t)ids, 1));
-    if (!w.rank[0] || !w.rank[1] || !w.flag) {
+    w.ranks = static_cast<int32_t*>(std::calloc((size_t)ids * 2, sizeof(int32_t)));
+    w.bits = static_cast<uint64_t*>(std::calloc((size_t)(ids + 63) / 64, sizeof(uint64_t)));
+    if (!w.ranks || !w.bits) {
         w.release();
         return false;
     }
@@ -218,8 +218,8 @@ class Driver {
     int32_t pulls[2] = {0, 0};
     int32_t checks = 0;
     std::vector<int32_t> prefix[2];
-    int32_t* rank[2] = {nullptr, nullptr};   // rank of id in list i (0: unread)
-    uint8_t* inA = nullptr;
+    int32_t* ranks = nullptr;    // ranks[2 x + i]: rank of id x in list i (0: unread)
+    uint64_t* bits = nullptr;    // bit x: x is certified (in A)
     int64_t id_space = 0;
     TopBoth both;
     size_t ptr[2] = {0, 0};
@@ -231,26 +231,28 @@ class Driver {
 
     Workspace ws;
 
-    // Every entry written is an id of prefix[i] (rank[i]) or of A (inA):
+    int32_t rank(int i, int32_t x) const { return ranks[2 * (size_t)x + (size_t)i]; }
+    bool inA(int32_t x) const { return (bits[(uint32_t)x >> 6] >> (x & 63)) & 1u; }
+
+    // Every entry written is an id of prefix[i] (ranks) or of A (bits):
     // clear those, or whole arrays when that is cheaper, and pool them.
     ~Driver() {
-        if (!ws.flag) return;
-        for (int i = 0; i < 2; ++i) {
-            if ((int64_t)prefix[i].size() > ws.cap / 16)
-                std::memset(rank[i], 0, (size_t)ws.cap * sizeof(int32_t));
-            else
-                for (int32_t x : prefix[i]) rank[i][x] = 0;
+        if (!ws.ranks) return;
+        if ((int64_t)(prefix[0].size() + prefix[1].size()) > ws.cap / 8) {
+            std::memset(ranks, 0, (size_t)ws.cap * 2 * sizeof(int32_t));
+        } else {
+            for (int i = 0; i < 2; ++i)
+                for (int32_t x : prefix[i]) ranks[2 * (size_t)x + (size_t)i] = 0;
         }
-        for (int32_t x : A) inA[x] = 0;
+        for (int32_t x : A) bits[(uint32_t)x >> 6] = 0;
         give_back(ws);
     }
 
     bool init(int64_t ids) {
         id_space = std::max<int64_t>(ids, 1);
         if (!acquire(id_space, &ws)) return false;
-        rank[0] = ws.rank[0];
-        rank[1] = ws.rank[1];
-        inA = ws.flag;
+        ranks = ws.ranks;
+        bits = ws.bits;
         return true;
     }
 
@@ -261,15 +263,16 @@ class Driver {
 
     Frac L(int32_t x) const {
         Frac f;
-        if (active[0] && rank[0][x]) f = add(f, g[0].at(rank[0][x]));
-        if (active[1] && rank[1][x]) f = add(f, g[1].at(rank[1][x]));
+        const int32_t r0 = rank(0, x), r1 = rank(1, x);
+        if (active[0] && r0) f = add(f, g[0].at(r0));
+        if (active[1] && r1) f = add(f, g[1].at(r1));
         return f;
     }
 
     Frac U(int32_t x) const {
         Frac f = L(x);
         for (int i = 0; i < 2; ++i)
-            if (active[i] && !exhausted[i] && !rank[i][x]) f = add(f, u(i));
+            if (active[i] && !exhausted[i] && !rank(i, x)) f = add(f, u(i));
         return f;
     }
 
@@ -280,17 +283,26 @@ class Driver {
         const int j = 1 - i;
         const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
                            src[i].merge == nullptr;
+        // ids arrive in rank order, scattered over the id space: fetch the
+        // rank pair of the id kAhead positions on while this one is handled
+        constexpr int64_t kAhead = 16;
+        if (prefix[i].capacity() < prefix[i].size() + (size_t)n)
+            prefix[i].reserve(std::max(2 * prefix[i].capacity(), prefix[i].size() + (size_t)n));
         for (int64_t t = 0; t < n; ++t) {
+            if (t + kAhead < n) {
+                const int64_t y = ids[t + kAhead];
+                if (y >= 0 && y < id_space) __builtin_prefetch(ranks + 2 * y, 1, 0);
+            }
             const int64_t x64 = ids[t];
             if (check) {
                 if (x64 < 0 || x64 >= id_space) return false;
                 if (snap && !snap->is_visible(x64)) return false;
-                if (rank[i][x64]) return false;
+                if (rank(i, (int32_t)x64)) return false;
             }
             const int32_t x = (int32_t)x64;
             prefix[i].push_back(x);
-            rank[i][x] = (int32_t)(depth[i] + t + 1);
-            if (active[j] && rank[j][x] && !inA[x]) both.insert(Node{L(x), x});
+            ranks[2 * (size_t)x + (size_t)i] = (int32_t)(depth[i] + t + 1);
+            if (active[j] && rank(j, x) && !inA(x)) both.insert(Node{L(x), x});
         }
         depth[i] += n;
         return true;
@@ -302,8 +314,8 @@ class Driver {
         const int j = 1 - i;
         for (size_t p = from; p < prefix[i].size(); ++p) {
             const int32_t x = prefix[i][p];
-            if (inA[x] || x == skip) continue;
-            if (active[j] && rank[j][x]) continue;
+            if (inA(x) || x == skip) continue;
+            if (active[j] && rank(j, x)) continue;
             return x;
         }
         return -1;
@@ -313,7 +325,7 @@ class Driver {
         const int j = 1 - i;
         while (ptr[i] < prefix[i].size()) {
             const int32_t x = prefix[i][ptr[i]];
-            if (inA[x] || (active[j] && rank[j][x])) {
+            if (inA(x) || (active[j] && rank(j, x))) {
                 ++ptr[i];
                 continue;
             }
@@ -361,9 +373,9 @@ class Driver {
                 return Lx.num == 0;
             }
             A.push_back(xp);
-            inA[xp] = 1;
+            bits[(uint32_t)xp >> 6] |= 1ull << (xp & 63);
             // read from both lists: then it was the best of that group
-            if (active[0] && active[1] && rank[0][xp] && rank[1][xp]) both.pop_front();
+            if (active[0] && active[1] && rank(0, xp) && rank(1, xp)) both.pop_front();
         }
         return true;
     }
@@ -494,7 +506,7 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
         if (out_F) {
             bool determined = true;
             for (int i = 0; i < 2; ++i)
-                if (d.active[i] && !d.exhausted[i] && !d.rank[i][x]) determined = false;
+                if (d.active[i] && !d.exhausted[i] && !d.rank(i, x)) determined = false;
             out_F[t] = determined ? frac_to_double(d.L(x)) : std::nan("");
         }
     }
