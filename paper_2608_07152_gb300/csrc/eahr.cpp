@@ -32,6 +32,7 @@
 #include <limits>
 #include <mutex>
 #include <new>
+#include <thread>
 #include <vector>
 
 #include "../../include/merge.h"
@@ -129,6 +130,34 @@ struct TopBoth {
     void pop_front() { v.erase(v.begin()); }
 };
 
+// The best `cap` nodes of a stream, whatever the order of arrival:
+// candidates gather in a buffer that is cut back to the best `cap` whenever
+// it fills; once `cap` are kept, anything not above the worst kept is
+// dropped at once.
+struct TopStream {
+    static constexpr size_t kCut = 4096;
+    size_t cap = 2;
+    std::vector<Node> buf;
+    bool full = false;
+    Node worst;
+    void push(const Node& n) {
+        if (full && !NodeCmp()(n, worst)) return;
+        buf.push_back(n);
+        if (buf.size() >= kCut) cut();
+    }
+    void cut() {
+        if (buf.size() > cap) {
+            std::nth_element(buf.begin(), buf.begin() + (std::ptrdiff_t)(cap - 1), buf.end(),
+                             NodeCmp());
+            buf.resize(cap);
+        }
+        if (buf.size() == cap) {
+            full = true;
+            worst = *std::max_element(buf.begin(), buf.end(), NodeCmp());
+        }
+    }
+};
+
 // (a, x) beats (b, y): a > b, or a == b and x has the smaller id.
 inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
     const int c = cmp(a, b);
@@ -154,6 +183,8 @@ struct Workspace {
 };
 
 constexpr size_t kPoolMax = 16;
+constexpr int64_t kParallelMin = int64_t(1) << 17;   // ranks per pull worth threads
+constexpr unsigned kMaxThreads = 8;
 constexpr size_t kPoolBytes = size_t(1) << 30;
 
 std::mutex g_pool_mutex;
@@ -223,6 +254,7 @@ class Driver {
     int64_t id_space = 0;
     TopBoth both;
     size_t ptr[2] = {0, 0};
+    int64_t both_read = 0;   // items read from both lists
     std::vector<int32_t> A;
     int K = 0;
     std::vector<int64_t> buf_ids;
@@ -280,6 +312,10 @@ class Driver {
     // checked as they are read: inside the id space, visible in the
     // snapshot (when there is one) and not repeated within the list.
     bool record(int i, const int64_t* ids, int64_t n) {
+        if (n >= kParallelMin) {
+            const int T = (int)std::min<unsigned>(kMaxThreads, std::thread::hardware_concurrency());
+            if (T > 1) return record_parallel(i, ids, n, T);
+        }
         const int j = 1 - i;
         const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
                            src[i].merge == nullptr;
@@ -302,8 +338,102 @@ class Driver {
             const int32_t x = (int32_t)x64;
             prefix[i].push_back(x);
             ranks[2 * (size_t)x + (size_t)i] = (int32_t)(depth[i] + t + 1);
-            if (active[j] && rank(j, x) && !inA(x)) both.insert(Node{L(x), x});
+            if (rank(j, x)) {
+                ++both_read;
+                if (!inA(x)) both.insert(Node{L(x), x});
+            }
         }
+        depth[i] += n;
+        return true;
+    }
+
+    // record() over T threads, for long pulls.  Phase 1 writes the ranks
+    // (and the prefix), each thread a contiguous part; phase 2 reads every
+    // written rank back (a repeated id leaves a rank that is not its own)
+    // and collects each part's best items read from both lists.  Which items
+    // enter `both`, the K + 2 best, does not depend on the order of inserts.
+    bool record_parallel(int i, const int64_t* ids, int64_t n, int T) {
+        const int j = 1 - i;
+        const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
+                           src[i].merge == nullptr;
+        std::vector<int32_t>& pre = prefix[i];
+        const size_t base = pre.size();
+        if (pre.capacity() < base + (size_t)n)
+            pre.reserve(std::max(2 * pre.capacity(), base + (size_t)n));
+        pre.resize(base + (size_t)n, 0);
+        const int64_t d0 = depth[i];
+        std::vector<uint8_t> bad((size_t)T, 0);
+        std::vector<std::vector<Node>> tops((size_t)T);
+        std::vector<int64_t> doubly((size_t)T, 0);
+        auto part = [&](int t, int64_t* lo, int64_t* hi) {
+            *lo = n * t / T;
+            *hi = n * (t + 1) / T;
+        };
+        auto phase1 = [&](int t) {
+            int64_t lo, hi;
+            part(t, &lo, &hi);
+            for (int64_t k = lo; k < hi; ++k) {
+                if (k + 16 < hi) {
+                    const int64_t y = ids[k + 16];
+                    if (y >= 0 && y < id_space) __builtin_prefetch(ranks + 2 * y, 1, 0);
+                }
+                const int64_t x64 = ids[k];
+                if (check && (x64 < 0 || x64 >= id_space || (snap && !snap->is_visible(x64)))) {
+                    bad[(size_t)t] = 1;
+                    return;
+                }
+                // host lists may repeat an id across parts: relaxed atomics
+                // keep those accesses defined (plain loads and stores)
+                int32_t* slot = ranks + 2 * x64 + i;
+                if (check && __atomic_load_n(slot, __ATOMIC_RELAXED)) {
+                    bad[(size_t)t] = 1;
+                    return;
+                }
+                __atomic_store_n(slot, (int32_t)(d0 + k + 1), __ATOMIC_RELAXED);
+                pre[base + (size_t)k] = (int32_t)x64;
+            }
+        };
+        auto phase2 = [&](int t) {
+            int64_t lo, hi;
+            part(t, &lo, &hi);
+            // thread-local until the end: neighbouring threads' counters and
+            // vectors would share cache lines
+            TopStream top;
+            top.cap = both.cap;
+            top.buf.reserve(TopStream::kCut);
+            int64_t count = 0;
+            for (int64_t k = lo; k < hi; ++k) {
+                if (k + 16 < hi) __builtin_prefetch(ranks + 2 * (size_t)pre[base + (size_t)k + 16], 0, 0);
+                const int32_t x = pre[base + (size_t)k];
+                if (check && rank(i, x) != (int32_t)(d0 + k + 1)) {
+                    bad[(size_t)t] = 1;
+                    return;
+                }
+                if (rank(j, x)) {
+                    ++count;
+                    if (!inA(x)) top.push(Node{L(x), x});
+                }
+            }
+            top.cut();
+            doubly[(size_t)t] = count;
+            tops[(size_t)t] = std::move(top.buf);
+        };
+        for (auto phase : {0, 1}) {
+            std::vector<std::thread> th;
+            th.reserve((size_t)T - 1);
+            for (int t = 1; t < T; ++t) {
+                if (phase == 0) th.emplace_back(phase1, t);
+                else th.emplace_back(phase2, t);
+            }
+            if (phase == 0) phase1(0);
+            else phase2(0);
+            for (auto& x : th) x.join();
+            for (uint8_t b : bad)
+                if (b) return false;
+        }
+        for (const std::vector<Node>& top : tops)
+            for (const Node& nd : top) both.insert(nd);
+        for (int64_t c : doubly) both_read += c;
         depth[i] += n;
         return true;
     }
@@ -311,9 +441,12 @@ class Driver {
     // First item of list i, at or after position `from` of its prefix, that
     // is read from list i only and not fixed; -1 if none.
     int32_t only_from(int i, size_t from, int32_t skip) const {
+        if (single(i) == 0) return -1;
         const int j = 1 - i;
-        for (size_t p = from; p < prefix[i].size(); ++p) {
-            const int32_t x = prefix[i][p];
+        const std::vector<int32_t>& pre = prefix[i];
+        for (size_t p = from; p < pre.size(); ++p) {
+            if (p + 16 < pre.size()) __builtin_prefetch(ranks + 2 * (size_t)pre[p + 16], 0, 0);
+            const int32_t x = pre[p];
             if (inA(x) || x == skip) continue;
             if (active[j] && rank(j, x)) continue;
             return x;
@@ -322,9 +455,16 @@ class Driver {
     }
 
     void advance_ptr(int i) {
+        if (single(i) == 0) {   // every item of list i was read from both lists
+            ptr[i] = prefix[i].size();
+            return;
+        }
         const int j = 1 - i;
-        while (ptr[i] < prefix[i].size()) {
-            const int32_t x = prefix[i][ptr[i]];
+        const std::vector<int32_t>& pre = prefix[i];
+        while (ptr[i] < pre.size()) {
+            if (ptr[i] + 16 < pre.size())
+                __builtin_prefetch(ranks + 2 * (size_t)pre[ptr[i] + 16], 0, 0);
+            const int32_t x = pre[ptr[i]];
             if (inA(x) || (active[j] && rank(j, x))) {
                 ++ptr[i];
                 continue;
@@ -332,6 +472,9 @@ class Driver {
             break;
         }
     }
+
+    // Items read from list i only (certified or not).
+    int64_t single(int i) const { return depth[i] - both_read; }
 
     // Sec. 2.2 certification; returns true when the result is complete.
     bool certify() {

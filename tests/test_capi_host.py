@@ -257,3 +257,44 @@ def test_executor_rejects_null_handles_without_a_gpu():
         pvs.PVS_ERR_INVALID
     assert pvs._lib.pvs_executor_stats_get(None, None) == pvs.PVS_ERR_INVALID
     pvs._lib.pvs_executor_destroy(None)
+
+
+@pytest.mark.parametrize("relation", ["independent", "reversed", "noisy-reversed"])
+def test_deep_lists_through_the_threaded_record_path(relation):
+    """Pulls of 2^17 ranks and more are recorded by several threads; the
+    ordered Top-K must still equal complete-list fusion (Sec. 2.1)."""
+    n = 600_000
+    rng = np.random.default_rng(31)
+    a = rng.permutation(n)
+    if relation == "independent":
+        b = rng.permutation(n)
+    elif relation == "reversed":
+        b = a[::-1].copy()
+    else:
+        b = a[::-1].copy()
+        swap = rng.integers(0, n - 64, 5_000)
+        for s in swap:
+            b[s], b[s + 63] = b[s + 63], b[s]
+    for form, rf in FORMS:
+        ids, F, st = pvs.eahr_topk_lists(a, b, K=20, k=60, form=form)
+        T = ro.target_topk_large([a, b], [1, 1], 60, 20, rf)
+        assert ids.tolist() == [x for x, _ in T]
+        assert max(st["depth"]) > 1 << 17
+        for (x, f), g in zip(T, F):
+            if not np.isnan(g):
+                assert g == ro.as_float(f)
+
+
+@pytest.mark.parametrize("where", [(100, 450_000), (300_000, 300_001), (420_000, 590_000)])
+def test_repeated_ids_are_rejected_in_long_pulls(where):
+    """A host list that repeats an id is rejected, also when both copies fall
+    in one long pull (one thread part or two)."""
+    n = 600_000
+    rng = np.random.default_rng(37)
+    a = rng.permutation(n)
+    b = a[::-1].copy()       # read to the end: every position is recorded
+    i, j = where
+    b[j] = b[i]
+    with pytest.raises(pvs.PvsError) as e:
+        pvs.eahr_topk_lists(a, b, K=20, k=60)
+    assert e.value.status == pvs.PVS_ERR_INVALID
