@@ -917,7 +917,9 @@ def main_segments(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     bounds = [(n * i // SEGMENTS, n * (i + 1) // SEGMENTS) for i in range(SEGMENTS)]
     t0 = time.perf_counter()
     d_full = pvs.pvs_build(rows, stream=stream.cuda_stream)
-    d_seg = [pvs.pvs_build(rows[a:b], stream=stream.cuda_stream) for a, b in bounds]
+    # each Segment index gets a stream of its own (the library creates it),
+    # so the merge's concurrent refills of Segment cursors overlap on the GPU
+    d_seg = [pvs.pvs_build(rows[a:b]) for a, b in bounds]
     del rows
     torch.cuda.synchronize()
     comps = synth.mixture_components(n, COMPONENTS, seed=2, device=dev)

@@ -187,8 +187,7 @@ static cudaError_t launch_tpl(const IntervalArgs& a, int num_sms, cudaStream_t s
     if (stages > 8) stages = 8;
     if (stages < 2) return cudaErrorInvalidValue;
     const size_t smem = (size_t)stages * stage_bytes + 2 * stages * sizeof(uint64_t);
-    cudaError_t e = cudaFuncSetAttribute(interval_pass_kernel<CPL>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit((const void*)interval_pass_kernel<CPL>, smem);
     if (e != cudaSuccess) return e;
     const int64_t ntiles = (a.rows + kTileRows - 1) / kTileRows;
     const int grid = (int)(ntiles < num_sms ? ntiles : num_sms);

@@ -8,9 +8,17 @@
 // the item precedes everything any child can still produce (each child's
 // later ranks have smaller keys than its buffered ones).  Refill sizes start
 // from the request size spread over the children and double per refill.
+//
+// Refills are host round trips to the children's devices.  When a child runs
+// dry, every other child whose buffer is down to a quarter of its next
+// refill is refilled with it, and a round of several refills runs on one
+// host thread per child (each child is its own cursor with its own state),
+// so the round trips of one round overlap.  What is read ahead stays in the
+// buffers; the merged order does not depend on it.
 #include <algorithm>
 #include <cstring>
 #include <new>
+#include <thread>
 #include <unordered_set>
 #include <vector>
 
@@ -34,7 +42,15 @@ struct Child {
     size_t head = 0;
     bool exhausted = false;
     int64_t chunk = 0;       // next refill size
+    // result of the last refill (written by the thread that ran it)
+    pvs_status status = PVS_OK;
+    int64_t got = 0;
+    uint64_t key = 0;        // rank key of the buffered head (while left() > 0)
+    size_t left() const { return ids.size() - head; }
+    void set_key() { key = pvs::rank_key(scores[head], (uint32_t)ids[head]); }
 };
+
+constexpr size_t kRefillThreads = 16;   // concurrent refills per round
 
 }  // namespace
 
@@ -88,39 +104,70 @@ pvs_status describe(const pvs_merge_child& c, int64_t* length, int64_t* id_space
     }
 }
 
-// Read up to n ranks of a child into its (empty) buffer.
-pvs_status refill(pvs_merge* m, Child& c, int64_t n) {
-    c.ids.resize((size_t)n);
-    c.scores.resize((size_t)n);
+// Append up to n ranks of a child to its buffer (what was delivered is
+// dropped first).  Touches only the child: rounds run children concurrently.
+void refill(Child& c, int64_t n) {
+    c.ids.erase(c.ids.begin(), c.ids.begin() + (std::ptrdiff_t)c.head);
+    c.scores.erase(c.scores.begin(), c.scores.begin() + (std::ptrdiff_t)c.head);
     c.head = 0;
+    const size_t old = c.ids.size();
+    c.ids.resize(old + (size_t)n);
+    c.scores.resize(old + (size_t)n);
     int32_t got = 0;
     pvs_status s;
+    int64_t* ids = c.ids.data() + old;
+    float* scores = c.scores.data() + old;
     switch (c.kind) {
         case PVS_CHILD_DENSE:
-            s = pvs_next(static_cast<pvs_cursor*>(c.cur), (int32_t)n, c.ids.data(), c.scores.data(),
-                         &got);
+            s = pvs_next(static_cast<pvs_cursor*>(c.cur), (int32_t)n, ids, scores, &got);
             break;
         case PVS_CHILD_SPARSE:
-            s = pbm_next(static_cast<pbm_cursor*>(c.cur), (int32_t)n, c.ids.data(), c.scores.data(),
-                         &got);
+            s = pbm_next(static_cast<pbm_cursor*>(c.cur), (int32_t)n, ids, scores, &got);
             break;
         default:
-            s = pvs_merge_next(static_cast<pvs_merge*>(c.cur), (int32_t)n, c.ids.data(),
-                               c.scores.data(), &got);
+            s = pvs_merge_next(static_cast<pvs_merge*>(c.cur), (int32_t)n, ids, scores, &got);
             break;
     }
-    ++m->child_pulls;
-    if (s < 0) {
-        c.ids.clear();
-        c.scores.clear();
-        return s;
-    }
-    c.ids.resize((size_t)got);
-    c.scores.resize((size_t)got);
-    for (auto& x : c.ids) x += c.off;
-    m->read += got;
+    if (s < 0) got = 0;
+    c.ids.resize(old + (size_t)got);
+    c.scores.resize(old + (size_t)got);
+    for (size_t k = old; k < c.ids.size(); ++k) c.ids[k] += c.off;
+    if (c.left()) c.set_key();
+    c.status = s;
+    c.got = got;
     if (s == PVS_EXHAUSTED) c.exhausted = true;
-    return PVS_OK;
+}
+
+// One round: refill every child that is dry, and with them every child that
+// is down to a quarter of its next refill.  Returns the first error.
+pvs_status refill_round(pvs_merge* m, int32_t n) {
+    const int64_t k = (int64_t)m->ch.size();
+    std::vector<Child*> due;
+    bool dry = false;
+    for (Child& c : m->ch) {
+        if (c.exhausted) continue;
+        if (c.chunk == 0) c.chunk = std::max<int64_t>(16, 2 * ((n + k - 1) / k));
+        if (c.left() == 0) dry = true;
+    }
+    if (!dry) return PVS_OK;
+    for (Child& c : m->ch)
+        if (!c.exhausted && (int64_t)c.left() * 4 <= c.chunk) due.push_back(&c);
+    for (size_t b = 0; b < due.size(); b += kRefillThreads) {
+        const size_t e = std::min(due.size(), b + kRefillThreads);
+        std::vector<std::thread> th;
+        th.reserve(e - b);
+        for (size_t t = b + 1; t < e; ++t) th.emplace_back(refill, std::ref(*due[t]), due[t]->chunk);
+        refill(*due[b], due[b]->chunk);
+        for (auto& x : th) x.join();
+    }
+    pvs_status first = PVS_OK;
+    for (Child* c : due) {
+        ++m->child_pulls;
+        m->read += c->got;
+        c->chunk = std::min<int64_t>(c->chunk * 2, kMaxChunk);
+        if (c->status < 0 && first == PVS_OK) first = c->status;
+    }
+    return first;
 }
 
 bool seen(const pvs_merge* m, int64_t id) {
@@ -174,31 +221,27 @@ pvs_status pvs_merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, 
     if (!m) return PVS_ERR_INVALID;
     if (m->state < 0) return PVS_ERR_FAILED;
     if (n < 1 || !ids || !scores || !n_out) return PVS_ERR_INVALID;
-    const int64_t k = (int64_t)m->ch.size();
     int32_t count = 0;
+    // every child that can still produce has a buffered head before each
+    // item: children left dry by an error-free earlier call are refilled
+    // here, and a child that runs dry below right away
+    pvs_status s = refill_round(m, n);
+    if (s != PVS_OK) return fail(m, s);
     while (count < n) {
-        // every child that can still produce has a buffered head
-        for (Child& c : m->ch) {
-            if (c.head < c.ids.size() || c.exhausted) continue;
-            if (c.chunk == 0) c.chunk = std::max<int64_t>(16, 2 * ((n + k - 1) / k));
-            pvs_status s = refill(m, c, c.chunk);
-            if (s != PVS_OK) return fail(m, s);
-            c.chunk = std::min<int64_t>(c.chunk * 2, kMaxChunk);
-        }
         Child* best = nullptr;
-        uint64_t best_key = 0;
-        for (Child& c : m->ch) {
-            if (c.head >= c.ids.size()) continue;
-            const uint64_t key = pvs::rank_key(c.scores[c.head], (uint32_t)c.ids[c.head]);
-            if (!best || key > best_key) {
-                best = &c;
-                best_key = key;
-            }
-        }
+        for (Child& c : m->ch)
+            if (c.left() && (!best || c.key > best->key)) best = &c;
         if (!best) break;   // every child exhausted and delivered
+        const uint64_t best_key = best->key;
         const int64_t id = best->ids[best->head];
         const float sc = best->scores[best->head];
         ++best->head;
+        if (best->left()) {
+            best->set_key();
+        } else if (!best->exhausted) {
+            s = refill_round(m, n);
+            if (s != PVS_OK) return fail(m, s);
+        }
         if (m->any && best_key == m->last_key) {   // another copy with the same score
             ++m->dups;
             continue;

@@ -424,9 +424,8 @@ __global__ void __launch_bounds__(kFinishThreads) pbm_finish_kernel(const uint64
 cudaError_t launch_pbm_finish(const uint64_t* keys, const PbmCounters* ctr, uint64_t need,
                               int64_t* h_ids, float* h_scores, PbmCounters* h_mirror,
                               cudaStream_t st) {
-    cudaError_t e = cudaFuncSetAttribute(pbm_finish_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         kPbmFastWindow * (int)sizeof(uint64_t));
+    cudaError_t e = raise_smem_limit((const void*)pbm_finish_kernel,
+                                     kPbmFastWindow * sizeof(uint64_t));
     if (e != cudaSuccess) return e;
     count_launches(1);
     pbm_finish_kernel<<<1, kFinishThreads, kPbmFastWindow * sizeof(uint64_t), st>>>(

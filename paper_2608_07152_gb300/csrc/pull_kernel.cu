@@ -934,8 +934,7 @@ cudaError_t launch_ws_sort(const int32_t* w_id_b, const float* w_lo_b, const flo
     int pow2 = 1;
     while (pow2 < cap) pow2 <<= 1;
     const size_t smem = (size_t)pow2 * sizeof(unsigned long long);
-    cudaError_t e = cudaFuncSetAttribute(ws_sort_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit((const void*)ws_sort_kernel, smem);
     if (e != cudaSuccess) return e;
     count_launches(1);
     ws_sort_kernel<<<nq, kPullThreads, smem, st>>>(w_id_b, w_lo_b, w_hi_b, cap, w_len_b, dst);

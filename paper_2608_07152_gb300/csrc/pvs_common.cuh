@@ -4,6 +4,9 @@
 
 #include <cstdint>
 #include <cuda_runtime.h>
+#include <map>
+#include <mutex>
+#include <utility>
 
 #include "../../include/pvs.h"
 #include "kernels.h"
@@ -197,6 +200,24 @@ __device__ inline RowQuant quantize_row_warp(const float* __restrict__ v, int m,
     if (isinf(r.vnorm) || isinf(r.enorm)) r.status = PVS_ERR_OVERFLOW;
     if (out_of_range) r.status = PVS_ERR_INVALID;
     return r;
+}
+
+// Raise, never lower, a kernel's dynamic shared-memory limit on the current
+// device.  The limit belongs to the function, not to a launch: host threads
+// that launch one kernel with different sizes would otherwise undo each
+// other's setting between one thread's set and its launch.
+inline cudaError_t raise_smem_limit(const void* fn, size_t bytes) {
+    static std::mutex mu;
+    static std::map<std::pair<int, const void*>, size_t> limits;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    size_t& cur = limits[std::make_pair(dev, fn)];
+    if (bytes <= cur) return cudaSuccess;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) cur = bytes;
+    return e;
 }
 
 }  // namespace pvs

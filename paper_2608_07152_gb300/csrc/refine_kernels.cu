@@ -256,7 +256,7 @@ static int ring_stages(int m_raw) {
 }
 
 static cudaError_t ring_attr(const void* fn, size_t smem) {
-    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return raise_smem_limit(fn, smem);
 }
 
 // Staging the query takes m_raw floats of shared memory; up to 48 KB.

@@ -289,8 +289,7 @@ cudaError_t launch_bitonic_desc(uint64_t* keys, int count, cudaStream_t st) {
     int pow2 = 2;
     while (pow2 < count) pow2 <<= 1;
     const size_t smem = (size_t)pow2 * sizeof(uint64_t);
-    cudaError_t e = cudaFuncSetAttribute(bitonic_desc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit((const void*)bitonic_desc_kernel, smem);
     if (e != cudaSuccess) return e;
     count_launches(1);
     bitonic_desc_kernel<<<1, 1024, smem, st>>>(keys, count, pow2);
