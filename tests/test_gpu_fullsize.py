@@ -126,3 +126,111 @@ def test_eahr_with_deep_pulls_matches_complete_list_fusion(tau):
                 assert got == ro.as_float(f)
     finally:
         pvs.pvs_index_free(index)
+
+
+def _oracle_check_ranks(q, V, ids, sc, visible=None):
+    """The oracle's complete ranking (Sec. 2.1) agrees with the delivered
+    prefix id by id and in the bits of every authoritative score."""
+    ref_ids, ref_sc = po.dense_ranking(q, V, visible)
+    k = ids.size
+    assert np.array_equal(ids, ref_ids[:k])
+    assert np.array_equal(sc.view(np.uint32), ref_sc[:k].view(np.uint32))
+
+
+def test_batched_configuration_at_full_size():
+    """1,000,000 x 768 (1,024 mixture components), one batch of 256 queries
+    opened together (tensor-core filter pass, horizon 200), then 4 batched
+    pulls of 50 ranks into device buffers on the batch's stream: the
+    benchmark's launch configuration.  Sampled queries are checked against
+    the oracle's complete ranking."""
+    dev = torch.device("cuda")
+    n = 1_000_000
+    centres = synth.mixture_centres(1024, DIM, seed=4, device=dev)
+    rows = torch.empty((n, DIM), dtype=torch.float32, device=dev)
+    for r in range(0, n, 1 << 20):
+        c = min(1 << 20, n - r)
+        rows[r:r + c] = synth.mixture_rows(c, centres, 0.35, seed=4, first=r)
+    index = pvs.pvs_build(rows)
+    Q = synth.mixture_queries(256, centres, 0.5, seed=5).contiguous()
+    st = torch.cuda.Stream()
+    ids_t = torch.empty((256, 50), dtype=torch.int64, device=dev)
+    sc_t = torch.empty((256, 50), dtype=torch.float32, device=dev)
+    got_ids, got_sc = [], []
+    try:
+        curs = pvs.pvs_cursor_open_batch(index, Q, horizon=200, stream=st)
+        try:
+            for _ in range(4):
+                n_out = pvs.pvs_next_batch(curs, 50, ids_t, sc_t)
+                assert all(n_out == 50)
+                st.synchronize()
+                got_ids.append(ids_t.cpu().numpy().copy())
+                got_sc.append(sc_t.cpu().numpy().copy())
+            assert all(s >= 0 for s in pvs.pvs_cursor_sync_batch(curs))
+        finally:
+            pvs.pvs_cursor_close_batch(curs)
+        V = rows.cpu().numpy()
+        Qh = Q.cpu().numpy()
+        for i in (0, 97, 255):
+            _oracle_check_ranks(Qh[i], V, np.concatenate([g[i] for g in got_ids]),
+                                np.concatenate([g[i] for g in got_sc]))
+    finally:
+        pvs.pvs_index_free(index)
+
+
+def test_snapshot_configuration_at_full_size():
+    """2,000,000 x 1,024 with 20 % near-duplicates (copies + N(0, 1e-4^2),
+    normalised); snapshot 1, then 200,000 appended rows and 2 % of the live
+    rows tombstoned, snapshot 2 (Sec. 2.4).  Per snapshot, sampled queries:
+    the first 1,000 dense ranks equal the oracle's over the snapshot's
+    visible rows, and EAHR Top-20 against a tau = 0.2 copula ranking of the
+    visible ids equals complete-list fusion (Sec. 2.1, 2.2)."""
+    dev = torch.device("cuda")
+    n0, d, add = 2_000_000, 1024, 200_000
+    centres = synth.mixture_centres(4096, d, seed=5, device=dev)
+    rows = torch.empty((n0 + add, d), dtype=torch.float32, device=dev)
+    n_mix = n0 - n0 // 5
+    rows[:n_mix] = synth.mixture_rows(n_mix, centres, 0.35, seed=5)
+    g = torch.Generator(device=dev)
+    g.manual_seed(55)
+    src = torch.randint(0, n_mix, (n0 - n_mix,), generator=g, device=dev)
+    rows[n_mix:n0] = synth.near_duplicate_rows(rows[src], 1e-4, seed=56)
+    rows[n0:] = synth.mixture_rows(add, centres, 0.35, seed=61)
+    index = pvs.pvs_build(rows[:n0])
+    Q = synth.mixture_queries(4, centres, 0.5, seed=58)
+    snaps = []
+    try:
+        snaps.append(pvs.pvs_snapshot_create(index))
+        pvs.pvs_append(index, rows[n0:])
+        rng = np.random.default_rng(57)
+        dead = rng.choice(n0 + add, int(0.02 * (n0 + add)), replace=False)
+        pvs.pvs_tombstone(index, dead)
+        snaps.append(pvs.pvs_snapshot_create(index))
+        vis = [np.zeros(n0 + add, bool), np.ones(n0 + add, bool)]
+        vis[0][:n0] = True
+        vis[1][dead] = False
+        V = rows.cpu().numpy()
+        for s, snap in enumerate(snaps):
+            vis_ids = torch.from_numpy(np.nonzero(vis[s])[0]).to(dev)
+            for j in (2 * s, 2 * s + 1):
+                q = Q[j].contiguous()
+                cur = pvs.pvs_cursor_open(index, q, snap)
+                ids, sc, _ = pvs.pvs_next(cur, 1000)
+                pvs.pvs_cursor_close(cur)
+                qh = q.cpu().numpy()
+                ref_ids, ref_sc = po.dense_ranking(qh, V, vis[s])
+                assert np.array_equal(ids, ref_ids[:1000])
+                assert np.array_equal(sc.view(np.uint32), ref_sc[:1000].view(np.uint32))
+                proxy = rows[vis_ids] @ q
+                sparse = vis_ids[synth.copula_ranking(proxy, 0.2, 900 + j)].cpu().numpy()
+                cur = pvs.pvs_cursor_open(index, q, snap)
+                got, F, _ = pvs.eahr_topk(cur, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+                pvs.pvs_cursor_close(cur)
+                T = ro.target_topk_large([ref_ids, sparse], [1, 1], 60, 20, ro.NUMERATOR)
+                assert got.tolist() == [x for x, _ in T]
+                for (x, f), v in zip(T, F):
+                    if not np.isnan(v):
+                        assert v == ro.as_float(f)
+    finally:
+        for snap in snaps:
+            pvs.pvs_snapshot_free(snap)
+        pvs.pvs_index_free(index)
