@@ -125,6 +125,11 @@ __global__ void __launch_bounds__(kIntervalThreads, 1)
         }
     }
 
+    // the slot's kSlotTop largest live lower bounds, descending
+    float top[kSlotTop];
+#pragma unroll
+    for (int j = 0; j < kSlotTop; ++j) top[j] = -INFINITY;
+
     int k = 0;
     for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++k) {
         const int s = k % stages;
@@ -174,9 +179,24 @@ __global__ void __launch_bounds__(kIntervalThreads, 1)
             if (tombstoned(a.tomb, row)) lo = hi = -INFINITY;
             a.lo[row] = lo;
             a.hi[row] = hi;
+            if (lo > top[kSlotTop - 1]) {   // insertion into the descending list
+                top[kSlotTop - 1] = lo;
+#pragma unroll
+                for (int j = kSlotTop - 1; j > 0; --j)
+                    if (top[j] > top[j - 1]) {
+                        const float x = top[j];
+                        top[j] = top[j - 1];
+                        top[j - 1] = x;
+                    }
+            }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[s]);
+    }
+    if (a.slot_top && p == 0) {
+        float* o = a.slot_top + ((size_t)blockIdx.x * TR + (size_t)r_in_tile) * kSlotTop;
+#pragma unroll
+        for (int j = 0; j < kSlotTop; ++j) o[j] = top[j];
     }
 }
 
@@ -197,6 +217,26 @@ static cudaError_t launch_tpl(const IntervalArgs& a, int num_sms, cudaStream_t s
     interval_pass_kernel<CPL><<<grid, kIntervalThreads, smem, st>>>(a, stages, rotate,
                                                                      a.m_pad / 64);
     return cudaGetLastError();
+}
+
+// The staged kernel serves these row widths (the others take the unstaged one).
+static bool staged_width(int m_pad) {
+    switch (m_pad / 64) {
+        case 1: case 2: case 4: case 6: case 8: case 12: case 16: return true;
+        default: break;
+    }
+    return kTileRows * m_pad + 3 * kTileRows * 4 <= 100 * 1024;
+}
+
+int64_t interval_slots(int64_t rows, int m_pad, int num_sms, int64_t* min_rows_per_slot) {
+    *min_rows_per_slot = 0;
+    if (rows <= 0 || !staged_width(m_pad)) return 0;
+    const int64_t ntiles = (rows + kTileRows - 1) / kTileRows;
+    const int64_t grid = ntiles < num_sms ? ntiles : num_sms;
+    // CTA b scans tiles b, b + grid, ...: at least ntiles / grid of them, of
+    // which only the very last tile of the pass can be partial
+    *min_rows_per_slot = ntiles / grid - 1;
+    return grid * kTileRows;
 }
 
 cudaError_t launch_interval_pass(const IntervalArgs& a, int num_sms, cudaStream_t st) {

@@ -162,8 +162,17 @@ struct IntervalArgs {
     float* lo;
     float* hi;
     int* status;
+    // optional: the kSlotTop largest live lower bounds of every row slot of
+    // the staged pass (slot = CTA x row position in a tile; each row belongs
+    // to one slot), kSlotTop per slot, -inf where a slot had fewer live rows
+    float* slot_top = nullptr;
 };
+constexpr int kSlotTop = 4;
 cudaError_t launch_interval_pass(const IntervalArgs& a, int num_sms, cudaStream_t st);
+// Slots whose kSlotTop lower bounds a pass over `rows` rows of m_pad bytes
+// writes to slot_top (0: that pass writes none), and the fewest rows any
+// of them scans.
+int64_t interval_slots(int64_t rows, int m_pad, int num_sms, int64_t* min_rows_per_slot);
 // Plain reference-style variant without staging (used for tiny inputs).
 cudaError_t launch_interval_simple(const IntervalArgs& a, cudaStream_t st);
 

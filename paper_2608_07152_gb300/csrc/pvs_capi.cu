@@ -199,7 +199,8 @@ void cursor_free_device(pvs_cursor* c) {
     dev_free(c->zq), dev_free(c->qraw), dev_free(c->qs);
     dev_free(c->lo), dev_free(c->hi);
     dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
-    dev_free(c->compact_scratch);
+    dev_free(c->compact_scratch), dev_free(c->slot_top);
+    c->slot_cap = 0;
     dev_free(c->cand), dev_free(c->keys), dev_free(c->keys_tmp), dev_free(c->front);
     if (c->sort_scratch) cudaFree(c->sort_scratch);
     c->sort_scratch = nullptr;
@@ -233,6 +234,8 @@ void cursor_reset(pvs_cursor* c) {
     c->batch_passes = 0;
     c->batch_ms = 0.0;
     c->ev_pending = false;
+    c->slot_fresh = false;
+    c->slot_n = 0;
     c->interval_ms = 0.0;
     c->generator = PVS_GEN_INTERVALS;
     c->scan_ready = false;
@@ -376,6 +379,23 @@ pvs_status interval_pass(pvs_cursor* c) {
     a.lo = c->lo;
     a.hi = c->hi;
     a.status = c->d_status;
+    // per-slot largest lower bounds, for the first working set (see
+    // build_working_set): only when no row is tombstoned and every slot
+    // scans at least kSlotTop rows, so that every entry is a live row's bound
+    int64_t min_rows = 0;
+    const int64_t slots = interval_slots(c->rows, x->m_pad, x->num_sms, &min_rows);
+    c->slot_fresh = false;
+    c->slot_n = 0;
+    if (slots > 0 && c->snap->d_tomb == nullptr && min_rows >= kSlotTop) {
+        if (c->slot_cap < slots * kSlotTop) {
+            dev_free(c->slot_top);
+            c->slot_cap = 0;
+            PVS_CUDA(dev_alloc(&c->slot_top, (size_t)(slots * kSlotTop)));
+            c->slot_cap = slots * kSlotTop;
+        }
+        a.slot_top = c->slot_top;
+        c->slot_n = slots * kSlotTop;
+    }
     if (!c->ev_begin) {
         PVS_CUDA(cudaEventCreate(&c->ev_begin));
         PVS_CUDA(cudaEventCreate(&c->ev_end));
@@ -388,6 +408,7 @@ pvs_status interval_pass(pvs_cursor* c) {
     else PVS_CUDA(cudaStreamWaitEvent(c->stream, x->pass_done, 0));
     PVS_CUDA(cudaEventRecord(c->ev_begin, c->stream));
     PVS_CUDA(launch_interval_pass(a, x->num_sms, c->stream));
+    c->slot_fresh = a.slot_top != nullptr;
     PVS_CUDA(cudaEventRecord(c->ev_end, c->stream));
     PVS_CUDA(cudaEventRecord(x->pass_done, c->stream));
     c->ev_pending = true;
@@ -402,7 +423,16 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     const int64_t remaining = c->visible - c->emitted;
     int64_t H = std::max<int64_t>({want, 2 * c->horizon, 2048});
     if (H > remaining) H = remaining;
-    if (H < remaining) {
+    if (H < remaining && c->slot_fresh && H <= c->slot_n) {
+        // Each of the slot_n per-slot entries is the lower bound of a
+        // distinct live row, so at least H rows have lo >= the H-th largest
+        // entry v: v is at most the H-th largest lo of all rows, and the
+        // rows with hi >= v hold the working set (a few more rows than the
+        // exact threshold keeps; a few thousand entries are selected from
+        // instead of every row).
+        PVS_CUDA(launch_select_f32_n(c->slot_top, c->slot_n, (uint64_t)H, c->sel,
+                                     grid_for(c, c->slot_n), c->stream));
+    } else if (H < remaining) {
         PVS_CUDA(launch_select_f32_n(c->lo, c->rows, (uint64_t)H, c->sel, grid_for(c, c->rows),
                                      c->stream));
     } else {
@@ -410,6 +440,7 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     }
     PVS_CUDA(launch_compact_ordered(c->lo, c->hi, c->rows, c->sel, c->w_id, c->w_lo, c->w_hi,
                                     &c->ctr->w_len, c->compact_scratch, c->stream));
+    c->slot_fresh = false;   // later builds select from the current bounds
     c->horizon = H;
     c->horizon_base = c->emitted;
     c->horizon_builds++;
@@ -428,6 +459,7 @@ pvs_status rescan_from_batch(pvs_cursor* c) {
     if (s != PVS_OK) return s;
     s = interval_pass(c);
     if (s != PVS_OK) return s;
+    c->slot_fresh = false;   // the scatter below changes bounds (delivered rows leave)
     PVS_CUDA(launch_scatter_ws(c->w_id, c->w_lo, c->w_hi, &c->ctr->w_len, c->lo, c->hi,
                                grid_for(c, c->cap_w), c->stream));
     // the working set is rebuilt from the full bounds; its arrays may grow

@@ -94,6 +94,13 @@ struct pvs_cursor {
     float* w_hi = nullptr;
     int64_t horizon = 0, horizon_base = 0;
     unsigned int* compact_scratch = nullptr;
+    // the interval pass's largest lower bounds per row slot (kSlotTop each):
+    // while fresh (the pass's bounds unchanged, every slot holding at least
+    // kSlotTop live rows), the H-th largest of them bounds the H-th largest
+    // lower bound of all rows from below
+    float* slot_top = nullptr;
+    int64_t slot_cap = 0, slot_n = 0;
+    bool slot_fresh = false;
     // pull scratch
     int32_t* cand = nullptr;
     int32_t* front = nullptr;         // frontier of the one-launch pull (kFrontCap entries)

@@ -494,3 +494,41 @@ def test_eahr_rejects_bad_sparse_lists_and_used_cursors():
         pvs.pvs_cursor_close(cur)
     finally:
         pvs.pvs_index_free(index)
+
+
+@pytest.mark.parametrize("crowded", [False, True])
+def test_first_working_set_from_per_slot_bounds(crowded):
+    """The first working set after an interval pass is selected from each row
+    slot's four largest lower bounds (a slot = a CTA's row position in a
+    64-row tile).  That threshold is never above the exact one, so the ranks
+    stay exact; with the best rows crowded into one slot it is much lower and
+    the working set larger, and the ranks must still be exact (Sec. 2.1,
+    2.3.1)."""
+    n, m = 2_000_003, 32
+    rng = np.random.default_rng(211)
+    V = rng.standard_normal((n, m)).astype(np.float32)
+    V /= np.linalg.norm(V, axis=1, keepdims=True)
+    q = rng.standard_normal(m).astype(np.float32)
+    q /= np.linalg.norm(q)
+    if crowded:
+        # rows of slot 5 of the first CTA (tiles 0, 152, 304, ... of 64 rows)
+        # are near-copies of the query: every one of them beats every other row
+        rows = np.arange(5, n, 64 * 152)
+        V[rows] = q + 0.01 * rng.standard_normal((rows.size, m)).astype(np.float32)
+        V[rows] /= np.linalg.norm(V[rows], axis=1, keepdims=True)
+    index = pvs.pvs_build(V)
+    try:
+        cur = pvs.pvs_cursor_open(index, q)
+        try:
+            got = [pvs.pvs_next(cur, 20) for _ in range(50)]
+            st = pvs.pvs_cursor_stats(cur)
+        finally:
+            pvs.pvs_cursor_close(cur)
+    finally:
+        pvs.pvs_index_free(index)
+    ids = np.concatenate([g[0] for g in got])
+    sc = np.concatenate([g[1] for g in got])
+    ref_ids, ref_sc = po.dense_ranking(q, V)
+    assert np.array_equal(ids, ref_ids[:1000])
+    assert np.array_equal(sc.view(np.uint32), ref_sc[:1000].view(np.uint32))
+    assert st["interval_passes"] == 1
