@@ -51,6 +51,8 @@ typedef struct pbm_stats {
     int64_t items_scored;      /* items of expanded ranges (scored exactly)  */
     int64_t pulls;             /* pbm_next calls                             */
     int64_t rounds;            /* expand-and-certify rounds over all pulls   */
+    int64_t pulls_from_window; /* pulls served on the host from an earlier
+                                  pull's certified window (no device work)  */
     int32_t state;             /* PVS_OK, PVS_EXHAUSTED or an error          */
     int32_t reserved;
 } pbm_stats;

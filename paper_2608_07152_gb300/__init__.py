@@ -76,7 +76,8 @@ class eahr_stats(ctypes.Structure):
 class pbm_stats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
         "items", "emitted", "ranges", "ranges_expanded", "postings_visited", "items_scored",
-        "pulls", "rounds")] + [("state", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+        "pulls", "rounds", "pulls_from_window")] + [("state", ctypes.c_int32),
+                                                    ("reserved", ctypes.c_int32)]
 
 
 class pvs_merge_child(ctypes.Structure):

@@ -109,12 +109,18 @@ struct pbm_cursor {
     void* sort_scratch = nullptr;
     int64_t* out_ids = nullptr;
     float* out_scores = nullptr;
-    int64_t* h_ids = nullptr;         // pinned: ranks of a pull served by the finish kernel
-    float* h_scores = nullptr;
+    int64_t* h_ids = nullptr;         // pinned: the sorted window of the last pull served by
+    float* h_scores = nullptr;        // the finish kernel
+    // entries [ahead_pos, ahead_len) of that window are certified ranks not
+    // yet delivered: the next ranks in order (their keys exceed the bound of
+    // every range not expanded when the window was taken, and the window held
+    // every scored item above that bound), served without device work
+    int64_t ahead_pos = 0, ahead_len = 0;
     uint64_t last_key = ~0ull;
     int64_t next = 0;                 // ranges expanded (a prefix of the sorted order)
     uint64_t E = 64;                  // ranges to expand in the next round
     int64_t emitted = 0, pulls = 0, rounds = 0;
+    int64_t served_ahead = 0;         // pulls served from the window without device work
     int state = PVS_OK;
 };
 
@@ -404,6 +410,22 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     cudaStream_t st = c->stream;
     ++c->pulls;
     const uint64_t need = (uint64_t)std::min<int64_t>(n, x->n_items - c->emitted);
+    if ((uint64_t)(c->ahead_len - c->ahead_pos) >= need) {   // certified ranks already here
+        std::memcpy(ids, c->h_ids + c->ahead_pos, need * sizeof(int64_t));
+        std::memcpy(scores, c->h_scores + c->ahead_pos, need * sizeof(float));
+        c->ahead_pos += (int64_t)need;
+        c->last_key = pvs::rank_key(scores[need - 1], (uint32_t)ids[need - 1]);
+        c->emitted += (int64_t)need;
+        ++c->served_ahead;
+        *n_out = (int32_t)need;
+        if (c->emitted == x->n_items) {
+            c->state = PVS_EXHAUSTED;
+            return PVS_EXHAUSTED;
+        }
+        return PVS_OK;
+    }
+    // too few: the device gathers them again (they lie below last_key)
+    c->ahead_pos = c->ahead_len = 0;
     uint64_t E = std::max<uint64_t>(c->E, 2 * ((need + x->block - 1) / x->block));
     uint64_t window = 0;
     uint64_t last = 0;   // size of the last expansion of this pull
@@ -456,6 +478,8 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     if (served) {
         std::memcpy(ids, c->h_ids, m * sizeof(int64_t));
         std::memcpy(scores, c->h_scores, m * sizeof(float));
+        c->ahead_pos = (int64_t)m;
+        c->ahead_len = (int64_t)window;
     } else if (m > 0) {
         // large window: the m-th largest key first (or the whole window when
         // it fits the gather buffer), then a device sort of the m keys
@@ -514,6 +538,7 @@ pvs_status pbm_cursor_stats(pbm_cursor* c, pbm_stats* out) {
     out->items_scored = (int64_t)c->h_ctr->items;
     out->pulls = c->pulls;
     out->rounds = c->rounds;
+    out->pulls_from_window = c->served_ahead;
     out->state = c->state;
     out->reserved = 0;
     return PVS_OK;

@@ -412,7 +412,9 @@ __global__ void __launch_bounds__(kFinishThreads) pbm_finish_kernel(const uint64
                 __syncthreads();
             }
         }
-        for (int i = threadIdx.x; (unsigned long long)i < need; i += blockDim.x) {
+        // the whole window, sorted: every key in it is certified, so the
+        // host can serve later pulls from what lies beyond `need`
+        for (int i = threadIdx.x; (unsigned long long)i < count; i += blockDim.x) {
             h_ids[i] = (int64_t)rank_key_id(keys[i]);
             h_scores[i] = rank_key_score(keys[i]);
         }

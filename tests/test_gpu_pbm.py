@@ -129,6 +129,8 @@ def test_bm25_corpus_deep_pulls_and_large_windows():
         q_postings = sum(int(off[t + 1] - off[t]) for t in terms)
         assert stats["postings_visited"] == q_postings      # every posting once, at the end
         assert stats["items_scored"] == n_items
+        # pulls of 20 inside an earlier pull's certified window need no device work
+        assert stats["pulls_from_window"] > 0
 
 
 def test_first_ranks_touch_few_ranges():
