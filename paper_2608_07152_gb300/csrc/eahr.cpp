@@ -419,14 +419,20 @@ class Driver {
             tops[(size_t)t] = std::move(top.buf);
         };
         for (auto phase : {0, 1}) {
+            auto run = [&](int t) {
+                if (phase == 0) phase1(t);
+                else phase2(t);
+            };
+            // parts whose thread could not be started run here, after part 0
             std::vector<std::thread> th;
-            th.reserve((size_t)T - 1);
-            for (int t = 1; t < T; ++t) {
-                if (phase == 0) th.emplace_back(phase1, t);
-                else th.emplace_back(phase2, t);
+            int started = 1;
+            try {
+                th.reserve((size_t)T - 1);
+                for (; started < T; ++started) th.emplace_back(run, started);
+            } catch (...) {
             }
-            if (phase == 0) phase1(0);
-            else phase2(0);
+            run(0);
+            for (int t = started; t < T; ++t) run(t);
             for (auto& x : th) x.join();
             for (uint8_t b : bad)
                 if (b) return false;
@@ -570,8 +576,22 @@ bool contrib_from(const eahr_params* p, int i, int64_t max_rank, Contrib* out) {
     return true;
 }
 
+pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
+                      int32_t* n_out, eahr_stats* st);
+
+// The driver behind every entry point: allocation failures (prefixes of
+// millions of ranks) become PVS_ERR_OOM instead of leaving the C ABI.
 pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F, int32_t* n_out,
                eahr_stats* st) {
+    try {
+        return run_driver(d, p, out_ids, out_F, n_out, st);
+    } catch (const std::bad_alloc&) {
+        return PVS_ERR_OOM;
+    }
+}
+
+pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
+                      int32_t* n_out, eahr_stats* st) {
     const int step0 = p->step > 0 ? p->step : 16;
     int64_t size[2] = {step0, step0};
     d.K = p->K;

@@ -154,10 +154,17 @@ pvs_status refill_round(pvs_merge* m, int32_t n) {
         if (!c.exhausted && (int64_t)c.left() * 4 <= c.chunk) due.push_back(&c);
     for (size_t b = 0; b < due.size(); b += kRefillThreads) {
         const size_t e = std::min(due.size(), b + kRefillThreads);
+        // refills whose thread could not be started run here
         std::vector<std::thread> th;
-        th.reserve(e - b);
-        for (size_t t = b + 1; t < e; ++t) th.emplace_back(refill, std::ref(*due[t]), due[t]->chunk);
+        size_t started = b + 1;
+        try {
+            th.reserve(e - b);
+            for (; started < e; ++started)
+                th.emplace_back(refill, std::ref(*due[started]), due[started]->chunk);
+        } catch (...) {
+        }
         refill(*due[b], due[b]->chunk);
+        for (size_t t = started; t < e; ++t) refill(*due[t], due[t]->chunk);
         for (auto& x : th) x.join();
     }
     pvs_status first = PVS_OK;
@@ -174,6 +181,10 @@ bool seen(const pvs_merge* m, int64_t id) {
     return (m->seen[(size_t)(id >> 6)] >> (id & 63)) & 1u;
 }
 
+}  // namespace
+
+namespace {
+pvs_status merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, int32_t* n_out);
 }  // namespace
 
 extern "C" {
@@ -216,7 +227,22 @@ pvs_status pvs_merge_open(const pvs_merge_child* children, int32_t count, pvs_me
     return PVS_OK;
 }
 
+// Buffer growth that fails fails the merge cursor (PVS_ERR_OOM) instead of
+// leaving the C ABI.
 pvs_status pvs_merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    try {
+        return merge_next(m, n, ids, scores, n_out);
+    } catch (const std::bad_alloc&) {
+        if (n_out) *n_out = 0;
+        return m ? fail(m, PVS_ERR_OOM) : PVS_ERR_OOM;
+    }
+}
+
+}  // extern "C"
+
+namespace {
+
+pvs_status merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
     if (n_out) *n_out = 0;
     if (!m) return PVS_ERR_INVALID;
     if (m->state < 0) return PVS_ERR_FAILED;
@@ -265,6 +291,10 @@ pvs_status pvs_merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, 
     }
     return PVS_OK;
 }
+
+}  // namespace
+
+extern "C" {
 
 pvs_status pvs_merge_stats_get(pvs_merge* m, pvs_merge_stats* out) {
     if (!m || !out) return PVS_ERR_INVALID;
