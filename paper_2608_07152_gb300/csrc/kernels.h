@@ -183,6 +183,10 @@ cudaError_t launch_interval_simple(const IntervalArgs& a, cudaStream_t st);
 cudaError_t launch_select_f32(const float* vals, const unsigned int* len, uint64_t k,
                               SelectState* sel, int grid, cudaStream_t st);
 // Same over `rows` entries with a host-known length.
+// As launch_select_f32_n in one single-CTA launch, for short arrays (tens of
+// thousands of values).
+cudaError_t launch_select_small(const float* vals, int64_t len, uint64_t k, SelectState* sel,
+                                cudaStream_t st);
 cudaError_t launch_select_f32_n(const float* vals, int64_t rows, uint64_t k, SelectState* sel,
                                 int grid, cudaStream_t st);
 // Ordered compaction: for i < rows with lo[i] != -inf and key(hi[i]) >=

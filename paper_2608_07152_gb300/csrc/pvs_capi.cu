@@ -430,8 +430,7 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
         // rows with hi >= v hold the working set (a few more rows than the
         // exact threshold keeps; a few thousand entries are selected from
         // instead of every row).
-        PVS_CUDA(launch_select_f32_n(c->slot_top, c->slot_n, (uint64_t)H, c->sel,
-                                     grid_for(c, c->slot_n), c->stream));
+        PVS_CUDA(launch_select_small(c->slot_top, c->slot_n, (uint64_t)H, c->sel, c->stream));
     } else if (H < remaining) {
         PVS_CUDA(launch_select_f32_n(c->lo, c->rows, (uint64_t)H, c->sel, grid_for(c, c->rows),
                                      c->stream));

@@ -97,6 +97,69 @@ cudaError_t launch_select_f32_n(const float* vals, int64_t rows, uint64_t k, Sel
     return select_f32(vals, nullptr, rows, k, sel, grid, st);
 }
 
+// The same selection for a short array in one launch: one CTA runs the four
+// digit rounds with its histogram in shared memory (the values are re-read
+// from L2 each round).
+__global__ void __launch_bounds__(1024) select_small_kernel(const float* __restrict__ vals,
+                                                            int64_t len, uint64_t k0,
+                                                            SelectState* sel) {
+    __shared__ unsigned int h[256];
+    __shared__ unsigned int suffix[256];
+    __shared__ uint32_t prefix;
+    __shared__ unsigned long long k;
+    const int t = threadIdx.x;
+    if (t == 0) {
+        prefix = 0;
+        k = k0;
+    }
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        if (t < 256) h[t] = 0;
+        __syncthreads();
+        const uint32_t hmask = shift >= 24 ? 0u : (0xffffffffu << (shift + 8));
+        const uint32_t pre = prefix;
+        for (int64_t i = t; i < len; i += blockDim.x) {
+            const float v = vals[i];
+            if (v == -INFINITY) continue;
+            const uint32_t key = fkey(v);
+            if ((key & hmask) != (pre & hmask)) continue;
+            atomicAdd(&h[(key >> shift) & 0xffu], 1u);
+        }
+        __syncthreads();
+        // suffix[u] = keys whose digit is 255 - u or above
+        if (t < 256) suffix[t] = h[255 - t];
+        __syncthreads();
+        for (int o = 1; o < 256; o <<= 1) {
+            unsigned int v = (t < 256 && t >= o) ? suffix[t - o] : 0u;
+            __syncthreads();
+            if (t < 256) suffix[t] += v;
+            __syncthreads();
+        }
+        // every thread reads k before the one thread holding the digit
+        // (exactly one: keys are counted once) rewrites it
+        const unsigned long long kk = k;
+        const unsigned long long above = (t < 256 && t > 0) ? suffix[t - 1] : 0u;
+        const bool mine = t < 256 && above < kk && kk <= (unsigned long long)suffix[t];
+        __syncthreads();
+        if (mine) {
+            prefix = pre | ((uint32_t)(255 - t) << shift);
+            k = kk - above;
+        }
+        __syncthreads();
+    }
+    if (t == 0) {
+        sel->prefix = prefix;
+        sel->k = k;
+    }
+    if (t < 256) sel->hist[t] = 0;
+}
+
+cudaError_t launch_select_small(const float* vals, int64_t len, uint64_t k, SelectState* sel,
+                                cudaStream_t st) {
+    count_launches(1);
+    select_small_kernel<<<1, 1024, 0, st>>>(vals, len, k, sel);
+    return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------
 // ordered compaction of the working set: {i : lo[i] live, key(hi[i]) >= tau}
 // ---------------------------------------------------------------------------
