@@ -97,12 +97,13 @@ cudaError_t launch_select_f32_n(const float* vals, int64_t rows, uint64_t k, Sel
     return select_f32(vals, nullptr, rows, k, sel, grid, st);
 }
 
-// The same selection for a short array in one launch: one CTA runs the four
-// digit rounds with its histogram in shared memory (the values are re-read
-// from L2 each round).
+// The same selection for a short array in one launch: one CTA copies the
+// values into shared memory once (16-byte loads; when they fit) and runs the
+// four digit rounds there, its histogram in shared memory too.
 __global__ void __launch_bounds__(1024) select_small_kernel(const float* __restrict__ vals,
                                                             int64_t len, uint64_t k0,
-                                                            SelectState* sel) {
+                                                            SelectState* sel, int staged) {
+    extern __shared__ float4 staged_vals[];
     __shared__ unsigned int h[256];
     __shared__ unsigned int suffix[256];
     __shared__ uint32_t prefix;
@@ -112,18 +113,38 @@ __global__ void __launch_bounds__(1024) select_small_kernel(const float* __restr
         prefix = 0;
         k = k0;
     }
+    const float* src = vals;
+    if (staged) {
+        const int64_t n4 = len / 4;
+        const float4* v4 = reinterpret_cast<const float4*>(vals);
+        for (int64_t i = t; i < n4; i += blockDim.x) staged_vals[i] = v4[i];
+        float* sf = reinterpret_cast<float*>(staged_vals);
+        for (int64_t i = n4 * 4 + t; i < len; i += blockDim.x) sf[i] = vals[i];
+        src = sf;
+    }
     for (int shift = 24; shift >= 0; shift -= 8) {
         if (t < 256) h[t] = 0;
         __syncthreads();
         const uint32_t hmask = shift >= 24 ? 0u : (0xffffffffu << (shift + 8));
         const uint32_t pre = prefix;
+        // close scores share their high digits: each thread counts a run of
+        // one digit in a register and adds it when the digit changes
+        uint32_t run_d = 256u;
+        unsigned int run_n = 0;
         for (int64_t i = t; i < len; i += blockDim.x) {
-            const float v = vals[i];
+            const float v = src[i];
             if (v == -INFINITY) continue;
             const uint32_t key = fkey(v);
             if ((key & hmask) != (pre & hmask)) continue;
-            atomicAdd(&h[(key >> shift) & 0xffu], 1u);
+            const uint32_t d = (key >> shift) & 0xffu;
+            if (d != run_d) {
+                if (run_n) atomicAdd(&h[run_d], run_n);
+                run_d = d;
+                run_n = 0;
+            }
+            ++run_n;
         }
+        if (run_n) atomicAdd(&h[run_d], run_n);
         __syncthreads();
         // suffix[u] = keys whose digit is 255 - u or above
         if (t < 256) suffix[t] = h[255 - t];
@@ -155,8 +176,17 @@ __global__ void __launch_bounds__(1024) select_small_kernel(const float* __restr
 
 cudaError_t launch_select_small(const float* vals, int64_t len, uint64_t k, SelectState* sel,
                                 cudaStream_t st) {
+    // staged in shared memory when the values fit in 200 KB and start on a
+    // 16-byte boundary (device allocations do)
+    const bool staged = len > 0 && len * (int64_t)sizeof(float) <= 200 * 1024 &&
+                        (reinterpret_cast<uintptr_t>(vals) & 15u) == 0;
+    const size_t smem = staged ? (size_t)((len + 3) / 4) * sizeof(float4) : 0;
+    if (smem > 0) {
+        cudaError_t e = raise_smem_limit((const void*)select_small_kernel, smem);
+        if (e != cudaSuccess) return e;
+    }
     count_launches(1);
-    select_small_kernel<<<1, 1024, 0, st>>>(vals, len, k, sel);
+    select_small_kernel<<<1, 1024, smem, st>>>(vals, len, k, sel, staged ? 1 : 0);
     return cudaGetLastError();
 }
 
@@ -171,10 +201,14 @@ size_t compact_scratch_elems(int64_t rows) {
     return (size_t)((rows + kCompactTile - 1) / kCompactTile) + 1;
 }
 
+// A row leaves (emitted, tombstoned) with lo = hi = -inf, and refinement
+// sets lo = hi = its score: lo is -inf exactly when hi is.  So a threshold
+// that is the key of a finite bound (tau != 0) is reached only by live rows
+// and needs hi alone; tau = 0 (every live row) reads lo.
 __device__ __forceinline__ bool ws_member(const float* lo, const float* hi, int64_t i,
                                           uint32_t tau) {
-    const float l = lo[i];
-    return l != -INFINITY && fkey(hi[i]) >= tau;
+    if (tau != 0u) return fkey(hi[i]) >= tau;
+    return lo[i] != -INFINITY;
 }
 
 __global__ void compact_count_kernel(const float* __restrict__ lo, const float* __restrict__ hi,
