@@ -168,19 +168,41 @@ inline bool beats(const Frac& a, int32_t x, const Frac& b, int32_t y) {
 // kPoolBytes in all; larger or surplus ones are freed).  The two lists'
 // ranks of one id sit side by side (one cache line serves both lookups), and
 // the certified-set flags are a bitset (1.1 MB at 8.8M ids, cache-resident).
+// The two lists' read ids are stored here too (a valid list repeats no id,
+// so cap entries hold it); their contents are always ids below cap.
 struct Workspace {
     int32_t* ranks = nullptr;    // [cap][2]
     uint64_t* bits = nullptr;    // [(cap + 63) / 64]
+    int32_t* read[2] = {nullptr, nullptr};   // [cap] each
     int64_t cap = 0;
-    size_t bytes() const { return (size_t)cap * 2 * sizeof(int32_t) + (size_t)(cap + 63) / 8; }
+    size_t bytes() const {
+        return (size_t)cap * 4 * sizeof(int32_t) + (size_t)(cap + 63) / 8;
+    }
     void release() {
         std::free(ranks);
         std::free(bits);
+        std::free(read[0]);
+        std::free(read[1]);
         ranks = nullptr;
         bits = nullptr;
+        read[0] = read[1] = nullptr;
         cap = 0;
     }
 };
+
+// The ids read from one list, in rank order, in workspace storage.
+struct IdList {
+    int32_t* p = nullptr;
+    size_t n = 0, cap = 0;
+    size_t size() const { return n; }
+    int32_t operator[](size_t i) const { return p[i]; }
+    const int32_t* begin() const { return p; }
+    const int32_t* end() const { return p + n; }
+};
+
+// memset of a large array over up to kMaxThreads threads (what a thread
+// that cannot start would have cleared is cleared here).
+void zero_parallel(void* dst, size_t bytes);
 
 constexpr size_t kPoolMax = 16;
 constexpr int64_t kParallelMin = int64_t(1) << 17;   // ranks per pull worth threads
@@ -211,7 +233,9 @@ bool acquire(int64_t ids, Workspace* out) {
     w.cap = ids;
     w.ranks = static_cast<int32_t*>(std::calloc((size_t)ids * 2, sizeof(int32_t)));
     w.bits = static_cast<uint64_t*>(std::calloc((size_t)(ids + 63) / 64, sizeof(uint64_t)));
-    if (!w.ranks || !w.bits) {
+    w.read[0] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
+    w.read[1] = static_cast<int32_t*>(std::calloc((size_t)ids, sizeof(int32_t)));
+    if (!w.ranks || !w.bits || !w.read[0] || !w.read[1]) {
         w.release();
         return false;
     }
@@ -228,6 +252,29 @@ void give_back(Workspace w) {
         return;
     }
     w.release();
+}
+
+void zero_parallel(void* dst, size_t bytes) {
+    const unsigned T = std::min<unsigned>(kMaxThreads, std::thread::hardware_concurrency());
+    if (bytes < (size_t(16) << 20) || T < 2) {
+        std::memset(dst, 0, bytes);
+        return;
+    }
+    uint8_t* b = static_cast<uint8_t*>(dst);
+    auto part = [&](unsigned t) {
+        const size_t lo = bytes * t / T, hi = bytes * (t + 1) / T;
+        std::memset(b + lo, 0, hi - lo);
+    };
+    std::vector<std::thread> th;
+    unsigned started = 1;
+    try {
+        th.reserve(T - 1);
+        for (; started < T; ++started) th.emplace_back(part, started);
+    } catch (...) {
+    }
+    part(0);
+    for (unsigned t = started; t < T; ++t) part(t);
+    for (auto& x : th) x.join();
 }
 
 struct Source {
@@ -248,7 +295,7 @@ class Driver {
     bool exhausted[2] = {false, false};
     int32_t pulls[2] = {0, 0};
     int32_t checks = 0;
-    std::vector<int32_t> prefix[2];
+    IdList prefix[2];
     int32_t* ranks = nullptr;    // ranks[2 x + i]: rank of id x in list i (0: unread)
     uint64_t* bits = nullptr;    // bit x: x is certified (in A)
     int64_t id_space = 0;
@@ -271,7 +318,7 @@ class Driver {
     ~Driver() {
         if (!ws.ranks) return;
         if ((int64_t)(prefix[0].size() + prefix[1].size()) > ws.cap / 8) {
-            std::memset(ranks, 0, (size_t)ws.cap * 2 * sizeof(int32_t));
+            zero_parallel(ranks, (size_t)ws.cap * 2 * sizeof(int32_t));
         } else {
             for (int i = 0; i < 2; ++i)
                 for (int32_t x : prefix[i]) ranks[2 * (size_t)x + (size_t)i] = 0;
@@ -285,6 +332,11 @@ class Driver {
         if (!acquire(id_space, &ws)) return false;
         ranks = ws.ranks;
         bits = ws.bits;
+        for (int i = 0; i < 2; ++i) {
+            prefix[i].p = ws.read[i];
+            prefix[i].n = 0;
+            prefix[i].cap = (size_t)ws.cap;
+        }
         return true;
     }
 
@@ -322,8 +374,7 @@ class Driver {
         // ids arrive in rank order, scattered over the id space: fetch the
         // rank pair of the id kAhead positions on while this one is handled
         constexpr int64_t kAhead = 16;
-        if (prefix[i].capacity() < prefix[i].size() + (size_t)n)
-            prefix[i].reserve(std::max(2 * prefix[i].capacity(), prefix[i].size() + (size_t)n));
+        if (prefix[i].n + (size_t)n > prefix[i].cap) return false;   // an id repeats
         for (int64_t t = 0; t < n; ++t) {
             if (t + kAhead < n) {
                 const int64_t y = ids[t + kAhead];
@@ -336,7 +387,7 @@ class Driver {
                 if (rank(i, (int32_t)x64)) return false;
             }
             const int32_t x = (int32_t)x64;
-            prefix[i].push_back(x);
+            prefix[i].p[prefix[i].n++] = x;
             ranks[2 * (size_t)x + (size_t)i] = (int32_t)(depth[i] + t + 1);
             if (rank(j, x)) {
                 ++both_read;
@@ -356,11 +407,12 @@ class Driver {
         const int j = 1 - i;
         const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
                            src[i].merge == nullptr;
-        std::vector<int32_t>& pre = prefix[i];
-        const size_t base = pre.size();
-        if (pre.capacity() < base + (size_t)n)
-            pre.reserve(std::max(2 * pre.capacity(), base + (size_t)n));
-        pre.resize(base + (size_t)n, 0);
+        IdList& pre = prefix[i];
+        const size_t base = pre.n;
+        if (base + (size_t)n > pre.cap) return false;   // an id repeats
+        // counted before the parts run: cleanup then covers whatever a part
+        // wrote before it stopped (stale entries are ids below cap)
+        pre.n = base + (size_t)n;
         const int64_t d0 = depth[i];
         std::vector<uint8_t> bad((size_t)T, 0);
         std::vector<std::vector<Node>> tops((size_t)T);
@@ -390,7 +442,7 @@ class Driver {
                     return;
                 }
                 __atomic_store_n(slot, (int32_t)(d0 + k + 1), __ATOMIC_RELAXED);
-                pre[base + (size_t)k] = (int32_t)x64;
+                pre.p[base + (size_t)k] = (int32_t)x64;
             }
         };
         auto phase2 = [&](int t) {
@@ -449,7 +501,7 @@ class Driver {
     int32_t only_from(int i, size_t from, int32_t skip) const {
         if (single(i) == 0) return -1;
         const int j = 1 - i;
-        const std::vector<int32_t>& pre = prefix[i];
+        const IdList& pre = prefix[i];
         for (size_t p = from; p < pre.size(); ++p) {
             if (p + 16 < pre.size()) __builtin_prefetch(ranks + 2 * (size_t)pre[p + 16], 0, 0);
             const int32_t x = pre[p];
@@ -466,7 +518,7 @@ class Driver {
             return;
         }
         const int j = 1 - i;
-        const std::vector<int32_t>& pre = prefix[i];
+        const IdList& pre = prefix[i];
         while (ptr[i] < pre.size()) {
             if (ptr[i] + 16 < pre.size())
                 __builtin_prefetch(ranks + 2 * (size_t)pre[ptr[i] + 16], 0, 0);
@@ -731,13 +783,20 @@ pvs_status eahr_topk_lists(const int64_t* list0, int64_t n0, const int64_t* list
     if (!params_ok(p) || !out_ids || !n_out || n0 < 0 || n1 < 0 || (n0 > 0 && !list0) ||
         (n1 > 0 && !list1))
         return PVS_ERR_INVALID;
-    int64_t id_space = 0;
-    for (int64_t t = 0; t < n0; ++t) id_space = std::max<int64_t>(id_space, list0[t] + 1);
-    for (int64_t t = 0; t < n1; ++t) id_space = std::max<int64_t>(id_space, list1[t] + 1);
-    for (int64_t t = 0; t < n0; ++t)
-        if (list0[t] < 0) return PVS_ERR_INVALID;
-    for (int64_t t = 0; t < n1; ++t)
-        if (list1[t] < 0) return PVS_ERR_INVALID;
+    // one pass per list: the id space (largest id + 1) and no negative id
+    int64_t id_space = 0, lowest = 0;
+    for (int i = 0; i < 2; ++i) {
+        const int64_t* l = i == 0 ? list0 : list1;
+        const int64_t len = i == 0 ? n0 : n1;
+        int64_t hi = -1, lo = 0;
+        for (int64_t t = 0; t < len; ++t) {
+            hi = std::max(hi, l[t]);
+            lo = std::min(lo, l[t]);
+        }
+        id_space = std::max(id_space, hi + 1);
+        lowest = std::min(lowest, lo);
+    }
+    if (lowest < 0) return PVS_ERR_INVALID;
     if (id_space > ((int64_t)1 << 31)) return PVS_ERR_INVALID;
     Driver d;
     d.src[0].list = list0;
