@@ -585,20 +585,26 @@ class Driver {
     pvs_status pull(int i, int64_t n) {
         if (exhausted[i] || !active[i]) return PVS_OK;
         pulls[i]++;
-        if (src[i].cursor || src[i].sparse || src[i].merge) {
-            if (n > (int64_t)std::numeric_limits<int32_t>::max()) n = std::numeric_limits<int32_t>::max();
+        if (n > (int64_t)std::numeric_limits<int32_t>::max()) n = std::numeric_limits<int32_t>::max();
+        if (src[i].cursor) {   // read where the pull left them (pinned), without a copy
+            const int64_t* ids = nullptr;
+            const float* scores = nullptr;
+            int32_t got = 0;
+            pvs_status s = pvs::next_pinned(src[i].cursor, (int32_t)n, &ids, &scores, &got);
+            if (s < 0) return s;
+            if (!record(i, ids, got)) return PVS_ERR_INVALID;
+            if (s == PVS_EXHAUSTED) exhausted[i] = true;
+        } else if (src[i].sparse || src[i].merge) {
             buf_ids.resize((size_t)n);
             buf_scores.resize((size_t)n);
             int32_t got = 0;
             pvs_status s =
-                src[i].cursor
-                    ? pvs_next(src[i].cursor, (int32_t)n, buf_ids.data(), buf_scores.data(), &got)
-                : src[i].sparse
+                src[i].sparse
                     ? pbm_next(src[i].sparse, (int32_t)n, buf_ids.data(), buf_scores.data(), &got)
                     : pvs_merge_next(src[i].merge, (int32_t)n, buf_ids.data(), buf_scores.data(),
                                      &got);
             if (s < 0) return s;
-            record(i, buf_ids.data(), got);
+            if (!record(i, buf_ids.data(), got)) return PVS_ERR_INVALID;
             if (s == PVS_EXHAUSTED) exhausted[i] = true;
         } else {
             const int64_t take = std::min<int64_t>(n, src[i].length - depth[i]);

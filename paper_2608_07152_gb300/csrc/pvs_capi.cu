@@ -1464,12 +1464,10 @@ static pvs_status next_common(pvs_cursor* c, int32_t n, int32_t* n_out, int64_t*
     return PVS_OK;
 }
 
-pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
-    DeviceGuard device_guard(cursor_device(c));
-    int64_t n_eff;
-    pvs_status s = next_common(c, n, n_out, &n_eff);
-    if (s != PVS_OK) return s;
-    if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
+// pvs_next's pull: the next n_eff >= 0 ranks end in the cursor's pinned
+// buffers (c->h_ids, c->h_scores; valid until its next pull).
+static pvs_status pull_to_pinned(pvs_cursor* c, int64_t n_eff) {
+    pvs_status s;
     if (n_eff > 0 && n_eff <= kPullFusedMax) {
         // the kernels write ids, scores and the status word straight into the
         // cursor's pinned host buffers: one launch, one wait
@@ -1488,8 +1486,6 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         harvest_interval_time(c);
         const int dev_status = *reinterpret_cast<volatile int*>(mirror);
         if (dev_status != 0) return fail(c, (pvs_status)dev_status);
-        std::memcpy(ids, c->h_ids, n_eff * sizeof(int64_t));
-        std::memcpy(scores, c->h_scores, n_eff * sizeof(float));
     } else if (n_eff > 0) {
         s = cursor_out_reserve(c, n_eff);
         if (s != PVS_OK) return fail(c, s);
@@ -1504,13 +1500,48 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         if (e != cudaSuccess) return fail(c, cuda_status(e));
         s = check_device_status(c);
         if (s != PVS_OK) return s;
+    }
+    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
+    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+}
+
+pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
+    DeviceGuard device_guard(cursor_device(c));
+    int64_t n_eff;
+    pvs_status s = next_common(c, n, n_out, &n_eff);
+    if (s != PVS_OK) return s;
+    if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
+    s = pull_to_pinned(c, n_eff);
+    if (s < 0) return s;
+    if (n_eff > 0) {
         std::memcpy(ids, c->h_ids, n_eff * sizeof(int64_t));
         std::memcpy(scores, c->h_scores, n_eff * sizeof(float));
     }
     *n_out = (int32_t)n_eff;
-    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
-    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+    return s;
 }
+
+}  // extern "C"
+
+// The next n ranks left in the cursor's pinned buffers, for host code of
+// this library that reads them once (the EAHR driver): *ids and *scores
+// point there and stay valid until the cursor's next pull.  As pvs_next.
+pvs_status pvs::next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
+                            int32_t* n_out) {
+    DeviceGuard device_guard(cursor_device(c));
+    int64_t n_eff;
+    pvs_status s = next_common(c, n, n_out, &n_eff);
+    if (s != PVS_OK) return s;
+    if (!ids || !scores) return PVS_ERR_INVALID;
+    s = pull_to_pinned(c, n_eff);
+    if (s < 0) return s;
+    *ids = c->h_ids;
+    *scores = c->h_scores;
+    *n_out = (int32_t)n_eff;
+    return s;
+}
+
+extern "C" {
 
 pvs_status pvs_next_device(pvs_cursor* c, int32_t n, int64_t* ids, float* scores,
                            int32_t* n_out) {

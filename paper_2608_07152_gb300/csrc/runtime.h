@@ -139,6 +139,10 @@ namespace pvs {
 int64_t cursor_visible(const pvs_cursor* c);
 int64_t cursor_emitted(const pvs_cursor* c);
 const SnapData* cursor_snapshot(const pvs_cursor* c);
+// pvs_next with the ranks left in the cursor's pinned buffers (valid until
+// its next pull) instead of copied out.
+pvs_status next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
+                       int32_t* n_out);
 // Open a cursor whose device work runs on `stream` (null: the index's stream).
 pvs_status cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const float* query,
                           int32_t query_on_device, cudaStream_t stream, pvs_cursor** out);
