@@ -1,6 +1,6 @@
 """GPU parity of the PVS path against the oracle, through the C ABI.
 
-Bars (BASELINE correctness rules, arXiv 2608.07152 Sec. 2.1, 2.3.1, App. A.1):
+Bars (arXiv 2608.07152 Sec. 2.1, 2.3.1, App. A.1):
   * codes, scales and norm bounds: bit-exact with the oracle quantizer;
   * intervals: bit-exact with the oracle's interval arithmetic, and sound
     (lo <= authoritative score <= hi) for every vector;
