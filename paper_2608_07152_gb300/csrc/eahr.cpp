@@ -207,6 +207,7 @@ void zero_parallel(void* dst, size_t bytes);
 constexpr size_t kPoolMax = 16;
 constexpr int64_t kParallelMin = int64_t(1) << 17;   // ranks per pull worth threads
 constexpr unsigned kMaxThreads = 8;
+constexpr int64_t kAheadMin = int64_t(1) << 17;   // dense pulls worth a helper thread
 constexpr size_t kPoolBytes = size_t(1) << 30;
 
 std::mutex g_pool_mutex;
@@ -310,12 +311,41 @@ class Driver {
 
     Workspace ws;
 
+    // A dense pull running on a helper thread while this one records the
+    // other list and certifies (long pulls of a dense cursor only).  The
+    // cursor is touched by that thread alone until it is joined; its ranks
+    // stay in the cursor's pinned buffers until they are recorded.
+    std::thread ahead;
+    bool ahead_live = false;
+    pvs_status ahead_status = PVS_OK;
+    const int64_t* ahead_ids = nullptr;
+    const float* ahead_scores = nullptr;
+    int32_t ahead_got = 0;
+
+    void start_ahead(int64_t n) {
+        if (ahead_live || !src[0].cursor || !active[0] || exhausted[0]) return;
+        n = std::min<int64_t>(n, std::numeric_limits<int32_t>::max());
+        try {
+            ahead = std::thread([this, n] {
+                ahead_status = pvs::next_pinned(src[0].cursor, (int32_t)n, &ahead_ids,
+                                                &ahead_scores, &ahead_got);
+            });
+            ahead_live = true;
+        } catch (...) {   // no thread: the pull runs when it is needed
+        }
+    }
+    void join_ahead() {
+        if (ahead_live) ahead.join();
+        ahead_live = false;
+    }
+
     int32_t rank(int i, int32_t x) const { return ranks[2 * (size_t)x + (size_t)i]; }
     bool inA(int32_t x) const { return (bits[(uint32_t)x >> 6] >> (x & 63)) & 1u; }
 
     // Every entry written is an id of prefix[i] (ranks) or of A (bits):
     // clear those, or whole arrays when that is cheaper, and pool them.
     ~Driver() {
+        join_ahead();
         if (!ws.ranks) return;
         if ((int64_t)(prefix[0].size() + prefix[1].size()) > ws.cap / 8) {
             zero_parallel(ranks, (size_t)ws.cap * 2 * sizeof(int32_t));
@@ -590,7 +620,16 @@ class Driver {
             const int64_t* ids = nullptr;
             const float* scores = nullptr;
             int32_t got = 0;
-            pvs_status s = pvs::next_pinned(src[i].cursor, (int32_t)n, &ids, &scores, &got);
+            pvs_status s;
+            if (ahead_live) {   // the pull started earlier: its ranks are the next ones
+                join_ahead();
+                s = ahead_status;
+                ids = ahead_ids;
+                scores = ahead_scores;
+                got = ahead_got;
+            } else {
+                s = pvs::next_pinned(src[i].cursor, (int32_t)n, &ids, &scores, &got);
+            }
             if (s < 0) return s;
             if (!record(i, ids, got)) return PVS_ERR_INVALID;
             if (s == PVS_EXHAUSTED) exhausted[i] = true;
@@ -712,6 +751,9 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
                 if (s < 0) return s;
                 size[pick] = std::min<int64_t>(2 * size[pick], (int64_t)1 << 24);
             }
+            // long dense pulls: the next one starts now, beside certification
+            // and the other list's pull (ranks read ahead change no result)
+            if (size[0] >= kAheadMin) d.start_ahead(size[0]);
         }
         done = d.certify();
         if (!done) {
