@@ -56,6 +56,10 @@ constexpr size_t kRefillThreads = 16;   // concurrent refills per round
 
 struct pvs_merge {
     std::vector<Child> ch;
+    // winner tree over the children's head keys: node i holds the child with
+    // the larger key of nodes 2i and 2i+1, leaf P + c child c (-1: none)
+    std::vector<int32_t> tree;
+    int32_t P = 1;
     int64_t id_space = 0, length = 0;
     std::vector<uint64_t> seen;   // delivered request ids (bitmap)
     uint64_t last_key = 0;
@@ -177,6 +181,31 @@ pvs_status refill_round(pvs_merge* m, int32_t n) {
     return first;
 }
 
+// Key of child c's buffered head; 0 when it has none (real rank keys are
+// larger: a finite score's ordered key is at least 2^23).
+uint64_t head_key(const pvs_merge* m, int32_t c) {
+    if (c < 0) return 0;
+    const Child& x = m->ch[(size_t)c];
+    return x.left() ? x.key : 0;
+}
+
+int32_t winner(const pvs_merge* m, int32_t a, int32_t b) {
+    return head_key(m, a) >= head_key(m, b) ? a : b;
+}
+
+void tree_build(pvs_merge* m) {
+    const int32_t k = (int32_t)m->ch.size();
+    for (int32_t c = 0; c < m->P; ++c) m->tree[(size_t)(m->P + c)] = c < k ? c : -1;
+    for (int32_t i = m->P - 1; i >= 1; --i)
+        m->tree[(size_t)i] = winner(m, m->tree[(size_t)(2 * i)], m->tree[(size_t)(2 * i + 1)]);
+}
+
+// Child c's head changed: replay its path to the root.
+void tree_update(pvs_merge* m, int32_t c) {
+    for (int32_t i = (m->P + c) >> 1; i >= 1; i >>= 1)
+        m->tree[(size_t)i] = winner(m, m->tree[(size_t)(2 * i)], m->tree[(size_t)(2 * i + 1)]);
+}
+
 bool seen(const pvs_merge* m, int64_t id) {
     return (m->seen[(size_t)(id >> 6)] >> (id & 63)) & 1u;
 }
@@ -223,6 +252,8 @@ pvs_status pvs_merge_open(const pvs_merge_child* children, int32_t count, pvs_me
         return PVS_ERR_INVALID;
     }
     m->seen.assign((size_t)((m->id_space + 63) / 64), 0ull);
+    while (m->P < count) m->P *= 2;
+    m->tree.assign((size_t)(2 * m->P), -1);
     *out = m;
     return PVS_OK;
 }
@@ -253,20 +284,24 @@ pvs_status merge_next(pvs_merge* m, int32_t n, int64_t* ids, float* scores, int3
     // here, and a child that runs dry below right away
     pvs_status s = refill_round(m, n);
     if (s != PVS_OK) return fail(m, s);
+    tree_build(m);
     while (count < n) {
-        Child* best = nullptr;
-        for (Child& c : m->ch)
-            if (c.left() && (!best || c.key > best->key)) best = &c;
-        if (!best) break;   // every child exhausted and delivered
+        const int32_t b = m->tree[1];
+        if (head_key(m, b) == 0) break;   // every child exhausted and delivered
+        Child* best = &m->ch[(size_t)b];
         const uint64_t best_key = best->key;
         const int64_t id = best->ids[best->head];
         const float sc = best->scores[best->head];
         ++best->head;
         if (best->left()) {
             best->set_key();
+            tree_update(m, b);
         } else if (!best->exhausted) {
-            s = refill_round(m, n);
+            s = refill_round(m, n);   // may refill several children
             if (s != PVS_OK) return fail(m, s);
+            tree_build(m);
+        } else {
+            tree_update(m, b);
         }
         if (m->any && best_key == m->last_key) {   // another copy with the same score
             ++m->dups;
