@@ -1,7 +1,8 @@
 """The multi-rank logic of bench.py on CPU with the gloo backend (world size
 2): one process per rank, the job's time is the slowest rank's, throughput
 counts every rank's units, every rank draws its own queries, and only rank 0
-runs the reference arm."""
+runs the reference arm; the clock record keeps only samples of the timed
+region."""
 import os
 import socket
 
@@ -58,3 +59,25 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
     monkeypatch.setenv("WORLD_SIZE", "2")
     bench.reference_arm(object())                # returns before reading any argument
     assert capsys.readouterr().out == ""
+
+
+def test_clock_summary_keeps_the_samples_of_the_timed_region():
+    """The clock record of a bench line: only samples that arrived between the
+    region's start and one sampling period after its end count; throttle
+    reasons are collected from those samples alone."""
+    cs = bench.ClockSampler(0)
+    cs.t0, cs.t1 = 10.0, 11.0
+    row = "0, {sm}, 2070, 900.00, 0x0, {hw}, Not Active, Not Active, {pc}\n"
+    cs.rows = [
+        (9.5, row.format(sm=1200, hw="Active", pc="Not Active")),      # before: dropped
+        (10.2, row.format(sm=2070, hw="Not Active", pc="Not Active")),
+        (10.6, row.format(sm=2055, hw="Not Active", pc="Active")),
+        (11.05, row.format(sm=2070, hw="Not Active", pc="Not Active")),  # last period: kept
+        (11.5, row.format(sm=900, hw="Active", pc="Not Active")),       # after: dropped
+    ]
+    s = cs.summary()
+    assert s["samples"] == 3
+    assert s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0
+    assert s["reasons"] == ["sw_power_cap"]
+    cs.rows = [(12.0, row.format(sm=2070, hw="Not Active", pc="Not Active"))]
+    assert cs.summary()["reasons"] == ["unsampled"]
