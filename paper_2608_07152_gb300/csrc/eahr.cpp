@@ -500,10 +500,34 @@ class Driver {
             doubly[(size_t)t] = count;
             tops[(size_t)t] = std::move(top.buf);
         };
-        for (auto phase : {0, 1}) {
+        // a cursor's ids never repeat: one pass per part writes the ranks and
+        // collects the doubly-read items (the other list is not written here)
+        auto single = [&](int t) {
+            int64_t lo, hi;
+            part(t, &lo, &hi);
+            TopStream top;
+            top.cap = both.cap;
+            top.buf.reserve(TopStream::kCut);
+            int64_t count = 0;
+            for (int64_t k = lo; k < hi; ++k) {
+                if (k + 16 < hi) __builtin_prefetch(ranks + 2 * ids[k + 16], 1, 0);
+                const int32_t x = (int32_t)ids[k];
+                ranks[2 * (size_t)x + (size_t)i] = (int32_t)(d0 + k + 1);
+                pre.p[base + (size_t)k] = x;
+                if (rank(j, x)) {
+                    ++count;
+                    if (!inA(x)) top.push(Node{L(x), x});
+                }
+            }
+            top.cut();
+            doubly[(size_t)t] = count;
+            tops[(size_t)t] = std::move(top.buf);
+        };
+        for (int phase = check ? 0 : 2; phase < (check ? 2 : 3); ++phase) {
             auto run = [&](int t) {
                 if (phase == 0) phase1(t);
-                else phase2(t);
+                else if (phase == 1) phase2(t);
+                else single(t);
             };
             // parts whose thread could not be started run here, after part 0
             std::vector<std::thread> th;
