@@ -96,8 +96,12 @@ pvs_status pbm_cursor_open(pbm_index* index, const int32_t* terms, const float* 
  * (float32) in host memory, *n_out of them.  Returns PVS_OK, or
  * PVS_EXHAUSTED once all N items have been delivered (then *n_out < n, or
  * *n_out == n for the call that delivers the last item).  Output is an
- * append-only exact prefix (Sec. 2.1).  Errors: PVS_ERR_INVALID (n < 1, null
- * pointer), PVS_ERR_OVERFLOW (a score or bound overflowed float32),
+ * append-only exact prefix (Sec. 2.1).  A pull whose certified window (every
+ * scored item above the bound of every range not yet expanded, at most 8,192
+ * of them) holds more ranks than requested keeps the rest in the cursor's
+ * pinned memory: later pulls that fit in them are served there, with no
+ * device work (pbm_stats.pulls_from_window).  Errors: PVS_ERR_INVALID (n < 1,
+ * null pointer), PVS_ERR_OVERFLOW (a score or bound overflowed float32),
  * PVS_ERR_OOM, PVS_ERR_CUDA, PVS_ERR_FAILED (the cursor failed earlier).
  */
 pvs_status pbm_next(pbm_cursor* cursor, int32_t n, int64_t* ids, float* scores, int32_t* n_out);
