@@ -11,7 +11,10 @@
  * A merge cursor reads its children (PVS cursors, PBM cursors or other merge
  * cursors, so a Shard of Segments and a request of Shards are both merge
  * cursors) in chunks, keeps what it has read but not yet delivered, and
- * delivers the merged order.  A child's ids are mapped to the request's id
+ * delivers the merged order.  Children due for more ranks at the same time
+ * are read concurrently, one host thread each: children on streams of their
+ * own (e.g. Segment indexes built without a shared stream) then also overlap
+ * on the device.  A child's ids are mapped to the request's id
  * space by adding the child's id_offset.  Copies: an item delivered by two
  * children with the same score is delivered once (they are adjacent in the
  * merged order); the same id with another score fails the merge cursor with
