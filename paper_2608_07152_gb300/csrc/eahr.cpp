@@ -278,6 +278,39 @@ void zero_parallel(void* dst, size_t bytes) {
     for (auto& x : th) x.join();
 }
 
+// Smallest (at most 0) and largest (at least -1) id of a host list, long
+// lists over up to kMaxThreads threads.
+void id_range(const int64_t* l, int64_t len, int64_t* lo_out, int64_t* hi_out) {
+    const unsigned T = len >= (int64_t(1) << 20)
+                           ? std::min<unsigned>(kMaxThreads, std::thread::hardware_concurrency())
+                           : 1u;
+    std::vector<int64_t> lo((size_t)std::max(T, 1u), 0), hi((size_t)std::max(T, 1u), -1);
+    auto part = [&](unsigned t) {
+        const int64_t a = len * (int64_t)t / (int64_t)T, b = len * (int64_t)(t + 1) / (int64_t)T;
+        int64_t x = 0, y = -1;
+        for (int64_t k = a; k < b; ++k) {
+            x = std::min(x, l[k]);
+            y = std::max(y, l[k]);
+        }
+        lo[t] = x;
+        hi[t] = y;
+    };
+    std::vector<std::thread> th;
+    unsigned started = 1;
+    if (T > 1) {
+        try {
+            th.reserve(T - 1);
+            for (; started < T; ++started) th.emplace_back(part, started);
+        } catch (...) {
+        }
+    }
+    if (T >= 1) part(0);
+    for (unsigned t = started; t < T; ++t) part(t);
+    for (auto& x : th) x.join();
+    *lo_out = *std::min_element(lo.begin(), lo.end());
+    *hi_out = *std::max_element(hi.begin(), hi.end());
+}
+
 struct Source {
     // dense cursor, sparse PBM cursor, merge cursor or host list
     pvs_cursor* cursor = nullptr;
@@ -858,13 +891,8 @@ pvs_status eahr_topk_lists(const int64_t* list0, int64_t n0, const int64_t* list
     // one pass per list: the id space (largest id + 1) and no negative id
     int64_t id_space = 0, lowest = 0;
     for (int i = 0; i < 2; ++i) {
-        const int64_t* l = i == 0 ? list0 : list1;
-        const int64_t len = i == 0 ? n0 : n1;
         int64_t hi = -1, lo = 0;
-        for (int64_t t = 0; t < len; ++t) {
-            hi = std::max(hi, l[t]);
-            lo = std::min(lo, l[t]);
-        }
+        id_range(i == 0 ? list0 : list1, i == 0 ? n0 : n1, &lo, &hi);
         id_space = std::max(id_space, hi + 1);
         lowest = std::min(lowest, lo);
     }

@@ -298,3 +298,16 @@ def test_repeated_ids_are_rejected_in_long_pulls(where):
     with pytest.raises(pvs.PvsError) as e:
         pvs.eahr_topk_lists(a, b, K=20, k=60)
     assert e.value.status == pvs.PVS_ERR_INVALID
+
+
+@pytest.mark.parametrize("where", [0, 1_234_567, 2_099_999])
+def test_negative_ids_are_rejected_in_long_host_lists(where):
+    """Long host lists are validated over several threads: a negative id
+    anywhere is rejected."""
+    n = 2_100_000
+    a = np.arange(n, dtype=np.int64)
+    b = a[::-1].copy()
+    b[where] = -3
+    with pytest.raises(pvs.PvsError) as e:
+        pvs.eahr_topk_lists(a, b, K=20, k=60)
+    assert e.value.status == pvs.PVS_ERR_INVALID
