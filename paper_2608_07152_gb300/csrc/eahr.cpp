@@ -461,11 +461,16 @@ class Driver {
         return true;
     }
 
-    // record() over T threads, for long pulls.  Phase 1 writes the ranks
-    // (and the prefix), each thread a contiguous part; phase 2 reads every
-    // written rank back (a repeated id leaves a rank that is not its own)
-    // and collects each part's best items read from both lists.  Which items
+    // record() over T threads, for long pulls: each thread takes a
+    // contiguous part and, in one pass, writes the ranks (and the read ids)
+    // and collects its part's best items read from both lists.  Which items
     // enter `both`, the K + 2 best, does not depend on the order of inserts.
+    // A cursor's ids never repeat; a host list's are checked as they are
+    // written: the rank slot is exchanged, and a slot that already held a
+    // rank (from an earlier pull, or from another part of this one) means a
+    // repeated id.  L of a doubly-read item comes from the rank just written
+    // and the other list's rank (that list is not written here), so no slot
+    // of list i is read while other parts may write it.
     bool record_parallel(int i, const int64_t* ids, int64_t n, int T) {
         const int j = 1 - i;
         const bool check = src[i].cursor == nullptr && src[i].sparse == nullptr &&
@@ -480,37 +485,8 @@ class Driver {
         std::vector<uint8_t> bad((size_t)T, 0);
         std::vector<std::vector<Node>> tops((size_t)T);
         std::vector<int64_t> doubly((size_t)T, 0);
-        auto part = [&](int t, int64_t* lo, int64_t* hi) {
-            *lo = n * t / T;
-            *hi = n * (t + 1) / T;
-        };
-        auto phase1 = [&](int t) {
-            int64_t lo, hi;
-            part(t, &lo, &hi);
-            for (int64_t k = lo; k < hi; ++k) {
-                if (k + 16 < hi) {
-                    const int64_t y = ids[k + 16];
-                    if (y >= 0 && y < id_space) __builtin_prefetch(ranks + 2 * y, 1, 0);
-                }
-                const int64_t x64 = ids[k];
-                if (check && (x64 < 0 || x64 >= id_space || (snap && !snap->is_visible(x64)))) {
-                    bad[(size_t)t] = 1;
-                    return;
-                }
-                // host lists may repeat an id across parts: relaxed atomics
-                // keep those accesses defined (plain loads and stores)
-                int32_t* slot = ranks + 2 * x64 + i;
-                if (check && __atomic_load_n(slot, __ATOMIC_RELAXED)) {
-                    bad[(size_t)t] = 1;
-                    return;
-                }
-                __atomic_store_n(slot, (int32_t)(d0 + k + 1), __ATOMIC_RELAXED);
-                pre.p[base + (size_t)k] = (int32_t)x64;
-            }
-        };
-        auto phase2 = [&](int t) {
-            int64_t lo, hi;
-            part(t, &lo, &hi);
+        auto part = [&](int t) {
+            const int64_t lo = n * t / T, hi = n * (t + 1) / T;
             // thread-local until the end: neighbouring threads' counters and
             // vectors would share cache lines
             TopStream top;
@@ -518,64 +494,55 @@ class Driver {
             top.buf.reserve(TopStream::kCut);
             int64_t count = 0;
             for (int64_t k = lo; k < hi; ++k) {
-                if (k + 16 < hi) __builtin_prefetch(ranks + 2 * (size_t)pre[base + (size_t)k + 16], 0, 0);
-                const int32_t x = pre[base + (size_t)k];
-                if (check && rank(i, x) != (int32_t)(d0 + k + 1)) {
-                    bad[(size_t)t] = 1;
-                    return;
+                if (k + 16 < hi) {
+                    const int64_t y = ids[k + 16];
+                    if (y >= 0 && y < id_space) __builtin_prefetch(ranks + 2 * y, 1, 0);
                 }
-                if (rank(j, x)) {
+                const int64_t x64 = ids[k];
+                const int32_t r = (int32_t)(d0 + k + 1);
+                if (check) {
+                    if (x64 < 0 || x64 >= id_space || (snap && !snap->is_visible(x64))) {
+                        bad[(size_t)t] = 1;
+                        break;
+                    }
+                    pre.p[base + (size_t)k] = (int32_t)x64;   // recorded before the write
+                    if (__atomic_exchange_n(ranks + 2 * x64 + i, r, __ATOMIC_RELAXED) != 0) {
+                        bad[(size_t)t] = 1;
+                        break;
+                    }
+                } else {
+                    ranks[2 * (size_t)x64 + (size_t)i] = r;
+                    pre.p[base + (size_t)k] = (int32_t)x64;
+                }
+                const int32_t x = (int32_t)x64;
+                const int32_t rj = rank(j, x);
+                if (rj) {
                     ++count;
-                    if (!inA(x)) top.push(Node{L(x), x});
+                    if (!inA(x)) {
+                        Frac f;
+                        if (active[i]) f = add(f, g[i].at(r));
+                        if (active[j]) f = add(f, g[j].at(rj));
+                        top.push(Node{f, x});
+                    }
                 }
             }
             top.cut();
             doubly[(size_t)t] = count;
             tops[(size_t)t] = std::move(top.buf);
         };
-        // a cursor's ids never repeat: one pass per part writes the ranks and
-        // collects the doubly-read items (the other list is not written here)
-        auto single = [&](int t) {
-            int64_t lo, hi;
-            part(t, &lo, &hi);
-            TopStream top;
-            top.cap = both.cap;
-            top.buf.reserve(TopStream::kCut);
-            int64_t count = 0;
-            for (int64_t k = lo; k < hi; ++k) {
-                if (k + 16 < hi) __builtin_prefetch(ranks + 2 * ids[k + 16], 1, 0);
-                const int32_t x = (int32_t)ids[k];
-                ranks[2 * (size_t)x + (size_t)i] = (int32_t)(d0 + k + 1);
-                pre.p[base + (size_t)k] = x;
-                if (rank(j, x)) {
-                    ++count;
-                    if (!inA(x)) top.push(Node{L(x), x});
-                }
-            }
-            top.cut();
-            doubly[(size_t)t] = count;
-            tops[(size_t)t] = std::move(top.buf);
-        };
-        for (int phase = check ? 0 : 2; phase < (check ? 2 : 3); ++phase) {
-            auto run = [&](int t) {
-                if (phase == 0) phase1(t);
-                else if (phase == 1) phase2(t);
-                else single(t);
-            };
-            // parts whose thread could not be started run here, after part 0
-            std::vector<std::thread> th;
-            int started = 1;
-            try {
-                th.reserve((size_t)T - 1);
-                for (; started < T; ++started) th.emplace_back(run, started);
-            } catch (...) {
-            }
-            run(0);
-            for (int t = started; t < T; ++t) run(t);
-            for (auto& x : th) x.join();
-            for (uint8_t b : bad)
-                if (b) return false;
+        // parts whose thread could not be started run here, after part 0
+        std::vector<std::thread> th;
+        int started = 1;
+        try {
+            th.reserve((size_t)T - 1);
+            for (; started < T; ++started) th.emplace_back(part, started);
+        } catch (...) {
         }
+        part(0);
+        for (int t = started; t < T; ++t) part(t);
+        for (auto& x : th) x.join();
+        for (uint8_t b : bad)
+            if (b) return false;
         for (const std::vector<Node>& top : tops)
             for (const Node& nd : top) both.insert(nd);
         for (int64_t c : doubly) both_read += c;
