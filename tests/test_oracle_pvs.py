@@ -147,6 +147,41 @@ def test_gamma_is_smallest_f32_above_a_over_one_minus_a():
         assert F(float(np.nextafter(g, np.float32(0)))) < target
 
 
+def _qhat_queries():
+    rng = np.random.default_rng(31)
+    out = [rng.standard_normal(m).astype(np.float32) for m in (1, 7, 128, 768)]
+    out.append((rng.standard_normal(96) * 1e30).astype(np.float32))
+    # subnormal scale: max |q_j| / 127 lies below the smallest normal float32
+    out.append((rng.standard_normal(64) * 1e-40).astype(np.float32))
+    # one dominant entry and one that quantizes far from its value:
+    # ||q_hat|| exceeds ||q|| by ~2e-5 relative (below)
+    out.append(np.array([1.0, 0.004], np.float32))
+    return out
+
+
+@pytest.mark.parametrize("k", range(len(_qhat_queries())))
+def test_query_encoding_bounds_the_norm_of_the_dequantized_query(k):
+    """Sec. 2.3.1: q_hat = s_q z_q, and E needs ||q_hat||_2; App. A.1 wants it
+    rounded up.  The stored bound must satisfy, in exact rationals,
+    ||s_q z_q|| <= qhat <= (1 + 2^-20) ||s_q z_q|| (+ one subnormal step where
+    the bound itself is subnormal).  Neither ||z_q|| (s_q dropped) nor ||q||
+    (the query before quantization) passes this on the cases below."""
+    q = _qhat_queries()[k]
+    qe = po.encode_query(q)
+    Q = po.quantize(q.reshape(1, -1))
+    assert qe.status == 0
+    assert np.array_equal(qe.z, Q.z[0]) and qe.s == Q.s[0]
+    n2 = sum(((F(float(qe.s)) * int(z)) ** 2 for z in qe.z.tolist()), F(0))
+    qh = F(float(qe.qhat))
+    assert qh * qh >= n2                                     # an upper bound
+    slack = qh - F(2.0 ** -149) if qh < F(2.0 ** -126) else qh
+    assert slack * slack <= (1 + F(1, 2 ** 20)) ** 2 * n2   # and a tight one
+    if k == len(_qhat_queries()) - 1:
+        # this case separates ||q_hat|| from ||q|| by more than the tolerance
+        qn2 = sum((F(float(x)) ** 2 for x in q.tolist()), F(0))
+        assert qn2 * (1 + F(1, 2 ** 19)) < n2
+
+
 # --------------------------------------------------------------------------
 # intervals (Sec. 2.3.1 + App. A.1)
 # --------------------------------------------------------------------------
