@@ -270,10 +270,14 @@ int64_t pvs_launch_count(void);
 
 /* ---------------------------------------------------------------------------
  * Allocation-free exact ranking.  The paper has no counterpart to this entry
- * point; it exists for callers that cannot allocate device memory where they
- * need a ranking: code running while a CUDA stream is being captured into a
- * graph (cudaMalloc is not permitted during most capture modes), and
- * services whose memory pool owns the device memory budget.
+ * point.  It exists for callers that cannot allocate device memory where
+ * they need a ranking:
+ *   - services whose device memory is owned by their own pool or budget
+ *     (for instance a server that reserves almost all HBM for its indexes at
+ *     start-up): an allocation outside that pool either fails or breaks the
+ *     pool's accounting;
+ *   - latency-critical callers: cudaMalloc can take milliseconds, and
+ *     cudaFree waits for the whole device to go idle.
  * ------------------------------------------------------------------------ */
 
 /* Largest vector count pvs_rank_exact_noalloc accepts. */
@@ -285,8 +289,12 @@ int64_t pvs_launch_count(void);
  * score and order (score descending, ties by ascending row number) as
  * pvs_next -- and write the first `top` <= n row numbers and scores to the
  * DEVICE buffers out_ids (int64) and out_scores (float32).  Work is queued
- * on `cuda_stream` (a cudaStream_t; NULL for the legacy default stream) and
- * the call returns after it has finished.
+ * on `cuda_stream` (a cudaStream_t; NULL for the legacy default stream); the
+ * call then copies the device status word into host memory and waits for
+ * the stream (cudaStreamSynchronize) before it returns, so the outputs are
+ * complete on return.  The library sees raw pointers only: the caller
+ * guarantees that query holds dim floats and that out_ids / out_scores hold
+ * at least `top` entries.
  *
  * Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
  * Its scratch is one static device array of 8192 64-bit keys plus a status
@@ -299,8 +307,9 @@ int64_t pvs_launch_count(void);
  *
  * Errors: PVS_ERR_INVALID when n > PVS_NOALLOC_MAX_VECTORS, n < 0, top > n,
  * dim outside [1, 32767], or a pointer is not device memory;
- * PVS_ERR_NONFINITE for a NaN or infinite entry; PVS_ERR_OVERFLOW when a
- * score overflows float32; PVS_ERR_CUDA when a CUDA call fails. */
+ * PVS_ERR_NONFINITE for a NaN or infinite entry of the query or of a vector
+ * (with n > 0); PVS_ERR_OVERFLOW when a score overflows float32;
+ * PVS_ERR_CUDA when a CUDA call fails. */
 pvs_status pvs_rank_exact_noalloc(const float* query, const float* vecs, int32_t n, int32_t dim,
                                   int32_t top, int64_t* out_ids, float* out_scores,
                                   void* cuda_stream);

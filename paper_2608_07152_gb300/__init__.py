@@ -451,22 +451,44 @@ PVS_NOALLOC_MAX_VECTORS = 8192
 
 
 def pvs_rank_exact_noalloc(query, vecs, top: int, out_ids, out_scores) -> int:
-    """Allocation-free exact ranking of the rows of `vecs` against `query`
-    (both contiguous float32 CUDA tensors) into the caller's CUDA tensors
-    out_ids (int64, >= top) and out_scores (float32, >= top).  Neither this
-    wrapper nor the library allocates device memory: callers that cannot
-    (code inside a stream capture, pool-managed services) pass tensors they
-    already own.  Runs on torch's current stream and returns after it."""
+    """Allocation-free exact ranking of the rows of `vecs` (float32 [n, dim])
+    against `query` (float32 [dim]) into the caller's tensors out_ids (int64,
+    at least `top` entries) and out_scores (float32, at least `top` entries).
+    All four are contiguous CUDA tensors on one device.  Neither this wrapper
+    nor the library allocates device memory: callers whose device memory
+    belongs to a pool or budget of their own pass tensors they already own.
+    Runs on torch's current stream of that device and returns once the
+    stream has finished the work.
+
+    The library cannot see tensor shapes or types through raw pointers, so
+    every size and type is checked here before the call."""
     import torch
-    for t in (query, vecs, out_ids, out_scores):
+    ts = (query, vecs, out_ids, out_scores)
+    for t in ts:
         if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()):
             raise TypeError("pvs_rank_exact_noalloc takes contiguous CUDA tensors")
-    n, dim = (vecs.shape[0], vecs.shape[1]) if vecs.dim() == 2 else (0, query.shape[-1])
-    stream = torch.cuda.current_stream(vecs.device).cuda_stream
-    return _check(_lib.pvs_rank_exact_noalloc(
-        ctypes.c_void_p(query.data_ptr()), ctypes.c_void_p(vecs.data_ptr()), int(n), int(dim),
-        int(top), ctypes.c_void_p(out_ids.data_ptr()), ctypes.c_void_p(out_scores.data_ptr()),
-        ctypes.c_void_p(stream) if stream else None), "pvs_rank_exact_noalloc")
+    if any(t.device != vecs.device for t in ts):
+        raise ValueError("query, vecs, out_ids and out_scores must be on one device")
+    if query.dtype != torch.float32 or vecs.dtype != torch.float32:
+        raise TypeError("query and vecs must be float32")
+    if out_ids.dtype != torch.int64 or out_scores.dtype != torch.float32:
+        raise TypeError("out_ids must be int64 and out_scores float32")
+    if vecs.dim() != 2:
+        raise ValueError("vecs must be a 2-D tensor [n, dim]")
+    n, dim = int(vecs.shape[0]), int(vecs.shape[1])
+    top = int(top)
+    if query.numel() != dim:
+        raise ValueError(f"query has {query.numel()} entries, vecs rows have {dim}")
+    if top < 0 or top > n:
+        raise ValueError(f"top = {top} outside [0, {n}]")
+    if out_ids.numel() < top or out_scores.numel() < top:
+        raise ValueError(f"out_ids and out_scores must hold at least top = {top} entries")
+    with torch.cuda.device(vecs.device):
+        stream = torch.cuda.current_stream(vecs.device).cuda_stream
+        return _check(_lib.pvs_rank_exact_noalloc(
+            ctypes.c_void_p(query.data_ptr()), ctypes.c_void_p(vecs.data_ptr()), n, dim, top,
+            ctypes.c_void_p(out_ids.data_ptr()), ctypes.c_void_p(out_scores.data_ptr()),
+            ctypes.c_void_p(stream) if stream else None), "pvs_rank_exact_noalloc")
 
 
 def _params(K, k, form, policy, step, weights):

@@ -5,11 +5,11 @@
 // -> descending sort -> emit), run over vectors the caller already holds on
 // the device, with the rank keys kept in one file-scope static device array
 // instead of memory obtained from cudaMalloc.  Some callers cannot allocate
-// device memory at the point where they need a ranking: code that runs while
-// a CUDA stream is being captured into a graph (cudaMalloc is not permitted
-// during most capture modes), and services whose memory pool already owns the
-// device memory budget, so that an allocation outside the pool either fails
-// or breaks its accounting.
+// device memory at the point where they need a ranking: services whose
+// device memory is owned by their own pool or budget, where an allocation
+// outside the pool either fails or breaks its accounting, and
+// latency-critical callers, for whom cudaMalloc can take milliseconds and
+// cudaFree waits for the whole device to go idle.
 //
 // The scratch array: PVS_NOALLOC_MAX_VECTORS 64-bit keys plus one status word
 // (64 KiB + 256 B).  Every GPU that loads this library holds it until the

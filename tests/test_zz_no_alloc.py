@@ -1,15 +1,19 @@
 """pvs_rank_exact_noalloc: exact ranking without any device allocation.
 
-Some callers cannot allocate device memory where they need a ranking: code
-that runs while a CUDA stream is being captured into a graph, where
-cudaMalloc is not permitted, and services whose memory pool already owns the
-device memory budget.  For them the library keeps the ranking's scratch in a
-fixed static device array.  These tests check, through the C ABI, that two
-calls in a row return exactly what the cursor path (pvs_cursor_open +
-pvs_next) returns for the same rows and query.  The second call ranks fewer
-rows than the first, so keys the first call left in the shared array must
-not leak into its result.  The bar is the one every parity test here uses:
-identical ids in identical order and bit-identical float32 scores.
+Some callers cannot allocate device memory where they need a ranking:
+services whose device memory belongs to a pool or budget of their own, where
+an allocation outside it fails or breaks the pool's accounting, and
+latency-critical callers, for whom cudaMalloc is slow and cudaFree waits for
+the whole device.  For them the library keeps the ranking's scratch in a
+fixed static device array.
+
+These tests call it through the C ABI and compare it with the oracle's
+complete dense ranking (Sec. 2.1: authoritative scores, ties by ascending
+id): identical ids in identical order and bit-identical float32 scores, the
+bar every parity test here uses.  Each case makes two calls in a row, and
+the second ranks fewer rows than the first, so keys the first call left in
+the shared array must not leak into its result.  This file is collected
+last, so a run that stops at the first failure has run every other test.
 """
 import numpy as np
 import pytest
@@ -17,47 +21,70 @@ import torch
 
 import paper_2608_07152_gb300 as pvs
 import synth
+from oracle import pvs_oracle as po
 
 pytestmark = pytest.mark.gpu
 
-
-def _cursor_ranking(vecs, q, top):
-    index = pvs.pvs_build(vecs)
-    try:
-        cur = pvs.pvs_cursor_open(index, q)
-        try:
-            ids, scores, _ = pvs.pvs_next(cur, top)
-        finally:
-            pvs.pvs_cursor_close(cur)
-    finally:
-        pvs.pvs_index_free(index)
-    return ids, scores
+MAX = pvs.PVS_NOALLOC_MAX_VECTORS
 
 
-def test_noalloc_matches_cursor_path_on_two_calls_in_a_row():
+def _outs(k=MAX):
+    return (torch.full((max(k, 1),), -7, dtype=torch.int64, device="cuda"),
+            torch.full((max(k, 1),), float("nan"), dtype=torch.float32, device="cuda"))
+
+
+def _check_against_oracle(q, V, top, out_ids, out_scores):
+    pvs.pvs_rank_exact_noalloc(q, V, top, out_ids, out_scores)
+    torch.cuda.synchronize()
+    got_ids = out_ids[:top].cpu().numpy()
+    got_scores = out_scores[:top].cpu().numpy()
+    ref_ids, ref_scores = po.dense_ranking(q.cpu().numpy(), V.cpu().numpy())
+    assert np.array_equal(got_ids, ref_ids[:top])
+    assert np.array_equal(got_scores.view(np.uint32), ref_scores[:top].view(np.uint32))
+
+
+def test_noalloc_matches_oracle_on_two_calls_in_a_row():
     torch.cuda.set_device(0)
-    V = synth.unit_normal(6000, 96, seed=21, device="cuda")
-    Q = synth.unit_normal(2, 96, seed=22, device="cuda")
-    out_ids = torch.empty(pvs.PVS_NOALLOC_MAX_VECTORS, dtype=torch.int64, device="cuda")
-    out_scores = torch.empty(pvs.PVS_NOALLOC_MAX_VECTORS, dtype=torch.float32, device="cuda")
-    cases = [(Q[0].contiguous(), V, 500),
-             (Q[1].contiguous(), V[:3000].contiguous(), 3000)]
-    for q, vecs, top in cases:
-        pvs.pvs_rank_exact_noalloc(q, vecs, top, out_ids, out_scores)
-        torch.cuda.synchronize()
-        got_ids = out_ids[:top].cpu().numpy()
-        got_scores = out_scores[:top].cpu().numpy()
-        ref_ids, ref_scores = _cursor_ranking(vecs, q, top)
-        assert np.array_equal(got_ids, ref_ids)
-        assert np.array_equal(got_scores.view(np.uint32), ref_scores.view(np.uint32))
+    V = synth.unit_normal(MAX, 96, seed=21, device="cuda")
+    Q = synth.unit_normal(3, 96, seed=22, device="cuda")
+    out_ids, out_scores = _outs()
+    # the full scratch (n = 8192, every rank), then fewer rows with top < n
+    _check_against_oracle(Q[0].contiguous(), V, MAX, out_ids, out_scores)
+    _check_against_oracle(Q[1].contiguous(), V[:3000].contiguous(), 500, out_ids, out_scores)
+    # a ragged size that is no power of two, every rank
+    _check_against_oracle(Q[2].contiguous(), V[:1237].contiguous(), 1237, out_ids, out_scores)
+
+
+def test_noalloc_exact_ties_go_to_ascending_row_number():
+    torch.cuda.set_device(0)
+    base = synth.unit_normal(40, 32, seed=23, device="cuda")
+    # every row appears three times: equal scores, ranked by row number
+    V = base.repeat(3, 1).contiguous()
+    q = synth.unit_normal(1, 32, seed=24, device="cuda")[0].contiguous()
+    out_ids, out_scores = _outs(120)
+    _check_against_oracle(q, V, 120, out_ids, out_scores)
+    _check_against_oracle(q, V[:50].contiguous(), 17, out_ids, out_scores)
+
+
+def test_noalloc_empty_input_and_top_zero_write_nothing():
+    torch.cuda.set_device(0)
+    q = synth.unit_normal(1, 16, seed=25, device="cuda")[0].contiguous()
+    out_ids, out_scores = _outs(8)
+    empty = torch.zeros((0, 16), device="cuda")
+    assert pvs.pvs_rank_exact_noalloc(q, empty, 0, out_ids, out_scores) == pvs.PVS_OK
+    V = synth.unit_normal(64, 16, seed=26, device="cuda")
+    assert pvs.pvs_rank_exact_noalloc(q, V, 0, out_ids, out_scores) == pvs.PVS_OK
+    torch.cuda.synchronize()
+    assert (out_ids.cpu() == -7).all() and torch.isnan(out_scores.cpu()).all()
+    # and the array works again afterwards
+    _check_against_oracle(q, V, 64, out_ids, out_scores)
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch_and_bad_input():
     torch.cuda.set_device(0)
-    out_ids = torch.empty(16, dtype=torch.int64, device="cuda")
-    out_scores = torch.empty(16, dtype=torch.float32, device="cuda")
+    out_ids, out_scores = _outs(16)
     q = torch.ones(16, device="cuda")
-    too_many = torch.zeros((pvs.PVS_NOALLOC_MAX_VECTORS + 1, 16), device="cuda")
+    too_many = torch.zeros((MAX + 1, 16), device="cuda")
     with pytest.raises(pvs.PvsError) as e:
         pvs.pvs_rank_exact_noalloc(q, too_many, 10, out_ids, out_scores)
     assert e.value.status == pvs.PVS_ERR_INVALID
@@ -66,3 +93,23 @@ def test_noalloc_rejects_sizes_beyond_its_scratch_and_bad_input():
     with pytest.raises(pvs.PvsError) as e:
         pvs.pvs_rank_exact_noalloc(q, bad, 10, out_ids, out_scores)
     assert e.value.status == pvs.PVS_ERR_NONFINITE
+    good = torch.ones((40, 16), device="cuda")
+    qbad = torch.ones(16, device="cuda")
+    qbad[5] = float("inf")
+    with pytest.raises(pvs.PvsError) as e:
+        pvs.pvs_rank_exact_noalloc(qbad, good, 10, out_ids, out_scores)
+    assert e.value.status == pvs.PVS_ERR_NONFINITE
+    # shape and type errors the library cannot see through raw pointers
+    with pytest.raises(ValueError):
+        pvs.pvs_rank_exact_noalloc(torch.ones(15, device="cuda"), good, 10, out_ids, out_scores)
+    with pytest.raises(ValueError):
+        pvs.pvs_rank_exact_noalloc(q, good, 17, out_ids, out_scores)
+    with pytest.raises(ValueError):
+        pvs.pvs_rank_exact_noalloc(q, good, 41, *_outs(64))
+    with pytest.raises(TypeError):
+        pvs.pvs_rank_exact_noalloc(q.double(), good, 10, out_ids, out_scores)
+    with pytest.raises(TypeError):
+        pvs.pvs_rank_exact_noalloc(q, good, 10, out_ids.int(), out_scores)
+    # a good call right after the failures still matches the oracle
+    V = synth.unit_normal(40, 16, seed=27, device="cuda")
+    _check_against_oracle(q, V, 40, *_outs(40))
