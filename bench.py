@@ -559,7 +559,8 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         rd[order] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
         rs = torch.empty(n, dtype=torch.float64, device=dev)
         rs[sparse_dev] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
-        fused = 1.0 / (EAHR_RRF_K + rd) + 1.0 / (EAHR_RRF_K + rs)
+        # the sparse list is the positive-score support (Sec. 2.1)
+        fused = 1.0 / (EAHR_RRF_K + rd) + torch.where(ss > 0, 1.0 / (EAHR_RRF_K + rs), 0.0)
         top = torch.topk(fused, EAHR_K).indices
         top.cpu()
         return (time.perf_counter() - t) * 1e3
@@ -661,7 +662,8 @@ def build_sparse_index(pvs, synth, torch, n, dev, seed):
 def sparse_complete(torch, n, post, terms, weights, dev):
     """The complete sparse ranking in plain torch (the comparator): every
     query term's postings scattered into a score per item, then a full stable
-    sort; returns the first SPARSE_RANKS ids (host) and the time in ms."""
+    sort; returns the first SPARSE_RANKS ids of the positive-score support
+    (host) and the time in ms."""
     off, docs, imps = post
     torch.cuda.synchronize()
     t = time.perf_counter()
@@ -670,7 +672,8 @@ def sparse_complete(torch, n, post, terms, weights, dev):
         a, b = int(off[term]), int(off[term + 1])
         sc.index_put_((docs[a:b].long(),), imps[a:b] * w, accumulate=True)
     order = torch.argsort(sc, descending=True, stable=True)
-    head = order[:SPARSE_RANKS].cpu()
+    head = order[:SPARSE_RANKS]
+    head = head[sc[head] > 0].cpu()
     return head, (time.perf_counter() - t) * 1e3
 
 
@@ -1112,25 +1115,26 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
             a, b = int(off[term]), int(off[term + 1])
             ss.index_put_((docs[a:b].long(),), imps[a:b] * w, accumulate=True)
         sorder = torch.argsort(ss, descending=True, stable=True)
-        return dorder, sorder
+        return dorder, sorder, ss
 
     def comparator(i):
         torch.cuda.synchronize()
         t = time.perf_counter()
-        dorder, sorder = full_orders(i)
+        dorder, sorder, ss = full_orders(i)
         ar = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
         rd = torch.empty(n, dtype=torch.float64, device=dev)
         rd[dorder] = ar
         rs = torch.empty(n, dtype=torch.float64, device=dev)
         rs[sorder] = ar
-        fused = 1.0 / (EAHR_RRF_K + rd) + 1.0 / (EAHR_RRF_K + rs)
+        # the sparse list is the positive-score support (Sec. 2.1)
+        fused = 1.0 / (EAHR_RRF_K + rd) + torch.where(ss > 0, 1.0 / (EAHR_RRF_K + rs), 0.0)
         torch.topk(fused, EAHR_K).indices.cpu()
         return (time.perf_counter() - t) * 1e3
 
     for w in range(2):
         one(w)
         comparator(w)
-    dorder, sorder = full_orders(2)
+    dorder, sorder, _ = full_orders(2)
     ktau = synth.kendall_tau_sample(dorder.cpu().numpy(), sorder.cpu().numpy(), 200_000, seed=5)
     del dorder, sorder
     if pg:

@@ -4,15 +4,19 @@
  * Method: arXiv 2608.07152, Sec. 2.3.2 (Posting Block-Max) and Appendix A.2
  * (its float32 range bound); the ranked-list contract is Sec. 2.1.
  *
- * PBM produces the complete exact sparse ranking of the items 0 .. N-1
- * under a query: items ordered by the sparse score S(x) = sum_t q_t p_t(x)
- * (descending), ties by ascending id, items without any matching posting at
- * score +0.  It partitions the id space into ranges of `block` consecutive
- * ids, bounds every range by H(R) = sum_t q_t m_t(R) with the block maxima
- * m_t(R), expands ranges in decreasing order of H and publishes a rank once
- * no unexpanded range can hold an item ranked before it.  Ranks come in
- * chunks on demand; the cursor keeps the unexpanded ranges and the scored
- * items between calls.
+ * PBM produces the complete exact sparse ranked list of a query: its
+ * support U_s is the set of items with a positive sparse score
+ * S(x) = sum_t q_t p_t(x) (Sec. 2.1: items outside U_s have no rank and
+ * contribute nothing to fusion), ordered by S descending, ties by ascending
+ * id.  Items with no matching posting, with only zero impacts or zero-weight
+ * terms, or whose float32 score rounds to 0, are not in the list; neither
+ * are items a snapshot deletes (pbm_cursor_open_snapshot).  PBM partitions
+ * the id space into ranges of `block` consecutive ids, bounds every range by
+ * H(R) = sum_t q_t m_t(R) with the block maxima m_t(R), expands the ranges
+ * with H > 0 in decreasing order of H and publishes a rank once no
+ * unexpanded range can hold an item ranked before it.  Ranks come in chunks
+ * on demand; the cursor keeps the unexpanded ranges and the scored items
+ * between calls.
  *
  * Float32 evaluation (App. A.2; readings of this library): both S and H
  * are accumulated term by term in the order the query lists its terms, each
@@ -43,8 +47,9 @@ typedef struct pbm_cursor pbm_cursor;
 
 /* Counters of one PBM cursor (the sparse counters of Sec. 3.5). */
 typedef struct pbm_stats {
-    int64_t items;             /* N                                          */
-    int64_t emitted;           /* ranks delivered so far                     */
+    int64_t items;             /* N, the id space (|U_s| <= N)               */
+    int64_t emitted;           /* ranks delivered so far (= |U_s| once the
+                                  list is Exhausted)                         */
     int64_t ranges;            /* ranges of the id space                     */
     int64_t ranges_expanded;   /* ranges whose items were scored             */
     int64_t postings_visited;  /* postings read while scoring               */
@@ -83,7 +88,7 @@ void pbm_index_free(pbm_index* index);   /* cursors must be closed first */
  * Open a cursor for the query {(terms[i], weights[i])}, i < nq, whose
  * listed order is the summation order sigma (App. A.2).  terms: distinct
  * ids in [0, n_terms); weights: finite, >= 0 (a zero weight contributes
- * nothing).  nq may be 0 (every score is 0: the ranking is id order);
+ * nothing).  nq may be 0 (every score is 0: the ranked list is empty);
  * nq <= 1024.  Host arrays; copied.  The range bounds H(R) are computed
  * here.  Errors: PVS_ERR_INVALID (bad term, repeated term, nq out of
  * range), PVS_ERR_NONFINITE (non-finite weight), PVS_ERR_OOM, PVS_ERR_CUDA.
@@ -92,10 +97,24 @@ pvs_status pbm_cursor_open(pbm_index* index, const int32_t* terms, const float* 
                            int32_t nq, pbm_cursor** out);
 
 /*
+ * pbm_cursor_open over the visible set of a PVS snapshot (Sec. 2.4: every
+ * channel of a request ranks the items of one fixed snapshot): items the
+ * snapshot deletes are outside the ranked list.  The snapshot's rows must
+ * be the PBM index's items (same id space, snapshot rows == n_items) and its
+ * index on the same device; the snapshot may be freed while the cursor is
+ * open.  snap NULL is pbm_cursor_open.  Errors as pbm_cursor_open, and
+ * PVS_ERR_INVALID for a snapshot of another size or device.
+ */
+pvs_status pbm_cursor_open_snapshot(pbm_index* index, const pvs_snapshot* snap,
+                                    const int32_t* terms, const float* weights, int32_t nq,
+                                    pbm_cursor** out);
+
+/*
  * The next up to n ranks (n >= 1): ids (int64) and their scores S_hat
- * (float32) in host memory, *n_out of them.  Returns PVS_OK, or
- * PVS_EXHAUSTED once all N items have been delivered (then *n_out < n, or
- * *n_out == n for the call that delivers the last item).  Output is an
+ * (float32, all > 0) in host memory, *n_out of them.  Returns PVS_OK, or
+ * PVS_EXHAUSTED once the last item of the support has been delivered (then
+ * *n_out < n, or *n_out == n for the call that delivers the last item;
+ * later calls deliver 0).  Output is an
  * append-only exact prefix (Sec. 2.1).  A pull whose certified window (every
  * scored item above the bound of every range not yet expanded, at most 8,192
  * of them) holds more ranks than requested keeps the rest in the cursor's
@@ -119,9 +138,13 @@ void pbm_cursor_close(pbm_cursor* cursor);
 /*
  * EAHR (Sec. 2.2) over a dense PVS cursor and a sparse PBM cursor, both
  * unused so far: the same contract as eahr_topk with the sparse ranks pulled
- * from PBM instead of a host array.  Both must rank the same items: the
- * PBM index holds exactly the dense snapshot's rows and the snapshot has no
- * deleted rows (else PVS_ERR_INVALID).
+ * from PBM instead of a host array.  Both channels must see one visible set
+ * (Sec. 2.4): the PBM index's items are the dense snapshot's rows, and the
+ * PBM cursor deletes what the dense cursor's snapshot deletes (open it with
+ * pbm_cursor_open_snapshot on that snapshot, or with pbm_cursor_open when
+ * nothing is deleted); else PVS_ERR_INVALID.  The sparse support U_s is
+ * usually much smaller than the visible set; items outside it contribute
+ * nothing (Sec. 2.1).
  */
 pvs_status eahr_topk_pbm(pvs_cursor* dense, pbm_cursor* sparse, const eahr_params* p,
                          int64_t* out_ids, double* out_F, int32_t* n_out, eahr_stats* st);

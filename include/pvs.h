@@ -142,6 +142,33 @@ pvs_status pvs_index_export(const pvs_index* index, int64_t first, int64_t count
                             int8_t* codes, float* scale, float* vnorm, float* enorm);
 void pvs_index_free(pvs_index* index);
 
+/* Load an index from data saved earlier (pvs_index_export gives codes,
+ * scales and norm bounds; the caller keeps the raw vectors): n rows of
+ * dimension dim, all HOST buffers -- vecs float32 [n x dim], codes int8
+ * [n x dim], scale / vnorm / enorm float32 [n].  Nothing is re-quantized:
+ * the library checks only what it relies on to stay in bounds (codes in
+ * [-127, 127], finite vectors, finite positive scales, finite nonnegative
+ * norm bounds) and otherwise trusts the parameters.  Parameters that do not
+ * bound a row's score are caught by the failure rule of App. A.1 when that
+ * row is scored exactly: the pull fails with PVS_ERR_INTERVAL and the cursor
+ * is Failed.  `cuda_stream` as in pvs_build.  Errors: PVS_ERR_INVALID,
+ * PVS_ERR_NONFINITE (a non-finite vector entry), PVS_ERR_OOM, PVS_ERR_CUDA. */
+pvs_status pvs_index_import(const float* vecs, const int8_t* codes, const float* scale,
+                            const float* vnorm, const float* enorm, int64_t n, int32_t dim,
+                            void* cuda_stream, pvs_index** out);
+
+/* Device-side time limit, in nanoseconds, of each wait of this index's
+ * interval passes for a tile of codes or a free pipeline stage (default and
+ * maximum 2e9, i.e. 2 s).  A wait that runs out sets PVS_ERR_TIMEOUT: the
+ * pull fails and the cursor is Failed (Sec. 2.1); the GPU context stays
+ * usable and other cursors are unaffected.  0 makes every such wait give up
+ * at once unless its tile has already arrived, which lets tests reach the
+ * timeout rule without a fault.  While the limit is below 2 s, each pass's
+ * status is read on the host before the pull goes on.  The pass's waits for
+ * its own copies in flight always keep the 2 s limit.  Must not overlap
+ * other calls on the index.  Errors: PVS_ERR_INVALID (null index, ns < 0). */
+pvs_status pvs_index_set_wait_limit(pvs_index* index, int64_t ns);
+
 /* Freeze the currently visible set (rows inserted so far minus tombstones).
  * A snapshot may be freed while cursors opened on it are still open. */
 pvs_status pvs_snapshot_create(pvs_index* index, pvs_snapshot** out);

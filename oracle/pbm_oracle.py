@@ -22,8 +22,11 @@ Readings (the paper fixes neither):
         acc <- RN(acc + RN(q_t * p_t(x)))   for t in sigma, acc starting at +0;
   * the ranges are the fixed blocks [r B, (r + 1) B) of the identifier
     space for a block size B;
-  * the sparse ranking covers every item 0 .. N-1: items without a posting of
-    any query term have score +0 and follow all others in ascending id.
+  * the sparse ranking's support is U_s = {x : S_hat(x) > 0} (Sec. 2.1: the
+    sparse retriever ranks the items with positive query scores; items
+    outside U_s have no rank and contribute nothing to fusion).  An item
+    with no posting of a query term, with only zero impacts or zero-weight
+    terms, or whose float32 products all round to zero, is outside U_s.
 
 Postings are term-major (CSR): the postings of term t are entries
 term_off[t] .. term_off[t+1]-1 of (docs, imps), docs strictly ascending.
@@ -86,12 +89,13 @@ def sparse_scores(q_terms, q_weights, term_off, docs, imps, n_items: int) -> np.
 
 
 def sparse_ranking(q_terms, q_weights, term_off, docs, imps, n_items: int):
-    """The complete sparse ranking (Sec. 2.1): every item id ordered by
-    (S_hat desc, id asc); returns (ids int64, scores float32)."""
+    """The complete sparse ranked list (Sec. 2.1): the support U_s = {x :
+    S_hat(x) > 0} ordered by (S_hat desc, id asc); returns (ids int64,
+    scores float32), both of length |U_s|."""
     S = sparse_scores(q_terms, q_weights, term_off, docs, imps, n_items)
-    ids = np.arange(n_items, dtype=np.int64)
-    order = np.lexsort((ids, -S.astype(np.float64)))
-    return order.astype(np.int64), S[order]
+    ids = np.nonzero(S > 0)[0].astype(np.int64)
+    order = np.lexsort((ids, -S[ids].astype(np.float64)))
+    return ids[order], S[ids[order]]
 
 
 def block_maxima(term_off, docs, imps, n_items: int, block: int):

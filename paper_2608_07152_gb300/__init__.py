@@ -136,6 +136,8 @@ def _load() -> ctypes.CDLL:
         "pvs_status_string": (ctypes.c_char_p, [i32]),
         "pvs_launch_count": (i64, []),
         "pvs_rank_exact_noalloc": (i32, [P, P, i32, i32, i32, P, P, P]),
+        "pvs_index_import": (i32, [P, P, P, P, P, i64, i32, P, pp]),
+        "pvs_index_set_wait_limit": (i32, [P, i64]),
         "eahr_topk": (i32, [P, P, i64, ctypes.POINTER(eahr_params), P, P, P,
                             ctypes.POINTER(eahr_stats)]),
         "eahr_topk_lists": (i32, [P, i64, P, i64, ctypes.POINTER(eahr_params), P, P, P,
@@ -145,6 +147,7 @@ def _load() -> ctypes.CDLL:
         "pbm_index_ranges": (i64, [P]),
         "pbm_index_free": (None, [P]),
         "pbm_cursor_open": (i32, [P, P, P, i32, pp]),
+        "pbm_cursor_open_snapshot": (i32, [P, P, P, P, i32, pp]),
         "pbm_next": (i32, [P, i32, P, P, P]),
         "pbm_cursor_range_bounds": (i32, [P, i64, i64, P]),
         "pbm_cursor_stats": (i32, [P, ctypes.POINTER(pbm_stats)]),
@@ -178,9 +181,10 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pvs_cursor_set_stream", "pvs_next_batch", "pvs_batch_bounds",
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_cursor_sync_batch", "pvs_cursor_stats_batch", "pvs_cursor_close_batch",
-            "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc", "eahr_topk",
+            "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc",
+            "pvs_index_import", "pvs_index_set_wait_limit", "eahr_topk",
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
-            "pbm_index_free", "pbm_cursor_open", "pbm_next", "pbm_cursor_range_bounds",
+            "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
             "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge",
             "pvs_executor_create", "pvs_executor_run", "pvs_executor_stats_get",
@@ -271,6 +275,28 @@ def pvs_index_export(index, first: int, count: int):
     _check(_lib.pvs_index_export(index, first, count, codes.ctypes.data, scale.ctypes.data,
                                  vnorm.ctypes.data, enorm.ctypes.data), "pvs_index_export")
     return codes, scale, vnorm, enorm
+
+
+def pvs_index_import(vecs, codes, scale, vnorm, enorm, stream=None):
+    """Index from saved parameters (host arrays): vecs float32 [n, dim],
+    codes int8 [n, dim], scale / vnorm / enorm float32 [n].  Nothing is
+    re-quantized; a parameter that does not bound its row's score fails the
+    pull that scores the row (App. A.1 failure rule)."""
+    v = np.ascontiguousarray(vecs, dtype=np.float32)
+    z = np.ascontiguousarray(codes, dtype=np.int8)
+    s, vn, en = (np.ascontiguousarray(a, dtype=np.float32) for a in (scale, vnorm, enorm))
+    n, dim = v.shape
+    if z.shape != (n, dim) or s.shape != (n,) or vn.shape != (n,) or en.shape != (n,):
+        raise ValueError("codes [n, dim] and scale / vnorm / enorm [n] must match vecs")
+    out = ctypes.c_void_p()
+    _check(_lib.pvs_index_import(v.ctypes.data, z.ctypes.data, s.ctypes.data, vn.ctypes.data,
+                                 en.ctypes.data, n, dim, stream, ctypes.byref(out)),
+           "pvs_index_import")
+    return out
+
+
+def pvs_index_set_wait_limit(index, ns: int) -> None:
+    _check(_lib.pvs_index_set_wait_limit(index, int(ns)), "pvs_index_set_wait_limit")
 
 
 def pvs_index_free(index) -> None:
@@ -588,14 +614,20 @@ def pbm_index_free(index) -> None:
     _lib.pbm_index_free(index)
 
 
-def pbm_cursor_open(index, terms, weights):
+def pbm_cursor_open(index, terms, weights, snap=None):
+    """PBM cursor for the query (terms, weights); with `snap` (a PVS snapshot
+    of the same id space) the items it deletes are left out of the ranking."""
     t = np.ascontiguousarray(terms, dtype=np.int32)
     w = np.ascontiguousarray(weights, dtype=np.float32)
     if t.shape != w.shape:
         raise ValueError("one weight per query term")
     out = ctypes.c_void_p()
-    _check(_lib.pbm_cursor_open(index, t.ctypes.data, w.ctypes.data, t.size, ctypes.byref(out)),
-           "pbm_cursor_open")
+    if snap is None:
+        _check(_lib.pbm_cursor_open(index, t.ctypes.data, w.ctypes.data, t.size,
+                                    ctypes.byref(out)), "pbm_cursor_open")
+    else:
+        _check(_lib.pbm_cursor_open_snapshot(index, snap, t.ctypes.data, w.ctypes.data, t.size,
+                                             ctypes.byref(out)), "pbm_cursor_open_snapshot")
     return out
 
 

@@ -40,11 +40,12 @@
 #include "../../include/pvs.h"
 #include "runtime.h"
 
-// facts about merge cursors (merge.cu)
+// facts about merge cursors (merge.cu) and PBM cursors (pbm_capi.cu)
 namespace pvs {
 int64_t merge_id_space(const pvs_merge* m);
 int64_t merge_length(const pvs_merge* m);
 bool merge_fresh(const pvs_merge* m);
+const SnapData* pbm_cursor_snapshot(const pbm_cursor* c);
 }  // namespace pvs
 
 namespace {
@@ -635,7 +636,9 @@ class Driver {
         return true;
     }
 
-    // Pull up to n ranks from list i.
+    // Pull up to n ranks from list i.  A producer's list length is only an
+    // upper bound until it reports Exhausted (a sparse support U_s is known
+    // only then); from then on it is the depth read.
     pvs_status pull(int i, int64_t n) {
         if (exhausted[i] || !active[i]) return PVS_OK;
         pulls[i]++;
@@ -675,9 +678,20 @@ class Driver {
             if (depth[i] == src[i].length) exhausted[i] = true;
         }
         if (depth[i] >= src[i].length) exhausted[i] = true;
+        if (exhausted[i]) src[i].length = depth[i];
         return PVS_OK;
     }
 };
+
+// Whether two snapshots (null: every row of `rows` visible) have one visible set.
+bool same_visible(const pvs::SnapData* a, const pvs::SnapData* b, int64_t rows) {
+    if (a == b) return true;
+    const bool a_all = !a || a->visible == a->rows;
+    const bool b_all = !b || b->visible == b->rows;
+    if ((a && a->rows != rows) || (b && b->rows != rows)) return false;
+    if (a_all || b_all) return a_all && b_all;
+    return a->h_tomb == b->h_tomb;
+}
 
 bool contrib_from(const eahr_params* p, int i, int64_t max_rank, Contrib* out) {
     const int64_t wn = p->w_num[i], wd = p->w_den[i];
@@ -888,8 +902,9 @@ pvs_status eahr_topk_pbm(pvs_cursor* dense, pbm_cursor* sparse, const eahr_param
     if (pbm_cursor_stats(sparse, &ps) != PVS_OK || ps.emitted != 0 || ps.state < 0)
         return PVS_ERR_INVALID;
     const pvs::SnapData* snap = pvs::cursor_snapshot(dense);
-    // both channels rank the same items: every row of the snapshot, no deletions
-    if (ps.items != snap->rows || snap->visible != snap->rows) return PVS_ERR_INVALID;
+    // both channels rank items of one visible set (Sec. 2.4)
+    if (ps.items != snap->rows || !same_visible(snap, pvs::pbm_cursor_snapshot(sparse), snap->rows))
+        return PVS_ERR_INVALID;
     Driver d;
     d.snap = snap;
     d.src[0].cursor = dense;

@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(kIntervalThreads, 1)
             for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++k) {
                 const int s = k % stages;
                 const uint32_t ph = (uint32_t)(k / stages) & 1u;
-                if (!mbar_wait(&empty[s], ph ^ 1u)) {
+                if (!mbar_wait(&empty[s], ph ^ 1u, a.wait_ns)) {
                     set_status(a.status, PVS_ERR_TIMEOUT);
                     ok = false;
                     break;
@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(kIntervalThreads, 1)
     for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++k) {
         const int s = k % stages;
         const uint32_t ph = (uint32_t)(k / stages) & 1u;
-        if (!mbar_wait(&full[s], ph)) {
+        if (!mbar_wait(&full[s], ph, a.wait_ns)) {
             if (lane == 0) set_status(a.status, PVS_ERR_TIMEOUT);
             break;
         }

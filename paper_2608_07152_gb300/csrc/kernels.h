@@ -12,6 +12,7 @@ void count_launches(int k);
 constexpr int kTileRows = 64;         // rows per interval-pass tile
 constexpr int kCodeAlign = 64;        // code rows padded to a multiple of 64 bytes
 constexpr int kMaxDim = 32767;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s device-side wait limit
 
 // Encoded query scalars (Sec. 2.3.1, App. A.1).
 struct QueryScalars {
@@ -166,6 +167,10 @@ struct IntervalArgs {
     // the staged pass (slot = CTA x row position in a tile; each row belongs
     // to one slot), kSlotTop per slot, -inf where a slot had fewer live rows
     float* slot_top = nullptr;
+    // limit of each wait for a tile or a free stage (device ns; 0: never
+    // wait).  Waits for the pass's own copies in flight before it exits keep
+    // the full 2 s limit whatever this is, so no copy outlives the kernel.
+    unsigned long long wait_ns = kWaitLimitNs;
 };
 constexpr int kSlotTop = 4;
 cudaError_t launch_interval_pass(const IntervalArgs& a, int num_sms, cudaStream_t st);

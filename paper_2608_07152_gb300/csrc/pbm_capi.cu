@@ -13,6 +13,14 @@
 // The certified items are then emitted in key order.  The pool is
 // append-only: emission runs in strictly decreasing key order, so the items
 // not yet emitted are exactly the pool keys below the last emitted key.
+//
+// The ranked list is the support U_s = {x : S(x) > 0} (Sec. 2.1), minus the
+// items a snapshot deletes.  A range with H(R) = 0 holds no item of U_s
+// (S <= H), so only the ranges with H > 0 -- a prefix of the sorted order --
+// are ever expanded; zero-score and deleted items of an expanded range enter
+// the pool with key 0, which no window takes.  The list is Exhausted once
+// every range with H > 0 is expanded and the window below the last emitted
+// key has been delivered.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -25,6 +33,7 @@
 #include "kernels.h"
 #include "pbm_kernels.h"
 #include "pvs_common.cuh"
+#include "runtime.h"
 
 namespace {
 
@@ -116,7 +125,10 @@ struct pbm_cursor {
     // every range not expanded when the window was taken, and the window held
     // every scored item above that bound), served without device work
     int64_t ahead_pos = 0, ahead_len = 0;
+    bool ahead_complete = false;      // that window held every remaining rank
     uint64_t last_key = ~0ull;
+    int64_t n_pos = 0;                // ranges with H > 0: the only ones expanded
+    std::shared_ptr<pvs::SnapData> snap;   // visible set (null: every item)
     int64_t next = 0;                 // ranges expanded (a prefix of the sorted order)
     uint64_t E = 64;                  // ranges to expand in the next round
     int64_t emitted = 0, pulls = 0, rounds = 0;
@@ -326,12 +338,17 @@ void pbm_index_free(pbm_index* x) {
     delete x;
 }
 
-pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weights, int32_t nq,
-                           pbm_cursor** out) {
+}  // extern "C"
+
+namespace {
+
+pvs_status open_cursor(pbm_index* x, const std::shared_ptr<pvs::SnapData>& snap,
+                       const int32_t* terms, const float* weights, int32_t nq, pbm_cursor** out) {
     if (!out) return PVS_ERR_INVALID;
     *out = nullptr;
     if (!x || nq < 0 || nq > pvs::kPbmMaxTerms || (nq > 0 && (!terms || !weights)))
         return PVS_ERR_INVALID;
+    if (snap && snap->rows != x->n_items) return PVS_ERR_INVALID;
     DeviceGuard device_guard(x->device);
     std::vector<int32_t> sorted(terms, terms + nq);
     std::sort(sorted.begin(), sorted.end());
@@ -348,6 +365,7 @@ pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weig
     c->index = x;
     c->stream = x->stream;
     c->nq = nq;
+    if (snap && snap->d_tomb) c->snap = snap;   // deletions apply
     auto bail = [&](pvs_status s) {
         free_cursor(c);
         return s;
@@ -379,7 +397,7 @@ pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weig
         pvs::launch_pbm_starts(q, x->blk_off, x->blk_range, x->nchunk, c->starts, st) !=
             cudaSuccess ||
         pvs::launch_pbm_bounds(q, c->starts, x->blk_range, x->blk_max, x->n_ranges, x->nchunk,
-                               c->H, &c->ctr->status, st) != cudaSuccess ||
+                               c->H, &c->ctr->status, &c->ctr->pos_ranges, st) != cudaSuccess ||
         pvs::launch_pbm_range_keys(c->H, x->n_ranges, x->block, c->rkeys, st) != cudaSuccess)
         return bail(PVS_ERR_CUDA);
     // the expansion order: range keys sorted descending (the sort's scratch is
@@ -391,9 +409,33 @@ pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weig
              : pvs::launch_radix_sort_desc(c->rkeys, c->tmp, x->n_ranges, c->sort_scratch, st)) !=
             cudaSuccess)
         return bail(PVS_ERR_CUDA);
-    if (cudaStreamSynchronize(st) != cudaSuccess) return bail(PVS_ERR_CUDA);   // query copies
+    if (cudaMemcpyAsync(c->h_ctr, c->ctr, sizeof(pvs::PbmCounters), cudaMemcpyDeviceToHost,
+                        st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)   // query copies, the count of ranges
+        return bail(PVS_ERR_CUDA);
+    c->n_pos = (int64_t)c->h_ctr->pos_ranges;
     *out = c;
     return PVS_OK;
+}
+
+}  // namespace
+
+namespace pvs {
+const SnapData* pbm_cursor_snapshot(const pbm_cursor* c) { return c->snap.get(); }
+}  // namespace pvs
+
+extern "C" {
+
+pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weights, int32_t nq,
+                           pbm_cursor** out) {
+    return open_cursor(x, nullptr, terms, weights, nq, out);
+}
+
+pvs_status pbm_cursor_open_snapshot(pbm_index* x, const pvs_snapshot* snap, const int32_t* terms,
+                                    const float* weights, int32_t nq, pbm_cursor** out) {
+    if (out) *out = nullptr;
+    if (snap && (!x || !snap->index || snap->index->device != x->device)) return PVS_ERR_INVALID;
+    return open_cursor(x, snap ? snap->data : nullptr, terms, weights, nq, out);
 }
 
 pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
@@ -401,24 +443,28 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     if (!c) return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
     if (n < 1 || !ids || !scores || !n_out) return PVS_ERR_INVALID;
+    if (c->state == PVS_EXHAUSTED) return PVS_EXHAUSTED;
     pbm_index* x = c->index;
     DeviceGuard device_guard(x->device);
-    if (c->emitted == x->n_items) {
-        c->state = PVS_EXHAUSTED;
-        return PVS_EXHAUSTED;
-    }
     cudaStream_t st = c->stream;
     ++c->pulls;
     const uint64_t need = (uint64_t)std::min<int64_t>(n, x->n_items - c->emitted);
-    if ((uint64_t)(c->ahead_len - c->ahead_pos) >= need) {   // certified ranks already here
-        std::memcpy(ids, c->h_ids + c->ahead_pos, need * sizeof(int64_t));
-        std::memcpy(scores, c->h_scores + c->ahead_pos, need * sizeof(float));
-        c->ahead_pos += (int64_t)need;
-        c->last_key = pvs::rank_key(scores[need - 1], (uint32_t)ids[need - 1]);
-        c->emitted += (int64_t)need;
+    if (need == 0) {   // every item was delivered: the support is the whole id space
+        c->state = PVS_EXHAUSTED;
+        return PVS_EXHAUSTED;
+    }
+    const uint64_t avail = (uint64_t)(c->ahead_len - c->ahead_pos);
+    if (need > 0 && (avail >= need || (c->ahead_complete && avail > 0))) {
+        // certified ranks already here (all that remain, when the window was complete)
+        const uint64_t m = std::min(need, avail);
+        std::memcpy(ids, c->h_ids + c->ahead_pos, m * sizeof(int64_t));
+        std::memcpy(scores, c->h_scores + c->ahead_pos, m * sizeof(float));
+        c->ahead_pos += (int64_t)m;
+        c->last_key = pvs::rank_key(scores[m - 1], (uint32_t)ids[m - 1]);
+        c->emitted += (int64_t)m;
         ++c->served_ahead;
-        *n_out = (int32_t)need;
-        if (c->emitted == x->n_items) {
+        *n_out = (int32_t)m;
+        if (c->ahead_complete && c->ahead_pos == c->ahead_len) {
             c->state = PVS_EXHAUSTED;
             return PVS_EXHAUSTED;
         }
@@ -426,32 +472,34 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     }
     // too few: the device gathers them again (they lie below last_key)
     c->ahead_pos = c->ahead_len = 0;
+    c->ahead_complete = false;
     uint64_t E = std::max<uint64_t>(c->E, 2 * ((need + x->block - 1) / x->block));
     uint64_t window = 0;
     uint64_t last = 0;   // size of the last expansion of this pull
-    bool served = false;
+    bool served = false, complete = false;
     for (;;) {
         // the certified window, gathered; a window of at most kPbmFastWindow
-        // keys that covers the pull is sorted and written to pinned memory in
-        // the same step (one synchronisation)
-        cudaError_t e = pvs::launch_pbm_window(c->rkeys, c->next, x->n_ranges, c->pool,
-                                               c->last_key, c->buf, c->buf_cap, c->ctr, st);
+        // keys that covers the pull (or holds every remaining rank) is sorted
+        // and written to pinned memory in the same step (one synchronisation)
+        complete = c->next >= c->n_pos;
+        cudaError_t e = pvs::launch_pbm_window(c->rkeys, c->next, c->n_pos, c->pool, c->last_key,
+                                               c->buf, c->buf_cap, c->ctr, st);
         if (e == cudaSuccess)
-            e = pvs::launch_pbm_finish(c->buf, c->ctr, need, c->h_ids, c->h_scores, c->h_ctr,
-                                       st);
+            e = pvs::launch_pbm_finish(c->buf, c->ctr, need, complete, c->h_ids, c->h_scores,
+                                       c->h_ctr, st);
         if (e == cudaSuccess) e = cudaStreamSynchronize(st);
         if (e != cudaSuccess) return fail(c, cuda_status(e));
         if (c->h_ctr->status != 0) return fail(c, (pvs_status)c->h_ctr->status);
         window = c->h_ctr->collected;
-        if (window >= need && window <= (uint64_t)pvs::kPbmFastWindow) {
+        if (window >= 1 && (window >= need || complete) &&
+            window <= (uint64_t)pvs::kPbmFastWindow) {
             served = true;
             break;
         }
-        const uint64_t unexpanded = (uint64_t)(x->n_ranges - c->next);
-        if (window >= need || unexpanded == 0) break;
-        // expand the next E ranges of the sorted order
+        if (window >= need || complete) break;
+        // expand the next E ranges of the sorted order (ranges with H > 0 only)
         ++c->rounds;
-        const uint64_t k = std::min(E, unexpanded);
+        const uint64_t k = std::min(E, (uint64_t)(c->n_pos - c->next));
         pvs::PbmExpandArgs a{};
         a.ranges = c->rkeys + c->next;
         a.count = (int64_t)k;
@@ -464,6 +512,7 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         a.imps = x->imps;
         a.n_items = x->n_items;
         a.block = x->block;
+        a.tomb = c->snap ? c->snap->d_tomb : nullptr;
         a.pool = c->pool;
         a.ctr = c->ctr;
         e = pvs::launch_pbm_expand(a, (int)std::min<uint64_t>(k, (uint64_t)x->num_sms * 4), st);
@@ -480,6 +529,7 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         std::memcpy(scores, c->h_scores, m * sizeof(float));
         c->ahead_pos = (int64_t)m;
         c->ahead_len = (int64_t)window;
+        c->ahead_complete = complete;
     } else if (m > 0) {
         // large window: the m-th largest key first (or the whole window when
         // it fits the gather buffer), then a device sort of the m keys
@@ -507,7 +557,9 @@ pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32
         c->emitted += (int64_t)m;
     }
     *n_out = (int32_t)m;
-    if (c->emitted == x->n_items) {
+    // with every range of positive bound expanded, the window held every
+    // remaining rank: delivering all of it ends the list
+    if (complete && m == window) {
         c->state = PVS_EXHAUSTED;
         return PVS_EXHAUSTED;
     }

@@ -284,7 +284,8 @@ __global__ void __launch_bounds__(256) pbm_bounds_kernel(PbmQuery q,
                                                          const int32_t* __restrict__ blk_range,
                                                          const float* __restrict__ blk_max,
                                                          int64_t n_ranges, int64_t nchunk,
-                                                         float* H, int* status) {
+                                                         float* H, int* status,
+                                                         unsigned long long* pos_ranges) {
     __shared__ float h[kPbmChunk];
     const int64_t k = blockIdx.x;
     const int64_t r0 = k * kPbmChunk;
@@ -303,20 +304,28 @@ __global__ void __launch_bounds__(256) pbm_bounds_kernel(PbmQuery q,
         }
         __syncthreads();
     }
-    for (int x = threadIdx.x; x < kPbmChunk && r0 + x < n_ranges; x += blockDim.x) {
-        const float v = h[x];
-        if (!isfinite(v)) set_status(status, PVS_ERR_OVERFLOW);
-        H[r0 + x] = v;
+    // kPbmChunk is a multiple of the block size: whole warps run every trip
+    for (int x = threadIdx.x; x < kPbmChunk; x += blockDim.x) {
+        const bool in = r0 + x < n_ranges;
+        const float v = in ? h[x] : 0.0f;
+        if (in) {
+            if (!isfinite(v)) set_status(status, PVS_ERR_OVERFLOW);
+            H[r0 + x] = v;
+        }
+        const unsigned int pos = __ballot_sync(0xffffffffu, in && v > 0.0f);
+        if ((threadIdx.x & 31) == 0 && pos)
+            atomicAdd(pos_ranges, (unsigned long long)__popc(pos));
     }
 }
 
 cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const int32_t* blk_range,
                               const float* blk_max, int64_t n_ranges, int64_t nchunk, float* H,
-                              int* status, cudaStream_t st) {
+                              int* status, unsigned long long* pos_ranges, cudaStream_t st) {
+    static_assert(kPbmChunk % 256 == 0, "whole warps in the bound pass's count");
     if (nchunk <= 0) return cudaSuccess;
     count_launches(1);
     pbm_bounds_kernel<<<(unsigned)nchunk, 256, 0, st>>>(q, starts, blk_range, blk_max, n_ranges,
-                                                        nchunk, H, status);
+                                                        nchunk, H, status, pos_ranges);
     return cudaGetLastError();
 }
 
@@ -384,12 +393,14 @@ constexpr int kFinishThreads = 1024;
 
 __global__ void __launch_bounds__(kFinishThreads) pbm_finish_kernel(const uint64_t* keys_in,
                                                                     const PbmCounters* ctr,
-                                                                    uint64_t need, int64_t* h_ids,
+                                                                    uint64_t need, int complete,
+                                                                    int64_t* h_ids,
                                                                     float* h_scores,
                                                                     PbmCounters* h_mirror) {
     extern __shared__ uint64_t keys[];
     const unsigned long long count = ctr->collected;
-    if (need > 0 && count >= need && count <= (unsigned long long)kPbmFastWindow) {
+    if (need > 0 && count >= 1 && (count >= need || complete) &&
+        count <= (unsigned long long)kPbmFastWindow) {
         int pow2 = 1;
         while ((unsigned long long)pow2 < count) pow2 <<= 1;
         for (int i = threadIdx.x; i < pow2; i += blockDim.x)
@@ -424,21 +435,24 @@ __global__ void __launch_bounds__(kFinishThreads) pbm_finish_kernel(const uint64
 }
 
 cudaError_t launch_pbm_finish(const uint64_t* keys, const PbmCounters* ctr, uint64_t need,
-                              int64_t* h_ids, float* h_scores, PbmCounters* h_mirror,
-                              cudaStream_t st) {
+                              bool complete, int64_t* h_ids, float* h_scores,
+                              PbmCounters* h_mirror, cudaStream_t st) {
     cudaError_t e = raise_smem_limit((const void*)pbm_finish_kernel,
                                      kPbmFastWindow * sizeof(uint64_t));
     if (e != cudaSuccess) return e;
     count_launches(1);
     pbm_finish_kernel<<<1, kFinishThreads, kPbmFastWindow * sizeof(uint64_t), st>>>(
-        keys, ctr, need, h_ids, h_scores, h_mirror);
+        keys, ctr, need, complete ? 1 : 0, h_ids, h_scores, h_mirror);
     return cudaGetLastError();
 }
 
 // One CTA per range at a time: the range's block of every query term
 // (binary search within the term's blocks of the range's chunk), then the
 // postings term by term in query order into the items' float32 scores,
-// then every item of the range goes to the pool with its rank key.
+// then every item of the range goes to the pool with its rank key.  Items
+// outside the support (S = 0, Sec. 2.1: no rank) and deleted items get key 0,
+// which lies below every real key and every window bound, so no window takes
+// them.
 constexpr int kExpandThreads = 256;
 
 __global__ void __launch_bounds__(kExpandThreads) pbm_expand_kernel(PbmExpandArgs a) {
@@ -494,7 +508,10 @@ __global__ void __launch_bounds__(kExpandThreads) pbm_expand_kernel(PbmExpandArg
         for (int x = threadIdx.x; x < cnt; x += blockDim.x) {
             const float v = s[x];
             if (!isfinite(v)) set_status(&a.ctr->status, PVS_ERR_OVERFLOW);
-            a.pool[base + x] = rank_key(v, (uint32_t)(first + x));
+            const int64_t id = first + x;
+            const bool dead =
+                a.tomb != nullptr && ((__ldg(a.tomb + (id >> 5)) >> (id & 31)) & 1u);
+            a.pool[base + x] = (v > 0.0f && !dead) ? rank_key(v, (uint32_t)id) : 0ull;
         }
         __syncthreads();   // s, pb, pe are reused by the next range
     }

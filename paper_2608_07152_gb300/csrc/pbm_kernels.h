@@ -22,6 +22,7 @@ struct PbmCounters {
     unsigned long long postings;
     unsigned long long items;
     unsigned long long collected;        // pool keys gathered for an emission
+    unsigned long long pos_ranges;       // ranges with H > 0 (set at open)
     int status;
     int pad;
 };
@@ -58,10 +59,11 @@ struct PbmQuery {
 // starts[i * (nchunk + 1) + k] = first block of query term i with range >= k * kPbmChunk.
 cudaError_t launch_pbm_starts(const PbmQuery& q, const int64_t* blk_off, const int32_t* blk_range,
                               int64_t nchunk, int64_t* starts, cudaStream_t st);
-// H[r] for every range, term by term in query order.
+// H[r] for every range, term by term in query order; *pos_ranges counts the
+// ranges with H > 0 (only they can hold an item of the support U_s).
 cudaError_t launch_pbm_bounds(const PbmQuery& q, const int64_t* starts, const int32_t* blk_range,
                               const float* blk_max, int64_t n_ranges, int64_t nchunk, float* H,
-                              int* status, cudaStream_t st);
+                              int* status, unsigned long long* pos_ranges, cudaStream_t st);
 
 // ---- pulls ---------------------------------------------------------------------
 // rkeys[r] = key(H[r], r * block): the ranges' competition keys (sorted once,
@@ -74,13 +76,15 @@ cudaError_t launch_pbm_range_keys(const float* H, int64_t n_ranges, int block, u
 cudaError_t launch_pbm_window(const uint64_t* sorted, int64_t next, int64_t n_ranges,
                               const uint64_t* pool, uint64_t hi, uint64_t* out, uint64_t cap,
                               PbmCounters* ctr, cudaStream_t st);
-// One CTA: when need <= ctr->collected <= kPbmFastWindow, sorts the collected
-// keys and writes the first `need` ids / scores to h_ids / h_scores; always
-// copies *ctr to *h_mirror last.  h_* may be pinned host memory.
+// One CTA: when 1 <= ctr->collected <= kPbmFastWindow and either need <=
+// ctr->collected or `complete` (the window holds every remaining rank),
+// sorts the collected keys and writes all of them as ids / scores to h_ids /
+// h_scores; always copies *ctr to *h_mirror last.  h_* may be pinned host
+// memory.
 constexpr int kPbmFastWindow = 8192;
 cudaError_t launch_pbm_finish(const uint64_t* keys, const PbmCounters* ctr, uint64_t need,
-                              int64_t* h_ids, float* h_scores, PbmCounters* h_mirror,
-                              cudaStream_t st);
+                              bool complete, int64_t* h_ids, float* h_scores,
+                              PbmCounters* h_mirror, cudaStream_t st);
 struct PbmExpandArgs {
     const uint64_t* ranges;       // sorted range keys of the ranges to expand
     int64_t count;                // how many
@@ -93,6 +97,7 @@ struct PbmExpandArgs {
     const float* imps;
     int64_t n_items;
     int block;
+    const uint32_t* tomb;         // deleted items (bit per id), null: none
     uint64_t* pool;
     PbmCounters* ctr;
 };

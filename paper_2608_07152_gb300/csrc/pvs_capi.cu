@@ -379,6 +379,7 @@ pvs_status interval_pass(pvs_cursor* c) {
     a.lo = c->lo;
     a.hi = c->hi;
     a.status = c->d_status;
+    a.wait_ns = x->wait_ns;
     // per-slot largest lower bounds, for the first working set (see
     // build_working_set): only when no row is tombstoned and every slot
     // scans at least kSlotTop rows, so that every entry is a live row's bound
@@ -414,6 +415,12 @@ pvs_status interval_pass(pvs_cursor* c) {
     c->ev_pending = true;
     c->interval_passes++;
     c->scanned = true;
+    if (x->wait_ns < kWaitLimitNs) {
+        // a shortened wait limit (pvs_index_set_wait_limit) makes a timed-out
+        // pass likely: its bounds are then incomplete, so its status is read
+        // here, before any later kernel of the pull uses them
+        return check_device_status(c);
+    }
     return PVS_OK;
 }
 
@@ -1023,13 +1030,13 @@ pvs_status pvs_build(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_
     return pvs_build_ex(vecs, n, dim, vecs_on_device, cuda_stream, PVS_QUANT_PER_VECTOR, out);
 }
 
-pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
-                        void* cuda_stream, int32_t quantization, pvs_index** out) {
-    if (!out) return PVS_ERR_INVALID;
-    *out = nullptr;
-    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) || (n > 0 && !vecs) ||
-        (quantization != PVS_QUANT_PER_VECTOR && quantization != PVS_QUANT_GLOBAL))
-        return PVS_ERR_INVALID;
+}  // extern "C"
+
+namespace {
+
+// An empty index for vectors of dimension dim: device, stream, status word
+// and scratch pool (no rows yet).
+pvs_status index_create(int32_t dim, void* cuda_stream, pvs_index** out) {
     pvs_index* x = new (std::nothrow) pvs_index();
     if (!x) return PVS_ERR_OOM;
     auto bail = [&](pvs_status s) {
@@ -1063,6 +1070,28 @@ pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_
         uint64_t keep = UINT64_MAX;
         cudaMemPoolSetAttribute(x->scratch_pool, cudaMemPoolAttrReleaseThreshold, &keep);
     }
+    *out = x;
+    return PVS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_on_device,
+                        void* cuda_stream, int32_t quantization, pvs_index** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) || (n > 0 && !vecs) ||
+        (quantization != PVS_QUANT_PER_VECTOR && quantization != PVS_QUANT_GLOBAL))
+        return PVS_ERR_INVALID;
+    pvs_index* x = nullptr;
+    pvs_status s0 = index_create(dim, cuda_stream, &x);
+    if (s0 != PVS_OK) return s0;
+    auto bail = [&](pvs_status s) {
+        pvs_index_free(x);
+        return s;
+    };
     if (vecs_on_device && n > 0 && !is_device_ptr(vecs)) return bail(PVS_ERR_INVALID);
     if (quantization == PVS_QUANT_GLOBAL) {
         // one scale for the corpus: RN(max |v_j| / 127), from the largest entry
@@ -1096,6 +1125,71 @@ pvs_status pvs_build_ex(const float* vecs, int64_t n, int32_t dim, int32_t vecs_
     s = refresh_norm_maxes(x);
     if (s != PVS_OK) return bail(s);
     *out = x;
+    return PVS_OK;
+}
+
+pvs_status pvs_index_import(const float* vecs, const int8_t* codes, const float* scale,
+                            const float* vnorm, const float* enorm, int64_t n, int32_t dim,
+                            void* cuda_stream, pvs_index** out) {
+    if (!out) return PVS_ERR_INVALID;
+    *out = nullptr;
+    if (dim < 1 || dim > kMaxDim || n < 0 || n >= ((int64_t)1 << 31) ||
+        (n > 0 && (!vecs || !codes || !scale || !vnorm || !enorm)))
+        return PVS_ERR_INVALID;
+    // what the method relies on without recomputing it: codes in [-127, 127]
+    // (the Int8 dot products cannot overflow), finite inputs, positive scales
+    for (int64_t i = 0; i < n; ++i) {
+        if (!(std::isfinite(scale[i]) && scale[i] > 0.0f) || !std::isfinite(vnorm[i]) ||
+            !std::isfinite(enorm[i]) || vnorm[i] < 0.0f || enorm[i] < 0.0f)
+            return PVS_ERR_INVALID;
+        for (int32_t j = 0; j < dim; ++j) {
+            const int8_t z = codes[i * (int64_t)dim + j];
+            if (z < -127) return PVS_ERR_INVALID;
+            if (!std::isfinite(vecs[i * (int64_t)dim + j])) return PVS_ERR_NONFINITE;
+        }
+    }
+    pvs_index* x = nullptr;
+    pvs_status s = index_create(dim, cuda_stream, &x);
+    if (s != PVS_OK) return s;
+    auto bail = [&](pvs_status st) {
+        pvs_index_free(x);
+        return st;
+    };
+    s = index_reserve(x, n);
+    if (s != PVS_OK) return bail(s);
+    cudaStream_t st = x->stream;
+    if (n > 0) {
+        // padded rows: zero bytes and floats beyond dim, as the builder writes them
+        cudaError_t e = cudaMemsetAsync(x->codes, 0, (size_t)n * x->m_pad, st);
+        if (e == cudaSuccess)
+            e = cudaMemsetAsync(x->raw, 0, (size_t)n * x->m_raw * sizeof(float), st);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(x->codes, (size_t)x->m_pad, codes, (size_t)dim, (size_t)dim,
+                                  (size_t)n, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(x->raw, (size_t)x->m_raw * sizeof(float), vecs,
+                                  (size_t)dim * sizeof(float), (size_t)dim * sizeof(float),
+                                  (size_t)n, cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(x->scale, scale, n * sizeof(float), cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(x->vnorm, vnorm, n * sizeof(float), cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(x->enorm, enorm, n * sizeof(float), cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) return bail(cuda_status(e));
+    }
+    x->size = n;
+    x->live = n;
+    s = refresh_norm_maxes(x);
+    if (s != PVS_OK) return bail(s);
+    *out = x;
+    return PVS_OK;
+}
+
+pvs_status pvs_index_set_wait_limit(pvs_index* x, int64_t ns) {
+    if (!x || ns < 0) return PVS_ERR_INVALID;
+    x->wait_ns = (unsigned long long)std::min<int64_t>(ns, (int64_t)kWaitLimitNs);
     return PVS_OK;
 }
 

@@ -14,7 +14,6 @@
 namespace pvs {
 
 constexpr int kWarp = 32;
-constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s device-side wait limit
 
 // ---------------------------------------------------------------------------
 // Ordered 32-bit keys of float32 values: key(a) < key(b) iff a < b, with -0

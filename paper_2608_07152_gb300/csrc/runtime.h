@@ -63,6 +63,8 @@ struct pvs_index {
     // scalar-quantization intervals: one scale for every row (else null)
     int quant = PVS_QUANT_PER_VECTOR;
     float* gscale = nullptr;                // device, one float
+    // device-side wait limit of this index's interval passes (ns; 0: no wait)
+    unsigned long long wait_ns = pvs::kWaitLimitNs;
 };
 
 struct pvs_snapshot {

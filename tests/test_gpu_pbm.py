@@ -1,8 +1,9 @@
 """PBM sparse rank generator through the C ABI against the oracle
-(arXiv 2608.07152 Sec. 2.1, Sec. 2.3.2, App. A.2).
+(arXiv 2608.07152 Sec. 2.1, Sec. 2.3.2, Sec. 2.4, App. A.2).
 
 Every emitted rank and score is compared bit for bit with the oracle's
-complete sparse ranking; the range bounds with the oracle's H_hat(R).
+complete sparse ranked list, whose support U_s is the items with a positive
+score (Sec. 2.1); the range bounds with the oracle's H_hat(R).
 """
 import numpy as np
 import pytest
@@ -40,7 +41,7 @@ def random_postings(rng, n_items, n_terms, max_df, integer=False):
     return csr(n_terms, postings)
 
 
-def pull_all(cur, chunks, n_items):
+def pull_all(cur, chunks, n_support):
     ids, sc = [], []
     k = 0
     while True:
@@ -50,13 +51,17 @@ def pull_all(cur, chunks, n_items):
         ids.append(i)
         sc.append(s)
         if st == pvs.PVS_EXHAUSTED:
-            assert sum(len(x) for x in ids) == n_items
+            assert sum(len(x) for x in ids) == n_support
             break
         assert len(i) == n
+    # an exhausted list stays exhausted and delivers nothing
+    i, s, st = pvs.pbm_next(cur, 5)
+    assert st == pvs.PVS_EXHAUSTED and len(i) == 0
     return np.concatenate(ids), np.concatenate(sc)
 
 
 def check_against_oracle(off, docs, imps, n_items, terms, weights, block, chunks):
+    ref_ids, ref_sc = po.sparse_ranking(terms, weights, off, docs, imps, n_items)
     index = pvs.pbm_build(off, docs, imps, n_items, block=block)
     try:
         cur = pvs.pbm_cursor_open(index, terms, weights)
@@ -65,16 +70,18 @@ def check_against_oracle(off, docs, imps, n_items, terms, weights, block, chunks
             H = pvs.pbm_cursor_range_bounds(cur, 0, nr)
             ref_H = po.range_bounds(terms, weights, off, docs, imps, n_items, block)
             assert np.array_equal(H.view(np.uint32), ref_H.view(np.uint32))
-            ids, sc = pull_all(cur, chunks, n_items)
+            ids, sc = pull_all(cur, chunks, len(ref_ids))
             stats = pvs.pbm_cursor_stats(cur)
         finally:
             pvs.pbm_cursor_close(cur)
     finally:
         pvs.pbm_index_free(index)
-    ref_ids, ref_sc = po.sparse_ranking(terms, weights, off, docs, imps, n_items)
     assert np.array_equal(ids, ref_ids)
     assert np.array_equal(sc.view(np.uint32), ref_sc.view(np.uint32))
-    assert stats["emitted"] == n_items and stats["state"] == pvs.PVS_EXHAUSTED
+    assert stats["emitted"] == len(ref_ids) and stats["state"] == pvs.PVS_EXHAUSTED
+    # only ranges with a positive bound are expanded (S <= H: the others hold
+    # no item of U_s)
+    assert stats["ranges_expanded"] == int(np.count_nonzero(ref_H > 0))
     return stats
 
 
@@ -111,9 +118,17 @@ def test_ties_zero_weights_and_empty_terms():
     terms2 = np.array([3, 11] + empty[:1], np.int32)
     w2 = np.array([0.0, 2.0] + [1.0] * len(empty[:1]), np.float32)
     check_against_oracle(off, docs, imps, n_items, terms2, w2, 64, [100])
-    # no query terms: every score is 0 and the ranking is id order
+    # no query terms, or only zero weights: every score is 0, U_s is empty
     check_against_oracle(off, docs, imps, n_items, np.zeros(0, np.int32),
                          np.zeros(0, np.float32), 16, [999])
+    check_against_oracle(off, docs, imps, n_items, np.array([3, 11], np.int32),
+                         np.zeros(2, np.float32), 16, [1])
+    # every item in U_s: one term posted on every item
+    full = csr(2, {0: [(x, 1.0 + (x % 5)) for x in range(700)], 1: [(3, 2.0)]})
+    check_against_oracle(*full, 700, np.array([0], np.int32), np.ones(1, np.float32), 32,
+                         [700])
+    check_against_oracle(*full, 700, np.array([0], np.int32), np.ones(1, np.float32), 32,
+                         [699, 1, 5])
 
 
 def test_bm25_corpus_deep_pulls_and_large_windows():
@@ -128,7 +143,9 @@ def test_bm25_corpus_deep_pulls_and_large_windows():
                                      [20] * 50 + [70_000, 100_000])
         q_postings = sum(int(off[t + 1] - off[t]) for t in terms)
         assert stats["postings_visited"] == q_postings      # every posting once, at the end
-        assert stats["items_scored"] == n_items
+        H = po.range_bounds(terms, weights, off, docs, imps, n_items, 128)
+        sizes = np.minimum(128, n_items - 128 * np.arange(H.size))
+        assert stats["items_scored"] == int(sizes[H > 0].sum())
         # pulls of 20 inside an earlier pull's certified window need no device work
         assert stats["pulls_from_window"] > 0
 
@@ -187,7 +204,8 @@ def test_invalid_inputs_fail_loudly():
             with pytest.raises(pvs.PvsError):
                 pvs.pbm_next(cur, 0)
             i, s, st = pvs.pbm_next(cur, 10)
-            assert st == pvs.PVS_EXHAUSTED and i.tolist() == [3, 1, 0, 2]
+            # item 2 has no posting: score 0, outside U_s
+            assert st == pvs.PVS_EXHAUSTED and i.tolist() == [3, 1, 0]
             i, s, st = pvs.pbm_next(cur, 10)
             assert st == pvs.PVS_EXHAUSTED and len(i) == 0
         finally:
@@ -225,3 +243,115 @@ def test_eahr_with_pbm_matches_complete_list_fusion(tau_terms):
     for (x, f), got in zip(T, F):
         if not np.isnan(got):
             assert got == ro.as_float(f)
+
+
+def _eahr_pbm(V, q, off, docs, imps, n, terms, weights, snap_ids=None):
+    """eahr_topk_pbm over a fresh PVS index of V and PBM index of the postings;
+    snap_ids: ids to delete in a snapshot that both cursors see."""
+    dindex = pvs.pvs_build(V)
+    sindex = pvs.pbm_build(off, docs, imps, n)
+    snap = None
+    try:
+        if snap_ids is not None:
+            pvs.pvs_tombstone(dindex, snap_ids)
+            snap = pvs.pvs_snapshot_create(dindex)
+        dcur = pvs.pvs_cursor_open(dindex, q, snap=snap)
+        scur = pvs.pbm_cursor_open(sindex, terms, weights, snap=snap)
+        try:
+            return pvs.eahr_topk_pbm(dcur, scur, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+        finally:
+            pvs.pbm_cursor_close(scur)
+            pvs.pvs_cursor_close(dcur)
+    finally:
+        if snap is not None:
+            pvs.pvs_snapshot_free(snap)
+        pvs.pbm_index_free(sindex)
+        pvs.pvs_index_free(dindex)
+
+
+def test_eahr_over_the_positive_score_support_differs_from_ranking_every_item():
+    """Sec. 2.1: the sparse channel ranks only U_s = {S > 0}; an item outside
+    it contributes nothing.  With BM25 queries of 1-3 terms U_s is a small
+    part of the corpus, and ranking every item (zero scores last, by id)
+    would hand each zero-score item a spurious 1 / (60 + r): the two targets
+    differ, and EAHR must return the one over U_s."""
+    n, m = 40_000, 64
+    V = synth.unit_normal(n, m, seed=51).numpy()
+    Q = synth.unit_normal(6, m, seed=52).numpy()
+    off, docs, imps = synth.bm25_postings(n, 8_000, 25.0, seed=53)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    queries = synth.sparse_queries(6, torch.from_numpy(off), seed=54, mean_terms=1.0)
+    differ = 0
+    for qi, (terms, weights) in enumerate(queries):
+        terms, weights = terms[:3], weights[:3]
+        dense_ids, _ = pvo.dense_ranking(Q[qi], V)
+        sparse_ids, _ = po.sparse_ranking(terms, weights, off, docs, imps, n)
+        assert 0 < sparse_ids.size < n // 4
+        T = ro.target_topk_large([dense_ids, sparse_ids], [1, 1], 60, 20, ro.NUMERATOR)
+        S = po.sparse_scores(terms, weights, off, docs, imps, n)
+        every = np.concatenate([sparse_ids, np.nonzero(S == 0)[0]])   # zero scores last, by id
+        T_every = ro.target_topk_large([dense_ids, every], [1, 1], 60, 20, ro.NUMERATOR)
+        differ += [x for x, _ in T] != [x for x, _ in T_every]
+        ids, F, st = _eahr_pbm(V, Q[qi], off, docs, imps, n, terms, weights)
+        assert ids.tolist() == [x for x, _ in T]
+        for (x, f), got in zip(T, F):
+            if not np.isnan(got):
+                assert got == ro.as_float(f)
+        assert st["length"][1] == sparse_ids.size or not st["exhausted"][1]
+    assert differ > 0
+
+
+def test_pbm_on_a_snapshot_with_deletions():
+    """Sec. 2.4: both channels of a request rank one fixed snapshot.  A PBM
+    cursor opened on a PVS snapshot leaves deleted items out of its list,
+    and EAHR over the two matches complete-list fusion of the visible items."""
+    n, m = 30_000, 64
+    rng = np.random.default_rng(61)
+    V = synth.unit_normal(n, m, seed=62).numpy()
+    q = synth.unit_normal(1, m, seed=63).numpy()[0]
+    off, docs, imps = synth.bm25_postings(n, 5_000, 25.0, seed=64)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    terms, weights = synth.sparse_queries(1, torch.from_numpy(off), seed=65, mean_terms=4.0)[0]
+    S = po.sparse_scores(terms, weights, off, docs, imps, n)
+    # delete 5 % of the items, among them the ten best sparse ones
+    dead = np.unique(np.concatenate([rng.choice(n, n // 20, replace=False),
+                                     po.sparse_ranking(terms, weights, off, docs, imps, n)[0][:10]]))
+    visible = np.ones(n, bool)
+    visible[dead] = False
+    ref_ids, ref_sc = po.sparse_ranking(terms, weights, off, docs, imps, n)
+    keep = visible[ref_ids]
+    ref_ids, ref_sc = ref_ids[keep], ref_sc[keep]
+    dindex = pvs.pvs_build(V)
+    sindex = pvs.pbm_build(off, docs, imps, n, block=64)
+    try:
+        pvs.pvs_tombstone(dindex, dead)
+        snap = pvs.pvs_snapshot_create(dindex)
+        try:
+            cur = pvs.pbm_cursor_open(sindex, terms, weights, snap=snap)
+            try:
+                ids, sc = pull_all(cur, [20, 333], len(ref_ids))
+            finally:
+                pvs.pbm_cursor_close(cur)
+            # a cursor without the snapshot does not see the same items
+            dcur = pvs.pvs_cursor_open(dindex, q, snap=snap)
+            scur = pvs.pbm_cursor_open(sindex, terms, weights)
+            try:
+                with pytest.raises(pvs.PvsError) as e:
+                    pvs.eahr_topk_pbm(dcur, scur, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+                assert e.value.status == pvs.PVS_ERR_INVALID
+            finally:
+                pvs.pbm_cursor_close(scur)
+                pvs.pvs_cursor_close(dcur)
+        finally:
+            pvs.pvs_snapshot_free(snap)
+    finally:
+        pvs.pbm_index_free(sindex)
+        pvs.pvs_index_free(dindex)
+    assert np.array_equal(ids, ref_ids)
+    assert np.array_equal(sc.view(np.uint32), ref_sc.view(np.uint32))
+    dense_ids, _ = pvo.dense_ranking(q, V, visible=visible)
+    T = ro.target_topk_large([dense_ids, ref_ids], [1, 1], 60, 20, ro.NUMERATOR)
+    got, F, _ = _eahr_pbm(V, q, off, docs, imps, n, terms, weights, snap_ids=dead)
+    assert got.tolist() == [x for x, _ in T]
+    assert not visible[got].size or visible[got].all()
+    assert S[dead].max() > 0      # deleted items that PBM would otherwise rank

@@ -36,13 +36,41 @@ def test_hand_worked_case():
     S = po.sparse_scores([0, 2], [2.0, 0.5], off, docs, imps, 6)
     assert S.tolist() == [5.0, 1.0, 1.0, 0.0, 6.0, 0.0]
     ids, sc = po.sparse_ranking([0, 2], [2.0, 0.5], off, docs, imps, 6)
-    # Sec. 2.1: ties (items 1 and 2 at 1; items 3 and 5 at 0) by ascending id
-    assert ids.tolist() == [4, 0, 1, 2, 3, 5]
-    assert sc.tolist() == [6.0, 5.0, 1.0, 1.0, 0.0, 0.0]
+    # Sec. 2.1: ties (items 1 and 2 at 1) by ascending id; items 3 and 5 score
+    # 0, so they are outside the support U_s and have no rank
+    assert ids.tolist() == [4, 0, 1, 2]
+    assert sc.tolist() == [6.0, 5.0, 1.0, 1.0]
     # blocks of 2 ids: R0 = {0,1}, R1 = {2,3}, R2 = {4,5}
     # m_0 = (1.5, 0.5, 3), m_2 = (4, 0, 0) -> H = (2*1.5 + 0.5*4, 2*0.5, 2*3)
     H = po.range_bounds([0, 2], [2.0, 0.5], off, docs, imps, 6, 2)
     assert H.tolist() == [5.0, 1.0, 6.0]
+
+
+def test_support_is_the_items_with_positive_score():
+    # Sec. 2.1: the sparse retriever ranks U_s, the items with positive query
+    # scores; items outside it have no rank (and contribute 0 to fusion).
+    # Query: term 0 (q = 1), term 1 (q = 0), term 2 (q = 2^-100).
+    #   item 0: p_0 = 3                      -> S = 3           in U_s
+    #   item 1: only term 1 (zero weight)    -> S = RN(0 * 5) = 0
+    #   item 2: p_0 = 0 (a zero impact)      -> S = 0
+    #   item 3: p_2 = 2^-60: 2^-160 is below half the smallest subnormal
+    #           (2^-150), so RN(q_2 p_2) = 0 -> S = 0
+    #   item 4: no posting at all            -> S = 0
+    #   item 5: p_2 = 2^-40: q_2 p_2 = 2^-140, a float32 subnormal > 0
+    #   item 6: p_0 = 3, tie with item 0     -> after it by id
+    tiny = 2.0 ** -100
+    off, docs, imps = csr(4, {0: [(0, 3.0), (2, 0.0), (6, 3.0)],
+                              1: [(1, 5.0)],
+                              2: [(3, 2.0 ** -60), (5, 2.0 ** -40)],
+                              3: [(4, 9.0)]})
+    S = po.sparse_scores([0, 1, 2], [1.0, 0.0, tiny], off, docs, imps, 7)
+    assert S[3] == 0 and S[5] == np.float32(2.0 ** -140) and S[5] > 0
+    ids, sc = po.sparse_ranking([0, 1, 2], [1.0, 0.0, tiny], off, docs, imps, 7)
+    assert ids.tolist() == [0, 6, 5]
+    assert sc.tolist() == [3.0, 3.0, float(np.float32(2.0 ** -140))]
+    # a query that matches nothing has an empty ranked list
+    ids, sc = po.sparse_ranking([1], [0.0], off, docs, imps, 7)
+    assert ids.size == 0 and sc.size == 0
 
 
 def _dyadic_instance(rng, n_items, n_terms, nnz):
@@ -73,7 +101,7 @@ def test_exact_rational_sums_on_dyadic_inputs():
         # complete ranking by (score desc, id asc) against a sort of the
         # exact rationals
         ids, _ = po.sparse_ranking(q_terms, q_w, off, docs, imps, n_items)
-        want = sorted(range(n_items), key=lambda x: (-exact[x], x))
+        want = sorted((x for x in range(n_items) if exact[x] > 0), key=lambda x: (-exact[x], x))
         assert ids.tolist() == want
 
 
@@ -101,8 +129,8 @@ def test_sum_follows_the_query_term_order():
 
 
 def test_single_term_closed_form():
-    # one query term: the ranking is that term's postings by (impact desc,
-    # id asc), then every other item in ascending id at score 0
+    # one query term: the ranking is that term's postings with a positive
+    # impact, by (impact desc, id asc); nothing else has a rank
     rng = np.random.default_rng(3)
     n_items = 200
     d = np.sort(rng.choice(n_items, size=60, replace=False))
@@ -111,9 +139,8 @@ def test_single_term_closed_form():
     ids, sc = po.sparse_ranking([0], [1.0], off, docs, imps, n_items)
     pos = [(float(np.float32(x)), int(y)) for x, y in zip(p, d) if x > 0]
     want = [y for _, y in sorted(pos, key=lambda z: (-z[0], z[1]))]
-    rest = sorted(set(range(n_items)) - set(want))
-    assert ids.tolist() == want + rest
-    assert np.all(sc[len(want):] == 0)
+    assert ids.tolist() == want
+    assert np.all(sc > 0)
 
 
 def test_range_bound_covers_every_item():
@@ -133,9 +160,9 @@ def test_range_bound_covers_every_item():
         S = po.sparse_scores(q_terms, q_w, off, docs, imps, n_items)
         H = po.range_bounds(q_terms, q_w, off, docs, imps, n_items, block)
         assert np.all(S <= H[np.arange(n_items) // block])
-        # the complete ranking is a permutation with nonincreasing scores
+        # the complete ranking is U_s without repeats, scores nonincreasing
         ids, sc = po.sparse_ranking(q_terms, q_w, off, docs, imps, n_items)
-        assert sorted(ids.tolist()) == list(range(n_items))
+        assert sorted(ids.tolist()) == np.nonzero(S > 0)[0].tolist()
         assert np.all(np.diff(sc.astype(np.float64)) <= 0)
 
 
