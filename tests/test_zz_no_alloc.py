@@ -77,7 +77,7 @@ def test_noalloc_empty_input_and_top_zero_write_nothing():
     torch.cuda.synchronize()
     assert (out_ids.cpu() == -7).all() and torch.isnan(out_scores.cpu()).all()
     # and the array works again afterwards
-    _check_against_oracle(q, V, 64, out_ids, out_scores)
+    _check_against_oracle(q, V, 64, *_outs(64))
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch_and_bad_input():
