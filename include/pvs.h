@@ -204,6 +204,32 @@ pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
                                  const float* queries, int32_t nq, int32_t queries_on_device,
                                  int32_t horizon, void* cuda_stream, pvs_cursor** out);
 
+/* Largest group of pvs_cursor_open_group. */
+#define PVS_GROUP_MAX 8
+
+/* Open nq (1 <= nq <= PVS_GROUP_MAX) cursors over one snapshot (`snap`, NULL:
+ * the index's current visible set) whose score intervals come from ONE
+ * streaming pass over the Int8 codes (Sec. 2.3.1, App. A.1): each tile of
+ * codes is read once and scored against all nq queries, instead of once per
+ * query.  Each cursor gets the same bounds, bit for bit, as a cursor of
+ * pvs_cursor_open, and afterwards behaves like one.  queries: nq x dim
+ * floats, host or device per queries_on_device.  The pass runs on
+ * `pass_stream` (a cudaStream_t; NULL: the index's stream) after the
+ * queries' encoding; cursor i's later work runs on cursor_streams[i] (an
+ * array of nq cudaStream_t, or NULL; a NULL array or entry means
+ * pass_stream), ordered after the pass, so the pulls of the group's queries
+ * can run on their own streams while the next group's pass streams the
+ * codes.  The call returns once the queries are encoded and the pass is
+ * queued.  Row widths the grouped pass does not serve (dim rounded up to 64
+ * not in {128, 256, 384, 512, 768, 1024}) and nq == 1 give plain cursors
+ * with a pass of their own at the first pull.  out[0..nq-1] receive the
+ * cursors; close each with pvs_cursor_close.  Errors as pvs_cursor_open; on
+ * error no cursor is returned. */
+pvs_status pvs_cursor_open_group(pvs_index* index, const pvs_snapshot* snap,
+                                 const float* queries, int32_t nq, int32_t queries_on_device,
+                                 void* pass_stream, void* const* cursor_streams,
+                                 pvs_cursor** out);
+
 /* The next n ranks of each of nc cursors in one set of launches (all
  * cursors of one index and one stream).  Row i of ids / scores (nc x n,
  * int64 / float32, device or host per outputs_on_device) receives cursor i's

@@ -137,6 +137,7 @@ def _load() -> ctypes.CDLL:
         "pvs_launch_count": (i64, []),
         "pvs_rank_exact_noalloc": (i32, [P, P, i32, i32, i32, P, P, P]),
         "pvs_index_import": (i32, [P, P, P, P, P, i64, i32, P, pp]),
+        "pvs_cursor_open_group": (i32, [P, P, P, i32, i32, P, P, P]),
         "pvs_index_set_wait_limit": (i32, [P, i64]),
         "eahr_topk": (i32, [P, P, i64, ctypes.POINTER(eahr_params), P, P, P,
                             ctypes.POINTER(eahr_stats)]),
@@ -182,7 +183,7 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_cursor_sync_batch", "pvs_cursor_stats_batch", "pvs_cursor_close_batch",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc",
-            "pvs_index_import", "pvs_index_set_wait_limit", "eahr_topk",
+            "pvs_index_import", "pvs_index_set_wait_limit", "pvs_cursor_open_group", "eahr_topk",
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
             "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
@@ -322,6 +323,31 @@ def pvs_cursor_open(index, query, snap=None):
     out = ctypes.c_void_p()
     _check(_lib.pvs_cursor_open(index, snap, ptr, on_dev, ctypes.byref(out)), "pvs_cursor_open")
     return out
+
+
+PVS_GROUP_MAX = 8
+
+
+def pvs_cursor_open_group(index, queries, snap=None, pass_stream=None, cursor_streams=None):
+    """Open one cursor per query row (at most PVS_GROUP_MAX) whose bounds come
+    from one grouped pass over the codes -> list of cursors.  pass_stream and
+    the entries of cursor_streams: torch.cuda.Stream or raw cudaStream_t
+    (None: the index's stream / the pass stream)."""
+    ptr, shape, on_dev, keep = _vec_arg(queries)
+    nq = shape[0] if len(shape) == 2 else 1
+    arr = (ctypes.c_void_p * max(nq, 1))()
+    ps = getattr(pass_stream, "cuda_stream", pass_stream)
+    streams = None
+    if cursor_streams is not None:
+        if len(cursor_streams) != nq:
+            raise ValueError("one stream per query")
+        streams = (ctypes.c_void_p * nq)(*[getattr(s, "cuda_stream", s) for s in cursor_streams])
+    _check(_lib.pvs_cursor_open_group(index, snap, ptr, nq, on_dev,
+                                      ctypes.c_void_p(ps) if ps else None,
+                                      ctypes.cast(streams, ctypes.c_void_p) if streams else None,
+                                      ctypes.cast(arr, ctypes.POINTER(ctypes.c_void_p))),
+           "pvs_cursor_open_group")
+    return [ctypes.c_void_p(arr[i]) for i in range(nq)]
 
 
 class CursorBatch(tuple):

@@ -22,29 +22,6 @@
 
 namespace pvs {
 
-// Interval of Sec. 2.3.1 / App. A.1 from the exact Int8 dot product, in the
-// operation order the oracle states (RN centre, RU/RD bounds).
-__device__ __forceinline__ void interval_epilogue(int dot, const QueryScalars& q, float sv,
-                                                  float vn, float en, float& lo, float& hi) {
-    float fdot = __int2float_rn(dot);
-    float ss = __fmul_rn(q.s, sv);
-    float c = __fmul_rn(ss, fdot);
-    float e1 = __fmul_ru(q.enorm, vn);
-    float e2 = __fmul_ru(q.qhat, en);
-    float E = __fadd_ru(e1, e2);
-    float g1 = __fadd_ru(fabsf(c), E);
-    float g2 = __fmul_ru(q.qnorm, vn);
-    float g3 = __fadd_ru(g1, g2);
-    float G = __fmul_ru(g3, q.gamma);
-    float r = __fadd_ru(E, G);
-    lo = __fsub_rd(c, r);
-    hi = __fadd_ru(c, r);
-}
-
-__device__ __forceinline__ bool tombstoned(const uint32_t* tomb, int64_t row) {
-    return tomb != nullptr && ((__ldg(tomb + (row >> 5)) >> (row & 31)) & 1u);
-}
-
 constexpr int kConsumerWarps = 8;
 constexpr int kIntervalThreads = (kConsumerWarps + 1) * 32;
 

@@ -181,6 +181,36 @@ int64_t interval_slots(int64_t rows, int m_pad, int num_sms, int64_t* min_rows_p
 // Plain reference-style variant without staging (used for tiny inputs).
 cudaError_t launch_interval_simple(const IntervalArgs& a, cudaStream_t st);
 
+// Grouped pass: the intervals of up to kGroupMax queries from one read of the
+// codes (each code tile is staged once and scored against every query of
+// the group).  Per query g < nq: its codes zq[g] and scalars qs[g], and its
+// own outputs lo[g], hi[g], status[g] and slot_top[g] (may be null).  A
+// slot of the grouped pass is (CTA, consumer warp, MMA row pair):
+// interval_group_slots gives their count and the fewest rows any scans.
+constexpr int kGroupMax = 8;
+struct IntervalGroupArgs {
+    const int8_t* codes;
+    const float* scale;
+    const float* vnorm;
+    const float* enorm;
+    const uint32_t* tomb;
+    int64_t rows;
+    int m_pad;
+    int nq;
+    const int8_t* zq[kGroupMax];
+    const QueryScalars* qs[kGroupMax];
+    float* lo[kGroupMax];
+    float* hi[kGroupMax];
+    int* status[kGroupMax];
+    float* slot_top[kGroupMax];
+    unsigned long long wait_ns = kWaitLimitNs;
+};
+// True when a grouped pass serves nq queries over rows of m_pad bytes.
+bool interval_group_supported(int m_pad, int nq);
+cudaError_t launch_interval_group(const IntervalGroupArgs& a, int num_sms, cudaStream_t st);
+int64_t interval_group_slots(int64_t rows, int m_pad, int nq, int num_sms,
+                             int64_t* min_rows_per_slot);
+
 // ---- selection / compaction / sort (select_kernels.cu) ----------------------
 // k-th largest key (1-based) among live entries of a float array: key of
 // vals[i] with vals[i] != -inf, i < *len (len in device memory).  Result in

@@ -231,6 +231,8 @@ void cursor_reset(pvs_cursor* c) {
     c->fresh_ws = false;
     c->horizon = c->horizon_base = 0;
     c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
+    c->code_bytes = 0;
+    c->group_size = 1;
     c->batch_passes = 0;
     c->batch_ms = 0.0;
     c->ev_pending = false;
@@ -414,6 +416,7 @@ pvs_status interval_pass(pvs_cursor* c) {
     PVS_CUDA(cudaEventRecord(x->pass_done, c->stream));
     c->ev_pending = true;
     c->interval_passes++;
+    c->code_bytes += c->rows * (int64_t)(x->m_pad + 12);
     c->scanned = true;
     if (x->wait_ns < kWaitLimitNs) {
         // a shortened wait limit (pvs_index_set_wait_limit) makes a timed-out
@@ -1361,11 +1364,152 @@ pvs_status pvs::cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const flo
     return PVS_OK;
 }
 
+static_assert(pvs::kGroupMax == PVS_GROUP_MAX, "group size of the C ABI");
+
+namespace {
+
+// One grouped interval pass for the nq (>= 2) freshly opened cursors cs[],
+// which share one snapshot: their bounds and per-slot lower bounds, on
+// stream `ps`; every cursor's own stream then waits for the pass.
+pvs_status group_pass(pvs_index* x, pvs_cursor* const* cs, int nq, cudaStream_t ps) {
+    IntervalGroupArgs a;
+    a.codes = x->codes;
+    a.scale = x->scale;
+    a.vnorm = x->vnorm;
+    a.enorm = x->enorm;
+    a.tomb = cs[0]->snap->d_tomb;
+    a.rows = cs[0]->rows;
+    a.m_pad = x->m_pad;
+    a.nq = nq;
+    a.wait_ns = x->wait_ns;
+    int64_t min_rows = 0;
+    const int64_t slots = interval_group_slots(a.rows, x->m_pad, nq, x->num_sms, &min_rows);
+    const bool use_slots = slots > 0 && a.tomb == nullptr && min_rows >= kSlotTop;
+    for (int i = 0; i < nq; ++i) {
+        pvs_cursor* c = cs[i];
+        pvs_status s = cursor_alloc_rows(c);
+        if (s != PVS_OK) return s;
+        c->slot_fresh = false;
+        c->slot_n = 0;
+        a.slot_top[i] = nullptr;
+        if (use_slots) {
+            if (c->slot_cap < slots * kSlotTop) {
+                dev_free(c->slot_top);
+                c->slot_cap = 0;
+                PVS_CUDA(dev_alloc(&c->slot_top, (size_t)(slots * kSlotTop)));
+                c->slot_cap = slots * kSlotTop;
+            }
+            a.slot_top[i] = c->slot_top;
+            c->slot_n = slots * kSlotTop;
+        }
+        a.zq[i] = c->zq;
+        a.qs[i] = c->qs;
+        a.lo[i] = c->lo;
+        a.hi[i] = c->hi;
+        a.status[i] = c->d_status;
+        if (!c->ev_begin) {
+            PVS_CUDA(cudaEventCreate(&c->ev_begin));
+            PVS_CUDA(cudaEventCreate(&c->ev_end));
+        }
+    }
+    {
+        // passes of one index run one after another (each saturates HBM)
+        std::lock_guard<std::mutex> lock(x->pass_mutex);
+        if (!x->pass_done)
+            PVS_CUDA(cudaEventCreateWithFlags(&x->pass_done, cudaEventDisableTiming));
+        else
+            PVS_CUDA(cudaStreamWaitEvent(ps, x->pass_done, 0));
+        for (int i = 0; i < nq; ++i) PVS_CUDA(cudaEventRecord(cs[i]->ev_begin, ps));
+        PVS_CUDA(launch_interval_group(a, x->num_sms, ps));
+        for (int i = 0; i < nq; ++i) PVS_CUDA(cudaEventRecord(cs[i]->ev_end, ps));
+        PVS_CUDA(cudaEventRecord(x->pass_done, ps));
+    }
+    for (int i = 0; i < nq; ++i) {
+        pvs_cursor* c = cs[i];
+        if (c->stream != ps) PVS_CUDA(cudaStreamWaitEvent(c->stream, c->ev_end, 0));
+        c->slot_fresh = a.slot_top[i] != nullptr;
+        c->ev_pending = true;
+        c->interval_passes++;
+        c->code_bytes += c->rows * (int64_t)(x->m_pad + 12) / nq;
+        c->group_size = nq;
+        c->scanned = true;
+    }
+    if (x->wait_ns < kWaitLimitNs) {   // as in interval_pass: check before any pull
+        PVS_CUDA(cudaStreamSynchronize(ps));
+        for (int i = 0; i < nq; ++i) {
+            pvs_status s = check_device_status(cs[i]);
+            if (s != PVS_OK) return s;
+        }
+    }
+    return PVS_OK;
+}
+
+}  // namespace
+
+pvs_status pvs::cursor_open_group(pvs_index* x, const pvs_snapshot* snap, const float* queries,
+                                  int32_t nq, int32_t queries_on_device, cudaStream_t pass_stream,
+                                  const cudaStream_t* cursor_streams, pvs_cursor** out) {
+    DeviceGuard device_guard(index_device(x));
+    if (!out || nq < 1 || nq > kGroupMax) return PVS_ERR_INVALID;
+    for (int i = 0; i < nq; ++i) out[i] = nullptr;
+    if (!x || !queries || (snap && snap->index != x)) return PVS_ERR_INVALID;
+    if (queries_on_device && !is_device_ptr(queries)) return PVS_ERR_INVALID;
+    cudaStream_t ps = pass_stream ? pass_stream : x->stream;
+    // one visible set for the whole group
+    pvs_snapshot own;
+    if (!snap) {
+        own.index = x;
+        own.data = make_snapdata(x);
+        if (!own.data) return PVS_ERR_OOM;
+        snap = &own;
+    }
+    pvs_cursor* cs[kGroupMax] = {nullptr};
+    auto bail = [&](pvs_status s) {
+        for (int i = 0; i < nq; ++i)
+            if (cs[i]) pvs_cursor_close(cs[i]);
+        return s;
+    };
+    for (int i = 0; i < nq; ++i) {
+        cudaStream_t st = cursor_streams && cursor_streams[i] ? cursor_streams[i] : ps;
+        pvs_status s = cursor_open_on(x, snap, queries + (int64_t)i * x->m, queries_on_device,
+                                      st, &cs[i]);
+        if (s != PVS_OK) return bail(s);
+    }
+    // one query, nothing visible, or rows the grouped pass does not serve:
+    // each cursor runs its own pass at its first pull
+    if (nq >= 2 && cs[0]->visible > 0 && interval_group_supported(x->m_pad, nq)) {
+        // the pass runs on ps after every cursor's queued work (their queries)
+        for (int i = 0; i < nq; ++i) {
+            if (cs[i]->stream == ps) continue;
+            cudaError_t e = cudaSuccess;
+            if (!cs[i]->ev_order) e = cudaEventCreateWithFlags(&cs[i]->ev_order, cudaEventDisableTiming);
+            if (e == cudaSuccess) e = cudaEventRecord(cs[i]->ev_order, cs[i]->stream);
+            if (e == cudaSuccess) e = cudaStreamWaitEvent(ps, cs[i]->ev_order, 0);
+            if (e != cudaSuccess) return bail(cuda_status(e));
+        }
+        pvs_status s = group_pass(x, cs, nq, ps);
+        if (s != PVS_OK) {
+            for (int i = 0; i < nq; ++i) fail(cs[i], s);
+            return bail(s);
+        }
+    }
+    for (int i = 0; i < nq; ++i) out[i] = cs[i];
+    return PVS_OK;
+}
+
 extern "C" {
 
 pvs_status pvs_cursor_open(pvs_index* x, const pvs_snapshot* snap, const float* query,
                            int32_t query_on_device, pvs_cursor** out) {
     return pvs::cursor_open_on(x, snap, query, query_on_device, nullptr, out);
+}
+
+pvs_status pvs_cursor_open_group(pvs_index* x, const pvs_snapshot* snap, const float* queries,
+                                 int32_t nq, int32_t queries_on_device, void* pass_stream,
+                                 void* const* cursor_streams, pvs_cursor** out) {
+    return pvs::cursor_open_group(x, snap, queries, nq, queries_on_device,
+                                  static_cast<cudaStream_t>(pass_stream),
+                                  reinterpret_cast<const cudaStream_t*>(cursor_streams), out);
 }
 
 pvs_status pvs_cursor_open_batch(pvs_index* x, const pvs_snapshot* snap, const float* queries,
@@ -1672,7 +1816,7 @@ static void fill_stats(pvs_cursor* c, const DevCounters& d, pvs_stats* out) {
     out->horizon_builds = c->horizon_builds;
     out->pulls = c->pulls;
     out->candidates = c->candidates + (int64_t)d.cand_total;
-    out->code_bytes = c->interval_passes * c->rows * (int64_t)(c->index->m_pad + 12);
+    out->code_bytes = c->code_bytes;
     out->state = c->state;
     harvest_interval_time(c);
     out->interval_ms = c->interval_ms;

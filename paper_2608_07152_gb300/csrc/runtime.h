@@ -121,6 +121,9 @@ struct pvs_cursor {
     unsigned int* h_small = nullptr;  // pinned scratch (counts, status)
     // stats
     int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;
+    int64_t code_bytes = 0;           // code + parameter bytes read for this cursor (a
+                                      // grouped pass's bytes are split among its queries)
+    int32_t group_size = 1;           // queries that shared the cursor's interval pass
     int64_t batch_passes = 0;         // batched (tensor-core) passes this cursor took part in
     double batch_ms = 0.0;            // device time of that pass (shared by its cursors)
     cudaEvent_t ev_begin = nullptr, ev_end = nullptr;   // around the last interval pass
@@ -145,6 +148,12 @@ const SnapData* cursor_snapshot(const pvs_cursor* c);
 // its next pull) instead of copied out.
 pvs_status next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
                        int32_t* n_out);
+// Open nq <= kGroupMax cursors whose bounds come from one grouped interval
+// pass on pass_stream (null: the index's stream); cursor i's later work runs
+// on cursor_streams[i] (null array or entry: pass_stream).
+pvs_status cursor_open_group(pvs_index* x, const pvs_snapshot* snap, const float* queries,
+                             int32_t nq, int32_t queries_on_device, cudaStream_t pass_stream,
+                             const cudaStream_t* cursor_streams, pvs_cursor** out);
 // Open a cursor whose device work runs on `stream` (null: the index's stream).
 pvs_status cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const float* query,
                           int32_t query_on_device, cudaStream_t stream, pvs_cursor** out);
