@@ -4,20 +4,23 @@ Workload (the passage-scale single-query configuration): a corpus of
 N = 8,841,823 vectors of d = 768 drawn from a 4,096-component Gaussian
 mixture (standard-normal centres, within-component std 0.35, L2-normalised);
 queries are perturbed mixture centres (noise std 0.5, normalised).  One step
-= a batch of queries; per query the cursor delivers the first 1,000 exact
-ranks in chunks of 20 (open, 50 pulls, close).  The corpus codes (6.9 GB per
+= a batch of queries; per query a cursor delivers the first 1,000 exact ranks
+in chunks of 20 (open, 50 pulls, close).  The corpus codes (6.9 GB per
 interval pass) are far larger than the 129 MB L2, so no L2 flush is needed.
 
-`value` (exact dense ranks/s) is timed with CUDA events on the library's
-stream with queries resident in HBM and ranks written to device buffers;
-`e2e` repeats the step through the library's native request executor
-(pvs_executor_run: host query buffers in pinned memory, host output buffers,
-every 20-rank page read through pvs_next onto the host before the next is
-requested, PIPELINE native worker threads), the copies inside the timed
-region.
-`roofline` reports the interval pass (the dominant kernel): algorithmic bytes
-N * (m_pad + 12) per pass over its CUDA-event duration, against the measured
-HBM copy bandwidth.
+Both legs run through the library's native request executor
+(pvs_executor_run_ex): WORKERS native threads, each serving GROUP queries
+at a time from one grouped interval pass over the codes
+(pvs_cursor_open_group) and pulling every 20-rank page of the group's
+cursors in one batched launch; every query still gets its own pages.
+`value` (exact dense ranks/s) has the queries resident in HBM and the ranks
+written to device buffers, timed with CUDA events; `e2e` is the same
+through host buffers (pinned queries in, every page on the host before the
+next is requested), the copies inside the timed region.
+`roofline` reports the grouped interval pass (the dominant kernel):
+algorithmic bytes N * (m_pad + 12) read plus 8 * N * GROUP bytes of bounds
+written per pass, over its CUDA-event duration (the library's events on the
+pass's stream), against the measured HBM copy bandwidth.
 
 `--impl reference` times the oracle (a plain CPU implementation, run as it
 stands) on a bounded sample of the same workload.  Under torchrun every rank
@@ -56,7 +59,9 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="pvs", choices=["pvs", "reference"])
-    p.add_argument("--queries", type=int, default=50, help="queries per step")
+    p.add_argument("--queries", type=int, default=64, help="queries per step")
+    p.add_argument("--group", type=int, default=8,
+                   help="passage: queries per grouped pass over the codes (1: one pass each)")
     p.add_argument("--n", type=int, default=N_CORPUS, help="corpus rows (default: full)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="passage",
@@ -236,8 +241,7 @@ def build_corpus_index(pvs, synth, torch, n, stream, device, components=COMPONEN
     return index, centres, time.perf_counter() - t0
 
 
-PIPELINE = 8   # queries in flight, each on its own stream (measured plateau: 2 -> 704k,
-               # 4 -> 827k, 6 -> 876k, 8 -> 903k, 10 -> 881k ranks/s)
+PIPELINE = 4   # passage: executor worker threads, each with a group of queries in flight
 
 
 def _finish(pvs, cur, stats_acc):
@@ -248,26 +252,6 @@ def _finish(pvs, cur, stats_acc):
         raise RuntimeError(f"cursor failed: {st}")
     if stats_acc is not None:
         stats_acc.append(s)
-
-
-def run_step_device(pvs, index, queries, out_ids, out_scores, streams, stats_acc):
-    """One step: every query opens a cursor and pulls 1,000 ranks in chunks
-    of 20 into device buffers.  Up to PIPELINE queries are in flight on their
-    own streams, so one query's pulls overlap the next query's interval pass;
-    every pull is still a separate pvs_next_device call."""
-    pending = []
-    for qi in range(queries.shape[0]):
-        slot = qi % PIPELINE
-        cur = pvs.pvs_cursor_open(index, queries[qi])
-        pvs.pvs_cursor_set_stream(cur, streams[slot])
-        for p in range(RANKS_PER_QUERY // CHUNK):
-            off = p * CHUNK
-            pvs.pvs_next_device(cur, CHUNK, out_ids[slot, off:], out_scores[slot, off:])
-        pending.append(cur)
-        if len(pending) >= PIPELINE:
-            _finish(pvs, pending.pop(0), stats_acc)
-    while pending:
-        _finish(pvs, pending.pop(0), stats_acc)
 
 
 def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, count):
@@ -311,10 +295,11 @@ def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget
     dt = time.perf_counter() - t0
     per_query_full = dt / done * (n_full / rows)
     return {"value": RANKS_PER_QUERY / per_query_full, "unit": UNIT,
-            "cores": os.cpu_count(), "kind": "oracle",
+            "cores": os.cpu_count(), "kind": "oracle", "projected": True,
             "sample": f"{done} queries x first {RANKS_PER_QUERY} exact ranks over the first "
-                      f"{rows:,} corpus rows (oracle: binary64 scoring + exact fallback + full "
-                      f"sort), time scaled by N/{rows:,}"}
+                      f"{rows:,} corpus rows (oracle: binary64 scoring by numpy's BLAS on "
+                      f"{os.cpu_count()} threads + exact fallback + full sort); projected to "
+                      f"N by scaling the time by N/{rows:,}"}
 
 
 def reference_arm(args):
@@ -344,9 +329,9 @@ def reference_arm(args):
             "config": {"workload": WORKLOAD, "N": args.n, "d": DIM,
                        "step": "1 query, first 1,000 ranks"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
-                             "kind": "oracle",
-                             "sample": f"1 query per step over the first {rows:,} rows, "
-                                       f"time scaled by N/{rows:,}"},
+                             "kind": "oracle", "projected": True,
+                             "sample": f"1 query per step over the first {rows:,} rows; "
+                                       f"projected to N by scaling the time by N/{rows:,}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -1315,6 +1300,139 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
+    """The passage workload (the default): the queries of a step served by
+    the native executor, GROUP at a time from one grouped pass over the
+    codes, every 20-rank page of a group's cursors in one batched pull."""
+    stream = torch.cuda.Stream(device=dev)
+    n = args.n
+    group = max(1, min(args.group, pvs.PVS_GROUP_MAX))
+    index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev)
+    nq = args.queries
+    total_q = (args.warmup + args.steps) * nq
+    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
+    queries = queries.reshape(total_q, DIM).contiguous()
+    warm_q = queries[:args.warmup * nq]
+    timed_q = queries[args.warmup * nq:]
+    n_timed = timed_q.shape[0]
+    ids = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
+    scores = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    executor = pvs.pvs_executor_create(index, PIPELINE)
+    try:
+        pvs.pvs_executor_set_group(executor, group)
+        if warm_q.shape[0]:
+            pvs.pvs_executor_run_device(executor, warm_q, RANKS_PER_QUERY, CHUNK,
+                                        ids[:warm_q.shape[0]], scores[:warm_q.shape[0]])
+        st0 = pvs.pvs_executor_stats(executor)
+
+        # ---- timed region: device-resident queries and outputs ----
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        launches0 = pvs.pvs_launch_count()
+        start = torch.cuda.Event(enable_timing=True)
+        end = torch.cuda.Event(enable_timing=True)
+        with ClockSampler(local) as clk:
+            start.record(stream)
+            n_out, status, rc = pvs.pvs_executor_run_device(executor, timed_q, RANKS_PER_QUERY,
+                                                            CHUNK, ids, scores)
+            end.record(stream)
+            stream.synchronize()
+        torch.cuda.synchronize()
+        launches = pvs.pvs_launch_count() - launches0
+        st1 = pvs.pvs_executor_stats(executor)
+        if rc != pvs.PVS_OK or int(n_out.min()) != RANKS_PER_QUERY:
+            raise RuntimeError(f"executor run failed: {rc}")
+        elapsed = start.elapsed_time(end) / 1e3
+        elapsed = slowest(pg, elapsed, dev)
+        ranks_total = n_timed * RANKS_PER_QUERY * world
+        value = job_rate(n_timed * RANKS_PER_QUERY, world, elapsed)
+
+        # ---- e2e: pinned host queries and outputs through the same executor ----
+        qh = timed_q.cpu().pin_memory()
+        h_ids = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.int64).pin_memory()
+        h_sc = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.float32).pin_memory()
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        _, _, n_got, _, rc = pvs.pvs_executor_run(executor, qh, RANKS_PER_QUERY, CHUNK,
+                                                  ids=h_ids, scores=h_sc)
+        torch.cuda.synchronize()
+        e2e_elapsed = time.perf_counter() - t0
+        if rc != pvs.PVS_OK or int(n_got.min()) != RANKS_PER_QUERY:
+            raise RuntimeError(f"executor run failed: {rc}")
+        # the two legs deliver the same ranks
+        same = bool(torch.equal(h_ids, ids.cpu()))
+    finally:
+        pvs.pvs_executor_destroy(executor)
+
+    # ---- latency of a lone query (its own cursor and pass), one at a time ----
+    out_ids = torch.empty((1, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
+    out_scores = torch.empty((1, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    lat20, lat1000 = measure_latency(pvs, torch, index, timed_q, out_ids, out_scores, stream,
+                                     min(n_timed, 20))
+    e2e_elapsed = slowest(pg, e2e_elapsed, dev)
+    e2e_value = ranks_total / e2e_elapsed
+
+    # ---- roofline of the grouped interval pass ----
+    m_pad = ((DIM + 63) // 64) * 64
+    passes = st1["interval_passes"] - st0["interval_passes"]
+    pass_ms = (st1["interval_ms"] - st0["interval_ms"]) / max(passes, 1)
+    read_bytes = n * (m_pad + 12)
+    write_bytes = 8 * n * group
+    alg_bytes = read_bytes + write_bytes
+    achieved = alg_bytes / (pass_ms / 1e3) / 1e9
+    peak, peak_kind = measured_peaks()
+    kernel = "interval_group_kernel" if group > 1 else "interval_pass_kernel"
+    traffic = (interval_traffic(n, "interval_group_kernel_passage_traffic.json") if group > 1
+               else interval_traffic(n))
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "N": n, "d": DIM, "queries_per_step": nq,
+                   "ranks_per_query": RANKS_PER_QUERY, "chunk": CHUNK,
+                   "queries_per_pass": group, "executor_workers": PIPELINE,
+                   "l2": "no flush: each interval pass streams 6.9 GB of codes (> 129 MB L2)",
+                   "parallelism": f"replicas x{world} (queries sharded, no collective)"},
+        "e2e": {"value": e2e_value, "unit": UNIT,
+                "h2d_bytes_per_step": nq * DIM * 4,
+                "d2h_bytes_per_step": nq * RANKS_PER_QUERY * (8 + 4),
+                "path": f"pvs_executor_run: {PIPELINE} native workers, {group} queries per "
+                        f"pass, pages of {CHUNK} through batched pulls, pinned host queries and "
+                        "outputs",
+                "same_ranks_as_value_leg": same},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_kind": peak_kind, "kernel": kernel,
+                     "frac_of_8tbs_nominal": achieved / 8000.0,
+                     "algorithmic_bytes": {"codes_and_params_read": read_bytes,
+                                           "bounds_written": write_bytes}},
+        "gpu_launches": launches,
+        "latency_ms": {"first_20_p50": statistics.median(lat20),
+                       "first_1000_p50": statistics.median(lat1000),
+                       "first_1000_p95": sorted(lat1000)[int(0.95 * (len(lat1000) - 1))],
+                       "note": "a lone query with its own cursor and single-query pass"},
+        "interval_pass": {"ms": pass_ms, "GBps": achieved, "queries_per_pass": group,
+                          "ms_per_query": pass_ms / group, "passes_timed": passes},
+        "per_query": {"refined_mean": (st1["refined"] - st0["refined"]) / n_timed},
+        "build_s": build_s,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        qb = timed_q[:64].cpu().numpy()
+        line["cpu_baseline"] = cpu_baseline(synth, torch, centres, qb, n)
+    pvs.pvs_index_free(index)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
 def main():
     global PIPELINE, BATCH_PIPELINE
     args = parse()
@@ -1358,122 +1476,7 @@ def main():
         main_segments(args, pvs, synth, torch, np, rank, world, local, dev, pg)
         return
 
-    stream = torch.cuda.Stream(device=dev)
-    n = args.n
-    index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev)
-    total_q = (args.warmup + args.steps) * args.queries
-    queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
-    queries = queries.reshape(args.warmup + args.steps, args.queries, DIM).contiguous()
-    out_ids = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
-    out_scores = torch.empty((PIPELINE, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
-    streams = [torch.cuda.Stream(device=dev) for _ in range(PIPELINE)]
-    torch.cuda.synchronize()
-
-    stats = []
-    for w in range(args.warmup):
-        run_step_device(pvs, index, queries[w], out_ids, out_scores, streams, None)
-
-    # ---- timed region: device-resident queries and outputs ----
-    if pg:
-        pg.barrier()
-    torch.cuda.synchronize()
-    launches0 = pvs.pvs_launch_count()
-    start = torch.cuda.Event(enable_timing=True)
-    end = torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
-        start.record(stream)
-        for s_ in streams:
-            s_.wait_event(start)
-        for s in range(args.steps):
-            run_step_device(pvs, index, queries[args.warmup + s], out_ids, out_scores, streams,
-                            stats)
-        for s_ in streams:                      # join every stream's work
-            done = torch.cuda.Event()
-            done.record(s_)
-            stream.wait_event(done)
-        end.record(stream)
-        stream.synchronize()
-    torch.cuda.synchronize()
-    launches = pvs.pvs_launch_count() - launches0
-    elapsed = start.elapsed_time(end) / 1e3
-    elapsed = slowest(pg, elapsed, dev)
-    ranks_total = args.steps * args.queries * RANKS_PER_QUERY * world
-    value = job_rate(args.steps * args.queries * RANKS_PER_QUERY, world, elapsed)
-
-    # ---- e2e: pinned host queries, host outputs, through the native executor ----
-    qh = [queries[args.warmup + s].cpu().pin_memory() for s in range(args.steps)]
-    h_ids = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.int64).pin_memory()
-    h_sc = torch.empty((args.queries, RANKS_PER_QUERY), dtype=torch.float32).pin_memory()
-    executor = pvs.pvs_executor_create(index, PIPELINE)
-    try:
-        if pg:
-            pg.barrier()
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for s in range(args.steps):
-            _, _, n_got, _, rc = pvs.pvs_executor_run(executor, qh[s], RANKS_PER_QUERY, CHUNK,
-                                                      ids=h_ids, scores=h_sc)
-            if rc != pvs.PVS_OK or int(n_got.min()) != RANKS_PER_QUERY:
-                raise RuntimeError(f"executor run failed: {rc}")
-        torch.cuda.synchronize()
-        e2e_elapsed = time.perf_counter() - t0
-    finally:
-        pvs.pvs_executor_destroy(executor)
-
-    # ---- latency, one query at a time ----
-    lat20, lat1000 = measure_latency(pvs, torch, index, queries[args.warmup],
-                                     out_ids, out_scores, stream, min(args.queries, 20))
-    e2e_elapsed = slowest(pg, e2e_elapsed, dev)
-    e2e_value = ranks_total / e2e_elapsed
-
-    # ---- roofline of the interval pass ----
-    m_pad = ((DIM + 63) // 64) * 64
-    passes = sum(s["interval_passes"] for s in stats)
-    interval_ms = sum(s["interval_ms"] for s in stats) / max(passes, 1)
-    alg_bytes = n * (m_pad + 12)
-    achieved = alg_bytes / (interval_ms / 1e3) / 1e9
-    peak, peak_kind = measured_peaks()
-    traffic = interval_traffic(n)
-
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": elapsed / args.steps * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "N": n, "d": DIM, "queries_per_step": args.queries,
-                   "ranks_per_query": RANKS_PER_QUERY, "chunk": CHUNK,
-                   "queries_in_flight": PIPELINE,
-                   "l2": "no flush: each query's interval pass streams 6.9 GB of codes (> 129 MB L2)",
-                   "parallelism": f"replicas x{world} (queries sharded, no collective)"},
-        "e2e": {"value": e2e_value, "unit": UNIT,
-                "h2d_bytes_per_step": args.queries * DIM * 4,
-                "d2h_bytes_per_step": args.queries * RANKS_PER_QUERY * (8 + 4),
-                "path": f"pvs_executor_run: {PIPELINE} native workers, pages of {CHUNK} "
-                        "through pvs_next, pinned host queries and outputs"},
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic,
-                     "peak_kind": peak_kind, "kernel": "interval_pass_kernel",
-                     "frac_of_8tbs_nominal": achieved / 8000.0},
-        "gpu_launches": launches,
-        "latency_ms": {"first_20_p50": statistics.median(lat20),
-                       "first_1000_p50": statistics.median(lat1000),
-                       "first_1000_p95": sorted(lat1000)[int(0.95 * (len(lat1000) - 1))]},
-        "interval_pass": {"ms": interval_ms, "GBps": achieved, "bytes": alg_bytes},
-        "per_query": {"refined_mean": statistics.mean(s["refined"] for s in stats),
-                      "candidates_mean": statistics.mean(s["candidates"] for s in stats),
-                      "exact_fallbacks": sum(s["exact_fallbacks"] for s in stats)},
-        "build_s": build_s,
-        "clocks": clk.summary(),
-    }
-    if rank == 0 and not args.no_cpu_baseline:
-        qb = queries[0].cpu().numpy()
-        line["cpu_baseline"] = cpu_baseline(synth, torch, centres, qb, n)
-    pvs.pvs_index_free(index)
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if pg:
-        pg.barrier()
-        pg.destroy_process_group()
+    main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg)
 
 
 if __name__ == "__main__":

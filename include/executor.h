@@ -13,7 +13,11 @@
  * A fixed pool of native worker threads, each with its own CUDA stream on
  * the index's device, keeps up to `workers` requests in flight, so the
  * interval pass of one request overlaps the pages of the others on the
- * device.  No host interpreter is involved between pages.
+ * device.  No host interpreter is involved between pages.  With a group
+ * size G >= 2 (pvs_executor_set_group) a worker serves G requests at a time:
+ * their cursors come from one pvs_cursor_open_group (one pass over the Int8
+ * codes for all G queries) and each page of the G cursors is one batched
+ * pull; every request still receives its own pages.
  *
  * Conventions as pvs.h: the caller owns every buffer; the index must
  * outlive the executor and must not be changed (append, delete) while a run
@@ -38,7 +42,11 @@ typedef struct pvs_executor_stats {
     int64_t pages;       /* pvs_next calls                                    */
     int64_t ranks;       /* ranks delivered                                   */
     int32_t workers;     /* worker threads (and streams)                      */
-    int32_t reserved;
+    int32_t group;       /* requests per grouped open (1: none)               */
+    int64_t interval_passes; /* passes over the Int8 codes (a grouped pass
+                                counts once)                                 */
+    double interval_ms;  /* their device time, CUDA events, summed           */
+    int64_t refined;     /* authoritative float32 evaluations                 */
 } pvs_executor_stats;
 
 /*
@@ -66,6 +74,24 @@ pvs_status pvs_executor_create(pvs_index* index, int32_t workers, pvs_executor**
 pvs_status pvs_executor_run(pvs_executor* ex, const pvs_snapshot* snap, const float* queries,
                             int32_t nq, int32_t ranks, int32_t page, int64_t* ids, float* scores,
                             int32_t* n_out, int32_t* status);
+
+/*
+ * pvs_executor_run with buffers_on_device selecting where queries, ids and
+ * scores live: 0 as pvs_executor_run (host memory); 1 for device memory of
+ * the index's device (nothing crosses the bus: each page is queued on the
+ * worker's stream and a request is complete when the call returns).  n_out
+ * and status are host arrays in both cases.
+ */
+pvs_status pvs_executor_run_ex(pvs_executor* ex, const pvs_snapshot* snap, const float* queries,
+                               int32_t nq, int32_t ranks, int32_t page, int32_t buffers_on_device,
+                               int64_t* ids, float* scores, int32_t* n_out, int32_t* status);
+
+/*
+ * Serve requests in groups of `group` (1 .. PVS_GROUP_MAX; default 1): the
+ * queries of a group share one pass over the codes.  Must not be called
+ * during a run.  Errors: PVS_ERR_INVALID.
+ */
+pvs_status pvs_executor_set_group(pvs_executor* ex, int32_t group);
 
 pvs_status pvs_executor_stats_get(pvs_executor* ex, pvs_executor_stats* out);
 

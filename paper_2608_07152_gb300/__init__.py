@@ -93,7 +93,9 @@ class pvs_merge_stats_t(ctypes.Structure):
 
 class pvs_executor_stats_t(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in ("requests", "failed", "pages", "ranks")] + [
-        ("workers", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+        ("workers", ctypes.c_int32), ("group", ctypes.c_int32),
+        ("interval_passes", ctypes.c_int64), ("interval_ms", ctypes.c_double),
+        ("refined", ctypes.c_int64)]
 
 
 def _load() -> ctypes.CDLL:
@@ -163,6 +165,8 @@ def _load() -> ctypes.CDLL:
                                   ctypes.POINTER(eahr_stats)]),
         "pvs_executor_create": (i32, [P, i32, pp]),
         "pvs_executor_run": (i32, [P, P, P, i32, i32, i32, P, P, P, P]),
+        "pvs_executor_run_ex": (i32, [P, P, P, i32, i32, i32, i32, P, P, P, P]),
+        "pvs_executor_set_group": (i32, [P, i32]),
         "pvs_executor_stats_get": (i32, [P, ctypes.POINTER(pvs_executor_stats_t)]),
         "pvs_executor_destroy": (None, [P]),
     }
@@ -188,7 +192,8 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
             "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge",
-            "pvs_executor_create", "pvs_executor_run", "pvs_executor_stats_get",
+            "pvs_executor_create", "pvs_executor_run", "pvs_executor_run_ex",
+            "pvs_executor_set_group", "pvs_executor_stats_get",
             "pvs_executor_destroy")
 
 
@@ -807,10 +812,41 @@ def pvs_executor_run(ex, queries, ranks: int, page: int, snap=None, ids=None, sc
     return ids, scores, n_out, status, rc
 
 
+def pvs_executor_set_group(ex, group: int) -> None:
+    """Serve requests `group` at a time from one grouped pass over the codes."""
+    _check(_lib.pvs_executor_set_group(ex, int(group)), "pvs_executor_set_group")
+
+
+def pvs_executor_run_device(ex, queries, ranks: int, page: int, ids, scores, snap=None):
+    """pvs_executor_run with device-resident buffers: queries (CUDA float32
+    [nq, dim]), ids (CUDA int64 [nq, ranks]) and scores (CUDA float32 [nq,
+    ranks]), all contiguous on the index's device.  Returns (n_out [nq],
+    status [nq], rc) as host arrays."""
+    import torch
+    for t, dt, shape, what in ((queries, torch.float32, None, "queries"),
+                               (ids, torch.int64, None, "ids"),
+                               (scores, torch.float32, None, "scores")):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous() and
+                t.dtype == dt and t.dim() == 2):
+            raise ValueError(f"{what}: want a contiguous 2-D CUDA {dt} tensor")
+    nq = int(queries.shape[0])
+    if tuple(ids.shape) != (nq, ranks) or tuple(scores.shape) != (nq, ranks):
+        raise ValueError(f"ids and scores: want shape ({nq}, {ranks})")
+    n_out = np.zeros(nq, np.int32)
+    status = np.zeros(nq, np.int32)
+    rc = _lib.pvs_executor_run_ex(ex, snap, ctypes.c_void_p(queries.data_ptr()), nq, int(ranks),
+                                  int(page), 1, ctypes.c_void_p(ids.data_ptr()),
+                                  ctypes.c_void_p(scores.data_ptr()), n_out.ctypes.data,
+                                  status.ctypes.data)
+    if rc < 0 and not any(int(v) == rc for v in status):
+        raise PvsError(rc, "pvs_executor_run_ex")
+    return n_out, status, rc
+
+
 def pvs_executor_stats(ex) -> dict:
     st = pvs_executor_stats_t()
     _check(_lib.pvs_executor_stats_get(ex, ctypes.byref(st)), "pvs_executor_stats_get")
-    return {n: getattr(st, n) for n, _ in pvs_executor_stats_t._fields_ if n != "reserved"}
+    return {n: getattr(st, n) for n, _ in pvs_executor_stats_t._fields_}
 
 
 def pvs_executor_destroy(ex) -> None:

@@ -1587,9 +1587,15 @@ pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float*
     return (pvs_status)h_status;
 }
 
-pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
-                          int64_t* ids, float* scores, int32_t* n_out) {
-    DeviceGuard device_guard(first_cursor_device(cursors, nc));
+}  // extern "C"
+
+// The next n ranks of each of nc cursors (one index, one stream) in one set
+// of launches; cursor i's ranks go to ids[i][0 .. n) and scores[i][0 .. n)
+// (device or host per outputs_on_device).
+pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,
+                                int32_t outputs_on_device, int64_t* const* ids,
+                                float* const* scores, int32_t* n_out) {
+    DeviceGuard device_guard(first_cursor_device(const_cast<pvs_cursor**>(cursors), nc));
     if (!cursors || nc < 0 || n < 0 || !n_out || (nc > 0 && n > 0 && (!ids || !scores)))
         return PVS_ERR_INVALID;
     if (nc == 0) return PVS_OK;
@@ -1599,29 +1605,26 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
     for (int32_t i = 0; i < nc; ++i) {
         n_out[i] = 0;
         if (!cursors[i] || cursors[i]->index != x || cursors[i]->stream != st ||
-            cursors[i]->generator != PVS_GEN_INTERVALS)
+            cursors[i]->generator != PVS_GEN_INTERVALS || (n > 0 && (!ids[i] || !scores[i])))
             return PVS_ERR_INVALID;
     }
     for (int32_t i = 0; i < nc; ++i)
         if (cursors[i]->state < 0) return PVS_ERR_FAILED;
     const bool fused = n <= kPullFusedMax;
     if (!fused) {   // large pulls: one cursor at a time
-        pvs_status worst = PVS_OK;
         for (int32_t i = 0; i < nc; ++i) {
             pvs_status s = outputs_on_device
-                               ? pvs_next_device(cursors[i], n, ids + (int64_t)i * n,
-                                                 scores + (int64_t)i * n, &n_out[i])
-                               : pvs_next(cursors[i], n, ids + (int64_t)i * n,
-                                          scores + (int64_t)i * n, &n_out[i]);
+                               ? pvs_next_device(cursors[i], n, ids[i], scores[i], &n_out[i])
+                               : pvs_next(cursors[i], n, ids[i], scores[i], &n_out[i]);
             if (s < 0) return s;
         }
-        return worst;
+        return PVS_OK;
     }
     DevBuf buf(st, x->scratch_pool);   // released in stream order after the launches that read it
-    int64_t* d_ids = outputs_on_device ? ids : buf.get<int64_t>((size_t)nc * n);
-    float* d_scores = outputs_on_device ? scores : buf.get<float>((size_t)nc * n);
+    int64_t* d_ids = outputs_on_device ? nullptr : buf.get<int64_t>((size_t)nc * n);
+    float* d_scores = outputs_on_device ? nullptr : buf.get<float>((size_t)nc * n);
     PullArgs* d_args = buf.get<PullArgs>((size_t)nc);
-    if (!d_ids || !d_scores || !d_args) return PVS_ERR_OOM;
+    if ((!outputs_on_device && (!d_ids || !d_scores)) || !d_args) return PVS_ERR_OOM;
     std::vector<PullArgs> args;
     std::vector<int32_t> who;
     args.reserve(nc);
@@ -1645,8 +1648,8 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         a.n = (int)n_eff;
         a.cand = c->cand;
         a.keys = reinterpret_cast<unsigned long long*>(c->keys);
-        a.out_ids = d_ids + (int64_t)i * n;
-        a.out_scores = d_scores + (int64_t)i * n;
+        a.out_ids = outputs_on_device ? ids[i] : d_ids + (int64_t)i * n;
+        a.out_scores = outputs_on_device ? scores[i] : d_scores + (int64_t)i * n;
         a.status = c->d_status;
         a.ctr = c->ctr;
         a.front = nullptr;   // a few pulls per batch: a frontier would not pay for itself
@@ -1669,18 +1672,32 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         cursors[i]->pulls++;
         cursors[i]->fresh_ws = false;
     }
-    pvs_status result = PVS_OK;
     if (!outputs_on_device) {
-        PVS_CUDA(cudaMemcpyAsync(ids, d_ids, (size_t)nc * n * sizeof(int64_t),
-                                 cudaMemcpyDeviceToHost, st));
-        PVS_CUDA(cudaMemcpyAsync(scores, d_scores, (size_t)nc * n * sizeof(float),
-                                 cudaMemcpyDeviceToHost, st));
+        bool contiguous = true;   // rows i at ids[0] + i n: one copy each for ids and scores
+        for (int32_t i = 1; i < nc && contiguous; ++i)
+            contiguous = ids[i] == ids[0] + (int64_t)i * n && scores[i] == scores[0] + (int64_t)i * n;
+        if (contiguous) {
+            PVS_CUDA(cudaMemcpyAsync(ids[0], d_ids, (size_t)nc * n * sizeof(int64_t),
+                                     cudaMemcpyDeviceToHost, st));
+            PVS_CUDA(cudaMemcpyAsync(scores[0], d_scores, (size_t)nc * n * sizeof(float),
+                                     cudaMemcpyDeviceToHost, st));
+        } else {
+            for (int32_t i : who) {
+                PVS_CUDA(cudaMemcpyAsync(ids[i], d_ids + (int64_t)i * n,
+                                         (size_t)n_out[i] * sizeof(int64_t),
+                                         cudaMemcpyDeviceToHost, st));
+                PVS_CUDA(cudaMemcpyAsync(scores[i], d_scores + (int64_t)i * n,
+                                         (size_t)n_out[i] * sizeof(float),
+                                         cudaMemcpyDeviceToHost, st));
+            }
+        }
         std::vector<pvs_cursor*> pulled;
         for (int32_t i : who) pulled.push_back(cursors[i]);
         std::vector<int> dev_status(pulled.size(), 0);
         pvs_status s = gather_state(pulled.data(), (int)pulled.size(), st, dev_status.data(),
                                     nullptr);
         if (s != PVS_OK) return s;
+        pvs_status result = PVS_OK;
         for (size_t j = 0; j < pulled.size(); ++j)
             if (dev_status[j] != 0) result = fail(pulled[j], (pvs_status)dev_status[j]);
         if (result != PVS_OK) return result;
@@ -1690,6 +1707,22 @@ pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t o
         if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
     }
     return PVS_OK;
+}
+
+extern "C" {
+
+pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
+                          int64_t* ids, float* scores, int32_t* n_out) {
+    if (!cursors || nc < 0 || n < 0 || !n_out || (nc > 0 && n > 0 && (!ids || !scores)))
+        return PVS_ERR_INVALID;
+    std::vector<int64_t*> id_rows((size_t)std::max(nc, 1));
+    std::vector<float*> score_rows((size_t)std::max(nc, 1));
+    for (int32_t i = 0; i < nc; ++i) {
+        id_rows[(size_t)i] = ids ? ids + (int64_t)i * n : nullptr;
+        score_rows[(size_t)i] = scores ? scores + (int64_t)i * n : nullptr;
+    }
+    return pvs::next_batch_rows(cursors, nc, n, outputs_on_device, id_rows.data(),
+                                score_rows.data(), n_out);
 }
 
 static pvs_status next_common(pvs_cursor* c, int32_t n, int32_t* n_out, int64_t* n_eff) {

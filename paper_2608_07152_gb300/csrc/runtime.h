@@ -148,6 +148,11 @@ const SnapData* cursor_snapshot(const pvs_cursor* c);
 // its next pull) instead of copied out.
 pvs_status next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
                        int32_t* n_out);
+// pvs_next_batch with each cursor's outputs at its own address: cursor i's
+// next n ranks to ids[i], scores[i] (device or host per outputs_on_device).
+pvs_status next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,
+                           int32_t outputs_on_device, int64_t* const* ids, float* const* scores,
+                           int32_t* n_out);
 // Open nq <= kGroupMax cursors whose bounds come from one grouped interval
 // pass on pass_stream (null: the index's stream); cursor i's later work runs
 // on cursor_streams[i] (null array or entry: pass_stream).

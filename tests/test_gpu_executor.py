@@ -152,3 +152,72 @@ def test_executor_argument_errors():
     finally:
         pvs.pvs_index_free(other)
         pvs.pvs_index_free(index)
+
+
+@pytest.mark.parametrize("group,workers", [(8, 3), (3, 2), (5, 1)])
+def test_grouped_requests_equal_the_oracle_ranking(group, workers):
+    """Requests served `group` at a time share one pass over the codes
+    (pvs_cursor_open_group) and one batched pull per page; every request's
+    ranks are still the oracle's."""
+    V, Q = _mixture(9_001, 96, 23, seed=300 + group)
+    index = pvs.pvs_build(V)
+    try:
+        ex = pvs.pvs_executor_create(index, workers)
+        try:
+            pvs.pvs_executor_set_group(ex, group)
+            ids, sc, n_out, status, rc = pvs.pvs_executor_run(ex, Q, 300, 20)
+            st = pvs.pvs_executor_stats(ex)
+        finally:
+            pvs.pvs_executor_destroy(ex)
+    finally:
+        pvs.pvs_index_free(index)
+    assert rc == pvs.PVS_OK and np.all(status == pvs.PVS_OK)
+    _check_rows(V, Q, ids, sc, n_out, 300)
+    assert st["group"] == group and st["interval_passes"] == -(-23 // group)
+    assert st["requests"] == 23 and st["failed"] == 0 and st["ranks"] == 23 * 300
+    assert st["interval_ms"] > 0 and st["refined"] >= 23 * 300
+
+
+@pytest.mark.parametrize("group", [1, 8])
+def test_device_buffers_grouped_and_not(group):
+    V, Q = _mixture(12_345, 128, 19, seed=400 + group)
+    index = pvs.pvs_build(V)
+    try:
+        ex = pvs.pvs_executor_create(index, 4)
+        try:
+            pvs.pvs_executor_set_group(ex, group)
+            q = torch.from_numpy(Q).cuda()
+            ids = torch.zeros((19, 250), dtype=torch.int64, device="cuda")
+            sc = torch.zeros((19, 250), dtype=torch.float32, device="cuda")
+            n_out, status, rc = pvs.pvs_executor_run_device(ex, q, 250, 20, ids, sc)
+        finally:
+            pvs.pvs_executor_destroy(ex)
+    finally:
+        pvs.pvs_index_free(index)
+    assert rc == pvs.PVS_OK and np.all(status == pvs.PVS_OK)
+    _check_rows(V, Q, ids.cpu().numpy(), sc.cpu().numpy(), n_out, 250)
+
+
+def test_grouped_requests_with_exhaustion_and_a_failed_query():
+    V, Q = _mixture(61, 32, 17, seed=15, comps=4)
+    index = pvs.pvs_build(V)
+    try:
+        ex = pvs.pvs_executor_create(index, 2)
+        try:
+            pvs.pvs_executor_set_group(ex, 8)
+            _, _, n_out, status, rc = pvs.pvs_executor_run(ex, Q, 80, 9)
+            assert rc == pvs.PVS_OK and np.all(status == pvs.PVS_EXHAUSTED)
+            ids, sc, n_out, status, rc = pvs.pvs_executor_run(ex, Q, 80, 9)
+            _check_rows(V, Q, ids, sc, n_out, 80)
+            bad = Q.copy()
+            bad[9, 1] = np.inf        # the second group's open fails; its others go on
+            ids, sc, n_out, status, rc = pvs.pvs_executor_run(ex, bad, 80, 9)
+            assert status[9] == pvs.PVS_ERR_NONFINITE and rc == pvs.PVS_ERR_NONFINITE
+            assert n_out[9] == 0 and np.all(ids[9] == -1)
+            _check_rows(V, Q, ids, sc, n_out, 80, rows=[i for i in range(17) if i != 9])
+            with pytest.raises(pvs.PvsError):
+                pvs.pvs_executor_set_group(ex, 9)
+        finally:
+            pvs.pvs_executor_destroy(ex)
+    finally:
+        pvs.pvs_index_free(index)

@@ -1,8 +1,10 @@
 """Parity at full size and in deep pulls, through the C ABI.
 
 * Passage scale (8,841,823 x 768, the mixture corpus of the benchmark), in
-  the launch configuration the benchmark times: one cursor on its own stream,
-  50 pulls of 20 ranks into device buffers.  The oracle cannot rank 8.8M rows
+  the launch configuration the benchmark times -- the native executor with
+  four workers, eight queries per grouped pass over the codes, 50 batched
+  pulls of 20 ranks into device buffers -- and for a lone cursor on its own
+  stream (the latency figures' path).  The oracle cannot rank 8.8M rows
   in a test, so it checks what it can compute one by one and what holds at
   any size (Sec. 2.1, 2.3.1, App. A.1):
     - every emitted score equals the oracle's exact score of that row;
@@ -30,7 +32,8 @@ N_PASSAGE = 8_841_823
 DIM = 768
 
 
-def test_passage_scale_pulls_in_the_benchmark_configuration():
+@pytest.fixture(scope="module")
+def passage():
     dev = torch.device("cuda")
     centres = synth.mixture_centres(4096, DIM, seed=2, device=dev)
     rows = torch.empty((N_PASSAGE, DIM), dtype=torch.float32, device=dev)
@@ -38,67 +41,119 @@ def test_passage_scale_pulls_in_the_benchmark_configuration():
         c = min(1 << 20, N_PASSAGE - r)
         rows[r:r + c] = synth.mixture_rows(c, centres, 0.35, seed=2, first=r)
     index = pvs.pvs_build(rows)
+    try:
+        yield dev, centres, rows, index
+    finally:
+        pvs.pvs_index_free(index)
+
+
+def _check_prefix(rows, dev, qh, ids, sc, sample):
+    """The three checks of a first-1,000 prefix that the oracle can make at
+    this size: exact scores of the emitted rows, (score desc, id asc) order,
+    and nothing of a row sample outside the prefix ahead of its last rank."""
+    V_ids = rows[torch.from_numpy(ids).to(dev)].cpu().numpy()
+    ref = np.array([po.exact_score_one(qh, v) for v in V_ids], np.float32)
+    assert np.array_equal(sc.view(np.uint32), ref.view(np.uint32))
+    key = list(zip((-sc.astype(np.float64)).tolist(), ids.tolist()))
+    assert key == sorted(key)
+    assert len(set(ids.tolist())) == ids.size
+    Vs = rows[torch.from_numpy(sample).to(dev)].cpu().numpy()
+    s_sample = po.exact_scores(qh, Vs)
+    emitted = set(ids.tolist())
+    last_s, last_id = float(sc[-1]), int(ids[-1])
+    for i, s in zip(sample.tolist(), s_sample.tolist()):
+        if i not in emitted:
+            assert s < last_s or (s == last_s and i > last_id), i
+    return s_sample
+
+
+def test_passage_scale_grouped_executor_in_the_benchmark_configuration(passage):
+    dev, centres, rows, index = passage
+    Q = synth.mixture_queries(16, centres, 0.5, seed=3).contiguous()
+    ids_t = torch.empty((16, 1000), dtype=torch.int64, device=dev)
+    sc_t = torch.empty((16, 1000), dtype=torch.float32, device=dev)
+    ex = pvs.pvs_executor_create(index, 4)
+    try:
+        pvs.pvs_executor_set_group(ex, 8)
+        n_out, status, rc = pvs.pvs_executor_run_device(ex, Q, 1000, 20, ids_t, sc_t)
+        st = pvs.pvs_executor_stats(ex)
+    finally:
+        pvs.pvs_executor_destroy(ex)
+    assert rc == pvs.PVS_OK and np.all(n_out == 1000)
+    assert st["interval_passes"] == 2          # two groups of eight, one pass each
+    ids_all, sc_all = ids_t.cpu().numpy(), sc_t.cpu().numpy()
+    Qh = Q.cpu().numpy()
+    rng = np.random.default_rng(6)
+    base = rng.integers(0, N_PASSAGE, 50_000)
+    for i in range(16):
+        sample = np.unique(np.concatenate([base, ids_all[i]]))
+        _check_prefix(rows, dev, Qh[i], ids_all[i], sc_all[i], sample)
+    # the grouped pass's bounds of a row sample: the oracle's, for each query
+    first = np.unique(rng.integers(0, N_PASSAGE, 3000))
+    Qs = po.quantize(rows[torch.from_numpy(first).to(dev)].cpu().numpy())
+    curs = pvs.pvs_cursor_open_group(index, Q[:8])
+    try:
+        for i, cur in enumerate(curs):
+            lo = np.empty(first.size, np.float32)
+            hi = np.empty(first.size, np.float32)
+            for k, r in enumerate(first.tolist()):
+                l, h = pvs.pvs_cursor_bounds(cur, int(r), 1)
+                lo[k], hi[k] = l[0], h[0]
+            ref_lo, ref_hi = po.intervals(po.encode_query(Qh[i]), Qs, DIM)
+            assert np.array_equal(lo.view(np.uint32), ref_lo.view(np.uint32))
+            assert np.array_equal(hi.view(np.uint32), ref_hi.view(np.uint32))
+    finally:
+        for cur in curs:
+            pvs.pvs_cursor_close(cur)
+
+
+def test_passage_scale_lone_cursor(passage):
+    dev, centres, rows, index = passage
     q = synth.mixture_queries(1, centres, 0.5, seed=3)[0].contiguous()
     side = torch.cuda.Stream()
     ids_t = torch.empty(1000, dtype=torch.int64, device=dev)
     sc_t = torch.empty(1000, dtype=torch.float32, device=dev)
+    cur = pvs.pvs_cursor_open(index, q)
+    pvs.pvs_cursor_set_stream(cur, side)
     try:
-        cur = pvs.pvs_cursor_open(index, q)
-        pvs.pvs_cursor_set_stream(cur, side)
-        try:
-            for p in range(50):
-                n_out, _ = pvs.pvs_next_device(cur, 20, ids_t[20 * p:], sc_t[20 * p:])
-                assert n_out == 20
-            assert pvs.pvs_cursor_sync(cur) >= 0
-            side.synchronize()
-            ids = ids_t.cpu().numpy()
-            sc = sc_t.cpu().numpy()
-            rng = np.random.default_rng(5)
-            sample = np.unique(np.concatenate([rng.integers(0, N_PASSAGE, 100_000), ids]))
-            lo, hi = [], []
-            for i in sample[:4096]:      # bounds of a sample (ids sorted; contiguous reads)
-                l, h = pvs.pvs_cursor_bounds(cur, int(i), 1)
-                lo.append(l[0])
-                hi.append(h[0])
-        finally:
-            pvs.pvs_cursor_close(cur)
-        qh = q.cpu().numpy()
-        V_ids = rows[torch.from_numpy(ids).to(dev)].cpu().numpy()
-        # 1. emitted scores are the exact scores of those rows
-        ref = np.array([po.exact_score_one(qh, v) for v in V_ids], np.float32)
-        assert np.array_equal(sc.view(np.uint32), ref.view(np.uint32))
-        # 2. order: score desc, id asc
-        key = list(zip((-sc.astype(np.float64)).tolist(), ids.tolist()))
-        assert key == sorted(key)
-        assert len(set(ids.tolist())) == 1000
-        # 3. completeness on a sample: nothing outside the prefix beats rank 1,000
-        Vs = rows[torch.from_numpy(sample).to(dev)].cpu().numpy()
-        s_sample = po.exact_scores(qh, Vs)
-        emitted = set(ids.tolist())
-        last_s, last_id = float(sc[-1]), int(ids[-1])
-        for i, s in zip(sample.tolist(), s_sample.tolist()):
-            if i not in emitted:
-                assert s < last_s or (s == last_s and i > last_id), i
-        # 4. intervals of sampled rows: the oracle's (or, for a row already
-        # refined, lo == hi == its exact score; -inf once delivered), and sound
-        qe = po.encode_query(qh)
-        first = sample[:4096]
-        Qs = po.quantize(rows[torch.from_numpy(first).to(dev)].cpu().numpy())
-        ref_lo, ref_hi = po.intervals(qe, Qs, DIM)
-        lo = np.array(lo, np.float32)
-        hi = np.array(hi, np.float32)
-        s_first = s_sample[np.searchsorted(sample, first)]
-        for k, i in enumerate(first.tolist()):
-            if i in emitted:
-                assert lo[k] == -np.inf and hi[k] == -np.inf
-            elif lo[k] == hi[k]:
-                assert lo[k].view(np.uint32) == s_first[k].view(np.uint32)
-            else:
-                assert lo[k].view(np.uint32) == ref_lo[k].view(np.uint32)
-                assert hi[k].view(np.uint32) == ref_hi[k].view(np.uint32)
-        assert np.all(ref_lo <= s_first) and np.all(s_first <= ref_hi)
+        for p in range(50):
+            n_out, _ = pvs.pvs_next_device(cur, 20, ids_t[20 * p:], sc_t[20 * p:])
+            assert n_out == 20
+        assert pvs.pvs_cursor_sync(cur) >= 0
+        side.synchronize()
+        ids = ids_t.cpu().numpy()
+        sc = sc_t.cpu().numpy()
+        rng = np.random.default_rng(5)
+        sample = np.unique(np.concatenate([rng.integers(0, N_PASSAGE, 100_000), ids]))
+        lo, hi = [], []
+        for i in sample[:4096]:      # bounds of a sample (ids sorted; contiguous reads)
+            l, h = pvs.pvs_cursor_bounds(cur, int(i), 1)
+            lo.append(l[0])
+            hi.append(h[0])
     finally:
-        pvs.pvs_index_free(index)
+        pvs.pvs_cursor_close(cur)
+    qh = q.cpu().numpy()
+    # 1-3. exact scores, order, completeness on a sample
+    s_sample = _check_prefix(rows, dev, qh, ids, sc, sample)
+    emitted = set(ids.tolist())
+    # 4. intervals of sampled rows: the oracle's (or, for a row already
+    # refined, lo == hi == its exact score; -inf once delivered), and sound
+    qe = po.encode_query(qh)
+    first = sample[:4096]
+    Qs = po.quantize(rows[torch.from_numpy(first).to(dev)].cpu().numpy())
+    ref_lo, ref_hi = po.intervals(qe, Qs, DIM)
+    lo = np.array(lo, np.float32)
+    hi = np.array(hi, np.float32)
+    s_first = s_sample[np.searchsorted(sample, first)]
+    for k, i in enumerate(first.tolist()):
+        if i in emitted:
+            assert lo[k] == -np.inf and hi[k] == -np.inf
+        elif lo[k] == hi[k]:
+            assert lo[k].view(np.uint32) == s_first[k].view(np.uint32)
+        else:
+            assert lo[k].view(np.uint32) == ref_lo[k].view(np.uint32)
+            assert hi[k].view(np.uint32) == ref_hi[k].view(np.uint32)
+    assert np.all(ref_lo <= s_first) and np.all(s_first <= ref_hi)
 
 
 @pytest.mark.parametrize("tau", [0.0, -0.5])

@@ -532,3 +532,38 @@ def test_first_working_set_from_per_slot_bounds(crowded):
     assert np.array_equal(ids, ref_ids[:1000])
     assert np.array_equal(sc.view(np.uint32), ref_sc[:1000].view(np.uint32))
     assert st["interval_passes"] == 1
+
+
+@pytest.mark.parametrize("tau", [0.5, 0.0])
+def test_frozen_scheduler_over_a_pvs_cursor(tau):
+    """Sec. 3.5's frozen scheduler (EAHR_POLICY_FROZEN) driving a real dense
+    cursor: the ordered Top-20 equals complete-list fusion, and every pull of
+    either list reads one 16-rank step (the last pull of a list that runs out
+    may read fewer)."""
+    n, m = 30_000, 64
+    centres = synth.mixture_centres(64, m, seed=80, device="cpu")
+    V = synth.mixture_rows(n, centres, 0.35, seed=81).numpy()
+    q = synth.mixture_queries(1, centres, 0.5, seed=82).numpy()[0]
+    dense_ids, dense_sc = po.dense_ranking(q, V)
+    proxy = torch.from_numpy(dense_sc[np.argsort(dense_ids)].astype(np.float64))
+    sparse = synth.copula_ranking(proxy, tau, seed=83).numpy()
+    T = ro.target_topk_large([dense_ids, sparse], [1, 1], 60, 20, ro.NUMERATOR)
+    index = pvs.pvs_build(V)
+    try:
+        cur = pvs.pvs_cursor_open(index, q)
+        try:
+            ids, F, st = pvs.eahr_topk(cur, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                       policy=pvs.EAHR_POLICY_FROZEN, step=16)
+        finally:
+            pvs.pvs_cursor_close(cur)
+    finally:
+        pvs.pvs_index_free(index)
+    assert ids.tolist() == [x for x, _ in T]
+    for (x, f), got in zip(T, F):
+        if not np.isnan(got):
+            assert got == ro.as_float(f)
+    for i in range(2):
+        d, p = st["depth"][i], st["pulls"][i]
+        assert p >= 1 and 16 * (p - 1) < d <= 16 * p
+        if not st["exhausted"][i]:
+            assert d == 16 * p
