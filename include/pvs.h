@@ -80,7 +80,8 @@ typedef struct pvs_stats {
     int64_t exact_fallbacks;  /* evaluations that needed the exact accumulator */
     int64_t interval_passes;  /* full passes over the Int8 codes               */
     int64_t horizon_builds;   /* candidate-set (re)builds from the bounds      */
-    int64_t pulls;            /* pvs_next / pvs_next_device calls              */
+    int64_t pulls;            /* device pulls (a call served from ranks computed
+                                 ahead of it needs none)                       */
     int64_t candidates;       /* candidate entries certified over all pulls    */
     int64_t code_bytes;       /* bytes of codes + per-vector params scanned    */
     int32_t state;            /* PVS_OK (Open), PVS_EXHAUSTED, or the failure  */
@@ -239,6 +240,14 @@ pvs_status pvs_cursor_open_group(pvs_index* index, const pvs_snapshot* snap,
 pvs_status pvs_next_batch(pvs_cursor** cursors, int32_t nc, int32_t n, int32_t outputs_on_device,
                           int64_t* ids, float* scores, int32_t* n_out);
 
+/* Read-ahead: a pull of n <= 256 ranks computes up to `pages` x n of them
+ * (at most 256; default 4) and keeps the ones not asked for in the cursor,
+ * so the next calls are served without device work (host outputs) or by a
+ * copy (device outputs).  Exact either way (Sec. 2.1: the list is a stable
+ * prefix, so a rank computed early is the rank delivered later).  pages = 1
+ * computes exactly what is asked.  Errors: PVS_ERR_INVALID (pages < 1). */
+pvs_status pvs_cursor_set_readahead(pvs_cursor* cursor, int32_t pages);
+
 /* Deliver the next n exact ranks (Sec. 2.1: a stable exact prefix that is
  * only ever extended).  ids (int64) and scores (the authoritative float32
  * scores: the correctly rounded value of the exact inner product) are HOST
@@ -298,7 +307,8 @@ void pvs_cursor_close_batch(pvs_cursor** cursors, int32_t nc);
 /* Diagnostics.  Copy to host the score interval [lo, hi] that the cursor
  * holds for ids first .. first+count-1 of its snapshot: the App. A.1 interval
  * before an item is scored, lo == hi == its authoritative score after, and
- * -inf once the item is delivered or if it is deleted.  Runs the interval
+ * -inf once the item is delivered or computed ahead of the caller (read-ahead,
+ * pvs_cursor_set_readahead) or if it is deleted.  Runs the interval
  * pass first if no pull has run it yet. */
 pvs_status pvs_cursor_bounds(pvs_cursor* cursor, int64_t first, int64_t count, float* lo,
                              float* hi);

@@ -140,6 +140,7 @@ def _load() -> ctypes.CDLL:
         "pvs_rank_exact_noalloc": (i32, [P, P, i32, i32, i32, P, P, P]),
         "pvs_index_import": (i32, [P, P, P, P, P, i64, i32, P, pp]),
         "pvs_cursor_open_group": (i32, [P, P, P, i32, i32, P, P, P]),
+        "pvs_cursor_set_readahead": (i32, [P, i32]),
         "pvs_index_set_wait_limit": (i32, [P, i64]),
         "eahr_topk": (i32, [P, P, i64, ctypes.POINTER(eahr_params), P, P, P,
                             ctypes.POINTER(eahr_stats)]),
@@ -187,7 +188,8 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pvs_cursor_stats", "pvs_cursor_bounds", "pvs_cursor_score_ids", "pvs_cursor_close",
             "pvs_cursor_sync_batch", "pvs_cursor_stats_batch", "pvs_cursor_close_batch",
             "pvs_status_string", "pvs_launch_count", "pvs_rank_exact_noalloc",
-            "pvs_index_import", "pvs_index_set_wait_limit", "pvs_cursor_open_group", "eahr_topk",
+            "pvs_index_import", "pvs_index_set_wait_limit", "pvs_cursor_open_group",
+            "pvs_cursor_set_readahead", "eahr_topk",
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
             "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
@@ -448,6 +450,10 @@ def pvs_cursor_sync(cursor) -> int:
 def pvs_cursor_set_generator(cursor, generator: int) -> None:
     """PVS_GEN_INTERVALS (default) or PVS_GEN_FULL_SCAN, before the first pull."""
     _check(_lib.pvs_cursor_set_generator(cursor, int(generator)), "pvs_cursor_set_generator")
+
+
+def pvs_cursor_set_readahead(cursor, pages: int) -> None:
+    _check(_lib.pvs_cursor_set_readahead(cursor, int(pages)), "pvs_cursor_set_readahead")
 
 
 def pvs_cursor_set_stream(cursor, stream) -> None:

@@ -83,6 +83,19 @@ cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t s
 // refines and emits (one cluster per cursor in the batch form).
 cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st);
 cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st);
+// dev[0 .. n) = host[0 .. n), in stream order, the host array read at launch.
+cudaError_t launch_stage_pull_args(const PullArgs* host, int n, PullArgs* dev, cudaStream_t st);
+// Ranks computed ahead, handed to the callers' buffers: for every entry,
+// count ids and scores from src to dst (device or pinned host memory), in
+// stream order, one launch per 64 entries (the entries are read at launch).
+struct RankCopy {
+    const int64_t* src_ids;
+    const float* src_scores;
+    int64_t* dst_ids;
+    float* dst_scores;
+    int count;
+};
+cudaError_t launch_copy_ranks(const RankCopy* host, int n, cudaStream_t st);
 cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
                               int m_raw, cudaStream_t st);
 cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
@@ -208,6 +221,28 @@ struct IntervalGroupArgs {
 // True when a grouped pass serves nq queries over rows of m_pad bytes.
 bool interval_group_supported(int m_pad, int nq);
 cudaError_t launch_interval_group(const IntervalGroupArgs& a, int num_sms, cudaStream_t st);
+
+// First working sets of the n <= kGroupMax cursors of a grouped pass, in four
+// launches for all of them (grid dimension y = the cursor): per cursor g the
+// k[g]-th largest of its slot_n per-slot lower bounds (select_small), then the
+// ordered compaction of its rows with key(hi) >= that threshold
+// (launch_compact_ordered's count, scan and scatter).
+struct WsGroupArgs {
+    int n;
+    int64_t rows;
+    int64_t slot_n;
+    const float* slot[kGroupMax];
+    uint64_t k[kGroupMax];
+    SelectState* sel[kGroupMax];
+    const float* lo[kGroupMax];
+    const float* hi[kGroupMax];
+    int32_t* w_id[kGroupMax];
+    float* w_lo[kGroupMax];
+    float* w_hi[kGroupMax];
+    unsigned int* w_len[kGroupMax];
+    unsigned int* scratch[kGroupMax];   // compact_scratch_elems(rows) each
+};
+cudaError_t launch_ws_group(const WsGroupArgs& a, cudaStream_t st);
 int64_t interval_group_slots(int64_t rows, int m_pad, int nq, int num_sms,
                              int64_t* min_rows_per_slot);
 

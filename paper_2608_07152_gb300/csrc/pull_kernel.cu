@@ -759,6 +759,60 @@ cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
     return cudaGetLastError();
 }
 
+// Per-cursor arguments of a batched pull written to device memory in stream
+// order by a kernel that receives them as parameters: the host's copy of
+// the arguments is captured at launch, so neither a pageable copy (which
+// can wait for the stream) nor a reused pinned buffer (which the next pull
+// could overwrite before the copy runs) is involved.
+constexpr int kArgsPerStage = 64;
+struct PullArgsPack {
+    PullArgs a[kArgsPerStage];
+};
+
+__global__ void stage_pull_args_kernel(const __grid_constant__ PullArgsPack p, int count,
+                                       PullArgs* out) {
+    for (int i = threadIdx.x; i < count; i += blockDim.x) out[i] = p.a[i];
+}
+
+cudaError_t launch_stage_pull_args(const PullArgs* host, int n, PullArgs* dev, cudaStream_t st) {
+    for (int first = 0; first < n; first += kArgsPerStage) {
+        const int count = n - first < kArgsPerStage ? n - first : kArgsPerStage;
+        PullArgsPack p;
+        for (int i = 0; i < count; ++i) p.a[i] = host[first + i];
+        count_launches(1);
+        stage_pull_args_kernel<<<1, 64, 0, st>>>(p, count, dev + first);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+constexpr int kCopiesPerLaunch = 64;
+struct RankCopyPack {
+    RankCopy e[kCopiesPerLaunch];
+};
+
+__global__ void copy_ranks_kernel(const __grid_constant__ RankCopyPack p) {
+    const RankCopy& e = p.e[blockIdx.x];
+    for (int i = threadIdx.x; i < e.count; i += blockDim.x) {
+        e.dst_ids[i] = e.src_ids[i];
+        e.dst_scores[i] = e.src_scores[i];
+    }
+}
+
+cudaError_t launch_copy_ranks(const RankCopy* host, int n, cudaStream_t st) {
+    for (int first = 0; first < n; first += kCopiesPerLaunch) {
+        const int count = n - first < kCopiesPerLaunch ? n - first : kCopiesPerLaunch;
+        RankCopyPack p;
+        for (int i = 0; i < count; ++i) p.e[i] = host[first + i];
+        count_launches(1);
+        copy_ranks_kernel<<<count, 128, 0, st>>>(p);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
 cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
     count_launches(1);

@@ -37,7 +37,7 @@ SnapData::~SnapData() {
 }
 
 int64_t cursor_visible(const pvs_cursor* c) { return c->visible; }
-int64_t cursor_emitted(const pvs_cursor* c) { return c->emitted; }
+int64_t cursor_emitted(const pvs_cursor* c) { return c->emitted - c->ahead; }
 const SnapData* cursor_snapshot(const pvs_cursor* c) { return c->snap.get(); }
 
 }  // namespace pvs
@@ -233,6 +233,9 @@ void cursor_reset(pvs_cursor* c) {
     c->pulls = c->interval_passes = c->horizon_builds = c->candidates = 0;
     c->code_bytes = 0;
     c->group_size = 1;
+    c->ahead = c->ahead_pos = 0;
+    c->ahead_host = false;
+    c->readahead = 4;
     c->batch_passes = 0;
     c->batch_ms = 0.0;
     c->ev_pending = false;
@@ -244,8 +247,11 @@ void cursor_reset(pvs_cursor* c) {
 }
 
 // Closed cursors kept per index for reuse: at most kCursorPool of them and
-// kCursorPoolBytes of device buffers (batched opens reuse hundreds of small
-// cursors; single-query cursors hold buffers for every row).
+// a quarter of the device's memory (at least kCursorPoolBytes) in device
+// buffers.  Batched opens reuse hundreds of small cursors; single-query
+// cursors hold buffers for every row (~460 MB at 8.8M rows), and grouped
+// opens keep dozens of them in flight: a cursor that is not pooled frees its
+// buffers, and cudaFree waits for the whole device.
 constexpr size_t kCursorPool = 1024;
 constexpr size_t kCursorPoolBytes = size_t(4) << 30;
 
@@ -456,6 +462,59 @@ pvs_status build_working_set(pvs_cursor* c, int64_t want) {
     c->fresh_ws = true;
     // new indices: no frontier, default hint (front_k and front_hint are adjacent)
     PVS_CUDA(cudaMemsetAsync(&c->ctr->front_k, 0, 2 * sizeof(unsigned int), c->stream));
+    return PVS_OK;
+}
+
+// The first working sets of the cursors of one stream that are due for
+// one from their pass's per-slot lower bounds (build_working_set's first
+// case), built together: four launches for all of them instead of four per
+// cursor.  Cursors of one grouped pass share rows and slot count.  Cursors
+// that do not qualify are left to prepare_pull.
+// pulls[i]: the ranks cursor i's next pull computes (0: no pull).
+pvs_status build_first_working_sets(pvs_cursor* const* cs, int32_t nc, const int64_t* pulls) {
+    WsGroupArgs a;
+    a.n = 0;
+    pvs_cursor* picked[kGroupMax];
+    int64_t H_of[kGroupMax];
+    for (int32_t i = 0; i < nc && a.n < kGroupMax; ++i) {
+        pvs_cursor* c = cs[i];
+        if (c->state != PVS_OK || c->batch_ws || !c->scanned || !c->slot_fresh) continue;
+        const int64_t n_eff = pulls[i];
+        if (n_eff <= 0 || c->emitted + n_eff - c->horizon_base <= c->horizon) continue;
+        const int64_t remaining = c->visible - c->emitted;
+        const int64_t H = std::min<int64_t>(std::max<int64_t>({n_eff, 2 * c->horizon, 2048}),
+                                            remaining);
+        if (H >= remaining || H > c->slot_n) continue;
+        if (a.n > 0 && (c->rows != a.rows || c->slot_n != a.slot_n)) continue;
+        a.rows = c->rows;
+        a.slot_n = c->slot_n;
+        a.slot[a.n] = c->slot_top;
+        a.k[a.n] = (uint64_t)H;
+        a.sel[a.n] = c->sel;
+        a.lo[a.n] = c->lo;
+        a.hi[a.n] = c->hi;
+        a.w_id[a.n] = c->w_id;
+        a.w_lo[a.n] = c->w_lo;
+        a.w_hi[a.n] = c->w_hi;
+        a.w_len[a.n] = &c->ctr->w_len;
+        a.scratch[a.n] = c->compact_scratch;
+        picked[a.n] = c;
+        H_of[a.n] = H;
+        ++a.n;
+    }
+    if (a.n < 2) return PVS_OK;   // prepare_pull builds a lone one
+    cudaStream_t st = picked[0]->stream;
+    PVS_CUDA(launch_ws_group(a, st));
+    for (int i = 0; i < a.n; ++i) {
+        pvs_cursor* c = picked[i];
+        c->slot_fresh = false;
+        c->horizon = H_of[i];
+        c->horizon_base = c->emitted;
+        c->horizon_builds++;
+        c->fresh_ws = true;
+        // new indices: no frontier, default hint (front_k and front_hint are adjacent)
+        PVS_CUDA(cudaMemsetAsync(&c->ctr->front_k, 0, 2 * sizeof(unsigned int), st));
+    }
     return PVS_OK;
 }
 
@@ -1053,6 +1112,11 @@ pvs_status index_create(int32_t dim, void* cuda_stream, pvs_index** out) {
     x->m = dim;
     x->m_pad = (int)round_up(dim, kCodeAlign);
     x->m_raw = (int)round_up(dim, 4);
+    {
+        size_t free_b = 0, total_b = 0;
+        if (cudaMemGetInfo(&free_b, &total_b) != cudaSuccess) return bail(PVS_ERR_CUDA);
+        x->pool_limit = std::max(kCursorPoolBytes, total_b / 4);
+    }
     if (cuda_stream) {
         x->stream = static_cast<cudaStream_t>(cuda_stream);
     } else {
@@ -1366,6 +1430,13 @@ pvs_status pvs::cursor_open_on(pvs_index* x, const pvs_snapshot* snap, const flo
 
 static_assert(pvs::kGroupMax == PVS_GROUP_MAX, "group size of the C ABI");
 
+// SMs left free of the grouped pass.  Measured at 8.8M x 768 with eight
+// queries per pass and eight groups in flight (ranks/s; pass ms): 0 SMs
+// 4.78M (1.24 ms), 16 4.80M (1.19), 32 5.19M (1.22), 48 5.26M (1.29), 56
+// 5.54M (1.40), 64 5.17M (1.51), 80 4.31M (1.82); 32 keeps the pass near
+// the HBM roofline.
+constexpr int kGroupReserveSms = 32;
+
 namespace {
 
 // One grouped interval pass for the nq (>= 2) freshly opened cursors cs[],
@@ -1382,8 +1453,12 @@ pvs_status group_pass(pvs_index* x, pvs_cursor* const* cs, int nq, cudaStream_t 
     a.m_pad = x->m_pad;
     a.nq = nq;
     a.wait_ns = x->wait_ns;
+    // the pass runs on all but kGroupReserveSms SMs: pulls and working-set
+    // builds of other groups run beside it (the pass's shared memory and
+    // registers leave no room for them on its own SMs)
+    const int pass_sms = std::max(x->num_sms / 2, x->num_sms - kGroupReserveSms);
     int64_t min_rows = 0;
-    const int64_t slots = interval_group_slots(a.rows, x->m_pad, nq, x->num_sms, &min_rows);
+    const int64_t slots = interval_group_slots(a.rows, x->m_pad, nq, pass_sms, &min_rows);
     const bool use_slots = slots > 0 && a.tomb == nullptr && min_rows >= kSlotTop;
     for (int i = 0; i < nq; ++i) {
         pvs_cursor* c = cs[i];
@@ -1420,7 +1495,7 @@ pvs_status group_pass(pvs_index* x, pvs_cursor* const* cs, int nq, cudaStream_t 
         else
             PVS_CUDA(cudaStreamWaitEvent(ps, x->pass_done, 0));
         for (int i = 0; i < nq; ++i) PVS_CUDA(cudaEventRecord(cs[i]->ev_begin, ps));
-        PVS_CUDA(launch_interval_group(a, x->num_sms, ps));
+        PVS_CUDA(launch_interval_group(a, pass_sms, ps));
         for (int i = 0; i < nq; ++i) PVS_CUDA(cudaEventRecord(cs[i]->ev_end, ps));
         PVS_CUDA(cudaEventRecord(x->pass_done, ps));
     }
@@ -1592,6 +1667,21 @@ pvs_status pvs_batch_bounds(pvs_index* x, const pvs_snapshot* snap, const float*
 // The next n ranks of each of nc cursors (one index, one stream) in one set
 // of launches; cursor i's ranks go to ids[i][0 .. n) and scores[i][0 .. n)
 // (device or host per outputs_on_device).
+// The cursor's state after a delivery: Exhausted once the caller has every rank.
+static pvs_status delivery_state(pvs_cursor* c) {
+    if (c->state >= 0 && c->emitted - c->ahead == c->visible) c->state = PVS_EXHAUSTED;
+    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+}
+
+// Ranks a pull computes for a request of `need` while nothing is ahead: up
+// to `readahead` times the request (at most one fused launch's worth, and
+// never past the list's end); large requests exactly.
+static int64_t pull_size(const pvs_cursor* c, int64_t need, int32_t readahead) {
+    if (need > kPullFusedMax) return need;
+    const int64_t want = std::min<int64_t>(kPullFusedMax, need * std::max<int32_t>(1, readahead));
+    return std::min<int64_t>(std::max(want, need), c->visible - c->emitted);
+}
+
 pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,
                                 int32_t outputs_on_device, int64_t* const* ids,
                                 float* const* scores, int32_t* n_out) {
@@ -1610,8 +1700,7 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
     }
     for (int32_t i = 0; i < nc; ++i)
         if (cursors[i]->state < 0) return PVS_ERR_FAILED;
-    const bool fused = n <= kPullFusedMax;
-    if (!fused) {   // large pulls: one cursor at a time
+    if (n > kPullFusedMax) {   // large pulls: one cursor at a time
         for (int32_t i = 0; i < nc; ++i) {
             pvs_status s = outputs_on_device
                                ? pvs_next_device(cursors[i], n, ids[i], scores[i], &n_out[i])
@@ -1620,20 +1709,56 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
         }
         return PVS_OK;
     }
+    // per cursor: the ranks delivered now, first from those computed ahead
+    // (take), then from this call's pull (rest), which computes pulls[i]
+    std::vector<int64_t> take((size_t)nc), rest((size_t)nc), pulls((size_t)nc);
+    std::vector<RankCopy> copies;
+    bool host_async = false;   // device ranks copied to host rows, not yet waited for
+    for (int32_t i = 0; i < nc; ++i) {
+        pvs_cursor* c = cursors[i];
+        const int64_t need = std::min<int64_t>(n, c->visible - (c->emitted - c->ahead));
+        n_out[i] = (int32_t)need;
+        take[i] = std::min(need, c->ahead);
+        rest[i] = need - take[i];
+        pulls[i] = rest[i] > 0 ? pull_size(c, rest[i], c->readahead) : 0;
+        if (take[i] > 0) {
+            const int64_t* si = (c->ahead_host ? c->h_ids : c->d_ids) + c->ahead_pos;
+            const float* ss = (c->ahead_host ? c->h_scores : c->d_scores) + c->ahead_pos;
+            if (outputs_on_device) {
+                copies.push_back(RankCopy{si, ss, ids[i], scores[i], (int)take[i]});
+            } else if (c->ahead_host) {
+                std::memcpy(ids[i], si, take[i] * sizeof(int64_t));
+                std::memcpy(scores[i], ss, take[i] * sizeof(float));
+            } else {
+                PVS_CUDA(cudaMemcpyAsync(ids[i], si, take[i] * sizeof(int64_t),
+                                         cudaMemcpyDeviceToHost, st));
+                PVS_CUDA(cudaMemcpyAsync(scores[i], ss, take[i] * sizeof(float),
+                                         cudaMemcpyDeviceToHost, st));
+                host_async = true;
+            }
+            c->ahead_pos += take[i];
+            c->ahead -= take[i];
+        }
+    }
+    // ranks taken from the buffers leave them before a pull refills them
+    if (!copies.empty()) PVS_CUDA(launch_copy_ranks(copies.data(), (int)copies.size(), st));
+    copies.clear();
+    {
+        pvs_status s = build_first_working_sets(cursors, nc, pulls.data());
+        if (s != PVS_OK) return s;
+    }
     DevBuf buf(st, x->scratch_pool);   // released in stream order after the launches that read it
-    int64_t* d_ids = outputs_on_device ? nullptr : buf.get<int64_t>((size_t)nc * n);
-    float* d_scores = outputs_on_device ? nullptr : buf.get<float>((size_t)nc * n);
     PullArgs* d_args = buf.get<PullArgs>((size_t)nc);
-    if ((!outputs_on_device && (!d_ids || !d_scores)) || !d_args) return PVS_ERR_OOM;
+    if (!d_args) return PVS_ERR_OOM;
     std::vector<PullArgs> args;
     std::vector<int32_t> who;
     args.reserve(nc);
     for (int32_t i = 0; i < nc; ++i) {
+        if (pulls[i] <= 0) continue;
         pvs_cursor* c = cursors[i];
-        const int64_t n_eff = std::min<int64_t>(n, c->visible - c->emitted);
-        n_out[i] = (int32_t)n_eff;
-        if (n_eff <= 0) continue;
-        pvs_status s = prepare_pull(c, n_eff);
+        pvs_status s = cursor_out_reserve(c, pulls[i]);   // nothing is ahead now
+        if (s != PVS_OK) return fail(c, s);
+        s = prepare_pull(c, pulls[i]);
         if (s != PVS_OK) return fail(c, s);
         PullArgs a;
         a.w_id = c->w_id;
@@ -1645,11 +1770,13 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
         a.qraw = c->qraw;
         a.raw = x->raw;
         a.m_raw = x->m_raw;
-        a.n = (int)n_eff;
+        a.n = (int)pulls[i];
         a.cand = c->cand;
         a.keys = reinterpret_cast<unsigned long long*>(c->keys);
-        a.out_ids = outputs_on_device ? ids[i] : d_ids + (int64_t)i * n;
-        a.out_scores = outputs_on_device ? scores[i] : d_scores + (int64_t)i * n;
+        // device outputs: the cursor's device buffers; host outputs: its
+        // pinned buffers, which the kernels write directly
+        a.out_ids = outputs_on_device ? c->d_ids : c->h_ids;
+        a.out_scores = outputs_on_device ? c->d_scores : c->h_scores;
         a.status = c->d_status;
         a.ctr = c->ctr;
         a.front = nullptr;   // a few pulls per batch: a frontier would not pay for itself
@@ -1658,54 +1785,58 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
         who.push_back(i);
     }
     if (!args.empty()) {
-        PVS_CUDA(cudaMemcpyAsync(d_args, args.data(), args.size() * sizeof(PullArgs),
-                                 cudaMemcpyHostToDevice, st));
+        PVS_CUDA(launch_stage_pull_args(args.data(), (int)args.size(), d_args, st));
         bool fresh = false;
         for (int32_t i : who) fresh = fresh || cursors[i]->fresh_ws;
-        if (fresh)   // first pull of new working sets: refinement on every SM
-            PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), 4, x->m_raw, st));
-        else
+        if (fresh) {   // first pull of new working sets: refinement on every SM
+            const int per = std::min(64, std::max(4, 2 * x->num_sms / (int)args.size()));
+            PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), per, x->m_raw, st));
+        } else {
             PVS_CUDA(launch_pull_cluster_batch(d_args, (int)args.size(), st));
+        }
     }
     for (int32_t i : who) {
-        cursors[i]->emitted += n_out[i];
-        cursors[i]->pulls++;
-        cursors[i]->fresh_ws = false;
-    }
-    if (!outputs_on_device) {
-        bool contiguous = true;   // rows i at ids[0] + i n: one copy each for ids and scores
-        for (int32_t i = 1; i < nc && contiguous; ++i)
-            contiguous = ids[i] == ids[0] + (int64_t)i * n && scores[i] == scores[0] + (int64_t)i * n;
-        if (contiguous) {
-            PVS_CUDA(cudaMemcpyAsync(ids[0], d_ids, (size_t)nc * n * sizeof(int64_t),
-                                     cudaMemcpyDeviceToHost, st));
-            PVS_CUDA(cudaMemcpyAsync(scores[0], d_scores, (size_t)nc * n * sizeof(float),
-                                     cudaMemcpyDeviceToHost, st));
-        } else {
-            for (int32_t i : who) {
-                PVS_CUDA(cudaMemcpyAsync(ids[i], d_ids + (int64_t)i * n,
-                                         (size_t)n_out[i] * sizeof(int64_t),
-                                         cudaMemcpyDeviceToHost, st));
-                PVS_CUDA(cudaMemcpyAsync(scores[i], d_scores + (int64_t)i * n,
-                                         (size_t)n_out[i] * sizeof(float),
-                                         cudaMemcpyDeviceToHost, st));
-            }
-        }
-        std::vector<pvs_cursor*> pulled;
-        for (int32_t i : who) pulled.push_back(cursors[i]);
-        std::vector<int> dev_status(pulled.size(), 0);
-        pvs_status s = gather_state(pulled.data(), (int)pulled.size(), st, dev_status.data(),
-                                    nullptr);
-        if (s != PVS_OK) return s;
-        pvs_status result = PVS_OK;
-        for (size_t j = 0; j < pulled.size(); ++j)
-            if (dev_status[j] != 0) result = fail(pulled[j], (pvs_status)dev_status[j]);
-        if (result != PVS_OK) return result;
-    }
-    for (int32_t i = 0; i < nc; ++i) {
         pvs_cursor* c = cursors[i];
-        if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
+        c->emitted += pulls[i];
+        c->pulls++;
+        c->fresh_ws = false;
+        c->ahead = pulls[i];
+        c->ahead_pos = 0;
+        c->ahead_host = !outputs_on_device;
     }
+    if (outputs_on_device) {
+        for (int32_t i : who) {
+            pvs_cursor* c = cursors[i];
+            copies.push_back(RankCopy{c->d_ids, c->d_scores, ids[i] + take[i],
+                                      scores[i] + take[i], (int)rest[i]});
+        }
+        if (!copies.empty()) PVS_CUDA(launch_copy_ranks(copies.data(), (int)copies.size(), st));
+    } else {
+        if (!who.empty()) {
+            std::vector<pvs_cursor*> pulled;
+            for (int32_t i : who) pulled.push_back(cursors[i]);
+            std::vector<int> dev_status(pulled.size(), 0);
+            pvs_status s = gather_state(pulled.data(), (int)pulled.size(), st, dev_status.data(),
+                                        nullptr);   // also waits for the pulls' outputs
+            if (s != PVS_OK) return s;
+            pvs_status result = PVS_OK;
+            for (size_t j = 0; j < pulled.size(); ++j)
+                if (dev_status[j] != 0) result = fail(pulled[j], (pvs_status)dev_status[j]);
+            if (result != PVS_OK) return result;
+            for (int32_t i : who) {
+                pvs_cursor* c = cursors[i];
+                std::memcpy(ids[i] + take[i], c->h_ids, rest[i] * sizeof(int64_t));
+                std::memcpy(scores[i] + take[i], c->h_scores, rest[i] * sizeof(float));
+            }
+        } else if (host_async) {
+            PVS_CUDA(cudaStreamSynchronize(st));
+        }
+    }
+    for (int32_t i : who) {
+        cursors[i]->ahead_pos = rest[i];
+        cursors[i]->ahead -= rest[i];
+    }
+    for (int32_t i = 0; i < nc; ++i) delivery_state(cursors[i]);
     return PVS_OK;
 }
 
@@ -1730,23 +1861,28 @@ static pvs_status next_common(pvs_cursor* c, int32_t n, int32_t* n_out, int64_t*
     if (n_out) *n_out = 0;
     if (!c || n < 0 || !n_out) return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
-    const int64_t remaining = c->visible - c->emitted;
+    const int64_t remaining = c->visible - (c->emitted - c->ahead);
     *n_eff = std::min<int64_t>(n, remaining);
     return PVS_OK;
 }
 
-// pvs_next's pull: the next n_eff >= 0 ranks end in the cursor's pinned
-// buffers (c->h_ids, c->h_scores; valid until its next pull).
-static pvs_status pull_to_pinned(pvs_cursor* c, int64_t n_eff) {
+// A pull of r >= 1 ranks into the cursor's pinned buffers at [at, at + r);
+// they become the ranks ahead (ahead_pos = at).  The buffers must already
+// hold at + r entries when at > 0 (they are only reallocated while empty).
+static pvs_status pull_to_pinned(pvs_cursor* c, int64_t r, int64_t at = 0) {
     pvs_status s;
-    if (n_eff > 0 && n_eff <= kPullFusedMax) {
+    if (at == 0) {
+        s = cursor_out_reserve(c, r);
+        if (s != PVS_OK) return fail(c, s);
+    } else if (at + r > c->out_cap) {
+        return fail(c, PVS_ERR_INVALID);   // internal invariant
+    }
+    if (r <= kPullFusedMax) {
         // the kernels write ids, scores and the status word straight into the
         // cursor's pinned host buffers: one launch, one wait
-        s = cursor_out_reserve(c, n_eff);
-        if (s != PVS_OK) return fail(c, s);
         int* mirror = reinterpret_cast<int*>(c->h_small) + 2;
         *reinterpret_cast<volatile int*>(mirror) = kStatusPending;
-        s = pull(c, n_eff, c->h_ids, c->h_scores, mirror);
+        s = pull(c, r, c->h_ids + at, c->h_scores + at, mirror);
         if (s != PVS_OK) return s;
         if (!wait_published(mirror)) {
             // nothing published within the limit: an asynchronous error, or a
@@ -1757,23 +1893,50 @@ static pvs_status pull_to_pinned(pvs_cursor* c, int64_t n_eff) {
         harvest_interval_time(c);
         const int dev_status = *reinterpret_cast<volatile int*>(mirror);
         if (dev_status != 0) return fail(c, (pvs_status)dev_status);
-    } else if (n_eff > 0) {
-        s = cursor_out_reserve(c, n_eff);
-        if (s != PVS_OK) return fail(c, s);
-        s = pull(c, n_eff, c->d_ids, c->d_scores);
+    } else {
+        s = pull(c, r, c->d_ids + at, c->d_scores + at);
         if (s != PVS_OK) return s;
         cudaStream_t st = c->stream;
-        cudaError_t e = cudaMemcpyAsync(c->h_ids, c->d_ids, n_eff * sizeof(int64_t),
+        cudaError_t e = cudaMemcpyAsync(c->h_ids + at, c->d_ids + at, r * sizeof(int64_t),
                                         cudaMemcpyDeviceToHost, st);
         if (e == cudaSuccess)
-            e = cudaMemcpyAsync(c->h_scores, c->d_scores, n_eff * sizeof(float),
+            e = cudaMemcpyAsync(c->h_scores + at, c->d_scores + at, r * sizeof(float),
                                 cudaMemcpyDeviceToHost, st);
         if (e != cudaSuccess) return fail(c, cuda_status(e));
         s = check_device_status(c);
         if (s != PVS_OK) return s;
     }
-    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
-    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+    c->ahead = r;
+    c->ahead_pos = at;
+    c->ahead_host = true;
+    return PVS_OK;
+}
+
+// Ranks ahead in the device buffers moved to the front of the pinned ones.
+static pvs_status ahead_to_host(pvs_cursor* c) {
+    if (c->ahead == 0) {
+        c->ahead_pos = 0;
+        c->ahead_host = true;
+        return PVS_OK;
+    }
+    if (c->ahead_host) {
+        if (c->ahead_pos > 0) {
+            std::memmove(c->h_ids, c->h_ids + c->ahead_pos, c->ahead * sizeof(int64_t));
+            std::memmove(c->h_scores, c->h_scores + c->ahead_pos, c->ahead * sizeof(float));
+        }
+    } else {
+        cudaStream_t st = c->stream;
+        cudaError_t e = cudaMemcpyAsync(c->h_ids, c->d_ids + c->ahead_pos,
+                                        c->ahead * sizeof(int64_t), cudaMemcpyDeviceToHost, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(c->h_scores, c->d_scores + c->ahead_pos, c->ahead * sizeof(float),
+                                cudaMemcpyDeviceToHost, st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+        if (e != cudaSuccess) return fail(c, cuda_status(e));
+    }
+    c->ahead_pos = 0;
+    c->ahead_host = true;
+    return PVS_OK;
 }
 
 pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
@@ -1782,21 +1945,32 @@ pvs_status pvs_next(pvs_cursor* c, int32_t n, int64_t* ids, float* scores, int32
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
     if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
-    s = pull_to_pinned(c, n_eff);
-    if (s < 0) return s;
-    if (n_eff > 0) {
-        std::memcpy(ids, c->h_ids, n_eff * sizeof(int64_t));
-        std::memcpy(scores, c->h_scores, n_eff * sizeof(float));
+    int64_t off = 0;
+    while (off < n_eff) {
+        if (c->ahead == 0) {
+            s = pull_to_pinned(c, pull_size(c, n_eff - off, c->readahead));
+            if (s < 0) return s;
+        } else if (!c->ahead_host) {
+            s = ahead_to_host(c);
+            if (s < 0) return s;
+        }
+        const int64_t take = std::min(n_eff - off, c->ahead);
+        std::memcpy(ids + off, c->h_ids + c->ahead_pos, take * sizeof(int64_t));
+        std::memcpy(scores + off, c->h_scores + c->ahead_pos, take * sizeof(float));
+        c->ahead_pos += take;
+        c->ahead -= take;
+        off += take;
     }
     *n_out = (int32_t)n_eff;
-    return s;
+    return delivery_state(c);
 }
 
 }  // extern "C"
 
-// The next n ranks left in the cursor's pinned buffers, for host code of
-// this library that reads them once (the EAHR driver): *ids and *scores
-// point there and stay valid until the cursor's next pull.  As pvs_next.
+// The next n ranks in the cursor's pinned buffers, for host code of this
+// library that reads them once (the EAHR driver): *ids and *scores point
+// there and stay valid until the cursor's next pull.  As pvs_next, without
+// read-ahead (the driver sizes its pulls itself).
 pvs_status pvs::next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
                             int32_t* n_out) {
     DeviceGuard device_guard(cursor_device(c));
@@ -1804,12 +1978,44 @@ pvs_status pvs::next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
     if (!ids || !scores) return PVS_ERR_INVALID;
-    s = pull_to_pinned(c, n_eff);
-    if (s < 0) return s;
-    *ids = c->h_ids;
-    *scores = c->h_scores;
+    if (n_eff > c->ahead) {
+        if (c->ahead == 0) {
+            s = pull_to_pinned(c, n_eff);
+        } else {
+            // ranks a pvs_next left ahead come first, the rest right after them
+            s = ahead_to_host(c);
+            if (s == PVS_OK && c->ahead + (n_eff - c->ahead) > c->out_cap) {
+                std::vector<int64_t> keep_ids(c->h_ids, c->h_ids + c->ahead);
+                std::vector<float> keep_sc(c->h_scores, c->h_scores + c->ahead);
+                const int64_t k = c->ahead;
+                c->ahead = 0;
+                s = cursor_out_reserve(c, n_eff);
+                if (s == PVS_OK) {
+                    std::memcpy(c->h_ids, keep_ids.data(), k * sizeof(int64_t));
+                    std::memcpy(c->h_scores, keep_sc.data(), k * sizeof(float));
+                    c->ahead = k;
+                } else {
+                    fail(c, s);
+                }
+            }
+            if (s == PVS_OK) {
+                const int64_t k = c->ahead;
+                s = pull_to_pinned(c, n_eff - k, k);
+                c->ahead += k;
+                c->ahead_pos = 0;
+            }
+        }
+        if (s < 0) return s;
+    } else if (!c->ahead_host) {
+        s = ahead_to_host(c);
+        if (s < 0) return s;
+    }
+    *ids = c->h_ids + c->ahead_pos;
+    *scores = c->h_scores + c->ahead_pos;
+    c->ahead_pos += n_eff;
+    c->ahead -= n_eff;
     *n_out = (int32_t)n_eff;
-    return s;
+    return delivery_state(c);
 }
 
 extern "C" {
@@ -1821,13 +2027,51 @@ pvs_status pvs_next_device(pvs_cursor* c, int32_t n, int64_t* ids, float* scores
     pvs_status s = next_common(c, n, n_out, &n_eff);
     if (s != PVS_OK) return s;
     if (n_eff > 0 && (!ids || !scores)) return PVS_ERR_INVALID;
-    if (n_eff > 0) {
-        s = pull(c, n_eff, ids, scores);
-        if (s != PVS_OK) return s;
+    int64_t off = 0;
+    RankCopy copies[2];
+    int ncopy = 0;
+    while (off < n_eff) {
+        if (c->ahead == 0) {
+            const int64_t r = pull_size(c, n_eff - off, c->readahead);
+            if (r > kPullFusedMax) {   // a large pull goes straight to the caller
+                if (ncopy) {
+                    PVS_CUDA(launch_copy_ranks(copies, ncopy, c->stream));
+                    ncopy = 0;
+                }
+                s = pull(c, r, ids + off, scores + off);
+                if (s != PVS_OK) return s;
+                off += r;
+                break;
+            }
+            if (ncopy) {   // the buffer is reused: earlier copies first
+                PVS_CUDA(launch_copy_ranks(copies, ncopy, c->stream));
+                ncopy = 0;
+            }
+            s = cursor_out_reserve(c, r);
+            if (s != PVS_OK) return fail(c, s);
+            s = pull(c, r, c->d_ids, c->d_scores);
+            if (s != PVS_OK) return s;
+            c->ahead = r;
+            c->ahead_pos = 0;
+            c->ahead_host = false;
+        }
+        const int64_t take = std::min(n_eff - off, c->ahead);
+        const int64_t* src_i = (c->ahead_host ? c->h_ids : c->d_ids) + c->ahead_pos;
+        const float* src_s = (c->ahead_host ? c->h_scores : c->d_scores) + c->ahead_pos;
+        copies[ncopy++] = RankCopy{src_i, src_s, ids + off, scores + off, (int)take};
+        c->ahead_pos += take;
+        c->ahead -= take;
+        off += take;
     }
+    if (ncopy) PVS_CUDA(launch_copy_ranks(copies, ncopy, c->stream));
     *n_out = (int32_t)n_eff;
-    if (c->emitted == c->visible) c->state = PVS_EXHAUSTED;
-    return c->state == PVS_EXHAUSTED ? PVS_EXHAUSTED : PVS_OK;
+    return delivery_state(c);
+}
+
+pvs_status pvs_cursor_set_readahead(pvs_cursor* c, int32_t pages) {
+    if (!c || pages < 1) return PVS_ERR_INVALID;
+    c->readahead = pages;
+    return PVS_OK;
 }
 
 pvs_status pvs_cursor_sync(pvs_cursor* c) {
@@ -1842,7 +2086,7 @@ pvs_status pvs_cursor_sync(pvs_cursor* c) {
 static void fill_stats(pvs_cursor* c, const DevCounters& d, pvs_stats* out) {
     std::memset(out, 0, sizeof(*out));
     out->visible = c->visible;
-    out->emitted = c->emitted;
+    out->emitted = c->emitted - c->ahead;   // delivered to the caller
     out->refined = (int64_t)d.refined;
     out->exact_fallbacks = (int64_t)d.exact_fallbacks;
     out->interval_passes = c->interval_passes;
@@ -1965,7 +2209,7 @@ static void release_cursor(pvs_cursor* c) {
         std::lock_guard<std::mutex> lock(x->pool_mutex);
         const size_t bytes = cursor_device_bytes(c);
         if (x->cursor_pool.size() < kCursorPool &&
-            x->pool_bytes + bytes <= kCursorPoolBytes) {   // keep the buffers for the next cursor
+            x->pool_bytes + bytes <= x->pool_limit) {   // keep the buffers for the next cursor
             x->pool_bytes += bytes;
             cursor_reset(c);
             x->cursor_pool.push_back(c);

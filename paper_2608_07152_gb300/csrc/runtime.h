@@ -47,6 +47,7 @@ struct pvs_index {
     size_t stage_floats = 0;
     std::vector<pvs_cursor*> cursor_pool;   // closed cursors whose buffers are reused
     size_t pool_bytes = 0;                  // device bytes held by pooled cursors
+    size_t pool_limit = 0;                  // at most this many (a quarter of the device)
     std::mutex pool_mutex;                  // cursors may open / close on several threads
     std::mutex pass_mutex;                  // orders interval passes of this index
     cudaEvent_t pass_done = nullptr;        // end of the last interval pass queued
@@ -118,6 +119,14 @@ struct pvs_cursor {
     int64_t out_cap = 0;
     int64_t* h_ids = nullptr;         // pinned
     float* h_scores = nullptr;        // pinned
+    // ranks computed ahead of the caller (Sec. 2.1: the list is a stable
+    // prefix, so a rank computed early is the rank delivered later): they sit
+    // at [ahead_pos, ahead_pos + ahead) of h_ids / h_scores when ahead_host,
+    // else of d_ids / d_scores.  `emitted` counts them; the caller has
+    // received emitted - ahead ranks.
+    int64_t ahead = 0, ahead_pos = 0;
+    bool ahead_host = false;
+    int32_t readahead = 4;            // a pull computes up to this many pages
     unsigned int* h_small = nullptr;  // pinned scratch (counts, status)
     // stats
     int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;

@@ -100,9 +100,8 @@ cudaError_t launch_select_f32_n(const float* vals, int64_t rows, uint64_t k, Sel
 // The same selection for a short array in one launch: one CTA copies the
 // values into shared memory once (16-byte loads; when they fit) and runs the
 // four digit rounds there, its histogram in shared memory too.
-__global__ void __launch_bounds__(1024) select_small_kernel(const float* __restrict__ vals,
-                                                            int64_t len, uint64_t k0,
-                                                            SelectState* sel, int staged) {
+__device__ __forceinline__ void select_small_body(const float* __restrict__ vals, int64_t len,
+                                                  uint64_t k0, SelectState* sel, int staged) {
     extern __shared__ float4 staged_vals[];
     __shared__ unsigned int h[256];
     __shared__ unsigned int suffix[256];
@@ -174,6 +173,12 @@ __global__ void __launch_bounds__(1024) select_small_kernel(const float* __restr
     if (t < 256) sel->hist[t] = 0;
 }
 
+__global__ void __launch_bounds__(1024) select_small_kernel(const float* __restrict__ vals,
+                                                            int64_t len, uint64_t k0,
+                                                            SelectState* sel, int staged) {
+    select_small_body(vals, len, k0, sel, staged);
+}
+
 cudaError_t launch_select_small(const float* vals, int64_t len, uint64_t k, SelectState* sel,
                                 cudaStream_t st) {
     // staged in shared memory when the values fit in 200 KB and start on a
@@ -211,9 +216,10 @@ __device__ __forceinline__ bool ws_member(const float* lo, const float* hi, int6
     return lo[i] != -INFINITY;
 }
 
-__global__ void compact_count_kernel(const float* __restrict__ lo, const float* __restrict__ hi,
-                                     int64_t rows, const SelectState* sel,
-                                     unsigned int* block_counts) {
+__device__ __forceinline__ void compact_count_body(const float* __restrict__ lo,
+                                                   const float* __restrict__ hi, int64_t rows,
+                                                   const SelectState* sel,
+                                                   unsigned int* block_counts) {
     __shared__ unsigned int wsum[kCompactBlock / 32];
     const uint32_t tau = (uint32_t)sel->prefix;
     const int64_t base = (int64_t)blockIdx.x * kCompactTile;
@@ -232,8 +238,15 @@ __global__ void compact_count_kernel(const float* __restrict__ lo, const float* 
     }
 }
 
+__global__ void compact_count_kernel(const float* __restrict__ lo, const float* __restrict__ hi,
+                                     int64_t rows, const SelectState* sel,
+                                     unsigned int* block_counts) {
+    compact_count_body(lo, hi, rows, sel, block_counts);
+}
+
 // Exclusive scan of n block counts by one block; total to *total.
-__global__ void scan_counts_kernel(unsigned int* counts, int64_t n, unsigned int* total) {
+__device__ __forceinline__ void scan_counts_body(unsigned int* counts, int64_t n,
+                                                 unsigned int* total) {
     __shared__ unsigned int part[1024];
     const int t = threadIdx.x;
     const int64_t per = (n + blockDim.x - 1) / blockDim.x;
@@ -257,10 +270,15 @@ __global__ void scan_counts_kernel(unsigned int* counts, int64_t n, unsigned int
     if (t == (int)blockDim.x - 1) *total = part[t];
 }
 
-__global__ void compact_scatter_kernel(const float* __restrict__ lo, const float* __restrict__ hi,
-                                       int64_t rows, const SelectState* sel,
-                                       const unsigned int* block_offsets, int32_t* w_id,
-                                       float* w_lo, float* w_hi) {
+__global__ void scan_counts_kernel(unsigned int* counts, int64_t n, unsigned int* total) {
+    scan_counts_body(counts, n, total);
+}
+
+__device__ __forceinline__ void compact_scatter_body(const float* __restrict__ lo,
+                                                     const float* __restrict__ hi, int64_t rows,
+                                                     const SelectState* sel,
+                                                     const unsigned int* block_offsets,
+                                                     int32_t* w_id, float* w_lo, float* w_hi) {
     __shared__ unsigned int wbase[kCompactBlock / 32];
     __shared__ unsigned int run;
     const uint32_t tau = (uint32_t)sel->prefix;
@@ -292,6 +310,13 @@ __global__ void compact_scatter_kernel(const float* __restrict__ lo, const float
     }
 }
 
+__global__ void compact_scatter_kernel(const float* __restrict__ lo, const float* __restrict__ hi,
+                                       int64_t rows, const SelectState* sel,
+                                       const unsigned int* block_offsets, int32_t* w_id,
+                                       float* w_lo, float* w_hi) {
+    compact_scatter_body(lo, hi, rows, sel, block_offsets, w_id, w_lo, w_hi);
+}
+
 cudaError_t launch_compact_ordered(const float* lo, const float* hi, int64_t rows,
                                    const SelectState* sel, int32_t* w_id, float* w_lo,
                                    float* w_hi, unsigned int* w_len, unsigned int* scratch,
@@ -305,6 +330,59 @@ cudaError_t launch_compact_ordered(const float* lo, const float* hi, int64_t row
     count_launches(1);
     compact_scatter_kernel<<<(unsigned)nb, kCompactBlock, 0, st>>>(lo, hi, rows, sel, scratch,
                                                                    w_id, w_lo, w_hi);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// the same steps for the cursors of a grouped pass, one launch per step
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(1024) select_small_group_kernel(const __grid_constant__ WsGroupArgs a,
+                                                                  int staged) {
+    const int g = blockIdx.y;
+    select_small_body(a.slot[g], a.slot_n, a.k[g], a.sel[g], staged);
+}
+
+__global__ void compact_count_group_kernel(const __grid_constant__ WsGroupArgs a) {
+    const int g = blockIdx.y;
+    compact_count_body(a.lo[g], a.hi[g], a.rows, a.sel[g], a.scratch[g]);
+}
+
+__global__ void scan_counts_group_kernel(const __grid_constant__ WsGroupArgs a, int64_t nb) {
+    const int g = blockIdx.x;
+    scan_counts_body(a.scratch[g], nb, a.w_len[g]);
+}
+
+__global__ void compact_scatter_group_kernel(const __grid_constant__ WsGroupArgs a) {
+    const int g = blockIdx.y;
+    compact_scatter_body(a.lo[g], a.hi[g], a.rows, a.sel[g], a.scratch[g], a.w_id[g], a.w_lo[g],
+                         a.w_hi[g]);
+}
+
+cudaError_t launch_ws_group(const WsGroupArgs& a, cudaStream_t st) {
+    if (a.n <= 0) return cudaSuccess;
+    if (a.n > kGroupMax || a.slot_n <= 0) return cudaErrorInvalidValue;
+    bool staged = a.slot_n * (int64_t)sizeof(float) <= 200 * 1024;
+    for (int g = 0; g < a.n; ++g)
+        staged = staged && (reinterpret_cast<uintptr_t>(a.slot[g]) & 15u) == 0;
+    const size_t smem = staged ? (size_t)((a.slot_n + 3) / 4) * sizeof(float4) : 0;
+    if (smem > 0) {
+        cudaError_t e = raise_smem_limit((const void*)select_small_group_kernel, smem);
+        if (e != cudaSuccess) return e;
+    }
+    count_launches(1);
+    select_small_group_kernel<<<dim3(1, a.n), 1024, smem, st>>>(a, staged ? 1 : 0);
+    const int64_t nb = (a.rows + kCompactTile - 1) / kCompactTile;
+    if (nb == 0) {
+        for (int g = 0; g < a.n; ++g) {
+            cudaError_t e = cudaMemsetAsync(a.w_len[g], 0, sizeof(unsigned int), st);
+            if (e != cudaSuccess) return e;
+        }
+        return cudaGetLastError();
+    }
+    count_launches(3);
+    compact_count_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+    scan_counts_group_kernel<<<a.n, 1024, 0, st>>>(a, nb);
+    compact_scatter_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -145,9 +145,14 @@ def test_passage_scale_lone_cursor(passage):
     lo = np.array(lo, np.float32)
     hi = np.array(hi, np.float32)
     s_first = s_sample[np.searchsorted(sample, first)]
+    last_s, last_id = float(sc[-1]), int(ids[-1])
     for k, i in enumerate(first.tolist()):
         if i in emitted:
             assert lo[k] == -np.inf and hi[k] == -np.inf
+        elif lo[k] == -np.inf:
+            # computed ahead of the caller: it ranks right after the prefix
+            s = float(s_first[k])
+            assert hi[k] == -np.inf and (s < last_s or (s == last_s and i > last_id))
         elif lo[k] == hi[k]:
             assert lo[k].view(np.uint32) == s_first[k].view(np.uint32)
         else:

@@ -567,3 +567,53 @@ def test_frozen_scheduler_over_a_pvs_cursor(tau):
         assert p >= 1 and 16 * (p - 1) < d <= 16 * p
         if not st["exhausted"][i]:
             assert d == 16 * p
+
+
+@pytest.mark.parametrize("pages", [1, 4, 13])
+def test_readahead_with_mixed_calls_matches_the_oracle(pages):
+    """A pull may compute ranks ahead of the caller (pvs_cursor_set_readahead);
+    Sec. 2.1's stable prefix makes any mix of host, device and batched calls
+    of any sizes deliver the complete ranking in order."""
+    n, m = 20_011, 128
+    V = synth.unit_normal(n, m, seed=90).numpy()
+    q = synth.unit_normal(1, m, seed=91).numpy()[0]
+    ref_ids, ref_sc = po.dense_ranking(q, V)
+    index = pvs.pvs_build(V)
+    got_i, got_s = [], []
+    try:
+        cur = pvs.pvs_cursor_open(index, q)
+        try:
+            pvs.pvs_cursor_set_readahead(cur, pages)
+            for k, kind in ((7, "host"), (20, "dev"), (3, "host"), (20, "batch_host"),
+                            (11, "batch_dev"), (300, "host"), (257, "dev"), (64, "batch_dev"),
+                            (1, "dev"), (999, "batch_host"), (5, "host")):
+                if kind == "host":
+                    i, s, _ = pvs.pvs_next(cur, k)
+                elif kind == "dev":
+                    ti = torch.empty(k, dtype=torch.int64, device="cuda")
+                    ts = torch.empty(k, dtype=torch.float32, device="cuda")
+                    got, _ = pvs.pvs_next_device(cur, k, ti, ts)
+                    assert pvs.pvs_cursor_sync(cur) >= 0
+                    i, s = ti[:got].cpu().numpy(), ts[:got].cpu().numpy()
+                elif kind == "batch_host":
+                    ib, sb, nb = pvs.pvs_next_batch([cur], k)
+                    i, s = ib[0, :nb[0]], sb[0, :nb[0]]
+                else:
+                    ti = torch.empty((1, k), dtype=torch.int64, device="cuda")
+                    ts = torch.empty((1, k), dtype=torch.float32, device="cuda")
+                    nb = pvs.pvs_next_batch([cur], k, ti, ts)
+                    assert pvs.pvs_cursor_sync(cur) >= 0
+                    i, s = ti[0, :nb[0]].cpu().numpy(), ts[0, :nb[0]].cpu().numpy()
+                assert len(i) == k
+                got_i.append(np.asarray(i))
+                got_s.append(np.asarray(s))
+            st = pvs.pvs_cursor_stats(cur)
+        finally:
+            pvs.pvs_cursor_close(cur)
+    finally:
+        pvs.pvs_index_free(index)
+    ids = np.concatenate(got_i)
+    sc = np.concatenate(got_s).astype(np.float32)
+    assert st["emitted"] == ids.size
+    assert np.array_equal(ids, ref_ids[:ids.size])
+    assert np.array_equal(sc.view(np.uint32), ref_sc[:ids.size].view(np.uint32))
