@@ -76,13 +76,17 @@ def parse():
                         "vs full scan; segments: EAHR over 8 merged Segments")
     p.add_argument("--eahr-queries", type=int, default=200,
                    help="queries per correlation level (tau = +0.5, 0)")
-    p.add_argument("--eahr-exhaust-queries", type=int, default=10,
+    p.add_argument("--eahr-exhaust-queries", type=int, default=200,
                    help="queries at tau = -0.5 (both lists are read to the end)")
     p.add_argument("--snap-queries", type=int, default=100, help="queries per snapshot")
     p.add_argument("--eahr-levels", default="0.5,0,-0.5",
                    help="Kendall tau levels of --workload eahr (comma-separated)")
-    p.add_argument("--eahr-policy", default="geometric", choices=["geometric", "frozen", "equal"],
-                   help="EAHR scheduling policy of --workload eahr")
+    p.add_argument("--eahr-policy", default="adaptive",
+                   choices=["adaptive", "geometric", "frozen", "equal"],
+                   help="EAHR scheduling policy (adaptive: geometric reading, then complete-list "
+                        "fusion on the device once the lists are read deep)")
+    p.add_argument("--no-eahr", action="store_true",
+                   help="passage: leave out the EAHR Top-20 record of the default line")
     p.add_argument("--ablation-queries", type=int, default=30,
                    help="queries per generator in --workload ablation")
     p.add_argument("--pipeline", type=int, default=0,
@@ -504,6 +508,84 @@ EAHR_RRF_K = 60   # the build target's w / (60 + rank), w_d = w_s = 1
 EAHR_LEVELS = (0.5, 0.0, -0.5)
 
 
+def eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts, rank, dev,
+                warmup=2, comparator_queries=None):
+    """EAHR Top-20 per Kendall-tau level: per query a Gaussian-copula sparse
+    ranking of every id (an fp32 torch product of the corpus with the query is
+    the copula's proxy: input generation only), then, timed on the host,
+    cursor open + eahr_topk (dense pulls through the library, sparse ids from
+    host memory) + close.  Beside it, the exhaustive comparator: fp32 scores
+    of every row, a full sort and complete-list fusion in plain torch (for the
+    first `comparator_queries` queries of a level; all when None).
+    counts: {tau: queries}.  Returns (levels, latencies)."""
+    n = rows.shape[0]
+
+    def sparse_for(q, tau, seed):
+        proxy = rows @ q
+        return synth.copula_ranking(proxy, tau, seed).cpu().numpy(), proxy
+
+    def comparator(q, sparse_dev):
+        """Exhaustive fp32 scoring + full sort + complete-list fusion, ms."""
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        sc = rows @ q
+        order = torch.argsort(sc, descending=True, stable=True)
+        rd = torch.empty(n, dtype=torch.float64, device=dev)
+        rd[order] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
+        rs = torch.empty(n, dtype=torch.float64, device=dev)
+        rs[sparse_dev] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
+        fused = 1.0 / (EAHR_RRF_K + rd) + 1.0 / (EAHR_RRF_K + rs)
+        top = torch.topk(fused, EAHR_K).indices
+        top.cpu()
+        return (time.perf_counter() - t) * 1e3
+
+    qi = 0
+    for w in range(warmup):   # library paths, torch kernels
+        sp, _ = sparse_for(queries[qi], 0.5, 7 + w)
+        cur = pvs.pvs_cursor_open(index, queries[qi])
+        pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR, policy=policy)
+        pvs.pvs_cursor_close(cur)
+        comparator(queries[qi], torch.from_numpy(sp).to(dev))
+        qi += 1
+    levels, lat_all = {}, []
+    for tau, count in counts.items():
+        lat, cmp_ms, dd, ds, ex, pulls, complete = [], [], [], [], 0, [], 0
+        ktau = None
+        for j in range(count):
+            q = queries[qi]
+            qi += 1
+            sp, proxy = sparse_for(q, tau, query_seed(1000, rank) + qi)
+            if j == 0:   # realised Kendall tau of the generated channel
+                dense_order = torch.argsort(proxy, descending=True, stable=True).cpu().numpy()
+                ktau = synth.kendall_tau_sample(dense_order, sp, 200_000, seed=qi)
+            torch.cuda.synchronize()
+            t = time.perf_counter()
+            cur = pvs.pvs_cursor_open(index, q)
+            ids, F, st = pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K,
+                                       form=pvs.EAHR_NUMERATOR, policy=policy)
+            pvs.pvs_cursor_close(cur)
+            lat.append((time.perf_counter() - t) * 1e3)
+            if len(ids) != EAHR_K:
+                raise RuntimeError("EAHR returned a short list")
+            dd.append(st["depth"][0])
+            ds.append(st["depth"][1])
+            ex += int(st["exhausted"][0] and st["exhausted"][1])
+            complete += int(st.get("complete", 0))
+            pulls.append(st["pulls"][0])
+            if comparator_queries is None or j < comparator_queries:
+                cmp_ms.append(comparator(q, torch.from_numpy(sp).to(dev)))
+        lat_all.extend(lat)
+        levels[f"{tau:+.1f}"] = {
+            "queries": count, "kendall_tau_realised": ktau,
+            "latency_ms_p50": float(np.median(lat)), "latency_ms_p95": float(np.percentile(lat, 95)),
+            "exhaustive_fp32_ms_p50": float(np.median(cmp_ms)) if cmp_ms else None,
+            "dense_depth_p50": float(np.median(dd)), "dense_depth_mean": float(np.mean(dd)),
+            "sparse_depth_p50": float(np.median(ds)), "both_exhausted": ex,
+            "finished_by_complete_fusion": complete,
+            "dense_pulls_p50": float(np.median(pulls))}
+    return levels, lat_all
+
+
 def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     """EAHR end to end over the passage corpus: per query a sparse channel that
     is a complete ranking of all N ids, a Gaussian-copula permutation of the
@@ -525,78 +607,20 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     index = pvs.pvs_build(rows, stream=stream.cuda_stream)
     torch.cuda.synchronize()
     build_s = time.perf_counter() - t0
-    total_q = 2 * args.eahr_queries + args.eahr_exhaust_queries + 2
+    counts = {t: (args.eahr_exhaust_queries if t < 0 else args.eahr_queries)
+              for t in [float(x) for x in args.eahr_levels.split(",")]}
+    total_q = sum(counts.values()) + 2
     queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
     policy = {"geometric": pvs.EAHR_POLICY_GEOMETRIC, "frozen": pvs.EAHR_POLICY_FROZEN,
-              "equal": pvs.EAHR_POLICY_EQUAL_DEPTH}[args.eahr_policy]
+              "equal": pvs.EAHR_POLICY_EQUAL_DEPTH,
+              "adaptive": pvs.EAHR_POLICY_ADAPTIVE}[args.eahr_policy]
 
-    def sparse_for(q, tau, seed):
-        proxy = rows @ q
-        return synth.copula_ranking(proxy, tau, seed).cpu().numpy(), proxy
-
-    def comparator(q, sparse_dev):
-        """Exhaustive fp32 scoring + full sort + complete-list fusion, ms."""
-        torch.cuda.synchronize()
-        t = time.perf_counter()
-        sc = rows @ q
-        order = torch.argsort(sc, descending=True, stable=True)
-        rd = torch.empty(n, dtype=torch.float64, device=dev)
-        rd[order] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
-        rs = torch.empty(n, dtype=torch.float64, device=dev)
-        rs[sparse_dev] = torch.arange(1, n + 1, dtype=torch.float64, device=dev)
-        # the sparse list is the positive-score support (Sec. 2.1)
-        fused = 1.0 / (EAHR_RRF_K + rd) + torch.where(ss > 0, 1.0 / (EAHR_RRF_K + rs), 0.0)
-        top = torch.topk(fused, EAHR_K).indices
-        top.cpu()
-        return (time.perf_counter() - t) * 1e3
-
-    # warm-up (library paths, torch kernels)
-    for w in range(2):
-        sp, _ = sparse_for(queries[w], 0.5, 7 + w)
-        cur = pvs.pvs_cursor_open(index, queries[w])
-        pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K, form=pvs.EAHR_NUMERATOR, policy=policy)
-        pvs.pvs_cursor_close(cur)
-        comparator(queries[w], torch.from_numpy(sp).to(dev))
     if pg:
         pg.barrier()
     launches0 = pvs.pvs_launch_count()
-    levels = {}
-    qi = 2
-    lat_all = []
     with ClockSampler(local) as clk:
-        for tau in [float(x) for x in args.eahr_levels.split(",")]:
-            count = args.eahr_exhaust_queries if tau < 0 else args.eahr_queries
-            lat, cmp_ms, dd, ds, ex, pulls = [], [], [], [], 0, []
-            ktau = None
-            for j in range(count):
-                q = queries[qi]
-                qi += 1
-                sp, proxy = sparse_for(q, tau, query_seed(1000, rank) + qi)
-                if j == 0:   # realised Kendall tau of the generated channel
-                    dense_order = torch.argsort(proxy, descending=True, stable=True).cpu().numpy()
-                    ktau = synth.kendall_tau_sample(dense_order, sp, 200_000, seed=qi)
-                torch.cuda.synchronize()
-                t = time.perf_counter()
-                cur = pvs.pvs_cursor_open(index, q)
-                ids, F, st = pvs.eahr_topk(cur, sp, K=EAHR_K, k=EAHR_RRF_K,
-                                           form=pvs.EAHR_NUMERATOR, policy=policy)
-                pvs.pvs_cursor_close(cur)
-                lat.append((time.perf_counter() - t) * 1e3)
-                if len(ids) != EAHR_K:
-                    raise RuntimeError("EAHR returned a short list")
-                dd.append(st["depth"][0])
-                ds.append(st["depth"][1])
-                ex += int(st["exhausted"][0] and st["exhausted"][1])
-                pulls.append(st["pulls"][0])
-                cmp_ms.append(comparator(q, torch.from_numpy(sp).to(dev)))
-            lat_all.extend(lat)
-            levels[f"{tau:+.1f}"] = {
-                "queries": count, "kendall_tau_realised": ktau,
-                "latency_ms_p50": float(np.median(lat)), "latency_ms_p95": float(np.percentile(lat, 95)),
-                "exhaustive_fp32_ms_p50": float(np.median(cmp_ms)),
-                "dense_depth_p50": float(np.median(dd)), "dense_depth_mean": float(np.mean(dd)),
-                "sparse_depth_p50": float(np.median(ds)), "both_exhausted": ex,
-                "dense_pulls_p50": float(np.median(pulls))}
+        levels, lat_all = eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts,
+                                      rank, dev, warmup=2)
     launches = pvs.pvs_launch_count() - launches0
     head = levels.get("+0.5", next(iter(levels.values())))
     line = {
@@ -1300,6 +1324,32 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.destroy_process_group()
 
 
+def eahr_record(args, pvs, synth, torch, np, index, centres, n, rank, dev):
+    """The EAHR Top-20 configuration on the passage index (K = 20, weighted
+    RRF 1 / (60 + rank), a Gaussian-copula sparse ranking of every id per
+    query at Kendall tau +0.5 / 0 / -0.5, the adaptive policy): per-level
+    latency, depth and the exhaustive comparator, for the default line."""
+    rows = torch.empty((n, DIM), dtype=torch.float32, device=dev)   # the copula's proxy
+    for r in range(0, n, 1 << 20):
+        c = min(1 << 20, n - r)
+        rows[r:r + c] = synth.mixture_rows(c, centres, WITHIN_STD, seed=2, first=r)
+    counts = {0.5: args.eahr_queries, 0.0: args.eahr_queries, -0.5: args.eahr_exhaust_queries}
+    queries = synth.mixture_queries(sum(counts.values()) + 2, centres, QUERY_NOISE,
+                                    seed=query_seed(5003, rank))
+    levels, _ = eahr_levels(pvs, synth, torch, np, index, rows, queries,
+                            pvs.EAHR_POLICY_ADAPTIVE, counts, rank, dev, warmup=2,
+                            comparator_queries=20)
+    del rows
+    torch.cuda.empty_cache()
+    return {"metric": "EAHR Top-20 latency", "unit": "ms", "higher_is_better": False,
+            "K": EAHR_K, "rrf": "1/(60+rank), w_d = w_s = 1", "policy": "adaptive",
+            "timed": "cursor open + eahr_topk + close per query, host clock, sparse ids in "
+                     "host memory",
+            "comparator": "exhaustive fp32 scoring + full sort + complete-list fusion in plain "
+                          "torch, first 20 queries of each level",
+            "levels": levels}
+
+
 def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     """The passage workload (the default): the queries of a step served by
     the native executor, GROUP at a time from one grouped pass over the
@@ -1422,6 +1472,8 @@ def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         "build_s": build_s,
         "clocks": clk.summary(),
     }
+    if rank == 0 and not args.no_eahr:
+        line["eahr"] = eahr_record(args, pvs, synth, torch, np, index, centres, n, rank, dev)
     if rank == 0 and not args.no_cpu_baseline:
         qb = timed_q[:64].cpu().numpy()
         line["cpu_baseline"] = cpu_baseline(synth, torch, centres, qb, n)

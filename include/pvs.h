@@ -393,7 +393,7 @@ enum {
     EAHR_POLICY_EQUAL_DEPTH = 1, /* both lists advance by `step` ranks, and
                                     certification runs after every step
                                     (the controlled-stream protocol, Sec. 3.4) */
-    EAHR_POLICY_FROZEN = 2       /* the paper's frozen scheduler (Sec. 3.5):
+    EAHR_POLICY_FROZEN = 2,      /* the paper's frozen scheduler (Sec. 3.5):
                                     each step reads `step` ranks from the list
                                     whose next unread rank contributes more; a
                                     list skipped 16 steps in a row is advanced;
@@ -402,6 +402,17 @@ enum {
                                     has grown by clamp(access / 8, 64, 1024)
                                     since the last check, and at once when a
                                     list is exhausted                          */
+    EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk only: GEOMETRIC until the ranks
+                                    read reach max(2^18, (n_dense + n_sparse)
+                                    / 16), then complete-list fusion on the
+                                    device (Sec. 2.2: when early determination
+                                    is impossible, fusing the complete lists
+                                    gives the same result): every visible
+                                    row's authoritative score, both lists'
+                                    ranks, the fused order, exact rational
+                                    comparison of the items near the K-th.
+                                    The whole sparse list is then checked.
+                                    Other entry points treat it as GEOMETRIC  */
 };
 
 typedef struct eahr_params {
@@ -422,7 +433,8 @@ typedef struct eahr_stats {
     int32_t exhausted[2];   /* list i reached Exhausted                        */
     int32_t pulls[2];       /* producer calls per list                         */
     int32_t checks;         /* certification rounds                            */
-    int32_t reserved;
+    int32_t complete;       /* 1: finished by complete-list fusion on the
+                               device (EAHR_POLICY_ADAPTIVE)                   */
 } eahr_stats;
 
 /* EAHR over a freshly opened dense cursor (no ranks delivered yet) and a

@@ -44,6 +44,7 @@ EAHR_NUMERATOR = 1
 EAHR_POLICY_GEOMETRIC = 0
 EAHR_POLICY_EQUAL_DEPTH = 1
 EAHR_POLICY_FROZEN = 2
+EAHR_POLICY_ADAPTIVE = 3
 
 
 class PvsError(RuntimeError):
@@ -70,7 +71,7 @@ class eahr_params(ctypes.Structure):
 class eahr_stats(ctypes.Structure):
     _fields_ = [("depth", ctypes.c_int64 * 2), ("length", ctypes.c_int64 * 2),
                 ("exhausted", ctypes.c_int32 * 2), ("pulls", ctypes.c_int32 * 2),
-                ("checks", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("checks", ctypes.c_int32), ("complete", ctypes.c_int32)]
 
 
 class pbm_stats(ctypes.Structure):
@@ -566,7 +567,7 @@ def _params(K, k, form, policy, step, weights):
 def _eahr_result(st, ids, F, got, stats):
     s = {"depth": list(stats.depth), "length": list(stats.length),
          "exhausted": list(stats.exhausted), "pulls": list(stats.pulls),
-         "checks": stats.checks}
+         "checks": stats.checks, "complete": stats.complete}
     return ids[:got.value], F[:got.value], s
 
 

@@ -725,9 +725,59 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
     }
 }
 
+// EAHR_POLICY_ADAPTIVE's finish (Sec. 2.2, last paragraph): complete-list
+// fusion of the dense cursor's query and the host sparse list on the device,
+// then T*_K from the candidates it returns, ordered by exact rational F
+// (ties: smaller id first), zero-score items never appended (Sec. 2.1).
+constexpr int64_t kCompleteMin = (int64_t)1 << 18;
+
+pvs_status finish_complete(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
+                           int32_t* n_out, eahr_stats* st) {
+    d.join_ahead();
+    pvs::FuseWeights w;
+    for (int i = 0; i < 2; ++i) {
+        w.a[i] = d.active[i] ? (double)d.g[i].a : 0.0;
+        w.b[i] = (double)d.g[i].b;
+        w.c[i] = (double)d.g[i].c;
+    }
+    std::vector<pvs::FusedCand> cand;
+    pvs_status s = pvs::fuse_complete(d.src[0].cursor, d.src[1].list, d.src[1].length, w, p->K,
+                                      &cand);
+    if (s != PVS_OK) return s;
+    std::vector<Node> nodes;
+    nodes.reserve(cand.size());
+    for (const pvs::FusedCand& c : cand) {
+        Frac F;
+        if (d.active[0] && c.rd > 0) F = add(F, d.g[0].at(c.rd));
+        if (d.active[1] && c.rs > 0) F = add(F, d.g[1].at(c.rs));
+        if (F.num != 0) nodes.push_back(Node{F, c.id});
+    }
+    std::sort(nodes.begin(), nodes.end(), NodeCmp());
+    const int32_t q = (int32_t)std::min<size_t>((size_t)p->K, nodes.size());
+    for (int32_t t = 0; t < q; ++t) {
+        out_ids[t] = nodes[(size_t)t].id;
+        if (out_F) out_F[t] = frac_to_double(nodes[(size_t)t].F);
+    }
+    *n_out = q;
+    if (st) {
+        for (int i = 0; i < 2; ++i) {
+            st->depth[i] = d.src[i].length;   // both lists used to the end
+            st->length[i] = d.src[i].length;
+            st->exhausted[i] = d.active[i] ? 1 : 0;
+            st->pulls[i] = d.pulls[i];
+        }
+        st->checks = d.checks;
+        st->complete = 1;
+    }
+    return PVS_OK;
+}
+
 pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
                       int32_t* n_out, eahr_stats* st) {
     const int step0 = p->step > 0 ? p->step : 16;
+    const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor && d.src[1].list;
+    const int64_t complete_at =
+        std::max<int64_t>(kCompleteMin, (d.src[0].length + d.src[1].length) / 16);
     int64_t size[2] = {step0, step0};
     d.K = p->K;
     d.both.cap = (size_t)p->K + 2;
@@ -794,6 +844,8 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
             if (size[0] >= kAheadMin) d.start_ahead(size[0]);
         }
         done = d.certify();
+        if (!done && adaptive && d.depth[0] + d.depth[1] >= complete_at)
+            return finish_complete(d, p, out_ids, out_F, n_out, st);
         if (!done) {
             bool any_open = false;
             for (int i = 0; i < 2; ++i) any_open |= d.active[i] && !d.exhausted[i];
@@ -820,7 +872,7 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
             st->pulls[i] = d.pulls[i];
         }
         st->checks = d.checks;
-        st->reserved = 0;
+        st->complete = 0;
     }
     return PVS_OK;
 }
@@ -828,7 +880,7 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
 bool params_ok(const eahr_params* p) {
     return p && p->K >= 1 && p->k >= 1 && (p->form == EAHR_RANK_SCALED || p->form == EAHR_NUMERATOR) &&
            (p->policy == EAHR_POLICY_GEOMETRIC || p->policy == EAHR_POLICY_EQUAL_DEPTH ||
-            p->policy == EAHR_POLICY_FROZEN) &&
+            p->policy == EAHR_POLICY_FROZEN || p->policy == EAHR_POLICY_ADAPTIVE) &&
            p->step >= 0;
 }
 

@@ -157,6 +157,25 @@ const SnapData* cursor_snapshot(const pvs_cursor* c);
 // its next pull) instead of copied out.
 pvs_status next_pinned(pvs_cursor* c, int32_t n, const int64_t** ids, const float** scores,
                        int32_t* n_out);
+// Complete-list weighted RRF on the device (fusion.cu).  Per list i the
+// contribution of rank r is a[i] / (b[i] r + c[i]) (0 when a[i] == 0).
+struct FuseWeights {
+    double a[2], b[2], c[2];
+};
+// One item near the top of the fused order: the binary32 value of its fused
+// score (bits), its id and its ranks in the two lists (0: not in the list).
+struct FusedCand {
+    uint32_t fbits;
+    int32_t id, rd, rs;
+};
+// The candidates for T*_K of the complete dense ranking of `dense`'s query
+// over its snapshot and the host sparse list: every item of T*_K is among
+// them, in descending binary32 fused-score order (the caller orders them
+// exactly).  Does not use or change the cursor's ranked state.  Errors:
+// PVS_ERR_INVALID (a sparse id outside the snapshot, deleted or repeated),
+// PVS_ERR_OVERFLOW, PVS_ERR_OOM, PVS_ERR_CUDA.
+pvs_status fuse_complete(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
+                         const FuseWeights& w, int32_t K, std::vector<FusedCand>* out);
 // pvs_next_batch with each cursor's outputs at its own address: cursor i's
 // next n ranks to ids[i], scores[i] (device or host per outputs_on_device).
 pvs_status next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,

@@ -294,3 +294,82 @@ def test_snapshot_configuration_at_full_size():
         for snap in snaps:
             pvs.pvs_snapshot_free(snap)
         pvs.pvs_index_free(index)
+
+
+@pytest.mark.parametrize("tau", [0.5, 0.0, -0.5])
+def test_eahr_adaptive_policy_equals_complete_list_fusion(tau):
+    """EAHR_POLICY_ADAPTIVE (Sec. 2.2, last paragraph): geometric reading
+    until the lists are deep, then complete-list fusion on the device; the
+    ordered Top-K and its F equal the oracle's complete-list fusion."""
+    m, n = 256, 200_003
+    centres = synth.mixture_centres(256, m, seed=74, device="cpu")
+    V = synth.mixture_rows(n, centres, 0.35, seed=75).numpy()
+    q = synth.mixture_queries(1, centres, 0.5, seed=76).numpy()[0]
+    dense_ids, dense_sc = po.dense_ranking(q, V)
+    proxy = torch.from_numpy(dense_sc[np.argsort(dense_ids)].astype(np.float64))
+    sparse = synth.copula_ranking(proxy, tau, seed=77).numpy()
+    T = ro.target_topk_large([dense_ids, sparse], [1, 1], 60, 20, ro.NUMERATOR)
+    index = pvs.pvs_build(V)
+    try:
+        for policy in (pvs.EAHR_POLICY_ADAPTIVE, pvs.EAHR_POLICY_GEOMETRIC):
+            cur = pvs.pvs_cursor_open(index, q)
+            try:
+                ids, F, st = pvs.eahr_topk(cur, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                           policy=policy)
+            finally:
+                pvs.pvs_cursor_close(cur)
+            assert ids.tolist() == [x for x, _ in T]
+            for (x, f), got in zip(T, F):
+                if not np.isnan(got):
+                    assert got == ro.as_float(f)
+            if policy == pvs.EAHR_POLICY_ADAPTIVE:
+                assert st["complete"] == (1 if tau <= 0 else 0)
+                if st["complete"]:
+                    assert not np.isnan(F).any()
+        # the device finish checks the whole sparse list
+        if tau <= 0:
+            bad = sparse.copy()
+            bad[-1] = bad[0]                      # a repeated id, far down the list
+            cur = pvs.pvs_cursor_open(index, q)
+            try:
+                with pytest.raises(pvs.PvsError) as e:
+                    pvs.eahr_topk(cur, bad, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                  policy=pvs.EAHR_POLICY_ADAPTIVE)
+                assert e.value.status == pvs.PVS_ERR_INVALID
+            finally:
+                pvs.pvs_cursor_close(cur)
+    finally:
+        pvs.pvs_index_free(index)
+
+
+def test_eahr_at_passage_scale_equals_complete_list_fusion(passage):
+    """The EAHR configuration at full size (8,841,823 x 768, K = 20,
+    w / (60 + r)): one query per Kendall-tau level, a Gaussian-copula sparse
+    ranking of every id, both scheduling policies, against complete-list
+    fusion of the oracle's complete dense ranking (scored in row chunks)."""
+    dev, centres, rows, index = passage
+    Q = synth.mixture_queries(3, centres, 0.5, seed=1003)
+    Qh = Q.cpu().numpy()
+    scores = [[] for _ in range(3)]
+    for r in range(0, N_PASSAGE, 1 << 20):
+        Vh = rows[r:r + (1 << 20)].cpu().numpy()
+        for i in range(3):
+            scores[i].append(po.exact_scores(Qh[i], Vh))
+    ids_all = np.arange(N_PASSAGE, dtype=np.int64)
+    for i, tau in enumerate((0.5, 0.0, -0.5)):
+        s = np.concatenate(scores[i])
+        dense_ids = np.lexsort((ids_all, -s.astype(np.float64))).astype(np.int64)
+        sparse = synth.copula_ranking(torch.from_numpy(s.astype(np.float64)), tau,
+                                      seed=2003 + i).numpy()
+        T = ro.target_topk_large([dense_ids, sparse], [1, 1], 60, 20, ro.NUMERATOR)
+        for policy in (pvs.EAHR_POLICY_ADAPTIVE, pvs.EAHR_POLICY_GEOMETRIC):
+            cur = pvs.pvs_cursor_open(index, Q[i].contiguous())
+            try:
+                ids, F, st = pvs.eahr_topk(cur, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                           policy=policy)
+            finally:
+                pvs.pvs_cursor_close(cur)
+            assert ids.tolist() == [x for x, _ in T], (tau, policy)
+            for (x, f), got in zip(T, F):
+                if not np.isnan(got):
+                    assert got == ro.as_float(f)
