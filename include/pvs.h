@@ -403,8 +403,9 @@ enum {
                                     since the last check, and at once when a
                                     list is exhausted                          */
     EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk only: GEOMETRIC until the ranks
-                                    read reach max(2^18, (n_dense + n_sparse)
-                                    / 16), then complete-list fusion on the
+                                    read reach (n_dense + n_sparse) / 16,
+                                    clamped to [2^16, 2^18], then complete-list
+                                    fusion on the
                                     device (Sec. 2.2: when early determination
                                     is impossible, fusing the complete lists
                                     gives the same result): every visible

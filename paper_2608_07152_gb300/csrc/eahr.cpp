@@ -729,7 +729,11 @@ pvs_status run(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
 // fusion of the dense cursor's query and the host sparse list on the device,
 // then T*_K from the candidates it returns, ordered by exact rational F
 // (ties: smaller id first), zero-score items never appended (Sec. 2.1).
-constexpr int64_t kCompleteMin = (int64_t)1 << 18;
+// The switch: once the ranks read reach a sixteenth of both lists, but at
+// least kCompleteMin and at most kCompleteMax (the device finish costs about
+// one full scoring of the corpus, which reading deeper soon exceeds).
+constexpr int64_t kCompleteMin = (int64_t)1 << 16;
+constexpr int64_t kCompleteMax = (int64_t)1 << 18;
 
 pvs_status finish_complete(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
                            int32_t* n_out, eahr_stats* st) {
@@ -776,8 +780,8 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
                       int32_t* n_out, eahr_stats* st) {
     const int step0 = p->step > 0 ? p->step : 16;
     const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor && d.src[1].list;
-    const int64_t complete_at =
-        std::max<int64_t>(kCompleteMin, (d.src[0].length + d.src[1].length) / 16);
+    const int64_t complete_at = std::min(
+        kCompleteMax, std::max<int64_t>(kCompleteMin, (d.src[0].length + d.src[1].length) / 16));
     int64_t size[2] = {step0, step0};
     d.K = p->K;
     d.both.cap = (size_t)p->K + 2;
