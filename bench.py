@@ -83,8 +83,9 @@ def parse():
                    help="Kendall tau levels of --workload eahr (comma-separated)")
     p.add_argument("--eahr-policy", default="adaptive",
                    choices=["adaptive", "geometric", "frozen", "equal"],
-                   help="EAHR scheduling policy (adaptive: geometric reading, then complete-list "
-                        "fusion on the device once the lists are read deep)")
+                   help="EAHR scheduling policy (adaptive: geometric reading, then an exact finish "
+                        "on the device: ranks of the remaining candidates, else complete-list "
+                        "fusion)")
     p.add_argument("--no-eahr", action="store_true",
                    help="passage: leave out the EAHR Top-20 record of the default line")
     p.add_argument("--ablation-queries", type=int, default=30,
@@ -549,7 +550,8 @@ def eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts, ran
         qi += 1
     levels, lat_all = {}, []
     for tau, count in counts.items():
-        lat, cmp_ms, dd, ds, ex, pulls, complete = [], [], [], [], 0, [], 0
+        lat, cmp_ms, dd, ds, ex, pulls = [], [], [], [], 0, []
+        finish = {0: 0, 1: 0, 2: 0, 3: 0}
         ktau = None
         for j in range(count):
             q = queries[qi]
@@ -570,7 +572,7 @@ def eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts, ran
             dd.append(st["depth"][0])
             ds.append(st["depth"][1])
             ex += int(st["exhausted"][0] and st["exhausted"][1])
-            complete += int(st.get("complete", 0))
+            finish[int(st.get("complete", 0))] += 1
             pulls.append(st["pulls"][0])
             if comparator_queries is None or j < comparator_queries:
                 cmp_ms.append(comparator(q, torch.from_numpy(sp).to(dev)))
@@ -581,7 +583,8 @@ def eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts, ran
             "exhaustive_fp32_ms_p50": float(np.median(cmp_ms)) if cmp_ms else None,
             "dense_depth_p50": float(np.median(dd)), "dense_depth_mean": float(np.mean(dd)),
             "sparse_depth_p50": float(np.median(ds)), "both_exhausted": ex,
-            "finished_by_complete_fusion": complete,
+            "finished_by": {"reading": finish[0], "rank_intervals": finish[2],
+                            "exact_ranks": finish[3], "complete_list_fusion": finish[1]},
             "dense_pulls_p50": float(np.median(pulls))}
     return levels, lat_all
 

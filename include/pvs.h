@@ -402,17 +402,37 @@ enum {
                                     has grown by clamp(access / 8, 64, 1024)
                                     since the last check, and at once when a
                                     list is exhausted                          */
-    EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk only: GEOMETRIC until the ranks
-                                    read reach (n_dense + n_sparse) / 16,
-                                    clamped to [2^16, 2^18], then complete-list
-                                    fusion on the
-                                    device (Sec. 2.2: when early determination
-                                    is impossible, fusing the complete lists
-                                    gives the same result): every visible
-                                    row's authoritative score, both lists'
-                                    ranks, the fused order, exact rational
-                                    comparison of the items near the K-th.
-                                    The whole sparse list is then checked.
+    EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk only: GEOMETRIC reading, and
+                                    once the ranks read reach 2^12 (again
+                                    each time they double) an exact finish:
+                                    with LB the K-th largest L(x) of the
+                                    items read, and B < LB, only the items
+                                    with U(x) >= LB can be in T*_K; their
+                                    missing ranks come from the device: a
+                                    sparse rank from the host list, a dense
+                                    rank as an interval from counting the
+                                    rows whose bounds lie above or around
+                                    the item's authoritative score.  When
+                                    those intervals do not certify the order
+                                    (Sec. 2.2 over the candidates), the rows
+                                    around each score are scored and the
+                                    ranks are exact.  An F known only as an
+                                    interval is reported as NaN (its
+                                    position is certified).  Failing that
+                                    (too many candidates,
+                                    a cursor without bounds of every row),
+                                    once the ranks read reach (n_dense +
+                                    n_sparse) / 16 clamped to [2^16, 2^18]:
+                                    complete-list fusion on the device (every
+                                    visible row's authoritative score, both
+                                    lists' ranks, the fused order).  Both
+                                    finishes rest on Sec. 2.2 (when early
+                                    determination is impossible, fusing the
+                                    complete lists gives the same result).
+                                    Complete-list fusion, and an exact finish
+                                    that needs a sparse rank, read the whole
+                                    sparse list: an invalid id anywhere in it
+                                    then fails the call.
                                     Other entry points treat it as GEOMETRIC  */
 };
 
@@ -434,8 +454,12 @@ typedef struct eahr_stats {
     int32_t exhausted[2];   /* list i reached Exhausted                        */
     int32_t pulls[2];       /* producer calls per list                         */
     int32_t checks;         /* certification rounds                            */
-    int32_t complete;       /* 1: finished by complete-list fusion on the
-                               device (EAHR_POLICY_ADAPTIVE)                   */
+    int32_t complete;       /* how EAHR_POLICY_ADAPTIVE finished: 0 certified
+                               from the ranks read (Sec. 2.2), 1 complete-list
+                               fusion on the device, 2 the remaining
+                               candidates ordered by the rank intervals their
+                               rows' bounds give, 3 by exact ranks (rows
+                               scored)                                        */
 } eahr_stats;
 
 /* EAHR over a freshly opened dense cursor (no ranks delivered yet) and a

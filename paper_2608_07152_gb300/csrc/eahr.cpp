@@ -776,12 +776,198 @@ pvs_status finish_complete(Driver& d, const eahr_params* p, int64_t* out_ids, do
     return PVS_OK;
 }
 
+// EAHR_POLICY_ADAPTIVE's cheaper finish: exact ranks for the few items that
+// can still be in T*_K.  Let LB be the K-th largest L(x) over the items read
+// so far.  An item y with U(y) < LB cannot be in T*_K, because K items have
+// F >= L >= LB > F(y); neither can an unread item when B < LB.  The others
+// (the candidates) get their missing ranks from the device: the dense rank
+// by counting the rows above the item's exact score, the sparse one from the
+// host list.  Their F is then exact, and T*_K is their best K by (F desc, id
+// asc), zero scores excluded (Sec. 2.1).  Returns PVS_OK with *handled false
+// when it does not apply (B >= LB, fewer than K items read, too many
+// candidates: *retry stays true; a cursor without bounds of every row:
+// *retry false); the driver then reads on.
+constexpr int64_t kQueryAt = (int64_t)1 << 12;   // ranks read (both lists) before it is tried
+
+// Certification (Sec. 2.2) over a closed candidate set whose F lies in
+// [lo[t].F, hi[t].F]: repeatedly, the candidate first by (lower bound desc,
+// id asc) is next when its (lower bound, id) beats the (upper bound, id) of
+// every other candidate left.  Fills *order with up to K candidate indices,
+// zero scores excluded (Sec. 2.1); false when the bounds leave the order
+// open.
+bool order_by_bounds(const std::vector<Node>& lo, const std::vector<Node>& hi, int K,
+                     std::vector<int32_t>* order) {
+    order->clear();
+    const size_t n = lo.size();
+    std::vector<int32_t> by_lo(n), by_hi(n);
+    for (size_t t = 0; t < n; ++t) by_lo[t] = by_hi[t] = (int32_t)t;
+    std::sort(by_lo.begin(), by_lo.end(),
+              [&](int32_t a, int32_t b) { return NodeCmp()(lo[(size_t)a], lo[(size_t)b]); });
+    std::sort(by_hi.begin(), by_hi.end(),
+              [&](int32_t a, int32_t b) { return NodeCmp()(hi[(size_t)a], hi[(size_t)b]); });
+    std::vector<uint8_t> taken(n, 0);
+    size_t p_lo = 0, p_hi = 0;
+    while ((int)order->size() < K) {
+        while (p_lo < n && taken[(size_t)by_lo[p_lo]]) ++p_lo;
+        if (p_lo == n) break;
+        const int32_t x = by_lo[p_lo];
+        while (p_hi < n && taken[(size_t)by_hi[p_hi]]) ++p_hi;
+        // the strongest other candidate by (upper bound, id)
+        size_t q = p_hi;
+        if (q < n && by_hi[q] == x) {
+            ++q;
+            while (q < n && taken[(size_t)by_hi[q]]) ++q;
+        }
+        if (q < n && !beats(lo[(size_t)x].F, lo[(size_t)x].id, hi[(size_t)by_hi[q]].F,
+                            hi[(size_t)by_hi[q]].id))
+            return false;
+        if (lo[(size_t)x].F.num == 0) {   // nothing left with a positive score
+            if (hi[(size_t)x].F.num != 0) return false;
+            break;
+        }
+        order->push_back(x);
+        taken[(size_t)x] = 1;
+    }
+    return true;
+}
+
+pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
+                               int32_t* n_out, eahr_stats* st, bool* handled, bool* retry) {
+    *handled = false;
+    *retry = true;
+    pvs_cursor* c = d.src[0].cursor;
+    // ranks already pulled are recorded first: the helper thread's pull, and
+    // any ranks the cursor computed ahead (served without device work), so
+    // that every item still unread is also undelivered by the cursor
+    if (d.ahead_live) {
+        d.join_ahead();
+        if (d.ahead_status < 0) return d.ahead_status;
+        d.pulls[0]++;
+        if (!d.record(0, d.ahead_ids, d.ahead_got)) return PVS_ERR_INVALID;
+        if (d.ahead_status == PVS_EXHAUSTED || d.depth[0] >= d.src[0].length) {
+            d.exhausted[0] = true;
+            d.src[0].length = d.depth[0];
+        }
+        if (d.certify()) return PVS_OK;   // the extra ranks decided it: the caller reports
+    }
+    if (!d.exhausted[0] && c->ahead > 0) {
+        pvs_status s = d.pull(0, c->ahead);
+        if (s < 0) return s;
+        if (d.certify()) return PVS_OK;
+    }
+    const int K = p->K;
+    // the K-th largest L over the items read (each once)
+    std::vector<Node> known;
+    known.reserve(d.prefix[0].size() + d.prefix[1].size());
+    for (int32_t x : d.prefix[0]) known.push_back(Node{d.L(x), x});
+    for (int32_t x : d.prefix[1])
+        if (!d.rank(0, x)) known.push_back(Node{d.L(x), x});
+    if ((int64_t)known.size() < K) return PVS_OK;
+    std::nth_element(known.begin(), known.begin() + (K - 1), known.end(), NodeCmp());
+    const Frac LB = known[(size_t)K - 1].F;
+    if (LB.num == 0 || cmp(add(d.u(0), d.u(1)), LB) >= 0) return PVS_OK;
+    // candidates and the ranks they miss
+    std::vector<int32_t> cand, need_d, need_s;
+    for (const Node& nd : known) {
+        if (cmp(d.U(nd.id), LB) < 0) continue;
+        cand.push_back(nd.id);
+        for (int i = 0; i < 2; ++i) {
+            if (!d.active[i] || d.exhausted[i] || d.rank(i, nd.id)) continue;
+            (i == 0 ? need_d : need_s).push_back(nd.id);
+        }
+    }
+    if ((int64_t)need_d.size() > pvs::kRankQueryMax || (int64_t)need_s.size() > pvs::kRankQueryMax)
+        return PVS_OK;
+    // first the dense rank intervals the rows' bounds give (no row scored)
+    std::vector<int64_t> rd_lo(need_d.size()), rd_hi(need_d.size()), rs(need_s.size());
+    bool supported = false;
+    pvs_status s = pvs::rank_queries(c, need_d.data(), (int32_t)need_d.size(), false,
+                                     d.src[1].list, d.src[1].length, need_s.data(),
+                                     (int32_t)need_s.size(), rd_lo.data(), rd_hi.data(), rs.data(),
+                                     &supported);
+    if (s != PVS_OK) return s;
+    if (!supported) {   // this cursor never supports it
+        *retry = false;
+        return PVS_OK;
+    }
+    // F of every candidate, an interval while a dense rank is one
+    std::vector<size_t> at_d(cand.size(), SIZE_MAX), at_s(cand.size(), SIZE_MAX);
+    {
+        std::vector<std::pair<int32_t, size_t>> pos(cand.size());
+        for (size_t t = 0; t < cand.size(); ++t) pos[t] = {cand[t], t};
+        std::sort(pos.begin(), pos.end());
+        auto slot = [&](int32_t x) {
+            return std::lower_bound(pos.begin(), pos.end(), std::make_pair(x, (size_t)0))->second;
+        };
+        for (size_t t = 0; t < need_d.size(); ++t) at_d[slot(need_d[t])] = t;
+        for (size_t t = 0; t < need_s.size(); ++t) at_s[slot(need_s[t])] = t;
+    }
+    std::vector<Node> lo(cand.size()), hi(cand.size());
+    auto fill = [&]() {
+        for (size_t t = 0; t < cand.size(); ++t) {
+            const int32_t x = cand[t];
+            Frac Fl, Fh;
+            for (int i = 0; i < 2; ++i) {
+                if (!d.active[i]) continue;
+                int64_t r = d.rank(i, x), r_hi = r;
+                if (!r && i == 0 && at_d[t] != SIZE_MAX) {
+                    r = rd_lo[at_d[t]];
+                    r_hi = rd_hi[at_d[t]];
+                } else if (!r && i == 1 && at_s[t] != SIZE_MAX) {
+                    r = r_hi = rs[at_s[t]];
+                }
+                if (r > 0) {
+                    Fh = add(Fh, d.g[i].at(r));
+                    Fl = add(Fl, d.g[i].at(r_hi));
+                }
+            }
+            lo[t] = Node{Fl, x};
+            hi[t] = Node{Fh, x};
+        }
+    };
+    fill();
+    std::vector<int32_t> order;
+    bool scored = false;
+    if (!order_by_bounds(lo, hi, K, &order)) {
+        scored = true;
+        // the intervals leave the order open: exact dense ranks
+        s = pvs::rank_queries(c, need_d.data(), (int32_t)need_d.size(), true, nullptr, 0, nullptr,
+                              0, rd_lo.data(), rd_hi.data(), nullptr, &supported);
+        if (s != PVS_OK) return s;
+        fill();
+        order_by_bounds(lo, hi, K, &order);   // decided now: lo == hi
+    }
+    // F is reported where it is known exactly (a point interval), NaN where
+    // only the position is certified (as for an item unread in an Open list)
+    const int32_t q = (int32_t)order.size();
+    for (int32_t t = 0; t < q; ++t) {
+        const size_t u = (size_t)order[(size_t)t];
+        out_ids[t] = lo[u].id;
+        if (out_F)
+            out_F[t] = cmp(lo[u].F, hi[u].F) == 0 ? frac_to_double(lo[u].F) : std::nan("");
+    }
+    *n_out = q;
+    if (st) {
+        for (int i = 0; i < 2; ++i) {
+            st->depth[i] = d.depth[i];
+            st->length[i] = d.src[i].length;
+            st->exhausted[i] = d.exhausted[i] ? 1 : 0;
+            st->pulls[i] = d.pulls[i];
+        }
+        st->checks = d.checks;
+        st->complete = scored ? 3 : 2;
+    }
+    *handled = true;
+    return PVS_OK;
+}
+
 pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
                       int32_t* n_out, eahr_stats* st) {
     const int step0 = p->step > 0 ? p->step : 16;
     const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor && d.src[1].list;
     const int64_t complete_at = std::min(
         kCompleteMax, std::max<int64_t>(kCompleteMin, (d.src[0].length + d.src[1].length) / 16));
+    int64_t query_at = kQueryAt;
     int64_t size[2] = {step0, step0};
     d.K = p->K;
     d.both.cap = (size_t)p->K + 2;
@@ -848,6 +1034,15 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
             if (size[0] >= kAheadMin) d.start_ahead(size[0]);
         }
         done = d.certify();
+        if (!done && adaptive && d.depth[0] + d.depth[1] >= query_at) {
+            bool handled = false, retry = true;
+            pvs_status s = finish_rank_queries(d, p, out_ids, out_F, n_out, st, &handled, &retry);
+            if (s < 0) return s;
+            if (handled) return PVS_OK;
+            done = d.certify();   // ranks the attempt recorded may have decided it
+            // else again after as much reading, or never
+            query_at = retry ? 2 * (d.depth[0] + d.depth[1]) : std::numeric_limits<int64_t>::max();
+        }
         if (!done && adaptive && d.depth[0] + d.depth[1] >= complete_at)
             return finish_complete(d, p, out_ids, out_F, n_out, st);
         if (!done) {

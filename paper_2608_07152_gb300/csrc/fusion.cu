@@ -1,10 +1,10 @@
-// Complete-list weighted RRF on the device: the fallback of EAHR's adaptive
-// policy when both ranked lists must be read deep (arXiv 2608.07152, Sec. 2.1
-// defines T*_K over the complete lists; Sec. 2.2's last paragraph notes that
-// when early determination is impossible, fusing the complete lists gives
-// the same result).
+// Complete-list weighted RRF on the device: the finishes of EAHR's adaptive
+// policy when both ranked lists would have to be read deep (arXiv 2608.07152,
+// Sec. 2.1 defines T*_K over the complete lists; Sec. 2.2's last paragraph
+// notes that when early determination is impossible, fusing the complete
+// lists gives the same result).
 //
-// Steps, one request, on the dense cursor's stream:
+// fuse_complete, one request, on the dense cursor's stream:
 //   1. the complete dense ranking: the authoritative score of every visible
 //      row (the exhaustive scanning generator's kernel) and one sort by
 //      (score desc, id asc); rank_d[x] = position + 1;
@@ -18,11 +18,25 @@
 //      below the K-th key's: every item of T*_K is among them (the binary64
 //      error of F is far below a binary32 step), and the caller orders them
 //      with exact rational arithmetic.
+//
+// rank_queries, the cheaper finish: the exact ranks of a few items only, in
+// the list they have not been read from.
+//   dense  the item's authoritative score s_x fixes its key (s_x, x); its
+//          rank is one plus the number of visible rows whose key is larger.
+//          Every row's interval [lo, hi] (App. A.1) decides that comparison
+//          unless s_x lies inside it; only such rows are scored exactly.
+//          Rows the cursor has delivered (bounds set to -inf) rank before
+//          every item not yet delivered.  One pass over the bounds counts
+//          for all items at once: a row adds one to the items whose keys
+//          are below its own, a prefix of the items' sorted keys;
+//   sparse one scatter of the host list (as step 2 above), read at the
+//          items' ids.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <vector>
 
+#include "exact_dot.cuh"
 #include "kernels.h"
 #include "pvs_common.cuh"
 #include "runtime.h"
@@ -86,6 +100,161 @@ __global__ void top_entries_kernel(const uint64_t* __restrict__ keys, int64_t m,
 int grid_of(int64_t n) {
     const int64_t g = (n + 255) / 256;
     return (int)std::max<int64_t>(1, std::min<int64_t>(g, 152 * 8));
+}
+
+// The queried items' keys (score, id) in ascending order, in one CTA:
+// keys[i] = rank_key(score of ids[i], ids[i]), bitonic sort in shared memory.
+__global__ void __launch_bounds__(kRankQueryMax) query_keys_kernel(const int64_t* __restrict__ ids,
+                                                                   const float* __restrict__ scores,
+                                                                   int n, uint64_t* keys,
+                                                                   int* status) {
+    __shared__ uint64_t sk[kRankQueryMax];
+    int pow2 = 1;
+    while (pow2 < n) pow2 <<= 1;
+    for (int i = threadIdx.x; i < pow2; i += blockDim.x) {
+        uint64_t k = ~0ull;   // padding sorts last
+        if (i < n) {
+            const float s = scores[i];
+            if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
+            k = rank_key(s, (uint32_t)ids[i]);
+        }
+        sk[i] = k;
+    }
+    __syncthreads();
+    for (int size = 2; size <= pow2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = threadIdx.x; i < pow2; i += blockDim.x) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool up = (i & size) == 0;
+                    const uint64_t a = sk[i], b = sk[j];
+                    if ((a > b) == up) {
+                        sk[i] = b;
+                        sk[j] = a;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) keys[i] = sk[i];
+}
+
+// Number of keys below x, and at most x (keys ascending).
+__device__ __forceinline__ int keys_below(const uint64_t* k, int n, uint64_t x) {
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (k[mid] < x) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+__device__ __forceinline__ int keys_at_most(const uint64_t* k, int n, uint64_t x) {
+    int lo = 0, hi = n;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (k[mid] <= x) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+constexpr int kCountWarps = 8;
+
+// hist[j] = number of visible rows whose key lies above exactly j of the
+// queried keys (sorted ascending); the rank of the item with the j-th
+// smallest key is then 1 + sum of hist[t] for t > j.  A row's key lies in
+// [key(lo, y), key(hi, y)]; when no queried key falls in that range the
+// count is fixed by the bounds.  Otherwise, with `exact`, the row's
+// authoritative score is computed (and must lie in its interval, App. A.1);
+// without, the row counts in hist[a] (a = the queried keys below key(lo, y):
+// it is surely above those) and may lie above the keys a .. b-1 (b = the
+// keys at most key(hi, y)): maybe[a] += 1, maybe[b] -= 1, so that the prefix
+// sum of `maybe` at j counts the rows that may lie above the j-th key.  A
+// row with hi = -inf has been delivered and lies above every queried key.
+__global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
+    const float* __restrict__ lo, const float* __restrict__ hi, int64_t rows,
+    const uint32_t* __restrict__ tomb, const float* __restrict__ qraw,
+    const float* __restrict__ raw, int m_raw, const uint64_t* __restrict__ qkeys, int nq,
+    int exact, unsigned long long* hist, unsigned long long* maybe, int* status,
+    DevCounters* ctr) {
+    __shared__ uint64_t sk[kRankQueryMax];
+    __shared__ unsigned int sh[kRankQueryMax + 1];
+    __shared__ int sm[kRankQueryMax + 1];
+    for (int i = threadIdx.x; i < nq; i += blockDim.x) sk[i] = qkeys[i];
+    for (int i = threadIdx.x; i <= nq; i += blockDim.x) {
+        sh[i] = 0;
+        sm[i] = 0;
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int64_t step = (int64_t)gridDim.x * kCountWarps * 32;
+    unsigned long long scored = 0, fallbacks = 0;
+    for (int64_t base = ((int64_t)blockIdx.x * kCountWarps + (threadIdx.x >> 5)) * 32; base < rows;
+         base += step) {
+        const int64_t y = base + lane;
+        int bin = -1;   // -1: nothing to count from the bounds
+        bool straddle = false;
+        float l = 0.f, h = 0.f;
+        if (y < rows && !tombstoned(tomb, y)) {
+            l = lo[y];
+            h = hi[y];
+            if (h == -INFINITY) {
+                bin = nq;
+            } else {
+                const int a = keys_below(sk, nq, rank_key(l, (uint32_t)y));
+                const int b = keys_at_most(sk, nq, rank_key(h, (uint32_t)y));
+                if (a == b) {
+                    bin = a;
+                } else if (exact) {
+                    straddle = true;
+                } else {
+                    bin = a;
+                    atomicAdd(&sm[a], 1);
+                    atomicAdd(&sm[b], -1);
+                }
+            }
+        }
+        // one shared-memory add per distinct bin of the warp
+        const unsigned int live = __ballot_sync(0xffffffffu, bin >= 0);
+        if (bin >= 0) {
+            const unsigned int same = __match_any_sync(live, bin);
+            if (lane == __ffs(same) - 1) atomicAdd(&sh[bin], (unsigned int)__popc(same));
+        }
+        unsigned int todo = __ballot_sync(0xffffffffu, straddle);
+        while (todo) {
+            const int src = __ffs(todo) - 1;
+            todo &= todo - 1;
+            const int64_t r = base + src;
+            bool fb = false;
+            const float s = exact_dot_warp_eft(qraw, qraw, raw + r * (int64_t)m_raw, m_raw, &fb);
+            const float lr = __shfl_sync(0xffffffffu, l, src);
+            const float hr = __shfl_sync(0xffffffffu, h, src);
+            if (lane == 0) {
+                if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
+                else if (s < lr || s > hr) set_status(status, PVS_ERR_INTERVAL);
+                atomicAdd(&sh[keys_below(sk, nq, rank_key(s, (uint32_t)r))], 1u);
+                ++scored;
+                fallbacks += fb ? 1 : 0;
+            }
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i <= nq; i += blockDim.x) {
+        if (sh[i]) atomicAdd(&hist[i], (unsigned long long)sh[i]);
+        if (sm[i]) atomicAdd(&maybe[i], (unsigned long long)(long long)sm[i]);   // mod 2^64
+    }
+    if (lane == 0 && scored) {
+        atomicAdd(&ctr->refined, scored);
+        if (fallbacks) atomicAdd(&ctr->exact_fallbacks, fallbacks);
+    }
+}
+
+__global__ void gather_ranks_kernel(const int32_t* __restrict__ rank_of,
+                                    const int32_t* __restrict__ ids, int n, int32_t* out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) out[i] = rank_of[ids[i]];
 }
 
 }  // namespace
@@ -223,6 +392,215 @@ pvs_status fuse_complete(pvs_cursor* c, const int64_t* sparse, int64_t ns, const
     }
     cleanup();
 #undef FUSE_CUDA
+    return result;
+}
+
+pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, bool exact,
+                        const int64_t* sparse, int64_t ns, const int32_t* sparse_ids, int32_t nsq,
+                        int64_t* dense_lo, int64_t* dense_hi, int64_t* sparse_rank,
+                        bool* supported) {
+    if (supported) *supported = false;
+    if (!c || !c->index || !supported || nd < 0 || nsq < 0 || nd > kRankQueryMax ||
+        nsq > kRankQueryMax || ns < 0 || (nd > 0 && (!dense_ids || !dense_lo || !dense_hi)) ||
+        (nsq > 0 && (!sparse_ids || !sparse_rank || (ns > 0 && !sparse))))
+        return PVS_ERR_INVALID;
+    if (c->state < 0) return PVS_ERR_FAILED;
+    if (nd > 0 && (c->generator != PVS_GEN_INTERVALS || c->batch_ws || !c->scanned || !c->lo ||
+                   c->ahead != 0))
+        return PVS_OK;   // not supported: the caller finishes another way
+    *supported = true;
+    pvs_index* x = c->index;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (prev != x->device) cudaSetDevice(x->device);
+    struct Restore {
+        int dev;
+        ~Restore() {
+            if (dev >= 0) cudaSetDevice(dev);
+        }
+    } restore{prev != x->device ? prev : -1};
+
+    const SnapData* sd = c->snap.get();
+    const int64_t rows = sd->rows;
+    for (int32_t i = 0; i < nd; ++i)
+        if (dense_ids[i] < 0 || dense_ids[i] >= rows || !sd->is_visible(dense_ids[i]))
+            return PVS_ERR_INVALID;
+    for (int32_t i = 0; i < nsq; ++i)
+        if (sparse_ids[i] < 0 || sparse_ids[i] >= rows) return PVS_ERR_INVALID;
+    const uint32_t* tomb = sd->d_tomb;
+    cudaStream_t st = c->stream;
+    cudaStream_t st2 = nullptr;
+    cudaEvent_t ev = nullptr;
+    std::vector<void*> held;
+    auto alloc = [&](size_t bytes, cudaStream_t s) -> void* {
+        void* p = nullptr;
+        if (cudaMallocFromPoolAsync(&p, std::max<size_t>(bytes, 16), x->scratch_pool, s) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        held.push_back(p);
+        return p;
+    };
+    auto cleanup = [&]() {
+        if (st2 && ev && cudaEventRecord(ev, st2) == cudaSuccess) cudaStreamWaitEvent(st, ev, 0);
+        for (void* p : held) cudaFreeAsync(p, st);
+        if (ev) cudaEventDestroy(ev);
+        if (st2) cudaStreamDestroy(st2);
+        cudaGetLastError();
+    };
+#define RQ_CUDA(expr)                                              \
+    do {                                                           \
+        cudaError_t e_ = (expr);                                   \
+        if (e_ != cudaSuccess) {                                   \
+            cudaGetLastError();                                    \
+            cleanup();                                             \
+            return e_ == cudaErrorMemoryAllocation ? PVS_ERR_OOM   \
+                                                   : PVS_ERR_CUDA; \
+        }                                                          \
+    } while (0)
+    if (cudaStreamCreateWithFlags(&st2, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        cleanup();
+        return PVS_ERR_CUDA;
+    }
+    // host staging: the queried ids in, the counts and ranks out (pinned,
+    // so the copies are asynchronous; freed after the final wait)
+    struct Pinned {
+        void* p = nullptr;
+        ~Pinned() {
+            if (p) cudaFreeHost(p);
+        }
+    } pin;
+    const size_t id_bytes = (size_t)std::max(nd, 1) * 8 + (size_t)std::max(nsq, 1) * 4;
+    const size_t out_bytes = (size_t)(nd + 1) * 16 + (size_t)std::max(nd, 1) * 8 +
+                             (size_t)std::max(nsq, 1) * 4 + 2 * sizeof(int);
+    if (cudaMallocHost(&pin.p, id_bytes + out_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        cleanup();
+        return PVS_ERR_OOM;
+    }
+    int64_t* h_dids = static_cast<int64_t*>(pin.p);
+    int32_t* h_sids = reinterpret_cast<int32_t*>(h_dids + std::max(nd, 1));
+    unsigned long long* h_hist =
+        reinterpret_cast<unsigned long long*>(static_cast<char*>(pin.p) + id_bytes);
+    unsigned long long* h_maybe = h_hist + nd + 1;
+    uint64_t* h_keys = reinterpret_cast<uint64_t*>(h_maybe + nd + 1);
+    int32_t* h_srank = reinterpret_cast<int32_t*>(h_keys + std::max(nd, 1));
+    int* h_status = reinterpret_cast<int*>(h_srank + std::max(nsq, 1));
+    for (int32_t i = 0; i < nd; ++i) h_dids[i] = dense_ids[i];
+    for (int32_t i = 0; i < nsq; ++i) h_sids[i] = sparse_ids[i];
+    h_status[0] = h_status[1] = 0;
+
+    int* status = static_cast<int*>(alloc(2 * sizeof(int), st));
+    if (!status) {
+        cleanup();
+        return PVS_ERR_OOM;
+    }
+    RQ_CUDA(cudaMemsetAsync(status, 0, 2 * sizeof(int), st));
+    RQ_CUDA(cudaEventRecord(ev, st));   // st2 uses the status word too
+    RQ_CUDA(cudaStreamWaitEvent(st2, ev, 0));
+    // dense: the items' scores and sorted keys, then one pass over the bounds
+    if (nd > 0) {
+        int64_t* d_dids = static_cast<int64_t*>(alloc((size_t)nd * 8, st));
+        float* d_score = static_cast<float*>(alloc((size_t)nd * 4, st));
+        uint64_t* d_keys = static_cast<uint64_t*>(alloc((size_t)nd * 8, st));
+        unsigned long long* d_hist =
+            static_cast<unsigned long long*>(alloc((size_t)(nd + 1) * 16, st));
+        unsigned long long* d_maybe = d_hist + nd + 1;
+        if (!d_dids || !d_score || !d_keys || !d_hist) {
+            cleanup();
+            return PVS_ERR_OOM;
+        }
+        RQ_CUDA(cudaMemcpyAsync(d_dids, h_dids, (size_t)nd * 8, cudaMemcpyHostToDevice, st));
+        RQ_CUDA(cudaMemsetAsync(d_hist, 0, (size_t)(nd + 1) * 16, st));
+        RQ_CUDA(launch_score_ids(d_dids, nd, c->qraw, x->raw, x->m_raw, d_score, c->ctr, st));
+        count_launches(1);
+        query_keys_kernel<<<1, kRankQueryMax, 0, st>>>(d_dids, d_score, nd, d_keys, status);
+        RQ_CUDA(cudaGetLastError());
+        int grid = 0;
+        RQ_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&grid, rank_count_kernel,
+                                                              kCountWarps * 32, 0));
+        int64_t blocks = (int64_t)std::max(grid, 1) * std::max(x->num_sms, 1);
+        blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, (rows + kCountWarps * 32 - 1) /
+                                                                    (kCountWarps * 32)));
+        count_launches(1);
+        rank_count_kernel<<<(unsigned)blocks, kCountWarps * 32, 0, st>>>(
+            c->lo, c->hi, rows, tomb, c->qraw, x->raw, x->m_raw, d_keys, nd, exact ? 1 : 0,
+            d_hist, d_maybe, status, c->ctr);
+        RQ_CUDA(cudaGetLastError());
+        RQ_CUDA(cudaMemcpyAsync(h_hist, d_hist, (size_t)(nd + 1) * 16, cudaMemcpyDeviceToHost,
+                                st));
+        RQ_CUDA(cudaMemcpyAsync(h_keys, d_keys, (size_t)nd * 8, cudaMemcpyDeviceToHost, st));
+    }
+    // sparse: scatter the list, read the queried ids (second stream; a copy
+    // from pageable memory may hold this thread until it is done, so the
+    // dense work is queued first)
+    int32_t* d_srank = nullptr;
+    if (nsq > 0) {
+        int32_t* rank_of = static_cast<int32_t*>(alloc((size_t)std::max<int64_t>(rows, 1) * 4, st2));
+        int64_t* d_list = static_cast<int64_t*>(alloc((size_t)std::max<int64_t>(ns, 1) * 8, st2));
+        int32_t* d_sids = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
+        d_srank = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
+        if (!rank_of || !d_list || !d_sids || !d_srank) {
+            cleanup();
+            return PVS_ERR_OOM;
+        }
+        RQ_CUDA(cudaMemsetAsync(rank_of, 0, (size_t)std::max<int64_t>(rows, 1) * 4, st2));
+        RQ_CUDA(cudaMemcpyAsync(d_sids, h_sids, (size_t)nsq * 4, cudaMemcpyHostToDevice, st2));
+        if (ns > 0) {
+            RQ_CUDA(cudaMemcpyAsync(d_list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice, st2));
+            count_launches(1);
+            list_rank_kernel<<<grid_of(ns), 256, 0, st2>>>(d_list, ns, rows, tomb, rank_of,
+                                                           status + 1);
+            RQ_CUDA(cudaGetLastError());
+        }
+        count_launches(1);
+        gather_ranks_kernel<<<(nsq + 255) / 256, 256, 0, st2>>>(rank_of, d_sids, nsq, d_srank);
+        RQ_CUDA(cudaGetLastError());
+        RQ_CUDA(cudaMemcpyAsync(h_srank, d_srank, (size_t)nsq * 4, cudaMemcpyDeviceToHost, st2));
+    }
+    RQ_CUDA(cudaEventRecord(ev, st2));
+    RQ_CUDA(cudaStreamWaitEvent(st, ev, 0));
+    RQ_CUDA(cudaMemcpyAsync(h_status, status, 2 * sizeof(int), cudaMemcpyDeviceToHost, st));
+    RQ_CUDA(cudaStreamSynchronize(st));
+    pvs_status result = PVS_OK;
+    if (h_status[0] != 0) result = (pvs_status)h_status[0];
+    else if (h_status[1] != 0) result = (pvs_status)h_status[1];
+    if (result == PVS_OK) {
+        // the item with the j-th smallest key: 1 + rows surely above it, plus
+        // the rows that may be above it
+        unsigned long long above = 0, may = 0;
+        struct Ranks {
+            int32_t id;
+            int64_t lo, hi;
+            bool operator<(const Ranks& o) const { return id < o.id; }
+        };
+        std::vector<Ranks> by_id((size_t)nd);
+        for (int32_t j = nd - 1; j >= 0; --j) {
+            above += h_hist[j + 1];
+            by_id[(size_t)j].id = (int32_t)rank_key_id(h_keys[j]);
+            by_id[(size_t)j].lo = (int64_t)above + 1;
+        }
+        for (int32_t j = 0; j < nd; ++j) {
+            may += h_maybe[j];   // prefix sum of the differences (mod 2^64)
+            by_id[(size_t)j].hi = by_id[(size_t)j].lo + (int64_t)may;
+        }
+        std::sort(by_id.begin(), by_id.end());
+        for (int32_t i = 0; i < nd; ++i) {
+            const auto it = std::lower_bound(by_id.begin(), by_id.end(), Ranks{dense_ids[i], 0, 0});
+            if (it == by_id.end() || it->id != dense_ids[i]) {
+                result = PVS_ERR_INVALID;   // a repeated item
+                break;
+            }
+            dense_lo[i] = it->lo;
+            dense_hi[i] = it->hi;
+        }
+        for (int32_t i = 0; i < nsq; ++i) sparse_rank[i] = h_srank[i];
+    }
+    cleanup();
+#undef RQ_CUDA
     return result;
 }
 

@@ -176,6 +176,24 @@ struct FusedCand {
 // PVS_ERR_OVERFLOW, PVS_ERR_OOM, PVS_ERR_CUDA.
 pvs_status fuse_complete(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
                          const FuseWeights& w, int32_t K, std::vector<FusedCand>* out);
+// Ranks of a few items (fusion.cu).  Dense: row dense_ids[i]'s rank in the
+// complete dense ranking of `dense`'s query over its snapshot (1-based) lies
+// in [dense_lo[i], dense_hi[i]]; with `exact` the two are equal, else they
+// come from the rows' intervals alone (no row is scored exactly; the item's
+// own row may be counted in the width).  Sparse: sparse_rank[i] = the
+// position + 1 of sparse_ids[i] in the host list `sparse` (0: not in it).
+// The dense items must be visible and not yet delivered by the cursor, and
+// the cursor must hold no ranks computed ahead of delivery.  *supported is
+// false, and nothing runs, when the cursor keeps no bounds of every row (a
+// batched working set, the full-scan generator).  At most kRankQueryMax
+// items per list.  Errors: PVS_ERR_INVALID (a bad argument, or a sparse id
+// outside the snapshot, deleted or repeated), PVS_ERR_INTERVAL (an exact
+// score outside its interval), PVS_ERR_OVERFLOW, PVS_ERR_OOM, PVS_ERR_CUDA.
+constexpr int32_t kRankQueryMax = 1024;
+pvs_status rank_queries(pvs_cursor* dense, const int32_t* dense_ids, int32_t nd, bool exact,
+                        const int64_t* sparse, int64_t ns, const int32_t* sparse_ids, int32_t nsq,
+                        int64_t* dense_lo, int64_t* dense_hi, int64_t* sparse_rank,
+                        bool* supported);
 // pvs_next_batch with each cursor's outputs at its own address: cursor i's
 // next n ranks to ids[i], scores[i] (device or host per outputs_on_device).
 pvs_status next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,
