@@ -56,7 +56,7 @@ WORKLOAD = ("passage-scale single-query ranking: N=8,841,823 x d=768 Gaussian mi
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--steps", type=int, default=60)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="pvs", choices=["pvs", "reference"])
     p.add_argument("--queries", type=int, default=64, help="queries per step")
@@ -246,7 +246,7 @@ def build_corpus_index(pvs, synth, torch, n, stream, device, components=COMPONEN
     return index, centres, time.perf_counter() - t0
 
 
-PIPELINE = 4   # passage: executor worker threads, each with a group of queries in flight
+PIPELINE = 8   # passage: executor worker threads, each with a group of queries in flight
 
 
 def _finish(pvs, cur, stats_acc):
@@ -290,6 +290,7 @@ def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget
     rows = 1 << 20
     V = synth.mixture_rows(rows, centres_dev, WITHIN_STD, seed=2, first=0).cpu().numpy()
     t0 = time.perf_counter()
+    c0 = time.process_time()
     done = 0
     while done < len(queries_host):
         ids, sc = po.dense_ranking(queries_host[done], V)
@@ -298,13 +299,15 @@ def cpu_baseline(synth, torch, centres_dev, queries_host, n_full, seconds_budget
         if time.perf_counter() - t0 > seconds_budget:
             break
     dt = time.perf_counter() - t0
+    cores = (time.process_time() - c0) / dt   # the cores it kept busy on average
     per_query_full = dt / done * (n_full / rows)
     return {"value": RANKS_PER_QUERY / per_query_full, "unit": UNIT,
-            "cores": os.cpu_count(), "kind": "oracle", "projected": True,
+            "cores": round(cores, 1), "host_cores": os.cpu_count(), "kind": "oracle",
+            "projected": True,
             "sample": f"{done} queries x first {RANKS_PER_QUERY} exact ranks over the first "
-                      f"{rows:,} corpus rows (oracle: binary64 scoring by numpy's BLAS on "
-                      f"{os.cpu_count()} threads + exact fallback + full sort); projected to "
-                      f"N by scaling the time by N/{rows:,}"}
+                      f"{rows:,} corpus rows (oracle: binary64 scoring by numpy's BLAS, "
+                      f"exact fallback in Python, full sort; cores = process CPU time / wall "
+                      f"time); projected to N by scaling the time by N/{rows:,}"}
 
 
 def reference_arm(args):
@@ -323,9 +326,12 @@ def reference_arm(args):
     for w in range(args.warmup):
         po.dense_ranking(Q[w], V)
     t0 = time.perf_counter()
+    c0 = time.process_time()
     for s in range(args.steps):
         po.dense_ranking(Q[args.warmup + s], V)
-    dt = (time.perf_counter() - t0) / args.steps * (args.n / rows)
+    wall = time.perf_counter() - t0
+    cores = (time.process_time() - c0) / wall   # the cores it kept busy on average
+    dt = wall / args.steps * (args.n / rows)
     value = RANKS_PER_QUERY / dt
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -333,8 +339,8 @@ def reference_arm(args):
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": WORKLOAD, "N": args.n, "d": DIM,
                        "step": "1 query, first 1,000 ranks"},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(),
-                             "kind": "oracle", "projected": True,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": round(cores, 1),
+                             "host_cores": os.cpu_count(), "kind": "oracle", "projected": True,
                              "sample": f"1 query per step over the first {rows:,} rows; "
                                        f"projected to N by scaling the time by N/{rows:,}"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -392,7 +398,10 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     n = BATCH_N if args.n == N_CORPUS else args.n
     index, centres, build_s = build_corpus_index(pvs, synth, torch, n, stream.cuda_stream, dev,
                                                  components=BATCH_COMPONENTS, seed=4)
-    nb = args.warmup + args.steps
+    # every host thread warms up on its own batches (the cursor pool and the
+    # scratch pool grow to what four batches in flight hold)
+    warm = max(args.warmup, 2 * BATCH_PIPELINE)
+    nb = warm + args.steps
     queries = synth.mixture_queries(nb * BATCH_Q, centres, QUERY_NOISE, seed=query_seed(5, rank))
     queries = queries.reshape(nb, BATCH_Q, DIM).contiguous()
     streams = [torch.cuda.Stream(device=dev) for _ in range(BATCH_PIPELINE)]
@@ -423,7 +432,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                 step(queries[b], k, pass_ms)
         _run_threads(worker, BATCH_PIPELINE)
 
-    run(list(range(args.warmup)), None)
+    run(list(range(warm)), None)
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
@@ -435,7 +444,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         start.record(stream)
         for s_ in streams:
             s_.wait_event(start)
-        run(list(range(args.warmup, nb)), pass_ms)
+        run(list(range(warm, nb)), pass_ms)
         for s_ in streams:                      # join every stream's work
             done = torch.cuda.Event()
             done.record(s_)
@@ -444,7 +453,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         stream.synchronize()
     launches = pvs.pvs_launch_count() - launches0
     stats = []   # per-query counters from one more (untimed) batch of the same queries
-    step(queries[args.warmup], 0, None, stats)
+    step(queries[warm], 0, None, stats)
     elapsed = start.elapsed_time(end) / 1e3
     elapsed = slowest(pg, elapsed, dev)
     ranks_total = args.steps * BATCH_Q * BATCH_RANKS * world
@@ -456,7 +465,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
 
     def e2e_worker(k):
         torch.cuda.set_device(dev)
-        for b in range(args.warmup + k, nb, BATCH_PIPELINE):
+        for b in range(warm + k, nb, BATCH_PIPELINE):
             curs = pvs.pvs_cursor_open_batch(index, qh[b], horizon=BATCH_RANKS,
                                              stream=streams[k])
             for _ in range(BATCH_RANKS // BATCH_CHUNK):
@@ -474,7 +483,7 @@ def main_batched(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     peak, peak_kind = bf16_peak()
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": elapsed / args.steps * 1e3,
+        "warmup": warm, "ms_per_step": elapsed / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": BATCH_WORKLOAD, "N": n, "d": DIM, "queries_per_batch": BATCH_Q,
