@@ -441,8 +441,10 @@ typedef struct eahr_params {
     int32_t k;          /* RRF rank constant, >= 1                             */
     int32_t form;       /* EAHR_RANK_SCALED or EAHR_NUMERATOR                  */
     int32_t policy;     /* EAHR_POLICY_*                                       */
-    int32_t step;       /* first pull size (GEOMETRIC) or step (EQUAL_DEPTH,
-                           FROZEN); 0 selects 16                               */
+    int32_t step;       /* first pull size (GEOMETRIC, ADAPTIVE) or step
+                           (EQUAL_DEPTH, FROZEN); 0 selects 16, or 2^11 for
+                           ADAPTIVE (its exact finish is first tried once
+                           2^12 ranks are read)                              */
     int32_t w_num[2];   /* channel weights w_i = w_num[i] / w_den[i];          */
     int32_t w_den[2];   /* [0] dense, [1] sparse; 0 <= w_num < 2^16,
                            1 <= w_den < 2^16                                   */

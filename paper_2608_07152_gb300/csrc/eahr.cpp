@@ -373,6 +373,31 @@ class Driver {
         ahead_live = false;
     }
 
+    // The host sparse list scattered on the device by a helper thread while
+    // the dense list is read (EAHR_POLICY_ADAPTIVE's finishes use it).
+    std::thread stage;
+    bool stage_live = false;
+    pvs_status stage_status = PVS_OK;
+    pvs::StagedList* staged = nullptr;
+
+    void start_stage() {
+        if (stage_live || !src[0].cursor || !src[1].list || src[1].length == 0) return;
+        try {
+            stage = std::thread([this] {
+                stage_status = pvs::stage_sparse_list(src[0].cursor, src[1].list,
+                                                      src[1].length, &staged);
+            });
+            stage_live = true;
+        } catch (...) {   // no thread: the finish copies the list itself
+        }
+    }
+    // The staged list once it is queued (null when staging failed).
+    const pvs::StagedList* staged_list() {
+        if (stage_live) stage.join();
+        stage_live = false;
+        return stage_status == PVS_OK ? staged : nullptr;
+    }
+
     int32_t rank(int i, int32_t x) const { return ranks[2 * (size_t)x + (size_t)i]; }
     bool inA(int32_t x) const { return (bits[(uint32_t)x >> 6] >> (x & 63)) & 1u; }
 
@@ -380,6 +405,8 @@ class Driver {
     // clear those, or whole arrays when that is cheaper, and pool them.
     ~Driver() {
         join_ahead();
+        staged_list();
+        pvs::free_staged_list(staged);
         if (!ws.ranks) return;
         if ((int64_t)(prefix[0].size() + prefix[1].size()) > ws.cap / 8) {
             zero_parallel(ranks, (size_t)ws.cap * 2 * sizeof(int32_t));
@@ -884,7 +911,7 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
     pvs_status s = pvs::rank_queries(c, need_d.data(), (int32_t)need_d.size(), false,
                                      d.src[1].list, d.src[1].length, need_s.data(),
                                      (int32_t)need_s.size(), rd_lo.data(), rd_hi.data(), rs.data(),
-                                     &supported);
+                                     &supported, need_s.empty() ? nullptr : d.staged_list());
     if (s != PVS_OK) return s;
     if (!supported) {   // this cursor never supports it
         *retry = false;
@@ -963,8 +990,11 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
 
 pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
                       int32_t* n_out, eahr_stats* st) {
-    const int step0 = p->step > 0 ? p->step : 16;
     const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor && d.src[1].list;
+    if (adaptive) d.start_stage();
+    // the adaptive policy reads its first kQueryAt ranks in one pull per list
+    // (its finish is tried there; fewer, larger pulls cost fewer round trips)
+    const int step0 = p->step > 0 ? p->step : (adaptive ? (int)(kQueryAt / 2) : 16);
     const int64_t complete_at = std::min(
         kCompleteMax, std::max<int64_t>(kCompleteMin, (d.src[0].length + d.src[1].length) / 16));
     int64_t query_at = kQueryAt;

@@ -34,6 +34,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <new>
 #include <vector>
 
 #include "exact_dot.cuh"
@@ -395,14 +396,91 @@ pvs_status fuse_complete(pvs_cursor* c, const int64_t* sparse, int64_t ns, const
     return result;
 }
 
+struct StagedList {
+    pvs_index* index = nullptr;
+    cudaStream_t stream = nullptr;
+    cudaEvent_t ready = nullptr;
+    int32_t* rank_of = nullptr;
+    int64_t* list = nullptr;
+    int* status = nullptr;
+    int64_t rows = 0;
+};
+
+void free_staged_list(StagedList* s) {
+    if (!s) return;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (s->index) cudaSetDevice(s->index->device);
+    if (s->stream) {
+        if (s->rank_of) cudaFreeAsync(s->rank_of, s->stream);
+        if (s->list) cudaFreeAsync(s->list, s->stream);
+        if (s->status) cudaFreeAsync(s->status, s->stream);
+        cudaStreamSynchronize(s->stream);
+        cudaStreamDestroy(s->stream);
+    }
+    if (s->ready) cudaEventDestroy(s->ready);
+    cudaGetLastError();
+    if (prev >= 0) cudaSetDevice(prev);
+    delete s;
+}
+
+pvs_status stage_sparse_list(pvs_cursor* c, const int64_t* sparse, int64_t ns,
+                             StagedList** out) {
+    *out = nullptr;
+    if (!c || !c->index || ns < 0 || (ns > 0 && !sparse)) return PVS_ERR_INVALID;
+    pvs_index* x = c->index;
+    if (cudaSetDevice(x->device) != cudaSuccess) {
+        cudaGetLastError();
+        return PVS_ERR_CUDA;
+    }
+    StagedList* s = new (std::nothrow) StagedList();
+    if (!s) return PVS_ERR_OOM;
+    s->index = x;
+    s->rows = c->snap->rows;
+    const uint32_t* tomb = c->snap->d_tomb;
+    const size_t rows = (size_t)std::max<int64_t>(s->rows, 1);
+    auto failed = [&](cudaError_t e) {
+        cudaGetLastError();
+        free_staged_list(s);
+        return e == cudaErrorMemoryAllocation ? PVS_ERR_OOM : PVS_ERR_CUDA;
+    };
+    cudaError_t e = cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&s->ready, cudaEventDisableTiming);
+    if (e == cudaSuccess)
+        e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->rank_of), rows * 4,
+                                    x->scratch_pool, s->stream);
+    if (e == cudaSuccess)
+        e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->list),
+                                    (size_t)std::max<int64_t>(ns, 1) * 8, x->scratch_pool,
+                                    s->stream);
+    if (e == cudaSuccess)
+        e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->status), sizeof(int),
+                                    x->scratch_pool, s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->rank_of, 0, rows * 4, s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->status, 0, sizeof(int), s->stream);
+    if (e == cudaSuccess && ns > 0)
+        e = cudaMemcpyAsync(s->list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice, s->stream);
+    if (e != cudaSuccess) return failed(e);
+    if (ns > 0) {
+        count_launches(1);
+        list_rank_kernel<<<grid_of(ns), 256, 0, s->stream>>>(s->list, ns, s->rows, tomb,
+                                                             s->rank_of, s->status);
+        e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(s->ready, s->stream);
+    if (e != cudaSuccess) return failed(e);
+    *out = s;
+    return PVS_OK;
+}
+
 pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, bool exact,
                         const int64_t* sparse, int64_t ns, const int32_t* sparse_ids, int32_t nsq,
                         int64_t* dense_lo, int64_t* dense_hi, int64_t* sparse_rank,
-                        bool* supported) {
+                        bool* supported, const StagedList* staged) {
     if (supported) *supported = false;
     if (!c || !c->index || !supported || nd < 0 || nsq < 0 || nd > kRankQueryMax ||
         nsq > kRankQueryMax || ns < 0 || (nd > 0 && (!dense_ids || !dense_lo || !dense_hi)) ||
-        (nsq > 0 && (!sparse_ids || !sparse_rank || (ns > 0 && !sparse))))
+        (nsq > 0 && (!sparse_ids || !sparse_rank || (ns > 0 && !sparse && !staged))))
         return PVS_ERR_INVALID;
     if (c->state < 0) return PVS_ERR_FAILED;
     if (nd > 0 && (c->generator != PVS_GEN_INTERVALS || c->batch_ws || !c->scanned || !c->lo ||
@@ -538,18 +616,31 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
     // from pageable memory may hold this thread until it is done, so the
     // dense work is queued first)
     int32_t* d_srank = nullptr;
+    if (nsq > 0 && staged && staged->rows != rows) {
+        cleanup();
+        return PVS_ERR_INVALID;
+    }
     if (nsq > 0) {
-        int32_t* rank_of = static_cast<int32_t*>(alloc((size_t)std::max<int64_t>(rows, 1) * 4, st2));
-        int64_t* d_list = static_cast<int64_t*>(alloc((size_t)std::max<int64_t>(ns, 1) * 8, st2));
+        const bool own = staged == nullptr;
+        int32_t* rank_of =
+            own ? static_cast<int32_t*>(alloc((size_t)std::max<int64_t>(rows, 1) * 4, st2))
+                : staged->rank_of;
+        int64_t* d_list =
+            own ? static_cast<int64_t*>(alloc((size_t)std::max<int64_t>(ns, 1) * 8, st2))
+                : staged->list;
         int32_t* d_sids = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
         d_srank = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
         if (!rank_of || !d_list || !d_sids || !d_srank) {
             cleanup();
             return PVS_ERR_OOM;
         }
-        RQ_CUDA(cudaMemsetAsync(rank_of, 0, (size_t)std::max<int64_t>(rows, 1) * 4, st2));
+        if (own) RQ_CUDA(cudaMemsetAsync(rank_of, 0, (size_t)std::max<int64_t>(rows, 1) * 4, st2));
         RQ_CUDA(cudaMemcpyAsync(d_sids, h_sids, (size_t)nsq * 4, cudaMemcpyHostToDevice, st2));
-        if (ns > 0) {
+        if (!own) {   // scattered already: its verdict becomes this call's
+            RQ_CUDA(cudaStreamWaitEvent(st2, staged->ready, 0));
+            RQ_CUDA(cudaMemcpyAsync(status + 1, staged->status, sizeof(int),
+                                    cudaMemcpyDeviceToDevice, st2));
+        } else if (ns > 0) {
             RQ_CUDA(cudaMemcpyAsync(d_list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice, st2));
             count_launches(1);
             list_rank_kernel<<<grid_of(ns), 256, 0, st2>>>(d_list, ns, rows, tomb, rank_of,

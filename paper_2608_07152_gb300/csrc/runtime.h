@@ -190,10 +190,20 @@ pvs_status fuse_complete(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
 // outside the snapshot, deleted or repeated), PVS_ERR_INTERVAL (an exact
 // score outside its interval), PVS_ERR_OVERFLOW, PVS_ERR_OOM, PVS_ERR_CUDA.
 constexpr int32_t kRankQueryMax = 1024;
+// A host sparse list scattered on the device ahead of need: rank_of[x] =
+// position + 1 of id x (0: not in the list), its ids checked as in
+// fuse_complete (the verdict is read when the ranks are used).  Built on its
+// own stream by stage_sparse_list (which may hold the calling thread while
+// the pageable list is copied); rank_queries orders its reads after it.
+struct StagedList;
+pvs_status stage_sparse_list(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
+                             StagedList** out);
+void free_staged_list(StagedList* s);
+// `staged` (or null): the same list, already scattered.
 pvs_status rank_queries(pvs_cursor* dense, const int32_t* dense_ids, int32_t nd, bool exact,
                         const int64_t* sparse, int64_t ns, const int32_t* sparse_ids, int32_t nsq,
                         int64_t* dense_lo, int64_t* dense_hi, int64_t* sparse_rank,
-                        bool* supported);
+                        bool* supported, const StagedList* staged = nullptr);
 // pvs_next_batch with each cursor's outputs at its own address: cursor i's
 // next n ranks to ids[i], scores[i] (device or host per outputs_on_device).
 pvs_status next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t n,

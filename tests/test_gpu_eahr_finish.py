@@ -57,10 +57,13 @@ def _check(got, F, T):
             assert v == ro.as_float(f)
 
 
-def _run(index, q, sparse, snap=None, **kw):
+def _run(index, q, sparse, snap=None, step=16, **kw):
+    """Adaptive EAHR; step = 16 keeps geometric pulls small, so that the
+    lists are read to the finish threshold before certification could end the
+    request (step = 0, the default, reads 2^11 ranks per list at once)."""
     cur = pvs.pvs_cursor_open(index, q, snap)
     try:
-        return pvs.eahr_topk(cur, sparse, policy=pvs.EAHR_POLICY_ADAPTIVE, **kw)
+        return pvs.eahr_topk(cur, sparse, policy=pvs.EAHR_POLICY_ADAPTIVE, step=step, **kw)
     finally:
         pvs.pvs_cursor_close(cur)
 
@@ -78,6 +81,10 @@ def test_rank_query_finish_matches_complete_list_fusion(corpus, tau):
     if tau <= 0:
         assert st["complete"] in (2, 3)
         assert st["depth"][0] + st["depth"][1] < N   # finished well before the end
+    # the default first pull (2^11 ranks per list): the same result
+    ids, F, st = _run(index, q, sparse, step=0, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+    _check(ids, F, T)
+    assert st["complete"] in (0, 2, 3)
 
 
 @pytest.mark.parametrize("K,weights,form", [
@@ -174,7 +181,7 @@ def test_complete_list_fusion_finish_and_many_candidates(corpus):
     try:
         pvs.pvs_cursor_set_generator(cur, pvs.PVS_GEN_FULL_SCAN)
         ids, F, st = pvs.eahr_topk(cur, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR,
-                                   policy=pvs.EAHR_POLICY_ADAPTIVE)
+                                   policy=pvs.EAHR_POLICY_ADAPTIVE, step=16)
     finally:
         pvs.pvs_cursor_close(cur)
     _check(ids, F, T)
@@ -200,7 +207,7 @@ def test_rank_query_finish_on_grouped_cursors_and_a_bad_sparse_list(corpus):
     try:
         for c, (sparse, T) in zip(curs, refs):
             ids, F, st = pvs.eahr_topk(c, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR,
-                                       policy=pvs.EAHR_POLICY_ADAPTIVE)
+                                       policy=pvs.EAHR_POLICY_ADAPTIVE, step=16)
             _check(ids, F, T)
             assert st["complete"] in (2, 3)
     finally:
