@@ -598,6 +598,12 @@ def eahr_levels(pvs, synth, torch, np, index, rows, queries, policy, counts, ran
     return levels, lat_all
 
 
+def eahr_policy(args, pvs):
+    return {"geometric": pvs.EAHR_POLICY_GEOMETRIC, "frozen": pvs.EAHR_POLICY_FROZEN,
+            "equal": pvs.EAHR_POLICY_EQUAL_DEPTH,
+            "adaptive": pvs.EAHR_POLICY_ADAPTIVE}[args.eahr_policy]
+
+
 def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     """EAHR end to end over the passage corpus: per query a sparse channel that
     is a complete ranking of all N ids, a Gaussian-copula permutation of the
@@ -623,9 +629,7 @@ def main_eahr(args, pvs, synth, torch, np, rank, world, local, dev, pg):
               for t in [float(x) for x in args.eahr_levels.split(",")]}
     total_q = sum(counts.values()) + 2
     queries = synth.mixture_queries(total_q, centres, QUERY_NOISE, seed=query_seed(3, rank))
-    policy = {"geometric": pvs.EAHR_POLICY_GEOMETRIC, "frozen": pvs.EAHR_POLICY_FROZEN,
-              "equal": pvs.EAHR_POLICY_EQUAL_DEPTH,
-              "adaptive": pvs.EAHR_POLICY_ADAPTIVE}[args.eahr_policy]
+    policy = eahr_policy(args, pvs)
 
     if pg:
         pg.barrier()
@@ -1268,6 +1272,7 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
             snap = pvs.pvs_snapshot_create(index)
             vis_ids = torch.nonzero(visible[:size]).squeeze(1)
             lat, depth, ex_any, ex_both, near_ties, swaps = [], [], 0, 0, None, None
+            finish = {0: 0, 1: 0, 2: 0, 3: 0}
             for j in range(args.snap_queries):
                 q = queries[qi]
                 qi += 1
@@ -1277,10 +1282,12 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                 t = time.perf_counter()
                 cur = pvs.pvs_cursor_open(index, q, snap)
                 ids, F, st = pvs.eahr_topk(cur, sparse, K=EAHR_K, k=EAHR_RRF_K,
-                                           form=pvs.EAHR_NUMERATOR)
+                                           form=pvs.EAHR_NUMERATOR,
+                                           policy=eahr_policy(args, pvs))
                 pvs.pvs_cursor_close(cur)
                 lat.append((time.perf_counter() - t) * 1e3)
                 depth.append(st["depth"][0])
+                finish[int(st.get("complete", 0))] += 1
                 ex_any += int(st["exhausted"][0] or st["exhausted"][1])
                 ex_both += int(st["exhausted"][0] and st["exhausted"][1])
                 if j == 0:   # near ties among the first 1,000 dense ranks of this snapshot
@@ -1307,7 +1314,9 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                 "exhaustion_rate_any": ex_any / args.snap_queries,
                 "exhaustion_rate_both": ex_both / args.snap_queries,
                 "near_tie_pairs_first_1000": near_ties,
-                "oracle_mismatches_first_1000": swaps})
+                "oracle_mismatches_first_1000": swaps,
+                "finished_by": {"reading": finish[0], "rank_intervals": finish[2],
+                                "exact_ranks": finish[3], "complete_list_fusion": finish[1]}})
     launches = pvs.pvs_launch_count() - launches0
     p50 = float(np.median(lat_all))
     line = {
@@ -1318,7 +1327,7 @@ def main_snapshots(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         "config": {"workload": "adversarial ties + snapshots: N=2,000,000 x d=1,024 mixture with "
                                "20% near-duplicates (std 1e-4), +10% appended and 2% tombstoned "
                                "per snapshot, 5 snapshots, EAHR Top-20, sparse Kendall tau 0.2",
-                   "N": n0, "d": d, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
+                   "N": n0, "d": d, "K": EAHR_K, "rrf_k": EAHR_RRF_K, "policy": args.eahr_policy,
                    "l2": "no flush: every query's interval pass streams >= 2 GB of codes",
                    "parallelism": f"replicas x{world}"},
         "e2e": {"value": p50, "unit": "ms", "h2d_bytes_per_step": d * 4,
