@@ -100,8 +100,9 @@ struct LaneQuery {
     bool on;
 };
 
-__device__ __forceinline__ void eval_row(const IntervalGroupArgs& a, LaneQuery& Q, float dot_f,
-                                         float sv, float vn, float en, int64_t row) {
+// Returns the row's upper bound (-inf for a deleted row).
+__device__ __forceinline__ float eval_row(const IntervalGroupArgs& a, LaneQuery& Q, float dot_f,
+                                          float sv, float vn, float en, int64_t row) {
     float lo, hi;
     interval_epilogue(__float2int_rn(dot_f), Q.q, sv, vn, en, lo, hi);
     if (!isfinite(lo) || !isfinite(hi)) set_status(a.status[Q.n], PVS_ERR_OVERFLOW);
@@ -109,6 +110,7 @@ __device__ __forceinline__ void eval_row(const IntervalGroupArgs& a, LaneQuery& 
     a.lo[Q.n][row] = lo;
     a.hi[Q.n][row] = hi;
     top_insert(Q.top, lo);
+    return hi;
 }
 
 // B fragments in shared memory for rows wider than this many 64-byte groups.
@@ -265,11 +267,26 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[s]);
         const int64_t row_a = t * TR + ia, row_b = t * TR + ib;
+        float bm[2] = {-INFINITY, -INFINITY};
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
             if (!Q[u].on) continue;
-            if (row_a < a.rows) eval_row(a, Q[u], d[0][u], sa, va, ea, row_a);
-            if (row_b < a.rows) eval_row(a, Q[u], d[0][2 + u], sb, vb, eb, row_b);
+            if (row_a < a.rows) bm[u] = eval_row(a, Q[u], d[0][u], sa, va, ea, row_a);
+            if (row_b < a.rows)
+                bm[u] = fmaxf(bm[u], eval_row(a, Q[u], d[0][2 + u], sb, vb, eb, row_b));
+        }
+        // the warp's 16 rows: the lanes of one query pair differ in bits 2-4
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            bm[u] = fmaxf(bm[u], __shfl_xor_sync(0xffffffffu, bm[u], 4));
+            bm[u] = fmaxf(bm[u], __shfl_xor_sync(0xffffffffu, bm[u], 8));
+            bm[u] = fmaxf(bm[u], __shfl_xor_sync(0xffffffffu, bm[u], 16));
+        }
+        if (g == 0) {
+            const int64_t b = t * (TR / kBmaxRows) + blk;
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+                if (Q[u].on && a.bmax[Q[u].n] && b * kBmaxRows < a.rows) a.bmax[Q[u].n][b] = bm[u];
         }
     }
     const size_t slot = ((size_t)blockIdx.x * kGroupWarps + warp) * 8 + g;

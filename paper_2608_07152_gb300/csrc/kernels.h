@@ -216,8 +216,12 @@ struct IntervalGroupArgs {
     float* hi[kGroupMax];
     int* status[kGroupMax];
     float* slot_top[kGroupMax];
+    // largest upper bound of each 16-row block ((rows + 15) / 16 floats per
+    // query; -inf where no row is live), or null
+    float* bmax[kGroupMax];
     unsigned long long wait_ns = kWaitLimitNs;
 };
+constexpr int kBmaxRows = 16;
 // True when a grouped pass serves nq queries over rows of m_pad bytes.
 bool interval_group_supported(int m_pad, int nq);
 cudaError_t launch_interval_group(const IntervalGroupArgs& a, int num_sms, cudaStream_t st);
@@ -241,6 +245,10 @@ struct WsGroupArgs {
     float* w_hi[kGroupMax];
     unsigned int* w_len[kGroupMax];
     unsigned int* scratch[kGroupMax];   // compact_scratch_elems(rows) each
+    // the pass's 16-row block maxima of hi (upper bounds of the current hi:
+    // refinement and delivery only lower a row's upper bound), or null; with
+    // all of them set, only the blocks that reach the threshold are read
+    const float* bmax[kGroupMax];
 };
 cudaError_t launch_ws_group(const WsGroupArgs& a, cudaStream_t st);
 int64_t interval_group_slots(int64_t rows, int m_pad, int nq, int num_sms,

@@ -197,7 +197,7 @@ std::shared_ptr<SnapData> make_snapdata(const pvs_index* x) {
 
 void cursor_free_device(pvs_cursor* c) {
     dev_free(c->zq), dev_free(c->qraw), dev_free(c->qs);
-    dev_free(c->lo), dev_free(c->hi);
+    dev_free(c->lo), dev_free(c->hi), dev_free(c->bmax);
     dev_free(c->w_id), dev_free(c->w_lo), dev_free(c->w_hi);
     dev_free(c->compact_scratch), dev_free(c->slot_top);
     c->slot_cap = 0;
@@ -227,6 +227,7 @@ void cursor_reset(pvs_cursor* c) {
     c->rows = c->visible = c->emitted = 0;
     c->state = PVS_OK;
     c->scanned = false;
+    c->bmax_valid = false;
     c->batch_ws = false;
     c->fresh_ws = false;
     c->horizon = c->horizon_base = 0;
@@ -256,7 +257,8 @@ constexpr size_t kCursorPool = 1024;
 constexpr size_t kCursorPoolBytes = size_t(4) << 30;
 
 size_t cursor_device_bytes(const pvs_cursor* c) {
-    return (size_t)c->cap_rows * 12 + (size_t)c->cap_w * 40 + 4096 + kFrontCap * 4 +
+    return (size_t)c->cap_rows * 12 + (size_t)c->cap_rows / 4 + (size_t)c->cap_w * 40 + 4096 +
+           kFrontCap * 4 +
            (size_t)c->scan_cap * 20;
 }
 
@@ -265,11 +267,13 @@ size_t cursor_device_bytes(const pvs_cursor* c) {
 // Bounds of every row of the snapshot (single-query interval pass).
 pvs_status cursor_alloc_full(pvs_cursor* c) {
     if (c->lo && c->cap_rows >= c->rows) return PVS_OK;
-    dev_free(c->lo), dev_free(c->hi), dev_free(c->compact_scratch);
+    dev_free(c->lo), dev_free(c->hi), dev_free(c->bmax), dev_free(c->compact_scratch);
     c->cap_rows = 0;
+    c->bmax_valid = false;
     const size_t n = (size_t)std::max<int64_t>(c->rows, 1);
     PVS_CUDA(dev_alloc(&c->lo, n));
     PVS_CUDA(dev_alloc(&c->hi, n));
+    PVS_CUDA(dev_alloc(&c->bmax, (n + kBmaxRows - 1) / kBmaxRows));
     PVS_CUDA(dev_alloc(&c->compact_scratch, compact_scratch_elems((int64_t)n)));
     c->cap_rows = (int64_t)n;
     return PVS_OK;
@@ -424,6 +428,7 @@ pvs_status interval_pass(pvs_cursor* c) {
     c->interval_passes++;
     c->code_bytes += c->rows * (int64_t)(x->m_pad + 12);
     c->scanned = true;
+    c->bmax_valid = false;   // this pass writes no block maxima
     if (x->wait_ns < kWaitLimitNs) {
         // a shortened wait limit (pvs_index_set_wait_limit) makes a timed-out
         // pass likely: its bounds are then incomplete, so its status is read
@@ -498,6 +503,7 @@ pvs_status build_first_working_sets(pvs_cursor* const* cs, int32_t nc, const int
         a.w_hi[a.n] = c->w_hi;
         a.w_len[a.n] = &c->ctr->w_len;
         a.scratch[a.n] = c->compact_scratch;
+        a.bmax[a.n] = c->bmax_valid ? c->bmax : nullptr;
         picked[a.n] = c;
         H_of[a.n] = H;
         ++a.n;
@@ -1481,6 +1487,7 @@ pvs_status group_pass(pvs_index* x, pvs_cursor* const* cs, int nq, cudaStream_t 
         a.qs[i] = c->qs;
         a.lo[i] = c->lo;
         a.hi[i] = c->hi;
+        a.bmax[i] = c->bmax;
         a.status[i] = c->d_status;
         if (!c->ev_begin) {
             PVS_CUDA(cudaEventCreate(&c->ev_begin));
@@ -1508,6 +1515,7 @@ pvs_status group_pass(pvs_index* x, pvs_cursor* const* cs, int nq, cudaStream_t 
         c->code_bytes += c->rows * (int64_t)(x->m_pad + 12) / nq;
         c->group_size = nq;
         c->scanned = true;
+        c->bmax_valid = true;
     }
     if (x->wait_ns < kWaitLimitNs) {   // as in interval_pass: check before any pull
         PVS_CUDA(cudaStreamSynchronize(ps));

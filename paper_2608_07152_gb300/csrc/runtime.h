@@ -88,6 +88,10 @@ struct pvs_cursor {
     int64_t cap_rows = 0;
     float* lo = nullptr;
     float* hi = nullptr;
+    // the largest hi of each 16-row block, written by a grouped pass (upper
+    // bounds of hi from then on: refinement and delivery only lower hi)
+    float* bmax = nullptr;
+    bool bmax_valid = false;
     // working set (ordered by id): rows that can hold the next `horizon` ranks
     int64_t cap_w = 0;                // capacity of the working-set arrays
     bool batch_ws = false;            // working set came from a batched pass (no full bounds)

@@ -358,6 +358,77 @@ __global__ void compact_scatter_group_kernel(const __grid_constant__ WsGroupArgs
                          a.w_hi[g]);
 }
 
+// The same count and ordered scatter from the 16-row block maxima of hi: a
+// thread takes one block of 16 rows (a CTA the same 4,096 rows as above, so
+// the block counts and their scan are shared), and reads its rows only when
+// the block's maximum reaches the threshold (for tau = 0, every live row:
+// when the block holds one).
+__device__ __forceinline__ bool bmax_reaches(const float* bmax, int64_t b, uint32_t tau) {
+    const float m = bmax[b];
+    return tau != 0u ? fkey(m) >= tau : m != -INFINITY;
+}
+
+__device__ __forceinline__ unsigned int bmax_block_members(const float* lo, const float* hi,
+                                                           int64_t r0, int64_t rows,
+                                                           uint32_t tau) {
+    unsigned int c = 0;
+    const int64_t r1 = r0 + kBmaxRows < rows ? r0 + kBmaxRows : rows;
+    for (int64_t i = r0; i < r1; ++i) c += ws_member(lo, hi, i, tau) ? 1u : 0u;
+    return c;
+}
+
+__global__ void compact_count_bmax_group_kernel(const __grid_constant__ WsGroupArgs a) {
+    __shared__ unsigned int wsum[kCompactBlock / 32];
+    const int g = blockIdx.y;
+    const uint32_t tau = (uint32_t)a.sel[g]->prefix;
+    const int64_t b = (int64_t)blockIdx.x * kCompactBlock + threadIdx.x;
+    const int64_t r0 = b * kBmaxRows;
+    unsigned int c = 0;
+    if (r0 < a.rows && bmax_reaches(a.bmax[g], b, tau))
+        c = bmax_block_members(a.lo[g], a.hi[g], r0, a.rows, tau);
+    c = warp_sum(c);
+    if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = c;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned int s = 0;
+        for (int w = 0; w < kCompactBlock / 32; ++w) s += wsum[w];
+        a.scratch[g][blockIdx.x] = s;
+    }
+}
+
+__global__ void compact_scatter_bmax_group_kernel(const __grid_constant__ WsGroupArgs a) {
+    __shared__ unsigned int wtot[kCompactBlock / 32];
+    const int g = blockIdx.y;
+    const uint32_t tau = (uint32_t)a.sel[g]->prefix;
+    const float* lo = a.lo[g];
+    const float* hi = a.hi[g];
+    const int64_t b = (int64_t)blockIdx.x * kCompactBlock + threadIdx.x;
+    const int64_t r0 = b * kBmaxRows;
+    const bool live = r0 < a.rows && bmax_reaches(a.bmax[g], b, tau);
+    const unsigned int c = live ? bmax_block_members(lo, hi, r0, a.rows, tau) : 0u;
+    // exclusive prefix of c over the CTA, in thread (= row) order
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned int inc = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int v = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += v;
+    }
+    if (lane == 31) wtot[warp] = inc;
+    __syncthreads();
+    unsigned int pos = a.scratch[g][blockIdx.x] + inc - c;
+    for (int w = 0; w < warp; ++w) pos += wtot[w];
+    if (c == 0) return;
+    const int64_t r1 = r0 + kBmaxRows < a.rows ? r0 + kBmaxRows : a.rows;
+    for (int64_t i = r0; i < r1; ++i) {
+        if (!ws_member(lo, hi, i, tau)) continue;
+        a.w_id[g][pos] = (int32_t)i;
+        a.w_lo[g][pos] = lo[i];
+        a.w_hi[g][pos] = hi[i];
+        ++pos;
+    }
+}
+
 cudaError_t launch_ws_group(const WsGroupArgs& a, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
     if (a.n > kGroupMax || a.slot_n <= 0) return cudaErrorInvalidValue;
@@ -379,10 +450,18 @@ cudaError_t launch_ws_group(const WsGroupArgs& a, cudaStream_t st) {
         }
         return cudaGetLastError();
     }
+    bool by_blocks = true;
+    for (int g = 0; g < a.n; ++g) by_blocks = by_blocks && a.bmax[g] != nullptr;
     count_launches(3);
-    compact_count_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
-    scan_counts_group_kernel<<<a.n, 1024, 0, st>>>(a, nb);
-    compact_scatter_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+    if (by_blocks) {
+        compact_count_bmax_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+        scan_counts_group_kernel<<<a.n, 1024, 0, st>>>(a, nb);
+        compact_scatter_bmax_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+    } else {
+        compact_count_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+        scan_counts_group_kernel<<<a.n, 1024, 0, st>>>(a, nb);
+        compact_scatter_group_kernel<<<dim3((unsigned)nb, a.n), kCompactBlock, 0, st>>>(a);
+    }
     return cudaGetLastError();
 }
 
