@@ -1451,7 +1451,9 @@ def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     passes = st1["interval_passes"] - st0["interval_passes"]
     pass_ms = (st1["interval_ms"] - st0["interval_ms"]) / max(passes, 1)
     read_bytes = n * (m_pad + 12)
-    write_bytes = 8 * n * group
+    # bounds (lo, hi) of every row per query, and with groups the largest
+    # upper bound of each 16-row block per query
+    write_bytes = 8 * n * group + (4 * ((n + 15) // 16) * group if group > 1 else 0)
     alg_bytes = read_bytes + write_bytes
     achieved = alg_bytes / (pass_ms / 1e3) / 1e9
     peak, peak_kind = measured_peaks()
