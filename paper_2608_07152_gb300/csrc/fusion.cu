@@ -163,6 +163,64 @@ __device__ __forceinline__ int keys_at_most(const uint64_t* k, int n, uint64_t x
 
 constexpr int kCountWarps = 8;
 
+// fp32 inner product of q and v (m_raw floats, 16-byte aligned, zero padded)
+// by one warp: each lane a chain of FMAs over its float4s, then a butterfly
+// sum; every lane returns the same f and the same *err >= |f - q.v|.  Each
+// product is exact inside its FMA and then takes part in at most
+// n = 4 ceil(n4 / 32) + 5 roundings, so (Higham, Accuracy and Stability of
+// Numerical Algorithms, Sec. 3.1 and 3.3; gamma_n = n u / (1 - n u), u = 2^-24)
+//   |f - q.v| <= gamma_n S + k 2^-150,   S = sum |q_j v_j|,
+// k the roundings that may fall in the subnormal range (32 n + 32 at most;
+// 2^-149 per rounding below covers the growth of those terms).  S is bounded
+// the same way from its own fp32 chain g:  S <= (g + k 2^-149) / (1 - gamma_n).
+// Nothing here relies on a stored norm.
+__device__ __forceinline__ float fast_dot_warp(const float* __restrict__ q,
+                                               const float* __restrict__ v, int m_raw,
+                                               float* err) {
+    const int lane = threadIdx.x & 31;
+    const float4* q4 = reinterpret_cast<const float4*>(q);
+    const float4* v4 = reinterpret_cast<const float4*>(v);
+    const int n4 = m_raw >> 2;
+    constexpr int kBatch = 8;   // float4 of the row in flight per lane: one round trip
+    float f = 0.0f, g = 0.0f;
+#pragma unroll 1
+    for (int j0 = lane; j0 < n4; j0 += 32 * kBatch) {
+        float4 y[kBatch];
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int j = j0 + 32 * b;
+            y[b] = j < n4 ? __ldg(v4 + j) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        }
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+            const int j = j0 + 32 * b;
+            if (j < n4) {
+                const float4 a = q4[j];
+                f = fmaf(a.x, y[b].x, f);
+                g = fmaf(fabsf(a.x), fabsf(y[b].x), g);
+                f = fmaf(a.y, y[b].y, f);
+                g = fmaf(fabsf(a.y), fabsf(y[b].y), g);
+                f = fmaf(a.z, y[b].z, f);
+                g = fmaf(fabsf(a.z), fabsf(y[b].z), g);
+                f = fmaf(a.w, y[b].w, f);
+                g = fmaf(fabsf(a.w), fabsf(y[b].w), g);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        f += __shfl_xor_sync(0xffffffffu, f, o);
+        g += __shfl_xor_sync(0xffffffffu, g, o);
+    }
+    const int n = 4 * ((n4 + 31) / 32) + 5;
+    const float nu = (float)n * 0x1p-24f;
+    const float gamma = __fdiv_ru(nu, __fsub_rd(1.0f, nu));
+    const float tiny = (float)(32 * n + 32) * 0x1p-149f;
+    const float S = __fdiv_ru(__fadd_ru(g, tiny), __fsub_rd(1.0f, gamma));
+    *err = __fadd_ru(__fmul_ru(gamma, S), tiny);
+    return f;
+}
+
 // hist[j] = number of visible rows whose key lies above exactly j of the
 // queried keys (sorted ascending); the rank of the item with the j-th
 // smallest key is then 1 + sum of hist[t] for t > j.  A row's key lies in
@@ -177,9 +235,8 @@ constexpr int kCountWarps = 8;
 __global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
     const float* __restrict__ lo, const float* __restrict__ hi, int64_t rows,
     const uint32_t* __restrict__ tomb, const float* __restrict__ qraw,
-    const float* __restrict__ raw, int m_raw, const uint64_t* __restrict__ qkeys, int nq,
-    int exact, unsigned long long* hist, unsigned long long* maybe, int* status,
-    DevCounters* ctr) {
+    const float* __restrict__ raw, int m_raw, const uint64_t* __restrict__ qkeys, int nq, int exact,
+    unsigned long long* hist, unsigned long long* maybe, int* status, DevCounters* ctr) {
     __shared__ uint64_t sk[kRankQueryMax];
     __shared__ unsigned int sh[kRankQueryMax + 1];
     __shared__ int sm[kRankQueryMax + 1];
@@ -228,10 +285,30 @@ __global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
             const int src = __ffs(todo) - 1;
             todo &= todo - 1;
             const int64_t r = base + src;
-            bool fb = false;
-            const float s = exact_dot_warp_eft(qraw, qraw, raw + r * (int64_t)m_raw, m_raw, &fb);
             const float lr = __shfl_sync(0xffffffffu, l, src);
             const float hr = __shfl_sync(0xffffffffu, h, src);
+            // first a plain fp32 dot with its error bound: it places the
+            // authoritative score RN(q.v) in [fl, fh], which fixes the row's
+            // bin unless a queried key falls in that range
+            float err;
+            const float f = fast_dot_warp(qraw, raw + r * (int64_t)m_raw, m_raw, &err);
+            int fast_bin = -1;
+            if (lane == 0 && isfinite(f) && isfinite(err)) {
+                // a score of zero is reported as +0, whose key is above -0's
+                const float fl = __fsub_rd(f, err);
+                const float fh = __fadd_ru(f, err) == 0.0f ? 0.0f : __fadd_ru(f, err);
+                const int a = keys_below(sk, nq, rank_key(fl, (uint32_t)r));
+                const int b = keys_at_most(sk, nq, rank_key(fh, (uint32_t)r));
+                if (a == b) {
+                    fast_bin = a;
+                    if (fh < lr || fl > hr) set_status(status, PVS_ERR_INTERVAL);
+                    atomicAdd(&sh[a], 1u);
+                    ++scored;
+                }
+            }
+            if (__shfl_sync(0xffffffffu, fast_bin, 0) >= 0) continue;
+            bool fb = false;
+            const float s = exact_dot_warp_eft(qraw, qraw, raw + r * (int64_t)m_raw, m_raw, &fb);
             if (lane == 0) {
                 if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
                 else if (s < lr || s > hr) set_status(status, PVS_ERR_INTERVAL);
