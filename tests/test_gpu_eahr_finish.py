@@ -218,3 +218,31 @@ def test_rank_query_finish_on_grouped_cursors_and_a_bad_sparse_list(corpus):
     with pytest.raises(pvs.PvsError) as e:
         _run(index, Qg[0], bad, K=20, k=60, form=pvs.EAHR_NUMERATOR)
     assert e.value.status == pvs.PVS_ERR_INVALID
+
+
+def test_exact_count_near_equal_scores():
+    """Rows whose scores sit within a few ulps of a candidate's: exact copies
+    of the top rows (equal scores, ids decide) and copies perturbed by 1e-7.
+    The bounded fp32 dot cannot place them, so the error-free dot must; the
+    reversed sparse list makes every finish take exact ranks."""
+    rng = np.random.default_rng(340)
+    m, base_n = 64, 30_000
+    V = synth.unit_normal(base_n, m, seed=341).numpy()
+    q = synth.unit_normal(1, m, seed=342).numpy()[0]
+    ids0, _ = po.dense_ranking(q, V)
+    bottom = ids0[-40:]                      # the sparse list's top items
+    copies = np.repeat(V[bottom], 3, axis=0)
+    near = copies + (1e-7 * rng.standard_normal(copies.shape)).astype(np.float32)
+    W = np.concatenate([V, copies, near]).astype(np.float32)
+    W = W[rng.permutation(W.shape[0])]
+    dense_ids, _ = po.dense_ranking(q, W)
+    sparse = dense_ids[::-1].copy()
+    T = ro.target_topk_large([dense_ids, sparse], [1, 1], 60, 20, ro.NUMERATOR)
+    index = pvs.pvs_build(W)
+    try:
+        ids, F, st = _run(index, q, sparse, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+    finally:
+        pvs.pvs_index_free(index)
+    _check(ids, F, T)
+    assert st["complete"] == 3
+    assert not np.isnan(F).any()
