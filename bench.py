@@ -1123,7 +1123,7 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         dcur = pvs.pvs_cursor_open(index, dq[i])
         scur = pvs.pbm_cursor_open(sindex, *sq[i])
         ids, F, st = pvs.eahr_topk_pbm(dcur, scur, K=EAHR_K, k=EAHR_RRF_K,
-                                       form=pvs.EAHR_NUMERATOR)
+                                       form=pvs.EAHR_NUMERATOR, policy=eahr_policy(args, pvs))
         ps = pvs.pbm_cursor_stats(scur)
         pvs.pbm_cursor_close(scur)
         pvs.pvs_cursor_close(dcur)
@@ -1166,6 +1166,7 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         pg.barrier()
     launches0 = pvs.pvs_launch_count()
     lat, dd, ds, ex, rexp = [], [], [], 0, []
+    finish = {0: 0, 1: 0, 2: 0, 3: 0}
     with ClockSampler(local) as clk:
         for i in range(2, nq):
             ms, st, ps = one(i)
@@ -1174,6 +1175,7 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
             ds.append(st["depth"][1])
             ex += int(st["exhausted"][0] and st["exhausted"][1])
             rexp.append(ps["ranges_expanded"])
+            finish[int(st.get("complete", 0))] += 1
     launches = pvs.pvs_launch_count() - launches0
     cmp_ms = [comparator(i) for i in range(2, min(nq, 22))]
     line = {
@@ -1187,7 +1189,7 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                                f"terms, topic share {HYBRID_TOPIC_SHARE}), weighted RRF "
                                f"1/(60+rank), K={EAHR_K}",
                    "N": n, "d": DIM, "K": EAHR_K, "rrf_k": EAHR_RRF_K,
-                   "postings": int(docs.numel()),
+                   "policy": args.eahr_policy, "postings": int(docs.numel()),
                    "l2": "no flush: every query's interval pass streams 6.9 GB of codes",
                    "parallelism": f"replicas x{world}"},
         "e2e": {"value": float(np.median(lat)), "unit": "ms",
@@ -1198,6 +1200,8 @@ def main_hybrid(args, pvs, synth, torch, np, rank, world, local, dev, pg):
         "kendall_tau_dense_sparse": ktau,
         "dense_depth_p50": float(np.median(dd)), "sparse_depth_p50": float(np.median(ds)),
         "both_exhausted": ex, "pbm_ranges_expanded_p50": float(np.median(rexp)),
+        "finished_by": {"reading": finish[0], "rank_intervals": finish[2],
+                        "exact_ranks": finish[3]},
         "pbm_ranges": pvs.pbm_index_ranges(sindex),
         "exhaustive_torch_ms_p50": float(np.median(cmp_ms)),
         "gpu_launches": launches,

@@ -144,7 +144,11 @@ void pbm_cursor_close(pbm_cursor* cursor);
  * pbm_cursor_open_snapshot on that snapshot, or with pbm_cursor_open when
  * nothing is deleted); else PVS_ERR_INVALID.  The sparse support U_s is
  * usually much smaller than the visible set; items outside it contribute
- * nothing (Sec. 2.1).
+ * nothing (Sec. 2.1).  Under EAHR_POLICY_ADAPTIVE a helper thread computes
+ * the query's complete PBM ranking on the device (every item's S in the
+ * query's term order, the visible items with S > 0 sorted by (S desc, id
+ * asc)) while the lists are read, and the exact finish takes the
+ * candidates' missing sparse ranks from it.
  */
 pvs_status eahr_topk_pbm(pvs_cursor* dense, pbm_cursor* sparse, const eahr_params* p,
                          int64_t* out_ids, double* out_F, int32_t* n_out, eahr_stats* st);

@@ -402,7 +402,10 @@ enum {
                                     has grown by clamp(access / 8, 64, 1024)
                                     since the last check, and at once when a
                                     list is exhausted                          */
-    EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk only: GEOMETRIC reading, and
+    EAHR_POLICY_ADAPTIVE = 3     /* eahr_topk and eahr_topk_pbm (where the
+                                    sparse ranks of the finish come from the
+                                    query's complete PBM ranking, computed
+                                    on the device): GEOMETRIC reading, and
                                     once the ranks read reach 2^12 (again
                                     each time they double) an exact finish:
                                     with LB the K-th largest L(x) of the
@@ -422,7 +425,8 @@ enum {
                                     (too many candidates,
                                     a cursor without bounds of every row),
                                     once the ranks read reach (n_dense +
-                                    n_sparse) / 16 clamped to [2^16, 2^18]:
+                                    n_sparse) / 16 clamped to [2^16, 2^18]
+                                    (eahr_topk only):
                                     complete-list fusion on the device (every
                                     visible row's authoritative score, both
                                     lists' ranks, the fused order).  Both

@@ -380,15 +380,20 @@ class Driver {
     pvs_status stage_status = PVS_OK;
     pvs::StagedList* staged = nullptr;
 
+    // (a PBM source: its complete ranking, computed on the device)
     void start_stage() {
-        if (stage_live || !src[0].cursor || !src[1].list || src[1].length == 0) return;
+        if (stage_live || !src[0].cursor) return;
+        const bool host_list = src[1].list && src[1].length > 0;
+        if (!host_list && !src[1].sparse) return;
         try {
-            stage = std::thread([this] {
-                stage_status = pvs::stage_sparse_list(src[0].cursor, src[1].list,
-                                                      src[1].length, &staged);
+            stage = std::thread([this, host_list] {
+                stage_status =
+                    host_list ? pvs::stage_sparse_list(src[0].cursor, src[1].list, src[1].length,
+                                                       &staged)
+                              : pvs::pbm_stage_ranks(src[1].sparse, src[0].cursor->index, &staged);
             });
             stage_live = true;
-        } catch (...) {   // no thread: the finish copies the list itself
+        } catch (...) {   // no thread: a host list is copied by the finish itself
         }
     }
     // The staged list once it is queued (null when staging failed).
@@ -907,11 +912,16 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
         return PVS_OK;
     // first the dense rank intervals the rows' bounds give (no row scored)
     std::vector<int64_t> rd_lo(need_d.size()), rd_hi(need_d.size()), rs(need_s.size());
+    const pvs::StagedList* staged = need_s.empty() ? nullptr : d.staged_list();
+    if (!need_s.empty() && !staged && !d.src[1].list) {   // a PBM source that could not be staged
+        *retry = false;
+        return PVS_OK;
+    }
     bool supported = false;
     pvs_status s = pvs::rank_queries(c, need_d.data(), (int32_t)need_d.size(), false,
-                                     d.src[1].list, d.src[1].length, need_s.data(),
-                                     (int32_t)need_s.size(), rd_lo.data(), rd_hi.data(), rs.data(),
-                                     &supported, need_s.empty() ? nullptr : d.staged_list());
+                                     d.src[1].list, d.src[1].list ? d.src[1].length : 0,
+                                     need_s.data(), (int32_t)need_s.size(), rd_lo.data(),
+                                     rd_hi.data(), rs.data(), &supported, staged);
     if (s != PVS_OK) return s;
     if (!supported) {   // this cursor never supports it
         *retry = false;
@@ -990,7 +1000,8 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
 
 pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double* out_F,
                       int32_t* n_out, eahr_stats* st) {
-    const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor && d.src[1].list;
+    const bool adaptive = p->policy == EAHR_POLICY_ADAPTIVE && d.src[0].cursor &&
+                          (d.src[1].list || d.src[1].sparse);
     if (adaptive) d.start_stage();
     // the adaptive policy reads its first kQueryAt ranks in one pull per list
     // (its finish is tried there; fewer, larger pulls cost fewer round trips)
@@ -1073,7 +1084,7 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
             // else again after as much reading, or never
             query_at = retry ? 2 * (d.depth[0] + d.depth[1]) : std::numeric_limits<int64_t>::max();
         }
-        if (!done && adaptive && d.depth[0] + d.depth[1] >= complete_at)
+        if (!done && adaptive && d.src[1].list && d.depth[0] + d.depth[1] >= complete_at)
             return finish_complete(d, p, out_ids, out_F, n_out, st);
         if (!done) {
             bool any_open = false;

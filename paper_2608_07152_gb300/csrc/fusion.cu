@@ -473,16 +473,6 @@ pvs_status fuse_complete(pvs_cursor* c, const int64_t* sparse, int64_t ns, const
     return result;
 }
 
-struct StagedList {
-    pvs_index* index = nullptr;
-    cudaStream_t stream = nullptr;
-    cudaEvent_t ready = nullptr;
-    int32_t* rank_of = nullptr;
-    int64_t* list = nullptr;
-    int* status = nullptr;
-    int64_t rows = 0;
-};
-
 void free_staged_list(StagedList* s) {
     if (!s) return;
     int prev = -1;
@@ -707,7 +697,7 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
                 : staged->list;
         int32_t* d_sids = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
         d_srank = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
-        if (!rank_of || !d_list || !d_sids || !d_srank) {
+        if (!rank_of || (own && !d_list) || !d_sids || !d_srank) {
             cleanup();
             return PVS_ERR_OOM;
         }

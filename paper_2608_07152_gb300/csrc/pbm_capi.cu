@@ -422,6 +422,78 @@ pvs_status open_cursor(pbm_index* x, const std::shared_ptr<pvs::SnapData>& snap,
 
 namespace pvs {
 const SnapData* pbm_cursor_snapshot(const pbm_cursor* c) { return c->snap.get(); }
+
+// The complete sparse ranking of the cursor's query as a staged list: every
+// item's S in the query's term order (the expand kernel's evaluation), the
+// visible items with S > 0 sorted by key, their positions scattered into
+// rank_of.  Runs on a stream of its own and waits for it once (for the
+// member count), so the caller may be a helper thread.
+pvs_status pbm_stage_ranks(pbm_cursor* c, pvs_index* owner, StagedList** out) {
+    *out = nullptr;
+    if (!c || !c->index || !owner || c->state < 0) return PVS_ERR_INVALID;
+    pbm_index* x = c->index;
+    if (cudaSetDevice(x->device) != cudaSuccess) {
+        cudaGetLastError();
+        return PVS_ERR_CUDA;
+    }
+    StagedList* s = new (std::nothrow) StagedList();
+    if (!s) return PVS_ERR_OOM;
+    s->index = owner;
+    s->rows = x->n_items;
+    const size_t n = (size_t)std::max<int64_t>(x->n_items, 1);
+    const uint32_t* tomb = c->snap ? c->snap->d_tomb : nullptr;
+    float* acc = nullptr;
+    uint64_t* keys = nullptr;
+    uint64_t* tmp = nullptr;
+    void* scratch = nullptr;
+    unsigned long long* count = nullptr;
+    unsigned long long* h_count = nullptr;
+    cudaError_t e = cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking);
+    auto pool_alloc = [&](void** p, size_t bytes) {
+        if (e == cudaSuccess)
+            e = cudaMallocFromPoolAsync(p, std::max<size_t>(bytes, 16), owner->scratch_pool,
+                                        s->stream);
+    };
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&s->ready, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaMallocHost(&h_count, sizeof(unsigned long long));
+    pool_alloc(reinterpret_cast<void**>(&s->rank_of), n * 4);
+    pool_alloc(reinterpret_cast<void**>(&s->status), sizeof(int));
+    pool_alloc(reinterpret_cast<void**>(&acc), n * 4);
+    pool_alloc(reinterpret_cast<void**>(&keys), n * 8);
+    pool_alloc(reinterpret_cast<void**>(&count), sizeof(unsigned long long));
+    const int grid = std::max(1, x->num_sms) * 8;
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->rank_of, 0, n * 4, s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->status, 0, sizeof(int), s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(acc, 0, n * 4, s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(count, 0, sizeof(unsigned long long), s->stream);
+    if (e == cudaSuccess)
+        e = launch_pbm_score_all(PbmQuery{c->terms, c->weights, c->nq}, x->term_off, x->docs,
+                                 x->imps, acc, grid, s->stream);
+    if (e == cudaSuccess)
+        e = launch_pbm_member_keys(acc, x->n_items, tomb, keys, count, grid, s->stream);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h_count, count, sizeof(unsigned long long), cudaMemcpyDeviceToHost,
+                            s->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s->stream);
+    const int64_t m = e == cudaSuccess ? (int64_t)*h_count : 0;
+    if (m > 1) {
+        pool_alloc(reinterpret_cast<void**>(&tmp), (size_t)m * 8);
+        pool_alloc(&scratch, radix_sort_scratch_bytes(m));
+        if (e == cudaSuccess) e = launch_radix_sort_desc(keys, tmp, m, scratch, s->stream);
+    }
+    if (e == cudaSuccess) e = launch_pbm_rank_of(keys, m, s->rank_of, grid, s->stream);
+    if (e == cudaSuccess) e = cudaEventRecord(s->ready, s->stream);
+    for (void* p : {(void*)acc, (void*)keys, (void*)tmp, scratch, (void*)count})
+        if (p) cudaFreeAsync(p, s->stream);
+    if (h_count) cudaFreeHost(h_count);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        free_staged_list(s);
+        return e == cudaErrorMemoryAllocation ? PVS_ERR_OOM : PVS_ERR_CUDA;
+    }
+    *out = s;
+    return PVS_OK;
+}
 }  // namespace pvs
 
 extern "C" {

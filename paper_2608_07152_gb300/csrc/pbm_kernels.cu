@@ -636,4 +636,67 @@ cudaError_t launch_pbm_emit(const uint64_t* keys, int m, int64_t* ids, float* sc
     return cudaGetLastError();
 }
 
+// One term's postings; a term lists an item at most once, so no two threads
+// of a launch touch one accumulator, and launches in term order keep each
+// item's additions in the query's order (App. A.2).
+__global__ void pbm_score_term_kernel(const int64_t* __restrict__ term_off,
+                                      const int32_t* __restrict__ docs,
+                                      const float* __restrict__ imps, const int32_t* terms,
+                                      const float* weights, int j, float* acc) {
+    const int32_t t = terms[j];
+    const float w = weights[j];
+    const int64_t b = term_off[t], e = term_off[t + 1];
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = b + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < e; i += stride) {
+        const int32_t x = docs[i];
+        acc[x] = __fadd_rn(acc[x], __fmul_rn(w, imps[i]));
+    }
+}
+
+cudaError_t launch_pbm_score_all(const PbmQuery& q, const int64_t* term_off, const int32_t* docs,
+                                 const float* imps, float* acc, int grid, cudaStream_t st) {
+    for (int j = 0; j < q.nq; ++j) {
+        count_launches(1);
+        pbm_score_term_kernel<<<grid, 256, 0, st>>>(term_off, docs, imps, q.terms, q.weights, j,
+                                                    acc);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+__global__ void pbm_member_keys_kernel(const float* __restrict__ acc, int64_t n,
+                                       const uint32_t* __restrict__ tomb, uint64_t* keys,
+                                       unsigned long long* count) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < n; x += stride) {
+        const float s = acc[x];
+        if (s > 0.0f && !tombstoned(tomb, x))
+            keys[atomicAdd(count, 1ull)] = rank_key(s, (uint32_t)x);
+    }
+}
+
+cudaError_t launch_pbm_member_keys(const float* acc, int64_t n, const uint32_t* tomb,
+                                   uint64_t* keys, unsigned long long* count, int grid,
+                                   cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    count_launches(1);
+    pbm_member_keys_kernel<<<grid, 256, 0, st>>>(acc, n, tomb, keys, count);
+    return cudaGetLastError();
+}
+
+__global__ void pbm_rank_of_kernel(const uint64_t* __restrict__ keys, int64_t m, int32_t* rank_of) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < m; i += stride)
+        rank_of[rank_key_id(keys[i])] = (int32_t)(i + 1);
+}
+
+cudaError_t launch_pbm_rank_of(const uint64_t* keys, int64_t m, int32_t* rank_of, int grid,
+                               cudaStream_t st) {
+    if (m <= 0) return cudaSuccess;
+    count_launches(1);
+    pbm_rank_of_kernel<<<grid, 256, 0, st>>>(keys, m, rank_of);
+    return cudaGetLastError();
+}
+
 }  // namespace pvs

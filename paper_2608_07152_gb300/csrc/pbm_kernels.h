@@ -113,5 +113,18 @@ cudaError_t launch_pbm_select64(const uint64_t* pool, const PbmCounters* ctr, ui
 // ids[i], scores[i] of the first m keys of a descending key array.
 cudaError_t launch_pbm_emit(const uint64_t* keys, int m, int64_t* ids, float* scores,
                             cudaStream_t st);
+// Complete sparse scores: for each query term j in order,
+// acc[x] = RN(acc[x] + RN(q_j p_j(x))) over the term's postings (acc zeroed
+// by the caller), the evaluation of the expand kernel for every item.
+cudaError_t launch_pbm_score_all(const PbmQuery& q, const int64_t* term_off, const int32_t* docs,
+                                 const float* imps, float* acc, int grid, cudaStream_t st);
+// keys[0 .. *count) = rank keys of the visible items with acc > 0, in any
+// order (*count zeroed by the caller).
+cudaError_t launch_pbm_member_keys(const float* acc, int64_t n, const uint32_t* tomb,
+                                   uint64_t* keys, unsigned long long* count, int grid,
+                                   cudaStream_t st);
+// rank_of[id of keys[i]] = i + 1 for i < m (keys sorted descending).
+cudaError_t launch_pbm_rank_of(const uint64_t* keys, int64_t m, int32_t* rank_of, int grid,
+                               cudaStream_t st);
 
 }  // namespace pvs

@@ -73,6 +73,8 @@ struct pvs_snapshot {
     std::shared_ptr<pvs::SnapData> data;
 };
 
+struct pbm_cursor;
+
 struct pvs_cursor {
     pvs_index* index = nullptr;
     cudaStream_t stream = nullptr;    // where this cursor's device work runs
@@ -199,9 +201,21 @@ constexpr int32_t kRankQueryMax = 1024;
 // fuse_complete (the verdict is read when the ranks are used).  Built on its
 // own stream by stage_sparse_list (which may hold the calling thread while
 // the pageable list is copied); rank_queries orders its reads after it.
-struct StagedList;
+struct StagedList {
+    pvs_index* index = nullptr;       // device and scratch pool
+    cudaStream_t stream = nullptr;
+    cudaEvent_t ready = nullptr;      // recorded after the scatter
+    int32_t* rank_of = nullptr;       // [rows]
+    int64_t* list = nullptr;          // the list's ids on the device (or null)
+    int* status = nullptr;            // the scatter's verdict on the ids
+    int64_t rows = 0;
+};
 pvs_status stage_sparse_list(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
                              StagedList** out);
+// The complete ranking of a PBM cursor's query (U_s = the visible items with
+// S > 0, by (S desc, id asc), S evaluated as the PBM kernels do, App. A.2)
+// staged the same way (pbm_capi.cu); scratch from pool_owner's pool.
+pvs_status pbm_stage_ranks(pbm_cursor* sparse, pvs_index* pool_owner, StagedList** out);
 void free_staged_list(StagedList* s);
 // `staged` (or null): the same list, already scattered.
 pvs_status rank_queries(pvs_cursor* dense, const int32_t* dense_ids, int32_t nd, bool exact,

@@ -245,7 +245,8 @@ def test_eahr_with_pbm_matches_complete_list_fusion(tau_terms):
             assert got == ro.as_float(f)
 
 
-def _eahr_pbm(V, q, off, docs, imps, n, terms, weights, snap_ids=None):
+def _eahr_pbm(V, q, off, docs, imps, n, terms, weights, snap_ids=None,
+              policy=pvs.EAHR_POLICY_GEOMETRIC, step=0):
     """eahr_topk_pbm over a fresh PVS index of V and PBM index of the postings;
     snap_ids: ids to delete in a snapshot that both cursors see."""
     dindex = pvs.pvs_build(V)
@@ -258,7 +259,8 @@ def _eahr_pbm(V, q, off, docs, imps, n, terms, weights, snap_ids=None):
         dcur = pvs.pvs_cursor_open(dindex, q, snap=snap)
         scur = pvs.pbm_cursor_open(sindex, terms, weights, snap=snap)
         try:
-            return pvs.eahr_topk_pbm(dcur, scur, K=20, k=60, form=pvs.EAHR_NUMERATOR)
+            return pvs.eahr_topk_pbm(dcur, scur, K=20, k=60, form=pvs.EAHR_NUMERATOR,
+                                     policy=policy, step=step)
         finally:
             pvs.pbm_cursor_close(scur)
             pvs.pvs_cursor_close(dcur)
@@ -355,3 +357,39 @@ def test_pbm_on_a_snapshot_with_deletions():
     assert got.tolist() == [x for x, _ in T]
     assert not visible[got].size or visible[got].all()
     assert S[dead].max() > 0      # deleted items that PBM would otherwise rank
+
+
+@pytest.mark.parametrize("deleted", [False, True])
+def test_eahr_pbm_adaptive_finish_matches_complete_list_fusion(deleted):
+    """EAHR_POLICY_ADAPTIVE over PVS + PBM (Sec. 2.2, last paragraph): after
+    2^12 ranks the candidates' missing sparse ranks come from the query's
+    complete PBM ranking computed on the device (S in the query's term order,
+    as the expand kernel evaluates it), the dense ones from the rows' bounds.
+    Independent channels make both lists deep; with deletions both cursors
+    rank one snapshot."""
+    n, m = 60_000, 64
+    rng = np.random.default_rng(71)
+    V = synth.unit_normal(n, m, seed=72).numpy()
+    Q = synth.unit_normal(3, m, seed=73).numpy()
+    off, docs, imps = synth.bm25_postings(n, 6_000, 25.0, seed=74)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    queries = synth.sparse_queries(3, torch.from_numpy(off), seed=75, mean_terms=8.0)
+    dead = rng.choice(n, n // 25, replace=False) if deleted else None
+    visible = np.ones(n, bool)
+    if deleted:
+        visible[dead] = False
+    finishes = []
+    for qi, (terms, weights) in enumerate(queries):
+        dense_ids, _ = pvo.dense_ranking(Q[qi], V, visible=visible)
+        sparse_ids, _ = po.sparse_ranking(terms, weights, off, docs, imps, n)
+        sparse_ids = sparse_ids[visible[sparse_ids]]
+        T = ro.target_topk_large([dense_ids, sparse_ids], [1, 1], 60, 20, ro.NUMERATOR)
+        for step in (16, 0):
+            ids, F, st = _eahr_pbm(V, Q[qi], off, docs, imps, n, terms, weights, snap_ids=dead,
+                                   policy=pvs.EAHR_POLICY_ADAPTIVE, step=step)
+            assert ids.tolist() == [x for x, _ in T]
+            for (x, f), got in zip(T, F):
+                if not np.isnan(got):
+                    assert got == ro.as_float(f)
+            finishes.append(st["complete"])
+    assert any(c in (2, 3) for c in finishes)
