@@ -78,13 +78,20 @@ struct PullArgs {
     int* status_mirror;       // pinned host word: the status after the pull (null: none)
 };
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st);
-// Many cursors at once (args_dev: device array of ncursors PullArgs).
+// Many cursors at once: the per-cursor arguments travel as kernel
+// parameters, up to kPullPack cursors per launch (the parameter space holds
+// 32,764 bytes), so no copy of them is staged; every CTA reads only its own
+// cursor's entry, one address for all its threads.  The host array is read
+// at launch.
+constexpr int kPullPack = 224;
+struct PullArgsPack {
+    PullArgs a[kPullPack];
+};
+static_assert(sizeof(PullArgsPack) <= 31 * 1024, "kernel parameter space");
 // One launch per pull (n <= kPullFusedMax): a cluster of CTAs selects,
 // refines and emits (one cluster per cursor in the batch form).
 cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st);
-cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st);
-// dev[0 .. n) = host[0 .. n), in stream order, the host array read at launch.
-cudaError_t launch_stage_pull_args(const PullArgs* host, int n, PullArgs* dev, cudaStream_t st);
+cudaError_t launch_pull_cluster_batch(const PullArgs* host_args, int ncursors, cudaStream_t st);
 // Ranks computed ahead, handed to the callers' buffers: for every entry,
 // count ids and scores from src to dst (device or pinned host memory), in
 // stream order, one launch per 64 entries (the entries are read at launch).
@@ -96,9 +103,10 @@ struct RankCopy {
     int count;
 };
 cudaError_t launch_copy_ranks(const RankCopy* host, int n, cudaStream_t st);
-cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
+cudaError_t launch_pull_batch(const PullArgs* host_args, int ncursors, int refine_blocks_per_cursor,
                               int m_raw, cudaStream_t st);
-cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
+// ncursors <= kPullPack entries of p.
+cudaError_t launch_refine_batch(const PullArgsPack& p, int ncursors, int blocks_per_cursor,
                                 int m_raw, cudaStream_t st);
 
 // ---- batched open support (pull_kernel.cu, batch_support.cu) ----------------

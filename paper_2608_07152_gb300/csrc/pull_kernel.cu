@@ -21,6 +21,8 @@
 // Every CTA has 512 threads (<= 64 registers) and ~25 KB of shared memory, so
 // it fits on an SM beside another cursor's interval-pass CTA.
 #include "exact_dot.cuh"
+#include <vector>
+
 #include "kernels.h"
 #include "pipeline.cuh"
 #include "pvs_common.cuh"
@@ -196,9 +198,10 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_select_kernel(PullArgs a
 }
 
 // One CTA per cursor.
-__global__ void __launch_bounds__(kPullThreads, 2) pull_select_batch_kernel(const PullArgs* args) {
+__global__ void __launch_bounds__(kPullThreads, 2)
+    pull_select_batch_kernel(const __grid_constant__ PullArgsPack p) {
     __shared__ PullShared sh;
-    pull_select_body(args[blockIdx.x], sh);
+    pull_select_body(p.a[blockIdx.x], sh);
 }
 
 // Sort the m keys in sh.sk (descending) and emit the first n: ids, scores,
@@ -339,9 +342,10 @@ __global__ void __launch_bounds__(kPullThreads, 2) pull_emit_kernel(PullArgs a) 
     pull_emit_body(a, sh);
 }
 
-__global__ void __launch_bounds__(kPullThreads, 2) pull_emit_batch_kernel(const PullArgs* args) {
+__global__ void __launch_bounds__(kPullThreads, 2)
+    pull_emit_batch_kernel(const __grid_constant__ PullArgsPack p) {
     __shared__ PullShared sh;
-    pull_emit_body(args[blockIdx.x], sh);
+    pull_emit_body(p.a[blockIdx.x], sh);
 }
 
 // ---- one launch per pull: a cluster of CTAs per cursor -------------------------
@@ -746,9 +750,9 @@ __global__ void __cluster_dims__(kPullCluster, 1, 1) __launch_bounds__(kPullThre
 
 // One cluster per cursor.
 __global__ void __cluster_dims__(kPullClusterBatch, 1, 1) __launch_bounds__(kPullThreads, 2)
-    pull_cluster_batch_kernel(const PullArgs* args) {
+    pull_cluster_batch_kernel(const __grid_constant__ PullArgsPack p) {
     __shared__ PullShared sh;
-    pull_cluster_body<kPullClusterBatch>(args[blockIdx.x / kPullClusterBatch], sh);
+    pull_cluster_body<kPullClusterBatch>(p.a[blockIdx.x / kPullClusterBatch], sh);
 }
 
 cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
@@ -757,34 +761,6 @@ cudaError_t launch_pull_cluster(const PullArgs& a, cudaStream_t st) {
     count_launches(1);
     pull_cluster_kernel<<<kPullCluster, kPullThreads, 0, st>>>(a);
     return cudaGetLastError();
-}
-
-// Per-cursor arguments of a batched pull written to device memory in stream
-// order by a kernel that receives them as parameters: the host's copy of
-// the arguments is captured at launch, so neither a pageable copy (which
-// can wait for the stream) nor a reused pinned buffer (which the next pull
-// could overwrite before the copy runs) is involved.
-constexpr int kArgsPerStage = 64;
-struct PullArgsPack {
-    PullArgs a[kArgsPerStage];
-};
-
-__global__ void stage_pull_args_kernel(const __grid_constant__ PullArgsPack p, int count,
-                                       PullArgs* out) {
-    for (int i = threadIdx.x; i < count; i += blockDim.x) out[i] = p.a[i];
-}
-
-cudaError_t launch_stage_pull_args(const PullArgs* host, int n, PullArgs* dev, cudaStream_t st) {
-    for (int first = 0; first < n; first += kArgsPerStage) {
-        const int count = n - first < kArgsPerStage ? n - first : kArgsPerStage;
-        PullArgsPack p;
-        for (int i = 0; i < count; ++i) p.a[i] = host[first + i];
-        count_launches(1);
-        stage_pull_args_kernel<<<1, 64, 0, st>>>(p, count, dev + first);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
-    return cudaSuccess;
 }
 
 constexpr int kCopiesPerLaunch = 64;
@@ -813,11 +789,28 @@ cudaError_t launch_copy_ranks(const RankCopy* host, int n, cudaStream_t st) {
     return cudaSuccess;
 }
 
-cudaError_t launch_pull_cluster_batch(const PullArgs* args_dev, int ncursors, cudaStream_t st) {
+// Packs of up to kPullPack cursors' arguments (the last one partial).
+static std::vector<PullArgsPack> pull_packs(const PullArgs* host, int n) {
+    std::vector<PullArgsPack> packs((size_t)((n + kPullPack - 1) / kPullPack));
+    for (int i = 0; i < n; ++i) packs[(size_t)(i / kPullPack)].a[i % kPullPack] = host[i];
+    return packs;
+}
+static int pack_count(int n, size_t k) {
+    const int rest = n - (int)k * kPullPack;
+    return rest < kPullPack ? rest : kPullPack;
+}
+
+cudaError_t launch_pull_cluster_batch(const PullArgs* host_args, int ncursors, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
-    count_launches(1);
-    pull_cluster_batch_kernel<<<ncursors * kPullClusterBatch, kPullThreads, 0, st>>>(args_dev);
-    return cudaGetLastError();
+    const std::vector<PullArgsPack> packs = pull_packs(host_args, ncursors);
+    for (size_t k = 0; k < packs.size(); ++k) {
+        count_launches(1);
+        pull_cluster_batch_kernel<<<pack_count(ncursors, k) * kPullClusterBatch, kPullThreads, 0,
+                                    st>>>(packs[k]);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_pull_fused(const PullArgs& a, int refine_grid, cudaStream_t st) {
@@ -995,18 +988,29 @@ cudaError_t launch_ws_sort(const int32_t* w_id_b, const float* w_lo_b, const flo
     return cudaGetLastError();
 }
 
-cudaError_t launch_pull_batch(const PullArgs* args_dev, int ncursors, int refine_blocks_per_cursor,
+// Selection for every pack, then refinement for every pack, then emission.
+cudaError_t launch_pull_batch(const PullArgs* host_args, int ncursors, int refine_blocks_per_cursor,
                               int m_raw, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
-    count_launches(1);
-    pull_select_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    e = launch_refine_batch(args_dev, ncursors, refine_blocks_per_cursor, m_raw, st);
-    if (e != cudaSuccess) return e;
-    count_launches(1);
-    pull_emit_batch_kernel<<<ncursors, kPullThreads, 0, st>>>(args_dev);
-    return cudaGetLastError();
+    const std::vector<PullArgsPack> packs = pull_packs(host_args, ncursors);
+    for (size_t k = 0; k < packs.size(); ++k) {
+        count_launches(1);
+        pull_select_batch_kernel<<<pack_count(ncursors, k), kPullThreads, 0, st>>>(packs[k]);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    for (size_t k = 0; k < packs.size(); ++k) {
+        cudaError_t e = launch_refine_batch(packs[k], pack_count(ncursors, k),
+                                            refine_blocks_per_cursor, m_raw, st);
+        if (e != cudaSuccess) return e;
+    }
+    for (size_t k = 0; k < packs.size(); ++k) {
+        count_launches(1);
+        pull_emit_batch_kernel<<<pack_count(ncursors, k), kPullThreads, 0, st>>>(packs[k]);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace pvs

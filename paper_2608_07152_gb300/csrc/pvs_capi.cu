@@ -1755,9 +1755,6 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
         pvs_status s = build_first_working_sets(cursors, nc, pulls.data());
         if (s != PVS_OK) return s;
     }
-    DevBuf buf(st, x->scratch_pool);   // released in stream order after the launches that read it
-    PullArgs* d_args = buf.get<PullArgs>((size_t)nc);
-    if (!d_args) return PVS_ERR_OOM;
     std::vector<PullArgs> args;
     std::vector<int32_t> who;
     args.reserve(nc);
@@ -1793,14 +1790,13 @@ pvs_status pvs::next_batch_rows(pvs_cursor* const* cursors, int32_t nc, int32_t 
         who.push_back(i);
     }
     if (!args.empty()) {
-        PVS_CUDA(launch_stage_pull_args(args.data(), (int)args.size(), d_args, st));
         bool fresh = false;
         for (int32_t i : who) fresh = fresh || cursors[i]->fresh_ws;
         if (fresh) {   // first pull of new working sets: refinement on every SM
             const int per = std::min(64, std::max(4, 2 * x->num_sms / (int)args.size()));
-            PVS_CUDA(launch_pull_batch(d_args, (int)args.size(), per, x->m_raw, st));
+            PVS_CUDA(launch_pull_batch(args.data(), (int)args.size(), per, x->m_raw, st));
         } else {
-            PVS_CUDA(launch_pull_cluster_batch(d_args, (int)args.size(), st));
+            PVS_CUDA(launch_pull_cluster_batch(args.data(), (int)args.size(), st));
         }
     }
     for (int32_t i : who) {

@@ -88,9 +88,10 @@ __global__ void __launch_bounds__(256, 3) refine_kernel(
 
 // Many cursors at once: blocks_per_cursor consecutive blocks serve cursor
 // blockIdx.x / blocks_per_cursor.
-__global__ void __launch_bounds__(256, 3) refine_batch_kernel(const PullArgs* args,
-                                                              int blocks_per_cursor, int stage_q) {
-    const PullArgs& a = args[blockIdx.x / blocks_per_cursor];
+__global__ void __launch_bounds__(256, 3)
+    refine_batch_kernel(const __grid_constant__ PullArgsPack args, int blocks_per_cursor,
+                        int stage_q) {
+    const PullArgs& a = args.a[blockIdx.x / blocks_per_cursor];
     const float* qf = stage_query(a.qraw, a.m_raw, stage_q);
     const int64_t warps_per_block = blockDim.x >> 5;
     refine_warps(a.cand, &a.ctr->cand, a.w_id, a.w_lo, a.w_hi, a.lo, a.hi, qf, a.qraw, a.raw,
@@ -238,8 +239,8 @@ __global__ void __launch_bounds__(kRingWarps * 32, 2) refine_ring_kernel(RingRef
 }
 
 __global__ void __launch_bounds__(kRingWarps * 32, 2) refine_ring_batch_kernel(
-    const PullArgs* args, int blocks_per_cursor, int stages) {
-    const PullArgs& p = args[blockIdx.x / blocks_per_cursor];
+    const __grid_constant__ PullArgsPack args, int blocks_per_cursor, int stages) {
+    const PullArgs& p = args.a[blockIdx.x / blocks_per_cursor];
     const RingRefs a{p.cand, &p.ctr->cand, p.w_id, p.w_lo, p.w_hi, p.lo, p.hi,
                      p.qraw, p.raw, p.m_raw, p.status, p.ctr};
     refine_ring(a, stages, (int64_t)(blockIdx.x % blocks_per_cursor) * kRingWarps +
@@ -265,7 +266,7 @@ static int query_stage_bytes(int m_raw) {
     return b <= 48 * 1024 ? (int)b : 0;
 }
 
-cudaError_t launch_refine_batch(const PullArgs* args_dev, int ncursors, int blocks_per_cursor,
+cudaError_t launch_refine_batch(const PullArgsPack& args_dev, int ncursors, int blocks_per_cursor,
                                 int m_raw, cudaStream_t st) {
     if (ncursors <= 0) return cudaSuccess;
     const int stages = ring_stages(m_raw);
