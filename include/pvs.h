@@ -418,8 +418,10 @@ enum {
                                     the item's authoritative score.  When
                                     those intervals do not certify the order
                                     (Sec. 2.2 over the candidates), the rows
-                                    around each score are scored and the
-                                    ranks are exact.  An F known only as an
+                                    around the scores of the candidates
+                                    whose intervals overlap are scored and
+                                    their ranks made exact (a few rounds,
+                                    then every candidate's).  An F known only as an
                                     interval is reported as NaN (its
                                     position is certified).  Failing that
                                     (too many candidates,

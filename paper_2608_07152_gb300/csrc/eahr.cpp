@@ -965,14 +965,46 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
     fill();
     std::vector<int32_t> order;
     bool scored = false;
-    if (!order_by_bounds(lo, hi, K, &order)) {
+    // While the intervals leave the order open, exact dense ranks for the
+    // candidates whose F interval is wider than a point and overlaps another
+    // one that can still reach the Top-K (only they can hold the order up);
+    // the rows around each such candidate's score are scored.  A last round
+    // makes every dense rank exact, which decides the order.
+    for (int round = 0; !order_by_bounds(lo, hi, K, &order); ++round) {
         scored = true;
-        // the intervals leave the order open: exact dense ranks
-        s = pvs::rank_queries(c, need_d.data(), (int32_t)need_d.size(), true, nullptr, 0, nullptr,
-                              0, rd_lo.data(), rd_hi.data(), nullptr, &supported);
+        std::vector<size_t> pick;   // indices into need_d
+        if (round < 3) {
+            std::vector<Node> lows(lo);
+            std::nth_element(lows.begin(), lows.begin() + (std::ptrdiff_t)(K - 1), lows.end(),
+                             NodeCmp());
+            const Frac floor_k = lows[(size_t)K - 1].F;   // the K-th largest lower bound
+            std::vector<size_t> rel;
+            for (size_t t = 0; t < cand.size(); ++t)
+                if (cmp(hi[t].F, floor_k) >= 0) rel.push_back(t);
+            for (size_t t : rel) {
+                if (at_d[t] == SIZE_MAX || cmp(lo[t].F, hi[t].F) == 0) continue;
+                for (size_t u : rel)
+                    if (u != t && cmp(lo[t].F, hi[u].F) <= 0 && cmp(lo[u].F, hi[t].F) <= 0) {
+                        pick.push_back(at_d[t]);
+                        break;
+                    }
+            }
+        }
+        if (pick.empty())   // the last round: every dense rank
+            for (size_t j = 0; j < need_d.size(); ++j)
+                if (rd_lo[j] != rd_hi[j]) pick.push_back(j);
+        if (pick.empty()) break;   // cannot happen: point intervals decide
+        std::vector<int32_t> ids(pick.size());
+        std::vector<int64_t> plo(pick.size()), phi(pick.size());
+        for (size_t j = 0; j < pick.size(); ++j) ids[j] = need_d[pick[j]];
+        s = pvs::rank_queries(c, ids.data(), (int32_t)ids.size(), true, nullptr, 0, nullptr, 0,
+                              plo.data(), phi.data(), nullptr, &supported);
         if (s != PVS_OK) return s;
+        for (size_t j = 0; j < pick.size(); ++j) {
+            rd_lo[pick[j]] = plo[j];
+            rd_hi[pick[j]] = phi[j];
+        }
         fill();
-        order_by_bounds(lo, hi, K, &order);   // decided now: lo == hi
     }
     // F is reported where it is known exactly (a point interval), NaN where
     // only the position is certified (as for an item unread in an Open list)
