@@ -285,6 +285,12 @@ __global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
             const int src = __ffs(todo) - 1;
             todo &= todo - 1;
             const int64_t r = base + src;
+            if (todo) {   // the next row to score, into L2 while this one is scored
+                const char* nrow =
+                    reinterpret_cast<const char*>(raw + (base + __ffs(todo) - 1) * (int64_t)m_raw);
+                for (int off = lane * 128; off < m_raw * 4; off += 32 * 128)
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(nrow + off));
+            }
             const float lr = __shfl_sync(0xffffffffu, l, src);
             const float hr = __shfl_sync(0xffffffffu, h, src);
             // first a plain fp32 dot with its error bound: it places the
