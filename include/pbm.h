@@ -110,6 +110,18 @@ pvs_status pbm_cursor_open_snapshot(pbm_index* index, const pvs_snapshot* snap,
                                     pbm_cursor** out);
 
 /*
+ * pbm_cursor_open_snapshot with the cursor's device work (the bounds at open
+ * and every pull) on cuda_stream (a cudaStream_t of the index's device, not
+ * owned; NULL: the index's stream).  Cursors on streams of their own serve
+ * requests from several host threads concurrently.  Closed cursors keep
+ * their buffers for later opens of the same index (up to 32 of them).
+ * Errors as pbm_cursor_open_snapshot.
+ */
+pvs_status pbm_cursor_open_stream(pbm_index* index, const pvs_snapshot* snap,
+                                  const int32_t* terms, const float* weights, int32_t nq,
+                                  void* cuda_stream, pbm_cursor** out);
+
+/*
  * The next up to n ranks (n >= 1): ids (int64) and their scores S_hat
  * (float32, all > 0) in host memory, *n_out of them.  Returns PVS_OK, or
  * PVS_EXHAUSTED once the last item of the support has been delivered (then

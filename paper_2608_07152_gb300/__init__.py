@@ -153,6 +153,7 @@ def _load() -> ctypes.CDLL:
         "pbm_index_free": (None, [P]),
         "pbm_cursor_open": (i32, [P, P, P, i32, pp]),
         "pbm_cursor_open_snapshot": (i32, [P, P, P, P, i32, pp]),
+        "pbm_cursor_open_stream": (i32, [P, P, P, P, i32, P, pp]),
         "pbm_next": (i32, [P, i32, P, P, P]),
         "pbm_cursor_range_bounds": (i32, [P, i64, i64, P]),
         "pbm_cursor_stats": (i32, [P, ctypes.POINTER(pbm_stats)]),
@@ -192,7 +193,7 @@ EXPORTED = ("pvs_build", "pvs_build_ex", "pvs_cursor_set_generator", "pvs_append
             "pvs_index_import", "pvs_index_set_wait_limit", "pvs_cursor_open_group",
             "pvs_cursor_set_readahead", "eahr_topk",
             "eahr_topk_lists", "pbm_build", "pbm_index_items", "pbm_index_ranges",
-            "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_next", "pbm_cursor_range_bounds",
+            "pbm_index_free", "pbm_cursor_open", "pbm_cursor_open_snapshot", "pbm_cursor_open_stream", "pbm_next", "pbm_cursor_range_bounds",
             "pbm_cursor_stats", "pbm_cursor_close", "eahr_topk_pbm", "pvs_merge_open",
             "pvs_merge_next", "pvs_merge_stats_get", "pvs_merge_close", "eahr_topk_merge",
             "pvs_executor_create", "pvs_executor_run", "pvs_executor_run_ex",
@@ -652,15 +653,22 @@ def pbm_index_free(index) -> None:
     _lib.pbm_index_free(index)
 
 
-def pbm_cursor_open(index, terms, weights, snap=None):
+def pbm_cursor_open(index, terms, weights, snap=None, stream=None):
     """PBM cursor for the query (terms, weights); with `snap` (a PVS snapshot
-    of the same id space) the items it deletes are left out of the ranking."""
+    of the same id space) the items it deletes are left out of the ranking;
+    `stream` (a CUDA stream handle, or an object with .cuda_stream) carries
+    the cursor's device work."""
     t = np.ascontiguousarray(terms, dtype=np.int32)
     w = np.ascontiguousarray(weights, dtype=np.float32)
     if t.shape != w.shape:
         raise ValueError("one weight per query term")
     out = ctypes.c_void_p()
-    if snap is None:
+    if stream is not None:
+        handle = getattr(stream, "cuda_stream", stream)
+        _check(_lib.pbm_cursor_open_stream(index, snap, t.ctypes.data, w.ctypes.data, t.size,
+                                           ctypes.c_void_p(int(handle)), ctypes.byref(out)),
+               "pbm_cursor_open_stream")
+    elif snap is None:
         _check(_lib.pbm_cursor_open(index, t.ctypes.data, w.ctypes.data, t.size,
                                     ctypes.byref(out)), "pbm_cursor_open")
     else:

@@ -24,6 +24,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -97,12 +98,18 @@ struct pbm_index {
     int64_t* blk_pbeg = nullptr;    // [nb + 1]
     float* blk_max = nullptr;       // [nb]
     int64_t* blk_off = nullptr;     // [n_terms + 1]
+    // closed cursors keep their device and pinned buffers here for the next
+    // open (allocating them per query cost a cudaMalloc of n_items keys and a
+    // cudaFree, which waits for the whole device)
+    std::vector<pbm_cursor*> cursor_pool;
+    std::mutex pool_mutex;
 };
 
 struct pbm_cursor {
     pbm_index* index = nullptr;
     cudaStream_t stream = nullptr;
     int nq = 0;
+    int nq_cap = 0;                   // capacity of terms, weights, starts
     int32_t* terms = nullptr;
     float* weights = nullptr;
     int64_t* starts = nullptr;        // [nq][nchunk + 1]
@@ -142,6 +149,8 @@ pvs_status fail(pbm_cursor* c, pvs_status s) {
     if (s < 0 && c->state >= 0) c->state = s;
     return s;
 }
+
+constexpr size_t kPbmCursorPool = 32;
 
 void free_cursor(pbm_cursor* c) {
     if (!c) return;
@@ -327,6 +336,8 @@ void pbm_index_free(pbm_index* x) {
     if (!x) return;
     DeviceGuard device_guard(x->device);
     if (x->stream) cudaStreamSynchronize(x->stream);
+    for (pbm_cursor* c : x->cursor_pool) free_cursor(c);
+    x->cursor_pool.clear();
     dfree(x->term_off);
     dfree(x->docs);
     dfree(x->imps);
@@ -343,7 +354,8 @@ void pbm_index_free(pbm_index* x) {
 namespace {
 
 pvs_status open_cursor(pbm_index* x, const std::shared_ptr<pvs::SnapData>& snap,
-                       const int32_t* terms, const float* weights, int32_t nq, pbm_cursor** out) {
+                       const int32_t* terms, const float* weights, int32_t nq,
+                       cudaStream_t stream, pbm_cursor** out) {
     if (!out) return PVS_ERR_INVALID;
     *out = nullptr;
     if (!x || nq < 0 || nq > pvs::kPbmMaxTerms || (nq > 0 && (!terms || !weights)))
@@ -360,30 +372,57 @@ pvs_status open_cursor(pbm_index* x, const std::shared_ptr<pvs::SnapData>& snap,
         if (!std::isfinite(weights[i])) return PVS_ERR_NONFINITE;
         if (weights[i] < 0.0f) return PVS_ERR_INVALID;
     }
-    pbm_cursor* c = new (std::nothrow) pbm_cursor();
+    pbm_cursor* c = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(x->pool_mutex);
+        if (!x->cursor_pool.empty()) {
+            c = x->cursor_pool.back();
+            x->cursor_pool.pop_back();
+        }
+    }
+    if (!c) c = new (std::nothrow) pbm_cursor();
     if (!c) return PVS_ERR_OOM;
+    // the state of a fresh cursor; buffers of a pooled one are kept
     c->index = x;
-    c->stream = x->stream;
+    c->stream = stream ? stream : x->stream;
     c->nq = nq;
+    c->snap.reset();
     if (snap && snap->d_tomb) c->snap = snap;   // deletions apply
+    c->ahead_pos = c->ahead_len = 0;
+    c->ahead_complete = false;
+    c->last_key = ~0ull;
+    c->n_pos = 0;
+    c->next = 0;
+    c->E = 64;
+    c->emitted = c->pulls = c->rounds = c->served_ahead = 0;
+    c->state = PVS_OK;
     auto bail = [&](pvs_status s) {
         free_cursor(c);
         return s;
     };
-    if (dalloc(&c->terms, (size_t)nq) != cudaSuccess ||
-        dalloc(&c->weights, (size_t)nq) != cudaSuccess ||
-        dalloc(&c->starts, (size_t)nq * (size_t)(x->nchunk + 1)) != cudaSuccess ||
-        dalloc(&c->H, (size_t)x->n_ranges) != cudaSuccess ||
-        dalloc(&c->rkeys, (size_t)x->n_ranges) != cudaSuccess ||
-        dalloc(&c->pool, (size_t)x->n_items) != cudaSuccess ||
-        dalloc(&c->ctr, 1) != cudaSuccess ||
-        dalloc(&c->sel64, 258) != cudaSuccess ||
-        cudaMallocHost(reinterpret_cast<void**>(&c->h_ctr), sizeof(pvs::PbmCounters)) !=
-            cudaSuccess ||
-        cudaMallocHost(reinterpret_cast<void**>(&c->h_ids),
-                       pvs::kPbmFastWindow * sizeof(int64_t)) != cudaSuccess ||
-        cudaMallocHost(reinterpret_cast<void**>(&c->h_scores),
-                       pvs::kPbmFastWindow * sizeof(float)) != cudaSuccess)
+    if (nq > c->nq_cap) {
+        dfree(c->terms);
+        dfree(c->weights);
+        dfree(c->starts);
+        c->nq_cap = 0;
+        const int cap = std::max(nq, 16);
+        if (dalloc(&c->terms, (size_t)cap) != cudaSuccess ||
+            dalloc(&c->weights, (size_t)cap) != cudaSuccess ||
+            dalloc(&c->starts, (size_t)cap * (size_t)(x->nchunk + 1)) != cudaSuccess)
+            return bail(PVS_ERR_OOM);
+        c->nq_cap = cap;
+    }
+    if ((!c->H && dalloc(&c->H, (size_t)x->n_ranges) != cudaSuccess) ||
+        (!c->rkeys && dalloc(&c->rkeys, (size_t)x->n_ranges) != cudaSuccess) ||
+        (!c->pool && dalloc(&c->pool, (size_t)x->n_items) != cudaSuccess) ||
+        (!c->ctr && dalloc(&c->ctr, 1) != cudaSuccess) ||
+        (!c->sel64 && dalloc(&c->sel64, 258) != cudaSuccess) ||
+        (!c->h_ctr && cudaMallocHost(reinterpret_cast<void**>(&c->h_ctr),
+                                     sizeof(pvs::PbmCounters)) != cudaSuccess) ||
+        (!c->h_ids && cudaMallocHost(reinterpret_cast<void**>(&c->h_ids),
+                                     pvs::kPbmFastWindow * sizeof(int64_t)) != cudaSuccess) ||
+        (!c->h_scores && cudaMallocHost(reinterpret_cast<void**>(&c->h_scores),
+                                        pvs::kPbmFastWindow * sizeof(float)) != cudaSuccess))
         return bail(PVS_ERR_OOM);
     std::memset(c->h_ctr, 0, sizeof(pvs::PbmCounters));
     cudaStream_t st = c->stream;
@@ -500,14 +539,21 @@ extern "C" {
 
 pvs_status pbm_cursor_open(pbm_index* x, const int32_t* terms, const float* weights, int32_t nq,
                            pbm_cursor** out) {
-    return open_cursor(x, nullptr, terms, weights, nq, out);
+    return open_cursor(x, nullptr, terms, weights, nq, nullptr, out);
 }
 
 pvs_status pbm_cursor_open_snapshot(pbm_index* x, const pvs_snapshot* snap, const int32_t* terms,
                                     const float* weights, int32_t nq, pbm_cursor** out) {
+    return pbm_cursor_open_stream(x, snap, terms, weights, nq, nullptr, out);
+}
+
+pvs_status pbm_cursor_open_stream(pbm_index* x, const pvs_snapshot* snap, const int32_t* terms,
+                                  const float* weights, int32_t nq, void* cuda_stream,
+                                  pbm_cursor** out) {
     if (out) *out = nullptr;
     if (snap && (!x || !snap->index || snap->index->device != x->device)) return PVS_ERR_INVALID;
-    return open_cursor(x, snap ? snap->data : nullptr, terms, weights, nq, out);
+    return open_cursor(x, snap ? snap->data : nullptr, terms, weights, nq,
+                       static_cast<cudaStream_t>(cuda_stream), out);
 }
 
 pvs_status pbm_next(pbm_cursor* c, int32_t n, int64_t* ids, float* scores, int32_t* n_out) {
@@ -672,6 +718,15 @@ void pbm_cursor_close(pbm_cursor* c) {
     if (!c) return;
     DeviceGuard device_guard(c->index ? c->index->device : -1);
     if (c->stream) cudaStreamSynchronize(c->stream);
+    pbm_index* x = c->index;
+    if (x) {   // the buffers serve the next open
+        c->snap.reset();
+        std::lock_guard<std::mutex> lock(x->pool_mutex);
+        if (x->cursor_pool.size() < kPbmCursorPool) {
+            x->cursor_pool.push_back(c);
+            return;
+        }
+    }
     free_cursor(c);
 }
 
