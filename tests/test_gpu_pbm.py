@@ -393,3 +393,49 @@ def test_eahr_pbm_adaptive_finish_matches_complete_list_fusion(deleted):
                     assert got == ro.as_float(f)
             finishes.append(st["complete"])
     assert any(c in (2, 3) for c in finishes)
+
+
+def test_pooled_cursors_on_streams_from_several_threads():
+    """Closed cursors are reused by later opens (term counts that grow and
+    shrink, with and without a snapshot), and cursors on their own streams
+    serve queries from four host threads at once: every ranking equals the
+    oracle's."""
+    import threading
+    n = 20_000
+    off, docs, imps = synth.bm25_postings(n, 4_000, 20.0, seed=81)
+    off, docs, imps = off.numpy(), docs.numpy(), imps.numpy()
+    rng = np.random.default_rng(82)
+    queries = []
+    for k in (1, 7, 20, 3, 12, 2, 9, 5):
+        terms = rng.choice(4_000, k, replace=False).astype(np.int32)
+        queries.append((terms, rng.uniform(0.5, 2.0, k).astype(np.float32)))
+    refs = [po.sparse_ranking(t, w, off, docs, imps, n) for t, w in queries]
+    index = pvs.pbm_build(off, docs, imps, n)
+    errors, results = [], {}
+    try:
+        def serve(k):
+            try:
+                torch.cuda.set_device(0)
+                stream = torch.cuda.Stream()
+                for j in range(k, len(queries), 4):
+                    for _ in range(2):   # the second open reuses a pooled cursor
+                        cur = pvs.pbm_cursor_open(index, *queries[j], stream=stream)
+                        try:
+                            results[(j, _)] = pull_all(cur, [20, 77], len(refs[j][0]))
+                        finally:
+                            pvs.pbm_cursor_close(cur)
+            except Exception as e:   # reported on the main thread
+                errors.append(e)
+        threads = [threading.Thread(target=serve, args=(k,)) for k in range(4)]
+        for t in threads:
+            t.start()
+        for t in threads:
+            t.join()
+    finally:
+        pvs.pbm_index_free(index)
+    assert not errors, errors
+    assert len(results) == 2 * len(queries)
+    for (j, _), (ids, sc) in results.items():
+        ref_ids, ref_sc = refs[j]
+        assert np.array_equal(ids, ref_ids)
+        assert np.array_equal(sc.view(np.uint32), ref_sc.view(np.uint32))
