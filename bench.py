@@ -261,8 +261,23 @@ def _finish(pvs, cur, stats_acc):
         stats_acc.append(s)
 
 
-def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, count):
-    """Latency to the first 20 and first 1,000 ranks, one query at a time."""
+def single_pass_record(stats, n, m_pad, peak):
+    """The lone queries' interval pass (interval_pass_kernel, one query per
+    read of the codes), timed by the library's CUDA events on each cursor's
+    stream: N (m_pad + 12) B read + 8 N B written per pass."""
+    ms = [s["interval_ms"] for s in stats if s.get("interval_ms", 0) > 0]
+    if not ms:
+        return None
+    med = float(statistics.median(ms))
+    gbps = (n * (m_pad + 12) + 8 * n) / (med / 1e3) / 1e9
+    return {"kernel": "interval_pass_kernel", "ms_p50": med, "GBps": gbps, "frac": gbps / peak,
+            "passes": len(ms)}
+
+
+def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, count,
+                    stats=None):
+    """Latency to the first 20 and first 1,000 ranks, one query at a time
+    (each cursor's statistics appended to `stats` when given)."""
     lat20, lat1000 = [], []
     for qi in range(count):
         t_open = torch.cuda.Event(enable_timing=True)
@@ -276,7 +291,7 @@ def measure_latency(pvs, torch, index, queries, out_ids, out_scores, stream, cou
             if p == 0:
                 t_20.record(stream)
         t_end.record(stream)
-        _finish(pvs, cur, None)
+        _finish(pvs, cur, stats)
         stream.synchronize()
         lat20.append(t_open.elapsed_time(t_20))
         lat1000.append(t_open.elapsed_time(t_end))
@@ -1465,8 +1480,9 @@ def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     # ---- latency of a lone query (its own cursor and pass), one at a time ----
     out_ids = torch.empty((1, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
     out_scores = torch.empty((1, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    lone = []
     lat20, lat1000 = measure_latency(pvs, torch, index, timed_q, out_ids, out_scores, stream,
-                                     min(n_timed, 20))
+                                     min(n_timed, 20), lone)
     e2e_elapsed = slowest(pg, e2e_elapsed, dev)
     e2e_value = ranks_total / e2e_elapsed
 
@@ -1515,6 +1531,7 @@ def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
                        "note": "a lone query with its own cursor and single-query pass"},
         "interval_pass": {"ms": pass_ms, "GBps": achieved, "queries_per_pass": group,
                           "ms_per_query": pass_ms / group, "passes_timed": passes},
+        "single_query_pass": single_pass_record(lone, n, m_pad, peak),
         "per_query": {"refined_mean": (st1["refined"] - st0["refined"]) / n_timed},
         "build_s": build_s,
         "clocks": clk.summary(),
