@@ -206,7 +206,7 @@ pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
                                  int32_t horizon, void* cuda_stream, pvs_cursor** out);
 
 /* Largest group of pvs_cursor_open_group. */
-#define PVS_GROUP_MAX 8
+#define PVS_GROUP_MAX 16
 
 /* Open nq (1 <= nq <= PVS_GROUP_MAX) cursors over one snapshot (`snap`, NULL:
  * the index's current visible set) whose score intervals come from ONE
@@ -222,7 +222,8 @@ pvs_status pvs_cursor_open_batch(pvs_index* index, const pvs_snapshot* snap,
  * can run on their own streams while the next group's pass streams the
  * codes.  The call returns once the queries are encoded and the pass is
  * queued.  Row widths the grouped pass does not serve (dim rounded up to 64
- * not in {128, 256, 384, 512, 768, 1024}) and nq == 1 give plain cursors
+ * not in {128, 256, 384, 512, 768, 1024}, or above 768 with nq > 8) and
+ * nq == 1 give plain cursors
  * with a pass of their own at the first pull.  out[0..nq-1] receive the
  * cursors; close each with pvs_cursor_close.  Errors as pvs_cursor_open; on
  * error no cursor is returned. */

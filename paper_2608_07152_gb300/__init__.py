@@ -334,7 +334,7 @@ def pvs_cursor_open(index, query, snap=None):
     return out
 
 
-PVS_GROUP_MAX = 8
+PVS_GROUP_MAX = 16
 
 
 def pvs_cursor_open_group(index, queries, snap=None, pass_stream=None, cursor_streams=None):

@@ -1,5 +1,5 @@
 // Grouped PVS interval pass (Sec. 2.3.1, App. A.1): the score intervals of
-// up to kGroupMax = 8 queries from one streaming read of the Int8 codes.
+// up to kGroupMax = 16 queries from one streaming read of the Int8 codes.
 //
 // A single query's pass is an HBM-bound GEMV at about one Int8 operation per
 // byte; queries answered together can share its code stream.  For 8
@@ -11,13 +11,21 @@
 // is exact: |z| <= 127, every product is an integer below 2^14 and every
 // partial sum an integer below 2^24, so the f32 accumulator holds the exact
 // Int8 dot product.  (dp4a on the CUDA cores, at two warp instructions per
-// clock per SM, made the 8-query pass compute-bound at 1.7 ms.)
+// clock per SM, made the 8-query pass compute-bound at 1.7 ms; s8 mma.sync
+// on the codes as they are, with eight consumer warps per SM, bound by the
+// tensor pipe at 1.49 ms.)  The conversion and the epilogue make the
+// consumers' arithmetic about as long as the code stream at 8 queries, so
+// 16 queries (split, below) take twice as long per pass: no gain per query.
 //
 // Structure: a persistent CTA per SM; a producer thread stages 64-row tiles
 // (codes, then the three per-vector parameter arrays) with four 1-D bulk
 // copies (the TMA engine's cp.async.bulk) through an mbarrier ring, as the
-// single-query pass does.  Eight consumer warps in two groups of four take
-// alternate tiles; warp b of a group owns rows 16b .. 16b+15 of its tiles.
+// single-query pass does.  Eight consumer warps form two groups of four;
+// warp b of a group owns rows 16b .. 16b+15 of the tiles it takes.  With up
+// to 8 queries the groups take alternate tiles, each for every query; with
+// 9 .. 16 (split) both take every tile, group 0 for queries 0 .. 7 and
+// group 1 for queries 8 .. 15, so a tile is released once all eight warps
+// have read it (query fragments in registers: m_pad up to 768).
 // (Rows staged one bulk copy each, into a padded pitch free of bank
 // conflicts, made the TMA issue rate the limit: 2.4 ms per pass.  With
 // unpadded rows the fragment loads below are 2-way bank conflicted, which
@@ -49,6 +57,7 @@ namespace pvs {
 namespace {
 
 constexpr int kGroupWarps = 8;                        // consumer warps
+constexpr int kGroupHalf = 8;                         // queries of one consumer group
 constexpr int kGroupThreads = (kGroupWarps + 1) * 32;
 constexpr int kGroupSmemMax = 220 * 1024;             // stage ring budget
 
@@ -140,7 +149,8 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < stages; ++s) {
             mbar_init(&full[s], 1);
-            mbar_init(&empty[s], kGroupWarps / 2);   // the four warps of one group
+            // the warps that read a tile: one group, or both when split
+            mbar_init(&empty[s], a.nq > kGroupHalf ? kGroupWarps : kGroupWarps / 2);
         }
         mbar_fence_init();
     }
@@ -186,19 +196,22 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
     }
 
     // ---------------- consumers ----------------
-    const int grp = warp / (kGroupWarps / 2);          // takes tiles k = grp, grp + 2, ...
+    const bool split = a.nq > kGroupHalf;
+    const int grp = warp / (kGroupWarps / 2);          // tiles k = grp, grp + 2, ... (or all)
     const int blk = warp % (kGroupWarps / 2);          // rows 16 blk .. 16 blk + 15
     const int g = lane >> 2, q = lane & 3;
+    const int qb = split ? kGroupHalf * grp : 0;       // this group's first query
 
-    // query g's B fragments for every step, converted once
+    // query qb + g's B fragments for every step, converted once
     uint32_t bf[kRegB ? STEPS : 1][2];
     {
-        const uint32_t* zq = reinterpret_cast<const uint32_t*>(a.zq[g < a.nq ? g : 0]);
+        const int qg = qb + g;
+        const uint32_t* zq = reinterpret_cast<const uint32_t*>(a.zq[qg < a.nq ? qg : 0]);
 #pragma unroll
         for (int j = 0; j < CPJ; ++j)
 #pragma unroll
             for (int s = 0; s < 4; ++s) {
-                const uint32_t w = g < a.nq ? zq[4 * (4 * j + q) + s] : 0u;
+                const uint32_t w = qg < a.nq ? zq[4 * (4 * j + q) + s] : 0u;
                 if constexpr (kRegB) {
                     codes_to_f16x2(w, bf[4 * j + s][0], bf[4 * j + s][1]);
                 } else if (warp == 0) {
@@ -213,16 +226,17 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
     LaneQuery Q[2];
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
-        Q[u].n = 2 * q + u;
+        Q[u].n = qb + 2 * q + u;
         Q[u].on = Q[u].n < a.nq;
         Q[u].q = Q[u].on ? *a.qs[Q[u].n] : QueryScalars{};
 #pragma unroll
         for (int j = 0; j < kSlotTop; ++j) Q[u].top[j] = -INFINITY;
     }
 
-    int k = grp;
-    for (int64_t t = blockIdx.x + (int64_t)grp * gridDim.x; t < ntiles;
-         t += 2 * (int64_t)gridDim.x, k += 2) {
+    const int kstep = split ? 1 : 2;
+    int k = split ? 0 : grp;
+    for (int64_t t = blockIdx.x + (split ? 0 : (int64_t)grp * gridDim.x); t < ntiles;
+         t += (int64_t)kstep * gridDim.x, k += kstep) {
         const int s = k % stages;
         const uint32_t ph = (uint32_t)(k / stages) & 1u;
         if (!mbar_wait(&full[s], ph, a.wait_ns)) {
@@ -297,6 +311,13 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
 #pragma unroll
             for (int j = 0; j < kSlotTop; ++j) dst[slot * kSlotTop + j] = Q[u].top[j];
         }
+        // split: this slot scanned nothing for the other group's queries
+        const int other = kGroupHalf * (1 - grp) + 2 * q + u;
+        float* dso = split && other < a.nq ? a.slot_top[other] : nullptr;
+        if (dso) {
+#pragma unroll
+            for (int j = 0; j < kSlotTop; ++j) dso[slot * kSlotTop + j] = -INFINITY;
+        }
     }
 }
 
@@ -321,6 +342,7 @@ cudaError_t launch_group_tpl(const IntervalGroupArgs& a, int num_sms, cudaStream
 
 bool interval_group_supported(int m_pad, int nq) {
     if (nq < 1 || nq > kGroupMax || m_pad < 64 || m_pad % 64 != 0) return false;
+    if (nq > kGroupHalf && m_pad / 64 > kGroupRegCPJ) return false;   // split: fragments in registers
     switch (m_pad / 64) {
         case 1: case 2: case 3: case 4: case 6: case 8: case 12: case 16: return true;
         default: return false;
@@ -334,9 +356,10 @@ int64_t interval_group_slots(int64_t rows, int m_pad, int nq, int num_sms,
     const int64_t ntiles = (rows + kTileRows - 1) / kTileRows;
     const int64_t grid = ntiles < num_sms ? ntiles : num_sms;
     // CTA b scans tiles b, b + grid, ... (at least ntiles / grid of them);
-    // its two warp groups take alternate ones, and only the pass's very last
-    // tile can be partial; a slot sees two rows of each tile of its group
-    const int64_t per_group = (ntiles / grid) / 2;
+    // its two warp groups take alternate ones (or, split, both take every
+    // one), and only the pass's very last tile can be partial; a slot sees
+    // two rows of each tile of its group
+    const int64_t per_group = nq > kGroupHalf ? ntiles / grid : (ntiles / grid) / 2;
     *min_rows_per_slot = per_group > 0 ? (per_group - 1) * 2 : 0;
     return grid * kGroupWarps * 8;
 }

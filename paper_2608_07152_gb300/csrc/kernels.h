@@ -208,7 +208,7 @@ cudaError_t launch_interval_simple(const IntervalArgs& a, cudaStream_t st);
 // own outputs lo[g], hi[g], status[g] and slot_top[g] (may be null).  A
 // slot of the grouped pass is (CTA, consumer warp, MMA row pair):
 // interval_group_slots gives their count and the fewest rows any scans.
-constexpr int kGroupMax = 8;
+constexpr int kGroupMax = 16;
 struct IntervalGroupArgs {
     const int8_t* codes;
     const float* scale;

@@ -216,7 +216,7 @@ def test_grouped_requests_with_exhaustion_and_a_failed_query():
             assert n_out[9] == 0 and np.all(ids[9] == -1)
             _check_rows(V, Q, ids, sc, n_out, 80, rows=[i for i in range(17) if i != 9])
             with pytest.raises(pvs.PvsError):
-                pvs.pvs_executor_set_group(ex, 9)
+                pvs.pvs_executor_set_group(ex, pvs.PVS_GROUP_MAX + 1)
         finally:
             pvs.pvs_executor_destroy(ex)
     finally:

@@ -30,7 +30,10 @@ def _oracle_bounds(V, q, m):
 
 @pytest.mark.parametrize("m,n,nq", [(128, 9_731, 8), (100, 20_123, 3), (768, 30_011, 8),
                                     (768, 12_345, 2), (1024, 17_777, 5), (384, 40_961, 8),
-                                    (256, 8_193, 4), (512, 25_000, 7)])
+                                    (256, 8_193, 4), (512, 25_000, 7),
+                                    # 9 .. 16 queries: both warp groups on every tile
+                                    (768, 30_011, 16), (128, 9_731, 12), (384, 40_961, 9),
+                                    (512, 25_000, 16)])
 def test_group_bounds_equal_single_pass_and_oracle(m, n, nq):
     V = synth.unit_normal(n, m, seed=81 + m, device="cuda")
     Q = synth.unit_normal(nq, m, seed=82 + m, device="cuda")
@@ -72,8 +75,9 @@ def test_group_bounds_equal_single_pass_and_oracle(m, n, nq):
         assert np.array_equal(sc.view(np.uint32), ref_sc[:300].view(np.uint32))
 
 
-def test_group_on_own_streams_with_deletions_and_deep_pulls():
-    n, m, nq = 60_000, 768, 8
+@pytest.mark.parametrize("nq", [8, 16])
+def test_group_on_own_streams_with_deletions_and_deep_pulls(nq):
+    n, m = 60_000, 768
     V = synth.unit_normal(n, m, seed=91, device="cuda")
     Q = synth.unit_normal(nq, m, seed=92)
     rng = np.random.default_rng(93)
@@ -111,7 +115,9 @@ def test_group_on_own_streams_with_deletions_and_deep_pulls():
 
 
 def test_group_with_a_width_the_grouped_pass_does_not_serve_and_one_query():
-    for m, nq in ((1100, 3), (768, 1)):
+    # 1100: no grouped kernel; 1024 with 16 queries: no split kernel (the
+    # query fragments would not fit in registers); one query: a plain cursor
+    for m, nq in ((1100, 3), (768, 1), (1024, 16)):
         n = 5_000
         V = synth.unit_normal(n, m, seed=95, device="cuda")
         Q = synth.unit_normal(nq, m, seed=96)
@@ -143,7 +149,7 @@ def test_group_errors_and_timeout():
             pvs.pvs_cursor_open_group(index, bad)
         assert e.value.status == pvs.PVS_ERR_NONFINITE
         with pytest.raises(pvs.PvsError) as e:
-            pvs.pvs_cursor_open_group(index, synth.unit_normal(9, m, seed=99))
+            pvs.pvs_cursor_open_group(index, synth.unit_normal(pvs.PVS_GROUP_MAX + 1, m, seed=99))
         assert e.value.status == pvs.PVS_ERR_INVALID
         # the grouped pass's waits give up at once: the open fails, no cursor
         pvs.pvs_index_set_wait_limit(index, 0)
