@@ -162,6 +162,18 @@ __device__ __forceinline__ int keys_at_most(const uint64_t* k, int n, uint64_t x
 }
 
 constexpr int kCountWarps = 8;
+// Straddling rows a block queues for the residual level (and for the fp32
+// rows after it), flushed before a tile of kCountWarps * 32 rows could overflow.
+constexpr int kPlaceQueue = 2048;
+
+// Pinned staging of one rank query: ids in (8 B dense, 4 B sparse), per dense
+// item two 8-byte counts (plus one) and its key, per sparse item its rank,
+// two status words.
+constexpr size_t kRankQueryPinned = size_t(64) << 10;
+static_assert((size_t)kRankQueryMax * 12 + ((size_t)kRankQueryMax + 1) * 16 +
+                      (size_t)kRankQueryMax * 12 + 8 <=
+                  kRankQueryPinned,
+              "rank-query staging");
 
 // fp32 inner product of q and v (m_raw floats, 16-byte aligned, zero padded)
 // by one warp: each lane a chain of FMAs over its float4s, then a butterfly
@@ -221,22 +233,246 @@ __device__ __forceinline__ float fast_dot_warp(const float* __restrict__ q,
     return f;
 }
 
+// Upper bound of |x|, x the exact value that y = RN(x) rounds (a single
+// binary32 rounding: |x - y| <= 2^-23 |y| + 2^-149 covers the relative error
+// u |x| <= u (|y| + |x - y|) and the subnormal range).
+__device__ __forceinline__ float abs_before_rn(float y) {
+    return __fadd_ru(__fadd_ru(fabsf(y), __fmul_ru(fabsf(y), 0x1p-23f)), 0x1p-149f);
+}
+
+// Residual codes of rows [r0, r0 + n), one warp per row, in binary32 with
+// directed rounding.  e_j = RN(v_j - s z_j) (one FMA; v the authoritative
+// row, s and z its scale and codes), s2 = RN(max_j |e_j| / 7), z2_j =
+// clip(rint(e_j / s2), -7, 7), r2_j = RN(e_j - s2 z2_j) (one FMA).  The true
+// residual v_j - s z_j - s2 z2_j is at most a_j = |r2_j|^ + (|e_j|^ -
+// |e_j|) in magnitude (^: the bound of abs_before_rn), so rnorm =
+// RU(sqrt(sum a_j^2)) with every operation rounded up, and wnorm =
+// RU(||v||^ + rnorm) bounds ||s z + s2 z2|| = ||v - r2||.  Both hold whatever
+// the stored codes are.
+__global__ void __launch_bounds__(256) resid_build_kernel(
+    const float* __restrict__ raw, const int8_t* __restrict__ codes,
+    const float* __restrict__ scale, int64_t r0, int64_t n, int m, int m_pad, int m_raw,
+    uint8_t* __restrict__ resid, float4* __restrict__ rparam, int* status) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+    const int nw = m_pad >> 3;   // 32-bit words of nibbles per row
+    for (int64_t i = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n;
+         i += warps) {
+        const int64_t row = r0 + i;
+        const float* v = raw + row * (int64_t)m_raw;
+        const int8_t* z = codes + row * (int64_t)m_pad;
+        const float s = scale[row];
+        auto e_of = [&](int d) { return d < m ? fmaf(-s, (float)z[d], v[d]) : 0.0f; };
+        float emax = 0.0f;
+        for (int d = lane; d < m; d += kWarp) emax = fmaxf(emax, fabsf(e_of(d)));
+        emax = warp_max(emax);
+        float s2 = 0.0f;
+        if (emax > 0.0f) {
+            s2 = __fdiv_rn(emax, 7.0f);
+            if (s2 == 0.0f) s2 = __uint_as_float(1u);   // 2^-149
+        }
+        if (!isfinite(s2)) s2 = 0.0f;
+        auto z2_of = [&](float e) {
+            if (s2 == 0.0f) return 0;
+            return (int)fminf(fmaxf(rintf(__fdiv_rn(e, s2)), -7.0f), 7.0f);
+        };
+        float ss = 0.0f, sv = 0.0f;   // sums of squares, rounded up
+        for (int t = lane; t < nw; t += kWarp) {
+            uint32_t w = 0;
+            for (int k = 0; k < 8; ++k) {
+                const int d = 8 * t + k;
+                const float e = e_of(d);
+                const int c = z2_of(e);
+                w |= (uint32_t)(c + 8) << (8 * (k >> 1) + 4 * (k & 1));
+                if (d < m) {
+                    const float r = fmaf(-s2, (float)c, e);
+                    const float a = __fadd_ru(abs_before_rn(r),
+                                              __fsub_ru(abs_before_rn(e), fabsf(e)));
+                    ss = __fadd_ru(ss, __fmul_ru(a, a));
+                    sv = __fadd_ru(sv, __fmul_ru(v[d], v[d]));
+                }
+            }
+            reinterpret_cast<uint32_t*>(resid + row * (int64_t)(m_pad >> 1))[t] = w;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            ss = __fadd_ru(ss, __shfl_xor_sync(0xffffffffu, ss, o));
+            sv = __fadd_ru(sv, __shfl_xor_sync(0xffffffffu, sv, o));
+        }
+        if (lane == 0) {
+            const float nb = __fsqrt_ru(ss);
+            const float wb = __fadd_ru(__fsqrt_ru(sv), nb);
+            if (!isfinite(wb)) set_status(status, PVS_ERR_OVERFLOW);
+            rparam[row] = make_float4(s, s2, nb, wb);
+        }
+    }
+}
+
+// Rows of at most this many padded dimensions get residual codes (the
+// query's 16-bit codes then fit in 16 KB of shared memory).
+constexpr int kResidMaxPad = 4096;
+
+// The residual codes of every row of the index, extended on stream st; st
+// then waits for the last build, whichever stream ran it.
+pvs_status ensure_resid(pvs_index* x, cudaStream_t st, int* status) {
+    std::lock_guard<std::mutex> lock(x->resid_mutex);
+    if (!x->resid) {
+        const size_t cap = (size_t)std::max<int64_t>(x->cap, 1);
+        if (cudaMalloc(reinterpret_cast<void**>(&x->resid), cap * (size_t)(x->m_pad >> 1)) !=
+                cudaSuccess ||
+            cudaMalloc(reinterpret_cast<void**>(&x->rparam), cap * sizeof(float4)) !=
+                cudaSuccess) {
+            const cudaError_t e = cudaGetLastError();
+            cudaFree(x->resid), cudaFree(x->rparam);
+            x->resid = nullptr, x->rparam = nullptr;
+            return e == cudaErrorMemoryAllocation ? PVS_ERR_OOM : PVS_ERR_CUDA;
+        }
+        x->resid_rows = 0;
+    }
+    if (!x->resid_ready &&
+        cudaEventCreateWithFlags(&x->resid_ready, cudaEventDisableTiming) != cudaSuccess) {
+        cudaGetLastError();
+        return PVS_ERR_CUDA;
+    }
+    cudaError_t e = cudaSuccess;
+    if (x->resid_rows < x->size) {
+        const int64_t r0 = x->resid_rows, n = x->size - r0;
+        count_launches(1);
+        resid_build_kernel<<<(unsigned)std::min<int64_t>((n + 7) / 8, 152 * 64), 256, 0, st>>>(
+            x->raw, x->codes, x->scale, r0, n, x->m, x->m_pad, x->m_raw, x->resid, x->rparam,
+            status);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = cudaEventRecord(x->resid_ready, st);
+        if (e == cudaSuccess) x->resid_rows = x->size;
+    } else {
+        e = cudaStreamWaitEvent(st, x->resid_ready, 0);
+    }
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return PVS_ERR_CUDA;
+    }
+    return PVS_OK;
+}
+
+// The query in integers for the residual level, computed by every block of
+// a rank count into shared memory: q = s_q zq + e_q with |zq_j| <= Q (Q
+// keeps every integer dot product below 2^31), zq as 16-bit pairs twice,
+// in dimension order (for the int8 codes) and in the residual codes' nibble
+// order (dims 8t + 0, 2, 4, 6, 1, 3, 5, 7: the pairs (0,2) (4,6) of the low
+// nibbles, (1,3) (5,7) of the high ones), eq >= ||e_q|| and bias = sum zq_j.
+struct ResidQuery {
+    float sq, eq;
+    int bias;
+};
+
+// D1 = zq.z and D2 = zq.z2 over one row, exact integers, by the eight
+// lanes of an aligned group (dp2a): lane sl of the group takes the 16-dim
+// chunks sl, sl + 8, ..., so the group reads whole 128-byte lines of codes;
+// every lane of the group returns the same sums.  Lanes whose row is not
+// valid take part in the shuffles with zero sums.
+__device__ __forceinline__ void resid_dots_group8(const int32_t* __restrict__ zqn,
+                                                  const int32_t* __restrict__ zqp, int bias,
+                                                  const int8_t* __restrict__ z,
+                                                  const uint8_t* __restrict__ z2, int m_pad,
+                                                  bool valid, int* D1, int* D2) {
+    const int sl = threadIdx.x & 7;
+    const int n16 = m_pad >> 4;   // 16 dims per chunk: 16 code bytes, 8 residual bytes
+    const uint4* zc = reinterpret_cast<const uint4*>(z);
+    const uint2* rc = reinterpret_cast<const uint2*>(z2);
+    const int4* qn = reinterpret_cast<const int4*>(zqn);
+    const int4* qp = reinterpret_cast<const int4*>(zqp);
+    int acc1 = 0, acc2 = 0;
+    if (valid) {
+#pragma unroll 1
+        for (int c0 = sl; c0 < n16; c0 += 24) {
+            uint4 a[3];
+            uint2 b[3];
+#pragma unroll
+            for (int u = 0; u < 3; ++u) {
+                const int c = c0 + 8 * u;
+                a[u] = c < n16 ? __ldg(zc + c) : make_uint4(0, 0, 0, 0);
+                b[u] = c < n16 ? __ldg(rc + c) : make_uint2(0x88888888u, 0x88888888u);
+            }
+#pragma unroll
+            for (int u = 0; u < 3; ++u) {
+                const int c = c0 + 8 * u;
+                if (c >= n16) break;
+                const int4 n0 = qn[2 * c], n1 = qn[2 * c + 1];
+                const int4 p0 = qp[2 * c], p1 = qp[2 * c + 1];
+                acc1 = __dp2a_lo(n0.x, (int)a[u].x, acc1);
+                acc1 = __dp2a_hi(n0.y, (int)a[u].x, acc1);
+                acc1 = __dp2a_lo(n0.z, (int)a[u].y, acc1);
+                acc1 = __dp2a_hi(n0.w, (int)a[u].y, acc1);
+                acc1 = __dp2a_lo(n1.x, (int)a[u].z, acc1);
+                acc1 = __dp2a_hi(n1.y, (int)a[u].z, acc1);
+                acc1 = __dp2a_lo(n1.z, (int)a[u].w, acc1);
+                acc1 = __dp2a_hi(n1.w, (int)a[u].w, acc1);
+                const int l0 = (int)(b[u].x & 0x0F0F0F0Fu), h0 = (int)((b[u].x >> 4) & 0x0F0F0F0Fu);
+                const int l1 = (int)(b[u].y & 0x0F0F0F0Fu), h1 = (int)((b[u].y >> 4) & 0x0F0F0F0Fu);
+                acc2 = __dp2a_lo(p0.x, l0, acc2);
+                acc2 = __dp2a_hi(p0.y, l0, acc2);
+                acc2 = __dp2a_lo(p0.z, h0, acc2);
+                acc2 = __dp2a_hi(p0.w, h0, acc2);
+                acc2 = __dp2a_lo(p1.x, l1, acc2);
+                acc2 = __dp2a_hi(p1.y, l1, acc2);
+                acc2 = __dp2a_lo(p1.z, h1, acc2);
+                acc2 = __dp2a_hi(p1.w, h1, acc2);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 4; o > 0; o >>= 1) {   // within the aligned group of eight
+        acc1 += __shfl_xor_sync(0xffffffffu, acc1, o);
+        acc2 += __shfl_xor_sync(0xffffffffu, acc2, o);
+    }
+    *D1 = acc1;
+    *D2 = acc2 - 8 * bias;   // nibbles hold z2 + 8
+}
+
+// The exact inner product q.v lies in [*fl, *fh], from the row's dots
+// D1 = zq.z and D2 = zq.z2 and rp = (s, s2, rnorm, wnorm).  With
+// w = s z + s2 z2 (so v = w + r2) and q = s_q zq + e_q:
+//   q.v = s_q (s D1 + s2 D2) + e_q.w + q.r2,
+// |e_q.w| <= eq wnorm, |q.r2| <= ||q|| rnorm.  The binary32 evaluation
+// c = RN(s_q RN(RN(s RN(D1)) + RN(s2 RN(D2)))) has six roundings of relative
+// error u = 2^-24 each, so |c - s_q (s D1 + s2 D2)| <= 8 u s_q (|s D1'| +
+// |s2 D2'|) with room (' the rounded terms), plus (s_q + 1) 2^-147 for the
+// subnormal range.  False when the bounds are not finite.
+__device__ __forceinline__ bool resid_bounds(int D1, int D2, const float4 rp,
+                                             const ResidQuery& rq, float qnorm, float* fl,
+                                             float* fh) {
+    const float a = __fmul_rn(rp.x, __int2float_rn(D1));
+    const float b = __fmul_rn(rp.y, __int2float_rn(D2));
+    const float c = __fmul_rn(rq.sq, __fadd_rn(a, b));
+    float E = __fmul_ru(__fmul_ru(rq.sq, __fadd_ru(fabsf(a), fabsf(b))), 0x1p-21f);
+    E = __fadd_ru(E, __fadd_ru(__fmul_ru(rq.sq, 0x1p-147f), 0x1p-147f));
+    E = __fadd_ru(E, __fmul_ru(rq.eq, rp.w));
+    E = __fadd_ru(E, __fmul_ru(qnorm, rp.z));
+    *fl = __fsub_rd(c, E);
+    *fh = __fadd_ru(c, E);
+    return isfinite(*fl) && isfinite(*fh);
+}
+
 // hist[j] = number of visible rows whose key lies above exactly j of the
 // queried keys (sorted ascending); the rank of the item with the j-th
 // smallest key is then 1 + sum of hist[t] for t > j.  A row's key lies in
 // [key(lo, y), key(hi, y)]; when no queried key falls in that range the
 // count is fixed by the bounds.  Otherwise, with `exact`, the row's
-// authoritative score is computed (and must lie in its interval, App. A.1);
+// authoritative score is placed: first by the bounds of its residual codes
+// (resid_dot_warp, 1.5 B per dimension), else by the fp32 dot with its error
+// bound, else exactly (and it must lie in its interval, App. A.1);
 // without, the row counts in hist[a] (a = the queried keys below key(lo, y):
 // it is surely above those) and may lie above the keys a .. b-1 (b = the
 // keys at most key(hi, y)): maybe[a] += 1, maybe[b] -= 1, so that the prefix
 // sum of `maybe` at j counts the rows that may lie above the j-th key.  A
 // row with hi = -inf has been delivered and lies above every queried key.
-__global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
+__global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
     const float* __restrict__ lo, const float* __restrict__ hi, int64_t rows,
     const uint32_t* __restrict__ tomb, const float* __restrict__ qraw,
     const float* __restrict__ raw, int m_raw, const uint64_t* __restrict__ qkeys, int nq, int exact,
-    unsigned long long* hist, unsigned long long* maybe, int* status, DevCounters* ctr) {
+    const int8_t* __restrict__ codes, const uint8_t* __restrict__ resid,
+    const float4* __restrict__ rparam, int m_pad, int qrange,
+    const QueryScalars* __restrict__ qs, unsigned long long* hist, unsigned long long* maybe, int* status, DevCounters* ctr) {
     __shared__ uint64_t sk[kRankQueryMax];
     __shared__ unsigned int sh[kRankQueryMax + 1];
     __shared__ int sm[kRankQueryMax + 1];
@@ -249,80 +485,232 @@ __global__ void __launch_bounds__(kCountWarps * 32) rank_count_kernel(
     const int lane = threadIdx.x & 31;
     const int64_t step = (int64_t)gridDim.x * kCountWarps * 32;
     unsigned long long scored = 0, fallbacks = 0;
-    for (int64_t base = ((int64_t)blockIdx.x * kCountWarps + (threadIdx.x >> 5)) * 32; base < rows;
-         base += step) {
-        const int64_t y = base + lane;
-        int bin = -1;   // -1: nothing to count from the bounds
-        bool straddle = false;
-        float l = 0.f, h = 0.f;
-        if (y < rows && !tombstoned(tomb, y)) {
-            l = lo[y];
-            h = hi[y];
-            if (h == -INFINITY) {
-                bin = nq;
-            } else {
-                const int a = keys_below(sk, nq, rank_key(l, (uint32_t)y));
-                const int b = keys_at_most(sk, nq, rank_key(h, (uint32_t)y));
-                if (a == b) {
-                    bin = a;
-                } else if (exact) {
-                    straddle = true;
-                } else {
-                    bin = a;
-                    atomicAdd(&sm[a], 1);
-                    atomicAdd(&sm[b], -1);
-                }
-            }
+    // the query's integer form for the residual level (every block computes
+    // the same): s_q = RN(max |q_j| / Q), zq_j = clip(rint(RN(q_j / s_q)),
+    // -Q, Q), e_j = RN(q_j - s_q zq_j) (one FMA), eq = RU(sqrt(sum of the
+    // bounds of |q_j - s_q zq_j| squared)) with every operation rounded up
+    extern __shared__ int4 rq_smem[];
+    int32_t* zqn = reinterpret_cast<int32_t*>(rq_smem);   // m_pad / 2 pairs
+    int32_t* zqp = zqn + (m_pad >> 1);
+    __shared__ ResidQuery srq;
+    __shared__ float red_f[kCountWarps];
+    __shared__ int red_i[kCountWarps];
+    const bool use_resid = exact && resid != nullptr;
+    float qnorm = 0.0f;
+    if (use_resid) {
+        const int w = threadIdx.x >> 5;
+        const float Qf = (float)qrange;
+        float mq = 0.0f;
+        for (int j = threadIdx.x; j < m_raw; j += blockDim.x) mq = fmaxf(mq, fabsf(qraw[j]));
+        mq = warp_max(mq);
+        if (lane == 0) red_f[w] = mq;
+        __syncthreads();
+        mq = red_f[0];
+        for (int i = 1; i < kCountWarps; ++i) mq = fmaxf(mq, red_f[i]);
+        __syncthreads();   // red_f is written again below
+        float sq = 1.0f;
+        if (mq > 0.0f) {
+            sq = __fdiv_rn(mq, Qf);
+            if (sq == 0.0f) sq = __uint_as_float(1u);   // 2^-149
         }
-        // one shared-memory add per distinct bin of the warp
-        const unsigned int live = __ballot_sync(0xffffffffu, bin >= 0);
-        if (bin >= 0) {
-            const unsigned int same = __match_any_sync(live, bin);
-            if (lane == __ffs(same) - 1) atomicAdd(&sh[bin], (unsigned int)__popc(same));
+        int16_t* n16 = reinterpret_cast<int16_t*>(zqn);
+        int16_t* p16 = reinterpret_cast<int16_t*>(zqp);
+        float ss = 0.0f;
+        int bias = 0;
+        for (int j = threadIdx.x; j < m_pad; j += blockDim.x) {
+            int c = 0;
+            if (j < m_raw && mq > 0.0f) {
+                c = (int)fminf(fmaxf(rintf(__fdiv_rn(qraw[j], sq)), -Qf), Qf);
+                const float a = abs_before_rn(fmaf(-sq, (float)c, qraw[j]));
+                ss = __fadd_ru(ss, __fmul_ru(a, a));
+            } else if (j < m_raw) {
+                ss = __fadd_ru(ss, __fmul_ru(qraw[j], qraw[j]));
+            }
+            const int k = j & 7;
+            n16[j] = (int16_t)c;
+            p16[(j & ~7) + ((k & 1) ? 4 + (k >> 1) : (k >> 1))] = (int16_t)c;
+            bias += c;
         }
-        unsigned int todo = __ballot_sync(0xffffffffu, straddle);
-        while (todo) {
-            const int src = __ffs(todo) - 1;
-            todo &= todo - 1;
-            const int64_t r = base + src;
-            if (todo) {   // the next row to score, into L2 while this one is scored
-                const char* nrow =
-                    reinterpret_cast<const char*>(raw + (base + __ffs(todo) - 1) * (int64_t)m_raw);
-                for (int off = lane * 128; off < m_raw * 4; off += 32 * 128)
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(nrow + off));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) ss = __fadd_ru(ss, __shfl_xor_sync(0xffffffffu, ss, o));
+        bias = __reduce_add_sync(0xffffffffu, bias);
+        if (lane == 0) {
+            red_f[w] = ss;
+            red_i[w] = bias;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float st = 0.0f;
+            int bt = 0;
+            for (int i = 0; i < kCountWarps; ++i) {
+                st = __fadd_ru(st, red_f[i]);
+                bt += red_i[i];
             }
-            const float lr = __shfl_sync(0xffffffffu, l, src);
-            const float hr = __shfl_sync(0xffffffffu, h, src);
-            // first a plain fp32 dot with its error bound: it places the
-            // authoritative score RN(q.v) in [fl, fh], which fixes the row's
-            // bin unless a queried key falls in that range
-            float err;
-            const float f = fast_dot_warp(qraw, raw + r * (int64_t)m_raw, m_raw, &err);
-            int fast_bin = -1;
-            if (lane == 0 && isfinite(f) && isfinite(err)) {
-                // a score of zero is reported as +0, whose key is above -0's
-                const float fl = __fsub_rd(f, err);
-                const float fh = __fadd_ru(f, err) == 0.0f ? 0.0f : __fadd_ru(f, err);
-                const int a = keys_below(sk, nq, rank_key(fl, (uint32_t)r));
-                const int b = keys_at_most(sk, nq, rank_key(fh, (uint32_t)r));
-                if (a == b) {
-                    fast_bin = a;
-                    if (fh < lr || fl > hr) set_status(status, PVS_ERR_INTERVAL);
-                    atomicAdd(&sh[a], 1u);
-                    ++scored;
-                }
-            }
-            if (__shfl_sync(0xffffffffu, fast_bin, 0) >= 0) continue;
-            bool fb = false;
-            const float s = exact_dot_warp_eft(qraw, qraw, raw + r * (int64_t)m_raw, m_raw, &fb);
-            if (lane == 0) {
-                if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
-                else if (s < lr || s > hr) set_status(status, PVS_ERR_INTERVAL);
-                atomicAdd(&sh[keys_below(sk, nq, rank_key(s, (uint32_t)r))], 1u);
+            srq.sq = sq;
+            srq.eq = __fsqrt_ru(st);
+            srq.bias = bt;
+        }
+        __syncthreads();
+        qnorm = qs->qnorm;
+    }
+    const int64_t rbytes = m_pad >> 1;
+    const int warp = threadIdx.x >> 5;
+    // row r's bin from its fp32 row, by the whole warp: first a plain fp32
+    // dot with its error bound, which places the authoritative score RN(q.v)
+    // in [fl, fh] and fixes the bin unless a queried key falls in that range;
+    // then the exact dot
+    auto place_fp32 = [&](int64_t r, float lr, float hr) {
+        float err;
+        const float f = fast_dot_warp(qraw, raw + r * (int64_t)m_raw, m_raw, &err);
+        int fast_bin = -1;
+        if (lane == 0 && isfinite(f) && isfinite(err)) {
+            // a score of zero is reported as +0, whose key is above -0's
+            const float fl = __fsub_rd(f, err);
+            const float fh = __fadd_ru(f, err) == 0.0f ? 0.0f : __fadd_ru(f, err);
+            const int a = keys_below(sk, nq, rank_key(fl, (uint32_t)r));
+            const int b = keys_at_most(sk, nq, rank_key(fh, (uint32_t)r));
+            if (a == b) {
+                fast_bin = a;
+                if (fh < lr || fl > hr) set_status(status, PVS_ERR_INTERVAL);
+                atomicAdd(&sh[a], 1u);
                 ++scored;
-                fallbacks += fb ? 1 : 0;
             }
         }
+        if (__shfl_sync(0xffffffffu, fast_bin, 0) >= 0) return;
+        bool fb = false;
+        const float s = exact_dot_warp_eft(qraw, qraw, raw + r * (int64_t)m_raw, m_raw, &fb);
+        if (lane == 0) {
+            if (!isfinite(s)) set_status(status, PVS_ERR_OVERFLOW);
+            else if (s < lr || s > hr) set_status(status, PVS_ERR_INTERVAL);
+            atomicAdd(&sh[keys_below(sk, nq, rank_key(s, (uint32_t)r))], 1u);
+            ++scored;
+            fallbacks += fb ? 1 : 0;
+        }
+    };
+    // with the residual codes, the block queues its straddling rows and
+    // places them eight lanes per row; the rows they leave open are queued
+    // again and scored one warp per row
+    __shared__ int32_t q_rows[kPlaceQueue];
+    __shared__ int32_t f_rows[kPlaceQueue];
+    __shared__ int q_n, f_n;
+    if (threadIdx.x == 0) q_n = f_n = 0;
+    __syncthreads();
+    for (int64_t tb = (int64_t)blockIdx.x * kCountWarps * 32;; tb += step) {
+        const int64_t base = tb + warp * 32;
+        if (base < rows) {
+            const int64_t y = base + lane;
+            int bin = -1;   // -1: nothing to count from the bounds
+            bool straddle = false;
+            float l = 0.f, h = 0.f;
+            if (y < rows && !tombstoned(tomb, y)) {
+                l = lo[y];
+                h = hi[y];
+                if (h == -INFINITY) {
+                    bin = nq;
+                } else {
+                    const int a = keys_below(sk, nq, rank_key(l, (uint32_t)y));
+                    const int b = keys_at_most(sk, nq, rank_key(h, (uint32_t)y));
+                    if (a == b) {
+                        bin = a;
+                    } else if (exact) {
+                        straddle = true;
+                    } else {
+                        bin = a;
+                        atomicAdd(&sm[a], 1);
+                        atomicAdd(&sm[b], -1);
+                    }
+                }
+            }
+            // one shared-memory add per distinct bin of the warp
+            const unsigned int live = __ballot_sync(0xffffffffu, bin >= 0);
+            if (bin >= 0) {
+                const unsigned int same = __match_any_sync(live, bin);
+                if (lane == __ffs(same) - 1) atomicAdd(&sh[bin], (unsigned int)__popc(same));
+            }
+            if (use_resid) {
+                if (straddle) q_rows[atomicAdd(&q_n, 1)] = (int32_t)y;
+            } else {
+                unsigned int todo = __ballot_sync(0xffffffffu, straddle);
+                while (todo) {
+                    const int src = __ffs(todo) - 1;
+                    todo &= todo - 1;
+                    if (todo) {   // the next row to score, into L2 while this one is scored
+                        const char* nrow = reinterpret_cast<const char*>(
+                            raw + (base + __ffs(todo) - 1) * (int64_t)m_raw);
+                        for (int off = lane * 128; off < m_raw * 4; off += 32 * 128)
+                            asm volatile("prefetch.global.L2 [%0];" ::"l"(nrow + off));
+                    }
+                    place_fp32(base + src, __shfl_sync(0xffffffffu, l, src),
+                               __shfl_sync(0xffffffffu, h, src));
+                }
+            }
+        }
+        const bool last = tb + step >= rows;   // the same in every thread of the block
+        if (!use_resid) {
+            if (last) break;
+            continue;
+        }
+        __syncthreads();
+        const int n = q_n;
+        if (n > kPlaceQueue - kCountWarps * 32 || last) {
+            // four rows per warp, eight lanes per row
+            const int sl = lane & 7;
+            for (int i0 = warp * 4; i0 < n; i0 += kCountWarps * 4) {
+                const int i = i0 + (lane >> 3);
+                const bool valid = i < n;
+                const int64_t r = valid ? q_rows[i] : 0;
+                const int inext = i + kCountWarps * 4;   // the group's next row, into L2
+                if (inext < n) {
+                    const int64_t pr = q_rows[inext];
+                    const char* zc = reinterpret_cast<const char*>(codes + pr * (int64_t)m_pad);
+                    const char* rc = reinterpret_cast<const char*>(resid + pr * rbytes);
+                    for (int off = sl * 128; off < m_pad; off += 8 * 128)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(zc + off));
+                    for (int off = sl * 128; off < rbytes; off += 8 * 128)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(rc + off));
+                    if (sl == 7) asm volatile("prefetch.global.L2 [%0];" ::"l"(rparam + pr));
+                }
+                int D1, D2;
+                resid_dots_group8(zqn, zqp, srq.bias, codes + r * (int64_t)m_pad,
+                                  resid + r * rbytes, m_pad, valid, &D1, &D2);
+                int open = 0;   // the row needs its fp32 row
+                if (valid && sl == 0) {
+                    float rl, rh;
+                    bool placed = false;
+                    if (resid_bounds(D1, D2, rparam[r], srq, qnorm, &rl, &rh)) {
+                        // RN(q.v) lies in [rl, rh] as q.v does; a score of
+                        // zero is reported as +0, whose key is above -0's
+                        const float rh0 = rh == 0.0f ? 0.0f : rh;
+                        const int a = keys_below(sk, nq, rank_key(rl, (uint32_t)r));
+                        const int b = keys_at_most(sk, nq, rank_key(rh0, (uint32_t)r));
+                        if (a == b) {
+                            placed = true;
+                            if (rh < lo[r] || rl > hi[r]) set_status(status, PVS_ERR_INTERVAL);
+                            atomicAdd(&sh[a], 1u);
+                        }
+                    }
+                    if (!placed) {
+                        f_rows[atomicAdd(&f_n, 1)] = (int32_t)r;
+                        open = 1;
+                    }
+                }
+                if (__shfl_sync(0xffffffffu, open, lane & ~7)) {   // its fp32 row, into L2
+                    const char* vr = reinterpret_cast<const char*>(raw + r * (int64_t)m_raw);
+                    for (int off = sl * 128; off < m_raw * 4; off += 8 * 128)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(vr + off));
+                }
+            }
+            __syncthreads();
+            const int nf = f_n;
+            for (int i = warp; i < nf; i += kCountWarps) {
+                const int64_t r = f_rows[i];
+                place_fp32(r, lo[r], hi[r]);
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) q_n = f_n = 0;
+            __syncthreads();
+        }
+        if (last) break;
     }
     __syncthreads();
     for (int i = threadIdx.x; i <= nq; i += blockDim.x) {
@@ -580,8 +968,20 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
         if (sparse_ids[i] < 0 || sparse_ids[i] >= rows) return PVS_ERR_INVALID;
     const uint32_t* tomb = sd->d_tomb;
     cudaStream_t st = c->stream;
-    cudaStream_t st2 = nullptr;
-    cudaEvent_t ev = nullptr;
+    // the second stream, its event and the pinned staging stay with the
+    // cursor (created at its first rank query, freed with its buffers)
+    if (!c->rq_stream || !c->rq_event || !c->rq_pinned) {
+        if ((!c->rq_stream &&
+             cudaStreamCreateWithFlags(&c->rq_stream, cudaStreamNonBlocking) != cudaSuccess) ||
+            (!c->rq_event &&
+             cudaEventCreateWithFlags(&c->rq_event, cudaEventDisableTiming) != cudaSuccess) ||
+            (!c->rq_pinned && cudaMallocHost(&c->rq_pinned, kRankQueryPinned) != cudaSuccess)) {
+            cudaGetLastError();
+            return PVS_ERR_CUDA;
+        }
+    }
+    cudaStream_t st2 = c->rq_stream;
+    cudaEvent_t ev = c->rq_event;
     std::vector<void*> held;
     auto alloc = [&](size_t bytes, cudaStream_t s) -> void* {
         void* p = nullptr;
@@ -593,11 +993,12 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
         held.push_back(p);
         return p;
     };
+    // st frees the scratch after whatever st2 still has queued, and ends
+    // every call joined (the next call's st2 work follows this call's st)
     auto cleanup = [&]() {
-        if (st2 && ev && cudaEventRecord(ev, st2) == cudaSuccess) cudaStreamWaitEvent(st, ev, 0);
+        if (cudaEventRecord(ev, st2) == cudaSuccess) cudaStreamWaitEvent(st, ev, 0);
         for (void* p : held) cudaFreeAsync(p, st);
-        if (ev) cudaEventDestroy(ev);
-        if (st2) cudaStreamDestroy(st2);
+        if (cudaEventRecord(ev, st) == cudaSuccess) cudaStreamWaitEvent(st2, ev, 0);
         cudaGetLastError();
     };
 #define RQ_CUDA(expr)                                              \
@@ -610,32 +1011,13 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
                                                    : PVS_ERR_CUDA; \
         }                                                          \
     } while (0)
-    if (cudaStreamCreateWithFlags(&st2, cudaStreamNonBlocking) != cudaSuccess ||
-        cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) {
-        cudaGetLastError();
-        cleanup();
-        return PVS_ERR_CUDA;
-    }
     // host staging: the queried ids in, the counts and ranks out (pinned,
-    // so the copies are asynchronous; freed after the final wait)
-    struct Pinned {
-        void* p = nullptr;
-        ~Pinned() {
-            if (p) cudaFreeHost(p);
-        }
-    } pin;
+    // so the copies are asynchronous; every use ends at this call's wait)
     const size_t id_bytes = (size_t)std::max(nd, 1) * 8 + (size_t)std::max(nsq, 1) * 4;
-    const size_t out_bytes = (size_t)(nd + 1) * 16 + (size_t)std::max(nd, 1) * 8 +
-                             (size_t)std::max(nsq, 1) * 4 + 2 * sizeof(int);
-    if (cudaMallocHost(&pin.p, id_bytes + out_bytes) != cudaSuccess) {
-        cudaGetLastError();
-        cleanup();
-        return PVS_ERR_OOM;
-    }
-    int64_t* h_dids = static_cast<int64_t*>(pin.p);
+    int64_t* h_dids = static_cast<int64_t*>(c->rq_pinned);
     int32_t* h_sids = reinterpret_cast<int32_t*>(h_dids + std::max(nd, 1));
     unsigned long long* h_hist =
-        reinterpret_cast<unsigned long long*>(static_cast<char*>(pin.p) + id_bytes);
+        reinterpret_cast<unsigned long long*>(static_cast<char*>(c->rq_pinned) + id_bytes);
     unsigned long long* h_maybe = h_hist + nd + 1;
     uint64_t* h_keys = reinterpret_cast<uint64_t*>(h_maybe + nd + 1);
     int32_t* h_srank = reinterpret_cast<int32_t*>(h_keys + std::max(nd, 1));
@@ -670,16 +1052,36 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
         count_launches(1);
         query_keys_kernel<<<1, kRankQueryMax, 0, st>>>(d_dids, d_score, nd, d_keys, status);
         RQ_CUDA(cudaGetLastError());
-        int grid = 0;
-        RQ_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&grid, rank_count_kernel,
-                                                              kCountWarps * 32, 0));
+        // the residual codes place most rows of an exact count without their fp32 row
+        const bool resid = exact && x->m_pad <= kResidMaxPad;
+        if (resid) {
+            const pvs_status rs = ensure_resid(x, st, status);
+            if (rs != PVS_OK) {
+                cleanup();
+                return rs;
+            }
+        }
+        static const int grid = [] {
+            int g = 0;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&g, rank_count_kernel,
+                                                              kCountWarps * 32, 0) != cudaSuccess) {
+                cudaGetLastError();
+                g = 1;
+            }
+            return g;
+        }();
         int64_t blocks = (int64_t)std::max(grid, 1) * std::max(x->num_sms, 1);
         blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, (rows + kCountWarps * 32 - 1) /
                                                                     (kCountWarps * 32)));
         count_launches(1);
-        rank_count_kernel<<<(unsigned)blocks, kCountWarps * 32, 0, st>>>(
+        // |zq_j| <= Q keeps sum |zq_j z_j| <= m_pad Q 127 below 2^31
+        const int qrange = (int)std::min<int64_t>(16383, ((int64_t(1) << 31) - 1) /
+                                                             (127 * (int64_t)x->m_pad));
+        rank_count_kernel<<<(unsigned)blocks, kCountWarps * 32,
+                            resid ? (size_t)x->m_pad * 4 : 0, st>>>(
             c->lo, c->hi, rows, tomb, c->qraw, x->raw, x->m_raw, d_keys, nd, exact ? 1 : 0,
-            d_hist, d_maybe, status, c->ctr);
+            resid ? x->codes : nullptr, resid ? x->resid : nullptr, x->rparam, x->m_pad, qrange,
+            c->qs, d_hist, d_maybe, status, c->ctr);
         RQ_CUDA(cudaGetLastError());
         RQ_CUDA(cudaMemcpyAsync(h_hist, d_hist, (size_t)(nd + 1) * 16, cudaMemcpyDeviceToHost,
                                 st));

@@ -128,6 +128,8 @@ pvs_status index_reserve(pvs_index* x, int64_t need) {
     dev_free(x->raw);
     dev_free(x->codes_bf16);   // rebuilt on demand at the new capacity
     x->bf16_rows = 0;
+    dev_free(x->resid), dev_free(x->rparam);   // likewise
+    x->resid_rows = 0;
     x->codes = codes, x->scale = scale, x->vnorm = vnorm, x->enorm = enorm, x->raw = raw;
     x->cap = cap;
     x->h_tomb.resize((size_t)(cap / 32), 0u);
@@ -210,6 +212,10 @@ void cursor_free_device(pvs_cursor* c) {
     if (c->h_scores) cudaFreeHost(c->h_scores);
     if (c->h_small) cudaFreeHost(c->h_small);
     c->h_ids = nullptr, c->h_scores = nullptr, c->h_small = nullptr;
+    if (c->rq_pinned) cudaFreeHost(c->rq_pinned);
+    if (c->rq_stream) cudaStreamDestroy(c->rq_stream);
+    if (c->rq_event) cudaEventDestroy(c->rq_event);
+    c->rq_pinned = nullptr, c->rq_stream = nullptr, c->rq_event = nullptr;
     if (c->ev_begin) cudaEventDestroy(c->ev_begin);
     if (c->ev_end) cudaEventDestroy(c->ev_end);
     if (c->ev_order) cudaEventDestroy(c->ev_order);
@@ -1335,6 +1341,8 @@ void pvs_index_free(pvs_index* x) {
     if (x->pass_done) cudaEventDestroy(x->pass_done);
     if (x->scratch_pool) cudaMemPoolDestroy(x->scratch_pool);
     if (x->bf16_ready) cudaEventDestroy(x->bf16_ready);
+    dev_free(x->resid), dev_free(x->rparam);
+    if (x->resid_ready) cudaEventDestroy(x->resid_ready);
     dev_free(x->norm_maxes);
     dev_free(x->gscale);
     if (x->own_stream && x->stream) cudaStreamDestroy(x->stream);

@@ -55,6 +55,17 @@ struct pvs_index {
     uint16_t* codes_bf16 = nullptr;         // [cap][m_pad]
     int64_t bf16_rows = 0;                  // rows converted so far
     cudaEvent_t bf16_ready = nullptr;       // end of the last conversion (any stream)
+    // 4-bit codes of each row's quantization residual, for the exact rank
+    // counts of the EAHR finish (built on demand, extended over appended
+    // rows): v = scale z + rscale z2 + r2 with ||r2|| <= rnorm, z2 in [-7, 7]
+    // stored as z2 + 8, two per byte (dims 8t + k: byte k / 2 of word t, the
+    // low nibble for even k); rparam[row] = (scale, rscale, rnorm, wnorm) with
+    // wnorm >= ||scale z + rscale z2||
+    uint8_t* resid = nullptr;               // [cap][m_pad / 2]
+    float4* rparam = nullptr;               // [cap]
+    int64_t resid_rows = 0;                 // rows coded so far
+    cudaEvent_t resid_ready = nullptr;      // end of the last residual build (any stream)
+    std::mutex resid_mutex;
     // max vnorm and max enorm (float bits) over every row; refreshed by build and
     // append (upper bounds for any snapshot), read by the batched pass
     unsigned int* norm_maxes = nullptr;
@@ -134,6 +145,11 @@ struct pvs_cursor {
     bool ahead_host = false;
     int32_t readahead = 4;            // a pull computes up to this many pages
     unsigned int* h_small = nullptr;  // pinned scratch (counts, status)
+    // rank queries (fusion.cu): pinned staging, a second stream and an
+    // event, kept between calls
+    void* rq_pinned = nullptr;
+    cudaStream_t rq_stream = nullptr;
+    cudaEvent_t rq_event = nullptr;
     // stats
     int64_t pulls = 0, interval_passes = 0, horizon_builds = 0, candidates = 0;
     int64_t code_bytes = 0;           // code + parameter bytes read for this cursor (a

@@ -246,3 +246,80 @@ def test_exact_count_near_equal_scores():
     _check(ids, F, T)
     assert st["complete"] == 3
     assert not np.isnan(F).any()
+
+
+def _tied_mid_sparse(dense_ids, pairs, rng):
+    """A sparse list whose first `pairs` items lie in the middle of the dense
+    ranking (B_k), with the dense top item A_k placed at B_k's dense rank:
+    F(A_k) = F(B_k) exactly, so only exact dense ranks of mid-distribution
+    scores order each pair (ties: smaller id first)."""
+    n = len(dense_ids)
+    mid = n // 2
+    B = dense_ids[mid - 5 * pairs:mid + 5 * pairs:10][:pairs]
+    A = dense_ids[:pairs]
+    rank = np.empty(int(dense_ids.max()) + 1, np.int64)
+    rank[dense_ids] = np.arange(1, n + 1)
+    S = np.full(n, -1, np.int64)
+    S[:pairs] = B
+    S[rank[B] - 1] = A
+    used = np.zeros(rank.shape[0], bool)
+    used[A] = used[B] = True
+    rest = dense_ids[~used[dense_ids]].copy()
+    rng.shuffle(rest)
+    S[S < 0] = rest
+    return S
+
+
+def test_exact_ranks_of_mid_scores_through_the_residual_codes():
+    """Exact dense ranks of items in the middle of the score distribution,
+    where a third of the rows' intervals straddle each score: the residual
+    codes place all but a few of those rows without their fp32 rows (the
+    refined count stays far below the straddlers), and the codes are
+    extended over rows appended after they were first built."""
+    rng = np.random.default_rng(350)
+    m, n0, n1 = 128, 50_000, 12_000
+    centres = synth.mixture_centres(64, m, seed=351, device="cpu")
+    V = synth.mixture_rows(n0, centres, 0.35, seed=352).numpy()
+    q = synth.mixture_queries(1, centres, 0.5, seed=353).numpy()[0]
+    pairs = 10
+    index = pvs.pvs_build(V)
+    try:
+        dense_ids, _ = po.dense_ranking(q, V)
+        S = _tied_mid_sparse(dense_ids, pairs, rng)
+        T = ro.target_topk_large([dense_ids, S], [1, 1], 60, 2 * pairs, ro.NUMERATOR)
+        assert T[0][1] == T[1][1]
+        cur = pvs.pvs_cursor_open(index, q)
+        try:
+            ids, F, st = pvs.eahr_topk(cur, S, K=2 * pairs, k=60, form=pvs.EAHR_NUMERATOR,
+                                       policy=pvs.EAHR_POLICY_ADAPTIVE)
+            refined = pvs.pvs_cursor_stats(cur)["refined"]
+        finally:
+            pvs.pvs_cursor_close(cur)
+        _check(ids, F, T)
+        assert st["complete"] == 3
+        assert not np.isnan(F).any()
+        assert refined < n0 // 8, refined
+        # rows near the middle scores appended after the codes were built,
+        # some rows deleted; a snapshot sees both
+        W = V[dense_ids[n0 // 2 - n1 // 2:n0 // 2 + n1 // 2]]
+        W = (W + 1e-3 * rng.standard_normal(W.shape)).astype(np.float32)
+        pvs.pvs_append(index, W)
+        U = np.concatenate([V, W])
+        dead = rng.choice(n0 + n1, 2_000, replace=False)
+        pvs.pvs_tombstone(index, dead)
+        visible = np.ones(n0 + n1, bool)
+        visible[dead] = False
+        snap = pvs.pvs_snapshot_create(index)
+        try:
+            dense_ids, _ = po.dense_ranking(q, U, visible=visible)
+            S = _tied_mid_sparse(dense_ids, pairs, rng)
+            T = ro.target_topk_large([dense_ids, S], [1, 1], 60, 2 * pairs, ro.NUMERATOR)
+            ids, F, st = _run(index, q, S, snap=snap, step=0, K=2 * pairs, k=60,
+                              form=pvs.EAHR_NUMERATOR)
+            _check(ids, F, T)
+            assert st["complete"] == 3
+            assert not np.isnan(F).any()
+        finally:
+            pvs.pvs_snapshot_free(snap)
+    finally:
+        pvs.pvs_index_free(index)
