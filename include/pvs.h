@@ -422,7 +422,13 @@ enum {
                                     around the scores of the candidates
                                     whose intervals overlap are scored and
                                     their ranks made exact (a few rounds,
-                                    then every candidate's).  An F known only as an
+                                    then every candidate's); the first such
+                                    count gives the index 4-bit codes of
+                                    each row's quantization residual
+                                    (m_pad / 2 + 16 bytes per row, kept and
+                                    extended over appended rows), whose
+                                    tighter intervals place most of those
+                                    rows without their fp32 rows.  An F known only as an
                                     interval is reported as NaN (its
                                     position is certified).  Failing that
                                     (too many candidates,
