@@ -359,7 +359,9 @@ pvs_status ensure_resid(pvs_index* x, cudaStream_t st, int* status) {
 // keeps every integer dot product below 2^31), zq as 16-bit pairs twice,
 // in dimension order (for the int8 codes) and in the residual codes' nibble
 // order (dims 8t + 0, 2, 4, 6, 1, 3, 5, 7: the pairs (0,2) (4,6) of the low
-// nibbles, (1,3) (5,7) of the high ones), eq >= ||e_q|| and bias = sum zq_j.
+// nibbles, (1,3) (5,7) of the high ones), each as 16-byte slots: the first
+// half of every 16-dim chunk, then the second halves; eq >= ||e_q|| and
+// bias = sum zq_j.
 struct ResidQuery {
     float sq, eq;
     int bias;
@@ -397,8 +399,8 @@ __device__ __forceinline__ void resid_dots_group8(const int32_t* __restrict__ zq
             for (int u = 0; u < 3; ++u) {
                 const int c = c0 + 8 * u;
                 if (c >= n16) break;
-                const int4 n0 = qn[2 * c], n1 = qn[2 * c + 1];
-                const int4 p0 = qp[2 * c], p1 = qp[2 * c + 1];
+                const int4 n0 = qn[c], n1 = qn[n16 + c];
+                const int4 p0 = qp[c], p1 = qp[n16 + c];
                 acc1 = __dp2a_lo(n0.x, (int)a[u].x, acc1);
                 acc1 = __dp2a_hi(n0.y, (int)a[u].x, acc1);
                 acc1 = __dp2a_lo(n0.z, (int)a[u].y, acc1);
@@ -513,8 +515,8 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
             sq = __fdiv_rn(mq, Qf);
             if (sq == 0.0f) sq = __uint_as_float(1u);   // 2^-149
         }
-        int16_t* n16 = reinterpret_cast<int16_t*>(zqn);
-        int16_t* p16 = reinterpret_cast<int16_t*>(zqp);
+        int16_t* zn16 = reinterpret_cast<int16_t*>(zqn);
+        int16_t* zp16 = reinterpret_cast<int16_t*>(zqp);
         float ss = 0.0f;
         int bias = 0;
         for (int j = threadIdx.x; j < m_pad; j += blockDim.x) {
@@ -526,9 +528,12 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
             } else if (j < m_raw) {
                 ss = __fadd_ru(ss, __fmul_ru(qraw[j], qraw[j]));
             }
-            const int k = j & 7;
-            n16[j] = (int16_t)c;
-            p16[(j & ~7) + ((k & 1) ? 4 + (k >> 1) : (k >> 1))] = (int16_t)c;
+            // half h of chunk j / 16 (dims 8h .. 8h + 7 of the chunk) sits at
+            // 16-byte slot h * (m_pad / 16) + j / 16, so that the eight lanes of a group
+            // read consecutive slots
+            const int k = j & 7, slot = ((j >> 3) & 1) * (m_pad >> 4) + (j >> 4);
+            zn16[slot * 8 + k] = (int16_t)c;
+            zp16[slot * 8 + ((k & 1) ? 4 + (k >> 1) : (k >> 1))] = (int16_t)c;
             bias += c;
         }
 #pragma unroll
