@@ -162,9 +162,12 @@ __device__ __forceinline__ int keys_at_most(const uint64_t* k, int n, uint64_t x
 }
 
 constexpr int kCountWarps = 8;
-// Straddling rows a block queues for the residual level (and for the fp32
-// rows after it), flushed before a tile of kCountWarps * 32 rows could overflow.
+// Rows a block classifies per step (four per lane), and the straddling rows
+// it queues for the residual level (and for the fp32 rows after it), flushed
+// before a tile could overflow the queue.
+constexpr int kCountTile = kCountWarps * 32 * 4;
 constexpr int kPlaceQueue = 2048;
+static_assert(kPlaceQueue >= 2 * kCountTile, "queue");
 
 // Pinned staging of one rank query: ids in (8 B dense, 4 B sparse), per dense
 // item two 8-byte counts (plus one) and its key, per sparse item its rank,
@@ -485,7 +488,7 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
     }
     __syncthreads();
     const int lane = threadIdx.x & 31;
-    const int64_t step = (int64_t)gridDim.x * kCountWarps * 32;
+    const int64_t step = (int64_t)gridDim.x * kCountTile;
     unsigned long long scored = 0, fallbacks = 0;
     // the query's integer form for the residual level (every block computes
     // the same): s_q = RN(max |q_j| / Q), zq_j = clip(rint(RN(q_j / s_q)),
@@ -600,53 +603,95 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
     __shared__ int q_n, f_n;
     if (threadIdx.x == 0) q_n = f_n = 0;
     __syncthreads();
-    for (int64_t tb = (int64_t)blockIdx.x * kCountWarps * 32;; tb += step) {
-        const int64_t base = tb + warp * 32;
+    // a block tile: kCountWarps warps x 32 lanes x 4 consecutive rows, the
+    // bounds read as float4 (scalars at a ragged end or unaligned buffers)
+    const bool vec_ok = ((reinterpret_cast<uintptr_t>(lo) | reinterpret_cast<uintptr_t>(hi)) & 15) == 0;
+    const unsigned int lanemask_lt = (1u << lane) - 1u;
+    for (int64_t tb = (int64_t)blockIdx.x * kCountTile;; tb += step) {
+        const int64_t base = tb + (int64_t)warp * 32 * 4;
         if (base < rows) {
-            const int64_t y = base + lane;
-            int bin = -1;   // -1: nothing to count from the bounds
-            bool straddle = false;
-            float l = 0.f, h = 0.f;
-            if (y < rows && !tombstoned(tomb, y)) {
-                l = lo[y];
-                h = hi[y];
-                if (h == -INFINITY) {
-                    bin = nq;
-                } else {
-                    const int a = keys_below(sk, nq, rank_key(l, (uint32_t)y));
-                    const int b = keys_at_most(sk, nq, rank_key(h, (uint32_t)y));
-                    if (a == b) {
-                        bin = a;
-                    } else if (exact) {
-                        straddle = true;
+            const int64_t y0 = base + 4 * lane;
+            float lv[4] = {0.f, 0.f, 0.f, 0.f}, hv[4] = {0.f, 0.f, 0.f, 0.f};
+            if (vec_ok && y0 + 3 < rows) {
+                const float4 L = *reinterpret_cast<const float4*>(lo + y0);
+                const float4 H = *reinterpret_cast<const float4*>(hi + y0);
+                lv[0] = L.x, lv[1] = L.y, lv[2] = L.z, lv[3] = L.w;
+                hv[0] = H.x, hv[1] = H.y, hv[2] = H.z, hv[3] = H.w;
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (y0 + u < rows) {
+                        lv[u] = lo[y0 + u];
+                        hv[u] = hi[y0 + u];
+                    }
+            }
+            // the four rows share one tombstone word
+            const uint32_t tw = (tomb && y0 < rows) ? tomb[y0 >> 5] >> (y0 & 31) : 0u;
+            unsigned int strad[4] = {0u, 0u, 0u, 0u};   // straddling lanes per row slot
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t y = y0 + u;
+                const float l = lv[u], h = hv[u];
+                int bin = -1;   // -1: nothing to count from the bounds
+                int mb = -1;    // bounds mode: the row may lie above keys bin .. mb - 1
+                bool straddle = false;
+                if (y < rows && !((tw >> u) & 1u)) {
+                    if (h == -INFINITY) {
+                        bin = nq;
                     } else {
-                        bin = a;
-                        atomicAdd(&sm[a], 1);
-                        atomicAdd(&sm[b], -1);
+                        const int a = keys_below(sk, nq, rank_key(l, (uint32_t)y));
+                        const int b = keys_at_most(sk, nq, rank_key(h, (uint32_t)y));
+                        if (a == b) {
+                            bin = a;
+                        } else if (exact) {
+                            straddle = true;
+                        } else {
+                            bin = a;
+                            mb = b;
+                        }
                     }
                 }
+                // one shared-memory add per distinct bin of the warp
+                const unsigned int live = __ballot_sync(0xffffffffu, bin >= 0);
+                if (bin >= 0) {
+                    const unsigned int same = __match_any_sync(live, bin);
+                    if (lane == __ffs(same) - 1) atomicAdd(&sh[bin], (unsigned int)__popc(same));
+                }
+                // bounds mode: maybe[a] += 1, maybe[b] -= 1, per distinct key of the warp
+                const unsigned int mlive = __ballot_sync(0xffffffffu, mb >= 0);
+                if (mb >= 0) {
+                    const unsigned int sa = __match_any_sync(mlive, bin);
+                    if (lane == __ffs(sa) - 1) atomicAdd(&sm[bin], __popc(sa));
+                    const unsigned int sb = __match_any_sync(mlive, mb);
+                    if (lane == __ffs(sb) - 1) atomicAdd(&sm[mb], -__popc(sb));
+                }
+                const unsigned int todo = __ballot_sync(0xffffffffu, straddle);
+                if (use_resid) {   // one queue reservation per warp
+                    if (todo) {
+                        int qb = 0;
+                        if (lane == __ffs(todo) - 1) qb = atomicAdd(&q_n, __popc(todo));
+                        qb = __shfl_sync(0xffffffffu, qb, __ffs(todo) - 1);
+                        if (straddle) q_rows[qb + __popc(todo & lanemask_lt)] = (int32_t)y;
+                    }
+                } else {
+                    strad[u] = todo;
+                }
             }
-            // one shared-memory add per distinct bin of the warp
-            const unsigned int live = __ballot_sync(0xffffffffu, bin >= 0);
-            if (bin >= 0) {
-                const unsigned int same = __match_any_sync(live, bin);
-                if (lane == __ffs(same) - 1) atomicAdd(&sh[bin], (unsigned int)__popc(same));
-            }
-            if (use_resid) {
-                if (straddle) q_rows[atomicAdd(&q_n, 1)] = (int32_t)y;
-            } else {
-                unsigned int todo = __ballot_sync(0xffffffffu, straddle);
-                while (todo) {
-                    const int src = __ffs(todo) - 1;
-                    todo &= todo - 1;
-                    if (todo) {   // the next row to score, into L2 while this one is scored
+            // without the residual codes, each straddling row from its fp32 row
+#pragma unroll 1
+            for (int u = 0; u < 4 && !use_resid; ++u) {
+                unsigned int rest = strad[u];
+                while (rest) {
+                    const int src = __ffs(rest) - 1;
+                    rest &= rest - 1;
+                    if (rest) {   // the next row to score, into L2 while this one is scored
                         const char* nrow = reinterpret_cast<const char*>(
-                            raw + (base + __ffs(todo) - 1) * (int64_t)m_raw);
+                            raw + (base + 4 * (__ffs(rest) - 1) + u) * (int64_t)m_raw);
                         for (int off = lane * 128; off < m_raw * 4; off += 32 * 128)
                             asm volatile("prefetch.global.L2 [%0];" ::"l"(nrow + off));
                     }
-                    place_fp32(base + src, __shfl_sync(0xffffffffu, l, src),
-                               __shfl_sync(0xffffffffu, h, src));
+                    const int64_t r = base + 4 * src + u;
+                    place_fp32(r, lo[r], hi[r]);
                 }
             }
         }
@@ -657,7 +702,7 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
         }
         __syncthreads();
         const int n = q_n;
-        if (n > kPlaceQueue - kCountWarps * 32 || last) {
+        if (n > kPlaceQueue - kCountTile || last) {
             // four rows per warp, eight lanes per row
             const int sl = lane & 7;
             for (int i0 = warp * 4; i0 < n; i0 += kCountWarps * 4) {
@@ -1076,8 +1121,7 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
             return g;
         }();
         int64_t blocks = (int64_t)std::max(grid, 1) * std::max(x->num_sms, 1);
-        blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, (rows + kCountWarps * 32 - 1) /
-                                                                    (kCountWarps * 32)));
+        blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, (rows + kCountTile - 1) / kCountTile));
         count_launches(1);
         // |zq_j| <= Q keeps sum |zq_j z_j| <= m_pad Q 127 below 2^31
         const int qrange = (int)std::min<int64_t>(16383, ((int64_t(1) << 31) - 1) /
