@@ -538,8 +538,84 @@ __global__ void __launch_bounds__(1024) bitonic_desc_kernel(uint64_t* keys, int 
     for (int i = threadIdx.x; i < count; i += blockDim.x) keys[i] = sk[i];
 }
 
+// The same network for at most 1024 E keys with E per thread in registers
+// (thread t holds positions tE .. tE + E - 1): a stride below E is a swap
+// within a thread, below 32 E a shuffle within a warp, and only the larger
+// strides go through shared memory (15 of the 78 stages at 4,096 keys).
+template <int E>
+__device__ __forceinline__ void bitonic_keep(uint64_t& v, uint64_t w, int i, int j, int size) {
+    const bool desc = (i & size) == 0;
+    const bool keep_max = (i < j) == desc;
+    v = keep_max ? (v > w ? v : w) : (v < w ? v : w);
+}
+
+template <int E>
+__global__ void __launch_bounds__(1024) bitonic_desc_reg_kernel(uint64_t* keys, int count) {
+    __shared__ uint64_t sk[1024 * E];
+    const int t = threadIdx.x;
+    constexpr int n = 1024 * E;
+    uint64_t v[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int i = t * E + e;
+        v[e] = i < count ? keys[i] : 0ull;
+    }
+    for (int size = 2; size <= n; size <<= 1) {
+        for (int s = size >> 1; s > 0; s >>= 1) {
+            if (s >= 32 * E) {   // another warp's element
+#pragma unroll
+                for (int e = 0; e < E; ++e) sk[t * E + e] = v[e];
+                __syncthreads();
+#pragma unroll
+                for (int e = 0; e < E; ++e) {
+                    const int i = t * E + e;
+                    bitonic_keep<E>(v[e], sk[i ^ s], i, i ^ s, size);
+                }
+                __syncthreads();
+            } else if (s >= E) {   // another lane's element
+#pragma unroll
+                for (int e = 0; e < E; ++e) {
+                    const int i = t * E + e;
+                    const uint64_t w = __shfl_xor_sync(0xffffffffu, v[e], s / E);
+                    bitonic_keep<E>(v[e], w, i, i ^ s, size);
+                }
+            } else {   // this thread's element: s is 1 or 2 (E = 2 or 4)
+                auto ex = [&](uint64_t& a, uint64_t& b, int e) {
+                    const bool desc = ((t * E + e) & size) == 0;
+                    const bool swap = (a < b) == desc;
+                    const uint64_t x = a;
+                    a = swap ? b : a;
+                    b = swap ? x : b;
+                };
+                if (E >= 2 && s == 1) {
+                    ex(v[0], v[E >= 2 ? 1 : 0], 0);
+                    if (E == 4) ex(v[E == 4 ? 2 : 0], v[E == 4 ? 3 : 0], 2);
+                } else if (E == 4 && s == 2) {
+                    ex(v[0], v[E == 4 ? 2 : 0], 0);
+                    ex(v[E == 4 ? 1 : 0], v[E == 4 ? 3 : 0], 1);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        const int i = t * E + e;
+        if (i < count) keys[i] = v[e];
+    }
+}
+
 cudaError_t launch_bitonic_desc(uint64_t* keys, int count, cudaStream_t st) {
     if (count <= 1) return cudaSuccess;
+    if (count <= 4096) {
+        count_launches(1);
+        if (count <= 1024)
+            bitonic_desc_reg_kernel<1><<<1, 1024, 0, st>>>(keys, count);
+        else if (count <= 2048)
+            bitonic_desc_reg_kernel<2><<<1, 1024, 0, st>>>(keys, count);
+        else
+            bitonic_desc_reg_kernel<4><<<1, 1024, 0, st>>>(keys, count);
+        return cudaGetLastError();
+    }
     int pow2 = 2;
     while (pow2 < count) pow2 <<= 1;
     const size_t smem = (size_t)pow2 * sizeof(uint64_t);
