@@ -396,10 +396,21 @@ class Driver {
         } catch (...) {   // no thread: a host list is copied by the finish itself
         }
     }
-    // The staged list once it is queued (null when staging failed).
-    const pvs::StagedList* staged_list() {
+    void join_stage() {
         if (stage_live) stage.join();
         stage_live = false;
+    }
+    // The check of a staged host list, queued once the dense list's first
+    // pull (and its interval pass) is done, so that it does not run beside
+    // the pass.
+    void check_stage() {
+        join_stage();
+        if (stage_status == PVS_OK && staged && !staged->checked)
+            stage_status = pvs::check_staged_list(staged);
+    }
+    // The staged list once it is queued and checked (null when staging failed).
+    const pvs::StagedList* staged_list() {
+        check_stage();
         return stage_status == PVS_OK ? staged : nullptr;
     }
 
@@ -410,7 +421,7 @@ class Driver {
     // clear those, or whole arrays when that is cheaper, and pool them.
     ~Driver() {
         join_ahead();
-        staged_list();
+        join_stage();
         pvs::free_staged_list(staged);
         if (!ws.ranks) return;
         if ((int64_t)(prefix[0].size() + prefix[1].size()) > ws.cap / 8) {
@@ -1101,6 +1112,7 @@ pvs_status run_driver(Driver& d, const eahr_params* p, int64_t* out_ids, double*
                 pvs_status s = d.pull(pick, size[pick]);
                 if (s < 0) return s;
                 size[pick] = std::min<int64_t>(2 * size[pick], (int64_t)1 << 24);
+                if (adaptive && pick == 0) d.check_stage();
             }
             // long dense pulls: the next one starts now, beside certification
             // and the other list's pull (ranks read ahead change no result)

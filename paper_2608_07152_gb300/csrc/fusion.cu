@@ -779,6 +779,46 @@ __global__ void gather_ranks_kernel(const int32_t* __restrict__ rank_of,
     if (i < n) out[i] = rank_of[ids[i]];
 }
 
+// Every id of a sparse list: inside the snapshot, not deleted, not repeated
+// (one bit per id in `seen`, zeroed before; the second setter of a bit finds
+// it set).  The verdict goes to *status.
+__global__ void list_check_kernel(const int64_t* __restrict__ ids, int64_t n, int64_t rows,
+                                  const uint32_t* __restrict__ tomb, uint32_t* seen, int* status) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int64_t x = ids[i];
+        if (x < 0 || x >= rows || tombstoned(tomb, x)) {
+            set_status(status, PVS_ERR_INVALID);
+            continue;
+        }
+        const uint32_t bit = 1u << (x & 31);
+        if (atomicOr(&seen[x >> 5], bit) & bit) set_status(status, PVS_ERR_INVALID);
+    }
+}
+
+// out[k] = position + 1 of q[k] in the list (0: absent), q ascending and
+// distinct (nq <= kRankQueryMax), one pass over the list.
+__global__ void list_find_kernel(const int64_t* __restrict__ ids, int64_t n,
+                                 const int32_t* __restrict__ q, int nq, int32_t* out) {
+    __shared__ int32_t sq[kRankQueryMax];
+    for (int i = threadIdx.x; i < nq; i += blockDim.x) sq[i] = q[i];
+    __syncthreads();
+    if (nq == 0) return;
+    const int64_t qlo = sq[0], qhi = sq[nq - 1];
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int64_t x = ids[i];
+        if (x < qlo || x > qhi) continue;
+        int lo = 0, hi = nq - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (sq[mid] < x) lo = mid + 1;
+            else hi = mid;
+        }
+        if (sq[lo] == x) out[lo] = (int32_t)(i + 1);
+    }
+}
+
 }  // namespace
 
 pvs_status fuse_complete(pvs_cursor* c, const int64_t* sparse, int64_t ns, const FuseWeights& w,
@@ -925,6 +965,7 @@ void free_staged_list(StagedList* s) {
     if (s->stream) {
         if (s->rank_of) cudaFreeAsync(s->rank_of, s->stream);
         if (s->list) cudaFreeAsync(s->list, s->stream);
+        if (s->seen) cudaFreeAsync(s->seen, s->stream);
         if (s->status) cudaFreeAsync(s->status, s->stream);
         cudaStreamSynchronize(s->stream);
         cudaStreamDestroy(s->stream);
@@ -957,30 +998,52 @@ pvs_status stage_sparse_list(pvs_cursor* c, const int64_t* sparse, int64_t ns,
     };
     cudaError_t e = cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&s->ready, cudaEventDisableTiming);
-    if (e == cudaSuccess)
-        e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->rank_of), rows * 4,
-                                    x->scratch_pool, s->stream);
+    // the ids on the device and their check (a bit per id: 1.1 MB at 8.8M
+    // rows, held in L2); the finish then finds its few ids in one pass over
+    // the list, so no table of every item's rank is written beside the
+    // interval pass
+    const size_t words = rows / 32 + 1;
     if (e == cudaSuccess)
         e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->list),
                                     (size_t)std::max<int64_t>(ns, 1) * 8, x->scratch_pool,
                                     s->stream);
     if (e == cudaSuccess)
+        e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->seen), words * 4,
+                                    x->scratch_pool, s->stream);
+    if (e == cudaSuccess)
         e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&s->status), sizeof(int),
                                     x->scratch_pool, s->stream);
-    if (e == cudaSuccess) e = cudaMemsetAsync(s->rank_of, 0, rows * 4, s->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(s->seen, 0, words * 4, s->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(s->status, 0, sizeof(int), s->stream);
     if (e == cudaSuccess && ns > 0)
         e = cudaMemcpyAsync(s->list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice, s->stream);
     if (e != cudaSuccess) return failed(e);
-    if (ns > 0) {
+    s->tomb = tomb;
+    s->n = ns;
+    s->checked = false;   // check_staged_list queues the check
+    *out = s;
+    return PVS_OK;
+}
+
+pvs_status check_staged_list(StagedList* s) {
+    if (!s || s->checked) return PVS_OK;
+    s->checked = true;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (s->index && prev != s->index->device) cudaSetDevice(s->index->device);
+    cudaError_t e = cudaSuccess;
+    if (s->n > 0) {
         count_launches(1);
-        list_rank_kernel<<<grid_of(ns), 256, 0, s->stream>>>(s->list, ns, s->rows, tomb,
-                                                             s->rank_of, s->status);
+        list_check_kernel<<<grid_of(s->n), 256, 0, s->stream>>>(s->list, s->n, s->rows, s->tomb,
+                                                                s->seen, s->status);
         e = cudaGetLastError();
     }
     if (e == cudaSuccess) e = cudaEventRecord(s->ready, s->stream);
-    if (e != cudaSuccess) return failed(e);
-    *out = s;
+    if (s->index && prev >= 0 && prev != s->index->device) cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return PVS_ERR_CUDA;
+    }
     return PVS_OK;
 }
 
@@ -1136,45 +1199,76 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
                                 st));
         RQ_CUDA(cudaMemcpyAsync(h_keys, d_keys, (size_t)nd * 8, cudaMemcpyDeviceToHost, st));
     }
-    // sparse: scatter the list, read the queried ids (second stream; a copy
-    // from pageable memory may hold this thread until it is done, so the
-    // dense work is queued first)
+    // sparse (second stream; a copy from pageable memory may hold this thread
+    // until it is done, so the dense work is queued first): a PBM ranking's
+    // table read at the queried ids, or one pass over a host list (staged
+    // ahead, or copied and checked here) that finds the queried ids, sorted
+    // and without repeats
     int32_t* d_srank = nullptr;
+    std::vector<int32_t> uniq, slot_of;   // distinct queried ids ascending; each query's slot
     if (nsq > 0 && staged && staged->rows != rows) {
         cleanup();
         return PVS_ERR_INVALID;
     }
     if (nsq > 0) {
-        const bool own = staged == nullptr;
-        int32_t* rank_of =
-            own ? static_cast<int32_t*>(alloc((size_t)std::max<int64_t>(rows, 1) * 4, st2))
-                : staged->rank_of;
-        int64_t* d_list =
-            own ? static_cast<int64_t*>(alloc((size_t)std::max<int64_t>(ns, 1) * 8, st2))
-                : staged->list;
-        int32_t* d_sids = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
-        d_srank = static_cast<int32_t*>(alloc((size_t)nsq * 4, st2));
-        if (!rank_of || (own && !d_list) || !d_sids || !d_srank) {
+        const bool table = staged && staged->rank_of;
+        int nfind = nsq;
+        if (!table) {
+            uniq.assign(sparse_ids, sparse_ids + nsq);
+            std::sort(uniq.begin(), uniq.end());
+            uniq.erase(std::unique(uniq.begin(), uniq.end()), uniq.end());
+            slot_of.resize((size_t)nsq);
+            for (int32_t i = 0; i < nsq; ++i)
+                slot_of[(size_t)i] = (int32_t)(std::lower_bound(uniq.begin(), uniq.end(),
+                                                                sparse_ids[i]) -
+                                               uniq.begin());
+            nfind = (int)uniq.size();
+            std::copy(uniq.begin(), uniq.end(), h_sids);
+        }
+        int32_t* d_sids = static_cast<int32_t*>(alloc((size_t)nfind * 4, st2));
+        d_srank = static_cast<int32_t*>(alloc((size_t)nfind * 4, st2));
+        int64_t* d_list = staged ? staged->list : nullptr;
+        if (!staged) {   // the host list, copied and checked by this call
+            const size_t words = (size_t)std::max<int64_t>(rows, 1) / 32 + 1;
+            d_list = static_cast<int64_t*>(alloc((size_t)std::max<int64_t>(ns, 1) * 8, st2));
+            uint32_t* seen = static_cast<uint32_t*>(alloc(words * 4, st2));
+            if (!d_list || !seen) {
+                cleanup();
+                return PVS_ERR_OOM;
+            }
+            RQ_CUDA(cudaMemsetAsync(seen, 0, words * 4, st2));
+            if (ns > 0) {
+                RQ_CUDA(cudaMemcpyAsync(d_list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice,
+                                        st2));
+                count_launches(1);
+                list_check_kernel<<<grid_of(ns), 256, 0, st2>>>(d_list, ns, rows, tomb, seen,
+                                                                status + 1);
+                RQ_CUDA(cudaGetLastError());
+            }
+        }
+        if (!d_sids || !d_srank || (!table && ns > 0 && !d_list)) {
             cleanup();
             return PVS_ERR_OOM;
         }
-        if (own) RQ_CUDA(cudaMemsetAsync(rank_of, 0, (size_t)std::max<int64_t>(rows, 1) * 4, st2));
-        RQ_CUDA(cudaMemcpyAsync(d_sids, h_sids, (size_t)nsq * 4, cudaMemcpyHostToDevice, st2));
-        if (!own) {   // scattered already: its verdict becomes this call's
+        RQ_CUDA(cudaMemcpyAsync(d_sids, h_sids, (size_t)nfind * 4, cudaMemcpyHostToDevice, st2));
+        if (staged) {   // staged ahead: its verdict becomes this call's
             RQ_CUDA(cudaStreamWaitEvent(st2, staged->ready, 0));
             RQ_CUDA(cudaMemcpyAsync(status + 1, staged->status, sizeof(int),
                                     cudaMemcpyDeviceToDevice, st2));
-        } else if (ns > 0) {
-            RQ_CUDA(cudaMemcpyAsync(d_list, sparse, (size_t)ns * 8, cudaMemcpyHostToDevice, st2));
-            count_launches(1);
-            list_rank_kernel<<<grid_of(ns), 256, 0, st2>>>(d_list, ns, rows, tomb, rank_of,
-                                                           status + 1);
-            RQ_CUDA(cudaGetLastError());
         }
-        count_launches(1);
-        gather_ranks_kernel<<<(nsq + 255) / 256, 256, 0, st2>>>(rank_of, d_sids, nsq, d_srank);
+        if (table) {
+            count_launches(1);
+            gather_ranks_kernel<<<(nsq + 255) / 256, 256, 0, st2>>>(staged->rank_of, d_sids, nsq,
+                                                                    d_srank);
+        } else {
+            const int64_t n_list = staged ? std::max<int64_t>(ns, 0) : ns;
+            RQ_CUDA(cudaMemsetAsync(d_srank, 0, (size_t)nfind * 4, st2));
+            count_launches(1);
+            list_find_kernel<<<grid_of(n_list), 256, 0, st2>>>(d_list, n_list, d_sids, nfind,
+                                                               d_srank);
+        }
         RQ_CUDA(cudaGetLastError());
-        RQ_CUDA(cudaMemcpyAsync(h_srank, d_srank, (size_t)nsq * 4, cudaMemcpyDeviceToHost, st2));
+        RQ_CUDA(cudaMemcpyAsync(h_srank, d_srank, (size_t)nfind * 4, cudaMemcpyDeviceToHost, st2));
     }
     RQ_CUDA(cudaEventRecord(ev, st2));
     RQ_CUDA(cudaStreamWaitEvent(st, ev, 0));
@@ -1212,7 +1306,8 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
             dense_lo[i] = it->lo;
             dense_hi[i] = it->hi;
         }
-        for (int32_t i = 0; i < nsq; ++i) sparse_rank[i] = h_srank[i];
+        for (int32_t i = 0; i < nsq; ++i)
+            sparse_rank[i] = slot_of.empty() ? h_srank[i] : h_srank[slot_of[(size_t)i]];
     }
     cleanup();
 #undef RQ_CUDA

@@ -212,22 +212,32 @@ pvs_status fuse_complete(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
 // outside the snapshot, deleted or repeated), PVS_ERR_INTERVAL (an exact
 // score outside its interval), PVS_ERR_OVERFLOW, PVS_ERR_OOM, PVS_ERR_CUDA.
 constexpr int32_t kRankQueryMax = 1024;
-// A host sparse list scattered on the device ahead of need: rank_of[x] =
-// position + 1 of id x (0: not in the list), its ids checked as in
-// fuse_complete (the verdict is read when the ranks are used).  Built on its
-// own stream by stage_sparse_list (which may hold the calling thread while
-// the pageable list is copied); rank_queries orders its reads after it.
+// A sparse list on the device ahead of need.  From a host list
+// (stage_sparse_list): the ids copied, and checked as in fuse_complete (the
+// verdict is read when the ranks are used); rank_queries finds its ids in the
+// list.  From a PBM query (pbm_stage_ranks): rank_of[x] = position + 1 of id
+// x (0: not in the list).  Built on its own stream (stage_sparse_list may hold
+// the calling thread while the pageable list is copied); rank_queries orders
+// its reads after it.
 struct StagedList {
     pvs_index* index = nullptr;       // device and scratch pool
     cudaStream_t stream = nullptr;
     cudaEvent_t ready = nullptr;      // recorded after the scatter
-    int32_t* rank_of = nullptr;       // [rows]
+    int32_t* rank_of = nullptr;       // [rows], or null: look the ids up in `list`
     int64_t* list = nullptr;          // the list's ids on the device (or null)
+    uint32_t* seen = nullptr;         // a bit per id, set by the check of `list`
+    const uint32_t* tomb = nullptr;   // the snapshot's deletions, for the check
+    int64_t n = 0;                    // ids in `list`
+    bool checked = true;              // the check of `list` is queued
     int* status = nullptr;            // the scatter's verdict on the ids
     int64_t rows = 0;
 };
 pvs_status stage_sparse_list(pvs_cursor* dense, const int64_t* sparse, int64_t ns,
                              StagedList** out);
+// Queue the check of a list staged by stage_sparse_list (once; `ready` then
+// marks its end).  Kept apart so that its kernel need not run beside the
+// dense list's interval pass.
+pvs_status check_staged_list(StagedList* s);
 // The complete ranking of a PBM cursor's query (U_s = the visible items with
 // S > 0, by (S desc, id asc), S evaluated as the PBM kernels do, App. A.2)
 // staged the same way (pbm_capi.cu); scratch from pool_owner's pool.
