@@ -464,8 +464,9 @@ __device__ __forceinline__ bool resid_bounds(int D1, int D2, const float4 rp,
 // [key(lo, y), key(hi, y)]; when no queried key falls in that range the
 // count is fixed by the bounds.  Otherwise, with `exact`, the row's
 // authoritative score is placed: first by the bounds of its residual codes
-// (resid_dot_warp, 1.5 B per dimension), else by the fp32 dot with its error
-// bound, else exactly (and it must lie in its interval, App. A.1);
+// (resid_dots_group8 and resid_bounds, 1.5 B per dimension; the block queues
+// such rows and places them eight lanes per row), else by the fp32 dot with
+// its error bound, else exactly (and it must lie in its interval, App. A.1);
 // without, the row counts in hist[a] (a = the queried keys below key(lo, y):
 // it is surely above those) and may lie above the keys a .. b-1 (b = the
 // keys at most key(hi, y)): maybe[a] += 1, maybe[b] -= 1, so that the prefix
@@ -477,7 +478,8 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
     const float* __restrict__ raw, int m_raw, const uint64_t* __restrict__ qkeys, int nq, int exact,
     const int8_t* __restrict__ codes, const uint8_t* __restrict__ resid,
     const float4* __restrict__ rparam, int m_pad, int qrange,
-    const QueryScalars* __restrict__ qs, unsigned long long* hist, unsigned long long* maybe, int* status, DevCounters* ctr) {
+    const QueryScalars* __restrict__ qs, unsigned long long* hist, unsigned long long* maybe,
+    int* status, DevCounters* ctr) {
     __shared__ uint64_t sk[kRankQueryMax];
     __shared__ unsigned int sh[kRankQueryMax + 1];
     __shared__ int sm[kRankQueryMax + 1];
@@ -532,8 +534,8 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
                 ss = __fadd_ru(ss, __fmul_ru(qraw[j], qraw[j]));
             }
             // half h of chunk j / 16 (dims 8h .. 8h + 7 of the chunk) sits at
-            // 16-byte slot h * (m_pad / 16) + j / 16, so that the eight lanes of a group
-            // read consecutive slots
+            // 16-byte slot h * (m_pad / 16) + j / 16, so that the eight lanes
+            // of a group read consecutive slots
             const int k = j & 7, slot = ((j >> 3) & 1) * (m_pad >> 4) + (j >> 4);
             zn16[slot * 8 + k] = (int16_t)c;
             zp16[slot * 8 + ((k & 1) ? 4 + (k >> 1) : (k >> 1))] = (int16_t)c;
@@ -605,7 +607,8 @@ __global__ void __launch_bounds__(kCountWarps * 32, 4) rank_count_kernel(
     __syncthreads();
     // a block tile: kCountWarps warps x 32 lanes x 4 consecutive rows, the
     // bounds read as float4 (scalars at a ragged end or unaligned buffers)
-    const bool vec_ok = ((reinterpret_cast<uintptr_t>(lo) | reinterpret_cast<uintptr_t>(hi)) & 15) == 0;
+    const bool vec_ok =
+        ((reinterpret_cast<uintptr_t>(lo) | reinterpret_cast<uintptr_t>(hi)) & 15) == 0;
     const unsigned int lanemask_lt = (1u << lane) - 1u;
     for (int64_t tb = (int64_t)blockIdx.x * kCountTile;; tb += step) {
         const int64_t base = tb + (int64_t)warp * 32 * 4;
@@ -1184,7 +1187,8 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
             return g;
         }();
         int64_t blocks = (int64_t)std::max(grid, 1) * std::max(x->num_sms, 1);
-        blocks = std::min<int64_t>(blocks, std::max<int64_t>(1, (rows + kCountTile - 1) / kCountTile));
+        blocks = std::min<int64_t>(blocks,
+                                   std::max<int64_t>(1, (rows + kCountTile - 1) / kCountTile));
         count_launches(1);
         // |zq_j| <= Q keeps sum |zq_j z_j| <= m_pad Q 127 below 2^31
         const int qrange = (int)std::min<int64_t>(16383, ((int64_t(1) << 31) - 1) /
