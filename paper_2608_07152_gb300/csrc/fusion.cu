@@ -1193,6 +1193,9 @@ pvs_status rank_queries(pvs_cursor* c, const int32_t* dense_ids, int32_t nd, boo
         // |zq_j| <= Q keeps sum |zq_j z_j| <= m_pad Q 127 below 2^31
         const int qrange = (int)std::min<int64_t>(16383, ((int64_t(1) << 31) - 1) /
                                                              (127 * (int64_t)x->m_pad));
+        // the query codes' 4 m_pad bytes beside 33 KB of static shared memory
+        // pass the default 48 KB once m_pad exceeds 3,840
+        if (resid) RQ_CUDA(raise_smem_limit((const void*)rank_count_kernel, (size_t)x->m_pad * 4));
         rank_count_kernel<<<(unsigned)blocks, kCountWarps * 32,
                             resid ? (size_t)x->m_pad * 4 : 0, st>>>(
             c->lo, c->hi, rows, tomb, c->qraw, x->raw, x->m_raw, d_keys, nd, exact ? 1 : 0,

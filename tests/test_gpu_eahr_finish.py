@@ -323,3 +323,25 @@ def test_exact_ranks_of_mid_scores_through_the_residual_codes():
             pvs.pvs_snapshot_free(snap)
     finally:
         pvs.pvs_index_free(index)
+
+
+@pytest.mark.parametrize("m", [4096, 4200])
+def test_exact_ranks_at_the_widest_residual_rows_and_beyond(m):
+    """m_pad = 4096, the widest rows given residual codes (16 KB of query
+    codes in shared memory), and m_pad = 4224, whose exact counts read the
+    fp32 rows of every straddling row: the same exact ranks either way."""
+    rng = np.random.default_rng(360 + m)
+    n, pairs = 6_000, 6
+    V = synth.unit_normal(n, m, seed=361 + m).numpy()
+    q = synth.unit_normal(1, m, seed=362 + m).numpy()[0]
+    dense_ids, _ = po.dense_ranking(q, V)
+    S = _tied_mid_sparse(dense_ids, pairs, rng)
+    T = ro.target_topk_large([dense_ids, S], [1, 1], 60, 2 * pairs, ro.NUMERATOR)
+    index = pvs.pvs_build(V)
+    try:
+        ids, F, st = _run(index, q, S, step=0, K=2 * pairs, k=60, form=pvs.EAHR_NUMERATOR)
+    finally:
+        pvs.pvs_index_free(index)
+    _check(ids, F, T)
+    assert st["complete"] == 3
+    assert not np.isnan(F).any()
