@@ -1425,14 +1425,16 @@ def main_passage(args, pvs, synth, torch, np, rank, world, local, dev, pg):
     warm_q = queries[:args.warmup * nq]
     timed_q = queries[args.warmup * nq:]
     n_timed = timed_q.shape[0]
-    ids = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
-    scores = torch.empty((n_timed, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    n_buf = max(n_timed, warm_q.shape[0])   # the warm-up may hold more queries than the timed steps
+    ids_buf = torch.empty((n_buf, RANKS_PER_QUERY), dtype=torch.int64, device=dev)
+    scores_buf = torch.empty((n_buf, RANKS_PER_QUERY), dtype=torch.float32, device=dev)
+    ids, scores = ids_buf[:n_timed], scores_buf[:n_timed]
     executor = pvs.pvs_executor_create(index, PIPELINE)
     try:
         pvs.pvs_executor_set_group(executor, group)
         if warm_q.shape[0]:
             pvs.pvs_executor_run_device(executor, warm_q, RANKS_PER_QUERY, CHUNK,
-                                        ids[:warm_q.shape[0]], scores[:warm_q.shape[0]])
+                                        ids_buf[:warm_q.shape[0]], scores_buf[:warm_q.shape[0]])
         st0 = pvs.pvs_executor_stats(executor)
 
         # ---- timed region: device-resident queries and outputs ----
