@@ -104,6 +104,10 @@ struct Contrib {
         f.den = b * (uint64_t)r + c;
         return f;
     }
+    // the same in binary64 (relative error within 2^-52)
+    double at_d(int64_t r) const {
+        return a == 0 ? 0.0 : (double)a / (double)(b * (uint64_t)r + c);
+    }
 };
 
 struct Node {
@@ -458,6 +462,25 @@ class Driver {
         if (active[0] && r0) f = add(f, g[0].at(r0));
         if (active[1] && r1) f = add(f, g[1].at(r1));
         return f;
+    }
+
+    // L and U in binary64, within 2^-50 of the exact values (relative)
+    double L_d(int32_t x) const {
+        double f = 0.0;
+        const int32_t r0 = rank(0, x), r1 = rank(1, x);
+        if (active[0] && r0) f += g[0].at_d(r0);
+        if (active[1] && r1) f += g[1].at_d(r1);
+        return f;
+    }
+    double U_d(int32_t x) const {
+        double f = L_d(x);
+        for (int i = 0; i < 2; ++i)
+            if (active[i] && !exhausted[i] && !rank(i, x)) f += u_d(i);
+        return f;
+    }
+    double u_d(int i) const {
+        if (!active[i] || exhausted[i]) return 0.0;
+        return g[i].at_d(depth[i] + 1);
     }
 
     Frac U(int32_t x) const {
@@ -899,24 +922,39 @@ pvs_status finish_rank_queries(Driver& d, const eahr_params* p, int64_t* out_ids
         if (d.certify()) return PVS_OK;
     }
     const int K = p->K;
-    // the K-th largest L over the items read (each once)
-    std::vector<Node> known;
+    // the K-th largest L over the items read (each once): binary64 values
+    // (within 2^-50, relative) find the items that can hold it, all those
+    // within 10^-12 of the K-th largest value or above, and exact rationals
+    // decide among them
+    struct Approx {
+        double v;
+        int32_t id;
+    };
+    std::vector<Approx> known;
     known.reserve(d.prefix[0].size() + d.prefix[1].size());
-    for (int32_t x : d.prefix[0]) known.push_back(Node{d.L(x), x});
+    for (int32_t x : d.prefix[0]) known.push_back(Approx{d.L_d(x), x});
     for (int32_t x : d.prefix[1])
-        if (!d.rank(0, x)) known.push_back(Node{d.L(x), x});
+        if (!d.rank(0, x)) known.push_back(Approx{d.L_d(x), x});
     if ((int64_t)known.size() < K) return PVS_OK;
-    std::nth_element(known.begin(), known.begin() + (K - 1), known.end(), NodeCmp());
-    const Frac LB = known[(size_t)K - 1].F;
+    std::nth_element(known.begin(), known.begin() + (K - 1), known.end(),
+                     [](const Approx& a, const Approx& b) { return a.v > b.v; });
+    const double near = known[(size_t)K - 1].v * (1.0 - 1e-12);
+    std::vector<Node> top;
+    for (const Approx& a : known)
+        if (a.v >= near) top.push_back(Node{d.L(a.id), a.id});
+    std::nth_element(top.begin(), top.begin() + (K - 1), top.end(), NodeCmp());
+    const Frac LB = top[(size_t)K - 1].F;
     if (LB.num == 0 || cmp(add(d.u(0), d.u(1)), LB) >= 0) return PVS_OK;
-    // candidates and the ranks they miss
+    // candidates and the ranks they miss (U below LB by more than 10^-12 in
+    // binary64 is below it exactly)
+    const double LB_d = (double)LB.num / (double)LB.den;
     std::vector<int32_t> cand, need_d, need_s;
-    for (const Node& nd : known) {
-        if (cmp(d.U(nd.id), LB) < 0) continue;
-        cand.push_back(nd.id);
+    for (const Approx& a : known) {
+        if (d.U_d(a.id) < LB_d * (1.0 - 1e-12) || cmp(d.U(a.id), LB) < 0) continue;
+        cand.push_back(a.id);
         for (int i = 0; i < 2; ++i) {
-            if (!d.active[i] || d.exhausted[i] || d.rank(i, nd.id)) continue;
-            (i == 0 ? need_d : need_s).push_back(nd.id);
+            if (!d.active[i] || d.exhausted[i] || d.rank(i, a.id)) continue;
+            (i == 0 ? need_d : need_s).push_back(a.id);
         }
     }
     if ((int64_t)need_d.size() > pvs::kRankQueryMax || (int64_t)need_s.size() > pvs::kRankQueryMax)
